@@ -1,0 +1,69 @@
+"""Whole-network forward passes composed from the oracle's layer routines
+(test infrastructure only).
+
+MINW-Net inference (Algorithm 1, inference branch): for l = 1..n the weights
+are quantized (W^ = h(W)), the layer computes a~_l = a^q_{l-1} W^_l, and every
+layer but the last quantizes its output (a^q_l = h(a~_l)).  Around the product
+sit the layer constructs of Sec. III-E: {QuantizedConv-pooling-BN-HardTanh}
+or {QuantizedConv-BN-HardTanh}; the input of the first convolution stays
+fp32 while its weights are quantized; batch normalisation also follows the
+fully connected layers; the last layer's BN output is the fp32 logits.
+"""
+import numpy as np
+
+from . import oracle as O
+
+
+def _layer_levels_w(layer, thr_w):
+    return O.quantize(layer["w"], layer["bits_w"], thr_w, layer["w_scale"])
+
+
+def convnet_layer(layer, a, thr_a, thr_w):
+    """One layer of the Model-A-shaped ConvNet.
+
+    ``a`` is the fp32 image for the first layer and the previous layer's
+    HardTanh output otherwise (its quantization h is applied here).  Returns
+    (acc, y): the integer accumulator (None for the fp32 first layer, whose raw
+    output is fp32) after pooling, and the layer's fp32 output after BN and,
+    unless it is the last layer, HardTanh."""
+    wl = _layer_levels_w(layer, thr_w)
+    acc = None
+    if layer["bits_in"] == 0:
+        z = O.conv2d_f32_seq(a, wl.astype(np.float32), layer["stride"], layer["pad"])
+        if layer["pool"]:
+            z = O.maxpool_f32(z, 2, 2, 0)
+        y = O.affine(z, layer["scale"], layer["shift"])
+    else:
+        al = O.quantize(a, layer["bits_in"], thr_a)
+        if layer["kind"] == "conv":
+            acc = O.conv2d_levels(al, wl, layer["stride"], layer["pad"],
+                                  layer["bits_in"], layer["bits_w"])
+            if layer["pool"]:
+                acc = O.maxpool_i32(acc, 2, 2)
+        else:
+            B = al.shape[0]
+            flat = al.reshape(B, -1)                       # (c, h, w) order
+            acc = O.conv2d_levels(flat[:, :, None, None], wl[:, :, None, None], 1, 0,
+                                  layer["bits_in"], layer["bits_w"])
+            acc = acc.reshape(B, -1)
+        y = O.affine(acc, layer["scale"], layer["shift"])
+    if layer["bits_out"] != 0:
+        y = O.hardtanh(y)
+    return acc, y
+
+
+def convnet_forward(net, x, keep=False):
+    """Forward pass of the ConvNet built by ``inputs.convnet_params``.
+    Returns the fp32 logits, and with ``keep`` also the per-layer (acc, y)."""
+    a = x
+    trace = []
+    for layer in net["layers"]:
+        acc, a = convnet_layer(layer, a, net["thr_a"], net["thr_w"])
+        if keep:
+            trace.append((acc, a))
+    return (a, trace) if keep else a
+
+
+def activation_levels(y, bits, thr):
+    """Quantized levels h(y) of a layer output (what the next layer consumes)."""
+    return O.quantize(y, bits, thr)
