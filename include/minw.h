@@ -1,0 +1,246 @@
+/*
+ * minw.h -- C ABI of libminw.so: the MINW-Net low-bit inference hot path and
+ * the AQE quantizer of "Propagating Asymptotic-Estimated Gradients for Low
+ * Bitwidth Quantized Neural Networks" (arXiv 2003.04296), on one GB300
+ * (sm_103a).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Every pointer argument is a DEVICE pointer unless its comment says host.
+ *   The caller allocates and frees all tensors; only a minw_net owns memory.
+ * - Calls are asynchronous on the given CUDA stream (`stream` is a
+ *   cudaStream_t passed as void*; NULL = legacy default stream).  The return
+ *   value reports argument validation and launch errors only.
+ * - Device-side failures (a bounded wait that ran out) are latched in a
+ *   device flag and read with minw_get_last_device_error().
+ * - No call allocates device memory except minw_net_create.
+ * - Tensors are dense and row-major in the order written; device pointers
+ *   must be 16-byte aligned.
+ *
+ * Packed bit-plane layout ("planes")
+ * ----------------------------------
+ * A quantized tensor with `bits` in {1,2,3} is stored as uint32 words
+ *     [N][H][W][P][NW],  P = bits, NW = ceil(C/32),
+ * bit (c % 32) of word (c / 32) holding channel c; bits of channels >= C are 0.
+ *   plane 0           : 1 iff the level is negative (1-bit: 1 iff level = -1)
+ *   2-bit plane 1     : 1 iff the level is non-zero
+ *   3-bit planes 1, 2 : bits 0 and 1 of the magnitude code k,
+ *                       |level| = 2^(k-3) for k in {1,2,3}, 0 for k = 0
+ * Levels (Sec. IV-A): 1 bit {-1, 1} (Eq. sign), 2 bit {-1, 0, 1} (Eq. tnn),
+ * 3 bit {0, +-1/4, +-1/2, +-1} (Eq. qnn).  Weights [O][C][kh][kw] pack to
+ * [O][kh][kw][P][NW] (the same layout with N = O, H = kh, W = kw).
+ *
+ * Integer accumulators
+ * --------------------
+ * A convolution of quantized operands returns the exact integer
+ *     acc = (sum over valid taps of a_level * w_level) * 2^(f_a + f_w),
+ * f = 2 for a 3-bit operand, 0 otherwise (3-bit levels are multiples of 1/4).
+ * Zero padding contributes nothing (padding of the dequantized tensor).
+ */
+#ifndef MINW_H
+#define MINW_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define MINW_API __attribute__((visibility("default")))
+#else
+#define MINW_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MINW_OK = 0,
+    MINW_EINVAL = 1,          /* bad argument: null pointer, size, alignment, bits */
+    MINW_EUNSUPPORTED = 2,    /* valid request outside what the kernels cover */
+    MINW_ECUDA = 3,           /* a CUDA runtime call or launch failed */
+    MINW_ETIMEOUT = 4,        /* a bounded device-side wait ran out */
+    MINW_EDEVICE = 5          /* no usable sm_103a device */
+} minw_status;
+
+/* Quantizer h of Eq. sign / Eq. tnn / Eq. qnn applied to u = x * scale
+ * (one fp32 multiply; scale = 1 is the paper's quantizer).
+ *   bits 1: level = +1 if u > 0, -1 otherwise (sign(0) = -1).
+ *   bits 2: level = 0 if |u| <= thr[0], sign(u) otherwise.
+ *   bits 3: |u| <= thr[2] -> 0; thr[2] < |u| <= thr[1] -> +-1/4;
+ *           thr[1] < |u| <= thr[0] -> +-1/2; |u| > thr[0] -> +-1.
+ * thr must be descending; unused entries are ignored.  Host struct. */
+typedef struct {
+    int32_t bits;
+    float thr[3];
+    float scale;
+} minw_quant;
+
+/* Human-readable name of a status code (static string). */
+MINW_API const char *minw_status_string(minw_status s);
+
+/* Version of the library as MAJOR*10000 + MINOR*100 + PATCH. */
+MINW_API int32_t minw_version(void);
+
+/* ---------------------------------------------------------------------- */
+/* AQE elementwise (Sec. III-C, Eq. activation / Eq. weight, Eq. ours)     */
+/* ---------------------------------------------------------------------- */
+
+/* AQE forward, Eq. ours: y = alpha * h(x) + (1 - alpha) * x, evaluated in
+ * fp32 as fmaf(alpha, h(x * q->scale), (1 - alpha) * x).
+ * x, y: n floats (may alias).  alpha in [0, 1].  q: host pointer.
+ * Errors: MINW_EINVAL for n < 0, null pointers, misalignment, bad q. */
+MINW_API minw_status aqe_forward(const float *x, float *y, int64_t n, float alpha,
+                        const minw_quant *q, void *stream);
+
+/* AQE backward, Eq. activation / Eq. weight:
+ * gx = (|x| <= 1) ? gy * (2 * alpha) : 0   (fp32, one rounding).
+ * x, gy, gx: n floats (gx may alias gy). */
+MINW_API minw_status aqe_backward(const float *x, const float *gy, float *gx,
+                         int64_t n, float alpha, void *stream);
+
+/* Quantize + pack (Eq. inference: a^ = h(a)) with the AQE forward and the
+ * backward mask of Eq. activation fused into the same pass over x.
+ * x: fp32 NCHW [B][C][H][W].  planes: packed layout above (q->bits planes).
+ * y (nullable): AQE forward output at `alpha`, NCHW fp32, as aqe_forward.
+ * mask (nullable): 1 bit per element of x in flat NCHW order,
+ *   bit (i % 32) of word (i / 32) = 1[|x_i| <= 1]; ceil(B*C*H*W/32) words.
+ * Errors: MINW_EINVAL for non-positive sizes, null x/planes, bad q. */
+MINW_API minw_status aqe_quantize_pack(const float *x, int32_t B, int32_t C, int32_t H,
+                              int32_t W, const minw_quant *q, uint32_t *planes,
+                              float alpha, float *y, uint32_t *mask,
+                              void *stream);
+
+/* AQE backward from the packed mask written by aqe_quantize_pack:
+ * gx_i = bit_i(mask) ? gy_i * (2 * alpha) : 0, n elements. */
+MINW_API minw_status aqe_backward_masked(const uint32_t *mask, const float *gy,
+                                float *gx, int64_t n, float alpha,
+                                void *stream);
+
+/* Quantize + pack latent weights w [O][C][kh][kw] (Eq. inference:
+ * W^ = h(W)) into planes [O][kh][kw][q->bits][ceil(C/32)].
+ * channel_scale (nullable): per-output-channel multiplier replacing
+ * q->scale, u = w * channel_scale[o]. */
+MINW_API minw_status minw_pack_weights(const float *w, int32_t O, int32_t C, int32_t kh,
+                              int32_t kw, const minw_quant *q,
+                              const float *channel_scale, uint32_t *planes,
+                              void *stream);
+
+/* ---------------------------------------------------------------------- */
+/* Quantized convolution (Algorithm 1, inference: a~ = a^q W^q)            */
+/* ---------------------------------------------------------------------- */
+
+enum {
+    MINW_VARIANT_AUTO = 0,    /* per-shape choice from measurements */
+    MINW_VARIANT_POPC = 1,    /* bit-serial XNOR/AND + popcount on the integer pipe */
+    MINW_VARIANT_TC = 2       /* tcgen05 tensor cores on exact FP8 level values */
+};
+
+/* Convolution of packed activations act [B][H][W][bits_a][C/32] with packed
+ * weights wgt [O][kh][kw][bits_w][C/32]; C must be a multiple of 32.
+ * Output size Ho = (H + 2 pad - kh)/stride + 1, Wo likewise.
+ * acc_out (nullable): int32 NCHW [B][O][Ho][Wo], the exact accumulator.
+ * y_out (nullable): fp32 NCHW, y = fmaf((float)acc, scale[o], shift[o]);
+ *   scale/shift (length O) are required when y_out is given.
+ * variant: MINW_VARIANT_*.  At least one output must be non-null.
+ * Errors: MINW_EINVAL (sizes, pointers, bits), MINW_EUNSUPPORTED (C % 32,
+ * a variant that does not cover the shape). */
+MINW_API minw_status minw_conv2d(const uint32_t *act, int32_t B, int32_t C, int32_t H,
+                        int32_t W, int32_t bits_a, const uint32_t *wgt,
+                        int32_t O, int32_t kh, int32_t kw, int32_t bits_w,
+                        int32_t stride, int32_t pad, int32_t *acc_out,
+                        const float *scale, const float *shift, float *y_out,
+                        int32_t variant, void *stream);
+
+/* One MINW-Net block (Sec. III-E): QuantizedConv - [2x2/2 max pool] - BN -
+ * HardTanh - quantize, the quantize + pack of the next layer's input fused
+ * into the epilogue.  Pooling acts on the integer accumulator (the order the
+ * paper's block prescribes); BN is y = fmaf((float)acc, scale[o], shift[o]).
+ * pool: 0 or 1 (requires even Ho, Wo).
+ * q_out (nullable, host): quantizer of the output; when given, the output is
+ *   HardTanh'ed and packed into planes_out [B][Hp][Wp][q_out->bits][ceil(O/32)]
+ *   (Hp, Wp = pooled size).  When NULL the block is a last layer: no
+ *   HardTanh, no quantization.
+ * y_out (nullable): fp32 NCHW output after BN (and HardTanh when q_out).
+ * At least one of planes_out / y_out must be given. */
+MINW_API minw_status minw_conv_block(const uint32_t *act, int32_t B, int32_t C,
+                            int32_t H, int32_t W, int32_t bits_a,
+                            const uint32_t *wgt, int32_t O, int32_t kh,
+                            int32_t kw, int32_t bits_w, int32_t stride,
+                            int32_t pad, int32_t pool, const float *scale,
+                            const float *shift, const minw_quant *q_out,
+                            uint32_t *planes_out, float *y_out,
+                            int32_t variant, void *stream);
+
+/* First layer (Sec. III-E): the fp32 image x [B][C][H][W] is NOT quantized;
+ * the weights are.  w: latent fp32 weights [O][C][kh][kw]; q_w (host) and
+ * channel_scale (nullable) quantize them as minw_pack_weights does; q_w NULL
+ * keeps the fp32 weights as they are.  Each output is one fp32 fmaf chain over
+ * (c, ky, kx) in that order, padded taps skipped.  Then [pool 2x2/2 on fp32],
+ * BN (fmaf), and, with q_out, HardTanh + quantize + pack as minw_conv_block. */
+MINW_API minw_status minw_conv_first(const float *x, int32_t B, int32_t C, int32_t H,
+                            int32_t W, const float *w, int32_t O, int32_t kh,
+                            int32_t kw, int32_t stride, int32_t pad,
+                            const minw_quant *q_w, const float *channel_scale,
+                            int32_t pool, const float *scale,
+                            const float *shift, const minw_quant *q_out,
+                            uint32_t *planes_out, float *y_out, void *stream);
+
+/* ---------------------------------------------------------------------- */
+/* Whole-network forward (Algorithm 1, inference branch)                   */
+/* ---------------------------------------------------------------------- */
+
+enum { MINW_LAYER_CONV = 0, MINW_LAYER_FC = 1 };
+
+/* One layer of a sequential MINW-Net.  Pointers are device pointers read
+ * during minw_net_create only (the net keeps its own packed copy).
+ * - CONV: input [C][H][W], kernel kh x kw, stride, pad, optional pool.
+ * - FC: input is the previous output flattened in (c, h, w) order; C, H, W
+ *   describe that input (K = C*H*W); w is [O][K].
+ * bits_in 0 marks the first layer (fp32 input, minw_conv_first);
+ * bits_out 0 marks the last layer (fp32 logits, no HardTanh). */
+typedef struct {
+    int32_t kind;
+    int32_t C, H, W, O;
+    int32_t kh, kw, stride, pad, pool;
+    int32_t bits_in, bits_w, bits_out;
+    float thr_w[3];           /* weight quantizer thresholds */
+    float thr_out[3];         /* output quantizer thresholds */
+    const float *w;           /* latent weights */
+    const float *w_scale;     /* per-output-channel prescale, nullable */
+    const float *scale;       /* BN scale (length O) */
+    const float *shift;       /* BN shift (length O) */
+} minw_layer_desc;
+
+typedef struct minw_net minw_net;
+
+/* Build a network: validates the layer chain, packs every weight tensor,
+ * plans a kernel per layer (variant: MINW_VARIANT_*) and allocates activation
+ * buffers for up to max_batch images.  layers: host array.  Synchronous. */
+MINW_API minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers,
+                            int32_t max_batch, int32_t variant, void *stream,
+                            minw_net **out);
+
+/* Forward pass of B <= max_batch images x [B][C][H][W] (fp32) to logits
+ * [B][O_last] (fp32).  All work is enqueued on `stream`. */
+MINW_API minw_status minw_forward(minw_net *net, const float *x, int32_t B,
+                         float *logits, void *stream);
+
+/* Number of kernels one minw_forward launches. */
+MINW_API int32_t minw_net_launches(const minw_net *net);
+
+/* Release a network (synchronises its device memory frees). */
+MINW_API void minw_net_destroy(minw_net *net);
+
+/* ---------------------------------------------------------------------- */
+/* Errors                                                                  */
+/* ---------------------------------------------------------------------- */
+
+/* Reads and clears the device error flag after synchronising `stream`:
+ * MINW_OK, or MINW_ETIMEOUT when a bounded wait inside a kernel gave up. */
+MINW_API minw_status minw_get_last_device_error(void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MINW_H */

@@ -1,0 +1,53 @@
+// kernels.cuh -- argument blocks and launchers shared by the translation units.
+#pragma once
+
+#include "common.cuh"
+
+namespace minw {
+
+// Everything one quantized-convolution launch needs (passed by value).
+struct ConvArgs {
+    const uint32_t *act;   // [B][H][W][PA][NW]
+    const uint32_t *wgt;   // [O][kh][kw][PW][NW]
+    int B, C, H, W, O, kh, kw, stride, pad;
+    int Ho, Wo, NW;
+    int bits_a, bits_w;
+    long long M;           // B * Ho * Wo output pixels
+    // epilogue
+    int32_t *acc_out;      // int32 NCHW, unpooled (nullable)
+    float *y_out;          // fp32 NCHW after BN [+HardTanh] (nullable)
+    const float *scale;    // BN scale [O]
+    const float *shift;    // BN shift [O]
+    int pool;              // 2x2/2 max pool on the accumulator before BN
+    int quant_out;         // HardTanh + quantize + pack into planes_out
+    QParams qo;            // quantizer of the output
+    uint32_t *planes_out;  // [B][Hp][Wp][qo.bits][ceil(O/32)]
+};
+
+// First-layer convolution on the fp32 image (see conv_first.cu).
+struct FirstArgs {
+    const float *x;            // [B][C][H][W]
+    const float *w;            // latent [O][C][kh][kw]
+    const float *cscale;       // per-output-channel weight prescale (nullable)
+    int quant_w;               // quantize weights with qw
+    QParams qw;
+    int B, C, H, W, O, kh, kw, stride, pad, Ho, Wo;
+    const float *scale, *shift;
+    int quant_out;
+    QParams qo;
+    uint32_t *planes_out;      // [B][Ho][Wo][qo.bits][ceil(O/32)]
+    float *y_out;              // [B][O][Ho][Wo] (nullable)
+};
+
+// Launchers (host).  Return MINW_OK or an error status.
+minw_status launch_conv_first(const FirstArgs &a, cudaStream_t s);
+minw_status launch_conv_popc(const ConvArgs &a, cudaStream_t s);
+minw_status make_conv_args(ConvArgs &a, const uint32_t *act, int B, int C, int H, int W,
+                           int bits_a, const uint32_t *wgt, int O, int kh, int kw, int bits_w,
+                           int stride, int pad);
+int choose_variant(const ConvArgs &a, int requested);
+minw_status run_conv(const ConvArgs &a, int variant, cudaStream_t s);
+minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s);
+bool conv_tc_supported(const ConvArgs &a);
+
+}  // namespace minw

@@ -1,0 +1,193 @@
+// net.cu -- whole-network forward of a sequential MINW-Net (Algorithm 1,
+// inference branch, with the layer constructs of Sec. III-E).
+//
+// minw_net_create packs every quantized weight tensor once (W^ = h(W)),
+// copies the BN affine maps, plans one kernel per layer and allocates two
+// ping-pong activation buffers holding packed planes.  minw_forward then
+// enqueues one kernel per layer: the fp32 first layer, then quantized
+// convolution blocks whose epilogues write the next layer's packed input, and
+// a last layer that writes fp32 logits.  Fully connected layers run as
+// convolutions whose kernel covers the whole input map (flatten order
+// (c, h, w) = OIHW weight order).
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <vector>
+
+#include "kernels.cuh"
+
+using namespace minw;
+using namespace minw_host;
+
+struct LayerPlan {
+    minw_layer_desc d;        // shape fields only; pointers are not kept
+    int C, H, W, O, kh, kw, stride, pad, pool;
+    int Ho, Wo, Hp, Wp;
+    uint32_t *wplanes = nullptr;   // packed weights (quantized layers)
+    float *wlatent = nullptr;      // fp32 weights (first layer)
+    float *wscale = nullptr;       // per-channel weight prescale (first layer)
+    float *scale = nullptr;
+    float *shift = nullptr;
+    minw_quant qw{}, qo{};
+    int variant = MINW_VARIANT_POPC;
+};
+
+struct minw_net {
+    std::vector<LayerPlan> L;
+    int max_batch = 0;
+    uint32_t *buf[2] = {nullptr, nullptr};
+    size_t buf_words = 0;
+    std::vector<void *> owned;
+};
+
+static void net_free(minw_net *n) {
+    if (!n) return;
+    for (void *p : n->owned) cudaFree(p);
+    delete n;
+}
+
+template <typename T>
+static minw_status net_alloc(minw_net *n, T **p, size_t count) {
+    void *q = nullptr;
+    if (cudaMalloc(&q, count * sizeof(T) + 16) != cudaSuccess) return MINW_ECUDA;
+    n->owned.push_back(q);
+    *p = reinterpret_cast<T *>(q);
+    return MINW_OK;
+}
+
+extern "C" {
+
+minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int32_t max_batch,
+                            int32_t variant, void *stream, minw_net **out) {
+    if (!layers || n_layers < 2 || max_batch <= 0 || !out) return MINW_EINVAL;
+    if (variant < 0 || variant > 2) return MINW_EINVAL;
+    *out = nullptr;
+    cudaStream_t s = (cudaStream_t)stream;
+    minw_net *n = new minw_net();
+    n->max_batch = max_batch;
+    int pc = 0, ph = 0, pw = 0, pbits = 0;     // previous output shape and bits
+    size_t max_words = 0;
+    for (int l = 0; l < n_layers; ++l) {
+        const minw_layer_desc &d = layers[l];
+        LayerPlan P;
+        P.d = d;
+        P.d.w = nullptr; P.d.w_scale = nullptr; P.d.scale = nullptr; P.d.shift = nullptr;
+        const bool first = l == 0, last = l == n_layers - 1;
+        if (!d.w || !d.scale || !d.shift || d.O <= 0 || d.C <= 0 || d.H <= 0 || d.W <= 0) {
+            net_free(n);
+            return MINW_EINVAL;
+        }
+        if ((first && (d.bits_in != 0 || d.kind != MINW_LAYER_CONV)) || (!first && d.bits_in != pbits) ||
+            (last && d.bits_out != 0) || (!last && (d.bits_out < 1 || d.bits_out > 3)) ||
+            (!first && (d.bits_w < 1 || d.bits_w > 3)) || (first && (d.bits_w < 0 || d.bits_w > 3)) ||
+            (!first && (d.C != pc || d.H != ph || d.W != pw))) {
+            net_free(n);
+            return MINW_EINVAL;
+        }
+        P.C = d.C; P.H = d.H; P.W = d.W; P.O = d.O;
+        if (d.kind == MINW_LAYER_FC) {
+            P.kh = d.H; P.kw = d.W; P.stride = 1; P.pad = 0; P.pool = 0;
+        } else {
+            P.kh = d.kh; P.kw = d.kw; P.stride = d.stride; P.pad = d.pad; P.pool = d.pool;
+        }
+        if (P.kh <= 0 || P.kw <= 0 || P.stride <= 0 || P.pad < 0) { net_free(n); return MINW_EINVAL; }
+        P.Ho = (P.H + 2 * P.pad - P.kh) / P.stride + 1;
+        P.Wo = (P.W + 2 * P.pad - P.kw) / P.stride + 1;
+        if (P.Ho <= 0 || P.Wo <= 0 || (P.pool && ((P.Ho & 1) || (P.Wo & 1)))) {
+            net_free(n);
+            return MINW_EINVAL;
+        }
+        P.Hp = P.pool ? P.Ho / 2 : P.Ho;
+        P.Wp = P.pool ? P.Wo / 2 : P.Wo;
+        P.qw.bits = d.bits_w; P.qw.scale = 1.0f;
+        for (int i = 0; i < 3; ++i) P.qw.thr[i] = d.thr_w[i];
+        P.qo.bits = d.bits_out; P.qo.scale = 1.0f;
+        for (int i = 0; i < 3; ++i) P.qo.thr[i] = d.thr_out[i];
+        if ((d.bits_w > 0 && !valid_quant(&P.qw)) || (!last && !valid_quant(&P.qo))) {
+            net_free(n);
+            return MINW_EINVAL;
+        }
+        minw_status st = MINW_OK;
+        if ((st = net_alloc(n, &P.scale, P.O)) != MINW_OK || (st = net_alloc(n, &P.shift, P.O)) != MINW_OK) {
+            net_free(n);
+            return st;
+        }
+        cudaMemcpyAsync(P.scale, d.scale, sizeof(float) * P.O, cudaMemcpyDeviceToDevice, s);
+        cudaMemcpyAsync(P.shift, d.shift, sizeof(float) * P.O, cudaMemcpyDeviceToDevice, s);
+        const size_t K = (size_t)P.C * P.kh * P.kw;
+        if (first) {
+            if ((st = net_alloc(n, &P.wlatent, (size_t)P.O * K)) != MINW_OK) { net_free(n); return st; }
+            cudaMemcpyAsync(P.wlatent, d.w, sizeof(float) * P.O * K, cudaMemcpyDeviceToDevice, s);
+            if (d.w_scale) {
+                if ((st = net_alloc(n, &P.wscale, P.O)) != MINW_OK) { net_free(n); return st; }
+                cudaMemcpyAsync(P.wscale, d.w_scale, sizeof(float) * P.O, cudaMemcpyDeviceToDevice, s);
+            }
+        } else {
+            if (P.C % 32 != 0) { net_free(n); return MINW_EUNSUPPORTED; }
+            const size_t words = (size_t)P.O * P.kh * P.kw * d.bits_w * (P.C / 32);
+            if ((st = net_alloc(n, &P.wplanes, words)) != MINW_OK) { net_free(n); return st; }
+            // the weights are [O][C][kh][kw]; an FC weight [O][K] with K in
+            // (c, h, w) order is the same array
+            st = minw_pack_weights(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, P.wplanes, stream);
+            if (st != MINW_OK) { net_free(n); return st; }
+            ConvArgs a;
+            st = make_conv_args(a, P.wplanes, max_batch, P.C, P.H, P.W, d.bits_in, P.wplanes, P.O,
+                                P.kh, P.kw, d.bits_w, P.stride, P.pad);
+            if (st != MINW_OK) { net_free(n); return st; }
+            a.pool = P.pool;
+            a.quant_out = !last;
+            if (!last) a.qo = to_qparams(&P.qo);
+            P.variant = choose_variant(a, variant);
+        }
+        if (!last) {
+            const size_t words = (size_t)max_batch * P.Hp * P.Wp * d.bits_out * ((P.O + 31) / 32);
+            if (words > max_words) max_words = words;
+        }
+        pc = P.O; ph = P.Hp; pw = P.Wp; pbits = d.bits_out;
+        n->L.push_back(P);
+    }
+    for (int i = 0; i < 2; ++i) {
+        minw_status st = net_alloc(n, &n->buf[i], max_words);
+        if (st != MINW_OK) { net_free(n); return st; }
+    }
+    n->buf_words = max_words;
+    if (cudaStreamSynchronize(s) != cudaSuccess) { net_free(n); return MINW_ECUDA; }
+    *out = n;
+    return MINW_OK;
+}
+
+minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits, void *stream) {
+    if (!net || !x || !logits || B <= 0 || B > net->max_batch) return MINW_EINVAL;
+    const int nl = (int)net->L.size();
+    int cur = 0;
+    for (int l = 0; l < nl; ++l) {
+        const LayerPlan &P = net->L[l];
+        const bool last = l == nl - 1;
+        uint32_t *dst = last ? nullptr : net->buf[cur];
+        float *y = last ? logits : nullptr;
+        minw_status st;
+        if (l == 0) {
+            st = minw_conv_first(x, B, P.C, P.H, P.W, P.wlatent, P.O, P.kh, P.kw, P.stride, P.pad,
+                                 P.d.bits_w > 0 ? &P.qw : nullptr, P.wscale, P.pool, P.scale, P.shift,
+                                 last ? nullptr : &P.qo, dst, y, stream);
+        } else {
+            const uint32_t *src = net->buf[cur ^ 1];
+            st = minw_conv_block(src, B, P.C, P.H, P.W, P.d.bits_in, P.wplanes, P.O, P.kh, P.kw,
+                                 P.d.bits_w, P.stride, P.pad, P.pool, P.scale, P.shift,
+                                 last ? nullptr : &P.qo, dst, y, P.variant, stream);
+        }
+        if (st != MINW_OK) return st;
+        cur ^= 1;
+    }
+    return MINW_OK;
+}
+
+int32_t minw_net_launches(const minw_net *net) { return net ? (int32_t)net->L.size() : 0; }
+
+void minw_net_destroy(minw_net *net) {
+    if (!net) return;
+    cudaDeviceSynchronize();
+    net_free(net);
+}
+
+}  // extern "C"

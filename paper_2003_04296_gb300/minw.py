@@ -1,0 +1,265 @@
+"""ctypes binding of libminw.so (include/minw.h).
+
+Argument marshalling only: every function passes device pointers, sizes and
+the current CUDA stream to the C entry point of the same name and raises on a
+non-OK status.  Every step of the computation runs in the library's CUDA
+kernels; there is no fallback of any kind.  torch provides device memory and
+streams.
+"""
+import ctypes
+import os
+
+import torch
+
+from . import build as _build
+
+_LIB = None
+
+MINW_OK, MINW_EINVAL, MINW_EUNSUPPORTED, MINW_ECUDA, MINW_ETIMEOUT, MINW_EDEVICE = range(6)
+VARIANT_AUTO, VARIANT_POPC, VARIANT_TC = 0, 1, 2
+LAYER_CONV, LAYER_FC = 0, 1
+
+
+class MinwError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} ({status})")
+
+
+class Quant(ctypes.Structure):
+    _fields_ = [("bits", ctypes.c_int32), ("thr", ctypes.c_float * 3), ("scale", ctypes.c_float)]
+
+
+class LayerDesc(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int32), ("C", ctypes.c_int32), ("H", ctypes.c_int32),
+                ("W", ctypes.c_int32), ("O", ctypes.c_int32), ("kh", ctypes.c_int32),
+                ("kw", ctypes.c_int32), ("stride", ctypes.c_int32), ("pad", ctypes.c_int32),
+                ("pool", ctypes.c_int32), ("bits_in", ctypes.c_int32), ("bits_w", ctypes.c_int32),
+                ("bits_out", ctypes.c_int32), ("thr_w", ctypes.c_float * 3),
+                ("thr_out", ctypes.c_float * 3), ("w", ctypes.c_void_p), ("w_scale", ctypes.c_void_p),
+                ("scale", ctypes.c_void_p), ("shift", ctypes.c_void_p)]
+
+
+# name -> (restype, argtypes)
+_P, _I32, _I64, _F = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float
+_QP = ctypes.POINTER(Quant)
+SIGNATURES = {
+    "minw_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "minw_version": (_I32, []),
+    "aqe_forward": (ctypes.c_int, [_P, _P, _I64, _F, _QP, _P]),
+    "aqe_backward": (ctypes.c_int, [_P, _P, _P, _I64, _F, _P]),
+    "aqe_quantize_pack": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _F, _P, _P, _P]),
+    "aqe_backward_masked": (ctypes.c_int, [_P, _P, _P, _I64, _F, _P]),
+    "minw_pack_weights": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
+    "minw_conv2d": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32,
+                                   _I32, _I32, _P, _P, _P, _P, _I32, _P]),
+    "minw_conv_block": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32,
+                                       _I32, _I32, _I32, _P, _P, _QP, _P, _P, _I32, _P]),
+    "minw_conv_first": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32, _I32,
+                                       _QP, _P, _I32, _P, _P, _QP, _P, _P, _P]),
+    "minw_net_create": (ctypes.c_int, [ctypes.POINTER(LayerDesc), _I32, _I32, _I32, _P,
+                                       ctypes.POINTER(ctypes.c_void_p)]),
+    "minw_forward": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
+    "minw_net_launches": (_I32, [_P]),
+    "minw_net_destroy": (None, [_P]),
+    "minw_get_last_device_error": (ctypes.c_int, [_P]),
+}
+
+
+def library_path():
+    return _build.LIB
+
+
+def lib(build_if_missing=False):
+    """Load libminw.so.  Raises if it is missing: there is no other path."""
+    global _LIB
+    if _LIB is None:
+        path = library_path()
+        if not os.path.exists(path):
+            if not build_if_missing:
+                raise RuntimeError(f"libminw.so not built ({path}); run __graft_entry__.build()")
+            _build.build()
+        L = ctypes.CDLL(path)
+        for name, (res, args) in SIGNATURES.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _LIB = L
+    return _LIB
+
+
+def status_string(s):
+    return lib().minw_status_string(int(s)).decode()
+
+
+def _check(status, where):
+    if status != MINW_OK:
+        raise MinwError(status, where)
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("device tensor expected")
+    if not t.is_contiguous():
+        raise ValueError("contiguous tensor expected")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def quant(bits, thr=(0.0, 0.0, 0.0), scale=1.0):
+    q = Quant()
+    q.bits = int(bits)
+    t = list(thr) + [0.0] * (3 - len(thr))
+    for i in range(3):
+        q.thr[i] = float(t[i])
+    q.scale = float(scale)
+    return q
+
+
+def packed_words(N, C, H, W, bits):
+    return N * H * W * bits * ((C + 31) // 32)
+
+
+# ---------------------------------------------------------------------------
+# entry points (same names as the C ABI)
+# ---------------------------------------------------------------------------
+
+def aqe_forward(x, y, alpha, q, stream=None):
+    _check(lib().aqe_forward(_ptr(x), _ptr(y), x.numel(), float(alpha), ctypes.byref(q), _stream(stream)),
+           "aqe_forward")
+
+
+def aqe_backward(x, gy, gx, alpha, stream=None):
+    _check(lib().aqe_backward(_ptr(x), _ptr(gy), _ptr(gx), x.numel(), float(alpha), _stream(stream)),
+           "aqe_backward")
+
+
+def aqe_quantize_pack(x, q, planes, alpha=1.0, y=None, mask=None, stream=None):
+    B, C, H, W = x.shape
+    _check(lib().aqe_quantize_pack(_ptr(x), B, C, H, W, ctypes.byref(q), _ptr(planes), float(alpha),
+                                   _ptr(y), _ptr(mask), _stream(stream)), "aqe_quantize_pack")
+
+
+def aqe_backward_masked(mask, gy, gx, alpha, stream=None):
+    _check(lib().aqe_backward_masked(_ptr(mask), _ptr(gy), _ptr(gx), gy.numel(), float(alpha),
+                                     _stream(stream)), "aqe_backward_masked")
+
+
+def minw_pack_weights(w, q, planes, channel_scale=None, stream=None):
+    O, C, kh, kw = w.shape
+    _check(lib().minw_pack_weights(_ptr(w), O, C, kh, kw, ctypes.byref(q), _ptr(channel_scale),
+                                   _ptr(planes), _stream(stream)), "minw_pack_weights")
+
+
+def minw_conv2d(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad, acc_out=None,
+                scale=None, shift=None, y_out=None, variant=VARIANT_AUTO, stream=None):
+    _check(lib().minw_conv2d(_ptr(act), B, C, H, W, bits_a, _ptr(wgt), O, kh, kw, bits_w, stride, pad,
+                             _ptr(acc_out), _ptr(scale), _ptr(shift), _ptr(y_out), int(variant),
+                             _stream(stream)), "minw_conv2d")
+
+
+def minw_conv_block(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad, pool, scale, shift,
+                    q_out=None, planes_out=None, y_out=None, variant=VARIANT_AUTO, stream=None):
+    _check(lib().minw_conv_block(_ptr(act), B, C, H, W, bits_a, _ptr(wgt), O, kh, kw, bits_w, stride,
+                                 pad, int(pool), _ptr(scale), _ptr(shift),
+                                 ctypes.byref(q_out) if q_out is not None else None,
+                                 _ptr(planes_out), _ptr(y_out), int(variant), _stream(stream)),
+           "minw_conv_block")
+
+
+def minw_conv_first(x, w, stride, pad, scale, shift, q_w=None, channel_scale=None, pool=0, q_out=None,
+                    planes_out=None, y_out=None, stream=None):
+    B, C, H, W = x.shape
+    O, _, kh, kw = w.shape
+    _check(lib().minw_conv_first(_ptr(x), B, C, H, W, _ptr(w), O, kh, kw, stride, pad,
+                                 ctypes.byref(q_w) if q_w is not None else None, _ptr(channel_scale),
+                                 int(pool), _ptr(scale), _ptr(shift),
+                                 ctypes.byref(q_out) if q_out is not None else None,
+                                 _ptr(planes_out), _ptr(y_out), _stream(stream)), "minw_conv_first")
+
+
+def minw_get_last_device_error(stream=None):
+    return lib().minw_get_last_device_error(_stream(stream))
+
+
+class Net:
+    """Owner of a minw_net (minw_net_create / minw_forward / minw_net_destroy).
+
+    ``layers`` is a list of dicts with the minw_layer_desc fields; ``w``,
+    ``w_scale``, ``scale`` and ``shift`` are device tensors."""
+
+    def __init__(self, layers, max_batch, variant=VARIANT_AUTO, stream=None):
+        arr = (LayerDesc * len(layers))()
+        keep = []
+        for d, L in zip(arr, layers):
+            d.kind = L["kind"]
+            d.C, d.H, d.W, d.O = L["C"], L["H"], L["W"], L["O"]
+            d.kh, d.kw, d.stride, d.pad, d.pool = L.get("kh", 1), L.get("kw", 1), L.get("stride", 1), \
+                L.get("pad", 0), int(L.get("pool", 0))
+            d.bits_in, d.bits_w, d.bits_out = L["bits_in"], L["bits_w"], L["bits_out"]
+            for i in range(3):
+                d.thr_w[i] = float(L["thr_w"][i])
+                d.thr_out[i] = float(L["thr_out"][i])
+            for k in ("w", "w_scale", "scale", "shift"):
+                t = L.get(k)
+                keep.append(t)
+                setattr(d, k, t.data_ptr() if t is not None else None)
+        h = ctypes.c_void_p()
+        _check(lib().minw_net_create(arr, len(layers), int(max_batch), int(variant), _stream(stream),
+                                     ctypes.byref(h)), "minw_net_create")
+        self._h = h
+        self.max_batch = max_batch
+        self.out_features = layers[-1]["O"]
+
+    def forward(self, x, logits, stream=None):
+        _check(lib().minw_forward(self._h, _ptr(x), x.shape[0], _ptr(logits), _stream(stream)),
+               "minw_forward")
+
+    @property
+    def launches(self):
+        return lib().minw_net_launches(self._h)
+
+    def close(self):
+        if self._h:
+            lib().minw_net_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def layer_descs(net_params, device):
+    """minw_layer_desc dicts (device tensors) for a network described by
+    ``inputs.convnet_params``: marshalling of the same fields, no compute."""
+    out = []
+    thr_a = net_params["thr_a"]
+    c, h, w = net_params["in_shape"]
+    for L in net_params["layers"]:
+        d = dict(bits_in=L["bits_in"], bits_w=L["bits_w"], bits_out=L["bits_out"],
+                 thr_w=list(net_params["thr_w"]), thr_out=list(thr_a) if L["bits_out"] else [0.0] * 3,
+                 w=torch.from_numpy(L["w"]).to(device).contiguous(),
+                 w_scale=torch.from_numpy(L["w_scale"]).to(device),
+                 scale=torch.from_numpy(L["scale"]).to(device),
+                 shift=torch.from_numpy(L["shift"]).to(device), O=L["O"])
+        if L["kind"] == "conv":
+            d.update(kind=LAYER_CONV, C=c, H=h, W=w, kh=L["kh"], kw=L["kw"], stride=L["stride"],
+                     pad=L["pad"], pool=int(L["pool"]))
+            h = (h + 2 * L["pad"] - L["kh"]) // L["stride"] + 1
+            w = (w + 2 * L["pad"] - L["kw"]) // L["stride"] + 1
+            if L["pool"]:
+                h, w = h // 2, w // 2
+            c = L["O"]
+        else:
+            d.update(kind=LAYER_FC, C=c, H=h, W=w)
+            c, h, w = L["O"], 1, 1
+        out.append(d)
+    return out

@@ -1,0 +1,60 @@
+"""GPU parity of the whole-network forward (minw_forward) against the oracle:
+a small Model-A-shaped ConvNet for every activation/weight bit pair the
+workloads use, and the full CIFAR ConvNet at batch 256 on sampled images."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from oracle import network as N  # noqa: E402
+from paper_2003_04296_gb300.inputs import convnet_input, convnet_params  # noqa: E402
+from tests._gpu import assert_close, dev_tensor  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dev():
+    import __graft_entry__ as g
+    g.build()
+    assert torch.cuda.is_available()
+    return torch.device("cuda:0")
+
+
+@pytest.fixture(scope="module")
+def M(dev):
+    from paper_2003_04296_gb300 import minw
+    return minw
+
+
+def _run(dev, M, net_p, x_np, variant):
+    net = M.Net(M.layer_descs(net_p, dev), max_batch=x_np.shape[0], variant=variant)
+    logits = torch.empty((x_np.shape[0], net.out_features), dtype=torch.float32, device=dev)
+    net.forward(dev_tensor(x_np, dev), logits)
+    torch.cuda.synchronize()
+    out = logits.cpu().numpy()
+    net.close()
+    return out
+
+
+@pytest.mark.parametrize("bits_a,bits_w", [(1, 1), (2, 1), (2, 2), (3, 3)])
+def test_small_convnet(dev, M, bits_a, bits_w):
+    net_p = convnet_params(41, bits_a=bits_a, bits_w=bits_w, widths=(64, 64, 128, 128),
+                           pools=(False, True, False, True), fcs=(256,), classes=10, hw=16)
+    x = convnet_input(42, 3, hw=16)
+    got = _run(dev, M, net_p, x, M.VARIANT_POPC)
+    ref = N.convnet_forward(net_p, x)
+    assert_close(got, ref)
+    assert np.array_equal(got, ref)     # same fp32 operations in the same order
+
+
+def test_cifar_convnet_batch256_sampled(dev, M):
+    """The full Model-A-shaped ConvNet (128-128-P-256-256-P-512-512-P,
+    FC 1024-1024-10), 1-bit, batch 256; images 0 and 255 re-run by the oracle."""
+    net_p = convnet_params(2, bits_a=1, bits_w=1)
+    x = convnet_input(2, 256)
+    got = _run(dev, M, net_p, x, M.VARIANT_AUTO)
+    assert np.all(np.isfinite(got))
+    for i in (0, 255):
+        ref = N.convnet_forward(net_p, x[i:i + 1])
+        assert_close(got[i:i + 1], ref)
