@@ -1,0 +1,318 @@
+#!/usr/bin/env python3
+"""Throughput of the MINW-Net inference path on GB300.
+
+Workload: the CIFAR-shaped Model-A ConvNet forward (conv 128-128-P-256-256-P-
+512-512-P, FC 1024-1024-10), batch 256 per GPU, 1-bit activations x 1-bit
+weights in every hidden layer, fp32 image into the first layer, fp32 logits
+out.  Synthetic seeded data (U(-1,1) images, N(0,0.05) latent weights, folded
+BN maps); no dataset.  One step = one minw_forward over the batch.
+
+Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle on
+a bounded sample of the same workload instead.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "MINW-Net conv effective binary TOPS and forward images/s; fraction of roofline"
+BATCH = 256
+SEED = 2
+L2_FLUSH_BYTES = 256 << 20
+SMS = 152
+SM_MAX_MHZ = 2070.0
+POPC_PER_CLK_SM = 16          # measured: 16 popcounts per clock per SM
+THROTTLE = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown")
+
+
+def workload_config(bits_a, bits_w, batch, n_gpus, l2):
+    return {"workload": f"cifar_convnet_fwd_a{bits_a}w{bits_w}", "batch_per_gpu": batch,
+            "global_batch": batch * n_gpus, "input": "3x32x32 fp32 U(-1,1)",
+            "layers": "conv3x3 128,128,P,256,256,P,512,512,P; fc 1024,1024,10",
+            "bits_a": bits_a, "bits_w": bits_w, "first_layer": "fp32 input, quantized weights",
+            "parallelism": f"replicas x{n_gpus} (batch-sharded, no collective)", "l2": l2}
+
+
+def layer_macs(net_p, hw=32):
+    """MACs per image of each layer, in network order."""
+    out = []
+    size = hw
+    for L in net_p["layers"]:
+        if L["kind"] == "conv":
+            out.append(size * size * L["O"] * L["C"] * L["kh"] * L["kw"])
+            if L["pool"]:
+                size //= 2
+        else:
+            out.append(L["O"] * L["K"])
+    return out
+
+
+# ------------------------------------------------------------------ clocks --
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons during timing."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.out, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.out.close()
+
+    def summary(self):
+        if self.proc is None or not self.path:
+            return None
+        mhz, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    mhz.append(float(parts[1]))
+                    mx = float(parts[2])
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not mhz:
+            return None
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(mhz)}
+
+
+# --------------------------------------------------------------- reference --
+
+def oracle_images_per_s(net_p, x, max_seconds):
+    """Time the oracle's network forward image by image until max_seconds."""
+    from oracle import network as N
+    N.convnet_forward(net_p, x[:1])           # builds and loads the oracle
+    done, t0 = 0, time.perf_counter()
+    while done < x.shape[0]:
+        N.convnet_forward(net_p, x[done:done + 1])
+        done += 1
+        if time.perf_counter() - t0 >= max_seconds:
+            break
+    dt = time.perf_counter() - t0
+    return done / dt, done, dt
+
+
+def run_reference(args, rank):
+    if rank != 0:
+        return 0
+    from paper_2003_04296_gb300.inputs import convnet_input, convnet_params
+    net_p = convnet_params(SEED, bits_a=args.bits_a, bits_w=args.bits_w)
+    x = convnet_input(SEED, BATCH)
+    from oracle import network as N
+    # per-step sample sized so that warmup + steps stay within ~3 minutes
+    t0 = time.perf_counter()
+    N.convnet_forward(net_p, x[:1])
+    t_img = time.perf_counter() - t0
+    per_step = max(1, min(BATCH, int(150.0 / max(args.warmup + args.steps, 1) / max(t_img, 1e-3))))
+    for _ in range(args.warmup):
+        N.convnet_forward(net_p, x[:per_step])
+    times = []
+    for k in range(args.steps):
+        lo = (k * per_step) % BATCH
+        xs = x[lo:lo + per_step]
+        t0 = time.perf_counter()
+        N.convnet_forward(net_p, xs)
+        times.append(time.perf_counter() - t0)
+    sec = sum(times) / len(times)
+    ips = per_step / sec
+    sample = f"{per_step} of the {BATCH} images per step, single-threaded C oracle, extrapolated to images/s"
+    line = {"metric": METRIC, "value": ips, "unit": "images/s", "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True, "impl": "reference",
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(args.bits_a, args.bits_w, BATCH, args.gpus,
+                                      "flushed between steps (256 MiB write outside the timed events)"),
+            "cpu_baseline": {"value": ips, "unit": "images/s", "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": ips, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# --------------------------------------------------------------------- GPU --
+
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    import __graft_entry__ as g
+    if rank == 0:
+        g.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2003_04296_gb300 import minw
+    from paper_2003_04296_gb300.inputs import convnet_input, convnet_params
+
+    net_p = convnet_params(SEED, bits_a=args.bits_a, bits_w=args.bits_w)
+    x_np = convnet_input(SEED + 1000 * rank, BATCH)
+    net = minw.Net(minw.layer_descs(net_p, dev), max_batch=BATCH, variant=args.variant)
+    x = torch.from_numpy(x_np).to(dev)
+    logits = torch.empty((BATCH, net.out_features), dtype=torch.float32, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    net.enable_timing(True)
+    macs = layer_macs(net_p)
+    nl = net.launches
+
+    for _ in range(max(args.warmup, 3)):
+        net.forward(x, logits)
+    torch.cuda.synchronize()
+
+    step_ms, layer_ms = [], np.zeros(nl)
+    ev0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clk:
+        for k in range(args.steps):
+            flush.zero_()                       # evict the previous step from L2
+            ev0[k].record(stream)
+            net.forward(x, logits)
+            ev1[k].record(stream)
+            layer_ms += np.array(net.layer_times())   # waits for this step only
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+    for k in range(args.steps):
+        step_ms.append(ev0[k].elapsed_time(ev1[k]))
+    ms = sum(step_ms) / len(step_ms)
+    t = torch.tensor([ms], device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_max = float(t.item())
+
+    # end to end through the public API: pinned host input -> logits on host
+    x_host = torch.from_numpy(x_np).pin_memory()
+    out_host = torch.empty((BATCH, net.out_features), dtype=torch.float32).pin_memory()
+    net.enable_timing(False)
+    for _ in range(2):
+        net.forward_host(x_host, out_host)
+    e2e_s = []
+    if world > 1:
+        dist.barrier()
+    for _ in range(args.steps):
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        net.forward_host(x_host, out_host)
+        e2e_s.append(time.perf_counter() - t0)
+    e2e = torch.tensor([sum(e2e_s) / len(e2e_s)], device=dev)
+    if world > 1:
+        dist.all_reduce(e2e, op=dist.ReduceOp.MAX)
+    e2e_sec = float(e2e.item())
+
+    if rank != 0:
+        return 0
+
+    clocks = clk.summary()
+    layer_ms /= args.steps
+    total_macs = sum(macs) * BATCH
+    value = BATCH * world / (ms_max * 1e-3)
+    eff_tops = 2.0 * total_macs * world / (ms_max * 1e-3) / 1e12
+
+    # roofline of the dominant kernel: the quantized convolution (layers 2..n)
+    q_ms = float(layer_ms[1:].sum())
+    q_ops = 2.0 * sum(macs[1:]) * BATCH
+    achieved = q_ops / (q_ms * 1e-3) / 1e12
+    peak = POPC_PER_CLK_SM * 32 * 2 * SMS * SM_MAX_MHZ * 1e6 / 1e12
+    roofline = {"bound": "alu", "kernel": "conv_popc_kernel<1,1,4> (all quantized layers)",
+                "achieved": achieved, "peak": peak, "unit": "TOPS (2 x binary MAC)",
+                "frac": achieved / peak, "traffic": None,
+                "peak_basis": "16 popc/clk/SM x 32 MAC/popc x 2 ops x 152 SMs x 2070 MHz"}
+
+    cpu = None
+    if world == 1 and not args.skip_cpu:
+        ips, n_img, secs = oracle_images_per_s(net_p, x_np, args.cpu_seconds)
+        cpu = {"value": ips, "unit": "images/s", "cores": 1, "kind": "oracle",
+               "sample": f"{n_img} images of the batch through the single-threaded C oracle ({secs:.1f} s)"}
+
+    line = {"metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "b1", "data": "synthetic",
+            "config": workload_config(args.bits_a, args.bits_w, BATCH, world,
+                                      "flushed between steps (256 MiB write outside the timed events)"),
+            "eff_tops": eff_tops,
+            "layer_ms": [round(v, 5) for v in layer_ms.tolist()],
+            "roofline": roofline, "cpu_baseline": cpu,
+            "e2e": {"value": BATCH * world / e2e_sec, "unit": "images/s",
+                    "h2d_bytes_per_step": int(x_host.numel() * 4),
+                    "d2h_bytes_per_step": int(out_host.numel() * 4)},
+            "gpu_launches": nl * args.steps, "clocks": clocks}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["minw", "reference"], default="minw")
+    ap.add_argument("--bits-a", type=int, default=1)
+    ap.add_argument("--bits-w", type=int, default=1)
+    ap.add_argument("--variant", type=int, default=0, help="0 auto, 1 popcount, 2 tensor cores")
+    ap.add_argument("--cpu-seconds", type=float, default=20.0)
+    ap.add_argument("--skip-cpu", action="store_true")
+    args = ap.parse_args()
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        return run_reference(args, rank)
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    try:
+        return run_gpu(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

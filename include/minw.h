@@ -225,6 +225,20 @@ MINW_API minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_la
 MINW_API minw_status minw_forward(minw_net *net, const float *x, int32_t B,
                          float *logits, void *stream);
 
+/* Forward pass from HOST buffers: copies x_host [B][C][H][W] (fp32; pinned
+ * memory gives asynchronous copies) into a device staging buffer the net owns,
+ * runs minw_forward and copies the logits back into logits_host [B][O_last];
+ * returns after the stream has finished (the logits are ready). */
+MINW_API minw_status minw_forward_host(minw_net *net, const float *x_host, int32_t B,
+                              float *logits_host, void *stream);
+
+/* Per-layer timing: with on != 0 every later minw_forward records a CUDA
+ * event after each layer's kernel; minw_net_layer_times then writes the
+ * elapsed milliseconds of each layer of the most recent forward into ms
+ * (host array of minw_net_launches() floats), synchronising on the events. */
+MINW_API minw_status minw_net_enable_timing(minw_net *net, int32_t on);
+MINW_API minw_status minw_net_layer_times(minw_net *net, float *ms);
+
 /* Number of kernels one minw_forward launches. */
 MINW_API int32_t minw_net_launches(const minw_net *net);
 

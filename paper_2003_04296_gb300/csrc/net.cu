@@ -38,11 +38,17 @@ struct minw_net {
     uint32_t *buf[2] = {nullptr, nullptr};
     size_t buf_words = 0;
     std::vector<void *> owned;
+    float *x_stage = nullptr;         // device staging of minw_forward_host
+    float *logits_stage = nullptr;
+    size_t x_elems = 0, logit_elems = 0;
+    std::vector<cudaEvent_t> events;  // [0] before the first layer, [l+1] after layer l
+    bool timing = false;
 };
 
 static void net_free(minw_net *n) {
     if (!n) return;
     for (void *p : n->owned) cudaFree(p);
+    for (cudaEvent_t e : n->events) cudaEventDestroy(e);
     delete n;
 }
 
@@ -151,6 +157,14 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
         if (st != MINW_OK) { net_free(n); return st; }
     }
     n->buf_words = max_words;
+    n->x_elems = (size_t)max_batch * layers[0].C * layers[0].H * layers[0].W;
+    const LayerPlan &PL = n->L.back();
+    n->logit_elems = (size_t)max_batch * PL.O * PL.Hp * PL.Wp;
+    {
+        minw_status st = net_alloc(n, &n->x_stage, n->x_elems);
+        if (st == MINW_OK) st = net_alloc(n, &n->logits_stage, n->logit_elems);
+        if (st != MINW_OK) { net_free(n); return st; }
+    }
     if (cudaStreamSynchronize(s) != cudaSuccess) { net_free(n); return MINW_ECUDA; }
     *out = n;
     return MINW_OK;
@@ -160,6 +174,8 @@ minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits
     if (!net || !x || !logits || B <= 0 || B > net->max_batch) return MINW_EINVAL;
     const int nl = (int)net->L.size();
     int cur = 0;
+    cudaStream_t cs = (cudaStream_t)stream;
+    if (net->timing && cudaEventRecord(net->events[0], cs) != cudaSuccess) return MINW_ECUDA;
     for (int l = 0; l < nl; ++l) {
         const LayerPlan &P = net->L[l];
         const bool last = l == nl - 1;
@@ -177,8 +193,45 @@ minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits
                                  last ? nullptr : &P.qo, dst, y, P.variant, stream);
         }
         if (st != MINW_OK) return st;
+        if (net->timing && cudaEventRecord(net->events[l + 1], cs) != cudaSuccess) return MINW_ECUDA;
         cur ^= 1;
     }
+    return MINW_OK;
+}
+
+minw_status minw_forward_host(minw_net *net, const float *x_host, int32_t B, float *logits_host,
+                              void *stream) {
+    if (!net || !x_host || !logits_host || B <= 0 || B > net->max_batch) return MINW_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    const LayerPlan &F = net->L.front(), &PL = net->L.back();
+    const size_t xin = (size_t)B * F.C * F.H * F.W;
+    const size_t lout = (size_t)B * PL.O * PL.Hp * PL.Wp;
+    if (cudaMemcpyAsync(net->x_stage, x_host, xin * sizeof(float), cudaMemcpyHostToDevice, s) != cudaSuccess)
+        return MINW_ECUDA;
+    minw_status st = minw_forward(net, net->x_stage, B, net->logits_stage, stream);
+    if (st != MINW_OK) return st;
+    if (cudaMemcpyAsync(logits_host, net->logits_stage, lout * sizeof(float), cudaMemcpyDeviceToHost, s) !=
+        cudaSuccess)
+        return MINW_ECUDA;
+    return cudaStreamSynchronize(s) == cudaSuccess ? MINW_OK : MINW_ECUDA;
+}
+
+minw_status minw_net_enable_timing(minw_net *net, int32_t on) {
+    if (!net) return MINW_EINVAL;
+    if (on && net->events.empty()) {
+        net->events.resize(net->L.size() + 1);
+        for (auto &e : net->events)
+            if (cudaEventCreate(&e) != cudaSuccess) return MINW_ECUDA;
+    }
+    net->timing = on != 0;
+    return MINW_OK;
+}
+
+minw_status minw_net_layer_times(minw_net *net, float *ms) {
+    if (!net || !ms || net->events.empty()) return MINW_EINVAL;
+    if (cudaEventSynchronize(net->events.back()) != cudaSuccess) return MINW_ECUDA;
+    for (size_t l = 0; l < net->L.size(); ++l)
+        if (cudaEventElapsedTime(&ms[l], net->events[l], net->events[l + 1]) != cudaSuccess) return MINW_ECUDA;
     return MINW_OK;
 }
 

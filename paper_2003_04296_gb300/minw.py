@@ -60,6 +60,9 @@ SIGNATURES = {
     "minw_net_create": (ctypes.c_int, [ctypes.POINTER(LayerDesc), _I32, _I32, _I32, _P,
                                        ctypes.POINTER(ctypes.c_void_p)]),
     "minw_forward": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
+    "minw_forward_host": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
+    "minw_net_enable_timing": (ctypes.c_int, [_P, _I32]),
+    "minw_net_layer_times": (ctypes.c_int, [_P, _P]),
     "minw_net_launches": (_I32, [_P]),
     "minw_net_destroy": (None, [_P]),
     "minw_get_last_device_error": (ctypes.c_int, [_P]),
@@ -105,6 +108,16 @@ def _ptr(t):
     if not t.is_contiguous():
         raise ValueError("contiguous tensor expected")
     return ctypes.c_void_p(t.data_ptr())
+
+
+def _host_ptr(a):
+    if isinstance(a, torch.Tensor):
+        if a.is_cuda or not a.is_contiguous():
+            raise ValueError("contiguous host tensor expected")
+        return a.data_ptr()
+    if not a.flags["C_CONTIGUOUS"]:
+        raise ValueError("contiguous host array expected")
+    return a.ctypes.data
 
 
 def _stream(stream):
@@ -220,6 +233,23 @@ class Net:
     def forward(self, x, logits, stream=None):
         _check(lib().minw_forward(self._h, _ptr(x), x.shape[0], _ptr(logits), _stream(stream)),
                "minw_forward")
+
+    def forward_host(self, x_host, logits_host, stream=None):
+        """Host-buffer forward (numpy or pinned CPU tensors): copies in, runs,
+        copies the logits out and waits for them."""
+        _check(lib().minw_forward_host(self._h, ctypes.c_void_p(_host_ptr(x_host)), x_host.shape[0],
+                                       ctypes.c_void_p(_host_ptr(logits_host)), _stream(stream)),
+               "minw_forward_host")
+
+    def enable_timing(self, on=True):
+        _check(lib().minw_net_enable_timing(self._h, int(on)), "minw_net_enable_timing")
+
+    def layer_times(self):
+        """Milliseconds of each layer's kernel in the most recent forward."""
+        n = self.launches
+        arr = (ctypes.c_float * n)()
+        _check(lib().minw_net_layer_times(self._h, arr), "minw_net_layer_times")
+        return list(arr)
 
     @property
     def launches(self):
