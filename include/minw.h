@@ -171,6 +171,51 @@ MINW_API minw_status minw_conv_block(const uint32_t *act, int32_t B, int32_t C,
                             uint32_t *planes_out, float *y_out,
                             int32_t variant, void *stream);
 
+/* ---------------------------------------------------------------------- */
+/* Level-code layout and the tensor-core convolution                       */
+/* ---------------------------------------------------------------------- */
+
+/* "Codes" layout: one byte per value, the level in integer units (3-bit:
+ * quarters) written as an FP8 E4M3 number -- 0 -> 0x00, +-1 -> 0x38/0xB8,
+ * +-2 -> 0x40/0xC0, +-4 -> 0x48/0xC8.  Activations [N][H][W][C] (channels
+ * innermost), weights [O][kh][kw][C].  Products of two codes are exact, so a
+ * tensor-core FP8 contraction with fp32 accumulation returns the same integer
+ * accumulator as the popcount path.  C must be a multiple of 16 (128 for the
+ * convolution). */
+
+/* Quantize (Eq. inference) NCHW fp32 activations into NHWC codes. */
+MINW_API minw_status aqe_quantize_codes(const float *x, int32_t B, int32_t C, int32_t H,
+                                        int32_t W, const minw_quant *q, uint8_t *codes,
+                                        void *stream);
+
+/* Quantize latent weights [O][C][kh][kw] into codes [O][kh][kw][C];
+ * channel_scale as in minw_pack_weights. */
+MINW_API minw_status minw_pack_weight_codes(const float *w, int32_t O, int32_t C, int32_t kh,
+                                            int32_t kw, const minw_quant *q,
+                                            const float *channel_scale, uint8_t *codes,
+                                            void *stream);
+
+/* minw_conv2d on codes operands, run on the tcgen05 tensor cores.
+ * Supported: stride 1, C % 128 == 0, pad < kh, kw; otherwise
+ * MINW_EUNSUPPORTED.  bits_a / bits_w document the operands (1..3). */
+MINW_API minw_status minw_conv2d_codes(const uint8_t *act, int32_t B, int32_t C, int32_t H,
+                                       int32_t W, int32_t bits_a, const uint8_t *wgt,
+                                       int32_t O, int32_t kh, int32_t kw, int32_t bits_w,
+                                       int32_t stride, int32_t pad, int32_t *acc_out,
+                                       const float *scale, const float *shift, float *y_out,
+                                       void *stream);
+
+/* minw_conv_block on codes operands (tensor cores).  With q_out the quantized
+ * output goes to codes_out [B][Hp][Wp][O] (O % 16 == 0) and/or planes_out. */
+MINW_API minw_status minw_conv_block_codes(const uint8_t *act, int32_t B, int32_t C,
+                                           int32_t H, int32_t W, int32_t bits_a,
+                                           const uint8_t *wgt, int32_t O, int32_t kh,
+                                           int32_t kw, int32_t bits_w, int32_t stride,
+                                           int32_t pad, int32_t pool, const float *scale,
+                                           const float *shift, const minw_quant *q_out,
+                                           uint8_t *codes_out, uint32_t *planes_out,
+                                           float *y_out, void *stream);
+
 /* First layer (Sec. III-E): the fp32 image x [B][C][H][W] is NOT quantized;
  * the weights are.  w: latent fp32 weights [O][C][kh][kw]; q_w (host) and
  * channel_scale (nullable) quantize them as minw_pack_weights does; q_w NULL

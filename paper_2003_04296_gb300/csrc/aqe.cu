@@ -245,6 +245,63 @@ __global__ void pack_weights_kernel(const float *__restrict__ w, int O, int C, i
     }
 }
 
+// ---------------------------------------------------------------------------
+// Level codes: NCHW fp32 -> NHWC bytes (E4M3 levels), the tensor-core operand.
+// One warp owns 32 pixels x 32 channels of an image: lane l reads pixel p0+l of
+// each channel (coalesced along the row) and writes its 32 channel bytes with
+// two 16-byte stores.  C % 16 == 0.
+// ---------------------------------------------------------------------------
+
+__global__ void __launch_bounds__(256) quantize_codes_kernel(const float *__restrict__ x, int B, int C,
+                                                             int HW, QParams q, uint8_t *__restrict__ codes) {
+    const int groups = (C + 31) >> 5;
+    const int chunks = (HW + 31) >> 5;
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int64_t total = (int64_t)B * groups * chunks;
+    for (int64_t t = warp; t < total; t += nwarps) {
+        const int chunk = (int)(t % chunks);
+        const int g = (int)((t / chunks) % groups);
+        const int b = (int)(t / ((int64_t)chunks * groups));
+        const int p = chunk * 32 + lane;
+        if (p >= HW) continue;
+        const int c0 = g * 32;
+        const int cmax = min(32, C - c0);
+        uint32_t w[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+#pragma unroll 8
+        for (int c = 0; c < cmax; ++c) {
+            const float v = __ldcs(x + ((int64_t)b * C + c0 + c) * HW + p);
+            w[c >> 2] |= (uint32_t)level_code_e4m3(level_units(v * q.scale, q)) << ((c & 3) * 8);
+        }
+        uint4 *dst = reinterpret_cast<uint4 *>(codes + ((int64_t)b * HW + p) * C + c0);
+        dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+        if (cmax > 16) dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+    }
+}
+
+// Weights [O][C][kh][kw] -> codes [O][kh][kw][C]: one thread per 16 channels.
+__global__ void weight_codes_kernel(const float *__restrict__ w, int O, int C, int kh, int kw, QParams q,
+                                    const float *__restrict__ cscale, uint8_t *__restrict__ codes) {
+    const int G = C >> 4;
+    const int taps = kh * kw;
+    const int64_t total = (int64_t)O * taps * G;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        const int g = (int)(t % G);
+        const int tap = (int)((t / G) % taps);
+        const int o = (int)(t / ((int64_t)G * taps));
+        const float s = cscale ? cscale[o] : q.scale;
+        uint32_t wd[4] = {0u, 0u, 0u, 0u};
+        for (int c = 0; c < 16; ++c) {
+            const float v = w[((int64_t)o * C + g * 16 + c) * taps + tap];
+            wd[c >> 2] |= (uint32_t)level_code_e4m3(level_units(v * s, q)) << ((c & 3) * 8);
+        }
+        *reinterpret_cast<uint4 *>(codes + ((int64_t)o * taps + tap) * C + g * 16) =
+            make_uint4(wd[0], wd[1], wd[2], wd[3]);
+    }
+}
+
 }  // namespace minw
 
 // ===========================================================================
@@ -393,6 +450,30 @@ minw_status minw_pack_weights(const float *w, int32_t O, int32_t C, int32_t kh, 
         case 2: pack_weights_kernel<2><<<(unsigned)g, 256, 0, s>>>(w, O, C, kh, kw, qp, channel_scale, planes); break;
         default: pack_weights_kernel<3><<<(unsigned)g, 256, 0, s>>>(w, O, C, kh, kw, qp, channel_scale, planes); break;
     }
+    return launch_status();
+}
+
+minw_status aqe_quantize_codes(const float *x, int32_t B, int32_t C, int32_t H, int32_t W,
+                               const minw_quant *q, uint8_t *codes, void *stream) {
+    if (B <= 0 || C <= 0 || H <= 0 || W <= 0 || !valid_quant(q) || !x || !codes) return MINW_EINVAL;
+    if (C % 16 != 0 || !aligned16(codes)) return MINW_EUNSUPPORTED;
+    const int64_t HW = (int64_t)H * W;
+    if (HW > (1ll << 30)) return MINW_EUNSUPPORTED;
+    const int64_t warps = (int64_t)B * ((C + 31) / 32) * ((HW + 31) / 32);
+    const int64_t g = grid_for(warps * 32, 256);
+    quantize_codes_kernel<<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(x, B, C, (int)HW, to_qparams(q), codes);
+    return launch_status();
+}
+
+minw_status minw_pack_weight_codes(const float *w, int32_t O, int32_t C, int32_t kh, int32_t kw,
+                                   const minw_quant *q, const float *channel_scale, uint8_t *codes,
+                                   void *stream) {
+    if (O <= 0 || C <= 0 || kh <= 0 || kw <= 0 || !valid_quant(q) || !w || !codes) return MINW_EINVAL;
+    if (C % 16 != 0 || !aligned16(codes)) return MINW_EUNSUPPORTED;
+    const int64_t items = (int64_t)O * kh * kw * (C / 16);
+    const int64_t g = grid_for(items, 256);
+    weight_codes_kernel<<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(w, O, C, kh, kw, to_qparams(q),
+                                                                      channel_scale, codes);
     return launch_status();
 }
 

@@ -61,6 +61,15 @@ __device__ __forceinline__ uint32_t level_plane_bits(int v, int bits) {
     return r;
 }
 
+// FP8 E4M3 encoding of a level in integer units {0, +-1, +-2, +-4}: the
+// tensor-core operand of the "codes" layout (exact: powers of two).
+__host__ __device__ __forceinline__ uint8_t level_code_e4m3(int v) {
+    if (v == 0) return 0u;
+    const int m = v < 0 ? -v : v;
+    const uint32_t e = (m == 4) ? 9u : (m == 2) ? 8u : 7u;     // biased exponent, bias 7
+    return (uint8_t)(((v < 0) ? 0x80u : 0u) | (e << 3));
+}
+
 }  // namespace minw
 
 // Host-side helpers shared by the translation units.

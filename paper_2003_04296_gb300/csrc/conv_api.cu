@@ -35,20 +35,19 @@ minw_status make_conv_args(ConvArgs &a, const uint32_t *act, int B, int C, int H
     return MINW_OK;
 }
 
-// Per-shape choice.  The tensor-core path covers the shapes listed by
-// conv_tc_supported; everything else runs on the popcount path.
+// Per-shape choice for a layer whose input layout is still free (the network
+// planner): the tensor-core path wherever it covers the shape, the popcount
+// path elsewhere.
 int choose_variant(const ConvArgs &a, int requested) {
     if (requested == MINW_VARIANT_POPC) return MINW_VARIANT_POPC;
     if (requested == MINW_VARIANT_TC) return MINW_VARIANT_TC;
     return conv_tc_supported(a) ? MINW_VARIANT_TC : MINW_VARIANT_POPC;
 }
 
+// Packed-plane operands run on the popcount path; the tensor-core path takes
+// its operands in the codes layout (minw_conv2d_codes / minw_conv_block_codes).
 minw_status run_conv(const ConvArgs &a, int variant, cudaStream_t s) {
-    const int v = choose_variant(a, variant);
-    if (v == MINW_VARIANT_TC) {
-        if (!conv_tc_supported(a)) return MINW_EUNSUPPORTED;
-        return launch_conv_tc(a, s);
-    }
+    if (variant == MINW_VARIANT_TC) return MINW_EUNSUPPORTED;
     return launch_conv_popc(a, s);
 }
 
@@ -96,6 +95,67 @@ minw_status minw_conv_block(const uint32_t *act, int32_t B, int32_t C, int32_t H
     a.planes_out = planes_out;
     a.y_out = y_out;
     return run_conv(a, variant, (cudaStream_t)stream);
+}
+
+static minw_status make_codes_args(ConvArgs &a, const uint8_t *act, int B, int C, int H, int W, int bits_a,
+                                   const uint8_t *wgt, int O, int kh, int kw, int bits_w, int stride, int pad) {
+    if (B <= 0 || C <= 0 || H <= 0 || W <= 0 || O <= 0 || kh <= 0 || kw <= 0 || stride <= 0 || pad < 0)
+        return MINW_EINVAL;
+    if (bits_a < 1 || bits_a > 3 || bits_w < 1 || bits_w > 3) return MINW_EINVAL;
+    if (!act || !wgt || !aligned16(act) || !aligned16(wgt)) return MINW_EINVAL;
+    if (C % 128 != 0 || stride != 1 || pad >= kh || pad >= kw) return MINW_EUNSUPPORTED;
+    const int Ho = (H + 2 * pad - kh) / stride + 1;
+    const int Wo = (W + 2 * pad - kw) / stride + 1;
+    if (Ho <= 0 || Wo <= 0) return MINW_EINVAL;
+    if ((long long)B * H * W * C >= (1ll << 40)) return MINW_EUNSUPPORTED;
+    a = ConvArgs{};
+    a.act8 = act; a.wgt8 = wgt;
+    a.B = B; a.C = C; a.H = H; a.W = W; a.O = O; a.kh = kh; a.kw = kw;
+    a.stride = stride; a.pad = pad; a.Ho = Ho; a.Wo = Wo; a.NW = C / 32;
+    a.bits_a = bits_a; a.bits_w = bits_w;
+    a.M = (long long)B * Ho * Wo;
+    return MINW_OK;
+}
+
+minw_status minw_conv2d_codes(const uint8_t *act, int32_t B, int32_t C, int32_t H, int32_t W, int32_t bits_a,
+                              const uint8_t *wgt, int32_t O, int32_t kh, int32_t kw, int32_t bits_w,
+                              int32_t stride, int32_t pad, int32_t *acc_out, const float *scale,
+                              const float *shift, float *y_out, void *stream) {
+    ConvArgs a;
+    minw_status st = make_codes_args(a, act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad);
+    if (st != MINW_OK) return st;
+    if (!acc_out && !y_out) return MINW_EINVAL;
+    if (y_out && (!scale || !shift)) return MINW_EINVAL;
+    a.acc_out = acc_out;
+    a.y_out = y_out;
+    a.scale = scale;
+    a.shift = shift;
+    return launch_conv_tc(a, (cudaStream_t)stream);
+}
+
+minw_status minw_conv_block_codes(const uint8_t *act, int32_t B, int32_t C, int32_t H, int32_t W,
+                                  int32_t bits_a, const uint8_t *wgt, int32_t O, int32_t kh, int32_t kw,
+                                  int32_t bits_w, int32_t stride, int32_t pad, int32_t pool, const float *scale,
+                                  const float *shift, const minw_quant *q_out, uint8_t *codes_out,
+                                  uint32_t *planes_out, float *y_out, void *stream) {
+    ConvArgs a;
+    minw_status st = make_codes_args(a, act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad);
+    if (st != MINW_OK) return st;
+    if (!scale || !shift) return MINW_EINVAL;
+    if (q_out && (!valid_quant(q_out) || (!planes_out && !codes_out))) return MINW_EINVAL;
+    if (codes_out && (O % 16 != 0 || !aligned16(codes_out))) return MINW_EUNSUPPORTED;
+    if (!q_out && !y_out) return MINW_EINVAL;
+    if (pool != 0 && pool != 1) return MINW_EINVAL;
+    if (pool && ((a.Ho & 1) || (a.Wo & 1))) return MINW_EUNSUPPORTED;
+    a.scale = scale;
+    a.shift = shift;
+    a.pool = pool;
+    a.quant_out = q_out != nullptr;
+    if (q_out) a.qo = to_qparams(q_out);
+    a.planes_out = planes_out;
+    a.codes_out = q_out ? codes_out : nullptr;
+    a.y_out = y_out;
+    return launch_conv_tc(a, (cudaStream_t)stream);
 }
 
 }  // extern "C"

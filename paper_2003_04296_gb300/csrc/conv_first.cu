@@ -64,6 +64,7 @@ __global__ void __launch_bounds__(FIRST_NT) conv_first_kernel(const FirstArgs a)
     }
 
     uint32_t words[3] = {0u, 0u, 0u};
+    uint32_t cw[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
 #pragma unroll
     for (int oc = 0; oc < 32; ++oc) {
         if (oc < ochan) {
@@ -71,7 +72,9 @@ __global__ void __launch_bounds__(FIRST_NT) conv_first_kernel(const FirstArgs a)
             float y = fmaf(acc[oc], __ldg(a.scale + o), __ldg(a.shift + o));
             if (a.quant_out) {
                 y = fminf(fmaxf(y, -1.0f), 1.0f);
-                const uint32_t pb = level_plane_bits(level_units(y * a.qo.scale, a.qo), a.qo.bits);
+                const int lv = level_units(y * a.qo.scale, a.qo);
+                const uint32_t pb = level_plane_bits(lv, a.qo.bits);
+                cw[oc >> 2] |= (uint32_t)level_code_e4m3(lv) << ((oc & 3) * 8);
                 words[0] |= (pb & 1u) << oc;
                 words[1] |= ((pb >> 1) & 1u) << oc;
                 words[2] |= ((pb >> 2) & 1u) << oc;
@@ -79,7 +82,12 @@ __global__ void __launch_bounds__(FIRST_NT) conv_first_kernel(const FirstArgs a)
             if (a.y_out) a.y_out[((long long)b * a.O + o) * HoWo + pix] = y;
         }
     }
-    if (a.quant_out) {
+    if (a.quant_out && a.codes_out != nullptr) {
+        uint4 *dst = reinterpret_cast<uint4 *>(a.codes_out + m * a.O + g * 32);
+        dst[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
+        if (ochan > 16) dst[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
+    }
+    if (a.quant_out && a.planes_out != nullptr) {
         const int NWo = (a.O + 31) >> 5;
         uint32_t *dst = a.planes_out + (m * a.qo.bits) * NWo + g;
         for (int p = 0; p < a.qo.bits; ++p) dst[p * NWo] = words[p];

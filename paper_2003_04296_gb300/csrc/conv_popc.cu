@@ -335,6 +335,7 @@ __global__ void __launch_bounds__(NT) conv_popc_kernel(const ConvArgs a) {
         const int yo = pix / a.Wo, xo = pix - (pix / a.Wo) * a.Wo;
         const int opix = a.pool ? (yo / 2) * Wp + (xo / 2) : pix;
         uint32_t words[3] = {0u, 0u, 0u};
+        uint32_t cw[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
         for (int c = 0; c < 32; ++c) {
             const int cc = g * 32 + c;
             const int o = o0 + cc;
@@ -348,14 +349,22 @@ __global__ void __launch_bounds__(NT) conv_popc_kernel(const ConvArgs a) {
             float y = fmaf((float)v, __ldg(a.scale + o), __ldg(a.shift + o));
             if (a.quant_out) {
                 y = fminf(fmaxf(y, -1.0f), 1.0f);
-                const uint32_t pb = level_plane_bits(level_units(y * a.qo.scale, a.qo), a.qo.bits);
+                const int lv = level_units(y * a.qo.scale, a.qo);
+                const uint32_t pb = level_plane_bits(lv, a.qo.bits);
+                cw[c >> 2] |= (uint32_t)level_code_e4m3(lv) << ((c & 3) * 8);
                 words[0] |= (pb & 1u) << c;
                 words[1] |= ((pb >> 1) & 1u) << c;
                 words[2] |= ((pb >> 2) & 1u) << c;
             }
             if (a.y_out != nullptr) a.y_out[(b * a.O + o) * HpWp + opix] = y;
         }
-        if (a.quant_out) {
+        if (a.quant_out && a.codes_out != nullptr) {
+            const int ob = o0 + g * 32;
+            uint4 *dst = reinterpret_cast<uint4 *>(a.codes_out + (b * HpWp + opix) * a.O + ob);
+            if (ob < a.O) dst[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
+            if (ob + 16 < a.O) dst[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
+        }
+        if (a.quant_out && a.planes_out != nullptr) {
             const int wi = (o0 >> 5) + g;
             if (wi < NWo) {
                 uint32_t *dst = a.planes_out + ((b * HpWp + opix) * a.qo.bits) * NWo + wi;

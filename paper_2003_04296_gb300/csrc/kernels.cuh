@@ -21,7 +21,11 @@ struct ConvArgs {
     int pool;              // 2x2/2 max pool on the accumulator before BN
     int quant_out;         // HardTanh + quantize + pack into planes_out
     QParams qo;            // quantizer of the output
-    uint32_t *planes_out;  // [B][Hp][Wp][qo.bits][ceil(O/32)]
+    uint32_t *planes_out;  // [B][Hp][Wp][qo.bits][ceil(O/32)] (nullable)
+    uint8_t *codes_out;    // [B][Hp][Wp][O] E4M3 level codes (nullable; O % 16 == 0)
+    // tensor-core operands: E4M3 level codes
+    const uint8_t *act8;   // [B][H][W][C]
+    const uint8_t *wgt8;   // [O][kh][kw][C]
 };
 
 // First-layer convolution on the fp32 image (see conv_first.cu).
@@ -35,7 +39,8 @@ struct FirstArgs {
     const float *scale, *shift;
     int quant_out;
     QParams qo;
-    uint32_t *planes_out;      // [B][Ho][Wo][qo.bits][ceil(O/32)]
+    uint32_t *planes_out;      // [B][Ho][Wo][qo.bits][ceil(O/32)] (nullable)
+    uint8_t *codes_out;        // [B][Ho][Wo][O] E4M3 level codes (nullable)
     float *y_out;              // [B][O][Ho][Wo] (nullable)
 };
 

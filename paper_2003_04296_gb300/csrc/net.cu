@@ -23,7 +23,9 @@ struct LayerPlan {
     minw_layer_desc d;        // shape fields only; pointers are not kept
     int C, H, W, O, kh, kw, stride, pad, pool;
     int Ho, Wo, Hp, Wp;
-    uint32_t *wplanes = nullptr;   // packed weights (quantized layers)
+    uint32_t *wplanes = nullptr;   // packed weights (popcount layers)
+    uint8_t *wcodes = nullptr;     // weight codes (tensor-core layers)
+    int in_codes = 0;              // input arrives in the codes layout
     float *wlatent = nullptr;      // fp32 weights (first layer)
     float *wscale = nullptr;       // per-channel weight prescale (first layer)
     float *scale = nullptr;
@@ -130,27 +132,46 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
             }
         } else {
             if (P.C % 32 != 0) { net_free(n); return MINW_EUNSUPPORTED; }
-            const size_t words = (size_t)P.O * P.kh * P.kw * d.bits_w * (P.C / 32);
-            if ((st = net_alloc(n, &P.wplanes, words)) != MINW_OK) { net_free(n); return st; }
-            // the weights are [O][C][kh][kw]; an FC weight [O][K] with K in
-            // (c, h, w) order is the same array
-            st = minw_pack_weights(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, P.wplanes, stream);
-            if (st != MINW_OK) { net_free(n); return st; }
-            ConvArgs a;
-            st = make_conv_args(a, P.wplanes, max_batch, P.C, P.H, P.W, d.bits_in, P.wplanes, P.O,
-                                P.kh, P.kw, d.bits_w, P.stride, P.pad);
-            if (st != MINW_OK) { net_free(n); return st; }
+            if (P.pad >= P.kh || P.pad >= P.kw) { net_free(n); return MINW_EUNSUPPORTED; }
+            ConvArgs a{};
+            a.B = max_batch; a.C = P.C; a.H = P.H; a.W = P.W; a.O = P.O; a.kh = P.kh; a.kw = P.kw;
+            a.stride = P.stride; a.pad = P.pad; a.Ho = P.Ho; a.Wo = P.Wo; a.NW = P.C / 32;
+            a.bits_a = d.bits_in; a.bits_w = d.bits_w;
+            a.M = (long long)max_batch * P.Ho * P.Wo;
             a.pool = P.pool;
             a.quant_out = !last;
             if (!last) a.qo = to_qparams(&P.qo);
             P.variant = choose_variant(a, variant);
-        }
-        if (!last) {
-            const size_t words = (size_t)max_batch * P.Hp * P.Wp * d.bits_out * ((P.O + 31) / 32);
-            if (words > max_words) max_words = words;
+            if (P.variant == MINW_VARIANT_TC && !conv_tc_supported(a)) { net_free(n); return MINW_EUNSUPPORTED; }
         }
         pc = P.O; ph = P.Hp; pw = P.Wp; pbits = d.bits_out;
         n->L.push_back(P);
+    }
+    // input layouts follow the consumer's kernel; weights are quantized once
+    for (int l = 1; l < n_layers; ++l) {
+        LayerPlan &P = n->L[l];
+        const minw_layer_desc &d = layers[l];
+        P.in_codes = P.variant == MINW_VARIANT_TC;
+        minw_status st;
+        // the weights are [O][C][kh][kw]; an FC weight [O][K] with K in
+        // (c, h, w) order is the same array
+        if (P.in_codes) {
+            const size_t bytes = (size_t)P.O * P.kh * P.kw * P.C;
+            if ((st = net_alloc(n, &P.wcodes, bytes)) != MINW_OK) { net_free(n); return st; }
+            st = minw_pack_weight_codes(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, P.wcodes, stream);
+        } else {
+            const size_t words = (size_t)P.O * P.kh * P.kw * d.bits_w * (P.C / 32);
+            if ((st = net_alloc(n, &P.wplanes, words)) != MINW_OK) { net_free(n); return st; }
+            st = minw_pack_weights(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, P.wplanes, stream);
+        }
+        if (st != MINW_OK) { net_free(n); return st; }
+    }
+    for (int l = 0; l + 1 < n_layers; ++l) {
+        const LayerPlan &P = n->L[l];
+        const bool codes = n->L[l + 1].in_codes;
+        const size_t words = codes ? ((size_t)max_batch * P.Hp * P.Wp * P.O + 3) / 4
+                                   : (size_t)max_batch * P.Hp * P.Wp * P.d.bits_out * ((P.O + 31) / 32);
+        if (words > max_words) max_words = words;
     }
     for (int i = 0; i < 2; ++i) {
         minw_status st = net_alloc(n, &n->buf[i], max_words);
@@ -179,18 +200,45 @@ minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits
     for (int l = 0; l < nl; ++l) {
         const LayerPlan &P = net->L[l];
         const bool last = l == nl - 1;
-        uint32_t *dst = last ? nullptr : net->buf[cur];
-        float *y = last ? logits : nullptr;
+        const bool out_codes = !last && net->L[l + 1].in_codes;
+        void *dst = last ? nullptr : (void *)net->buf[cur];
         minw_status st;
         if (l == 0) {
-            st = minw_conv_first(x, B, P.C, P.H, P.W, P.wlatent, P.O, P.kh, P.kw, P.stride, P.pad,
-                                 P.d.bits_w > 0 ? &P.qw : nullptr, P.wscale, P.pool, P.scale, P.shift,
-                                 last ? nullptr : &P.qo, dst, y, stream);
+            FirstArgs a{};
+            a.x = x; a.w = P.wlatent; a.cscale = P.wscale;
+            a.quant_w = P.d.bits_w > 0;
+            if (a.quant_w) a.qw = to_qparams(&P.qw);
+            a.B = B; a.C = P.C; a.H = P.H; a.W = P.W; a.O = P.O; a.kh = P.kh; a.kw = P.kw;
+            a.stride = P.stride; a.pad = P.pad; a.Ho = P.Ho; a.Wo = P.Wo;
+            a.scale = P.scale; a.shift = P.shift;
+            a.quant_out = !last;
+            if (!last) a.qo = to_qparams(&P.qo);
+            a.planes_out = out_codes ? nullptr : (uint32_t *)dst;
+            a.codes_out = out_codes ? (uint8_t *)dst : nullptr;
+            a.y_out = last ? logits : nullptr;
+            st = launch_conv_first(a, cs);
         } else {
-            const uint32_t *src = net->buf[cur ^ 1];
-            st = minw_conv_block(src, B, P.C, P.H, P.W, P.d.bits_in, P.wplanes, P.O, P.kh, P.kw,
-                                 P.d.bits_w, P.stride, P.pad, P.pool, P.scale, P.shift,
-                                 last ? nullptr : &P.qo, dst, y, P.variant, stream);
+            const void *src = net->buf[cur ^ 1];
+            ConvArgs a{};
+            a.B = B; a.C = P.C; a.H = P.H; a.W = P.W; a.O = P.O; a.kh = P.kh; a.kw = P.kw;
+            a.stride = P.stride; a.pad = P.pad; a.Ho = P.Ho; a.Wo = P.Wo; a.NW = P.C / 32;
+            a.bits_a = P.d.bits_in; a.bits_w = P.d.bits_w;
+            a.M = (long long)B * P.Ho * P.Wo;
+            a.scale = P.scale; a.shift = P.shift; a.pool = P.pool;
+            a.quant_out = !last;
+            if (!last) a.qo = to_qparams(&P.qo);
+            a.planes_out = (!last && !out_codes) ? (uint32_t *)dst : nullptr;
+            a.codes_out = out_codes ? (uint8_t *)dst : nullptr;
+            a.y_out = last ? logits : nullptr;
+            if (P.in_codes) {
+                a.act8 = (const uint8_t *)src;
+                a.wgt8 = P.wcodes;
+                st = launch_conv_tc(a, cs);
+            } else {
+                a.act = (const uint32_t *)src;
+                a.wgt = P.wplanes;
+                st = launch_conv_popc(a, cs);
+            }
         }
         if (st != MINW_OK) return st;
         if (net->timing && cudaEventRecord(net->events[l + 1], cs) != cudaSuccess) return MINW_ECUDA;

@@ -57,6 +57,12 @@ SIGNATURES = {
                                        _I32, _I32, _I32, _P, _P, _QP, _P, _P, _I32, _P]),
     "minw_conv_first": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32, _I32,
                                        _QP, _P, _I32, _P, _P, _QP, _P, _P, _P]),
+    "aqe_quantize_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P]),
+    "minw_pack_weight_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
+    "minw_conv2d_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32,
+                                         _I32, _I32, _P, _P, _P, _P, _P]),
+    "minw_conv_block_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32,
+                                             _I32, _I32, _I32, _P, _P, _QP, _P, _P, _P, _P]),
     "minw_net_create": (ctypes.c_int, [ctypes.POINTER(LayerDesc), _I32, _I32, _I32, _P,
                                        ctypes.POINTER(ctypes.c_void_p)]),
     "minw_forward": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
@@ -195,6 +201,34 @@ def minw_conv_first(x, w, stride, pad, scale, shift, q_w=None, channel_scale=Non
                                  int(pool), _ptr(scale), _ptr(shift),
                                  ctypes.byref(q_out) if q_out is not None else None,
                                  _ptr(planes_out), _ptr(y_out), _stream(stream)), "minw_conv_first")
+
+
+def aqe_quantize_codes(x, q, codes, stream=None):
+    B, C, H, W = x.shape
+    _check(lib().aqe_quantize_codes(_ptr(x), B, C, H, W, ctypes.byref(q), _ptr(codes), _stream(stream)),
+           "aqe_quantize_codes")
+
+
+def minw_pack_weight_codes(w, q, codes, channel_scale=None, stream=None):
+    O, C, kh, kw = w.shape
+    _check(lib().minw_pack_weight_codes(_ptr(w), O, C, kh, kw, ctypes.byref(q), _ptr(channel_scale),
+                                        _ptr(codes), _stream(stream)), "minw_pack_weight_codes")
+
+
+def minw_conv2d_codes(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad, acc_out=None,
+                      scale=None, shift=None, y_out=None, stream=None):
+    _check(lib().minw_conv2d_codes(_ptr(act), B, C, H, W, bits_a, _ptr(wgt), O, kh, kw, bits_w, stride, pad,
+                                   _ptr(acc_out), _ptr(scale), _ptr(shift), _ptr(y_out), _stream(stream)),
+           "minw_conv2d_codes")
+
+
+def minw_conv_block_codes(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad, pool, scale, shift,
+                          q_out=None, codes_out=None, planes_out=None, y_out=None, stream=None):
+    _check(lib().minw_conv_block_codes(_ptr(act), B, C, H, W, bits_a, _ptr(wgt), O, kh, kw, bits_w, stride,
+                                       pad, int(pool), _ptr(scale), _ptr(shift),
+                                       ctypes.byref(q_out) if q_out is not None else None,
+                                       _ptr(codes_out), _ptr(planes_out), _ptr(y_out), _stream(stream)),
+           "minw_conv_block_codes")
 
 
 def minw_get_last_device_error(stream=None):

@@ -48,6 +48,18 @@ def test_small_convnet(dev, M, bits_a, bits_w):
     assert np.array_equal(got, ref)     # same fp32 operations in the same order
 
 
+@pytest.mark.parametrize("bits_a,bits_w", [(1, 1), (2, 2), (3, 3)])
+def test_small_convnet_tensor_cores(dev, M, bits_a, bits_w):
+    """Widths that are multiples of 128 put every quantized layer on the
+    tensor-core path (codes layout between layers)."""
+    net_p = convnet_params(43, bits_a=bits_a, bits_w=bits_w, widths=(128, 128, 256, 256),
+                           pools=(False, True, False, True), fcs=(256,), classes=10, hw=16)
+    x = convnet_input(44, 5, hw=16)
+    got = _run(dev, M, net_p, x, M.VARIANT_AUTO)
+    ref = N.convnet_forward(net_p, x)
+    assert np.array_equal(got, ref)
+
+
 def test_cifar_convnet_batch256_sampled(dev, M):
     """The full Model-A-shaped ConvNet (128-128-P-256-256-P-512-512-P,
     FC 1024-1024-10), 1-bit, batch 256; images 0 and 255 re-run by the oracle."""

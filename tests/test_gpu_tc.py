@@ -1,0 +1,174 @@
+"""GPU parity of the tensor-core path (level codes + tcgen05 FP8 contraction)
+against the oracle, through the C ABI: the codes layout, the convolution for
+all nine bit-width pairs on ragged tiles, the fused block epilogue, and
+accumulators at the largest magnitudes the workloads reach."""
+from itertools import product
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from oracle import oracle as O  # noqa: E402
+from paper_2003_04296_gb300.inputs import DEFAULT_THR, conv_problem  # noqa: E402
+from tests._gpu import dev_tensor, planes_view  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dev():
+    import __graft_entry__ as g
+    g.build()
+    assert torch.cuda.is_available()
+    return torch.device("cuda:0")
+
+
+@pytest.fixture(scope="module")
+def M(dev):
+    from paper_2003_04296_gb300 import minw
+    return minw
+
+
+def decode_e4m3(b):
+    """FP8 E4M3 bytes to values from the format's definition (1 sign bit,
+    4 exponent bits with bias 7, 3 mantissa bits); normal numbers only plus 0."""
+    b = b.astype(np.int64)
+    sign = np.where(b & 0x80, -1.0, 1.0)
+    e = (b >> 3) & 0xF
+    m = b & 7
+    v = sign * (1.0 + m / 8.0) * np.power(2.0, e - 7.0)
+    return np.where((b & 0x7F) == 0, 0.0, v)
+
+
+@pytest.mark.parametrize("bits", [1, 2, 3])
+@pytest.mark.parametrize("shape", [(2, 128, 5, 7), (1, 48, 3, 3), (3, 16, 1, 1)])
+def test_quantize_codes(dev, M, bits, shape):
+    B, C, H, W = shape
+    x = np.random.default_rng(C + bits).standard_normal(shape).astype(np.float32)
+    codes = torch.empty((B, H, W, C), dtype=torch.uint8, device=dev)
+    M.aqe_quantize_codes(dev_tensor(x, dev), M.quant(bits, DEFAULT_THR[bits]), codes)
+    lv = O.quantize(x, bits, DEFAULT_THR[bits]) * 2.0 ** O.units_shift(bits)
+    assert np.array_equal(decode_e4m3(codes.cpu().numpy()), lv.transpose(0, 2, 3, 1))
+
+
+@pytest.mark.parametrize("bits", [1, 2, 3])
+def test_weight_codes(dev, M, bits):
+    w = np.random.default_rng(bits).normal(0, 0.05, (40, 256, 3, 3)).astype(np.float32)
+    cs = (1.0 / np.abs(w.reshape(40, -1)).max(1)).astype(np.float32)
+    codes = torch.empty((40, 3, 3, 256), dtype=torch.uint8, device=dev)
+    M.minw_pack_weight_codes(dev_tensor(w, dev), M.quant(bits, DEFAULT_THR[bits]), codes,
+                             channel_scale=dev_tensor(cs, dev))
+    lv = O.quantize(w, bits, DEFAULT_THR[bits], cs) * 2.0 ** O.units_shift(bits)
+    assert np.array_equal(decode_e4m3(codes.cpu().numpy()), lv.transpose(0, 2, 3, 1))
+
+
+def _operands(dev, M, p):
+    B, C, H, W, O_ = p["B"], p["C"], p["H"], p["W"], p["O"]
+    act = torch.empty((B, H, W, C), dtype=torch.uint8, device=dev)
+    wgt = torch.empty((O_, p["kh"], p["kw"], C), dtype=torch.uint8, device=dev)
+    M.aqe_quantize_codes(dev_tensor(p["x"], dev), M.quant(p["bits_a"], p["thr_a"]), act)
+    M.minw_pack_weight_codes(dev_tensor(p["w"], dev), M.quant(p["bits_w"], p["thr_w"]), wgt,
+                             channel_scale=dev_tensor(p["w_scale"], dev))
+    return act, wgt
+
+
+def _ref_acc(p):
+    al = O.quantize(p["x"], p["bits_a"], p["thr_a"])
+    wl = O.quantize(p["w"], p["bits_w"], p["thr_w"], p["w_scale"])
+    return O.conv2d_levels(al, wl, p["stride"], p["pad"], p["bits_a"], p["bits_w"])
+
+
+TC_CASES = [
+    # B, C, H, W, O, k, pad
+    (2, 128, 9, 7, 70, 3, 1),       # ragged rows/columns of the pixel tile, ragged O
+    (3, 256, 16, 16, 256, 3, 1),    # BN = 256
+    (2, 128, 8, 8, 10, 1, 0),       # O = 10 -> one 16-wide channel tile
+    (130, 512, 4, 4, 20, 4, 0),     # fully connected over a 4x4 map, 2 image tiles
+    (2, 128, 1, 1, 300, 1, 0),      # two channel tiles, the second ragged
+    (1, 128, 14, 14, 64, 3, 1),     # 14x14: tiles overhang both edges
+]
+
+
+@pytest.mark.parametrize("case", TC_CASES)
+@pytest.mark.parametrize("ba,bw", list(product([1, 2, 3], [1, 2, 3])))
+def test_conv2d_codes(dev, M, case, ba, bw):
+    B, C, H, W, O_, k, pad = case
+    p = conv_problem(hash((case, ba, bw, "tc")) % 1000, B, C, H, W, O_, k, k, 1, pad, ba, bw, w_sigma=0.5)
+    act, wgt = _operands(dev, M, p)
+    acc = torch.full((B, O_, p["H"] + 2 * pad - k + 1, p["W"] + 2 * pad - k + 1), -7, dtype=torch.int32,
+                     device=dev)
+    y = torch.empty(acc.shape, dtype=torch.float32, device=dev)
+    M.minw_conv2d_codes(act, B, C, H, W, ba, wgt, O_, k, k, bw, 1, pad, acc_out=acc,
+                        scale=dev_tensor(p["scale"], dev), shift=dev_tensor(p["shift"], dev), y_out=y)
+    ref = _ref_acc(p)
+    got = acc.cpu().numpy()
+    assert np.array_equal(got, ref), f"{np.sum(got != ref)} of {ref.size} accumulators differ"
+    assert np.array_equal(y.cpu().numpy(), O.affine(ref, p["scale"], p["shift"]))
+    assert M.minw_get_last_device_error() == M.MINW_OK
+
+
+@pytest.mark.parametrize("ba,bw,hw", [(1, 1, 32), (2, 2, 16), (3, 3, 8), (2, 1, 16)])
+def test_conv_block_codes_pool(dev, M, ba, bw, hw):
+    B, C, O_ = 2, 128, 96
+    p = conv_problem(61 + ba + 3 * bw + hw, B, C, hw, hw, O_, 3, 3, 1, 1, ba, bw, w_sigma=0.5)
+    act, wgt = _operands(dev, M, p)
+    bo = ba
+    h2 = hw // 2
+    codes = torch.full((B, h2, h2, O_), 0x77, dtype=torch.uint8, device=dev)
+    planes = torch.full((M.packed_words(B, O_, h2, h2, bo),), -1, dtype=torch.int32, device=dev)
+    y = torch.empty((B, O_, h2, h2), dtype=torch.float32, device=dev)
+    M.minw_conv_block_codes(act, B, C, hw, hw, ba, wgt, O_, 3, 3, bw, 1, 1, 1, dev_tensor(p["scale"], dev),
+                            dev_tensor(p["shift"], dev), q_out=M.quant(bo, DEFAULT_THR[bo]), codes_out=codes,
+                            planes_out=planes, y_out=y)
+    acc = O.maxpool_i32(_ref_acc(p), 2, 2)
+    yr = O.hardtanh(O.affine(acc, p["scale"], p["shift"]))
+    assert np.array_equal(y.cpu().numpy(), yr)
+    lv = O.quantize(yr, bo, DEFAULT_THR[bo])
+    assert np.array_equal(planes_view(planes, B, h2, h2, bo, O_), O.pack(lv, bo))
+    assert np.array_equal(decode_e4m3(codes.cpu().numpy()),
+                          (lv * 2.0 ** O.units_shift(bo)).transpose(0, 2, 3, 1))
+
+
+def _adversarial(bits, C, k, hw, B=2, O_=64):
+    """Image 0 at the largest level everywhere (all products maximal); image 1
+    at the largest level on the first half of the channels and the smallest
+    non-zero level on the rest, so unit products follow large partial sums.
+    Even output channels use the largest weight level, odd ones mix in the
+    smaller levels."""
+    big, small = 1.0, (0.2 if bits == 3 else 1.0)
+    x = np.full((B, C, hw, hw), big, dtype=np.float32)
+    x[1, C // 2:] = small
+    w = np.full((O_, C, k, k), big, dtype=np.float32)
+    if bits == 3:
+        w[1::2, ::7] = 0.45
+        w[1::2, 3::5] = 0.2
+    elif bits == 2:
+        w[1::2, ::3] = 0.0
+    return dict(x=x, w=w, w_scale=np.ones(O_, np.float32), thr_a=DEFAULT_THR[bits], thr_w=DEFAULT_THR[bits],
+                scale=np.ones(O_, np.float32), shift=np.zeros(O_, np.float32), B=B, C=C, H=hw, W=hw, O=O_,
+                kh=k, kw=k, stride=1, pad=(k - 1) // 2 if k == 3 else 0, bits_a=bits, bits_w=bits)
+
+
+@pytest.mark.parametrize("bits,C,k,hw", [(3, 512, 3, 6), (1, 512, 4, 4), (1, 1024, 1, 1), (2, 512, 3, 5)])
+def test_exact_at_largest_magnitudes(dev, M, bits, C, k, hw):
+    """|acc| up to 16 * 4608 (3-bit, 512 x 3 x 3) and 8192 (1-bit FC) with
+    unit products next to the largest: the fp32 tensor-core accumulator must
+    reproduce every integer exactly."""
+    p = _adversarial(bits, C, k, hw)
+    act, wgt = _operands(dev, M, p)
+    Ho = hw + 2 * p["pad"] - k + 1
+    acc = torch.empty((p["B"], p["O"], Ho, Ho), dtype=torch.int32, device=dev)
+    M.minw_conv2d_codes(act, p["B"], C, hw, hw, bits, wgt, p["O"], k, k, bits, 1, p["pad"], acc_out=acc)
+    ref = _ref_acc(p)
+    assert np.abs(ref).max() == (16 if bits == 3 else 1) * C * k * k
+    assert np.array_equal(acc.cpu().numpy(), ref)
+
+
+def test_codes_argument_errors(dev, M):
+    t = torch.empty(4096, dtype=torch.uint8, device=dev)
+    a = torch.empty(64, dtype=torch.int32, device=dev)
+    with pytest.raises(M.MinwError):   # C % 128 != 0 is outside the tensor-core path
+        M.minw_conv2d_codes(t, 1, 64, 4, 4, 1, t, 8, 3, 3, 1, 1, 1, acc_out=a)
+    with pytest.raises(M.MinwError):   # stride 2 is outside the tensor-core path
+        M.minw_conv2d_codes(t, 1, 128, 4, 4, 1, t, 8, 3, 3, 1, 2, 1, acc_out=a)
