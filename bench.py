@@ -35,6 +35,20 @@ POPC_PER_CLK_SM = 16          # measured: 16 popcounts per clock per SM
 THROTTLE = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown")
 
 
+def _measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops"]), float(d.get("hbm_gbs", 6800.0))
+    except (OSError, KeyError, ValueError):
+        return 1900.0, 6800.0          # fallback figures of an earlier GB300 measurement
+
+
+BF16_TFLOPS, HBM_GBS = _measured_peaks()
+FP8_TFLOPS = 2.0 * BF16_TFLOPS
+
+
 def workload_config(bits_a, bits_w, batch, n_gpus, l2):
     return {"workload": f"cifar_convnet_fwd_a{bits_a}w{bits_w}", "batch_per_gpu": batch,
             "global_batch": batch * n_gpus, "input": "3x32x32 fp32 U(-1,1)",
@@ -252,14 +266,24 @@ def run_gpu(args, rank, world, local_rank):
     eff_tops = 2.0 * total_macs * world / (ms_max * 1e-3) / 1e12
 
     # roofline of the dominant kernel: the quantized convolution (layers 2..n)
+    variants = net.layer_variants()
     q_ms = float(layer_ms[1:].sum())
     q_ops = 2.0 * sum(macs[1:]) * BATCH
     achieved = q_ops / (q_ms * 1e-3) / 1e12
-    peak = POPC_PER_CLK_SM * 32 * 2 * SMS * SM_MAX_MHZ * 1e6 / 1e12
-    roofline = {"bound": "alu", "kernel": "conv_popc_kernel<1,1,4> (all quantized layers)",
-                "achieved": achieved, "peak": peak, "unit": "TOPS (2 x binary MAC)",
-                "frac": achieved / peak, "traffic": None,
-                "peak_basis": "16 popc/clk/SM x 32 MAC/popc x 2 ops x 152 SMs x 2070 MHz"}
+    if all(v == minw.VARIANT_TC for v in variants[1:]):
+        peak = FP8_TFLOPS
+        roofline = {"bound": "tensor", "kernel": "conv_tc_kernel (tcgen05 kind::f8f6f4, all quantized layers)",
+                    "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                    "traffic": None,
+                    "peak_basis": f"measured dense bf16 {BF16_TFLOPS:.1f} TFLOP/s (burst) x 2 for FP8 "
+                                  "(nominal fp8/bf16 ratio), of measured"}
+    else:
+        peak = POPC_PER_CLK_SM * 32 * 2 * SMS * SM_MAX_MHZ * 1e6 / 1e12
+        roofline = {"bound": "alu", "kernel": "conv_popc_kernel (all quantized layers)",
+                    "achieved": achieved, "peak": peak, "unit": "TOPS (2 x binary MAC)",
+                    "frac": achieved / peak, "traffic": None,
+                    "peak_basis": "16 popc/clk/SM x 32 MAC/popc x 2 ops x 152 SMs x 2070 MHz"}
+    roofline["layer_variants"] = variants
 
     cpu = None
     if world == 1 and not args.skip_cpu:
@@ -269,7 +293,8 @@ def run_gpu(args, rank, world, local_rank):
 
     line = {"metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "b1", "data": "synthetic",
+            "vs_baseline": None, "dtype": "e4m3" if all(v == minw.VARIANT_TC for v in variants[1:]) else "b1",
+            "data": "synthetic",
             "config": workload_config(args.bits_a, args.bits_w, BATCH, world,
                                       "flushed between steps (256 MiB write outside the timed events)"),
             "eff_tops": eff_tops,

@@ -284,6 +284,10 @@ MINW_API minw_status minw_forward_host(minw_net *net, const float *x_host, int32
 MINW_API minw_status minw_net_enable_timing(minw_net *net, int32_t on);
 MINW_API minw_status minw_net_layer_times(minw_net *net, float *ms);
 
+/* Kernel chosen for each layer (host array of minw_net_launches() ints):
+ * 0 for the fp32 first layer, else MINW_VARIANT_POPC or MINW_VARIANT_TC. */
+MINW_API minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants);
+
 /* Number of kernels one minw_forward launches. */
 MINW_API int32_t minw_net_launches(const minw_net *net);
 

@@ -70,6 +70,77 @@ __host__ __device__ __forceinline__ uint8_t level_code_e4m3(int v) {
     return (uint8_t)(((v < 0) ? 0x80u : 0u) | (e << 3));
 }
 
+// ---------------------------------------------------------------------------
+// Output quantization as integer thresholds.
+//
+// A hidden layer's output level is L(acc) = h(HardTanh(fmaf(acc, s, t))).
+// fmaf is monotone in acc, HardTanh and h are monotone, so L is a monotone
+// step function of the integer accumulator: with sigma = sign(s) (+1 for
+// s = 0), level index k(acc) = #{j : sigma * acc >= T_j} for per-channel
+// integer breakpoints T_1 <= ... <= T_{n-1} (n levels).  The breakpoints are
+// found by binary search on the very same fp32 operations, so the decision is
+// bit-identical to evaluating the chain element by element.
+// ---------------------------------------------------------------------------
+
+// Number of levels of a quantizer and the level index of a BN output y.
+__host__ __device__ __forceinline__ int num_levels(int bits) { return bits == 1 ? 2 : bits == 2 ? 3 : 7; }
+
+__device__ __forceinline__ int level_index_of_y(float y, const QParams &q) {
+    y = fminf(fmaxf(y, -1.0f), 1.0f);
+    const int u = level_units(y * q.scale, q);
+    if (q.bits == 1) return u > 0 ? 1 : 0;
+    if (q.bits == 2) return u + 1;
+    const int m = u < 0 ? -u : u;
+    const int e = (m == 4) ? 3 : m;                    // 0,1,2,4 -> 0,1,2,3
+    return 3 + (u < 0 ? -e : e);
+}
+
+// E4M3 code and plane bits (sign | code << 1) of level index k, packed tables.
+__device__ __forceinline__ uint32_t code_of_index(int k, int bits) {
+    if (bits == 1) return k ? 0x38u : 0xB8u;
+    if (bits == 2) return (uint32_t)((0x3800B8ull >> (8 * k)) & 0xFF);
+    return (uint32_t)((0x0048403800B8C0C8ull >> (8 * k)) & 0xFF);
+}
+__device__ __forceinline__ uint32_t planes_of_index(int k, int bits) {
+    if (bits == 1) return k ? 0u : 1u;
+    if (bits == 2) return (0x0203u >> (4 * k)) & 0x3u;     // idx 0: 3, 1: 0, 2: 2
+    return (uint32_t)((06420357ull >> (3 * k)) & 7ull);     // octal digits, idx 0 = low
+}
+
+// Breakpoints of channel o: T[0 .. n-2] and sigma, written to out[0 .. n-1].
+__device__ __forceinline__ void channel_thresholds(float s, float t, const QParams &q, float *out) {
+    const float sigma = (s < 0.0f) ? -1.0f : 1.0f;
+    const int n = num_levels(q.bits);
+    const int V = (1 << 24) - 1;                       // |acc| < 2^24 always
+    for (int j = 1; j < n; ++j) {
+        auto idx = [&](int v) { return level_index_of_y(fmaf((float)v * sigma, s, t), q); };
+        float T;
+        if (idx(-V) >= j) {
+            T = -INFINITY;
+        } else if (idx(V) < j) {
+            T = INFINITY;
+        } else {
+            int lo = -V, hi = V;                       // idx(lo) < j <= idx(hi)
+            while (hi - lo > 1) {
+                const int mid = lo + ((hi - lo) >> 1);
+                if (idx(mid) >= j) hi = mid; else lo = mid;
+            }
+            T = (float)hi;
+        }
+        out[j - 1] = T;
+    }
+    out[n - 1] = sigma;
+}
+
+// Level index of an accumulator (exact integer held in fp32) from the
+// breakpoints of its channel (n - 1 thresholds then sigma).
+__device__ __forceinline__ int level_index_of_acc(float acc, const float *thr, int n) {
+    const float v = acc * thr[n - 1];
+    int k = 0;
+    for (int j = 0; j < n - 1; ++j) k += (v >= thr[j]) ? 1 : 0;
+    return k;
+}
+
 }  // namespace minw
 
 // Host-side helpers shared by the translation units.

@@ -15,11 +15,15 @@
 //     bytes = level 0: the zero padding of the dequantized tensor), and
 //   - one TMA 2D box {128, BN} of the [O][kh][kw][C] weight codes,
 // both with 128-byte swizzle, i.e. the canonical K-major layout the MMA reads.
-// Warp roles (192 threads): warp 0 issues TMA, warp 1 owns TMEM and issues
-// MMAs (4 x K=32 per stage), warps 2-5 drain TMEM (one lane quarter each) and
-// run the fused epilogue: exact int conversion, 2x2 max pool via warp
-// shuffles, BN fmaf, HardTanh, quantize, and stores of the next layer's codes
-// or bit-planes (or raw int32 / fp32 NCHW outputs).
+// Persistent CTAs (one per SM) walk the tiles; the stage ring runs across tile
+// boundaries, and two TMEM accumulators let the epilogue of one tile overlap
+// the MMAs of the next.  Warp roles (192 threads): warp 0 issues TMA, warp 1
+// owns TMEM and issues MMAs (4 x K=32 per stage), warps 2-5 drain TMEM (one
+// lane quarter each) and run the fused epilogue: 2x2 max pool via warp
+// shuffles on the exact accumulators, then BN + HardTanh + quantize as
+// per-channel integer thresholds (bit-identical to the fp32 chain, see
+// common.cuh), and stores of the next layer's codes or bit-planes; raw int32
+// or fp32 NCHW outputs go through fmaf as in the paper's block.
 //
 // Every mbarrier wait is bounded (about one second of clock64); a wait that
 // runs out sets the device error flag read by minw_get_last_device_error, the
@@ -42,9 +46,11 @@ constexpr long long WAIT_CYCLES = 1ll << 31;
 
 struct Params {
     int B, C, H, W, O, kh, kw, pad, Ho, Wo;
-    int bw, bh, bb, nbx, nby;
+    int bw, bh, bb, nbx, nby, nbb, ntn;
     int BN, nck, nk, S;
     uint32_t stage_bytes, idesc, tmem_cols;
+    const float *thr;          // precomputed breakpoints [O][nlev] (nullable)
+    int nlev;                  // levels of the output quantizer
     int32_t *acc_out;
     float *y_out;
     const float *scale, *shift;
@@ -146,30 +152,55 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
 __device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
 __device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// Compile-time tables of the OUTB-bit output quantizer (see common.cuh).
+template <int OUTB>
+__device__ __forceinline__ uint32_t code_k(int k) {
+    if constexpr (OUTB == 1) return k ? 0x38u : 0xB8u;
+    else if constexpr (OUTB == 2) return (uint32_t)((0x3800B8u >> (8 * k)) & 0xFFu);
+    else return (uint32_t)((0x0048403800B8C0C8ull >> (8 * k)) & 0xFFull);
+}
+template <int OUTB>
+__device__ __forceinline__ uint32_t planes_k(int k) {
+    if constexpr (OUTB == 1) return k ? 0u : 1u;
+    else if constexpr (OUTB == 2) return (0x203u >> (4 * k)) & 0x3u;
+    else return (uint32_t)((06420357ull >> (3 * k)) & 7ull);
+}
+
+// OUTB: bits of the quantized output (0 when the launch writes none).
+template <int OUTB>
 __global__ void __launch_bounds__(NT, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const Params p) {
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint64_t *full = reinterpret_cast<uint64_t *>(smem + (size_t)p.S * p.stage_bytes);
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    // 1024-byte aligned base (the 128-byte swizzle repeats every 1024 bytes);
+    // pointer arithmetic on the shared array keeps the shared address space
+    uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    constexpr int NL = OUTB == 0 ? 1 : (OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7));
+    float *sthr = reinterpret_cast<float *>(smem + (size_t)p.S * p.stage_bytes);   // [O][NL]
+    const int thr_floats = OUTB ? p.O * NL : 0;
+    uint64_t *full = reinterpret_cast<uint64_t *>(sthr + ((thr_floats + 1) & ~1));
     uint64_t *empty = full + p.S;
-    uint64_t *accum = empty + p.S;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(accum + 1);
+    uint64_t *tfull = empty + p.S;            // [2] accumulator ready
+    uint64_t *tempty = tfull + 2;             // [2] accumulator drained
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(tempty + 2);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int tile_m = blockIdx.x, tile_n = blockIdx.y;
-    const int xb = tile_m % p.nbx;
-    const int yb = (tile_m / p.nbx) % p.nby;
-    const int bbk = tile_m / (p.nbx * p.nby);
-    const int x0 = xb * p.bw, y0 = yb * p.bh, b0 = bbk * p.bb;
-    const int o0 = tile_n * p.BN;
+    const int tiles_m = p.nbx * p.nby * p.nbb;
+    const int tiles = tiles_m * p.ntn;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < p.S; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
-        mbar_init(accum, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);
+        }
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     if (warp == 1) {
@@ -177,79 +208,115 @@ __global__ void __launch_bounds__(NT, 1)
                      "r"(p.tmem_cols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n");
     }
+    // output-quantizer breakpoints of every channel, in shared memory
+    if constexpr (OUTB > 0) {
+        if (p.thr != nullptr) {
+            for (int i = threadIdx.x; i < thr_floats; i += NT) sthr[i] = __ldg(p.thr + i);
+        } else {
+            for (int o = threadIdx.x; o < p.O; o += NT)
+                channel_thresholds(__ldg(p.scale + o), __ldg(p.shift + o), p.qo, sthr + o * NL);
+        }
+    }
     fence_before();
     __syncthreads();
     fence_after();
-    const uint32_t tmem_d = *tmem_slot;
+    const uint32_t tmem_base = *tmem_slot;
 
     if (warp == 0) {
         if (lane == 0) {
             // ---------------- TMA producer ----------------
             asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
             asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
-            int issued = 0;
-            for (int ks = 0; ks < p.nk; ++ks) {
-                const int s = ks % p.S, u = ks / p.S;
-                if (u > 0 && !mbar_wait(&empty[s], (u - 1) & 1)) break;
-                const int tap = ks / p.nck;
-                const int c0 = (ks - tap * p.nck) * 128;
-                const int ky = tap / p.kw, kx = tap - (tap / p.kw) * p.kw;
-                uint8_t *sa = smem + (size_t)s * p.stage_bytes;
-                mbar_expect_tx(&full[s], p.stage_bytes);
-                tma_load_4d(sa, &tmA, &full[s], c0, x0 - p.pad + kx, y0 - p.pad + ky, b0);
-                tma_load_2d(sa + A_BYTES, &tmB, &full[s], tap * p.C + c0, o0);
-                ++issued;
+            int g = 0, s = 0, lap = 0;             // stages issued, ring slot, ring lap
+            bool alive = true;
+            for (int t = blockIdx.x; t < tiles && alive; t += gridDim.x) {
+                const int tn = t / tiles_m, tm = t - tn * tiles_m;
+                const int xb = tm % p.nbx, yb = (tm / p.nbx) % p.nby, bbk = tm / (p.nbx * p.nby);
+                const int x0 = xb * p.bw - p.pad, y0 = yb * p.bh - p.pad, b0 = bbk * p.bb;
+                const int o0 = tn * p.BN;
+                int c0 = 0, kx = 0, ky = 0, kcol = 0;  // channel chunk, tap, weight column
+                for (int ks = 0; ks < p.nk; ++ks, ++g) {
+                    // slot reuse: wait until the MMAs of the previous lap released it
+                    if (lap > 0 && !mbar_wait(&empty[s], (lap - 1) & 1)) { alive = false; break; }
+                    uint8_t *sa = smem + (size_t)s * p.stage_bytes;
+                    mbar_expect_tx(&full[s], p.stage_bytes);
+                    tma_load_4d(sa, &tmA, &full[s], c0, x0 + kx, y0 + ky, b0);
+                    tma_load_2d(sa + A_BYTES, &tmB, &full[s], kcol, o0);
+                    kcol += 128;
+                    c0 += 128;
+                    if (c0 == p.C) {
+                        c0 = 0;
+                        if (++kx == p.kw) { kx = 0; ++ky; }
+                    }
+                    if (++s == p.S) { s = 0; ++lap; }
+                }
             }
             // drain: every issued load has landed before the CTA can exit
-            for (int j = issued > p.S ? issued - p.S : 0; j < issued; ++j)
+            for (int j = g > p.S ? g - p.S : 0; j < g; ++j)
                 if (!mbar_wait(&full[j % p.S], (j / p.S) & 1)) break;
         }
     } else if (warp == 1) {
         if (lane == 0) {
             // ---------------- MMA issuer ----------------
-            for (int ks = 0; ks < p.nk; ++ks) {
-                const int s = ks % p.S, u = ks / p.S;
-                if (!mbar_wait(&full[s], u & 1)) break;
+            int s = 0, i = 0;
+            uint32_t fphase = 0;
+            bool alive = true;
+            const uint32_t sbase = smem_u32(smem);
+            for (int t = blockIdx.x; t < tiles && alive; t += gridDim.x, ++i) {
+                const int ab = i & 1, use = i >> 1;
+                if (use > 0 && !mbar_wait(&tempty[ab], (use - 1) & 1)) break;
                 fence_after();
-                const uint32_t sa = smem_u32(smem + (size_t)s * p.stage_bytes);
-                const uint64_t adesc = sw128_desc(sa);
-                const uint64_t bdesc = sw128_desc(sa + A_BYTES);
+                const uint32_t tmem_d = tmem_base + (uint32_t)(ab * p.BN);
+                for (int ks = 0; ks < p.nk; ++ks) {
+                    if (!mbar_wait(&full[s], fphase)) { alive = false; break; }
+                    fence_after();
+                    const uint32_t sa = sbase + (uint32_t)s * p.stage_bytes;
+                    const uint64_t adesc = sw128_desc(sa);
+                    const uint64_t bdesc = sw128_desc(sa + A_BYTES);
 #pragma unroll
-                for (int kk = 0; kk < 4; ++kk)
-                    mma_f8(tmem_d, adesc + 2 * kk, bdesc + 2 * kk, p.idesc, (ks | kk) != 0);
-                mma_commit(&empty[s]);
+                    for (int kk = 0; kk < 4; ++kk)
+                        mma_f8(tmem_d, adesc + 2 * kk, bdesc + 2 * kk, p.idesc, (ks | kk) != 0);
+                    mma_commit(&empty[s]);
+                    if (++s == p.S) { s = 0; fphase ^= 1; }
+                }
+                mma_commit(&tfull[ab]);
             }
-            mma_commit(accum);
         }
     } else {
         // ---------------- epilogue: warps 2..5 ----------------
         const int q = warp & 3;                   // TMEM lane quarter of this warp
         const int r = q * 32 + lane;              // tile row = output pixel
-        const int b = b0 + r / (p.bh * p.bw);
-        const int y = y0 + (r / p.bw) % p.bh;
-        const int x = x0 + r % p.bw;
-        const bool valid = b < p.B && y < p.Ho && x < p.Wo;
-        const bool ok = mbar_wait(accum, 0);
-        fence_after();
-        const bool writer = valid && (!p.pool || ((x & 1) == 0 && (y & 1) == 0));
         const int Hp = p.pool ? p.Ho / 2 : p.Ho, Wp = p.pool ? p.Wo / 2 : p.Wo;
-        const int yp = p.pool ? y / 2 : y, xp = p.pool ? x / 2 : x;
-        const long long opix = ((long long)b * Hp + yp) * Wp + xp;
         const int NWo = (p.O + 31) >> 5;
-        uint32_t pw[3] = {0u, 0u, 0u};
-        if (ok) {
+        const int rb = r / (p.bh * p.bw), ry = (r / p.bw) % p.bh, rx = r % p.bw;
+        int i = 0;
+        for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++i) {
+            const int ab = i & 1, use = i >> 1;
+            const int tn = t / tiles_m, tm = t - tn * tiles_m;
+            const int xb = tm % p.nbx, yb = (tm / p.nbx) % p.nby, bbk = tm / (p.nbx * p.nby);
+            const int b = bbk * p.bb + rb;
+            const int y = yb * p.bh + ry;
+            const int x = xb * p.bw + rx;
+            const int o0 = tn * p.BN;
+            const bool valid = b < p.B && y < p.Ho && x < p.Wo;
+            const bool writer = valid && (!p.pool || ((x & 1) == 0 && (y & 1) == 0));
+            const int yp = p.pool ? y / 2 : y, xp = p.pool ? x / 2 : x;
+            const long long opix = ((long long)b * Hp + yp) * Wp + xp;
+            if (!mbar_wait(&tfull[ab], use & 1)) break;
+            fence_after();
+            uint32_t pw[3] = {0u, 0u, 0u};
             for (int ch = 0; ch < p.BN / 16; ++ch) {
                 __syncwarp();
                 uint32_t v[16];
-                tmem_ld16(tmem_d + ((uint32_t)(q * 32) << 16) + (uint32_t)(ch * 16), v);
-                int a[16];
+                tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * p.BN + ch * 16), v);
+                float a[16];
 #pragma unroll
-                for (int j = 0; j < 16; ++j) a[j] = __float2int_rn(__uint_as_float(v[j]));
+                for (int j = 0; j < 16; ++j) a[j] = __uint_as_float(v[j]);
                 if (p.pool) {
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
-                        a[j] = max(a[j], __shfl_xor_sync(0xffffffffu, a[j], 1));
-                        a[j] = max(a[j], __shfl_xor_sync(0xffffffffu, a[j], p.bw));
+                        a[j] = fmaxf(a[j], __shfl_xor_sync(0xffffffffu, a[j], 1));
+                        a[j] = fmaxf(a[j], __shfl_xor_sync(0xffffffffu, a[j], p.bw));
                     }
                 }
                 const int ob = o0 + ch * 16;
@@ -257,51 +324,79 @@ __global__ void __launch_bounds__(NT, 1)
 #pragma unroll
                     for (int j = 0; j < 16; ++j)
                         if (ob + j < p.O)
-                            p.acc_out[(((long long)b * p.O + ob + j) * p.Ho + y) * p.Wo + x] = a[j];
+                            p.acc_out[(((long long)b * p.O + ob + j) * p.Ho + y) * p.Wo + x] = __float2int_rn(a[j]);
                 }
-                if (writer && (p.y_out != nullptr || p.quant_out)) {
-                uint32_t cw[4] = {0u, 0u, 0u, 0u};
-                uint32_t bits16[3] = {0u, 0u, 0u};
+                if (p.y_out != nullptr && writer) {
 #pragma unroll
-                for (int j = 0; j < 16; ++j) {
-                    const int o = ob + j;
-                    if (o >= p.O) break;
-                    float yv = fmaf((float)a[j], __ldg(p.scale + o), __ldg(p.shift + o));
-                    if (p.quant_out) {
-                        yv = fminf(fmaxf(yv, -1.0f), 1.0f);
-                        const int lv = level_units(yv * p.qo.scale, p.qo);
-                        cw[j >> 2] |= (uint32_t)level_code_e4m3(lv) << ((j & 3) * 8);
-                        const uint32_t pb = level_plane_bits(lv, p.qo.bits);
-                        bits16[0] |= (pb & 1u) << j;
-                        bits16[1] |= ((pb >> 1) & 1u) << j;
-                        bits16[2] |= ((pb >> 2) & 1u) << j;
-                    }
-                    if (p.y_out != nullptr)
-                        p.y_out[(((long long)b * p.O + o) * Hp + yp) * Wp + xp] = yv;
-                }
-                if (p.quant_out && p.codes_out != nullptr)
-                    *reinterpret_cast<uint4 *>(p.codes_out + opix * p.O + ob) = make_uint4(cw[0], cw[1], cw[2], cw[3]);
-                if (p.quant_out && p.planes_out != nullptr) {
-                    const int half = (ob >> 4) & 1;
-#pragma unroll
-                    for (int k = 0; k < 3; ++k) pw[k] |= bits16[k] << (16 * half);
-                    if (half == 1 || ch == p.BN / 16 - 1 || ob + 16 >= p.O) {
-                        uint32_t *dst = p.planes_out + (opix * p.qo.bits) * NWo + (ob >> 5);
-                        for (int k = 0; k < p.qo.bits; ++k) dst[k * NWo] = pw[k];
-                        pw[0] = pw[1] = pw[2] = 0u;
+                    for (int j = 0; j < 16; ++j) {
+                        const int o = ob + j;
+                        if (o < p.O) {
+                            float yv = fmaf(a[j], __ldg(p.scale + o), __ldg(p.shift + o));
+                            if (OUTB > 0) yv = fminf(fmaxf(yv, -1.0f), 1.0f);
+                            p.y_out[(((long long)b * p.O + o) * Hp + yp) * Wp + xp] = yv;
+                        }
                     }
                 }
-                }  // writer
+                if constexpr (OUTB > 0) {
+                    if (writer) {
+                        int kq[16];
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            const int o = min(ob + j, p.O - 1);
+                            const float *th = sthr + o * NL;
+                            const float vv = a[j] * th[NL - 1];
+                            int k = 0;
+#pragma unroll
+                            for (int u = 0; u < NL - 1; ++u) k += (vv >= th[u]) ? 1 : 0;
+                            kq[j] = k;
+                        }
+                        if (p.codes_out != nullptr) {
+                            uint32_t cw[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) cw[j >> 2] |= code_k<OUTB>(kq[j]) << ((j & 3) * 8);
+                            *reinterpret_cast<uint4 *>(p.codes_out + opix * p.O + ob) =
+                                make_uint4(cw[0], cw[1], cw[2], cw[3]);
+                        }
+                        if (p.planes_out != nullptr) {
+                            uint32_t bits16[3] = {0u, 0u, 0u};
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) {
+                                const uint32_t pb = (ob + j < p.O) ? planes_k<OUTB>(kq[j]) : 0u;
+#pragma unroll
+                                for (int u = 0; u < OUTB; ++u) bits16[u] |= ((pb >> u) & 1u) << j;
+                            }
+                            const int half = (ob >> 4) & 1;
+#pragma unroll
+                            for (int u = 0; u < OUTB; ++u) pw[u] |= bits16[u] << (16 * half);
+                            if (half == 1 || ch == p.BN / 16 - 1 || ob + 16 >= p.O) {
+                                uint32_t *dst = p.planes_out + (opix * OUTB) * NWo + (ob >> 5);
+#pragma unroll
+                                for (int u = 0; u < OUTB; ++u) {
+                                    dst[u * NWo] = pw[u];
+                                    pw[u] = 0u;
+                                }
+                            }
+                        }
+                    }
+                }
             }
+            fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[ab]);
         }
-        __syncwarp();
-        fence_before();
     }
     __syncthreads();
     if (warp == 1) {
         fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_d), "r"(p.tmem_cols));
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(p.tmem_cols));
     }
+}
+
+// Breakpoints of every channel (see channel_thresholds): one thread per channel.
+__global__ void thresholds_kernel(const float *__restrict__ scale, const float *__restrict__ shift, int O,
+                                  QParams q, float *__restrict__ out) {
+    const int o = blockIdx.x * blockDim.x + threadIdx.x;
+    if (o < O) channel_thresholds(scale[o], shift[o], q, out + o * num_levels(q.bits));
 }
 
 // ---------------------------------------------------------------------------
@@ -364,15 +459,20 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     p.Ho = a.Ho; p.Wo = a.Wo;
     p.nck = a.C / 128;
     p.nk = a.kh * a.kw * p.nck;
+    p.nbb = (a.B + p.bb - 1) / p.bb;
+    p.ntn = (a.O + p.BN - 1) / p.BN;
+    p.nlev = a.quant_out ? num_levels(a.qo.bits) : 0;
+    p.thr = a.thr;
     p.stage_bytes = (uint32_t)(A_BYTES + p.BN * 128);
-    const size_t budget = (p.BN <= 128) ? 110 * 1024 : 200 * 1024;
+    const size_t thr_bytes = a.quant_out ? ((size_t)a.O * p.nlev + 2) * sizeof(float) : 0;
+    const size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes;
     int S = (int)(budget / p.stage_bytes);
-    if (S > 6) S = 6;
-    if (S < 2) S = 2;
+    if (S > 8) S = 8;
+    if (S < 2) return MINW_EUNSUPPORTED;
     p.S = S;
     p.idesc = (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(p.BN >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
     uint32_t cols = 32;
-    while ((int)cols < p.BN) cols <<= 1;
+    while ((int)cols < 2 * p.BN) cols <<= 1;          // two accumulators
     p.tmem_cols = cols;
     p.acc_out = a.acc_out; p.y_out = a.y_out; p.scale = a.scale; p.shift = a.shift;
     p.pool = a.pool; p.quant_out = a.quant_out; p.qo = a.qo;
@@ -401,9 +501,13 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return MINW_ECUDA;
     }
-    const int nbb = (a.B + p.bb - 1) / p.bb;
-    pl.grid = dim3((unsigned)(p.nbx * p.nby * nbb), (unsigned)((a.O + p.BN - 1) / p.BN));
-    pl.smem = (size_t)p.S * p.stage_bytes + 1024 + 256;
+    const int tiles = p.nbx * p.nby * p.nbb * p.ntn;
+    const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
+    pl.grid = dim3((unsigned)(tiles < sms ? tiles : sms));
+    pl.smem = (size_t)p.S * p.stage_bytes + 1024 + 256 + thr_bytes;
+    // more than half of an SM's shared memory: exactly one CTA (and one TMEM
+    // allocation) per SM
+    if (pl.smem < 120 * 1024) pl.smem = 120 * 1024;
     return MINW_OK;
 }
 
@@ -412,9 +516,16 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
 bool conv_tc_supported(const ConvArgs &a) {
     tc::Params p{};
     if (!tc::plan_shape(a, p)) return false;
+    if (a.quant_out && (size_t)a.O * num_levels(a.qo.bits) * sizeof(float) > 64 * 1024) return false;
     if (a.quant_out && a.codes_out != nullptr && a.O % 16 != 0) return false;
     if (a.acc_out != nullptr && a.pool) return false;
     return true;
+}
+
+minw_status launch_thresholds(const float *scale, const float *shift, int O, const QParams &q, float *out,
+                              cudaStream_t s) {
+    tc::thresholds_kernel<<<(O + 127) / 128, 128, 0, s>>>(scale, shift, O, q, out);
+    return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
 }
 
 minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
@@ -423,14 +534,17 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
     tc::Plan pl;
     minw_status st = tc::make_plan(a, pl);
     if (st != MINW_OK) return st;
-    static size_t configured = 0;
-    if (pl.smem > configured) {
-        if (cudaFuncSetAttribute(tc::conv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem) !=
-            cudaSuccess)
+    const int outb = a.quant_out ? a.qo.bits : 0;
+    static size_t configured[4] = {0, 0, 0, 0};
+    void (*kern)(const CUtensorMap, const CUtensorMap, const tc::Params) =
+        outb == 1 ? tc::conv_tc_kernel<1> : outb == 2 ? tc::conv_tc_kernel<2> : outb == 3 ? tc::conv_tc_kernel<3>
+                                                                                         : tc::conv_tc_kernel<0>;
+    if (pl.smem > configured[outb]) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem) != cudaSuccess)
             return MINW_ECUDA;
-        configured = pl.smem;
+        configured[outb] = pl.smem;
     }
-    tc::conv_tc_kernel<<<pl.grid, tc::NT, pl.smem, s>>>(pl.tmA, pl.tmB, pl.p);
+    kern<<<pl.grid, tc::NT, pl.smem, s>>>(pl.tmA, pl.tmB, pl.p);
     return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
 }
 

@@ -26,6 +26,7 @@ struct ConvArgs {
     // tensor-core operands: E4M3 level codes
     const uint8_t *act8;   // [B][H][W][C]
     const uint8_t *wgt8;   // [O][kh][kw][C]
+    const float *thr;      // output-quantizer breakpoints [O][levels] (nullable: computed in-kernel)
 };
 
 // First-layer convolution on the fp32 image (see conv_first.cu).
@@ -54,5 +55,7 @@ int choose_variant(const ConvArgs &a, int requested);
 minw_status run_conv(const ConvArgs &a, int variant, cudaStream_t s);
 minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s);
 bool conv_tc_supported(const ConvArgs &a);
+minw_status launch_thresholds(const float *scale, const float *shift, int O, const QParams &q, float *out,
+                              cudaStream_t s);
 
 }  // namespace minw

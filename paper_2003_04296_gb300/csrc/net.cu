@@ -25,6 +25,7 @@ struct LayerPlan {
     int Ho, Wo, Hp, Wp;
     uint32_t *wplanes = nullptr;   // packed weights (popcount layers)
     uint8_t *wcodes = nullptr;     // weight codes (tensor-core layers)
+    float *thr = nullptr;          // output-quantizer breakpoints (tensor-core layers)
     int in_codes = 0;              // input arrives in the codes layout
     float *wlatent = nullptr;      // fp32 weights (first layer)
     float *wscale = nullptr;       // per-channel weight prescale (first layer)
@@ -159,6 +160,11 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
             const size_t bytes = (size_t)P.O * P.kh * P.kw * P.C;
             if ((st = net_alloc(n, &P.wcodes, bytes)) != MINW_OK) { net_free(n); return st; }
             st = minw_pack_weight_codes(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, P.wcodes, stream);
+            if (st == MINW_OK && l + 1 < n_layers) {
+                const QParams qo = to_qparams(&P.qo);
+                st = net_alloc(n, &P.thr, (size_t)P.O * num_levels(qo.bits));
+                if (st == MINW_OK) st = launch_thresholds(P.scale, P.shift, P.O, qo, P.thr, s);
+            }
         } else {
             const size_t words = (size_t)P.O * P.kh * P.kw * d.bits_w * (P.C / 32);
             if ((st = net_alloc(n, &P.wplanes, words)) != MINW_OK) { net_free(n); return st; }
@@ -233,6 +239,7 @@ minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits
             if (P.in_codes) {
                 a.act8 = (const uint8_t *)src;
                 a.wgt8 = P.wcodes;
+                a.thr = P.thr;
                 st = launch_conv_tc(a, cs);
             } else {
                 a.act = (const uint32_t *)src;
@@ -280,6 +287,12 @@ minw_status minw_net_layer_times(minw_net *net, float *ms) {
     if (cudaEventSynchronize(net->events.back()) != cudaSuccess) return MINW_ECUDA;
     for (size_t l = 0; l < net->L.size(); ++l)
         if (cudaEventElapsedTime(&ms[l], net->events[l], net->events[l + 1]) != cudaSuccess) return MINW_ECUDA;
+    return MINW_OK;
+}
+
+minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants) {
+    if (!net || !variants) return MINW_EINVAL;
+    for (size_t l = 0; l < net->L.size(); ++l) variants[l] = l == 0 ? 0 : net->L[l].variant;
     return MINW_OK;
 }
 

@@ -69,6 +69,7 @@ SIGNATURES = {
     "minw_forward_host": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
     "minw_net_enable_timing": (ctypes.c_int, [_P, _I32]),
     "minw_net_layer_times": (ctypes.c_int, [_P, _P]),
+    "minw_net_layer_variants": (ctypes.c_int, [_P, _P]),
     "minw_net_launches": (_I32, [_P]),
     "minw_net_destroy": (None, [_P]),
     "minw_get_last_device_error": (ctypes.c_int, [_P]),
@@ -283,6 +284,13 @@ class Net:
         n = self.launches
         arr = (ctypes.c_float * n)()
         _check(lib().minw_net_layer_times(self._h, arr), "minw_net_layer_times")
+        return list(arr)
+
+    def layer_variants(self):
+        """Kernel per layer: 0 fp32 first layer, VARIANT_POPC or VARIANT_TC."""
+        n = self.launches
+        arr = (ctypes.c_int32 * n)()
+        _check(lib().minw_net_layer_variants(self._h, arr), "minw_net_layer_variants")
         return list(arr)
 
     @property
