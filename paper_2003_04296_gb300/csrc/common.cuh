@@ -132,6 +132,41 @@ __device__ __forceinline__ void channel_thresholds(float s, float t, const QPara
     out[n - 1] = sigma;
 }
 
+// The same breakpoints for an fp32 accumulator (the first layer, whose input
+// is not quantized): T_j is the smallest fp32 v with level index >= j when
+// evaluated at acc = sigma * v, found by binary search over the ordered fp32
+// bit patterns (finite values only).
+__device__ __forceinline__ int f32_order(float v) {
+    const int i = __float_as_int(v);
+    return i >= 0 ? i : (int)(0x80000000u - (uint32_t)i);   // monotone in v; -0 -> 0
+}
+__device__ __forceinline__ float f32_from_order(int k) {
+    return k >= 0 ? __int_as_float(k) : __int_as_float((int)(0x80000000u - (uint32_t)k));
+}
+__device__ __forceinline__ void channel_thresholds_f32(float s, float t, const QParams &q, float *out) {
+    const float sigma = (s < 0.0f) ? -1.0f : 1.0f;
+    const int n = num_levels(q.bits);
+    const int V = 0x7F7FFFFF;                          // order of FLT_MAX
+    for (int j = 1; j < n; ++j) {
+        auto idx = [&](int k) { return level_index_of_y(fmaf(f32_from_order(k) * sigma, s, t), q); };
+        float T;
+        if (idx(-V) >= j) {
+            T = -INFINITY;
+        } else if (idx(V) < j) {
+            T = INFINITY;
+        } else {
+            int lo = -V, hi = V;
+            while ((long long)hi - lo > 1) {                  // 2V overflows int
+                const int mid = (int)(((long long)lo + hi) >> 1);
+                if (idx(mid) >= j) hi = mid; else lo = mid;
+            }
+            T = f32_from_order(hi);
+        }
+        out[j - 1] = T;
+    }
+    out[n - 1] = sigma;
+}
+
 // Level index of an accumulator (exact integer held in fp32) from the
 // breakpoints of its channel (n - 1 thresholds then sigma).
 __device__ __forceinline__ int level_index_of_acc(float acc, const float *thr, int n) {

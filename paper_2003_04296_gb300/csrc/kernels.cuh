@@ -43,10 +43,13 @@ struct FirstArgs {
     uint32_t *planes_out;      // [B][Ho][Wo][qo.bits][ceil(O/32)] (nullable)
     uint8_t *codes_out;        // [B][Ho][Wo][O] E4M3 level codes (nullable)
     float *y_out;              // [B][O][Ho][Wo] (nullable)
+    const float *thr;          // fp32 breakpoints [O][8] (nullable: computed in-kernel)
 };
 
 // Launchers (host).  Return MINW_OK or an error status.
 minw_status launch_conv_first(const FirstArgs &a, cudaStream_t s);
+minw_status launch_thresholds_f32(const float *scale, const float *shift, int O, const QParams &q, float *out,
+                                  cudaStream_t s);
 minw_status launch_conv_popc(const ConvArgs &a, cudaStream_t s);
 minw_status make_conv_args(ConvArgs &a, const uint32_t *act, int B, int C, int H, int W,
                            int bits_a, const uint32_t *wgt, int O, int kh, int kw, int bits_w,

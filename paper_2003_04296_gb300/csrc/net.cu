@@ -25,7 +25,8 @@ struct LayerPlan {
     int Ho, Wo, Hp, Wp;
     uint32_t *wplanes = nullptr;   // packed weights (popcount layers)
     uint8_t *wcodes = nullptr;     // weight codes (tensor-core layers)
-    float *thr = nullptr;          // output-quantizer breakpoints (tensor-core layers)
+    float *thr = nullptr;          // output-quantizer breakpoints (first layer: fp32 [O][8];
+                                   // tensor-core layers: integer-valued [O][levels])
     int in_codes = 0;              // input arrives in the codes layout
     float *wlatent = nullptr;      // fp32 weights (first layer)
     float *wscale = nullptr;       // per-channel weight prescale (first layer)
@@ -125,6 +126,13 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
         cudaMemcpyAsync(P.shift, d.shift, sizeof(float) * P.O, cudaMemcpyDeviceToDevice, s);
         const size_t K = (size_t)P.C * P.kh * P.kw;
         if (first) {
+            if (!last) {
+                if ((st = net_alloc(n, &P.thr, (size_t)P.O * 8)) != MINW_OK) { net_free(n); return st; }
+                if ((st = launch_thresholds_f32(P.scale, P.shift, P.O, to_qparams(&P.qo), P.thr, s)) != MINW_OK) {
+                    net_free(n);
+                    return st;
+                }
+            }
             if ((st = net_alloc(n, &P.wlatent, (size_t)P.O * K)) != MINW_OK) { net_free(n); return st; }
             cudaMemcpyAsync(P.wlatent, d.w, sizeof(float) * P.O * K, cudaMemcpyDeviceToDevice, s);
             if (d.w_scale) {
@@ -222,6 +230,7 @@ minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits
             a.planes_out = out_codes ? nullptr : (uint32_t *)dst;
             a.codes_out = out_codes ? (uint8_t *)dst : nullptr;
             a.y_out = last ? logits : nullptr;
+            a.thr = P.thr;
             st = launch_conv_first(a, cs);
         } else {
             const void *src = net->buf[cur ^ 1];

@@ -195,6 +195,34 @@ def test_conv_first(dev, M, bits_w, bits_out):
     assert np.array_equal(planes_view(planes, B, H, W, bits_out, O_), O.pack(lv, bits_out))
 
 
+@pytest.mark.parametrize("quant_w", [True, False])
+def test_conv_first_strided_stem(dev, M, quant_w):
+    """A 7x7 / stride 2 / pad 3 first layer (ResNet stem shape) on a ragged
+    23x23 image, with quantized or fp32 weights."""
+    B, C, H, W, O_, k = 2, 3, 23, 23, 64, 7
+    r = np.random.default_rng(17)
+    x = r.standard_normal((B, C, H, W)).astype(np.float32)
+    w = r.normal(0, 0.05, (O_, C, k, k)).astype(np.float32)
+    scale = (r.normal(1, 0.1, O_) / np.sqrt(147.0)).astype(np.float32)
+    shift = r.normal(0, 0.1, O_).astype(np.float32)
+    if quant_w:
+        cs = (1.0 / np.abs(w.reshape(O_, -1)).max(1)).astype(np.float32)
+        wl = O.quantize(w, 3, DEFAULT_THR[3], cs).astype(np.float32)
+        kw_ = dict(q_w=M.quant(3, DEFAULT_THR[3]), channel_scale=dev_tensor(cs, dev))
+    else:
+        wl = w
+        kw_ = {}
+    Ho = (H + 6 - k) // 2 + 1
+    planes = torch.empty(M.packed_words(B, O_, Ho, Ho, 2), dtype=torch.int32, device=dev)
+    y = torch.empty((B, O_, Ho, Ho), dtype=torch.float32, device=dev)
+    M.minw_conv_first(dev_tensor(x, dev), dev_tensor(w, dev), 2, 3, dev_tensor(scale, dev), dev_tensor(shift, dev),
+                      q_out=M.quant(2, DEFAULT_THR[2]), planes_out=planes, y_out=y, **kw_)
+    yr = O.hardtanh(O.affine(O.conv2d_f32_seq(x, wl, 2, 3), scale, shift))
+    assert np.array_equal(y.cpu().numpy(), yr)
+    lv = O.quantize(yr, 2, DEFAULT_THR[2])
+    assert np.array_equal(planes_view(planes, B, Ho, Ho, 2, O_), O.pack(lv, 2))
+
+
 def test_conv2d_adversarial_magnitudes(dev, M):
     """Largest accumulators of the bench shapes: every 3-bit level at +-1 on a
     512-channel 3x3 kernel (|acc| = 16 * 4608) next to small products."""
