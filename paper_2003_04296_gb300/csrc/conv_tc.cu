@@ -17,9 +17,10 @@
 // both with 128-byte swizzle, i.e. the canonical K-major layout the MMA reads.
 // Persistent CTAs (one per SM) walk the tiles; the stage ring runs across tile
 // boundaries, and two TMEM accumulators let the epilogue of one tile overlap
-// the MMAs of the next.  Warp roles (192 threads): warp 0 issues TMA, warp 1
-// owns TMEM and issues MMAs (4 x K=32 per stage), warps 2-5 drain TMEM (one
-// lane quarter each) and run the fused epilogue: 2x2 max pool via warp
+// the MMAs of the next.  Warp roles (352 threads): warp 0 issues the
+// activation TMA boxes and warp 10 the weight boxes, warp 1 owns TMEM and
+// issues MMAs (4 x K=32 per stage), warps 2-9 drain TMEM (two per lane
+// quarter, each half of the accumulator columns) and run the fused epilogue: 2x2 max pool via warp
 // shuffles on the exact accumulators, then BN + HardTanh + quantize as
 // per-channel integer thresholds (bit-identical to the fp32 chain, see
 // common.cuh), and stores of the next layer's codes or bit-planes; raw int32
@@ -40,7 +41,9 @@ __device__ int g_device_error = 0;
 
 namespace tc {
 
-constexpr int NT = 192;
+constexpr int NT = 352;                 // 11 warps: TMA (A), MMA, 8 epilogue, TMA (B)
+constexpr int EPI_WARPS = 8;            // two per TMEM lane quarter, each half of the columns
+constexpr int B_WARP = 2 + EPI_WARPS;   // the weight-box TMA warp
 constexpr int A_BYTES = 128 * 128;
 constexpr long long WAIT_CYCLES = 1ll << 31;
 
@@ -149,6 +152,18 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
 }
 
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
+        "%14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];\n"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
+          "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
+          "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
+}
+
 __device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
 __device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
 
@@ -194,12 +209,12 @@ __global__ void __launch_bounds__(NT, 1)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < p.S; ++s) {
-            mbar_init(&full[s], 1);
+            mbar_init(&full[s], 2);               // one arrival per TMA issuing warp
             mbar_init(&empty[s], 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
-            mbar_init(&tempty[i], 4);
+            mbar_init(&tempty[i], EPI_WARPS);
         }
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
@@ -222,11 +237,13 @@ __global__ void __launch_bounds__(NT, 1)
     fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
-    if (warp == 0) {
+    if (warp == 0 || warp == B_WARP) {
         if (lane == 0) {
-            // ---------------- TMA producer ----------------
-            asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
-            asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+            // ---------------- TMA producers: warp 0 activations, warp 6 weights ----------------
+            const bool act = warp == 0;
+            const CUtensorMap *map = act ? &tmA : &tmB;
+            asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+            const uint32_t bytes = act ? (uint32_t)A_BYTES : p.stage_bytes - (uint32_t)A_BYTES;
             int g = 0, s = 0, lap = 0;             // stages issued, ring slot, ring lap
             bool alive = true;
             for (int t = blockIdx.x; t < tiles && alive; t += gridDim.x) {
@@ -239,9 +256,11 @@ __global__ void __launch_bounds__(NT, 1)
                     // slot reuse: wait until the MMAs of the previous lap released it
                     if (lap > 0 && !mbar_wait(&empty[s], (lap - 1) & 1)) { alive = false; break; }
                     uint8_t *sa = smem + (size_t)s * p.stage_bytes;
-                    mbar_expect_tx(&full[s], p.stage_bytes);
-                    tma_load_4d(sa, &tmA, &full[s], c0, x0 + kx, y0 + ky, b0);
-                    tma_load_2d(sa + A_BYTES, &tmB, &full[s], kcol, o0);
+                    mbar_expect_tx(&full[s], bytes);
+                    if (act)
+                        tma_load_4d(sa, &tmA, &full[s], c0, x0 + kx, y0 + ky, b0);
+                    else
+                        tma_load_2d(sa + A_BYTES, &tmB, &full[s], kcol, o0);
                     kcol += 128;
                     c0 += 128;
                     if (c0 == p.C) {
@@ -282,9 +301,10 @@ __global__ void __launch_bounds__(NT, 1)
                 mma_commit(&tfull[ab]);
             }
         }
-    } else {
-        // ---------------- epilogue: warps 2..5 ----------------
+    } else if (warp < B_WARP) {
+        // ---------------- epilogue: warps 2..9 ----------------
         const int q = warp & 3;                   // TMEM lane quarter of this warp
+        const int half_cols = (warp - 2) >> 2;    // which half of the accumulator columns
         const int r = q * 32 + lane;              // tile row = output pixel
         const int Hp = p.pool ? p.Ho / 2 : p.Ho, Wp = p.pool ? p.Wo / 2 : p.Wo;
         const int NWo = (p.O + 31) >> 5;
@@ -305,13 +325,29 @@ __global__ void __launch_bounds__(NT, 1)
             if (!mbar_wait(&tfull[ab], use & 1)) break;
             fence_after();
             uint32_t pw[3] = {0u, 0u, 0u};
-            for (int ch = 0; ch < p.BN / 16; ++ch) {
+            // this warp's 16-column groups: the first or second half of BN/16
+            // (split at an even group so that no 32-channel plane word straddles the halves)
+            const int ngrp = p.BN / 16;
+            const int gmid = min(ngrp, (((ngrp + 1) / 2) + 1) & ~1);
+            const int gbeg = half_cols ? gmid : 0, gend = half_cols ? ngrp : gmid;
+            uint32_t v32[32];
+            for (int ch = gbeg; ch < gend; ++ch) {
                 __syncwarp();
-                uint32_t v[16];
-                tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * p.BN + ch * 16), v);
+                // two groups per TMEM load where possible (one wait for 32 columns)
+                const int sub = (ch - gbeg) & 1;
+                if (sub == 0) {
+                    if (ch + 1 < gend)
+                        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * p.BN + ch * 16), v32);
+                    else {
+                        uint32_t v16[16];
+                        tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * p.BN + ch * 16), v16);
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) v32[j] = v16[j];
+                    }
+                }
                 float a[16];
 #pragma unroll
-                for (int j = 0; j < 16; ++j) a[j] = __uint_as_float(v[j]);
+                for (int j = 0; j < 16; ++j) a[j] = __uint_as_float(sub ? v32[16 + j] : v32[j]);
                 if (p.pool) {
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
