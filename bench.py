@@ -303,7 +303,7 @@ def run_gpu(args, rank, world, local_rank):
             "e2e": {"value": BATCH * world / e2e_sec, "unit": "images/s",
                     "h2d_bytes_per_step": int(x_host.numel() * 4),
                     "d2h_bytes_per_step": int(out_host.numel() * 4)},
-            "gpu_launches": nl * args.steps, "clocks": clocks}
+            "gpu_launches": net.kernels * args.steps, "clocks": clocks}
     print(json.dumps(line), flush=True)
     return 0
 

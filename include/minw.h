@@ -216,6 +216,26 @@ MINW_API minw_status minw_conv_block_codes(const uint8_t *act, int32_t B, int32_
                                            uint8_t *codes_out, uint32_t *planes_out,
                                            float *y_out, void *stream);
 
+/* Fully connected layer a~ = a^q W^q (Algorithm 1, inference) on the tensor
+ * cores, with the reduction over K split across CTAs when the output alone
+ * would leave most SMs idle (split-K).  act: codes [B][K]; wgt: codes [O][K];
+ * K % 128 == 0.  Outputs as minw_conv_block_codes with H = W = 1: codes_out
+ * [B][O] (O % 16 == 0), planes_out [B][bits][ceil(O/32)], y_out fp32 [B][O];
+ * acc_out (nullable) int32 [B][O] exact accumulators.  q_out NULL = last layer.
+ * workspace: device scratch of minw_fc_workspace_bytes(B, K, O) bytes for
+ * the full split (a smaller one splits K into fewer slices; 0 bytes or NULL
+ * runs without the split).  Its contents need no initialisation and are
+ * meaningless after the call.  Calls that share a workspace must not run
+ * concurrently.  With a split the call launches a second kernel that sums
+ * the K slices and runs the epilogue. */
+MINW_API size_t minw_fc_workspace_bytes(int32_t B, int32_t K, int32_t O);
+MINW_API minw_status minw_fc_codes(const uint8_t *act, int32_t B, int32_t K, int32_t bits_a,
+                                   const uint8_t *wgt, int32_t O, int32_t bits_w,
+                                   const float *scale, const float *shift,
+                                   const minw_quant *q_out, uint8_t *codes_out,
+                                   uint32_t *planes_out, float *y_out, int32_t *acc_out,
+                                   void *workspace, size_t workspace_bytes, void *stream);
+
 /* First layer (Sec. III-E): the fp32 image x [B][C][H][W] is NOT quantized;
  * the weights are.  w: latent fp32 weights [O][C][kh][kw]; q_w (host) and
  * channel_scale (nullable) quantize them as minw_pack_weights does; q_w NULL
@@ -288,8 +308,12 @@ MINW_API minw_status minw_net_layer_times(minw_net *net, float *ms);
  * 0 for the fp32 first layer, else MINW_VARIANT_POPC or MINW_VARIANT_TC. */
 MINW_API minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants);
 
-/* Number of kernels one minw_forward launches. */
+/* Number of layers (and of entries minw_net_layer_times fills). */
 MINW_API int32_t minw_net_launches(const minw_net *net);
+
+/* Number of kernels one minw_forward launches (a layer whose K reduction is
+ * split across CTAs launches two). */
+MINW_API int32_t minw_net_kernels(const minw_net *net);
 
 /* Release a network (synchronises its device memory frees). */
 MINW_API void minw_net_destroy(minw_net *net);

@@ -158,4 +158,37 @@ minw_status minw_conv_block_codes(const uint8_t *act, int32_t B, int32_t C, int3
     return launch_conv_tc(a, (cudaStream_t)stream);
 }
 
+size_t minw_fc_workspace_bytes(int32_t B, int32_t K, int32_t O) {
+    if (B <= 0 || K <= 0 || O <= 0 || K % 128 != 0) return 0;
+    ConvArgs a{};
+    a.B = B; a.C = K; a.H = 1; a.W = 1; a.O = O; a.kh = 1; a.kw = 1; a.stride = 1; a.pad = 0;
+    a.Ho = 1; a.Wo = 1; a.NW = K / 32; a.M = B;
+    return conv_tc_workspace_bytes(a);
+}
+
+minw_status minw_fc_codes(const uint8_t *act, int32_t B, int32_t K, int32_t bits_a, const uint8_t *wgt, int32_t O,
+                          int32_t bits_w, const float *scale, const float *shift, const minw_quant *q_out,
+                          uint8_t *codes_out, uint32_t *planes_out, float *y_out, int32_t *acc_out,
+                          void *workspace, size_t workspace_bytes, void *stream) {
+    ConvArgs a;
+    minw_status st = make_codes_args(a, act, B, K, 1, 1, bits_a, wgt, O, 1, 1, bits_w, 1, 0);
+    if (st != MINW_OK) return st;
+    if (q_out && (!valid_quant(q_out) || (!planes_out && !codes_out))) return MINW_EINVAL;
+    if ((q_out || y_out) && (!scale || !shift)) return MINW_EINVAL;
+    if (codes_out && (O % 16 != 0 || !aligned16(codes_out))) return MINW_EUNSUPPORTED;
+    if (!q_out && !y_out && !acc_out) return MINW_EINVAL;
+    if (workspace && !aligned16(workspace)) return MINW_EINVAL;
+    a.scale = scale;
+    a.shift = shift;
+    a.quant_out = q_out != nullptr;
+    if (q_out) a.qo = to_qparams(q_out);
+    a.planes_out = planes_out;
+    a.codes_out = q_out ? codes_out : nullptr;
+    a.y_out = y_out;
+    a.acc_out = acc_out;
+    a.workspace = workspace_bytes ? workspace : nullptr;
+    a.workspace_bytes = workspace_bytes;
+    return launch_conv_tc(a, (cudaStream_t)stream);
+}
+
 }  // extern "C"

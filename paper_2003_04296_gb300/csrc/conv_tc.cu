@@ -54,6 +54,8 @@ struct Params {
     uint32_t stage_bytes, idesc, tmem_cols;
     const float *thr;          // precomputed breakpoints [O][nlev] (nullable)
     int nlev;                  // levels of the output quantizer
+    int ksplit;                // K slices per output tile (1: no split)
+    int32_t *part;             // split-K: int32 partial sums [ksplit][tiles][128][BN]
     int32_t *acc_out;
     float *y_out;
     const float *scale, *shift;
@@ -206,6 +208,7 @@ __global__ void __launch_bounds__(NT, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int tiles_m = p.nbx * p.nby * p.nbb;
     const int tiles = tiles_m * p.ntn;
+    const int items = tiles * p.ksplit;       // (output tile, K slice) work items
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < p.S; ++s) {
@@ -246,13 +249,18 @@ __global__ void __launch_bounds__(NT, 1)
             const uint32_t bytes = act ? (uint32_t)A_BYTES : p.stage_bytes - (uint32_t)A_BYTES;
             int g = 0, s = 0, lap = 0;             // stages issued, ring slot, ring lap
             bool alive = true;
-            for (int t = blockIdx.x; t < tiles && alive; t += gridDim.x) {
+            for (int w = blockIdx.x; w < items && alive; w += gridDim.x) {
+                const int t = w / p.ksplit, kp = w - t * p.ksplit;
+                const int kb = (int)((long long)kp * p.nk / p.ksplit), ke = (int)((long long)(kp + 1) * p.nk / p.ksplit);
                 const int tn = t / tiles_m, tm = t - tn * tiles_m;
                 const int xb = tm % p.nbx, yb = (tm / p.nbx) % p.nby, bbk = tm / (p.nbx * p.nby);
                 const int x0 = xb * p.bw - p.pad, y0 = yb * p.bh - p.pad, b0 = bbk * p.bb;
                 const int o0 = tn * p.BN;
-                int c0 = 0, kx = 0, ky = 0, kcol = 0;  // channel chunk, tap, weight column
-                for (int ks = 0; ks < p.nk; ++ks, ++g) {
+                // channel chunk, tap and weight column of stage kb
+                const int tap0 = kb / p.nck;
+                int c0 = (kb - tap0 * p.nck) * 128, ky = tap0 / p.kw, kx = tap0 - (tap0 / p.kw) * p.kw;
+                int kcol = kb * 128;
+                for (int ks = kb; ks < ke; ++ks, ++g) {
                     // slot reuse: wait until the MMAs of the previous lap released it
                     if (lap > 0 && !mbar_wait(&empty[s], (lap - 1) & 1)) { alive = false; break; }
                     uint8_t *sa = smem + (size_t)s * p.stage_bytes;
@@ -281,12 +289,14 @@ __global__ void __launch_bounds__(NT, 1)
             uint32_t fphase = 0;
             bool alive = true;
             const uint32_t sbase = smem_u32(smem);
-            for (int t = blockIdx.x; t < tiles && alive; t += gridDim.x, ++i) {
+            for (int w = blockIdx.x; w < items && alive; w += gridDim.x, ++i) {
                 const int ab = i & 1, use = i >> 1;
+                const int t = w / p.ksplit, kp = w - t * p.ksplit;
+                const int kb = (int)((long long)kp * p.nk / p.ksplit), ke = (int)((long long)(kp + 1) * p.nk / p.ksplit);
                 if (use > 0 && !mbar_wait(&tempty[ab], (use - 1) & 1)) break;
                 fence_after();
                 const uint32_t tmem_d = tmem_base + (uint32_t)(ab * p.BN);
-                for (int ks = 0; ks < p.nk; ++ks) {
+                for (int ks = kb; ks < ke; ++ks) {
                     if (!mbar_wait(&full[s], fphase)) { alive = false; break; }
                     fence_after();
                     const uint32_t sa = sbase + (uint32_t)s * p.stage_bytes;
@@ -294,7 +304,7 @@ __global__ void __launch_bounds__(NT, 1)
                     const uint64_t bdesc = sw128_desc(sa + A_BYTES);
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
-                        mma_f8(tmem_d, adesc + 2 * kk, bdesc + 2 * kk, p.idesc, (ks | kk) != 0);
+                        mma_f8(tmem_d, adesc + 2 * kk, bdesc + 2 * kk, p.idesc, (ks != kb) || (kk != 0));
                     mma_commit(&empty[s]);
                     if (++s == p.S) { s = 0; fphase ^= 1; }
                 }
@@ -309,9 +319,16 @@ __global__ void __launch_bounds__(NT, 1)
         const int Hp = p.pool ? p.Ho / 2 : p.Ho, Wp = p.pool ? p.Wo / 2 : p.Wo;
         const int NWo = (p.O + 31) >> 5;
         const int rb = r / (p.bh * p.bw), ry = (r / p.bw) % p.bh, rx = r % p.bw;
+        // this warp's 16-column groups: the first or second half of BN/16
+        // (split at an even group so that no 32-channel plane word straddles the halves)
+        const int ngrp = p.BN / 16;
+        const int gmid = min(ngrp, (((ngrp + 1) / 2) + 1) & ~1);
+        const int gbeg = half_cols ? gmid : 0, gend = half_cols ? ngrp : gmid;
         int i = 0;
-        for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++i) {
+        bool dead = false;           // a bounded wait ran out: skip work, keep the barrier sequence
+        for (int w = blockIdx.x; w < items; w += gridDim.x, ++i) {
             const int ab = i & 1, use = i >> 1;
+            const int t = w / p.ksplit, kp = w - t * p.ksplit;
             const int tn = t / tiles_m, tm = t - tn * tiles_m;
             const int xb = tm % p.nbx, yb = (tm / p.nbx) % p.nby, bbk = tm / (p.nbx * p.nby);
             const int b = bbk * p.bb + rb;
@@ -322,32 +339,10 @@ __global__ void __launch_bounds__(NT, 1)
             const bool writer = valid && (!p.pool || ((x & 1) == 0 && (y & 1) == 0));
             const int yp = p.pool ? y / 2 : y, xp = p.pool ? x / 2 : x;
             const long long opix = ((long long)b * Hp + yp) * Wp + xp;
-            if (!mbar_wait(&tfull[ab], use & 1)) break;
-            fence_after();
             uint32_t pw[3] = {0u, 0u, 0u};
-            // this warp's 16-column groups: the first or second half of BN/16
-            // (split at an even group so that no 32-channel plane word straddles the halves)
-            const int ngrp = p.BN / 16;
-            const int gmid = min(ngrp, (((ngrp + 1) / 2) + 1) & ~1);
-            const int gbeg = half_cols ? gmid : 0, gend = half_cols ? ngrp : gmid;
-            uint32_t v32[32];
-            for (int ch = gbeg; ch < gend; ++ch) {
-                __syncwarp();
-                // two groups per TMEM load where possible (one wait for 32 columns)
-                const int sub = (ch - gbeg) & 1;
-                if (sub == 0) {
-                    if (ch + 1 < gend)
-                        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * p.BN + ch * 16), v32);
-                    else {
-                        uint32_t v16[16];
-                        tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * p.BN + ch * 16), v16);
-#pragma unroll
-                        for (int j = 0; j < 16; ++j) v32[j] = v16[j];
-                    }
-                }
-                float a[16];
-#pragma unroll
-                for (int j = 0; j < 16; ++j) a[j] = __uint_as_float(sub ? v32[16 + j] : v32[j]);
+
+            // the fused block epilogue of one 16-column group of exact accumulators
+            auto finish = [&](float (&a)[16], int ch) {
                 if (p.pool) {
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
@@ -415,16 +410,132 @@ __global__ void __launch_bounds__(NT, 1)
                         }
                     }
                 }
+            };
+
+            if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
+            fence_after();
+            int32_t *prow = p.part + (((size_t)kp * tiles + t) * 128 + r) * p.BN;
+            uint32_t v32[32];
+            for (int ch = gbeg; ch < gend && !dead; ++ch) {
+                __syncwarp();
+                // two groups per TMEM load where possible (one wait for 32 columns)
+                const int sub = (ch - gbeg) & 1;
+                if (sub == 0) {
+                    if (ch + 1 < gend)
+                        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * p.BN + ch * 16), v32);
+                    else {
+                        uint32_t v16[16];
+                        tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * p.BN + ch * 16), v16);
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) v32[j] = v16[j];
+                    }
+                }
+                float a[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) a[j] = __uint_as_float(sub ? v32[16 + j] : v32[j]);
+                if (p.ksplit == 1) {
+                    finish(a, ch);
+                } else {
+                    // exact integer partial sums of this K slice (summed by splitk_reduce_kernel)
+                    int4 *dst = reinterpret_cast<int4 *>(prow + ch * 16);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        dst[j] = make_int4(__float2int_rn(a[4 * j]), __float2int_rn(a[4 * j + 1]),
+                                           __float2int_rn(a[4 * j + 2]), __float2int_rn(a[4 * j + 3]));
+                }
             }
             fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&tempty[ab]);
+            if (lane == 0 && !dead) mbar_arrive(&tempty[ab]);      // the accumulator can be reused
         }
     }
     __syncthreads();
     if (warp == 1) {
         fence_after();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(p.tmem_cols));
+    }
+}
+
+// Split-K second pass: sums the K slices of every accumulator and runs the
+// block epilogue (no pooling).  Thread = one tile row (output pixel) x four
+// channels; eight consecutive lanes cover 32 channels of one row, so the
+// partial-sum loads coalesce and plane words assemble with shuffles.
+template <int OUTB>
+__global__ void __launch_bounds__(256) splitk_reduce_kernel(const Params p, const float *__restrict__ thr) {
+    constexpr int NL = OUTB == 0 ? 1 : (OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7));
+    const int tiles_m = p.nbx * p.nby * p.nbb;
+    const int tiles = tiles_m * p.ntn;
+    const int g32 = (p.O + 31) >> 5;                 // 32-channel groups
+    const long long total = (long long)tiles_m * 128 * g32 * 8;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    const int lane8 = threadIdx.x & 7;
+    if (idx - lane8 >= total) return;               // whole 8-lane groups leave together
+    const long long rowgrp = idx >> 3;
+    const int g = (int)(rowgrp % g32);
+    const long long rr = rowgrp / g32;
+    const int tm = (int)(rr >> 7), r = (int)(rr & 127);
+    const int o = g * 32 + lane8 * 4;                // first of this thread's four channels
+    const bool live = o < p.O;
+    const int tn = live ? o / p.BN : 0, col = live ? o - tn * p.BN : 0;
+    const int t = tn * tiles_m + tm;
+    const int xb = tm % p.nbx, yb = (tm / p.nbx) % p.nby, bbk = tm / (p.nbx * p.nby);
+    const int b = bbk * p.bb + r / (p.bh * p.bw);
+    const int y = yb * p.bh + (r / p.bw) % p.bh;
+    const int x = xb * p.bw + r % p.bw;
+    const bool inside = b < p.B && y < p.Ho && x < p.Wo;
+    const bool valid = live && inside;
+    int acc[4] = {0, 0, 0, 0};
+    if (valid) {
+        const size_t slice4 = (size_t)tiles * 128 * p.BN / 4;
+        const int4 *src = reinterpret_cast<const int4 *>(p.part + ((size_t)t * 128 + r) * p.BN + col);
+        for (int kp = 0; kp < p.ksplit; ++kp) {
+            const int4 v = __ldcs(src + kp * slice4);
+            acc[0] += v.x; acc[1] += v.y; acc[2] += v.z; acc[3] += v.w;
+        }
+    }
+    const long long HoWo = (long long)p.Ho * p.Wo;
+    const long long pix = ((long long)b * p.Ho + y) * p.Wo + x;
+    if (valid && p.acc_out != nullptr)
+        for (int j = 0; j < 4; ++j)
+            if (o + j < p.O) p.acc_out[((long long)b * p.O + o + j) * HoWo + (long long)y * p.Wo + x] = acc[j];
+    if (valid && p.y_out != nullptr)
+        for (int j = 0; j < 4; ++j)
+            if (o + j < p.O) {
+                float yv = fmaf((float)acc[j], __ldg(p.scale + o + j), __ldg(p.shift + o + j));
+                if (OUTB > 0) yv = fminf(fmaxf(yv, -1.0f), 1.0f);
+                p.y_out[((long long)b * p.O + o + j) * HoWo + (long long)y * p.Wo + x] = yv;
+            }
+    if constexpr (OUTB > 0) {
+        uint32_t code = 0u, bits[3] = {0u, 0u, 0u};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (valid && o + j < p.O) {
+                const float *th = thr + (o + j) * NL;
+                const float v = (float)acc[j] * __ldg(th + NL - 1);
+                int k = 0;
+#pragma unroll
+                for (int u = 0; u < NL - 1; ++u) k += (v >= __ldg(th + u)) ? 1 : 0;
+                code |= code_k<OUTB>(k) << (8 * j);
+                const uint32_t pb = planes_k<OUTB>(k);
+#pragma unroll
+                for (int u = 0; u < OUTB; ++u) bits[u] |= ((pb >> u) & 1u) << (lane8 * 4 + j);
+            }
+        }
+        if (p.codes_out != nullptr && valid) *reinterpret_cast<uint32_t *>(p.codes_out + pix * p.O + o) = code;
+        if (p.planes_out != nullptr) {
+#pragma unroll
+            for (int u = 0; u < OUTB; ++u) {
+                bits[u] |= __shfl_xor_sync(__activemask(), bits[u], 1);
+                bits[u] |= __shfl_xor_sync(__activemask(), bits[u], 2);
+                bits[u] |= __shfl_xor_sync(__activemask(), bits[u], 4);
+            }
+            if (lane8 == 0 && inside) {
+                const int NWo = (p.O + 31) >> 5;
+                uint32_t *dst = p.planes_out + (pix * OUTB) * NWo + g;
+#pragma unroll
+                for (int u = 0; u < OUTB; ++u) dst[u * NWo] = bits[u];
+            }
+        }
     }
 }
 
@@ -467,6 +578,7 @@ struct Plan {
     CUtensorMap tmA, tmB;
     dim3 grid;
     size_t smem;
+    float *thr_ws;      // split-K: breakpoints computed into the workspace (nullable)
 };
 
 static bool plan_shape(const ConvArgs &a, Params &p) {
@@ -486,6 +598,18 @@ static bool plan_shape(const ConvArgs &a, Params &p) {
     p.BN = BN;
     return true;
 }
+
+// Split-K: a shape with fewer output tiles than half the SMs and a long K
+// loop (>= 16 stages) splits it into slices of at least four stages, up to
+// one work item per SM.  Short K loops gain less than the second launch costs.
+static int auto_ksplit(int tiles, int nk, int sms) {
+    if (tiles * 2 > sms || nk < 16) return 1;
+    int ks = sms / tiles;
+    if (ks > nk / 4) ks = nk / 4;
+    return ks < 2 ? 1 : ks;
+}
+static size_t slice_bytes(int tiles, int BN) { return (size_t)tiles * 128 * BN * sizeof(int32_t); }
+static size_t thr_ws_bytes(int O, int nlev) { return (((size_t)O * nlev * sizeof(float)) + 255) & ~(size_t)255; }
 
 static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     Params &p = pl.p;
@@ -539,7 +663,29 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     }
     const int tiles = p.nbx * p.nby * p.nbb * p.ntn;
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
-    pl.grid = dim3((unsigned)(tiles < sms ? tiles : sms));
+    p.ksplit = 1;
+    pl.thr_ws = nullptr;
+    if (a.workspace != nullptr && !a.pool) {
+        // workspace: [breakpoints, when not given][ksplit partial-sum slices]
+        const size_t tb = (a.quant_out && a.thr == nullptr) ? thr_ws_bytes(a.O, p.nlev) : 0;
+        const size_t sb = slice_bytes(tiles, p.BN);
+        int ks = a.ksplit > 0 ? a.ksplit : auto_ksplit(tiles, p.nk, sms);
+        if (a.workspace_bytes > tb) {
+            const size_t cap = (a.workspace_bytes - tb) / sb;
+            if ((size_t)ks > cap) ks = (int)cap;
+        } else {
+            ks = 1;
+        }
+        if (ks > p.nk) ks = p.nk;
+        if (ks > 1) {
+            p.ksplit = ks;
+            uint8_t *w = reinterpret_cast<uint8_t *>(a.workspace);
+            if (tb) pl.thr_ws = reinterpret_cast<float *>(w);
+            p.part = reinterpret_cast<int32_t *>(w + tb);
+        }
+    }
+    const int items = tiles * p.ksplit;
+    pl.grid = dim3((unsigned)(items < sms ? items : sms));
     pl.smem = (size_t)p.S * p.stage_bytes + 1024 + 256 + thr_bytes;
     // more than half of an SM's shared memory: exactly one CTA (and one TMEM
     // allocation) per SM
@@ -549,6 +695,18 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
 
 }  // namespace tc
 
+size_t conv_tc_workspace_bytes(const ConvArgs &a) {
+    tc::Params p{};
+    if (a.pool || !tc::plan_shape(a, p)) return 0;
+    const int nbb = (a.B + p.bb - 1) / p.bb;
+    const int tiles = p.nbx * p.nby * nbb * ((a.O + p.BN - 1) / p.BN);
+    const int nk = a.kh * a.kw * (a.C / 128);
+    const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
+    const int ks = tc::auto_ksplit(tiles, nk, sms);
+    if (ks < 2) return 0;
+    return tc::thr_ws_bytes(a.O, 7) + (size_t)ks * tc::slice_bytes(tiles, p.BN);
+}
+
 bool conv_tc_supported(const ConvArgs &a) {
     tc::Params p{};
     if (!tc::plan_shape(a, p)) return false;
@@ -556,6 +714,12 @@ bool conv_tc_supported(const ConvArgs &a) {
     if (a.quant_out && a.codes_out != nullptr && a.O % 16 != 0) return false;
     if (a.acc_out != nullptr && a.pool) return false;
     return true;
+}
+
+int conv_tc_launches(const ConvArgs &a) {
+    if (a.workspace == nullptr || a.pool) return 1;
+    tc::Plan pl;
+    return (tc::make_plan(a, pl) == MINW_OK && pl.p.ksplit > 1) ? 2 : 1;
 }
 
 minw_status launch_thresholds(const float *scale, const float *shift, int O, const QParams &q, float *out,
@@ -571,16 +735,40 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
     minw_status st = tc::make_plan(a, pl);
     if (st != MINW_OK) return st;
     const int outb = a.quant_out ? a.qo.bits : 0;
+    const bool split = pl.p.ksplit > 1;
+    const int kout = split ? 0 : outb;            // the split main pass writes only partial sums
     static size_t configured[4] = {0, 0, 0, 0};
     void (*kern)(const CUtensorMap, const CUtensorMap, const tc::Params) =
-        outb == 1 ? tc::conv_tc_kernel<1> : outb == 2 ? tc::conv_tc_kernel<2> : outb == 3 ? tc::conv_tc_kernel<3>
+        kout == 1 ? tc::conv_tc_kernel<1> : kout == 2 ? tc::conv_tc_kernel<2> : kout == 3 ? tc::conv_tc_kernel<3>
                                                                                          : tc::conv_tc_kernel<0>;
-    if (pl.smem > configured[outb]) {
+    if (pl.smem > configured[kout]) {
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem) != cudaSuccess)
             return MINW_ECUDA;
-        configured[outb] = pl.smem;
+        configured[kout] = pl.smem;
     }
-    kern<<<pl.grid, tc::NT, pl.smem, s>>>(pl.tmA, pl.tmB, pl.p);
+    const float *thr = a.thr;
+    if (split && a.quant_out && thr == nullptr) {
+        tc::thresholds_kernel<<<(a.O + 127) / 128, 128, 0, s>>>(a.scale, a.shift, a.O, a.qo, pl.thr_ws);
+        thr = pl.thr_ws;
+    }
+    tc::Params pm = pl.p;
+    if (split) {
+        pm.quant_out = 0;
+        pm.acc_out = nullptr;
+        pm.y_out = nullptr;
+    }
+    kern<<<pl.grid, tc::NT, pl.smem, s>>>(pl.tmA, pl.tmB, pm);
+    if (split) {
+        const int tiles_m = pl.p.nbx * pl.p.nby * pl.p.nbb;
+        const long long threads = (long long)tiles_m * 128 * ((a.O + 31) / 32) * 8;
+        const unsigned blocks = (unsigned)((threads + 255) / 256);
+        switch (outb) {
+            case 1: tc::splitk_reduce_kernel<1><<<blocks, 256, 0, s>>>(pl.p, thr); break;
+            case 2: tc::splitk_reduce_kernel<2><<<blocks, 256, 0, s>>>(pl.p, thr); break;
+            case 3: tc::splitk_reduce_kernel<3><<<blocks, 256, 0, s>>>(pl.p, thr); break;
+            default: tc::splitk_reduce_kernel<0><<<blocks, 256, 0, s>>>(pl.p, thr); break;
+        }
+    }
     return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
 }
 

@@ -27,6 +27,10 @@ struct ConvArgs {
     const uint8_t *act8;   // [B][H][W][C]
     const uint8_t *wgt8;   // [O][kh][kw][C]
     const float *thr;      // output-quantizer breakpoints [O][levels] (nullable: computed in-kernel)
+    // split-K (tensor-core path): zero-initialised workspace, left zero by every call
+    void *workspace;       // nullable: no split
+    size_t workspace_bytes;
+    int ksplit;            // 0: chosen from the shape
 };
 
 // First-layer convolution on the fp32 image (see conv_first.cu).
@@ -58,6 +62,10 @@ int choose_variant(const ConvArgs &a, int requested);
 minw_status run_conv(const ConvArgs &a, int variant, cudaStream_t s);
 minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s);
 bool conv_tc_supported(const ConvArgs &a);
+// Workspace the tensor-core path needs to split K for this shape (0: it does not split).
+size_t conv_tc_workspace_bytes(const ConvArgs &a);
+// Kernels one tensor-core launch issues for this shape and workspace (2 with a split).
+int conv_tc_launches(const ConvArgs &a);
 minw_status launch_thresholds(const float *scale, const float *shift, int O, const QParams &q, float *out,
                               cudaStream_t s);
 

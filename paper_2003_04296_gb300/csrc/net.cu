@@ -45,6 +45,8 @@ struct minw_net {
     float *x_stage = nullptr;         // device staging of minw_forward_host
     float *logits_stage = nullptr;
     size_t x_elems = 0, logit_elems = 0;
+    void *ws = nullptr;               // split-K workspace shared by the layers (zero between layers)
+    size_t ws_bytes = 0;
     std::vector<cudaEvent_t> events;  // [0] before the first layer, [l+1] after layer l
     bool timing = false;
 };
@@ -152,6 +154,10 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
             if (!last) a.qo = to_qparams(&P.qo);
             P.variant = choose_variant(a, variant);
             if (P.variant == MINW_VARIANT_TC && !conv_tc_supported(a)) { net_free(n); return MINW_EUNSUPPORTED; }
+            if (P.variant == MINW_VARIANT_TC) {
+                const size_t wb = conv_tc_workspace_bytes(a);
+                if (wb > n->ws_bytes) n->ws_bytes = wb;
+            }
         }
         pc = P.O; ph = P.Hp; pw = P.Wp; pbits = d.bits_out;
         n->L.push_back(P);
@@ -192,6 +198,13 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
         if (st != MINW_OK) { net_free(n); return st; }
     }
     n->buf_words = max_words;
+    if (n->ws_bytes) {
+        uint8_t *w = nullptr;
+        minw_status st = net_alloc(n, &w, n->ws_bytes);
+        if (st != MINW_OK) { net_free(n); return st; }
+        if (cudaMemsetAsync(w, 0, n->ws_bytes, s) != cudaSuccess) { net_free(n); return MINW_ECUDA; }
+        n->ws = w;
+    }
     n->x_elems = (size_t)max_batch * layers[0].C * layers[0].H * layers[0].W;
     const LayerPlan &PL = n->L.back();
     n->logit_elems = (size_t)max_batch * PL.O * PL.Hp * PL.Wp;
@@ -249,6 +262,8 @@ minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits
                 a.act8 = (const uint8_t *)src;
                 a.wgt8 = P.wcodes;
                 a.thr = P.thr;
+                a.workspace = net->ws;
+                a.workspace_bytes = net->ws_bytes;
                 st = launch_conv_tc(a, cs);
             } else {
                 a.act = (const uint32_t *)src;
@@ -306,6 +321,26 @@ minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants) {
 }
 
 int32_t minw_net_launches(const minw_net *net) { return net ? (int32_t)net->L.size() : 0; }
+
+// Kernels one minw_forward issues (a split-K layer issues two).
+int32_t minw_net_kernels(const minw_net *net) {
+    if (!net) return 0;
+    int32_t k = 0;
+    for (size_t l = 0; l < net->L.size(); ++l) {
+        const LayerPlan &P = net->L[l];
+        if (l == 0 || !P.in_codes) { ++k; continue; }
+        ConvArgs a{};
+        a.B = net->max_batch; a.C = P.C; a.H = P.H; a.W = P.W; a.O = P.O; a.kh = P.kh; a.kw = P.kw;
+        a.stride = P.stride; a.pad = P.pad; a.Ho = P.Ho; a.Wo = P.Wo; a.NW = P.C / 32;
+        a.M = (long long)net->max_batch * P.Ho * P.Wo; a.pool = P.pool;
+        a.quant_out = l + 1 < net->L.size();
+        if (a.quant_out) a.qo = to_qparams(&P.qo);
+        a.act8 = P.wcodes; a.wgt8 = P.wcodes; a.thr = P.thr;
+        a.workspace = net->ws; a.workspace_bytes = net->ws_bytes;
+        k += conv_tc_launches(a);
+    }
+    return k;
+}
 
 void minw_net_destroy(minw_net *net) {
     if (!net) return;

@@ -63,6 +63,9 @@ SIGNATURES = {
                                          _I32, _I32, _P, _P, _P, _P, _P]),
     "minw_conv_block_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32,
                                              _I32, _I32, _I32, _P, _P, _QP, _P, _P, _P, _P]),
+    "minw_fc_workspace_bytes": (ctypes.c_size_t, [_I32, _I32, _I32]),
+    "minw_fc_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _P, _I32, _I32, _P, _P, _QP, _P, _P, _P, _P, _P,
+                                     ctypes.c_size_t, _P]),
     "minw_net_create": (ctypes.c_int, [ctypes.POINTER(LayerDesc), _I32, _I32, _I32, _P,
                                        ctypes.POINTER(ctypes.c_void_p)]),
     "minw_forward": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
@@ -71,6 +74,7 @@ SIGNATURES = {
     "minw_net_layer_times": (ctypes.c_int, [_P, _P]),
     "minw_net_layer_variants": (ctypes.c_int, [_P, _P]),
     "minw_net_launches": (_I32, [_P]),
+    "minw_net_kernels": (_I32, [_P]),
     "minw_net_destroy": (None, [_P]),
     "minw_get_last_device_error": (ctypes.c_int, [_P]),
 }
@@ -232,6 +236,19 @@ def minw_conv_block_codes(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, strid
            "minw_conv_block_codes")
 
 
+def minw_fc_workspace_bytes(B, K, O):
+    return int(lib().minw_fc_workspace_bytes(B, K, O))
+
+
+def minw_fc_codes(act, B, K, bits_a, wgt, O, bits_w, scale=None, shift=None, q_out=None, codes_out=None,
+                  planes_out=None, y_out=None, acc_out=None, workspace=None, stream=None):
+    nbytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    _check(lib().minw_fc_codes(_ptr(act), B, K, bits_a, _ptr(wgt), O, bits_w, _ptr(scale), _ptr(shift),
+                               ctypes.byref(q_out) if q_out is not None else None, _ptr(codes_out),
+                               _ptr(planes_out), _ptr(y_out), _ptr(acc_out), _ptr(workspace), nbytes,
+                               _stream(stream)), "minw_fc_codes")
+
+
 def minw_get_last_device_error(stream=None):
     return lib().minw_get_last_device_error(_stream(stream))
 
@@ -292,6 +309,11 @@ class Net:
         arr = (ctypes.c_int32 * n)()
         _check(lib().minw_net_layer_variants(self._h, arr), "minw_net_layer_variants")
         return list(arr)
+
+    @property
+    def kernels(self):
+        """Kernels one forward launches."""
+        return lib().minw_net_kernels(self._h)
 
     @property
     def launches(self):

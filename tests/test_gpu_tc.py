@@ -172,3 +172,49 @@ def test_codes_argument_errors(dev, M):
         M.minw_conv2d_codes(t, 1, 64, 4, 4, 1, t, 8, 3, 3, 1, 1, 1, acc_out=a)
     with pytest.raises(M.MinwError):   # stride 2 is outside the tensor-core path
         M.minw_conv2d_codes(t, 1, 128, 4, 4, 1, t, 8, 3, 3, 1, 2, 1, acc_out=a)
+
+
+def _fc_problem(seed, B, K, O, ba, bw):
+    p = conv_problem(seed, B, K, 1, 1, O, 1, 1, 1, 0, ba, bw, w_sigma=0.5)
+    return p
+
+
+@pytest.mark.parametrize("B,K,Oc,ba,bw", [(256, 8192, 1024, 1, 1), (130, 4096, 1024, 2, 2), (256, 2048, 10, 1, 1),
+                                         (64, 4096, 512, 3, 3)])
+def test_fc_split_k(dev, M, B, K, Oc, ba, bw):
+    """Fully connected layer with the K reduction split across CTAs: equal to
+    the unsplit kernel and to the oracle, two calls in a row on one workspace
+    (whose contents are garbage between calls)."""
+    p = _fc_problem(B + K + Oc, B, K, Oc, ba, bw)
+    act = torch.empty((B, 1, 1, K), dtype=torch.uint8, device=dev)
+    wgt = torch.empty((Oc, 1, 1, K), dtype=torch.uint8, device=dev)
+    M.aqe_quantize_codes(dev_tensor(p["x"], dev), M.quant(ba, p["thr_a"]), act)
+    M.minw_pack_weight_codes(dev_tensor(p["w"], dev), M.quant(bw, p["thr_w"]), wgt,
+                             channel_scale=dev_tensor(p["w_scale"], dev))
+    nbytes = M.minw_fc_workspace_bytes(B, K, Oc)
+    assert nbytes > 0
+    ws = torch.full((nbytes,), 0x5A, dtype=torch.uint8, device=dev)
+    sc, sh = dev_tensor(p["scale"], dev), dev_tensor(p["shift"], dev)
+    ref = _ref_acc(p).reshape(B, Oc)
+    last = Oc % 16 != 0
+    q = None if last else M.quant(ba, DEFAULT_THR[ba])
+    outs = []
+    half = ws[: nbytes // 2]
+    for use_ws in (ws, ws, half, None):
+        acc = torch.full((B, Oc), -7, dtype=torch.int32, device=dev)
+        y = torch.empty((B, Oc), dtype=torch.float32, device=dev)
+        codes = None if last else torch.empty((B, Oc), dtype=torch.uint8, device=dev)
+        M.minw_fc_codes(act, B, K, ba, wgt, Oc, bw, scale=sc, shift=sh, q_out=q, codes_out=codes, y_out=y,
+                        acc_out=acc, workspace=use_ws)
+        torch.cuda.synchronize()
+        assert np.array_equal(acc.cpu().numpy(), ref)
+        yr = O.affine(ref, p["scale"], p["shift"])
+        if not last:
+            yr = O.hardtanh(yr)
+        assert np.array_equal(y.cpu().numpy(), yr)
+        outs.append(codes.cpu().numpy() if codes is not None else None)
+    if not last:
+        lv = O.quantize(O.hardtanh(O.affine(ref, p["scale"], p["shift"])), ba, DEFAULT_THR[ba])
+        assert np.array_equal(decode_e4m3(outs[0]), lv * 2.0 ** O.units_shift(ba))
+        assert np.array_equal(outs[0], outs[2]) and np.array_equal(outs[0], outs[3])
+    assert M.minw_get_last_device_error() == M.MINW_OK
