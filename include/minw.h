@@ -236,6 +236,33 @@ MINW_API minw_status minw_fc_codes(const uint8_t *act, int32_t B, int32_t K, int
                                    uint32_t *planes_out, float *y_out, int32_t *acc_out,
                                    void *workspace, size_t workspace_bytes, void *stream);
 
+/* minw_fc_codes for callers that cannot allocate device memory (no
+ * counterpart in the paper; an interface addition).  Such callers include a
+ * plugin run by a host framework that owns all device memory and passes in
+ * only the tensors of the call, and a service that reserves its memory at
+ * start-up and forbids allocations afterwards.  The split-K scratch lives
+ * in a fixed array of MINW_FC_NOALLOC_SCRATCH_BYTES inside the library, held
+ * on every GPU that loads the library until the process exits.  The call
+ * allocates nothing (no cudaMalloc/cudaFree, no allocating library routine).
+ * - The first call on each device looks up the array's device address
+ *   (cudaGetSymbolAddress, with that device current); make that first call
+ *   before any stream capture.
+ * - Every call shares the one array.  Nothing in it needs to start at zero
+ *   (each call overwrites what it reads) and it keeps the last call's
+ *   contents; calls that overlap on the GPU (other streams, other threads)
+ *   race on it and must be serialised by the caller.
+ * - K is split into as many slices as the array holds; a shape whose
+ *   smallest split (two slices of int32 partial sums plus the breakpoints)
+ *   needs more than the array returns MINW_EUNSUPPORTED before any launch.
+ * Arguments and outputs as minw_fc_codes. */
+#define MINW_FC_NOALLOC_SCRATCH_BYTES (8u << 20)
+MINW_API minw_status minw_fc_codes_noalloc(const uint8_t *act, int32_t B, int32_t K,
+                                           int32_t bits_a, const uint8_t *wgt, int32_t O,
+                                           int32_t bits_w, const float *scale,
+                                           const float *shift, const minw_quant *q_out,
+                                           uint8_t *codes_out, uint32_t *planes_out,
+                                           float *y_out, int32_t *acc_out, void *stream);
+
 /* First layer (Sec. III-E): the fp32 image x [B][C][H][W] is NOT quantized;
  * the weights are.  w: latent fp32 weights [O][C][kh][kw]; q_w (host) and
  * channel_scale (nullable) quantize them as minw_pack_weights does; q_w NULL

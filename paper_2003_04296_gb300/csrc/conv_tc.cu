@@ -707,6 +707,17 @@ size_t conv_tc_workspace_bytes(const ConvArgs &a) {
     return tc::thr_ws_bytes(a.O, 7) + (size_t)ks * tc::slice_bytes(tiles, p.BN);
 }
 
+size_t conv_tc_min_split_bytes(const ConvArgs &a) {
+    tc::Params p{};
+    if (a.pool || !tc::plan_shape(a, p)) return 0;
+    const int nbb = (a.B + p.bb - 1) / p.bb;
+    const int tiles = p.nbx * p.nby * nbb * ((a.O + p.BN - 1) / p.BN);
+    const int nk = a.kh * a.kw * (a.C / 128);
+    const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
+    if (tc::auto_ksplit(tiles, nk, sms) < 2) return 0;
+    return tc::thr_ws_bytes(a.O, 7) + 2 * tc::slice_bytes(tiles, p.BN);
+}
+
 bool conv_tc_supported(const ConvArgs &a) {
     tc::Params p{};
     if (!tc::plan_shape(a, p)) return false;

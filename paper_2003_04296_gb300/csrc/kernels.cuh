@@ -64,6 +64,8 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s);
 bool conv_tc_supported(const ConvArgs &a);
 // Workspace the tensor-core path needs to split K for this shape (0: it does not split).
 size_t conv_tc_workspace_bytes(const ConvArgs &a);
+// Smallest workspace with which this shape still splits K (two slices); 0 when it does not split.
+size_t conv_tc_min_split_bytes(const ConvArgs &a);
 // Kernels one tensor-core launch issues for this shape and workspace (2 with a split).
 int conv_tc_launches(const ConvArgs &a);
 minw_status launch_thresholds(const float *scale, const float *shift, int O, const QParams &q, float *out,

@@ -66,6 +66,8 @@ SIGNATURES = {
     "minw_fc_workspace_bytes": (ctypes.c_size_t, [_I32, _I32, _I32]),
     "minw_fc_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _P, _I32, _I32, _P, _P, _QP, _P, _P, _P, _P, _P,
                                      ctypes.c_size_t, _P]),
+    "minw_fc_codes_noalloc": (ctypes.c_int, [_P, _I32, _I32, _I32, _P, _I32, _I32, _P, _P, _QP, _P, _P, _P, _P,
+                                             _P]),
     "minw_net_create": (ctypes.c_int, [ctypes.POINTER(LayerDesc), _I32, _I32, _I32, _P,
                                        ctypes.POINTER(ctypes.c_void_p)]),
     "minw_forward": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
@@ -247,6 +249,15 @@ def minw_fc_codes(act, B, K, bits_a, wgt, O, bits_w, scale=None, shift=None, q_o
                                ctypes.byref(q_out) if q_out is not None else None, _ptr(codes_out),
                                _ptr(planes_out), _ptr(y_out), _ptr(acc_out), _ptr(workspace), nbytes,
                                _stream(stream)), "minw_fc_codes")
+
+
+def minw_fc_codes_noalloc(act, B, K, bits_a, wgt, O, bits_w, scale=None, shift=None, q_out=None,
+                          codes_out=None, planes_out=None, y_out=None, acc_out=None, stream=None):
+    """minw_fc_codes with the library's fixed scratch array (allocates nothing)."""
+    _check(lib().minw_fc_codes_noalloc(_ptr(act), B, K, bits_a, _ptr(wgt), O, bits_w, _ptr(scale), _ptr(shift),
+                                       ctypes.byref(q_out) if q_out is not None else None, _ptr(codes_out),
+                                       _ptr(planes_out), _ptr(y_out), _ptr(acc_out), _stream(stream)),
+           "minw_fc_codes_noalloc")
 
 
 def minw_get_last_device_error(stream=None):
