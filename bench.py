@@ -46,6 +46,28 @@ def _measured_peaks():
 
 
 BF16_TFLOPS, HBM_GBS = _measured_peaks()
+
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "conv_tc_cifar_convnet_a1w1_b256_traffic.json")
+
+
+def _captured_traffic(bound):
+    """DRAM bytes per launch of the tensor-core kernel from the committed ncu
+    capture, or None when the kernel sources changed since the capture."""
+    if bound != "tensor":
+        return None
+    try:
+        import hashlib
+        with open(TRAFFIC_FILE) as f:
+            cap = json.load(f)
+        h = hashlib.sha256()
+        for src in cap["sources"]:
+            with open(os.path.join(ROOT, src), "rb") as f:
+                h.update(f.read())
+        if h.hexdigest() != cap["sources_sha256"]:
+            return None
+        return cap["dram_bytes_per_launch"]
+    except (OSError, KeyError, ValueError):
+        return None
 FP8_TFLOPS = 2.0 * BF16_TFLOPS
 
 
@@ -284,6 +306,7 @@ def run_gpu(args, rank, world, local_rank):
                     "frac": achieved / peak, "traffic": None,
                     "peak_basis": "16 popc/clk/SM x 32 MAC/popc x 2 ops x 152 SMs x 2070 MHz"}
     roofline["layer_variants"] = variants
+    roofline["traffic"] = _captured_traffic(roofline["bound"])
 
     cpu = None
     if world == 1 and not args.skip_cpu:
