@@ -196,7 +196,7 @@ MINW_API minw_status minw_pack_weight_codes(const float *w, int32_t O, int32_t C
                                             void *stream);
 
 /* minw_conv2d on codes operands, run on the tcgen05 tensor cores.
- * Supported: stride 1, C % 128 == 0, pad < kh, kw; otherwise
+ * Supported: stride 1 or 2, C % 64 == 0, pad < kh, kw; otherwise
  * MINW_EUNSUPPORTED.  bits_a / bits_w document the operands (1..3). */
 MINW_API minw_status minw_conv2d_codes(const uint8_t *act, int32_t B, int32_t C, int32_t H,
                                        int32_t W, int32_t bits_a, const uint8_t *wgt,
@@ -215,6 +215,33 @@ MINW_API minw_status minw_conv_block_codes(const uint8_t *act, int32_t B, int32_
                                            const float *shift, const minw_quant *q_out,
                                            uint8_t *codes_out, uint32_t *planes_out,
                                            float *y_out, void *stream);
+
+/* Extra inputs and outputs of a residual block (ResNet-style MINW-Net,
+ * where the paper leaves the block wiring open).  Host struct.
+ * res_codes (nullable): shortcut as level codes [B][Hp][Wp][O] of bit width
+ *   res_bits (its levels are added as values: 3-bit codes count quarters).
+ * res_f32 (nullable): shortcut as fp32 NHWC [B][Hp][Wp][O].
+ * y_nhwc (nullable, output): the BN output before the shortcut, fp32 NHWC.
+ * With a shortcut the block computes y = fmaf(acc, scale, shift) + shortcut
+ * (one fp32 add), then HardTanh and the output quantizer. */
+typedef struct {
+    const uint8_t *res_codes;
+    int32_t res_bits;
+    const float *res_f32;
+    float *y_nhwc;
+} minw_block_extra;
+
+/* minw_conv_block_codes with the residual inputs / outputs of extra
+ * (nullable).  At most one shortcut. */
+MINW_API minw_status minw_conv_block_codes_ex(const uint8_t *act, int32_t B, int32_t C,
+                                              int32_t H, int32_t W, int32_t bits_a,
+                                              const uint8_t *wgt, int32_t O, int32_t kh,
+                                              int32_t kw, int32_t bits_w, int32_t stride,
+                                              int32_t pad, int32_t pool, const float *scale,
+                                              const float *shift, const minw_quant *q_out,
+                                              uint8_t *codes_out, uint32_t *planes_out,
+                                              float *y_out, const minw_block_extra *extra,
+                                              void *stream);
 
 /* Fully connected layer a~ = a^q W^q (Algorithm 1, inference) on the tensor
  * cores, with the reduction over K split across CTAs when the output alone

@@ -103,7 +103,7 @@ static minw_status make_codes_args(ConvArgs &a, const uint8_t *act, int B, int C
         return MINW_EINVAL;
     if (bits_a < 1 || bits_a > 3 || bits_w < 1 || bits_w > 3) return MINW_EINVAL;
     if (!act || !wgt || !aligned16(act) || !aligned16(wgt)) return MINW_EINVAL;
-    if (C % 128 != 0 || stride != 1 || pad >= kh || pad >= kw) return MINW_EUNSUPPORTED;
+    if (C % 64 != 0 || (stride != 1 && stride != 2) || pad >= kh || pad >= kw) return MINW_EUNSUPPORTED;
     const int Ho = (H + 2 * pad - kh) / stride + 1;
     const int Wo = (W + 2 * pad - kw) / stride + 1;
     if (Ho <= 0 || Wo <= 0) return MINW_EINVAL;
@@ -155,6 +155,41 @@ minw_status minw_conv_block_codes(const uint8_t *act, int32_t B, int32_t C, int3
     a.planes_out = planes_out;
     a.codes_out = q_out ? codes_out : nullptr;
     a.y_out = y_out;
+    return launch_conv_tc(a, (cudaStream_t)stream);
+}
+
+minw_status minw_conv_block_codes_ex(const uint8_t *act, int32_t B, int32_t C, int32_t H, int32_t W,
+                                     int32_t bits_a, const uint8_t *wgt, int32_t O, int32_t kh, int32_t kw,
+                                     int32_t bits_w, int32_t stride, int32_t pad, int32_t pool,
+                                     const float *scale, const float *shift, const minw_quant *q_out,
+                                     uint8_t *codes_out, uint32_t *planes_out, float *y_out,
+                                     const minw_block_extra *extra, void *stream) {
+    ConvArgs a;
+    minw_status st = make_codes_args(a, act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad);
+    if (st != MINW_OK) return st;
+    if (!scale || !shift) return MINW_EINVAL;
+    if (q_out && (!valid_quant(q_out) || (!planes_out && !codes_out))) return MINW_EINVAL;
+    if (codes_out && (O % 16 != 0 || !aligned16(codes_out))) return MINW_EUNSUPPORTED;
+    if (pool != 0 && pool != 1) return MINW_EINVAL;
+    if (pool && ((a.Ho & 1) || (a.Wo & 1))) return MINW_EUNSUPPORTED;
+    if (extra && extra->res_codes && extra->res_f32) return MINW_EINVAL;
+    if (extra && extra->res_codes && (extra->res_bits < 1 || extra->res_bits > 3)) return MINW_EINVAL;
+    const bool any_out = q_out || y_out || (extra && extra->y_nhwc);
+    if (!any_out) return MINW_EINVAL;
+    a.scale = scale;
+    a.shift = shift;
+    a.pool = pool;
+    a.quant_out = q_out != nullptr;
+    if (q_out) a.qo = to_qparams(q_out);
+    a.planes_out = planes_out;
+    a.codes_out = q_out ? codes_out : nullptr;
+    a.y_out = y_out;
+    if (extra) {
+        a.res_codes = extra->res_codes;
+        a.res_unit = extra->res_bits == 3 ? 0.25f : 1.0f;
+        a.res_f32 = extra->res_f32;
+        a.y_nhwc = extra->y_nhwc;
+    }
     return launch_conv_tc(a, (cudaStream_t)stream);
 }
 

@@ -44,11 +44,14 @@ namespace tc {
 constexpr int NT = 352;                 // 11 warps: TMA (A), MMA, 8 epilogue, TMA (B)
 constexpr int EPI_WARPS = 8;            // two per TMEM lane quarter, each half of the columns
 constexpr int B_WARP = 2 + EPI_WARPS;   // the weight-box TMA warp
-constexpr int A_BYTES = 128 * 128;
+
 constexpr long long WAIT_CYCLES = 1ll << 31;
 
 struct Params {
     int B, C, H, W, O, kh, kw, pad, Ho, Wo;
+    int stride;                // 1 or 2 (TMA element strides)
+    int ck;                    // bytes (= channels) per K chunk: 128 (128-byte swizzle) or 64 (64-byte swizzle)
+    uint32_t a_bytes;          // activation box bytes per stage: 128 rows x ck
     int bw, bh, bb, nbx, nby, nbb, ntn;
     int BN, nck, nk, S;
     uint32_t stage_bytes, idesc, tmem_cols;
@@ -56,6 +59,11 @@ struct Params {
     int nlev;                  // levels of the output quantizer
     int ksplit;                // K slices per output tile (1: no split)
     int32_t *part;             // split-K: int32 partial sums [ksplit][tiles][128][BN]
+    // residual blocks: y = BN(acc) + shortcut, then HardTanh + quantize
+    const uint8_t *res_codes;  // shortcut as level codes [B][Hp][Wp][O] (nullable)
+    float res_unit;            // value of one level unit of res_codes (1 or 1/4)
+    const float *res_f32;      // shortcut as fp32 NHWC [B][Hp][Wp][O] (nullable)
+    float *y_nhwc;             // BN output (before the shortcut) as fp32 NHWC (nullable)
     int32_t *acc_out;
     float *y_out;
     const float *scale, *shift;
@@ -120,14 +128,22 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, u
 }
 
 // Shared-memory matrix descriptor of a K-major operand tile stored as rows of
-// 128 bytes with the 128-byte swizzle: 8-row groups 1024 bytes apart.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+// ck bytes with the ck-byte swizzle (ck = 128 or 64): 8-row groups 8*ck bytes
+// apart.
+__device__ __forceinline__ uint64_t sw_desc(uint32_t saddr, int ck) {
     uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);   // start address
     d |= (uint64_t)1 << 16;                             // leading byte offset (unused here)
-    d |= (uint64_t)(1024 >> 4) << 32;                   // stride byte offset: next 8 rows
+    d |= (uint64_t)((8 * ck) >> 4) << 32;               // stride byte offset: next 8 rows
     d |= (uint64_t)1 << 46;                             // descriptor version
-    d |= (uint64_t)2 << 61;                             // 128-byte swizzle
+    d |= (uint64_t)(ck == 128 ? 2 : 4) << 61;           // 128- or 64-byte swizzle
     return d;
+}
+
+// Value of an E4M3 level code in integer units (0, +-1, +-2, +-4).
+__device__ __forceinline__ float code_units(uint32_t c) {
+    if ((c & 0x7Fu) == 0u) return 0.0f;
+    const float m = (float)(1u << (((c >> 3) & 0xFu) - 7u));
+    return (c & 0x80u) ? -m : m;
 }
 
 __device__ __forceinline__ void mma_f8(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
@@ -246,7 +262,7 @@ __global__ void __launch_bounds__(NT, 1)
             const bool act = warp == 0;
             const CUtensorMap *map = act ? &tmA : &tmB;
             asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
-            const uint32_t bytes = act ? (uint32_t)A_BYTES : p.stage_bytes - (uint32_t)A_BYTES;
+            const uint32_t bytes = act ? p.a_bytes : p.stage_bytes - p.a_bytes;
             int g = 0, s = 0, lap = 0;             // stages issued, ring slot, ring lap
             bool alive = true;
             for (int w = blockIdx.x; w < items && alive; w += gridDim.x) {
@@ -254,12 +270,12 @@ __global__ void __launch_bounds__(NT, 1)
                 const int kb = (int)((long long)kp * p.nk / p.ksplit), ke = (int)((long long)(kp + 1) * p.nk / p.ksplit);
                 const int tn = t / tiles_m, tm = t - tn * tiles_m;
                 const int xb = tm % p.nbx, yb = (tm / p.nbx) % p.nby, bbk = tm / (p.nbx * p.nby);
-                const int x0 = xb * p.bw - p.pad, y0 = yb * p.bh - p.pad, b0 = bbk * p.bb;
+                const int x0 = xb * p.bw * p.stride - p.pad, y0 = yb * p.bh * p.stride - p.pad, b0 = bbk * p.bb;
                 const int o0 = tn * p.BN;
                 // channel chunk, tap and weight column of stage kb
                 const int tap0 = kb / p.nck;
-                int c0 = (kb - tap0 * p.nck) * 128, ky = tap0 / p.kw, kx = tap0 - (tap0 / p.kw) * p.kw;
-                int kcol = kb * 128;
+                int c0 = (kb - tap0 * p.nck) * p.ck, ky = tap0 / p.kw, kx = tap0 - (tap0 / p.kw) * p.kw;
+                int kcol = kb * p.ck;
                 for (int ks = kb; ks < ke; ++ks, ++g) {
                     // slot reuse: wait until the MMAs of the previous lap released it
                     if (lap > 0 && !mbar_wait(&empty[s], (lap - 1) & 1)) { alive = false; break; }
@@ -268,9 +284,9 @@ __global__ void __launch_bounds__(NT, 1)
                     if (act)
                         tma_load_4d(sa, &tmA, &full[s], c0, x0 + kx, y0 + ky, b0);
                     else
-                        tma_load_2d(sa + A_BYTES, &tmB, &full[s], kcol, o0);
-                    kcol += 128;
-                    c0 += 128;
+                        tma_load_2d(sa + p.a_bytes, &tmB, &full[s], kcol, o0);
+                    kcol += p.ck;
+                    c0 += p.ck;
                     if (c0 == p.C) {
                         c0 = 0;
                         if (++kx == p.kw) { kx = 0; ++ky; }
@@ -300,10 +316,10 @@ __global__ void __launch_bounds__(NT, 1)
                     if (!mbar_wait(&full[s], fphase)) { alive = false; break; }
                     fence_after();
                     const uint32_t sa = sbase + (uint32_t)s * p.stage_bytes;
-                    const uint64_t adesc = sw128_desc(sa);
-                    const uint64_t bdesc = sw128_desc(sa + A_BYTES);
-#pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
+                    const uint64_t adesc = sw_desc(sa, p.ck);
+                    const uint64_t bdesc = sw_desc(sa + p.a_bytes, p.ck);
+                    const int nmma = p.ck >> 5;                  // K = 32 bytes per MMA
+                    for (int kk = 0; kk < nmma; ++kk)
                         mma_f8(tmem_d, adesc + 2 * kk, bdesc + 2 * kk, p.idesc, (ks != kb) || (kk != 0));
                     mma_commit(&empty[s]);
                     if (++s == p.S) { s = 0; fphase ^= 1; }
@@ -357,7 +373,8 @@ __global__ void __launch_bounds__(NT, 1)
                         if (ob + j < p.O)
                             p.acc_out[(((long long)b * p.O + ob + j) * p.Ho + y) * p.Wo + x] = __float2int_rn(a[j]);
                 }
-                if (p.y_out != nullptr && writer) {
+                const bool resid = p.res_codes != nullptr || p.res_f32 != nullptr || p.y_nhwc != nullptr;
+                if (p.y_out != nullptr && writer && !resid) {
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
                         const int o = ob + j;
@@ -368,7 +385,51 @@ __global__ void __launch_bounds__(NT, 1)
                         }
                     }
                 }
-                if constexpr (OUTB > 0) {
+                if (resid) {
+                    // residual block: y = BN(acc) [+ shortcut], HardTanh, quantize,
+                    // element by element in the fp32 order of the block
+                    if (writer) {
+                        uint32_t cw[4] = {0u, 0u, 0u, 0u};
+                        uint32_t bits16[3] = {0u, 0u, 0u};
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            const int o = ob + j;
+                            if (o >= p.O) continue;
+                            float yv = fmaf(a[j], __ldg(p.scale + o), __ldg(p.shift + o));
+                            if (p.y_nhwc != nullptr) p.y_nhwc[opix * p.O + o] = yv;
+                            if (p.res_codes != nullptr) yv += code_units(__ldg(p.res_codes + opix * p.O + o)) * p.res_unit;
+                            else if (p.res_f32 != nullptr) yv += __ldg(p.res_f32 + opix * p.O + o);
+                            if (p.y_out != nullptr)
+                                p.y_out[(((long long)b * p.O + o) * Hp + yp) * Wp + xp] =
+                                    (OUTB > 0) ? fminf(fmaxf(yv, -1.0f), 1.0f) : yv;
+                            if constexpr (OUTB > 0) {
+                                const int k = level_index_of_y(yv, p.qo);
+                                cw[j >> 2] |= code_k<OUTB>(k) << ((j & 3) * 8);
+                                const uint32_t pb = planes_k<OUTB>(k);
+#pragma unroll
+                                for (int u = 0; u < OUTB; ++u) bits16[u] |= ((pb >> u) & 1u) << j;
+                            }
+                        }
+                        if constexpr (OUTB > 0) {
+                            if (p.codes_out != nullptr)
+                                *reinterpret_cast<uint4 *>(p.codes_out + opix * p.O + ob) =
+                                    make_uint4(cw[0], cw[1], cw[2], cw[3]);
+                            if (p.planes_out != nullptr) {
+                                const int half = (ob >> 4) & 1;
+#pragma unroll
+                                for (int u = 0; u < OUTB; ++u) pw[u] |= bits16[u] << (16 * half);
+                                if (half == 1 || ch == p.BN / 16 - 1 || ob + 16 >= p.O) {
+                                    uint32_t *dst = p.planes_out + (opix * OUTB) * NWo + (ob >> 5);
+#pragma unroll
+                                    for (int u = 0; u < OUTB; ++u) {
+                                        dst[u * NWo] = pw[u];
+                                        pw[u] = 0u;
+                                    }
+                                }
+                            }
+                        }
+                    }
+                } else if constexpr (OUTB > 0) {
                     if (writer) {
                         int kq[16];
 #pragma unroll
@@ -582,7 +643,7 @@ struct Plan {
 };
 
 static bool plan_shape(const ConvArgs &a, Params &p) {
-    if (a.stride != 1 || a.C % 128 != 0 || a.pad >= a.kh || a.pad >= a.kw) return false;
+    if ((a.stride != 1 && a.stride != 2) || a.C % 64 != 0 || a.pad >= a.kh || a.pad >= a.kw) return false;
     int bw = pow2_ceil(a.Wo);
     if (bw > 128) bw = 128;
     if (a.pool && bw > 16) bw = 16;
@@ -617,13 +678,16 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     if (!plan_shape(a, p)) return MINW_EUNSUPPORTED;
     p.B = a.B; p.C = a.C; p.H = a.H; p.W = a.W; p.O = a.O; p.kh = a.kh; p.kw = a.kw; p.pad = a.pad;
     p.Ho = a.Ho; p.Wo = a.Wo;
-    p.nck = a.C / 128;
+    p.stride = a.stride;
+    p.ck = (a.C % 128 == 0) ? 128 : 64;
+    p.a_bytes = (uint32_t)(128 * p.ck);
+    p.nck = a.C / p.ck;
     p.nk = a.kh * a.kw * p.nck;
     p.nbb = (a.B + p.bb - 1) / p.bb;
     p.ntn = (a.O + p.BN - 1) / p.BN;
     p.nlev = a.quant_out ? num_levels(a.qo.bits) : 0;
     p.thr = a.thr;
-    p.stage_bytes = (uint32_t)(A_BYTES + p.BN * 128);
+    p.stage_bytes = p.a_bytes + (uint32_t)(p.BN * p.ck);
     const size_t thr_bytes = a.quant_out ? ((size_t)a.O * p.nlev + 2) * sizeof(float) : 0;
     const size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes;
     int S = (int)(budget / p.stage_bytes);
@@ -637,16 +701,19 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     p.acc_out = a.acc_out; p.y_out = a.y_out; p.scale = a.scale; p.shift = a.shift;
     p.pool = a.pool; p.quant_out = a.quant_out; p.qo = a.qo;
     p.planes_out = a.planes_out; p.codes_out = a.codes_out;
+    p.res_codes = a.res_codes; p.res_unit = a.res_unit; p.res_f32 = a.res_f32; p.y_nhwc = a.y_nhwc;
 
     EncodeTiledFn enc = encode_fn();
     if (enc == nullptr) return MINW_ECUDA;
+    const CUtensorMapSwizzle swz = p.ck == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
     {
         const cuuint64_t dims[4] = {(cuuint64_t)a.C, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.B};
         const cuuint64_t strides[3] = {(cuuint64_t)a.C, (cuuint64_t)a.W * a.C, (cuuint64_t)a.H * a.W * a.C};
-        const cuuint32_t box[4] = {128u, (cuuint32_t)p.bw, (cuuint32_t)p.bh, (cuuint32_t)p.bb};
-        const cuuint32_t es[4] = {1u, 1u, 1u, 1u};
+        const cuuint32_t sd = (cuuint32_t)p.stride;
+        const cuuint32_t box[4] = {(cuuint32_t)p.ck, (cuuint32_t)p.bw * sd, (cuuint32_t)p.bh * sd, (cuuint32_t)p.bb};
+        const cuuint32_t es[4] = {1u, sd, sd, 1u};
         if (enc(&pl.tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<uint8_t *>(a.act8), dims, strides, box, es,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return MINW_ECUDA;
     }
@@ -654,10 +721,10 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
         const long long K = (long long)a.kh * a.kw * a.C;
         const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)a.O};
         const cuuint64_t strides[1] = {(cuuint64_t)K};
-        const cuuint32_t box[2] = {128u, (cuuint32_t)p.BN};
+        const cuuint32_t box[2] = {(cuuint32_t)p.ck, (cuuint32_t)p.BN};
         const cuuint32_t es[2] = {1u, 1u};
         if (enc(&pl.tmB, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(a.wgt8), dims, strides, box, es,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return MINW_ECUDA;
     }
@@ -700,7 +767,7 @@ size_t conv_tc_workspace_bytes(const ConvArgs &a) {
     if (a.pool || !tc::plan_shape(a, p)) return 0;
     const int nbb = (a.B + p.bb - 1) / p.bb;
     const int tiles = p.nbx * p.nby * nbb * ((a.O + p.BN - 1) / p.BN);
-    const int nk = a.kh * a.kw * (a.C / 128);
+    const int nk = a.kh * a.kw * (a.C / ((a.C % 128 == 0) ? 128 : 64));
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
     const int ks = tc::auto_ksplit(tiles, nk, sms);
     if (ks < 2) return 0;
@@ -712,7 +779,7 @@ size_t conv_tc_min_split_bytes(const ConvArgs &a) {
     if (a.pool || !tc::plan_shape(a, p)) return 0;
     const int nbb = (a.B + p.bb - 1) / p.bb;
     const int tiles = p.nbx * p.nby * nbb * ((a.O + p.BN - 1) / p.BN);
-    const int nk = a.kh * a.kw * (a.C / 128);
+    const int nk = a.kh * a.kw * (a.C / ((a.C % 128 == 0) ? 128 : 64));
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
     if (tc::auto_ksplit(tiles, nk, sms) < 2) return 0;
     return tc::thr_ws_bytes(a.O, 7) + 2 * tc::slice_bytes(tiles, p.BN);

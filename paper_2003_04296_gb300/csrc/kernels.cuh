@@ -27,6 +27,11 @@ struct ConvArgs {
     const uint8_t *act8;   // [B][H][W][C]
     const uint8_t *wgt8;   // [O][kh][kw][C]
     const float *thr;      // output-quantizer breakpoints [O][levels] (nullable: computed in-kernel)
+    // residual blocks (tensor-core path): y = BN(acc) + shortcut before HardTanh + quantize
+    const uint8_t *res_codes;  // shortcut as level codes [B][Hp][Wp][O] (nullable)
+    float res_unit;            // value of one level unit of res_codes
+    const float *res_f32;      // shortcut as fp32 NHWC (nullable)
+    float *y_nhwc;             // BN output before the shortcut, fp32 NHWC (nullable)
     // split-K (tensor-core path): zero-initialised workspace, left zero by every call
     void *workspace;       // nullable: no split
     size_t workspace_bytes;

@@ -30,6 +30,11 @@ class Quant(ctypes.Structure):
     _fields_ = [("bits", ctypes.c_int32), ("thr", ctypes.c_float * 3), ("scale", ctypes.c_float)]
 
 
+class BlockExtra(ctypes.Structure):
+    _fields_ = [("res_codes", ctypes.c_void_p), ("res_bits", ctypes.c_int32), ("res_f32", ctypes.c_void_p),
+                ("y_nhwc", ctypes.c_void_p)]
+
+
 class LayerDesc(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int32), ("C", ctypes.c_int32), ("H", ctypes.c_int32),
                 ("W", ctypes.c_int32), ("O", ctypes.c_int32), ("kh", ctypes.c_int32),
@@ -63,6 +68,9 @@ SIGNATURES = {
                                          _I32, _I32, _P, _P, _P, _P, _P]),
     "minw_conv_block_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32,
                                              _I32, _I32, _I32, _P, _P, _QP, _P, _P, _P, _P]),
+    "minw_conv_block_codes_ex": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32,
+                                                _I32, _I32, _I32, _P, _P, _QP, _P, _P, _P,
+                                                ctypes.POINTER(BlockExtra), _P]),
     "minw_fc_workspace_bytes": (ctypes.c_size_t, [_I32, _I32, _I32]),
     "minw_fc_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _P, _I32, _I32, _P, _P, _QP, _P, _P, _P, _P, _P,
                                      ctypes.c_size_t, _P]),
@@ -236,6 +244,21 @@ def minw_conv_block_codes(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, strid
                                        ctypes.byref(q_out) if q_out is not None else None,
                                        _ptr(codes_out), _ptr(planes_out), _ptr(y_out), _stream(stream)),
            "minw_conv_block_codes")
+
+
+def minw_conv_block_codes_ex(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad, pool, scale, shift,
+                             q_out=None, codes_out=None, planes_out=None, y_out=None, res_codes=None, res_bits=0,
+                             res_f32=None, y_nhwc=None, stream=None):
+    ex = BlockExtra()
+    ex.res_codes = res_codes.data_ptr() if res_codes is not None else None
+    ex.res_bits = int(res_bits)
+    ex.res_f32 = res_f32.data_ptr() if res_f32 is not None else None
+    ex.y_nhwc = y_nhwc.data_ptr() if y_nhwc is not None else None
+    _check(lib().minw_conv_block_codes_ex(_ptr(act), B, C, H, W, bits_a, _ptr(wgt), O, kh, kw, bits_w, stride, pad,
+                                          int(pool), _ptr(scale), _ptr(shift),
+                                          ctypes.byref(q_out) if q_out is not None else None, _ptr(codes_out),
+                                          _ptr(planes_out), _ptr(y_out), ctypes.byref(ex), _stream(stream)),
+           "minw_conv_block_codes_ex")
 
 
 def minw_fc_workspace_bytes(B, K, O):

@@ -166,12 +166,16 @@ def test_exact_at_largest_magnitudes(dev, M, bits, C, k, hw):
 
 
 def test_codes_argument_errors(dev, M):
+    """Shapes outside the tensor-core path are rejected on the host before any
+    launch (the tiny buffers are never read)."""
     t = torch.empty(4096, dtype=torch.uint8, device=dev)
     a = torch.empty(64, dtype=torch.int32, device=dev)
-    with pytest.raises(M.MinwError):   # C % 128 != 0 is outside the tensor-core path
-        M.minw_conv2d_codes(t, 1, 64, 4, 4, 1, t, 8, 3, 3, 1, 1, 1, acc_out=a)
-    with pytest.raises(M.MinwError):   # stride 2 is outside the tensor-core path
-        M.minw_conv2d_codes(t, 1, 128, 4, 4, 1, t, 8, 3, 3, 1, 2, 1, acc_out=a)
+    with pytest.raises(M.MinwError) as e1:   # C % 64 != 0
+        M.minw_conv2d_codes(t, 1, 32, 4, 4, 1, t, 8, 3, 3, 1, 1, 1, acc_out=a)
+    assert e1.value.status == M.MINW_EUNSUPPORTED
+    with pytest.raises(M.MinwError) as e2:   # stride 3
+        M.minw_conv2d_codes(t, 1, 128, 4, 4, 1, t, 8, 3, 3, 1, 3, 1, acc_out=a)
+    assert e2.value.status == M.MINW_EUNSUPPORTED
 
 
 def _fc_problem(seed, B, K, O, ba, bw):
@@ -218,3 +222,64 @@ def test_fc_split_k(dev, M, B, K, Oc, ba, bw):
         assert np.array_equal(decode_e4m3(outs[0]), lv * 2.0 ** O.units_shift(ba))
         assert np.array_equal(outs[0], outs[2]) and np.array_equal(outs[0], outs[3])
     assert M.minw_get_last_device_error() == M.MINW_OK
+
+
+TC_STRIDED = [
+    # B, C, H, W, O, k, stride, pad
+    (2, 64, 9, 7, 70, 3, 1, 1),       # 64-channel input: 64-byte K chunks
+    (2, 128, 16, 16, 128, 3, 2, 1),   # stride 2
+    (1, 128, 15, 13, 32, 3, 2, 1),    # stride 2, odd sizes
+    (2, 64, 14, 14, 128, 1, 2, 0),    # 1x1 / 2 downsample, 64 channels
+    (3, 64, 56, 56, 64, 3, 1, 1),     # ResNet layer-1 shape (partial tiles at the right edge)
+]
+
+
+@pytest.mark.parametrize("case", TC_STRIDED)
+@pytest.mark.parametrize("ba,bw", [(1, 1), (3, 3), (2, 1)])
+def test_conv2d_codes_strided_and_64ch(dev, M, case, ba, bw):
+    B, C, H, W, O_, k, s, pad = case
+    p = conv_problem(hash((case, ba, bw, "s")) % 1000, B, C, H, W, O_, k, k, s, pad, ba, bw, w_sigma=0.5)
+    act, wgt = _operands(dev, M, p)
+    Ho = (H + 2 * pad - k) // s + 1
+    Wo = (W + 2 * pad - k) // s + 1
+    acc = torch.full((B, O_, Ho, Wo), -7, dtype=torch.int32, device=dev)
+    M.minw_conv2d_codes(act, B, C, H, W, ba, wgt, O_, k, k, bw, s, pad, acc_out=acc)
+    ref = _ref_acc(p)
+    got = acc.cpu().numpy()
+    assert np.array_equal(got, ref), f"{np.sum(got != ref)} of {ref.size} accumulators differ"
+
+
+@pytest.mark.parametrize("shortcut", ["codes", "f32"])
+@pytest.mark.parametrize("bits", [3, 1])
+def test_residual_block_epilogue(dev, M, shortcut, bits):
+    """y = fmaf(acc, scale, shift) + shortcut (one fp32 add), HardTanh, quantize;
+    the shortcut is a level-code tensor (identity path) or fp32 NHWC (the
+    downsample path, itself produced by a block that writes its BN output)."""
+    B, C, H, W, O_ = 2, 128, 10, 12, 128
+    p = conv_problem(71 + bits, B, C, H, W, O_, 3, 3, 1, 1, bits, bits, w_sigma=0.5)
+    act, wgt = _operands(dev, M, p)
+    sc, sh = dev_tensor(p["scale"], dev), dev_tensor(p["shift"], dev)
+    acc_ref = _ref_acc(p)
+    y_bn = O.affine(acc_ref, p["scale"], p["shift"])                      # NCHW fp32
+    r = np.random.default_rng(5)
+    if shortcut == "codes":
+        xs = (r.standard_normal((B, O_, H, W)) * 0.7).astype(np.float32)
+        res_lv = O.quantize(xs, bits, DEFAULT_THR[bits])                 # dequantized levels
+        res_codes = torch.empty((B, H, W, O_), dtype=torch.uint8, device=dev)
+        M.aqe_quantize_codes(dev_tensor(xs, dev), M.quant(bits, DEFAULT_THR[bits]), res_codes)
+        kw = dict(res_codes=res_codes, res_bits=bits)
+        res = res_lv.astype(np.float32)
+    else:
+        res = (r.standard_normal((B, O_, H, W)) * 0.5).astype(np.float32)
+        kw = dict(res_f32=dev_tensor(res.transpose(0, 2, 3, 1), dev))
+    y_nhwc = torch.empty((B, H, W, O_), dtype=torch.float32, device=dev)
+    codes = torch.empty((B, H, W, O_), dtype=torch.uint8, device=dev)
+    y = torch.empty((B, O_, H, W), dtype=torch.float32, device=dev)
+    M.minw_conv_block_codes_ex(act, B, C, H, W, bits, wgt, O_, 3, 3, bits, 1, 1, 0, sc, sh,
+                               q_out=M.quant(bits, DEFAULT_THR[bits]), codes_out=codes, y_out=y, y_nhwc=y_nhwc,
+                               **kw)
+    assert np.array_equal(y_nhwc.cpu().numpy(), y_bn.transpose(0, 2, 3, 1))
+    yr = O.hardtanh((y_bn + res).astype(np.float32))
+    assert np.array_equal(y.cpu().numpy(), yr)
+    lv = O.quantize(yr, bits, DEFAULT_THR[bits])
+    assert np.array_equal(decode_e4m3(codes.cpu().numpy()), (lv * 2.0 ** O.units_shift(bits)).transpose(0, 2, 3, 1))
