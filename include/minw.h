@@ -362,6 +362,37 @@ MINW_API minw_status minw_net_layer_times(minw_net *net, float *ms);
  * 0 for the fp32 first layer, else MINW_VARIANT_POPC or MINW_VARIANT_TC. */
 MINW_API minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants);
 
+/* ResNet-18-shaped MINW-Net (Table V's network).  The paper leaves the
+ * residual wiring open; the reading implemented here:
+ *   stem: fp32 7x7/2 conv (fp32 weights, pad 3) -> 3x3/2 max pool (pad 1) ->
+ *         BN -> HardTanh -> quantize (the block order of Sec. III-E);
+ *   block (widths 64-128-256-512, two per stage, stride 2 entering stages
+ *         2-4): u = quantized input; v = h(HardTanh(BN1(conv1(u))));
+ *         y = BN2(conv2(v)) + s with s = u, or s = BN_d(conv_d(u)) for the
+ *         1x1 / 2 shortcut of the first block of stages 2-4 (fp32 sum);
+ *         output h(HardTanh(y));
+ *   head: global average pool of the last levels -> fp32 fully connected
+ *         layer [classes][512] -> BN -> fp32 logits.
+ * Every convolution weight of the blocks is quantized with (bits_w, thr_w)
+ * and its per-output-channel prescale (nullable); activations with
+ * (bits_a, thr_a).  conv_w[2b], conv_w[2b+1]: block b's two convolutions
+ * [O][C][3][3]; down_*[i]: the shortcut of stage i+2 [O][C][1][1].
+ * image_hw: multiple of 32 (224 for ImageNet crops).  Device pointers, read
+ * during creation only.  minw_forward then takes x [B][3][hw][hw] and writes
+ * logits [B][num_classes]. */
+typedef struct {
+    int32_t bits_a, bits_w;
+    float thr_a[3], thr_w[3];
+    int32_t image_hw, num_classes;
+    const float *stem_w, *stem_scale, *stem_shift;
+    const float *conv_w[16], *conv_wscale[16], *conv_scale[16], *conv_shift[16];
+    const float *down_w[3], *down_wscale[3], *down_scale[3], *down_shift[3];
+    const float *fc_w, *fc_scale, *fc_shift;
+} minw_resnet18_desc;
+
+MINW_API minw_status minw_resnet18_create(const minw_resnet18_desc *desc, int32_t max_batch,
+                                          void *stream, minw_net **out);
+
 /* Number of layers (and of entries minw_net_layer_times fills). */
 MINW_API int32_t minw_net_launches(const minw_net *net);
 

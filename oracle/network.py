@@ -67,3 +67,43 @@ def convnet_forward(net, x, keep=False):
 def activation_levels(y, bits, thr):
     """Quantized levels h(y) of a layer output (what the next layer consumes)."""
     return O.quantize(y, bits, thr)
+
+
+def resnet18_forward(net, x, keep=False):
+    """Forward pass of the ResNet-18-shaped MINW-Net built by
+    ``inputs.resnet18_params``.  The paper leaves the residual wiring open;
+    the reading followed (one fp32 operation per written step):
+      stem : fp32 7x7/2 conv (fp32 weights, pad 3) -> 3x3/2 max pool (pad 1)
+             -> BN -> HardTanh -> h  (the block order of Sec. III-E)
+      block: u = h(x); v = h(HardTanh(BN1(conv1(u))));
+             y = BN2(conv2(v)) + s, s = u or BN_d(conv_d(u)) (1x1 / 2);
+             next input = HardTanh(y) (quantized by the next block's h)
+      head : global average pool of h(last output) -> fp32 FC -> BN."""
+    ba, bw = net["bits_a"], net["bits_w"]
+    ta, tw = net["thr_a"], net["thr_w"]
+    st = net["stem"]
+    z = O.conv2d_f32_seq(x, st["w"], 2, 3)
+    z = O.maxpool_f32(z, 3, 2, 1)
+    a = O.hardtanh(O.affine(z, st["scale"], st["shift"]))
+    trace = [a]
+    for blk in net["blocks"]:
+        u = O.quantize(a, ba, ta)
+        c1, c2 = blk["c1"], blk["c2"]
+        w1 = O.quantize(c1["w"], bw, tw, c1["w_scale"])
+        acc1 = O.conv2d_levels(u, w1, blk["stride"], 1, ba, bw)
+        v = O.quantize(O.hardtanh(O.affine(acc1, c1["scale"], c1["shift"])), ba, ta)
+        w2 = O.quantize(c2["w"], bw, tw, c2["w_scale"])
+        y = O.affine(O.conv2d_levels(v, w2, 1, 1, ba, bw), c2["scale"], c2["shift"])
+        if blk["down"] is None:
+            s = u.astype(np.float32)
+        else:
+            d = blk["down"]
+            wd = O.quantize(d["w"], bw, tw, d["w_scale"])
+            s = O.affine(O.conv2d_levels(u, wd, 2, 0, ba, bw), d["scale"], d["shift"])
+        a = O.hardtanh((y + s).astype(np.float32))
+        trace.append(a)
+    last = O.quantize(a, ba, ta).astype(np.float32)
+    pooled = O.avgpool_f32(last)
+    fc = net["fc"]
+    logits = O.affine(O.linear_f32_seq(pooled, fc["w"]), fc["scale"], fc["shift"])
+    return (logits, trace) if keep else logits

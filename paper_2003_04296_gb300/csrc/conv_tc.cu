@@ -559,10 +559,23 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const Params p, cons
     if (valid && p.acc_out != nullptr)
         for (int j = 0; j < 4; ++j)
             if (o + j < p.O) p.acc_out[((long long)b * p.O + o + j) * HoWo + (long long)y * p.Wo + x] = acc[j];
-    if (valid && p.y_out != nullptr)
+    // residual blocks: y = BN(acc) [+ shortcut], element by element as in the
+    // single-pass epilogue; yres holds the HardTanh input
+    const bool resid = p.res_codes != nullptr || p.res_f32 != nullptr || p.y_nhwc != nullptr;
+    float yres[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    if (valid && resid)
         for (int j = 0; j < 4; ++j)
             if (o + j < p.O) {
                 float yv = fmaf((float)acc[j], __ldg(p.scale + o + j), __ldg(p.shift + o + j));
+                if (p.y_nhwc != nullptr) p.y_nhwc[pix * p.O + o + j] = yv;
+                if (p.res_codes != nullptr) yv += code_units(__ldg(p.res_codes + pix * p.O + o + j)) * p.res_unit;
+                else if (p.res_f32 != nullptr) yv += __ldg(p.res_f32 + pix * p.O + o + j);
+                yres[j] = yv;
+            }
+    if (valid && p.y_out != nullptr)
+        for (int j = 0; j < 4; ++j)
+            if (o + j < p.O) {
+                float yv = resid ? yres[j] : fmaf((float)acc[j], __ldg(p.scale + o + j), __ldg(p.shift + o + j));
                 if (OUTB > 0) yv = fminf(fmaxf(yv, -1.0f), 1.0f);
                 p.y_out[((long long)b * p.O + o + j) * HoWo + (long long)y * p.Wo + x] = yv;
             }
@@ -571,11 +584,15 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const Params p, cons
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             if (valid && o + j < p.O) {
-                const float *th = thr + (o + j) * NL;
-                const float v = (float)acc[j] * __ldg(th + NL - 1);
                 int k = 0;
+                if (resid) {
+                    k = level_index_of_y(yres[j], p.qo);
+                } else {
+                    const float *th = thr + (o + j) * NL;
+                    const float v = (float)acc[j] * __ldg(th + NL - 1);
 #pragma unroll
-                for (int u = 0; u < NL - 1; ++u) k += (v >= __ldg(th + u)) ? 1 : 0;
+                    for (int u = 0; u < NL - 1; ++u) k += (v >= __ldg(th + u)) ? 1 : 0;
+                }
                 code |= code_k<OUTB>(k) << (8 * j);
                 const uint32_t pb = planes_k<OUTB>(k);
 #pragma unroll
@@ -794,10 +811,16 @@ bool conv_tc_supported(const ConvArgs &a) {
     return true;
 }
 
+static bool conv_tc_residual(const ConvArgs &a) {
+    return a.res_codes != nullptr || a.res_f32 != nullptr || a.y_nhwc != nullptr;
+}
+
 int conv_tc_launches(const ConvArgs &a) {
     if (a.workspace == nullptr || a.pool) return 1;
     tc::Plan pl;
-    return (tc::make_plan(a, pl) == MINW_OK && pl.p.ksplit > 1) ? 2 : 1;
+    if (tc::make_plan(a, pl) != MINW_OK || pl.p.ksplit < 2) return 1;
+    // main pass + reduction, plus the breakpoints when the reduction needs them
+    return (a.quant_out && a.thr == nullptr && !conv_tc_residual(a)) ? 3 : 2;
 }
 
 minw_status launch_thresholds(const float *scale, const float *shift, int O, const QParams &q, float *out,
@@ -825,7 +848,7 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
         configured[kout] = pl.smem;
     }
     const float *thr = a.thr;
-    if (split && a.quant_out && thr == nullptr) {
+    if (split && a.quant_out && thr == nullptr && !conv_tc_residual(a)) {
         tc::thresholds_kernel<<<(a.O + 127) / 128, 128, 0, s>>>(a.scale, a.shift, a.O, a.qo, pl.thr_ws);
         thr = pl.thr_ws;
     }

@@ -14,45 +14,14 @@
 
 #include <vector>
 
-#include "kernels.cuh"
+#include "net.cuh"
 
 using namespace minw;
 using namespace minw_host;
 
-struct LayerPlan {
-    minw_layer_desc d;        // shape fields only; pointers are not kept
-    int C, H, W, O, kh, kw, stride, pad, pool;
-    int Ho, Wo, Hp, Wp;
-    uint32_t *wplanes = nullptr;   // packed weights (popcount layers)
-    uint8_t *wcodes = nullptr;     // weight codes (tensor-core layers)
-    float *thr = nullptr;          // output-quantizer breakpoints (first layer: fp32 [O][8];
-                                   // tensor-core layers: integer-valued [O][levels])
-    int in_codes = 0;              // input arrives in the codes layout
-    float *wlatent = nullptr;      // fp32 weights (first layer)
-    float *wscale = nullptr;       // per-channel weight prescale (first layer)
-    float *scale = nullptr;
-    float *shift = nullptr;
-    minw_quant qw{}, qo{};
-    int variant = MINW_VARIANT_POPC;
-};
-
-struct minw_net {
-    std::vector<LayerPlan> L;
-    int max_batch = 0;
-    uint32_t *buf[2] = {nullptr, nullptr};
-    size_t buf_words = 0;
-    std::vector<void *> owned;
-    float *x_stage = nullptr;         // device staging of minw_forward_host
-    float *logits_stage = nullptr;
-    size_t x_elems = 0, logit_elems = 0;
-    void *ws = nullptr;               // split-K workspace shared by the layers (zero between layers)
-    size_t ws_bytes = 0;
-    std::vector<cudaEvent_t> events;  // [0] before the first layer, [l+1] after layer l
-    bool timing = false;
-};
-
 static void net_free(minw_net *n) {
     if (!n) return;
+    if (n->res) resnet_free(n);
     for (void *p : n->owned) cudaFree(p);
     for (cudaEvent_t e : n->events) cudaEventDestroy(e);
     delete n;
@@ -220,6 +189,7 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
 
 minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits, void *stream) {
     if (!net || !x || !logits || B <= 0 || B > net->max_batch) return MINW_EINVAL;
+    if (net->kind == 1) return resnet_forward(net, x, B, logits, (cudaStream_t)stream);
     const int nl = (int)net->L.size();
     int cur = 0;
     cudaStream_t cs = (cudaStream_t)stream;
@@ -282,9 +252,8 @@ minw_status minw_forward_host(minw_net *net, const float *x_host, int32_t B, flo
                               void *stream) {
     if (!net || !x_host || !logits_host || B <= 0 || B > net->max_batch) return MINW_EINVAL;
     cudaStream_t s = (cudaStream_t)stream;
-    const LayerPlan &F = net->L.front(), &PL = net->L.back();
-    const size_t xin = (size_t)B * F.C * F.H * F.W;
-    const size_t lout = (size_t)B * PL.O * PL.Hp * PL.Wp;
+    const size_t xin = net->x_elems / net->max_batch * B;
+    const size_t lout = net->logit_elems / net->max_batch * B;
     if (cudaMemcpyAsync(net->x_stage, x_host, xin * sizeof(float), cudaMemcpyHostToDevice, s) != cudaSuccess)
         return MINW_ECUDA;
     minw_status st = minw_forward(net, net->x_stage, B, net->logits_stage, stream);
@@ -298,7 +267,7 @@ minw_status minw_forward_host(minw_net *net, const float *x_host, int32_t B, flo
 minw_status minw_net_enable_timing(minw_net *net, int32_t on) {
     if (!net) return MINW_EINVAL;
     if (on && net->events.empty()) {
-        net->events.resize(net->L.size() + 1);
+        net->events.resize((size_t)minw_net_launches(net) + 1);
         for (auto &e : net->events)
             if (cudaEventCreate(&e) != cudaSuccess) return MINW_ECUDA;
     }
@@ -309,22 +278,32 @@ minw_status minw_net_enable_timing(minw_net *net, int32_t on) {
 minw_status minw_net_layer_times(minw_net *net, float *ms) {
     if (!net || !ms || net->events.empty()) return MINW_EINVAL;
     if (cudaEventSynchronize(net->events.back()) != cudaSuccess) return MINW_ECUDA;
-    for (size_t l = 0; l < net->L.size(); ++l)
+    for (size_t l = 0; l + 1 < net->events.size(); ++l)
         if (cudaEventElapsedTime(&ms[l], net->events[l], net->events[l + 1]) != cudaSuccess) return MINW_ECUDA;
     return MINW_OK;
 }
 
 minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants) {
     if (!net || !variants) return MINW_EINVAL;
+    if (net->kind == 1) {
+        // stem, pool, the block convolutions (tensor cores), head
+        const int n = minw_net_launches(net);
+        for (int l = 0; l < n; ++l) variants[l] = (l >= 2 && l < n - 1) ? MINW_VARIANT_TC : 0;
+        return MINW_OK;
+    }
     for (size_t l = 0; l < net->L.size(); ++l) variants[l] = l == 0 ? 0 : net->L[l].variant;
     return MINW_OK;
 }
 
-int32_t minw_net_launches(const minw_net *net) { return net ? (int32_t)net->L.size() : 0; }
+int32_t minw_net_launches(const minw_net *net) {
+    if (!net) return 0;
+    return net->kind == 1 ? resnet_ops(net) : (int32_t)net->L.size();
+}
 
 // Kernels one minw_forward issues (a split-K layer issues two).
 int32_t minw_net_kernels(const minw_net *net) {
     if (!net) return 0;
+    if (net->kind == 1) return resnet_kernels(net);
     int32_t k = 0;
     for (size_t l = 0; l < net->L.size(); ++l) {
         const LayerPlan &P = net->L[l];

@@ -42,18 +42,42 @@ def weight_prescale(w, bits_w):
     return f32(1.0 / m)
 
 
-def bn_affine(r, O, fan_in, bits_in, bits_w, w_prescale, units_shift):
+# Expected maximum of k independent standard normals (k = 4: a 2x2 pool,
+# k = 9: a 3x3 pool): the running mean a BN after a max pool would learn, in
+# units of the pre-pool standard deviation.
+POOL_MEAN = {1: 0.0, 4: 1.0294, 9: 1.4850}
+
+
+def weight_ms(w, w_prescale, bits_w):
+    """Per-output-channel second moment of the prescaled latent weights, a
+    stand-in for the second moment of their levels (1 for sign weights)."""
+    O = w.shape[0]
+    if bits_w == 1:
+        return np.ones(O)
+    v = w.reshape(O, -1).astype(np.float64) * w_prescale.astype(np.float64)[:, None]
+    return np.maximum((v * v).mean(axis=1), 1e-6)
+
+
+def bn_affine(r, O, fan_in, bits_in, bits_w, w_prescale, units_shift, w_ms=None, pool_k=1):
     """Synthetic inference-mode batch normalisation folded to a per-channel
     affine map on the layer's raw output: gamma ~ N(1, 0.1), beta ~ N(0, 0.1),
-    running mean 0, running variance ~ fan_in times the level second moments.
-    The returned scale also carries the accumulator unit 2^-units_shift and the
-    weight prescale, so that y = scale * acc + shift."""
+    running variance ~ fan_in times the input and weight second moments
+    (``w_ms`` per channel, else the level second moment of ``bits_w``),
+    running mean 0, or the expected window maximum when a k-element max pool
+    precedes the BN.  The returned scale also carries the accumulator unit
+    2^-units_shift, so that y = scale * acc + shift.  Without ``w_ms`` the
+    statistics are those of the latent-weight output (the scale also undoes
+    the weight prescale); with it, those of the level output itself."""
     gamma = r.normal(1.0, 0.1, O)
     beta = r.normal(0.0, 0.1, O)
-    var = fan_in * _LEVEL_MS[bits_in] * _LEVEL_MS[bits_w]
-    s = gamma / np.sqrt(var + 1e-5)
-    s = s * (2.0 ** -units_shift) / w_prescale.astype(np.float64)
-    return f32(s), f32(beta)
+    wm = _LEVEL_MS[bits_w] if w_ms is None else w_ms
+    var = fan_in * _LEVEL_MS[bits_in] * wm
+    inv = gamma / np.sqrt(var + 1e-5)
+    shift = beta - inv * POOL_MEAN[pool_k] * np.sqrt(var)
+    s = inv * (2.0 ** -units_shift)
+    if w_ms is None:
+        s = s / w_prescale.astype(np.float64)
+    return f32(s), f32(shift)
 
 
 def _units(bits):
@@ -111,7 +135,8 @@ def convnet_params(seed, bits_a=1, bits_w=1, widths=(128, 128, 256, 256, 512, 51
         w = f32(r.normal(0.0, w_sigma, (c_out, c_in, 3, 3)))
         ws = weight_prescale(w, bits_w)
         u = (0 if bits_in == 0 else _units(bits_in)) + _units(bits_w)
-        scale, shift = bn_affine(r, c_out, c_in * 9, bits_in, bits_w, ws, u)
+        scale, shift = bn_affine(r, c_out, c_in * 9, bits_in, bits_w, ws, u,
+                                 w_ms=weight_ms(w, ws, bits_w), pool_k=4 if pool else 1)
         layers.append(dict(kind="conv", w=w, w_scale=ws, scale=scale, shift=shift,
                            pool=pool, bits_in=bits_in, bits_w=bits_w,
                            bits_out=bits_a, C=c_in, O=c_out, H=size, W=size,
@@ -124,7 +149,8 @@ def convnet_params(seed, bits_a=1, bits_w=1, widths=(128, 128, 256, 256, 512, 51
     for j, o in enumerate(dims):
         w = f32(r.normal(0.0, w_sigma, (o, k)))
         ws = weight_prescale(w, bits_w)
-        scale, shift = bn_affine(r, o, k, bits_a, bits_w, ws, _units(bits_a) + _units(bits_w))
+        scale, shift = bn_affine(r, o, k, bits_a, bits_w, ws, _units(bits_a) + _units(bits_w),
+                                 w_ms=weight_ms(w, ws, bits_w))
         last = j == len(dims) - 1
         rec = dict(kind="fc", w=w, w_scale=ws, scale=scale, shift=shift, pool=False,
                    bits_in=bits_a, bits_w=bits_w, bits_out=0 if last else bits_a,
@@ -141,3 +167,46 @@ def convnet_params(seed, bits_a=1, bits_w=1, widths=(128, 128, 256, 256, 512, 51
 def convnet_input(seed, B, in_ch=3, hw=32):
     """CIFAR-shaped synthetic images, U(-1, 1)."""
     return f32(rng(seed).uniform(-1.0, 1.0, (B, in_ch, hw, hw)))
+
+
+def resnet18_params(seed, bits_a=3, bits_w=3, classes=1000, hw=224, w_sigma=0.02):
+    """ResNet-18-shaped MINW-Net (Table V's network): fp32 7x7/2 stem (fp32
+    weights), eight basic blocks (widths 64-128-256-512, stride 2 and a 1x1
+    shortcut entering stages 2-4) with quantized weights, fp32 classifier.
+    Latent weights ~ N(0, w_sigma); BN maps as ``bn_affine``."""
+    r = rng(seed)
+    out = dict(bits_a=bits_a, bits_w=bits_w, thr_a=DEFAULT_THR[bits_a], thr_w=DEFAULT_THR[bits_w],
+               classes=classes, hw=hw)
+    sw = f32(r.normal(0.0, w_sigma, (64, 3, 7, 7)))
+    g, b_ = r.normal(1.0, 0.1, 64), r.normal(0.0, 0.1, 64)
+    var = 147 * 1.0 * w_sigma ** 2                 # image ~ N(0, 1), fp32 weights
+    inv = g / np.sqrt(var + 1e-5)                  # BN follows the 3x3 max pool
+    out["stem"] = dict(w=sw, scale=f32(inv), shift=f32(b_ - inv * POOL_MEAN[9] * np.sqrt(var)))
+    u = _units(bits_a) + _units(bits_w)
+
+    def qconv(o, c, k):
+        w = f32(r.normal(0.0, w_sigma, (o, c, k, k)))
+        ws = weight_prescale(w, bits_w)
+        scale, shift = bn_affine(r, o, c * k * k, bits_a, bits_w, ws, u, w_ms=weight_ms(w, ws, bits_w))
+        return dict(w=w, w_scale=ws, scale=scale, shift=shift, k=k)
+
+    blocks = []
+    c_in = 64
+    for stage, width in enumerate((64, 128, 256, 512)):
+        for j in range(2):
+            stride = 2 if (stage > 0 and j == 0) else 1
+            blk = dict(stride=stride, c1=qconv(width, c_in, 3), c2=qconv(width, width, 3),
+                       down=qconv(width, c_in, 1) if stride == 2 else None)
+            blocks.append(blk)
+            c_in = width
+    out["blocks"] = blocks
+    fw = f32(r.normal(0.0, w_sigma, (classes, 512)))
+    g, b_ = r.normal(1.0, 0.1, classes), r.normal(0.0, 0.1, classes)
+    var = 512 * _LEVEL_MS[bits_a] * w_sigma ** 2
+    out["fc"] = dict(w=fw, scale=f32(g / np.sqrt(var + 1e-5)), shift=f32(b_))
+    return out
+
+
+def resnet18_input(seed, B, hw=224):
+    """ImageNet-shaped synthetic images, N(0, 1)."""
+    return f32(rng(seed).standard_normal((B, 3, hw, hw)))

@@ -45,6 +45,17 @@ class LayerDesc(ctypes.Structure):
                 ("scale", ctypes.c_void_p), ("shift", ctypes.c_void_p)]
 
 
+class ResNet18Desc(ctypes.Structure):
+    _fields_ = [("bits_a", ctypes.c_int32), ("bits_w", ctypes.c_int32), ("thr_a", ctypes.c_float * 3),
+                ("thr_w", ctypes.c_float * 3), ("image_hw", ctypes.c_int32), ("num_classes", ctypes.c_int32),
+                ("stem_w", ctypes.c_void_p), ("stem_scale", ctypes.c_void_p), ("stem_shift", ctypes.c_void_p),
+                ("conv_w", ctypes.c_void_p * 16), ("conv_wscale", ctypes.c_void_p * 16),
+                ("conv_scale", ctypes.c_void_p * 16), ("conv_shift", ctypes.c_void_p * 16),
+                ("down_w", ctypes.c_void_p * 3), ("down_wscale", ctypes.c_void_p * 3),
+                ("down_scale", ctypes.c_void_p * 3), ("down_shift", ctypes.c_void_p * 3),
+                ("fc_w", ctypes.c_void_p), ("fc_scale", ctypes.c_void_p), ("fc_shift", ctypes.c_void_p)]
+
+
 # name -> (restype, argtypes)
 _P, _I32, _I64, _F = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float
 _QP = ctypes.POINTER(Quant)
@@ -78,6 +89,8 @@ SIGNATURES = {
                                              _P]),
     "minw_net_create": (ctypes.c_int, [ctypes.POINTER(LayerDesc), _I32, _I32, _I32, _P,
                                        ctypes.POINTER(ctypes.c_void_p)]),
+    "minw_resnet18_create": (ctypes.c_int, [ctypes.POINTER(ResNet18Desc), _I32, _P,
+                                            ctypes.POINTER(ctypes.c_void_p)]),
     "minw_forward": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
     "minw_forward_host": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
     "minw_net_enable_timing": (ctypes.c_int, [_P, _I32]),
@@ -292,6 +305,46 @@ class Net:
 
     ``layers`` is a list of dicts with the minw_layer_desc fields; ``w``,
     ``w_scale``, ``scale`` and ``shift`` are device tensors."""
+
+    @classmethod
+    def resnet18(cls, params, max_batch, device, stream=None):
+        """minw_resnet18_create from a parameter dict shaped like
+        ``inputs.resnet18_params`` (latent fp32 weights, BN maps); the tensors
+        are copied to ``device`` for the call and released after it."""
+        d = ResNet18Desc()
+        d.bits_a, d.bits_w = params["bits_a"], params["bits_w"]
+        for i in range(3):
+            d.thr_a[i] = float(params["thr_a"][i])
+            d.thr_w[i] = float(params["thr_w"][i])
+        d.image_hw, d.num_classes = params["hw"], params["classes"]
+        keep = []
+
+        def dev(a):
+            t = torch.from_numpy(a).to(device).contiguous()
+            keep.append(t)
+            return t.data_ptr()
+        st = params["stem"]
+        d.stem_w, d.stem_scale, d.stem_shift = dev(st["w"]), dev(st["scale"]), dev(st["shift"])
+        nd = 0
+        for b, blk in enumerate(params["blocks"]):
+            for j, c in enumerate((blk["c1"], blk["c2"])):
+                d.conv_w[2 * b + j], d.conv_wscale[2 * b + j] = dev(c["w"]), dev(c["w_scale"])
+                d.conv_scale[2 * b + j], d.conv_shift[2 * b + j] = dev(c["scale"]), dev(c["shift"])
+            if blk["down"] is not None:
+                c = blk["down"]
+                d.down_w[nd], d.down_wscale[nd] = dev(c["w"]), dev(c["w_scale"])
+                d.down_scale[nd], d.down_shift[nd] = dev(c["scale"]), dev(c["shift"])
+                nd += 1
+        fc = params["fc"]
+        d.fc_w, d.fc_scale, d.fc_shift = dev(fc["w"]), dev(fc["scale"]), dev(fc["shift"])
+        h = ctypes.c_void_p()
+        _check(lib().minw_resnet18_create(ctypes.byref(d), int(max_batch), _stream(stream), ctypes.byref(h)),
+               "minw_resnet18_create")
+        net = cls.__new__(cls)
+        net._h = h
+        net.max_batch = max_batch
+        net.out_features = params["classes"]
+        return net
 
     def __init__(self, layers, max_batch, variant=VARIANT_AUTO, stream=None):
         arr = (LayerDesc * len(layers))()
