@@ -32,6 +32,9 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+#include <stdlib.h>
+
+#include <mutex>
 
 #include "kernels.cuh"
 
@@ -58,6 +61,8 @@ struct Params {
     const float *thr;          // precomputed breakpoints [O][nlev] (nullable)
     int nlev;                  // levels of the output quantizer
     int ksplit;                // K slices per output tile (1: no split)
+    int cl;                    // CTAs per cluster sharing each weight box (1, 2 or 4; 1 when split)
+    int tiles_mp;              // pixel tiles per channel tile, padded to a multiple of cl
     int32_t *part;             // split-K: int32 partial sums [ksplit][tiles][128][BN]
     // residual blocks: y = BN(acc) + shortcut, then HardTanh + quantize
     const uint8_t *res_codes;  // shortcut as level codes [B][Hp][Wp][O] (nullable)
@@ -89,7 +94,7 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
 __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, 100000;\n selp.u32 %0, 1, 0, p;\n}\n"
         : "=r"(ok)
         : "r"(smem_u32(bar)), "r"(parity)
         : "memory");
@@ -97,7 +102,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
 }
 
 // Bounded wait for the phase with the given parity; false (and the device
-// error flag set) when it does not complete within WAIT_CYCLES.
+// error flag set) when it does not complete within WAIT_CYCLES.  Each
+// try_wait may suspend the thread up to 100 us (the hint) until the phase
+// completes, so waiting warps do not take issue slots from the MMA thread.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
@@ -117,6 +124,27 @@ __device__ __forceinline__ void tma_load_4d(void *dst, const CUtensorMap *map, u
         " [%0], [%1, {%2, %3, %4, %5}], [%6];\n" ::"r"(smem_u32(dst)),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_u32(bar))
         : "memory");
+}
+
+// The same box delivered to every CTA of the cluster named in mask, at the
+// same shared-memory offset, completing bytes on each CTA's barrier there.
+__device__ __forceinline__ void tma_load_2d_mc(void *dst, const CUtensorMap *map, uint64_t *bar, int c0, int c1,
+                                               uint16_t mask) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
+        " [%0], [%1, {%2, %3}], [%4], %5;\n" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar)), "h"(mask)
+        : "memory");
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release;\nbarrier.cluster.wait.acquire;\n" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;\n" : "=r"(r));
+    return r;
 }
 
 __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, uint64_t *bar, int c0, int c1) {
@@ -158,6 +186,16 @@ __device__ __forceinline__ void mma_commit(uint64_t *bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(
                      smem_u32(bar))
                  : "memory");
+}
+
+// Arrive on the barrier at this offset in every CTA of mask once the MMAs
+// issued so far have completed.
+__device__ __forceinline__ void mma_commit_mc(uint64_t *bar, uint16_t mask) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n" ::"r"(
+            smem_u32(bar)),
+        "h"(mask)
+        : "memory");
 }
 
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
@@ -203,6 +241,98 @@ __device__ __forceinline__ uint32_t planes_k(int k) {
     else return (uint32_t)((06420357ull >> (3 * k)) & 7ull);
 }
 
+// Four channels' bits (nibble g of m) spread to the low bit of four bytes.
+__device__ __forceinline__ uint32_t spread4(uint32_t m, int g) {
+    return (((m >> (4 * g)) & 0xFu) * 0x00204081u) & 0x01010101u;
+}
+
+// Epilogue of one 32-column chunk (16 when tail16 is false) of exact
+// accumulators, one tile row per lane, when the only output is the next
+// layer's levels.  For each breakpoint u the chunk becomes one 32-bit mask
+// M_u (bit j set when channel j's sigma * acc stays below T_u, taken from the
+// sign of fmaf(acc, sigma, -T_u): exact, as acc and T_u are integers, and
+// never -0, as -T_u = 0 is held as +0), so the
+// level index is k = #{u : bit clear}.  A 2x2 max pool of the accumulators
+// maps to the masks: for sigma = +1 the pooled level is the window's largest
+// (M pooled = AND over the window), for sigma = -1 its smallest (OR).  Bit
+// planes and E4M3 codes follow from the masks with bitwise logic.
+template <int OUTB>
+__device__ __forceinline__ void mask_chunk(uint32_t taddr, bool full32, const float *th, uint32_t sig, int pool,
+                                           int bw, bool writer, int nvalid, uint32_t *planes, int NWo,
+                                           uint8_t *codes) {
+    constexpr int NL = OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7);
+    uint32_t v[32];
+    if (full32) {
+        tmem_ld32(taddr, v);
+    } else {
+        uint32_t v16[16];
+        tmem_ld16(taddr, v16);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            v[j] = v16[j];
+            v[j + 16] = 0u;
+        }
+    }
+    uint32_t M[NL - 1];
+#pragma unroll
+    for (int u = 0; u < NL - 1; ++u) M[u] = 0u;
+#pragma unroll
+    for (int j = 31; j >= 0; --j) {
+        const float a = __uint_as_float(v[j]);
+        const float sg = th[j * NL + NL - 1];
+#pragma unroll
+        for (int u = 0; u < NL - 1; ++u)
+            M[u] = __funnelshift_l(__float_as_uint(fmaf(a, sg, th[j * NL + u])), M[u], 1);
+    }
+    if (pool) {
+#pragma unroll
+        for (int u = 0; u < NL - 1; ++u) {
+            const uint32_t m = M[u];
+            const uint32_t n1 = __shfl_xor_sync(0xffffffffu, m, 1);
+            const uint32_t a1 = m & n1, o1 = m | n1;
+            const uint32_t a2 = a1 & __shfl_xor_sync(0xffffffffu, a1, bw);
+            const uint32_t o2 = o1 | __shfl_xor_sync(0xffffffffu, o1, bw);
+            M[u] = (sig & a2) | (~sig & o2);
+        }
+    }
+    if (!writer) return;
+    // planes: sign, then the non-zero mask (2 bits) or the magnitude code (3 bits)
+    uint32_t P[3];
+    if constexpr (OUTB == 1) {
+        P[0] = M[0];
+    } else if constexpr (OUTB == 2) {
+        P[0] = M[0];
+        P[1] = M[0] | ~M[1];
+    } else {
+        P[0] = M[2];
+        P[1] = M[0] | (M[2] & ~M[1]) | (M[4] & ~M[3]) | ~M[5];     // |k - 3| in {1, 3}
+        P[2] = M[1] | ~M[4];                                        // |k - 3| in {2, 3}
+    }
+    if (planes != nullptr) {
+        const uint32_t vm = nvalid >= 32 ? 0xffffffffu : ((1u << nvalid) - 1u);
+#pragma unroll
+        for (int u = 0; u < OUTB; ++u) planes[u * NWo] = P[u] & vm;
+    }
+    if (codes != nullptr) {
+        uint32_t cw[8];
+#pragma unroll
+        for (int g = 0; g < 8; ++g) {
+            if constexpr (OUTB == 1) {
+                cw[g] = (spread4(P[0], g) * 0x80u) | 0x38383838u;
+            } else if constexpr (OUTB == 2) {
+                cw[g] = spread4(P[1], g) * 0x38u + spread4(P[0], g) * 0x80u;
+            } else {
+                const uint32_t c0 = P[1], c1 = P[2];
+                cw[g] = spread4(c0, g) * 0x08u + spread4(c0 & ~c1, g) * 0x30u + spread4(c1, g) * 0x40u +
+                        spread4(P[0] & (c0 | c1), g) * 0x80u;
+            }
+        }
+        uint4 *dst = reinterpret_cast<uint4 *>(codes);
+        dst[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
+        if (nvalid > 16 && full32) dst[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
+    }
+}
+
 // OUTB: bits of the quantized output (0 when the launch writes none).
 template <int OUTB>
 __global__ void __launch_bounds__(NT, 1)
@@ -213,23 +343,33 @@ __global__ void __launch_bounds__(NT, 1)
     // pointer arithmetic on the shared array keeps the shared address space
     uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     constexpr int NL = OUTB == 0 ? 1 : (OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7));
-    float *sthr = reinterpret_cast<float *>(smem + (size_t)p.S * p.stage_bytes);   // [O][NL]
-    const int thr_floats = OUTB ? p.O * NL : 0;
-    uint64_t *full = reinterpret_cast<uint64_t *>(sthr + ((thr_floats + 1) & ~1));
+    // breakpoints [O32][NL] (channels padded to a multiple of 32), then the
+    // per-32-channel masks of channels with sigma = +1
+    const int O32 = (p.O + 31) & ~31;
+    float *sthr = reinterpret_cast<float *>(smem + (size_t)p.S * p.stage_bytes);
+    const int thr_floats = OUTB ? O32 * NL : 0;
+    uint32_t *ssig = reinterpret_cast<uint32_t *>(sthr + thr_floats);              // [O32 / 32]
+    const int sig_words = OUTB ? O32 / 32 : 0;
+    uint64_t *full = reinterpret_cast<uint64_t *>(ssig + ((sig_words + 1) & ~1));
     uint64_t *empty = full + p.S;
     uint64_t *tfull = empty + p.S;            // [2] accumulator ready
     uint64_t *tempty = tfull + 2;             // [2] accumulator drained
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(tempty + 2);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int tiles_m = p.nbx * p.nby * p.nbb;
+    // pixel tiles padded to a multiple of the cluster size: the CTAs of a
+    // cluster walk tiles of the same channel tile in lock step (a padded tile
+    // reads zero boxes and writes nothing)
+    const int tiles_m = p.tiles_mp;
     const int tiles = tiles_m * p.ntn;
     const int items = tiles * p.ksplit;       // (output tile, K slice) work items
+    const uint16_t cmask = (uint16_t)((1u << p.cl) - 1u);
+    const int crank = p.cl > 1 ? (int)cluster_ctarank() : 0;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < p.S; ++s) {
             mbar_init(&full[s], 2);               // one arrival per TMA issuing warp
-            mbar_init(&empty[s], 1);
+            mbar_init(&empty[s], p.cl);           // one release per CTA reading the weight box
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
@@ -244,15 +384,38 @@ __global__ void __launch_bounds__(NT, 1)
     }
     // output-quantizer breakpoints of every channel, in shared memory
     if constexpr (OUTB > 0) {
+        // held as (-T_1 .. -T_{n-1}, sigma) with -0 stored as +0, so that
+        // fmaf(acc, sigma, -T) is never -0 and its sign bit is [sigma * acc < T]
         if (p.thr != nullptr) {
-            for (int i = threadIdx.x; i < thr_floats; i += NT) sthr[i] = __ldg(p.thr + i);
+            for (int i = threadIdx.x; i < p.O * NL; i += NT) {
+                const float x = __ldg(p.thr + i);
+                sthr[i] = (i % NL == NL - 1) ? x : (x == 0.0f ? 0.0f : -x);
+            }
         } else {
-            for (int o = threadIdx.x; o < p.O; o += NT)
-                channel_thresholds(__ldg(p.scale + o), __ldg(p.shift + o), p.qo, sthr + o * NL);
+            for (int o = threadIdx.x; o < p.O; o += NT) {
+                float *t = sthr + o * NL;
+                channel_thresholds(__ldg(p.scale + o), __ldg(p.shift + o), p.qo, t);
+                for (int u = 0; u < NL - 1; ++u) t[u] = t[u] == 0.0f ? 0.0f : -t[u];
+            }
+        }
+        for (int i = p.O * NL + threadIdx.x; i < thr_floats; i += NT)        // padding channels
+            sthr[i] = ((i % NL) == NL - 1) ? 1.0f : 0.0f;
+        // sigma of a channel: the sign of its BN scale (+1 for 0)
+        for (int g = threadIdx.x; g < sig_words; g += NT) {
+            uint32_t m = 0u;
+            for (int j = 0; j < 32; ++j) {
+                const int o = g * 32 + j;
+                const float sg = o < p.O ? (p.thr != nullptr ? __ldg(p.thr + o * NL + NL - 1)
+                                                             : (__ldg(p.scale + o) < 0.0f ? -1.0f : 1.0f))
+                                         : 1.0f;
+                m |= (sg > 0.0f ? 1u : 0u) << j;
+            }
+            ssig[g] = m;
         }
     }
     fence_before();
     __syncthreads();
+    if (p.cl > 1) cluster_sync_all();         // every barrier of the cluster is initialised
     fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
@@ -262,7 +425,8 @@ __global__ void __launch_bounds__(NT, 1)
             const bool act = warp == 0;
             const CUtensorMap *map = act ? &tmA : &tmB;
             asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
-            const uint32_t bytes = act ? p.a_bytes : p.stage_bytes - p.a_bytes;
+            const uint32_t bytes = act ? p.a_bytes : p.stage_bytes - p.a_bytes;   // weights: all cl slices
+            const int bslice = p.BN / p.cl;        // weight rows this CTA loads (and multicasts)
             int g = 0, s = 0, lap = 0;             // stages issued, ring slot, ring lap
             bool alive = true;
             for (int w = blockIdx.x; w < items && alive; w += gridDim.x) {
@@ -283,8 +447,11 @@ __global__ void __launch_bounds__(NT, 1)
                     mbar_expect_tx(&full[s], bytes);
                     if (act)
                         tma_load_4d(sa, &tmA, &full[s], c0, x0 + kx, y0 + ky, b0);
-                    else
+                    else if (p.cl == 1)
                         tma_load_2d(sa + p.a_bytes, &tmB, &full[s], kcol, o0);
+                    else
+                        tma_load_2d_mc(sa + p.a_bytes + (size_t)crank * bslice * p.ck, &tmB, &full[s], kcol,
+                                       o0 + crank * bslice, cmask);
                     kcol += p.ck;
                     c0 += p.ck;
                     if (c0 == p.C) {
@@ -297,6 +464,11 @@ __global__ void __launch_bounds__(NT, 1)
             // drain: every issued load has landed before the CTA can exit
             for (int j = g > p.S ? g - p.S : 0; j < g; ++j)
                 if (!mbar_wait(&full[j % p.S], (j / p.S) & 1)) break;
+            // clusters: every CTA's release of every slot has arrived here too
+            // (no remote arrival may reach this shared memory after exit)
+            if (p.cl > 1 && !act)
+                for (int j = g > p.S ? g - p.S : 0; j < g; ++j)
+                    if (!mbar_wait(&empty[j % p.S], (j / p.S) & 1)) break;
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -304,7 +476,15 @@ __global__ void __launch_bounds__(NT, 1)
             int s = 0, i = 0;
             uint32_t fphase = 0;
             bool alive = true;
+            // One thread issues every MMA, and each tcgen05.mma costs it on the
+            // order of a hundred cycles to issue: the loop keeps its own work per
+            // stage minimal (descriptors advance by a constant per ring slot,
+            // the K = 32 steps are unrolled).
             const uint32_t sbase = smem_u32(smem);
+            const uint64_t adesc0 = sw_desc(sbase, p.ck), bdesc0 = sw_desc(sbase + p.a_bytes, p.ck);
+            const uint32_t dstep = p.stage_bytes >> 4;     // start-address step of one ring slot
+            const bool k128 = p.ck == 128;                 // four K = 32 steps per stage, else two
+            const uint32_t idesc = p.idesc;
             for (int w = blockIdx.x; w < items && alive; w += gridDim.x, ++i) {
                 const int ab = i & 1, use = i >> 1;
                 const int t = w / p.ksplit, kp = w - t * p.ksplit;
@@ -312,16 +492,23 @@ __global__ void __launch_bounds__(NT, 1)
                 if (use > 0 && !mbar_wait(&tempty[ab], (use - 1) & 1)) break;
                 fence_after();
                 const uint32_t tmem_d = tmem_base + (uint32_t)(ab * p.BN);
+                uint32_t acc = 0u;
                 for (int ks = kb; ks < ke; ++ks) {
                     if (!mbar_wait(&full[s], fphase)) { alive = false; break; }
                     fence_after();
-                    const uint32_t sa = sbase + (uint32_t)s * p.stage_bytes;
-                    const uint64_t adesc = sw_desc(sa, p.ck);
-                    const uint64_t bdesc = sw_desc(sa + p.a_bytes, p.ck);
-                    const int nmma = p.ck >> 5;                  // K = 32 bytes per MMA
-                    for (int kk = 0; kk < nmma; ++kk)
-                        mma_f8(tmem_d, adesc + 2 * kk, bdesc + 2 * kk, p.idesc, (ks != kb) || (kk != 0));
-                    mma_commit(&empty[s]);
+                    const uint64_t off = (uint64_t)((uint32_t)s * dstep);
+                    const uint64_t ad = adesc0 + off, bd = bdesc0 + off;
+                    mma_f8(tmem_d, ad, bd, idesc, acc);
+                    mma_f8(tmem_d, ad + 2, bd + 2, idesc, 1u);
+                    if (k128) {
+                        mma_f8(tmem_d, ad + 4, bd + 4, idesc, 1u);
+                        mma_f8(tmem_d, ad + 6, bd + 6, idesc, 1u);
+                    }
+                    acc = 1u;
+                    if (p.cl == 1)
+                        mma_commit(&empty[s]);
+                    else
+                        mma_commit_mc(&empty[s], cmask);     // the slot is free in every CTA's view
                     if (++s == p.S) { s = 0; fphase ^= 1; }
                 }
                 mma_commit(&tfull[ab]);
@@ -340,6 +527,12 @@ __global__ void __launch_bounds__(NT, 1)
         const int ngrp = p.BN / 16;
         const int gmid = min(ngrp, (((ngrp + 1) / 2) + 1) & ~1);
         const int gbeg = half_cols ? gmid : 0, gend = half_cols ? ngrp : gmid;
+        // mask epilogue (a layer whose only output is the next layer's levels):
+        // this warp's 32-column chunks
+        const bool resid = p.res_codes != nullptr || p.res_f32 != nullptr || p.y_nhwc != nullptr;
+        const bool masked = OUTB > 0 && p.ksplit == 1 && p.acc_out == nullptr && p.y_out == nullptr && !resid;
+        const int nch = (p.BN + 31) >> 5, cmid = (nch + 1) >> 1;
+        const int cbeg = half_cols ? cmid : 0, cend = half_cols ? nch : cmid;
         int i = 0;
         bool dead = false;           // a bounded wait ran out: skip work, keep the barrier sequence
         for (int w = blockIdx.x; w < items; w += gridDim.x, ++i) {
@@ -356,6 +549,27 @@ __global__ void __launch_bounds__(NT, 1)
             const int yp = p.pool ? y / 2 : y, xp = p.pool ? x / 2 : x;
             const long long opix = ((long long)b * Hp + yp) * Wp + xp;
             uint32_t pw[3] = {0u, 0u, 0u};
+
+            if constexpr (OUTB > 0) {
+                if (masked) {
+                    if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
+                    fence_after();
+                    for (int c = cbeg; c < cend && !dead; ++c) {
+                        const int ob = o0 + c * 32;
+                        if (ob >= p.O) break;                      // no channel of this tile left
+                        __syncwarp();
+                        mask_chunk<OUTB>(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * p.BN + c * 32),
+                                         c * 32 + 32 <= p.BN, sthr + ob * NL, p.pool ? ssig[ob >> 5] : 0u, p.pool,
+                                         p.bw, writer, p.O - ob,
+                                         p.planes_out ? p.planes_out + (opix * OUTB) * NWo + (ob >> 5) : nullptr,
+                                         NWo, p.codes_out ? p.codes_out + opix * p.O + ob : nullptr);
+                    }
+                    fence_before();
+                    __syncwarp();
+                    if (lane == 0 && !dead) mbar_arrive(&tempty[ab]);
+                    continue;
+                }
+            }
 
             // the fused block epilogue of one 16-column group of exact accumulators
             auto finish = [&](float (&a)[16], int ch) {
@@ -439,7 +653,7 @@ __global__ void __launch_bounds__(NT, 1)
                             const float vv = a[j] * th[NL - 1];
                             int k = 0;
 #pragma unroll
-                            for (int u = 0; u < NL - 1; ++u) k += (vv >= th[u]) ? 1 : 0;
+                            for (int u = 0; u < NL - 1; ++u) k += (vv + th[u] >= 0.0f) ? 1 : 0;   // th = -T
                             kq[j] = k;
                         }
                         if (p.codes_out != nullptr) {
@@ -515,6 +729,7 @@ __global__ void __launch_bounds__(NT, 1)
         fence_after();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(p.tmem_cols));
     }
+    if (p.cl > 1) cluster_sync_all();         // no CTA leaves while a peer may still address it
 }
 
 // Split-K second pass: sums the K slices of every accumulator and runs the
@@ -689,7 +904,20 @@ static int auto_ksplit(int tiles, int nk, int sms) {
 static size_t slice_bytes(int tiles, int BN) { return (size_t)tiles * 128 * BN * sizeof(int32_t); }
 static size_t thr_ws_bytes(int O, int nlev) { return (((size_t)O * nlev * sizeof(float)) + 255) & ~(size_t)255; }
 
-static minw_status make_plan(const ConvArgs &a, Plan &pl) {
+// CTAs per cluster sharing each weight box (MINW_TC_CLUSTER = 1, 2 or 4;
+// 1 by default: the kernel is bound by MMA issue, not by the L2 -> shared
+// memory feed, and clusters of 2 or 4 measured 1-2 % slower on GB300).
+static int cluster_pref() {
+    static int v = -1;
+    if (v < 0) {
+        const char *e = getenv("MINW_TC_CLUSTER");
+        const int x = e ? atoi(e) : 1;
+        v = (x == 1 || x == 2 || x == 4) ? x : 1;
+    }
+    return v;
+}
+
+static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_pref()) {
     Params &p = pl.p;
     p = Params{};
     if (!plan_shape(a, p)) return MINW_EUNSUPPORTED;
@@ -705,7 +933,8 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     p.nlev = a.quant_out ? num_levels(a.qo.bits) : 0;
     p.thr = a.thr;
     p.stage_bytes = p.a_bytes + (uint32_t)(p.BN * p.ck);
-    const size_t thr_bytes = a.quant_out ? ((size_t)a.O * p.nlev + 2) * sizeof(float) : 0;
+    const size_t o32 = ((size_t)a.O + 31) & ~(size_t)31;
+    const size_t thr_bytes = a.quant_out ? (o32 * p.nlev + o32 / 32 + 2) * sizeof(float) : 0;
     const size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes;
     int S = (int)(budget / p.stage_bytes);
     if (S > 8) S = 8;
@@ -720,31 +949,6 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     p.planes_out = a.planes_out; p.codes_out = a.codes_out;
     p.res_codes = a.res_codes; p.res_unit = a.res_unit; p.res_f32 = a.res_f32; p.y_nhwc = a.y_nhwc;
 
-    EncodeTiledFn enc = encode_fn();
-    if (enc == nullptr) return MINW_ECUDA;
-    const CUtensorMapSwizzle swz = p.ck == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
-    {
-        const cuuint64_t dims[4] = {(cuuint64_t)a.C, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.B};
-        const cuuint64_t strides[3] = {(cuuint64_t)a.C, (cuuint64_t)a.W * a.C, (cuuint64_t)a.H * a.W * a.C};
-        const cuuint32_t sd = (cuuint32_t)p.stride;
-        const cuuint32_t box[4] = {(cuuint32_t)p.ck, (cuuint32_t)p.bw * sd, (cuuint32_t)p.bh * sd, (cuuint32_t)p.bb};
-        const cuuint32_t es[4] = {1u, sd, sd, 1u};
-        if (enc(&pl.tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<uint8_t *>(a.act8), dims, strides, box, es,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-            return MINW_ECUDA;
-    }
-    {
-        const long long K = (long long)a.kh * a.kw * a.C;
-        const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)a.O};
-        const cuuint64_t strides[1] = {(cuuint64_t)K};
-        const cuuint32_t box[2] = {(cuuint32_t)p.ck, (cuuint32_t)p.BN};
-        const cuuint32_t es[2] = {1u, 1u};
-        if (enc(&pl.tmB, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(a.wgt8), dims, strides, box, es,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-            return MINW_ECUDA;
-    }
     const int tiles = p.nbx * p.nby * p.nbb * p.ntn;
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
     p.ksplit = 1;
@@ -768,13 +972,70 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
             p.part = reinterpret_cast<int32_t *>(w + tb);
         }
     }
-    const int items = tiles * p.ksplit;
-    pl.grid = dim3((unsigned)(items < sms ? items : sms));
+    // clusters sharing each weight box (multicast): cl CTAs walk pixel tiles
+    // of one channel tile together; each loads BN / cl weight rows for all
+    // (padding the pixel tiles to a multiple of cl may add at most 1/8)
+    const int tiles_m = p.nbx * p.nby * p.nbb;
+    p.cl = 1;
+    if (p.ksplit == 1) {
+        int cl = cl_max;
+        while (cl > 1 && (p.BN % (8 * cl) != 0 || ((tiles_m + cl - 1) / cl * cl - tiles_m) * 8 > tiles_m)) cl >>= 1;
+        p.cl = cl;
+    }
+    p.tiles_mp = (tiles_m + p.cl - 1) / p.cl * p.cl;
+    EncodeTiledFn enc = encode_fn();
+    if (enc == nullptr) return MINW_ECUDA;
+    const CUtensorMapSwizzle swz = p.ck == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+    {
+        const cuuint64_t dims[4] = {(cuuint64_t)a.C, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.B};
+        const cuuint64_t strides[3] = {(cuuint64_t)a.C, (cuuint64_t)a.W * a.C, (cuuint64_t)a.H * a.W * a.C};
+        const cuuint32_t sd = (cuuint32_t)p.stride;
+        const cuuint32_t box[4] = {(cuuint32_t)p.ck, (cuuint32_t)p.bw * sd, (cuuint32_t)p.bh * sd, (cuuint32_t)p.bb};
+        const cuuint32_t es[4] = {1u, sd, sd, 1u};
+        if (enc(&pl.tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<uint8_t *>(a.act8), dims, strides, box, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return MINW_ECUDA;
+    }
+    {
+        const long long K = (long long)a.kh * a.kw * a.C;
+        const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)a.O};
+        const cuuint64_t strides[1] = {(cuuint64_t)K};
+        const cuuint32_t box[2] = {(cuuint32_t)p.ck, (cuuint32_t)(p.BN / p.cl)};
+        const cuuint32_t es[2] = {1u, 1u};
+        if (enc(&pl.tmB, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(a.wgt8), dims, strides, box, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return MINW_ECUDA;
+    }
+    const int items = p.tiles_mp * p.ntn * p.ksplit;
+    int grid = items < sms ? items : sms;
+    grid -= grid % p.cl;
+    pl.grid = dim3((unsigned)grid);
     pl.smem = (size_t)p.S * p.stage_bytes + 1024 + 256 + thr_bytes;
     // more than half of an SM's shared memory: exactly one CTA (and one TMEM
     // allocation) per SM
     if (pl.smem < 120 * 1024) pl.smem = 120 * 1024;
     return MINW_OK;
+}
+
+// Resident clusters of cl CTAs for a launch of kern with smem bytes (cached:
+// the answer depends only on these three).
+static int max_active_clusters(const void *kern, int cl, size_t smem, const cudaLaunchConfig_t &cfg) {
+    struct Entry { const void *k; int cl; size_t smem; int n; };
+    static Entry cache[32];
+    static int used = 0;
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < used; ++i)
+        if (cache[i].k == kern && cache[i].cl == cl && cache[i].smem == smem) return cache[i].n;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        n = 0;
+    }
+    if (used < 32) cache[used++] = Entry{kern, cl, smem, n};
+    return n;
 }
 
 }  // namespace tc
@@ -858,7 +1119,27 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
         pm.acc_out = nullptr;
         pm.y_out = nullptr;
     }
-    kern<<<pl.grid, tc::NT, pl.smem, s>>>(pl.tmA, pl.tmB, pm);
+    if (pm.cl == 1) {
+        kern<<<pl.grid, tc::NT, pl.smem, s>>>(pl.tmA, pl.tmB, pm);
+    } else {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = pl.grid;
+        cfg.blockDim = dim3(tc::NT);
+        cfg.dynamicSmemBytes = pl.smem;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = (unsigned)pm.cl;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        // a persistent grid: no more clusters than can be resident at once
+        const int maxc = tc::max_active_clusters(reinterpret_cast<const void *>(kern), pm.cl, pl.smem, cfg);
+        if (maxc < 1) return MINW_EUNSUPPORTED;
+        if ((int)cfg.gridDim.x > maxc * pm.cl) cfg.gridDim.x = (unsigned)(maxc * pm.cl);
+        if (cudaLaunchKernelEx(&cfg, kern, pl.tmA, pl.tmB, pm) != cudaSuccess) return MINW_ECUDA;
+    }
     if (split) {
         const int tiles_m = pl.p.nbx * pl.p.nby * pl.p.nbb;
         const long long threads = (long long)tiles_m * 128 * ((a.O + 31) / 32) * 8;
