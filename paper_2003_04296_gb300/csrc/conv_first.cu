@@ -2,7 +2,8 @@
 // is not quantized, its weights are.  Each output is one fp32 fmaf chain over
 // (c, ky, kx) in that order with padded taps skipped, so the result does not
 // depend on the launch shape.  BN (fmaf), HardTanh and quantize + pack of the
-// next layer's input are fused into the epilogue.
+// next layer's input are fused into the epilogue.  The same kernel runs the
+// ResNet stem (7x7 / 2, fp32 weights).
 //
 // See conv_first_kernel for the tiling.
 #include <cuda_runtime.h>
@@ -13,192 +14,243 @@
 namespace minw {
 
 
-constexpr int FIRST_NT = 128;
-constexpr int FIRST_PPT = 4;                    // output pixels per thread
-constexpr int FIRST_MAXPIX = FIRST_PPT * FIRST_NT;
+constexpr int FIRST_NT = 256;                   // 8 warps
+constexpr int FIRST_PX = 2;                     // output pixels per thread (32 apart)
 
-template <int OUTB>
-__device__ __forceinline__ uint32_t first_code(int k) {
-    if constexpr (OUTB == 1) return k ? 0x38u : 0xB8u;
-    else if constexpr (OUTB == 2) return (uint32_t)((0x3800B8u >> (8 * k)) & 0xFFu);
-    else return (uint32_t)((0x0048403800B8C0C8ull >> (8 * k)) & 0xFFull);
+// Two fp32 lanes in one 64-bit register for the packed fma.rn.f32x2: each
+// lane is an IEEE fmaf of its own, so a chain of them is bit-identical to
+// the scalar chain.
+__device__ __forceinline__ unsigned long long dup2(float x) {
+    unsigned long long r;
+    asm("mov.b64 %0, {%1, %1};" : "=l"(r) : "f"(x));
+    return r;
 }
-template <int OUTB>
-__device__ __forceinline__ uint32_t first_planes(int k) {
-    if constexpr (OUTB == 1) return k ? 0u : 1u;
-    else if constexpr (OUTB == 2) return (0x203u >> (4 * k)) & 0x3u;
-    else return (uint32_t)((06420357ull >> (3 * k)) & 7ull);
+__device__ __forceinline__ void ffma2(unsigned long long &acc, unsigned long long a, unsigned long long b) {
+    asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(acc) : "l"(a), "l"(b));
+}
+__device__ __forceinline__ float lane2(unsigned long long v, int hi) {
+    float lo_, hi_;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo_), "=f"(hi_) : "l"(v));
+    return hi ? hi_ : lo_;
 }
 
 struct FirstTile {
-    int R;            // output rows per CTA
-    int Rin, Win;     // input patch rows / columns (zero padded)
+    int OCB;          // output channels per CTA (32 or 64)
+    int groups;       // 32-channel groups per CTA
+    int PB;           // output pixels per CTA (64 per pixel block, 8 / groups blocks)
+    int tiles;        // CTAs along the pixels of one image
+    int Rmax;         // input patch rows
+    int Ws;           // patch columns per stride phase
+    int RP;           // patch row pitch (stride x Ws)
+    int K;            // C x kh x kw
     size_t smem;      // bytes of dynamic shared memory
 };
 
 static FirstTile first_tile(const FirstArgs &a) {
     FirstTile t;
-    t.R = FIRST_MAXPIX / a.Wo;
-    if (t.R > a.Ho) t.R = a.Ho;
-    if (t.R < 1) t.R = 1;
-    t.Rin = (t.R - 1) * a.stride + a.kh;
-    t.Win = (a.Wo - 1) * a.stride + a.kw;
-    const int K = a.C * a.kh * a.kw;
-    t.smem = sizeof(float) * (32 * (size_t)K + (size_t)a.C * t.Rin * t.Win + 32 * 8) + sizeof(int) * K;
+    t.OCB = a.O > 32 ? 64 : 32;
+    t.groups = t.OCB / 32;
+    t.PB = 64 * (8 / t.groups);
+    const int npix = a.Ho * a.Wo;
+    t.tiles = (npix + t.PB - 1) / t.PB;
+    const int rows = min(a.Ho, (t.PB + a.Wo - 2) / a.Wo + 1);      // rows PB consecutive pixels can touch
+    t.Rmax = (rows - 1) * a.stride + a.kh;
+    const int Win = (a.Wo - 1) * a.stride + a.kw;
+    t.Ws = (Win + a.stride - 1) / a.stride;
+    t.RP = t.Ws * a.stride;
+    t.K = a.C * a.kh * a.kw;
+    t.smem = sizeof(float) * ((size_t)t.K * t.OCB + (size_t)t.OCB * 8 + (size_t)a.C * t.Rmax * t.RP);
     return t;
 }
 
-// A CTA owns R full output rows of one image (R * Wo <= 512 pixels) and one
-// group of 32 output channels.  Its zero-padded input patch, the group's
-// weights ([K][32]) and the tap offsets sit in shared memory; a thread holds
-// four output pixels x 32 channels and per tap does four patch loads, eight
-// 128-bit broadcast weight loads and 128 fmaf.  Zero padding: the accumulator
-// starts at +0, a sum that rounds to zero is +0 in round-to-nearest, so it
-// never becomes -0 and fmaf(0, w, acc) == acc exactly -- the same value as
-// skipping the tap.  BN + HardTanh + quantize use exact fp32 breakpoints.
-template <int OUTB>
-__global__ void __launch_bounds__(FIRST_NT) conv_first_kernel(const FirstArgs a, const FirstTile tl) {
+// A CTA owns PB consecutive output pixels (row-major) of one image and 32 or
+// 64 output channels.  Shared memory holds the CTA's weights [K][OCB], its
+// breakpoints and the zero-padded input patch [C][rows][columns], the columns
+// split by stride phase (column rx at (rx % S) * Ws + rx / S) so that threads
+// reading neighbouring output pixels read neighbouring words for any stride.
+// Warp = 32 output channels x 64 pixels; a thread holds two pixels (32 apart)
+// x 32 channels as 16 channel pairs and per tap does two patch loads, eight
+// broadcast 128-bit weight loads and 32 packed fma.rn.f32x2, one fmaf chain
+// per output over (c, ky, kx) in that order.  Zero padding: the accumulator
+// starts at +0 and a sum that rounds to zero is +0, so it is never -0 and
+// fmaf(0, w, acc) == acc: the padded taps change nothing, exactly as skipping
+// them.  The epilogue turns each pixel's 32 channels into level masks (the
+// sign bits of fmaf(acc, sigma, -T)) and stores planes or codes from them.
+// KH, KW, S = 0: runtime shape.
+template <int OUTB, int KH, int KW, int S>
+__global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs a, const FirstTile tl) {
     extern __shared__ float4 smem4[];
-    float *sW = reinterpret_cast<float *>(smem4);                 // [K][32]
-    const int K = a.C * a.kh * a.kw;
-    float *sX = sW + 32 * K;                                      // [C][Rin][Win]
-    float *sT = sX + (size_t)a.C * tl.Rin * tl.Win;               // [32][8] breakpoints
-    int *sOff = reinterpret_cast<int *>(sT + 32 * 8);             // [K] patch offsets
+    const int kh = KH ? KH : a.kh, kw = KW ? KW : a.kw, st = S ? S : a.stride;
+    const int OCB = tl.OCB, K = tl.K, RP = tl.RP, Ws = tl.Ws;
+    float *sW = reinterpret_cast<float *>(smem4);                 // [K][OCB]
+    float *sT = sW + (size_t)K * OCB;                             // [OCB][8] -breakpoints, sigma
+    float *sX = sT + OCB * 8;                                     // [C][Rmax][RP]
 
-    const int g = blockIdx.y;
-    const int ochan = min(32, a.O - g * 32);
-    const int rblocks = (a.Ho + tl.R - 1) / tl.R;
-    const int b = blockIdx.x / rblocks;
-    const int oy0 = (blockIdx.x - b * rblocks) * tl.R;
-    const int iy0 = oy0 * a.stride - a.pad, ix0 = -a.pad;
+    const int b = blockIdx.x / tl.tiles;
+    const int p0 = (blockIdx.x - b * tl.tiles) * tl.PB;
+    const int o0 = blockIdx.y * OCB;
+    const int ochan = min(OCB, a.O - o0);
+    const int npix = a.Ho * a.Wo;
+    const int pend = min(p0 + tl.PB, npix);
+    const int y_first = p0 / a.Wo, y_last = (pend - 1) / a.Wo;
+    const int rows_in = (y_last - y_first) * st + kh;
+    const int Win = (a.Wo - 1) * st + kw;
+    const int iy0 = y_first * st - a.pad, ix0 = -a.pad;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    for (int i = threadIdx.x; i < 32 * K; i += FIRST_NT) {
-        const int k = i >> 5, oc = i & 31;
+    // weights: prepared [K][O] levels (coalesced), else the latent [O][K] array
+    const int osh = OCB == 64 ? 6 : 5;
+    for (int i = threadIdx.x; i < K * OCB; i += FIRST_NT) {
+        const int k = i >> osh, oc = i & (OCB - 1);
         float v = 0.0f;
         if (oc < ochan) {
-            const int o = g * 32 + oc;
-            v = a.w[(long long)o * K + k];
-            if (a.quant_w) {
-                const float sc = a.cscale ? a.cscale[o] : a.qw.scale;
-                v = level_value(v * sc, a.qw);
+            const int o = o0 + oc;
+            if (a.wt != nullptr) {
+                v = __ldg(a.wt + (long long)k * a.O + o);
+            } else {
+                v = __ldg(a.w + (long long)o * K + k);
+                if (a.quant_w) v = level_value(v * (a.cscale ? __ldg(a.cscale + o) : a.qw.scale), a.qw);
             }
         }
         sW[i] = v;
     }
-    const int plane = tl.Rin * tl.Win;
-    for (int i = threadIdx.x; i < a.C * plane; i += FIRST_NT) {
-        const int c = i / plane, rem = i - c * plane;
-        const int ry = rem / tl.Win, rx = rem - ry * tl.Win;
-        const int yi = iy0 + ry, xi = ix0 + rx;
-        float v = 0.0f;
-        if (yi >= 0 && yi < a.H && xi >= 0 && xi < a.W) v = __ldg(a.x + (((long long)b * a.C + c) * a.H + yi) * a.W + xi);
-        sX[i] = v;
-    }
-    for (int k = threadIdx.x; k < K; k += FIRST_NT) {
-        const int c = k / (a.kh * a.kw), r = k - c * a.kh * a.kw;
-        const int ky = r / a.kw, kx = r - ky * a.kw;
-        sOff[k] = c * plane + ky * tl.Win + kx;
-    }
-    if (a.quant_out && threadIdx.x < ochan) {
-        const int o = g * 32 + threadIdx.x;
-        if (a.thr != nullptr) {
-#pragma unroll
-            for (int u = 0; u < 8; ++u) sT[threadIdx.x * 8 + u] = __ldg(a.thr + o * 8 + u);
+    // breakpoints held for the mask test: (-T_1 .. -T_{n-1}, sigma); padding channels never reached
+    if (a.quant_out && threadIdx.x < OCB) {
+        float *t = sT + threadIdx.x * 8;
+        const int o = o0 + threadIdx.x;
+        const int nl = num_levels(a.qo.bits);
+        if (threadIdx.x >= ochan) {
+            for (int u = 0; u < 8; ++u) t[u] = u == nl - 1 ? 1.0f : -INFINITY;
         } else {
-            channel_thresholds_f32(__ldg(a.scale + o), __ldg(a.shift + o), a.qo, sT + threadIdx.x * 8);
+            if (a.thr != nullptr) {
+#pragma unroll
+                for (int u = 0; u < 8; ++u) t[u] = __ldg(a.thr + o * 8 + u);
+            } else {
+                channel_thresholds_f32(__ldg(a.scale + o), __ldg(a.shift + o), a.qo, t);
+            }
+            for (int u = 0; u < nl - 1; ++u) t[u] = mask_breakpoint(t[u]);
+        }
+    }
+    // input patch: one warp per (channel, row), lanes along the row
+    for (int cr = warp; cr < a.C * rows_in; cr += FIRST_NT / 32) {
+        const int c = cr / rows_in, r = cr - c * rows_in;
+        const int yi = iy0 + r;
+        const bool row_ok = yi >= 0 && yi < a.H;
+        const float *src = a.x + (((long long)b * a.C + c) * a.H + (row_ok ? yi : 0)) * a.W;
+        float *dst = sX + ((size_t)c * tl.Rmax + r) * RP;
+        for (int rx = lane; rx < Win; rx += 32) {
+            const int xi = ix0 + rx;
+            const float v = (row_ok && xi >= 0 && xi < a.W) ? __ldg(src + xi) : 0.0f;
+            dst[(rx % st) * Ws + rx / st] = v;
         }
     }
     __syncthreads();
 
-    const int npix = min(tl.R, a.Ho - oy0) * a.Wo;
-    int base[FIRST_PPT];
-    bool live[FIRST_PPT];
+    const int g = warp % tl.groups, pb = warp / tl.groups;
+    int pofs[FIRST_PX], pix[FIRST_PX];
+    bool live[FIRST_PX];
 #pragma unroll
-    for (int i = 0; i < FIRST_PPT; ++i) {
-        const int pidx = threadIdx.x + i * FIRST_NT;
-        live[i] = pidx < npix;
-        const int ly = live[i] ? pidx / a.Wo : 0, lx = live[i] ? pidx - (pidx / a.Wo) * a.Wo : 0;
-        base[i] = ly * a.stride * tl.Win + lx * a.stride;
+    for (int i = 0; i < FIRST_PX; ++i) {
+        const int p = p0 + pb * 64 + lane + 32 * i;
+        live[i] = p < pend;
+        pix[i] = live[i] ? p : p0;
+        const int yy = pix[i] / a.Wo, xx = pix[i] - yy * a.Wo;
+        pofs[i] = (yy - y_first) * st * RP + xx;
     }
-    if (!live[0]) return;
+    if (!live[0] || g * 32 >= ochan) return;
 
-    float acc[FIRST_PPT][32];
+    // accumulators of channel pairs (2j, 2j + 1), packed for fma.rn.f32x2
+    unsigned long long acc[FIRST_PX][16];
 #pragma unroll
-    for (int i = 0; i < FIRST_PPT; ++i)
+    for (int i = 0; i < FIRST_PX; ++i)
 #pragma unroll
-        for (int o = 0; o < 32; ++o) acc[i][o] = 0.0f;
-    for (int k = 0; k < K; ++k) {
-        const int off = sOff[k];
-        float xv[FIRST_PPT];
+        for (int o = 0; o < 16; ++o) acc[i][o] = 0ull;
+    const float *wg = sW + g * 32;
+    for (int c = 0; c < a.C; ++c) {
+#pragma unroll (KH ? KH : 1)
+        for (int ky = 0; ky < kh; ++ky) {
+            const float *xrow = sX + ((size_t)c * tl.Rmax + ky) * RP;
+            const float *wrow = wg + (size_t)((c * kh + ky) * kw) * OCB;
+            const float *xp[FIRST_PX];
 #pragma unroll
-        for (int i = 0; i < FIRST_PPT; ++i) xv[i] = sX[base[i] + off];
+            for (int i = 0; i < FIRST_PX; ++i) xp[i] = xrow + pofs[i];
+#pragma unroll (KW ? KW : 1)
+            for (int kx = 0; kx < kw; ++kx) {
+                // tap column kx: stride phase kx % S, offset kx / S within the phase
+                const int ph = kx % st, xo = kx / st;
+                unsigned long long xv[FIRST_PX];
 #pragma unroll
-        for (int o4 = 0; o4 < 8; ++o4) {
-            const float4 w = smem4[k * 8 + o4];
+                for (int i = 0; i < FIRST_PX; ++i) xv[i] = dup2((ph == 0 ? xp[i] : xp[i] + ph * Ws)[xo]);
+                const ulonglong2 *w2 = reinterpret_cast<const ulonglong2 *>(wrow + kx * OCB);
 #pragma unroll
-            for (int i = 0; i < FIRST_PPT; ++i) {
-                acc[i][4 * o4 + 0] = fmaf(xv[i], w.x, acc[i][4 * o4 + 0]);
-                acc[i][4 * o4 + 1] = fmaf(xv[i], w.y, acc[i][4 * o4 + 1]);
-                acc[i][4 * o4 + 2] = fmaf(xv[i], w.z, acc[i][4 * o4 + 2]);
-                acc[i][4 * o4 + 3] = fmaf(xv[i], w.w, acc[i][4 * o4 + 3]);
+                for (int o4 = 0; o4 < 8; ++o4) {
+                    const ulonglong2 w = w2[o4];
+#pragma unroll
+                    for (int i = 0; i < FIRST_PX; ++i) {
+                        ffma2(acc[i][2 * o4], xv[i], w.x);
+                        ffma2(acc[i][2 * o4 + 1], xv[i], w.y);
+                    }
+                }
             }
         }
     }
 
-    const long long HoWo = (long long)a.Ho * a.Wo;
+    const long long HoWo = (long long)npix;
     const int NWo = (a.O + 31) >> 5;
+    const int gch = min(32, ochan - g * 32);                     // live channels of this warp
+    const int ob = o0 + g * 32;
     constexpr int NL = OUTB == 0 ? 1 : (OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7));
 #pragma unroll
-    for (int i = 0; i < FIRST_PPT; ++i) {
+    for (int i = 0; i < FIRST_PX; ++i) {
         if (!live[i]) continue;
-        const int pix = oy0 * a.Wo + threadIdx.x + i * FIRST_NT;
-        const long long m = (long long)b * HoWo + pix;
+        const long long m = (long long)b * HoWo + pix[i];
         if (a.y_out) {
 #pragma unroll
             for (int oc = 0; oc < 32; ++oc) {
-                if (oc < ochan) {
-                    const int o = g * 32 + oc;
-                    float y = fmaf(acc[i][oc], __ldg(a.scale + o), __ldg(a.shift + o));
+                if (oc < gch) {
+                    const int o = ob + oc;
+                    float y = fmaf(lane2(acc[i][oc >> 1], oc & 1), __ldg(a.scale + o), __ldg(a.shift + o));
                     if (OUTB > 0) y = fminf(fmaxf(y, -1.0f), 1.0f);
-                    a.y_out[((long long)b * a.O + o) * HoWo + pix] = y;
+                    a.y_out[((long long)b * a.O + o) * HoWo + pix[i]] = y;
                 }
             }
         }
         if constexpr (OUTB > 0) {
-            int kq[32];
+            // level masks: bit oc of M[u] = [sigma * acc < T_u], from the sign of fmaf(acc, sigma, -T_u)
+            uint32_t M[NL - 1];
 #pragma unroll
-            for (int oc = 0; oc < 32; ++oc) {
-                const float *th = sT + oc * 8;
-                const float v = acc[i][oc] * th[NL - 1];
-                int k = 0;
+            for (int u = 0; u < NL - 1; ++u) M[u] = 0u;
 #pragma unroll
-                for (int u = 0; u < NL - 1; ++u) k += (v >= th[u]) ? 1 : 0;
-                kq[oc] = k;
+            for (int oc = 31; oc >= 0; --oc) {
+                const float *th = sT + (g * 32 + oc) * 8;
+                const float v = lane2(acc[i][oc >> 1], oc & 1), sg = th[NL - 1];
+#pragma unroll
+                for (int u = 0; u < NL - 1; ++u)
+                    M[u] = __funnelshift_l(__float_as_uint(fmaf(v, sg, th[u])), M[u], 1);
             }
-            if (a.codes_out != nullptr) {
-                uint32_t cw[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-#pragma unroll
-                for (int oc = 0; oc < 32; ++oc) cw[oc >> 2] |= first_code<OUTB>(kq[oc]) << ((oc & 3) * 8);
-                uint4 *dst = reinterpret_cast<uint4 *>(a.codes_out + m * a.O + g * 32);
-                dst[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
-                if (ochan > 16) dst[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
-            }
-            if (a.planes_out != nullptr) {
-                uint32_t words[OUTB];
-#pragma unroll
-                for (int u = 0; u < OUTB; ++u) words[u] = 0u;
-#pragma unroll
-                for (int oc = 0; oc < 32; ++oc) {
-                    const uint32_t pb = (oc < ochan) ? first_planes<OUTB>(kq[oc]) : 0u;
-#pragma unroll
-                    for (int u = 0; u < OUTB; ++u) words[u] |= ((pb >> u) & 1u) << oc;
-                }
-                uint32_t *dst = a.planes_out + (m * OUTB) * NWo + g;
-#pragma unroll
-                for (int u = 0; u < OUTB; ++u) dst[u * NWo] = words[u];
-            }
+            store_level_masks<OUTB>(M, gch, 32, a.planes_out ? a.planes_out + (m * OUTB) * NWo + (ob >> 5) : nullptr,
+                                    NWo, a.codes_out ? a.codes_out + m * a.O + ob : nullptr);
         }
     }
+}
+
+// Weights of a first layer prepared once: [K][O] (output channel fastest),
+// quantized to their levels with the per-channel prescale when quant_w.
+__global__ void first_weights_kernel(const float *__restrict__ w, int O, int K, int quant_w, QParams qw,
+                                     const float *__restrict__ cscale, float *__restrict__ wt) {
+    const long long n = (long long)O * K;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        const int o = (int)(i / K), k = (int)(i - (long long)o * K);
+        float v = w[i];
+        if (quant_w) v = level_value(v * (cscale ? cscale[o] : qw.scale), qw);
+        wt[(long long)k * O + o] = v;
+    }
+}
+
+minw_status launch_first_weights(const float *w, int O, int K, int quant_w, const QParams &qw, const float *cscale,
+                                 float *wt, cudaStream_t s) {
+    first_weights_kernel<<<256, 256, 0, s>>>(w, O, K, quant_w, qw, cscale, wt);
+    return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
 }
 
 // fp32 breakpoints of every channel, [O][8]: one thread per channel.
@@ -214,24 +266,38 @@ minw_status launch_thresholds_f32(const float *scale, const float *shift, int O,
     return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
 }
 
-minw_status launch_conv_first(const FirstArgs &a, cudaStream_t s) {
-    if (a.Wo > FIRST_MAXPIX) return MINW_EUNSUPPORTED;
-    const FirstTile tl = first_tile(a);
-    if (tl.smem > 200 * 1024) return MINW_EUNSUPPORTED;
-    const int outb = a.quant_out ? a.qo.bits : 0;
-    void (*kern)(const FirstArgs, const FirstTile) =
-        outb == 1 ? conv_first_kernel<1> : outb == 2 ? conv_first_kernel<2> : outb == 3 ? conv_first_kernel<3>
-                                                                                       : conv_first_kernel<0>;
-    static size_t configured_bytes[4] = {0, 0, 0, 0};
-    if (tl.smem > configured_bytes[outb]) {
+template <int OUTB, int KH, int KW, int S>
+static minw_status launch_first_shape(const FirstArgs &a, const FirstTile &tl, cudaStream_t s) {
+    static size_t configured = 0;
+    void (*kern)(const FirstArgs, const FirstTile) = conv_first_kernel<OUTB, KH, KW, S>;
+    if (tl.smem > configured) {
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tl.smem) != cudaSuccess)
             return MINW_ECUDA;
-        configured_bytes[outb] = tl.smem;
+        configured = tl.smem;
     }
-    const int rblocks = (a.Ho + tl.R - 1) / tl.R;
-    const dim3 grid((unsigned)(a.B * rblocks), (unsigned)((a.O + 31) / 32));
+    const dim3 grid((unsigned)(a.B * tl.tiles), (unsigned)((a.O + tl.OCB - 1) / tl.OCB));
     kern<<<grid, FIRST_NT, tl.smem, s>>>(a, tl);
     return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
+}
+
+template <int OUTB>
+static minw_status launch_first_bits(const FirstArgs &a, const FirstTile &tl, cudaStream_t s) {
+    if (a.kh == 3 && a.kw == 3 && a.stride == 1) return launch_first_shape<OUTB, 3, 3, 1>(a, tl, s);
+    if (a.kh == 7 && a.kw == 7 && a.stride == 2) return launch_first_shape<OUTB, 7, 7, 2>(a, tl, s);
+    return launch_first_shape<OUTB, 0, 0, 0>(a, tl, s);
+}
+
+minw_status launch_conv_first(const FirstArgs &a, cudaStream_t s) {
+    const FirstTile tl = first_tile(a);
+    if (tl.smem > 200 * 1024) return MINW_EUNSUPPORTED;
+    if (a.codes_out != nullptr && a.O % 16 != 0) return MINW_EUNSUPPORTED;
+    const int outb = a.quant_out ? a.qo.bits : 0;
+    switch (outb) {
+        case 1: return launch_first_bits<1>(a, tl, s);
+        case 2: return launch_first_bits<2>(a, tl, s);
+        case 3: return launch_first_bits<3>(a, tl, s);
+        default: return launch_first_bits<0>(a, tl, s);
+    }
 }
 
 }  // namespace minw

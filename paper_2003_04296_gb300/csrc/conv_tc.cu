@@ -241,11 +241,6 @@ __device__ __forceinline__ uint32_t planes_k(int k) {
     else return (uint32_t)((06420357ull >> (3 * k)) & 7ull);
 }
 
-// Four channels' bits (nibble g of m) spread to the low bit of four bytes.
-__device__ __forceinline__ uint32_t spread4(uint32_t m, int g) {
-    return (((m >> (4 * g)) & 0xFu) * 0x00204081u) & 0x01010101u;
-}
-
 // Epilogue of one 32-column chunk (16 when tail16 is false) of exact
 // accumulators, one tile row per lane, when the only output is the next
 // layer's levels.  For each breakpoint u the chunk becomes one 32-bit mask
@@ -296,41 +291,7 @@ __device__ __forceinline__ void mask_chunk(uint32_t taddr, bool full32, const fl
         }
     }
     if (!writer) return;
-    // planes: sign, then the non-zero mask (2 bits) or the magnitude code (3 bits)
-    uint32_t P[3];
-    if constexpr (OUTB == 1) {
-        P[0] = M[0];
-    } else if constexpr (OUTB == 2) {
-        P[0] = M[0];
-        P[1] = M[0] | ~M[1];
-    } else {
-        P[0] = M[2];
-        P[1] = M[0] | (M[2] & ~M[1]) | (M[4] & ~M[3]) | ~M[5];     // |k - 3| in {1, 3}
-        P[2] = M[1] | ~M[4];                                        // |k - 3| in {2, 3}
-    }
-    if (planes != nullptr) {
-        const uint32_t vm = nvalid >= 32 ? 0xffffffffu : ((1u << nvalid) - 1u);
-#pragma unroll
-        for (int u = 0; u < OUTB; ++u) planes[u * NWo] = P[u] & vm;
-    }
-    if (codes != nullptr) {
-        uint32_t cw[8];
-#pragma unroll
-        for (int g = 0; g < 8; ++g) {
-            if constexpr (OUTB == 1) {
-                cw[g] = (spread4(P[0], g) * 0x80u) | 0x38383838u;
-            } else if constexpr (OUTB == 2) {
-                cw[g] = spread4(P[1], g) * 0x38u + spread4(P[0], g) * 0x80u;
-            } else {
-                const uint32_t c0 = P[1], c1 = P[2];
-                cw[g] = spread4(c0, g) * 0x08u + spread4(c0 & ~c1, g) * 0x30u + spread4(c1, g) * 0x40u +
-                        spread4(P[0] & (c0 | c1), g) * 0x80u;
-            }
-        }
-        uint4 *dst = reinterpret_cast<uint4 *>(codes);
-        dst[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
-        if (nvalid > 16 && full32) dst[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
-    }
+    store_level_masks<OUTB>(M, nvalid, full32 ? 32 : 16, planes, NWo, codes);
 }
 
 // OUTB: bits of the quantized output (0 when the launch writes none).
@@ -389,13 +350,13 @@ __global__ void __launch_bounds__(NT, 1)
         if (p.thr != nullptr) {
             for (int i = threadIdx.x; i < p.O * NL; i += NT) {
                 const float x = __ldg(p.thr + i);
-                sthr[i] = (i % NL == NL - 1) ? x : (x == 0.0f ? 0.0f : -x);
+                sthr[i] = (i % NL == NL - 1) ? x : mask_breakpoint(x);
             }
         } else {
             for (int o = threadIdx.x; o < p.O; o += NT) {
                 float *t = sthr + o * NL;
                 channel_thresholds(__ldg(p.scale + o), __ldg(p.shift + o), p.qo, t);
-                for (int u = 0; u < NL - 1; ++u) t[u] = t[u] == 0.0f ? 0.0f : -t[u];
+                for (int u = 0; u < NL - 1; ++u) t[u] = mask_breakpoint(t[u]);
             }
         }
         for (int i = p.O * NL + threadIdx.x; i < thr_floats; i += NT)        // padding channels

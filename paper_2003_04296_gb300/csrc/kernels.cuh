@@ -53,10 +53,13 @@ struct FirstArgs {
     uint8_t *codes_out;        // [B][Ho][Wo][O] E4M3 level codes (nullable)
     float *y_out;              // [B][O][Ho][Wo] (nullable)
     const float *thr;          // fp32 breakpoints [O][8] (nullable: computed in-kernel)
+    const float *wt;           // prepared weights [K][O] (levels when quantized; nullable: from w)
 };
 
 // Launchers (host).  Return MINW_OK or an error status.
 minw_status launch_conv_first(const FirstArgs &a, cudaStream_t s);
+minw_status launch_first_weights(const float *w, int O, int K, int quant_w, const QParams &qw, const float *cscale,
+                                 float *wt, cudaStream_t s);
 minw_status launch_thresholds_f32(const float *scale, const float *shift, int O, const QParams &q, float *out,
                                   cudaStream_t s);
 minw_status launch_conv_popc(const ConvArgs &a, cudaStream_t s);

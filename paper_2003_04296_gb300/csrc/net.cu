@@ -110,6 +110,12 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
                 if ((st = net_alloc(n, &P.wscale, P.O)) != MINW_OK) { net_free(n); return st; }
                 cudaMemcpyAsync(P.wscale, d.w_scale, sizeof(float) * P.O, cudaMemcpyDeviceToDevice, s);
             }
+            if ((st = net_alloc(n, &P.wt, (size_t)P.O * K)) != MINW_OK) { net_free(n); return st; }
+            if ((st = launch_first_weights(P.wlatent, P.O, (int)K, d.bits_w > 0, to_qparams(&P.qw), P.wscale, P.wt,
+                                           s)) != MINW_OK) {
+                net_free(n);
+                return st;
+            }
         } else {
             if (P.C % 32 != 0) { net_free(n); return MINW_EUNSUPPORTED; }
             if (P.pad >= P.kh || P.pad >= P.kw) { net_free(n); return MINW_EUNSUPPORTED; }
@@ -214,6 +220,7 @@ minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits
             a.codes_out = out_codes ? (uint8_t *)dst : nullptr;
             a.y_out = last ? logits : nullptr;
             a.thr = P.thr;
+            a.wt = P.wt;
             st = launch_conv_first(a, cs);
         } else {
             const void *src = net->buf[cur ^ 1];

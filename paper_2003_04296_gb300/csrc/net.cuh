@@ -19,6 +19,7 @@ struct LayerPlan {
                                    // tensor-core layers: integer-valued [O][levels])
     int in_codes = 0;              // input arrives in the codes layout
     float *wlatent = nullptr;      // fp32 weights (first layer)
+    float *wt = nullptr;           // first layer: weights prepared as [K][O] levels
     float *wscale = nullptr;       // per-channel weight prescale (first layer)
     float *scale = nullptr;
     float *shift = nullptr;

@@ -142,6 +142,7 @@ struct ResNetPlan {
     int hw = 0, classes = 0, bits_a = 0, bits_w = 0;
     minw_quant qa{};
     float *stem_w = nullptr, *stem_scale = nullptr, *stem_shift = nullptr, *stem_thr = nullptr;
+    float *stem_wt = nullptr;              // stem weights as [147][64]
     int Hs = 0, Hp = 0;                    // stem output, pooled size
     ResBlock blocks[8];
     float *fc_wt = nullptr, *fc_scale = nullptr, *fc_shift = nullptr;
@@ -271,6 +272,9 @@ extern "C" minw_status minw_resnet18_create(const minw_resnet18_desc *d, int32_t
     if ((st = copy_owned(n, &R->stem_scale, d->stem_scale, 64, s)) != MINW_OK) return fail(st);
     if ((st = copy_owned(n, &R->stem_shift, d->stem_shift, 64, s)) != MINW_OK) return fail(st);
     if ((st = alloc_owned(n, &R->stem_thr, 64 * 8)) != MINW_OK) return fail(st);
+    if ((st = alloc_owned(n, &R->stem_wt, 64 * 3 * 49)) != MINW_OK) return fail(st);
+    if ((st = launch_first_weights(R->stem_w, 64, 3 * 49, 0, QParams{}, nullptr, R->stem_wt, s)) != MINW_OK)
+        return fail(st);
     if ((st = launch_thresholds_f32(R->stem_scale, R->stem_shift, 64, to_qparams(&R->qa), R->stem_thr, s)) != MINW_OK)
         return fail(st);
 
@@ -375,6 +379,7 @@ minw_status resnet_forward(minw_net *net, const float *x, int B, float *logits, 
         a.quant_out = 1; a.qo = to_qparams(&R->qa);
         a.codes_out = R->S;
         a.thr = R->stem_thr;
+        a.wt = R->stem_wt;
         if ((st = launch_conv_first(a, s)) != MINW_OK) return st;
         if ((st = mark()) != MINW_OK) return st;
     }
