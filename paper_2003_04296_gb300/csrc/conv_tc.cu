@@ -294,6 +294,83 @@ __device__ __forceinline__ void mask_chunk(uint32_t taddr, bool full32, const fl
     store_level_masks<OUTB>(M, nvalid, full32 ? 32 : 16, planes, NWo, codes);
 }
 
+// Epilogue of one 32-column chunk (16 when full32 is false) of a residual
+// block, one output pixel per lane: y = fmaf(acc, scale, shift), stored as
+// fp32 NHWC when asked (the BN output before the shortcut), then y + shortcut
+// (one fp32 add) and the next layer's levels from the sign bits of
+// y + (-T_u) against the quantizer's own breakpoints on y (HardTanh included),
+// through the same level masks as the plain epilogue.
+template <int OUTB>
+__device__ __forceinline__ void resid_chunk(uint32_t taddr, bool full32, const Params &p, int ob, long long opix,
+                                            bool writer, const float *syt, int NWo) {
+    uint32_t v[32];
+    if (full32) {
+        tmem_ld32(taddr, v);
+    } else {
+        uint32_t v16[16];
+        tmem_ld16(taddr, v16);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            v[j] = v16[j];
+            v[j + 16] = 0u;
+        }
+    }
+    if (!writer) return;
+    const int nvalid = min(32, p.O - ob);                 // a multiple of 16
+    const int ncol = full32 ? 32 : 16;
+    float y[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+        const int o = min(ob + j, p.O - 1);
+        y[j] = fmaf(__uint_as_float(v[j]), __ldg(p.scale + o), __ldg(p.shift + o));
+    }
+    const long long base = opix * p.O + ob;
+    if (p.y_nhwc != nullptr) {
+        float4 *dst = reinterpret_cast<float4 *>(p.y_nhwc + base);
+#pragma unroll
+        for (int q4 = 0; q4 < 8; ++q4)
+            if (q4 * 4 < nvalid && q4 * 4 < ncol) dst[q4] = make_float4(y[4 * q4], y[4 * q4 + 1], y[4 * q4 + 2], y[4 * q4 + 3]);
+    }
+    if constexpr (OUTB > 0) {
+        if (p.res_codes != nullptr) {
+            const uint4 *src = reinterpret_cast<const uint4 *>(p.res_codes + base);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                if (h * 16 >= nvalid || h * 16 >= ncol) break;
+                const uint4 cv = __ldg(src + h);
+                const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                    y[h * 16 + j] += code_units((cw[j >> 2] >> (8 * (j & 3))) & 0xFFu) * p.res_unit;
+            }
+        } else if (p.res_f32 != nullptr) {
+            const float4 *src = reinterpret_cast<const float4 *>(p.res_f32 + base);
+#pragma unroll
+            for (int q4 = 0; q4 < 8; ++q4) {
+                if (q4 * 4 >= nvalid || q4 * 4 >= ncol) break;
+                const float4 r = __ldg(src + q4);
+                y[4 * q4] += r.x;
+                y[4 * q4 + 1] += r.y;
+                y[4 * q4 + 2] += r.z;
+                y[4 * q4 + 3] += r.w;
+            }
+        }
+        constexpr int NL = OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7);
+        float nt[NL - 1];
+#pragma unroll
+        for (int u = 0; u < NL - 1; ++u) nt[u] = syt[u];
+        uint32_t M[NL - 1];
+#pragma unroll
+        for (int u = 0; u < NL - 1; ++u) M[u] = 0u;
+#pragma unroll
+        for (int j = 31; j >= 0; --j)
+#pragma unroll
+            for (int u = 0; u < NL - 1; ++u) M[u] = __funnelshift_l(__float_as_uint(y[j] + nt[u]), M[u], 1);
+        store_level_masks<OUTB>(M, nvalid, ncol, p.planes_out ? p.planes_out + (opix * OUTB) * NWo + (ob >> 5) : nullptr,
+                                NWo, p.codes_out ? p.codes_out + base : nullptr);
+    }
+}
+
 // OUTB: bits of the quantized output (0 when the launch writes none).
 template <int OUTB>
 __global__ void __launch_bounds__(NT, 1)
@@ -311,7 +388,9 @@ __global__ void __launch_bounds__(NT, 1)
     const int thr_floats = OUTB ? O32 * NL : 0;
     uint32_t *ssig = reinterpret_cast<uint32_t *>(sthr + thr_floats);              // [O32 / 32]
     const int sig_words = OUTB ? O32 / 32 : 0;
-    uint64_t *full = reinterpret_cast<uint64_t *>(ssig + ((sig_words + 1) & ~1));
+    // breakpoints of the output quantizer on y itself (residual blocks), held as -T
+    float *syt = reinterpret_cast<float *>(ssig + ((sig_words + 1) & ~1));
+    uint64_t *full = reinterpret_cast<uint64_t *>(syt + (OUTB ? 8 : 0));
     uint64_t *empty = full + p.S;
     uint64_t *tfull = empty + p.S;            // [2] accumulator ready
     uint64_t *tempty = tfull + 2;             // [2] accumulator drained
@@ -361,6 +440,11 @@ __global__ void __launch_bounds__(NT, 1)
         }
         for (int i = p.O * NL + threadIdx.x; i < thr_floats; i += NT)        // padding channels
             sthr[i] = ((i % NL) == NL - 1) ? 1.0f : 0.0f;
+        if (threadIdx.x == 0 && (p.res_codes != nullptr || p.res_f32 != nullptr)) {
+            float t[8];
+            channel_thresholds_f32(1.0f, 0.0f, p.qo, t);            // level of y = #{u : y >= t[u]}
+            for (int u = 0; u < NL - 1; ++u) syt[u] = mask_breakpoint(t[u]);
+        }
         // sigma of a channel: the sign of its BN scale (+1 for 0)
         for (int g = threadIdx.x; g < sig_words; g += NT) {
             uint32_t m = 0u;
@@ -492,6 +576,9 @@ __global__ void __launch_bounds__(NT, 1)
         // this warp's 32-column chunks
         const bool resid = p.res_codes != nullptr || p.res_f32 != nullptr || p.y_nhwc != nullptr;
         const bool masked = OUTB > 0 && p.ksplit == 1 && p.acc_out == nullptr && p.y_out == nullptr && !resid;
+        // residual epilogue without per-element fp32 outputs: the same chunks
+        const bool rmasked = p.ksplit == 1 && p.acc_out == nullptr && p.y_out == nullptr && !p.pool && resid &&
+                             p.O % 16 == 0;
         const int nch = (p.BN + 31) >> 5, cmid = (nch + 1) >> 1;
         const int cbeg = half_cols ? cmid : 0, cend = half_cols ? nch : cmid;
         int i = 0;
@@ -530,6 +617,21 @@ __global__ void __launch_bounds__(NT, 1)
                     if (lane == 0 && !dead) mbar_arrive(&tempty[ab]);
                     continue;
                 }
+            }
+            if (rmasked) {
+                if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
+                fence_after();
+                for (int c = cbeg; c < cend && !dead; ++c) {
+                    const int ob = o0 + c * 32;
+                    if (ob >= p.O) break;
+                    __syncwarp();
+                    resid_chunk<OUTB>(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * p.BN + c * 32),
+                                      c * 32 + 32 <= p.BN, p, ob, opix, writer, syt, NWo);
+                }
+                fence_before();
+                __syncwarp();
+                if (lane == 0 && !dead) mbar_arrive(&tempty[ab]);
+                continue;
             }
 
             // the fused block epilogue of one 16-column group of exact accumulators
@@ -895,7 +997,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     p.thr = a.thr;
     p.stage_bytes = p.a_bytes + (uint32_t)(p.BN * p.ck);
     const size_t o32 = ((size_t)a.O + 31) & ~(size_t)31;
-    const size_t thr_bytes = a.quant_out ? (o32 * p.nlev + o32 / 32 + 2) * sizeof(float) : 0;
+    const size_t thr_bytes = a.quant_out ? (o32 * p.nlev + o32 / 32 + 10) * sizeof(float) : 0;
     const size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes;
     int S = (int)(budget / p.stage_bytes);
     if (S > 8) S = 8;

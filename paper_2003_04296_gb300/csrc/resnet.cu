@@ -82,38 +82,48 @@ __global__ void __launch_bounds__(256) pool_levels_kernel(const uint8_t *__restr
     }
 }
 
-// Head: global average pool of level codes [B][HW][C] (one fp32 sum over the
-// pixels in order, then one division), fp32 fully connected layer (one fmaf
-// chain over the features in order, weights transposed to [C][classes]) and
-// BN (fmaf).  CTA = 8 images; the pooled features sit in shared memory.
-constexpr int HEAD_IMGS = 8;
-__global__ void __launch_bounds__(256) head_kernel(const uint8_t *__restrict__ X, int B, int HW, int C, float unit,
-                                                   const float *__restrict__ wt, int classes,
-                                                   const float *__restrict__ scale, const float *__restrict__ shift,
-                                                   float *__restrict__ logits) {
-    extern __shared__ float pooled[];                 // [HEAD_IMGS][C]
+// Head, first part: global average pool of level codes [B][HW][C] -> fp32
+// [B][C]; thread = (image, channel), one fp32 sum over the pixels in order,
+// then one division.
+__global__ void __launch_bounds__(256) avgpool_levels_kernel(const uint8_t *__restrict__ X, int B, int HW, int C,
+                                                             float unit, float *__restrict__ pooled) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= B * C) return;
+    const int b = i / C, c = i - b * C;
+    const uint8_t *src = X + (long long)b * HW * C + c;
+    float s = 0.0f;
+    for (int p = 0; p < HW; ++p) s += (float)code_to_units(__ldg(src + (long long)p * C)) * unit;
+    pooled[i] = s / (float)HW;
+}
+
+// Head, second part: fp32 fully connected layer (one fmaf chain over the
+// features in order; weights transposed to [C][classes]) and BN (fmaf).
+// CTA = 8 images x 128 classes; the pooled features of its images sit in
+// shared memory.
+constexpr int HEAD_IMGS = 8, HEAD_CLS = 128;
+__global__ void __launch_bounds__(HEAD_CLS) fc_head_kernel(const float *__restrict__ pooled, int B, int C,
+                                                           const float *__restrict__ wt, int classes,
+                                                           const float *__restrict__ scale,
+                                                           const float *__restrict__ shift,
+                                                           float *__restrict__ logits) {
+    extern __shared__ float sp[];                    // [HEAD_IMGS][C]
     const int b0 = blockIdx.x * HEAD_IMGS;
     const int nimg = min(HEAD_IMGS, B - b0);
-    for (int i = threadIdx.x; i < nimg * C; i += blockDim.x) {
-        const int im = i / C, c = i - (i / C) * C;
-        const uint8_t *src = X + (long long)(b0 + im) * HW * C + c;
-        float s = 0.0f;
-        for (int p = 0; p < HW; ++p) s += (float)code_to_units(src[(long long)p * C]) * unit;
-        pooled[im * C + c] = s / (float)HW;
-    }
+    for (int i = threadIdx.x; i < HEAD_IMGS * C; i += HEAD_CLS)
+        sp[i] = i < nimg * C ? pooled[(long long)b0 * C + i] : 0.0f;
     __syncthreads();
-    for (int o = threadIdx.x; o < classes; o += blockDim.x) {
-        float acc[HEAD_IMGS];
+    const int o = blockIdx.y * HEAD_CLS + threadIdx.x;
+    if (o >= classes) return;
+    float acc[HEAD_IMGS];
 #pragma unroll
-        for (int im = 0; im < HEAD_IMGS; ++im) acc[im] = 0.0f;
-        for (int k = 0; k < C; ++k) {
-            const float w = __ldg(wt + (long long)k * classes + o);
+    for (int im = 0; im < HEAD_IMGS; ++im) acc[im] = 0.0f;
+    for (int k = 0; k < C; ++k) {
+        const float w = __ldg(wt + (long long)k * classes + o);
 #pragma unroll
-            for (int im = 0; im < HEAD_IMGS; ++im) acc[im] = fmaf(pooled[im * C + k], w, acc[im]);
-        }
-        const float sc = __ldg(scale + o), sh = __ldg(shift + o);
-        for (int im = 0; im < nimg; ++im) logits[(long long)(b0 + im) * classes + o] = fmaf(acc[im], sc, sh);
+        for (int im = 0; im < HEAD_IMGS; ++im) acc[im] = fmaf(sp[im * C + k], w, acc[im]);
     }
+    const float sc = __ldg(scale + o), sh = __ldg(shift + o);
+    for (int im = 0; im < nimg; ++im) logits[(long long)(b0 + im) * classes + o] = fmaf(acc[im], sc, sh);
 }
 
 __global__ void transpose_kernel(const float *__restrict__ in, int rows, int cols, float *__restrict__ out) {
@@ -146,6 +156,7 @@ struct ResNetPlan {
     int Hs = 0, Hp = 0;                    // stem output, pooled size
     ResBlock blocks[8];
     float *fc_wt = nullptr, *fc_scale = nullptr, *fc_shift = nullptr;
+    float *pooled = nullptr;               // head: average-pooled features [max_batch][512]
     uint8_t *S = nullptr, *X = nullptr, *Y = nullptr, *V = nullptr;
     float *D = nullptr;
 };
@@ -217,7 +228,7 @@ static ConvArgs block_conv(const minw_net *net, const ResBlock &bk, int which, i
 }
 
 int32_t resnet_kernels(const minw_net *net) {
-    int k = 3;
+    int k = 4;                             // stem, pool, average pool + classifier
     const ResNetPlan *R = net->res;
     for (const ResBlock &bk : R->blocks)
         for (int which = 0; which < 3; ++which)
@@ -344,6 +355,7 @@ extern "C" minw_status minw_resnet18_create(const minw_resnet18_desc *d, int32_t
     if ((st = alloc_owned(n, &R->Y, act_codes)) != MINW_OK) return fail(st);
     if ((st = alloc_owned(n, &R->V, act_codes)) != MINW_OK) return fail(st);
     if ((st = alloc_owned(n, &R->D, down_f32)) != MINW_OK) return fail(st);
+    if ((st = alloc_owned(n, &R->pooled, Bm * 512)) != MINW_OK) return fail(st);
     if (ws) {
         uint8_t *w = nullptr;
         if ((st = alloc_owned(n, &w, ws)) != MINW_OK) return fail(st);
@@ -407,9 +419,11 @@ minw_status resnet_forward(minw_net *net, const float *x, int B, float *logits, 
     {
         const ResConv &last = R->blocks[7].c2;
         const int HW = last.Ho * last.Wo;
+        avgpool_levels_kernel<<<(unsigned)((B * 512 + 255) / 256), 256, 0, s>>>(X, B, HW, 512, unit, R->pooled);
         const size_t smem = sizeof(float) * HEAD_IMGS * 512;
-        head_kernel<<<(unsigned)((B + HEAD_IMGS - 1) / HEAD_IMGS), 256, smem, s>>>(
-            X, B, HW, 512, unit, R->fc_wt, R->classes, R->fc_scale, R->fc_shift, logits);
+        const dim3 grid((unsigned)((B + HEAD_IMGS - 1) / HEAD_IMGS), (unsigned)((R->classes + HEAD_CLS - 1) / HEAD_CLS));
+        fc_head_kernel<<<grid, HEAD_CLS, smem, s>>>(R->pooled, B, 512, R->fc_wt, R->classes, R->fc_scale, R->fc_shift,
+                                                   logits);
         if (cudaGetLastError() != cudaSuccess) return MINW_ECUDA;
         if ((st = mark()) != MINW_OK) return st;
     }
