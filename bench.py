@@ -1,11 +1,13 @@
 #!/usr/bin/env python3
 """Throughput of the MINW-Net inference path on GB300.
 
-Workload: the CIFAR-shaped Model-A ConvNet forward (conv 128-128-P-256-256-P-
-512-512-P, FC 1024-1024-10), batch 256 per GPU, 1-bit activations x 1-bit
-weights in every hidden layer, fp32 image into the first layer, fp32 logits
-out.  Synthetic seeded data (U(-1,1) images, N(0,0.05) latent weights, folded
-BN maps); no dataset.  One step = one minw_forward over the batch.
+Default workload: the CIFAR-shaped Model-A ConvNet forward (conv 128-128-P-
+256-256-P-512-512-P, FC 1024-1024-10), batch 256 per GPU, 1-bit activations x
+1-bit weights in every hidden layer, fp32 image into the first layer, fp32
+logits out.  ``--workload resnet18``: the ResNet-18-shaped network, batch 128
+of 3x224x224 images, 3-bit activations and weights, fp32 stem and classifier.
+Synthetic seeded data (images, latent weights, folded BN maps); no dataset.
+One step = one minw_forward over the batch.
 
 Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle on
 a bounded sample of the same workload instead.
@@ -26,8 +28,6 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "MINW-Net conv effective binary TOPS and forward images/s; fraction of roofline"
-BATCH = 256
-SEED = 2
 L2_FLUSH_BYTES = 256 << 20
 SMS = 152
 SM_MAX_MHZ = 2070.0
@@ -71,12 +71,78 @@ def _captured_traffic(bound):
 FP8_TFLOPS = 2.0 * BF16_TFLOPS
 
 
-def workload_config(bits_a, bits_w, batch, n_gpus, l2):
-    return {"workload": f"cifar_convnet_fwd_a{bits_a}w{bits_w}", "batch_per_gpu": batch,
-            "global_batch": batch * n_gpus, "input": "3x32x32 fp32 U(-1,1)",
-            "layers": "conv3x3 128,128,P,256,256,P,512,512,P; fc 1024,1024,10",
-            "bits_a": bits_a, "bits_w": bits_w, "first_layer": "fp32 input, quantized weights",
-            "parallelism": f"replicas x{n_gpus} (batch-sharded, no collective)", "l2": l2}
+L2_NOTE = "flushed between steps (256 MiB write outside the timed events)"
+
+
+class Workload:
+    """One benchmarked network: its seeded parameters and images, the net
+    built through the library's API, the oracle forward, and the MACs of each
+    op the net times (``minw_net_layer_times`` order)."""
+
+    def __init__(self, name, args):
+        from paper_2003_04296_gb300 import inputs as I
+        self.name = name
+        if name == "cifar_convnet":
+            self.batch, self.seed = 256, 2
+            self.params = I.convnet_params(self.seed, bits_a=args.bits_a, bits_w=args.bits_w)
+            self.bits = (args.bits_a, args.bits_w)
+        else:
+            self.batch, self.seed = 128, 4
+            self.params = I.resnet18_params(self.seed, bits_a=args.bits_a_resnet, bits_w=args.bits_w_resnet)
+            self.bits = (args.bits_a_resnet, args.bits_w_resnet)
+
+    def images(self, rank):
+        from paper_2003_04296_gb300 import inputs as I
+        if self.name == "cifar_convnet":
+            return I.convnet_input(self.seed + 1000 * rank, self.batch)
+        return I.resnet18_input(self.seed + 1000 * rank, self.batch)
+
+    def net(self, minw, dev, variant):
+        if self.name == "cifar_convnet":
+            return minw.Net(minw.layer_descs(self.params, dev), max_batch=self.batch, variant=variant)
+        return minw.Net.resnet18(self.params, self.batch, dev)
+
+    def oracle(self, x):
+        from oracle import network as N
+        if self.name == "cifar_convnet":
+            return N.convnet_forward(self.params, x)
+        return N.resnet18_forward(self.params, x)
+
+    def op_macs(self):
+        """MACs per image of each timed op, and the indices of the ops that
+        run the quantized convolution (the roofline's kernel)."""
+        if self.name == "cifar_convnet":
+            m = layer_macs(self.params)
+            return m, list(range(1, len(m)))
+        hw = self.params["hw"]
+        s = hw // 2
+        macs = [s * s * 64 * 3 * 49, 0]
+        size = s // 2
+        for blk in self.params["blocks"]:
+            o, c = blk["c1"]["w"].shape[:2]
+            so = size // blk["stride"]
+            macs.append(so * so * o * c * 9)
+            if blk["down"] is not None:
+                macs.append(so * so * o * c)
+            macs.append(so * so * o * o * 9)
+            size = so
+        macs.append(512 * self.params["classes"])
+        return macs, list(range(2, len(macs) - 1))
+
+    def config(self, n_gpus):
+        ba, bw = self.bits
+        par = f"replicas x{n_gpus} (batch-sharded, no collective)"
+        if self.name == "cifar_convnet":
+            return {"workload": f"cifar_convnet_fwd_a{ba}w{bw}", "batch_per_gpu": self.batch,
+                    "global_batch": self.batch * n_gpus, "input": "3x32x32 fp32 U(-1,1)",
+                    "layers": "conv3x3 128,128,P,256,256,P,512,512,P; fc 1024,1024,10",
+                    "bits_a": ba, "bits_w": bw, "first_layer": "fp32 input, quantized weights",
+                    "parallelism": par, "l2": L2_NOTE}
+        return {"workload": f"resnet18_fwd_a{ba}w{bw}", "batch_per_gpu": self.batch,
+                "global_batch": self.batch * n_gpus, "input": "3x224x224 fp32 N(0,1)",
+                "layers": "stem 7x7/2 64 + maxpool 3x3/2; basic blocks [2,2,2,2] 64-128-256-512; avgpool; fc 1000",
+                "bits_a": ba, "bits_w": bw, "first_layer": "fp32 stem and classifier (fp32 weights)",
+                "parallelism": par, "l2": L2_NOTE}
 
 
 def layer_macs(net_p, hw=32):
@@ -112,8 +178,12 @@ class ClockSampler:
             os.close(fd)
             self.out = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
                                          stdout=self.out, stderr=subprocess.DEVNULL)
+            # the timed region starts once the sampler is running (first line written)
+            t0 = time.time()
+            while time.time() - t0 < 5.0 and os.path.getsize(self.path) == 0 and self.proc.poll() is None:
+                time.sleep(0.02)
         except (OSError, FileNotFoundError):
             self.proc = None
         return self
@@ -154,13 +224,12 @@ class ClockSampler:
 
 # --------------------------------------------------------------- reference --
 
-def oracle_images_per_s(net_p, x, max_seconds):
+def oracle_images_per_s(wl, x, max_seconds):
     """Time the oracle's network forward image by image until max_seconds."""
-    from oracle import network as N
-    N.convnet_forward(net_p, x[:1])           # builds and loads the oracle
+    wl.oracle(x[:1])                          # builds and loads the oracle
     done, t0 = 0, time.perf_counter()
     while done < x.shape[0]:
-        N.convnet_forward(net_p, x[done:done + 1])
+        wl.oracle(x[done:done + 1])
         done += 1
         if time.perf_counter() - t0 >= max_seconds:
             break
@@ -171,32 +240,30 @@ def oracle_images_per_s(net_p, x, max_seconds):
 def run_reference(args, rank):
     if rank != 0:
         return 0
-    from paper_2003_04296_gb300.inputs import convnet_input, convnet_params
-    net_p = convnet_params(SEED, bits_a=args.bits_a, bits_w=args.bits_w)
-    x = convnet_input(SEED, BATCH)
-    from oracle import network as N
+    wl = Workload(args.workload, args)
+    x = wl.images(0)
+    B = wl.batch
     # per-step sample sized so that warmup + steps stay within ~3 minutes
     t0 = time.perf_counter()
-    N.convnet_forward(net_p, x[:1])
+    wl.oracle(x[:1])
     t_img = time.perf_counter() - t0
-    per_step = max(1, min(BATCH, int(150.0 / max(args.warmup + args.steps, 1) / max(t_img, 1e-3))))
+    per_step = max(1, min(B, int(150.0 / max(args.warmup + args.steps, 1) / max(t_img, 1e-3))))
     for _ in range(args.warmup):
-        N.convnet_forward(net_p, x[:per_step])
+        wl.oracle(x[:per_step])
     times = []
     for k in range(args.steps):
-        lo = (k * per_step) % BATCH
+        lo = (k * per_step) % B
         xs = x[lo:lo + per_step]
         t0 = time.perf_counter()
-        N.convnet_forward(net_p, xs)
+        wl.oracle(xs)
         times.append(time.perf_counter() - t0)
     sec = sum(times) / len(times)
     ips = per_step / sec
-    sample = f"{per_step} of the {BATCH} images per step, single-threaded C oracle, extrapolated to images/s"
+    sample = f"{per_step} of the {B} images per step, single-threaded C oracle, extrapolated to images/s"
     line = {"metric": METRIC, "value": ips, "unit": "images/s", "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True, "impl": "reference",
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": workload_config(args.bits_a, args.bits_w, BATCH, args.gpus,
-                                      "flushed between steps (256 MiB write outside the timed events)"),
+            "config": wl.config(args.gpus),
             "cpu_baseline": {"value": ips, "unit": "images/s", "cores": 1, "kind": "oracle", "sample": sample},
             "e2e": {"value": ips, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -217,18 +284,19 @@ def run_gpu(args, rank, world, local_rank):
     if world > 1:
         dist.barrier()
     from paper_2003_04296_gb300 import minw
-    from paper_2003_04296_gb300.inputs import convnet_input, convnet_params
 
-    net_p = convnet_params(SEED, bits_a=args.bits_a, bits_w=args.bits_w)
-    x_np = convnet_input(SEED + 1000 * rank, BATCH)
-    net = minw.Net(minw.layer_descs(net_p, dev), max_batch=BATCH, variant=args.variant)
+    wl = Workload(args.workload, args)
+    BATCH = wl.batch
+    x_np = wl.images(rank)
+    net = wl.net(minw, dev, args.variant)
     x = torch.from_numpy(x_np).to(dev)
     logits = torch.empty((BATCH, net.out_features), dtype=torch.float32, device=dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
     net.enable_timing(True)
-    macs = layer_macs(net_p)
+    macs, q_ops_idx = wl.op_macs()
     nl = net.launches
+    assert len(macs) == nl, (len(macs), nl)
 
     for _ in range(max(args.warmup, 3)):
         net.forward(x, logits)
@@ -287,12 +355,13 @@ def run_gpu(args, rank, world, local_rank):
     value = BATCH * world / (ms_max * 1e-3)
     eff_tops = 2.0 * total_macs * world / (ms_max * 1e-3) / 1e12
 
-    # roofline of the dominant kernel: the quantized convolution (layers 2..n)
+    # roofline of the dominant kernel: the quantized convolution (every op in q_ops_idx)
     variants = net.layer_variants()
-    q_ms = float(layer_ms[1:].sum())
-    q_ops = 2.0 * sum(macs[1:]) * BATCH
+    q_ms = float(sum(layer_ms[i] for i in q_ops_idx))
+    q_ops = 2.0 * sum(macs[i] for i in q_ops_idx) * BATCH
     achieved = q_ops / (q_ms * 1e-3) / 1e12
-    if all(v == minw.VARIANT_TC for v in variants[1:]):
+    all_tc = all(variants[i] == minw.VARIANT_TC for i in q_ops_idx)
+    if all_tc:
         peak = FP8_TFLOPS
         roofline = {"bound": "tensor", "kernel": "conv_tc_kernel (tcgen05 kind::f8f6f4, all quantized layers)",
                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
@@ -306,20 +375,19 @@ def run_gpu(args, rank, world, local_rank):
                     "frac": achieved / peak, "traffic": None,
                     "peak_basis": "16 popc/clk/SM x 32 MAC/popc x 2 ops x 152 SMs x 2070 MHz"}
     roofline["layer_variants"] = variants
-    roofline["traffic"] = _captured_traffic(roofline["bound"])
+    roofline["traffic"] = _captured_traffic(roofline["bound"]) if wl.name == "cifar_convnet" else None
 
     cpu = None
     if world == 1 and not args.skip_cpu:
-        ips, n_img, secs = oracle_images_per_s(net_p, x_np, args.cpu_seconds)
+        ips, n_img, secs = oracle_images_per_s(wl, x_np, args.cpu_seconds)
         cpu = {"value": ips, "unit": "images/s", "cores": 1, "kind": "oracle",
                "sample": f"{n_img} images of the batch through the single-threaded C oracle ({secs:.1f} s)"}
 
     line = {"metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "e4m3" if all(v == minw.VARIANT_TC for v in variants[1:]) else "b1",
+            "vs_baseline": None, "dtype": "e4m3" if all_tc else "b1",
             "data": "synthetic",
-            "config": workload_config(args.bits_a, args.bits_w, BATCH, world,
-                                      "flushed between steps (256 MiB write outside the timed events)"),
+            "config": wl.config(world),
             "eff_tops": eff_tops,
             "layer_ms": [round(v, 5) for v in layer_ms.tolist()],
             "roofline": roofline, "cpu_baseline": cpu,
@@ -337,8 +405,11 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["minw", "reference"], default="minw")
-    ap.add_argument("--bits-a", type=int, default=1)
-    ap.add_argument("--bits-w", type=int, default=1)
+    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18"], default="cifar_convnet")
+    ap.add_argument("--bits-a", type=int, default=1, help="CIFAR ConvNet activation bits")
+    ap.add_argument("--bits-w", type=int, default=1, help="CIFAR ConvNet weight bits")
+    ap.add_argument("--bits-a-resnet", type=int, default=3)
+    ap.add_argument("--bits-w-resnet", type=int, default=3)
     ap.add_argument("--variant", type=int, default=0, help="0 auto, 1 popcount, 2 tensor cores")
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--skip-cpu", action="store_true")

@@ -59,44 +59,79 @@ static FirstTile first_tile(const FirstArgs &a) {
     t.Ws = (Win + a.stride - 1) / a.stride;
     t.RP = t.Ws * a.stride;
     t.K = a.C * a.kh * a.kw;
-    t.smem = sizeof(float) * ((size_t)t.K * t.OCB + (size_t)t.OCB * 8 + (size_t)a.C * t.Rmax * t.RP);
+    t.smem = sizeof(float) * ((size_t)t.K * t.OCB + (size_t)t.OCB * 8 + 2 * (size_t)a.C * t.Rmax * t.RP);
     return t;
 }
 
-// A CTA owns PB consecutive output pixels (row-major) of one image and 32 or
-// 64 output channels.  Shared memory holds the CTA's weights [K][OCB], its
-// breakpoints and the zero-padded input patch [C][rows][columns], the columns
-// split by stride phase (column rx at (rx % S) * Ws + rx / S) so that threads
-// reading neighbouring output pixels read neighbouring words for any stride.
-// Warp = 32 output channels x 64 pixels; a thread holds two pixels (32 apart)
-// x 32 channels as 16 channel pairs and per tap does two patch loads, eight
-// broadcast 128-bit weight loads and 32 packed fma.rn.f32x2, one fmaf chain
-// per output over (c, ky, kx) in that order.  Zero padding: the accumulator
-// starts at +0 and a sum that rounds to zero is +0, so it is never -0 and
-// fmaf(0, w, acc) == acc: the padded taps change nothing, exactly as skipping
-// them.  The epilogue turns each pixel's 32 channels into level masks (the
-// sign bits of fmaf(acc, sigma, -T)) and stores planes or codes from them.
-// KH, KW, S = 0: runtime shape.
+// 4-byte asynchronous global -> shared copy; src_bytes = 0 writes a zero.
+__device__ __forceinline__ void cp_async4(float *dst, const float *src, int src_bytes) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"((uint32_t)__cvta_generic_to_shared(dst)),
+                 "l"(src), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+// Persistent CTAs own 32 or 64 output channels and walk pixel tiles of PB
+// consecutive output pixels (row-major within one image).  Shared memory
+// holds the weights [K][OCB] and breakpoints, loaded once, and two input
+// patches [C][rows][columns] (zero padded; columns split by stride phase, column
+// rx at (rx % S) * Ws + rx / S, so that threads reading neighbouring output
+// pixels read neighbouring words for any stride): the next tile's patch
+// arrives by cp.async while the current one is computed.  Warp = 32 output
+// channels x 64 pixels; a thread holds two pixels (32 apart) x 32 channels as
+// 16 channel pairs and per tap does two patch loads, eight broadcast 128-bit
+// weight loads and 32 packed fma.rn.f32x2, one fmaf chain per output over
+// (c, ky, kx) in that order.  Zero padding: the accumulator starts at +0 and
+// a sum that rounds to zero is +0, so it is never -0 and fmaf(0, w, acc) ==
+// acc: the padded taps change nothing, exactly as skipping them.  The
+// epilogue turns each pixel's 32 channels into level masks (the sign bits of
+// fmaf(acc, sigma, -T)) and stores planes or codes from them.  KH, KW, S = 0:
+// runtime shape.
 template <int OUTB, int KH, int KW, int S>
 __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs a, const FirstTile tl) {
     extern __shared__ float4 smem4[];
     const int kh = KH ? KH : a.kh, kw = KW ? KW : a.kw, st = S ? S : a.stride;
     const int OCB = tl.OCB, K = tl.K, RP = tl.RP, Ws = tl.Ws;
+    const size_t patch = (size_t)a.C * tl.Rmax * RP;
     float *sW = reinterpret_cast<float *>(smem4);                 // [K][OCB]
     float *sT = sW + (size_t)K * OCB;                             // [OCB][8] -breakpoints, sigma
-    float *sX = sT + OCB * 8;                                     // [C][Rmax][RP]
+    float *sX0 = sT + OCB * 8;                                    // [2][C][Rmax][RP]
 
-    const int b = blockIdx.x / tl.tiles;
-    const int p0 = (blockIdx.x - b * tl.tiles) * tl.PB;
     const int o0 = blockIdx.y * OCB;
     const int ochan = min(OCB, a.O - o0);
     const int npix = a.Ho * a.Wo;
-    const int pend = min(p0 + tl.PB, npix);
-    const int y_first = p0 / a.Wo, y_last = (pend - 1) / a.Wo;
-    const int rows_in = (y_last - y_first) * st + kh;
     const int Win = (a.Wo - 1) * st + kw;
-    const int iy0 = y_first * st - a.pad, ix0 = -a.pad;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int total = a.B * tl.tiles;
+
+    // asynchronous load of tile t's input patch into buffer buf
+    auto load_patch = [&](int t, int buf) {
+        const int b = t / tl.tiles;
+        const int p0 = (t - b * tl.tiles) * tl.PB;
+        const int pend = min(p0 + tl.PB, npix);
+        const int y_first = p0 / a.Wo, y_last = (pend - 1) / a.Wo;
+        const int rows_in = (y_last - y_first) * st + kh;
+        const int iy0 = y_first * st - a.pad, ix0 = -a.pad;
+        float *sX = sX0 + buf * patch;
+        for (int cr = warp; cr < a.C * rows_in; cr += FIRST_NT / 32) {
+            const int c = cr / rows_in, r = cr - c * rows_in;
+            const int yi = iy0 + r;
+            const bool row_ok = yi >= 0 && yi < a.H;
+            const float *src = a.x + (((long long)b * a.C + c) * a.H + (row_ok ? yi : 0)) * a.W;
+            float *dst = sX + ((size_t)c * tl.Rmax + r) * RP;
+            for (int rx = lane; rx < Win; rx += 32) {
+                const int xi = ix0 + rx;
+                const bool ok = row_ok && xi >= 0 && xi < a.W;
+                cp_async4(dst + (rx % st) * Ws + rx / st, ok ? src + xi : src, ok ? 4 : 0);
+            }
+        }
+        cp_async_commit();
+    };
+
+    int t = blockIdx.x;
+    if (t < total) load_patch(t, 0);
 
     // weights: prepared [K][O] levels (coalesced), else the latent [O][K] array
     const int osh = OCB == 64 ? 6 : 5;
@@ -116,121 +151,136 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
     }
     // breakpoints held for the mask test: (-T_1 .. -T_{n-1}, sigma); padding channels never reached
     if (a.quant_out && threadIdx.x < OCB) {
-        float *t = sT + threadIdx.x * 8;
+        float *th = sT + threadIdx.x * 8;
         const int o = o0 + threadIdx.x;
         const int nl = num_levels(a.qo.bits);
         if (threadIdx.x >= ochan) {
-            for (int u = 0; u < 8; ++u) t[u] = u == nl - 1 ? 1.0f : -INFINITY;
+            for (int u = 0; u < 8; ++u) th[u] = u == nl - 1 ? 1.0f : -INFINITY;
         } else {
             if (a.thr != nullptr) {
 #pragma unroll
-                for (int u = 0; u < 8; ++u) t[u] = __ldg(a.thr + o * 8 + u);
+                for (int u = 0; u < 8; ++u) th[u] = __ldg(a.thr + o * 8 + u);
             } else {
-                channel_thresholds_f32(__ldg(a.scale + o), __ldg(a.shift + o), a.qo, t);
+                channel_thresholds_f32(__ldg(a.scale + o), __ldg(a.shift + o), a.qo, th);
             }
-            for (int u = 0; u < nl - 1; ++u) t[u] = mask_breakpoint(t[u]);
+            for (int u = 0; u < nl - 1; ++u) th[u] = mask_breakpoint(th[u]);
         }
     }
-    // input patch: one warp per (channel, row), lanes along the row
-    for (int cr = warp; cr < a.C * rows_in; cr += FIRST_NT / 32) {
-        const int c = cr / rows_in, r = cr - c * rows_in;
-        const int yi = iy0 + r;
-        const bool row_ok = yi >= 0 && yi < a.H;
-        const float *src = a.x + (((long long)b * a.C + c) * a.H + (row_ok ? yi : 0)) * a.W;
-        float *dst = sX + ((size_t)c * tl.Rmax + r) * RP;
-        for (int rx = lane; rx < Win; rx += 32) {
-            const int xi = ix0 + rx;
-            const float v = (row_ok && xi >= 0 && xi < a.W) ? __ldg(src + xi) : 0.0f;
-            dst[(rx % st) * Ws + rx / st] = v;
-        }
-    }
-    __syncthreads();
 
     const int g = warp % tl.groups, pb = warp / tl.groups;
-    int pofs[FIRST_PX], pix[FIRST_PX];
-    bool live[FIRST_PX];
-#pragma unroll
-    for (int i = 0; i < FIRST_PX; ++i) {
-        const int p = p0 + pb * 64 + lane + 32 * i;
-        live[i] = p < pend;
-        pix[i] = live[i] ? p : p0;
-        const int yy = pix[i] / a.Wo, xx = pix[i] - yy * a.Wo;
-        pofs[i] = (yy - y_first) * st * RP + xx;
-    }
-    if (!live[0] || g * 32 >= ochan) return;
-
-    // accumulators of channel pairs (2j, 2j + 1), packed for fma.rn.f32x2
-    unsigned long long acc[FIRST_PX][16];
-#pragma unroll
-    for (int i = 0; i < FIRST_PX; ++i)
-#pragma unroll
-        for (int o = 0; o < 16; ++o) acc[i][o] = 0ull;
+    const int NWo = (a.O + 31) >> 5;
+    const int gch = min(32, ochan - g * 32);                     // live channels of this warp (may be <= 0)
+    const int ob = o0 + g * 32;
     const float *wg = sW + g * 32;
-    for (int c = 0; c < a.C; ++c) {
+    constexpr int NL = OUTB == 0 ? 1 : (OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7));
+    for (int buf = 0; t < total; t += gridDim.x, buf ^= 1) {
+        const int tn = t + (int)gridDim.x;
+        if (tn < total) {
+            load_patch(tn, buf ^ 1);
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
+        __syncthreads();                                         // patch t (and the weights) visible
+
+        const int b = t / tl.tiles;
+        const int p0 = (t - b * tl.tiles) * tl.PB;
+        const int pend = min(p0 + tl.PB, npix);
+        const int y_first = p0 / a.Wo;
+        const float *sX = sX0 + buf * patch;
+        int pofs[FIRST_PX], pix[FIRST_PX];
+        bool live[FIRST_PX];
+#pragma unroll
+        for (int i = 0; i < FIRST_PX; ++i) {
+            const int p = p0 + pb * 64 + lane + 32 * i;
+            live[i] = p < pend;
+            pix[i] = live[i] ? p : p0;
+            const int yy = pix[i] / a.Wo, xx = pix[i] - yy * a.Wo;
+            pofs[i] = (yy - y_first) * st * RP + xx;
+        }
+        if (live[0] && gch > 0) {
+            // accumulators of channel pairs (2j, 2j + 1), packed for fma.rn.f32x2
+            unsigned long long acc[FIRST_PX][16];
+#pragma unroll
+            for (int i = 0; i < FIRST_PX; ++i)
+#pragma unroll
+                for (int o = 0; o < 16; ++o) acc[i][o] = 0ull;
+            for (int c = 0; c < a.C; ++c) {
 #pragma unroll (KH ? KH : 1)
-        for (int ky = 0; ky < kh; ++ky) {
-            const float *xrow = sX + ((size_t)c * tl.Rmax + ky) * RP;
-            const float *wrow = wg + (size_t)((c * kh + ky) * kw) * OCB;
-            const float *xp[FIRST_PX];
+                for (int ky = 0; ky < kh; ++ky) {
+                    const float *xrow = sX + ((size_t)c * tl.Rmax + ky) * RP;
+                    const float *wrow = wg + (size_t)((c * kh + ky) * kw) * OCB;
+                    const float *xp[FIRST_PX];
 #pragma unroll
-            for (int i = 0; i < FIRST_PX; ++i) xp[i] = xrow + pofs[i];
+                    for (int i = 0; i < FIRST_PX; ++i) xp[i] = xrow + pofs[i];
 #pragma unroll (KW ? KW : 1)
-            for (int kx = 0; kx < kw; ++kx) {
-                // tap column kx: stride phase kx % S, offset kx / S within the phase
-                const int ph = kx % st, xo = kx / st;
-                unsigned long long xv[FIRST_PX];
+                    for (int kx = 0; kx < kw; ++kx) {
+                        // tap column kx: stride phase kx % S, offset kx / S within the phase
+                        const int ph = kx % st, xo = kx / st;
+                        unsigned long long xv[FIRST_PX];
 #pragma unroll
-                for (int i = 0; i < FIRST_PX; ++i) xv[i] = dup2((ph == 0 ? xp[i] : xp[i] + ph * Ws)[xo]);
-                const ulonglong2 *w2 = reinterpret_cast<const ulonglong2 *>(wrow + kx * OCB);
+                        for (int i = 0; i < FIRST_PX; ++i) xv[i] = dup2((ph == 0 ? xp[i] : xp[i] + ph * Ws)[xo]);
+                        const ulonglong2 *w2 = reinterpret_cast<const ulonglong2 *>(wrow + kx * OCB);
 #pragma unroll
-                for (int o4 = 0; o4 < 8; ++o4) {
-                    const ulonglong2 w = w2[o4];
+                        for (int o4 = 0; o4 < 8; ++o4) {
+                            const ulonglong2 w = w2[o4];
 #pragma unroll
-                    for (int i = 0; i < FIRST_PX; ++i) {
-                        ffma2(acc[i][2 * o4], xv[i], w.x);
-                        ffma2(acc[i][2 * o4 + 1], xv[i], w.y);
+                            for (int i = 0; i < FIRST_PX; ++i) {
+                                ffma2(acc[i][2 * o4], xv[i], w.x);
+                                ffma2(acc[i][2 * o4 + 1], xv[i], w.y);
+                            }
+                        }
                     }
                 }
             }
-        }
-    }
 
-    const long long HoWo = (long long)npix;
-    const int NWo = (a.O + 31) >> 5;
-    const int gch = min(32, ochan - g * 32);                     // live channels of this warp
-    const int ob = o0 + g * 32;
-    constexpr int NL = OUTB == 0 ? 1 : (OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7));
+            if (a.y_out) {
 #pragma unroll
-    for (int i = 0; i < FIRST_PX; ++i) {
-        if (!live[i]) continue;
-        const long long m = (long long)b * HoWo + pix[i];
-        if (a.y_out) {
+                for (int i = 0; i < FIRST_PX; ++i) {
+                    if (!live[i]) continue;
 #pragma unroll
-            for (int oc = 0; oc < 32; ++oc) {
-                if (oc < gch) {
-                    const int o = ob + oc;
-                    float y = fmaf(lane2(acc[i][oc >> 1], oc & 1), __ldg(a.scale + o), __ldg(a.shift + o));
-                    if (OUTB > 0) y = fminf(fmaxf(y, -1.0f), 1.0f);
-                    a.y_out[((long long)b * a.O + o) * HoWo + pix[i]] = y;
+                    for (int oc = 0; oc < 32; ++oc) {
+                        if (oc < gch) {
+                            const int o = ob + oc;
+                            float y = fmaf(lane2(acc[i][oc >> 1], oc & 1), __ldg(a.scale + o), __ldg(a.shift + o));
+                            if (OUTB > 0) y = fminf(fmaxf(y, -1.0f), 1.0f);
+                            a.y_out[((long long)b * a.O + o) * npix + pix[i]] = y;
+                        }
+                    }
+                }
+            }
+            if constexpr (OUTB > 0) {
+                // level masks: bit oc of M[i][u] = [sigma * acc < T_u], from the sign of
+                // fmaf(acc, sigma, -T_u); each channel's breakpoints serve both pixels
+                uint32_t M[FIRST_PX][NL - 1];
+#pragma unroll
+                for (int i = 0; i < FIRST_PX; ++i)
+#pragma unroll
+                    for (int u = 0; u < NL - 1; ++u) M[i][u] = 0u;
+#pragma unroll
+                for (int oc = 31; oc >= 0; --oc) {
+                    const float *th = sT + (g * 32 + oc) * 8;
+                    const float sg = th[NL - 1];
+#pragma unroll
+                    for (int u = 0; u < NL - 1; ++u) {
+                        const float nt = th[u];
+#pragma unroll
+                        for (int i = 0; i < FIRST_PX; ++i)
+                            M[i][u] = __funnelshift_l(__float_as_uint(fmaf(lane2(acc[i][oc >> 1], oc & 1), sg, nt)),
+                                                      M[i][u], 1);
+                    }
+                }
+#pragma unroll
+                for (int i = 0; i < FIRST_PX; ++i) {
+                    if (!live[i]) continue;
+                    const long long m = (long long)b * npix + pix[i];
+                    store_level_masks<OUTB>(M[i], gch, 32,
+                                            a.planes_out ? a.planes_out + (m * OUTB) * NWo + (ob >> 5) : nullptr, NWo,
+                                            a.codes_out ? a.codes_out + m * a.O + ob : nullptr);
                 }
             }
         }
-        if constexpr (OUTB > 0) {
-            // level masks: bit oc of M[u] = [sigma * acc < T_u], from the sign of fmaf(acc, sigma, -T_u)
-            uint32_t M[NL - 1];
-#pragma unroll
-            for (int u = 0; u < NL - 1; ++u) M[u] = 0u;
-#pragma unroll
-            for (int oc = 31; oc >= 0; --oc) {
-                const float *th = sT + (g * 32 + oc) * 8;
-                const float v = lane2(acc[i][oc >> 1], oc & 1), sg = th[NL - 1];
-#pragma unroll
-                for (int u = 0; u < NL - 1; ++u)
-                    M[u] = __funnelshift_l(__float_as_uint(fmaf(v, sg, th[u])), M[u], 1);
-            }
-            store_level_masks<OUTB>(M, gch, 32, a.planes_out ? a.planes_out + (m * OUTB) * NWo + (ob >> 5) : nullptr,
-                                    NWo, a.codes_out ? a.codes_out + m * a.O + ob : nullptr);
-        }
+        __syncthreads();                                         // buffer buf is free for tile t + 2 G
     }
 }
 
@@ -275,7 +325,13 @@ static minw_status launch_first_shape(const FirstArgs &a, const FirstTile &tl, c
             return MINW_ECUDA;
         configured = tl.smem;
     }
-    const dim3 grid((unsigned)(a.B * tl.tiles), (unsigned)((a.O + tl.OCB - 1) / tl.OCB));
+    // persistent: two CTAs per SM over all channel tiles
+    const int octiles = (a.O + tl.OCB - 1) / tl.OCB;
+    const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 152;
+    const int total = a.B * tl.tiles;
+    int gx = (2 * sms + octiles - 1) / octiles;
+    if (gx > total) gx = total;
+    const dim3 grid((unsigned)gx, (unsigned)octiles);
     kern<<<grid, FIRST_NT, tl.smem, s>>>(a, tl);
     return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
 }
