@@ -310,6 +310,17 @@ __global__ void thresholds_f32_kernel(const float *__restrict__ scale, const flo
     if (o < O) channel_thresholds_f32(scale[o], shift[o], q, out + o * 8);
 }
 
+// Breakpoints of a quantizer on its input y itself (HardTanh included): the
+// level index of y is #{u : y >= out[u]}.
+__global__ void ythresholds_kernel(QParams q, float *__restrict__ out) {
+    if (threadIdx.x == 0 && blockIdx.x == 0) channel_thresholds_f32(1.0f, 0.0f, q, out);
+}
+
+minw_status launch_ythresholds(const QParams &q, float *out, cudaStream_t s) {
+    ythresholds_kernel<<<1, 32, 0, s>>>(q, out);
+    return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
+}
+
 minw_status launch_thresholds_f32(const float *scale, const float *shift, int O, const QParams &q, float *out,
                                   cudaStream_t s) {
     thresholds_f32_kernel<<<(O + 63) / 64, 64, 0, s>>>(scale, shift, O, q, out);

@@ -69,6 +69,7 @@ struct Params {
     float res_unit;            // value of one level unit of res_codes (1 or 1/4)
     const float *res_f32;      // shortcut as fp32 NHWC [B][Hp][Wp][O] (nullable)
     float *y_nhwc;             // BN output (before the shortcut) as fp32 NHWC (nullable)
+    const float *ythr;         // breakpoints of the output quantizer on y (nullable: computed here)
     int32_t *acc_out;
     float *y_out;
     const float *scale, *shift;
@@ -431,7 +432,8 @@ __global__ void __launch_bounds__(NT, 1)
                 const float x = __ldg(p.thr + i);
                 sthr[i] = (i % NL == NL - 1) ? x : mask_breakpoint(x);
             }
-        } else {
+        } else if (p.res_codes == nullptr && p.res_f32 == nullptr) {
+            // (a residual block quantizes y + shortcut: no per-channel breakpoints on acc)
             for (int o = threadIdx.x; o < p.O; o += NT) {
                 float *t = sthr + o * NL;
                 channel_thresholds(__ldg(p.scale + o), __ldg(p.shift + o), p.qo, t);
@@ -440,10 +442,14 @@ __global__ void __launch_bounds__(NT, 1)
         }
         for (int i = p.O * NL + threadIdx.x; i < thr_floats; i += NT)        // padding channels
             sthr[i] = ((i % NL) == NL - 1) ? 1.0f : 0.0f;
-        if (threadIdx.x == 0 && (p.res_codes != nullptr || p.res_f32 != nullptr)) {
-            float t[8];
-            channel_thresholds_f32(1.0f, 0.0f, p.qo, t);            // level of y = #{u : y >= t[u]}
-            for (int u = 0; u < NL - 1; ++u) syt[u] = mask_breakpoint(t[u]);
+        if (p.res_codes != nullptr || p.res_f32 != nullptr) {       // level of y = #{u : y >= T_u}
+            if (p.ythr != nullptr) {
+                if (threadIdx.x < NL - 1) syt[threadIdx.x] = mask_breakpoint(__ldg(p.ythr + threadIdx.x));
+            } else if (threadIdx.x == 0) {
+                float t[8];
+                channel_thresholds_f32(1.0f, 0.0f, p.qo, t);         // a long serial search: callers cache it
+                for (int u = 0; u < NL - 1; ++u) syt[u] = mask_breakpoint(t[u]);
+            }
         }
         // sigma of a channel: the sign of its BN scale (+1 for 0)
         for (int g = threadIdx.x; g < sig_words; g += NT) {
@@ -1011,6 +1017,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     p.pool = a.pool; p.quant_out = a.quant_out; p.qo = a.qo;
     p.planes_out = a.planes_out; p.codes_out = a.codes_out;
     p.res_codes = a.res_codes; p.res_unit = a.res_unit; p.res_f32 = a.res_f32; p.y_nhwc = a.y_nhwc;
+    p.ythr = a.ythr;
 
     const int tiles = p.nbx * p.nby * p.nbb * p.ntn;
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;

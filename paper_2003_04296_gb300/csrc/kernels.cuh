@@ -32,6 +32,7 @@ struct ConvArgs {
     float res_unit;            // value of one level unit of res_codes
     const float *res_f32;      // shortcut as fp32 NHWC (nullable)
     float *y_nhwc;             // BN output before the shortcut, fp32 NHWC (nullable)
+    const float *ythr;         // breakpoints of the output quantizer on y [8] (nullable: computed in-kernel)
     // split-K (tensor-core path): zero-initialised workspace, left zero by every call
     void *workspace;       // nullable: no split
     size_t workspace_bytes;
@@ -58,6 +59,7 @@ struct FirstArgs {
 
 // Launchers (host).  Return MINW_OK or an error status.
 minw_status launch_conv_first(const FirstArgs &a, cudaStream_t s);
+minw_status launch_ythresholds(const QParams &q, float *out, cudaStream_t s);
 minw_status launch_first_weights(const float *w, int O, int K, int quant_w, const QParams &qw, const float *cscale,
                                  float *wt, cudaStream_t s);
 minw_status launch_thresholds_f32(const float *scale, const float *shift, int O, const QParams &q, float *out,

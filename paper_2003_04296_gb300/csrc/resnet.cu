@@ -38,9 +38,20 @@ __device__ __forceinline__ int code_to_units(uint32_t c) {
     return (c & 0x80u) ? -m : m;
 }
 
+// E4M3 level codes (0x00, +-0x38, +-0x40, +-0x48), four per word, mapped to
+// bytes whose unsigned order is the order of the levels (positive c -> c ^ 0x80,
+// negative c -> c ^ 0xFF), and back.
+__device__ __forceinline__ uint32_t codes_to_ordered(uint32_t w) {
+    return w ^ 0x80808080u ^ (((w >> 7) & 0x01010101u) * 0x7Fu);
+}
+__device__ __forceinline__ uint32_t ordered_to_codes(uint32_t o) {
+    return o ^ 0x80808080u ^ (((~o >> 7) & 0x01010101u) * 0x7Fu);
+}
+
 // 3x3 / stride 2 / pad 1 pooling of level codes [B][H][W][C] -> [B][Ho][Wo][C]:
 // per channel the max of the levels when the stem's BN scale is >= 0, the min
-// otherwise.  Thread = one output pixel x 16 channels; padded taps are skipped.
+// otherwise (padded taps skipped).  Thread = one output pixel x 16 channels;
+// the codes are compared as order-preserving bytes, four per word.
 __global__ void __launch_bounds__(256) pool_levels_kernel(const uint8_t *__restrict__ in, int B, int H, int W, int C,
                                                           const float *__restrict__ scale, uint8_t *__restrict__ out,
                                                           int Ho, int Wo) {
@@ -53,12 +64,15 @@ __global__ void __launch_bounds__(256) pool_levels_kernel(const uint8_t *__restr
         const int xo = (int)(pix % Wo);
         const int yo = (int)((pix / Wo) % Ho);
         const int b = (int)(pix / ((long long)Wo * Ho));
-        int best[16];
-        bool up[16];
+        uint32_t up[4], mx[4], mn[4];
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            up[j] = __ldg(scale + g * 16 + j) >= 0.0f;
-            best[j] = up[j] ? -8 : 8;
+        for (int q = 0; q < 4; ++q) {
+            uint32_t m = 0u;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) m |= (__ldg(scale + g * 16 + 4 * q + j) >= 0.0f ? 0xFFu : 0u) << (8 * j);
+            up[q] = m;
+            mx[q] = 0x00000000u;
+            mn[q] = 0xFFFFFFFFu;
         }
         for (int ky = 0; ky < 3; ++ky) {
             const int yi = 2 * yo - 1 + ky;
@@ -69,16 +83,17 @@ __global__ void __launch_bounds__(256) pool_levels_kernel(const uint8_t *__restr
                 const uint4 v = __ldg(reinterpret_cast<const uint4 *>(in + (((long long)b * H + yi) * W + xi) * C + g * 16));
                 const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-                for (int j = 0; j < 16; ++j) {
-                    const int u = code_to_units((w[j >> 2] >> (8 * (j & 3))) & 0xFFu);
-                    best[j] = up[j] ? max(best[j], u) : min(best[j], u);
+                for (int q = 0; q < 4; ++q) {
+                    const uint32_t o = codes_to_ordered(w[q]);
+                    mx[q] = __vmaxu4(mx[q], o);
+                    mn[q] = __vminu4(mn[q], o);
                 }
             }
         }
-        uint32_t o[4] = {0u, 0u, 0u, 0u};
+        uint32_t r[4];
 #pragma unroll
-        for (int j = 0; j < 16; ++j) o[j >> 2] |= (uint32_t)level_code_e4m3(best[j]) << (8 * (j & 3));
-        *reinterpret_cast<uint4 *>(out + pix * C + g * 16) = make_uint4(o[0], o[1], o[2], o[3]);
+        for (int q = 0; q < 4; ++q) r[q] = ordered_to_codes((mx[q] & up[q]) | (mn[q] & ~up[q]));
+        *reinterpret_cast<uint4 *>(out + pix * C + g * 16) = make_uint4(r[0], r[1], r[2], r[3]);
     }
 }
 
@@ -98,32 +113,28 @@ __global__ void __launch_bounds__(256) avgpool_levels_kernel(const uint8_t *__re
 
 // Head, second part: fp32 fully connected layer (one fmaf chain over the
 // features in order; weights transposed to [C][classes]) and BN (fmaf).
-// CTA = 8 images x 128 classes; the pooled features of its images sit in
-// shared memory.
-constexpr int HEAD_IMGS = 8, HEAD_CLS = 128;
-__global__ void __launch_bounds__(HEAD_CLS) fc_head_kernel(const float *__restrict__ pooled, int B, int C,
-                                                           const float *__restrict__ wt, int classes,
-                                                           const float *__restrict__ scale,
-                                                           const float *__restrict__ shift,
-                                                           float *__restrict__ logits) {
+// CTA = 8 images x 32 classes, one output per thread (many small chains keep
+// the SMs busy); the pooled features of its images sit in shared memory.
+constexpr int HEAD_IMGS = 8, HEAD_CLS = 32;
+__global__ void __launch_bounds__(HEAD_IMGS * HEAD_CLS) fc_head_kernel(const float *__restrict__ pooled, int B, int C,
+                                                                       const float *__restrict__ wt, int classes,
+                                                                       const float *__restrict__ scale,
+                                                                       const float *__restrict__ shift,
+                                                                       float *__restrict__ logits) {
     extern __shared__ float sp[];                    // [HEAD_IMGS][C]
-    const int b0 = blockIdx.x * HEAD_IMGS;
+    const int b0 = blockIdx.y * HEAD_IMGS;
     const int nimg = min(HEAD_IMGS, B - b0);
-    for (int i = threadIdx.x; i < HEAD_IMGS * C; i += HEAD_CLS)
+    const int tid = threadIdx.y * HEAD_CLS + threadIdx.x;
+    for (int i = tid; i < HEAD_IMGS * C; i += HEAD_IMGS * HEAD_CLS)
         sp[i] = i < nimg * C ? pooled[(long long)b0 * C + i] : 0.0f;
     __syncthreads();
-    const int o = blockIdx.y * HEAD_CLS + threadIdx.x;
-    if (o >= classes) return;
-    float acc[HEAD_IMGS];
-#pragma unroll
-    for (int im = 0; im < HEAD_IMGS; ++im) acc[im] = 0.0f;
-    for (int k = 0; k < C; ++k) {
-        const float w = __ldg(wt + (long long)k * classes + o);
-#pragma unroll
-        for (int im = 0; im < HEAD_IMGS; ++im) acc[im] = fmaf(sp[im * C + k], w, acc[im]);
-    }
-    const float sc = __ldg(scale + o), sh = __ldg(shift + o);
-    for (int im = 0; im < nimg; ++im) logits[(long long)(b0 + im) * classes + o] = fmaf(acc[im], sc, sh);
+    const int o = blockIdx.x * HEAD_CLS + threadIdx.x, im = threadIdx.y;
+    if (o >= classes || im >= nimg) return;
+    const float *x = sp + im * C;
+    float acc = 0.0f;
+#pragma unroll 8
+    for (int k = 0; k < C; ++k) acc = fmaf(x[k], __ldg(wt + (long long)k * classes + o), acc);
+    logits[(long long)(b0 + im) * classes + o] = fmaf(acc, __ldg(scale + o), __ldg(shift + o));
 }
 
 __global__ void transpose_kernel(const float *__restrict__ in, int rows, int cols, float *__restrict__ out) {
@@ -157,6 +168,7 @@ struct ResNetPlan {
     ResBlock blocks[8];
     float *fc_wt = nullptr, *fc_scale = nullptr, *fc_shift = nullptr;
     float *pooled = nullptr;               // head: average-pooled features [max_batch][512]
+    float *ythr = nullptr;                 // breakpoints of the activation quantizer on y [8]
     uint8_t *S = nullptr, *X = nullptr, *Y = nullptr, *V = nullptr;
     float *D = nullptr;
 };
@@ -217,6 +229,7 @@ static ConvArgs block_conv(const minw_net *net, const ResBlock &bk, int which, i
         a.act8 = R->V;
         a.quant_out = 1; a.qo = to_qparams(&R->qa);
         a.codes_out = Y;
+        a.ythr = R->ythr;
         if (bk.down) {
             a.res_f32 = R->D;
         } else {
@@ -356,6 +369,8 @@ extern "C" minw_status minw_resnet18_create(const minw_resnet18_desc *d, int32_t
     if ((st = alloc_owned(n, &R->V, act_codes)) != MINW_OK) return fail(st);
     if ((st = alloc_owned(n, &R->D, down_f32)) != MINW_OK) return fail(st);
     if ((st = alloc_owned(n, &R->pooled, Bm * 512)) != MINW_OK) return fail(st);
+    if ((st = alloc_owned(n, &R->ythr, 8)) != MINW_OK) return fail(st);
+    if ((st = launch_ythresholds(to_qparams(&R->qa), R->ythr, s)) != MINW_OK) return fail(st);
     if (ws) {
         uint8_t *w = nullptr;
         if ((st = alloc_owned(n, &w, ws)) != MINW_OK) return fail(st);
@@ -421,9 +436,9 @@ minw_status resnet_forward(minw_net *net, const float *x, int B, float *logits, 
         const int HW = last.Ho * last.Wo;
         avgpool_levels_kernel<<<(unsigned)((B * 512 + 255) / 256), 256, 0, s>>>(X, B, HW, 512, unit, R->pooled);
         const size_t smem = sizeof(float) * HEAD_IMGS * 512;
-        const dim3 grid((unsigned)((B + HEAD_IMGS - 1) / HEAD_IMGS), (unsigned)((R->classes + HEAD_CLS - 1) / HEAD_CLS));
-        fc_head_kernel<<<grid, HEAD_CLS, smem, s>>>(R->pooled, B, 512, R->fc_wt, R->classes, R->fc_scale, R->fc_shift,
-                                                   logits);
+        const dim3 grid((unsigned)((R->classes + HEAD_CLS - 1) / HEAD_CLS), (unsigned)((B + HEAD_IMGS - 1) / HEAD_IMGS));
+        fc_head_kernel<<<grid, dim3(HEAD_CLS, HEAD_IMGS), smem, s>>>(R->pooled, B, 512, R->fc_wt, R->classes,
+                                                                    R->fc_scale, R->fc_shift, logits);
         if (cudaGetLastError() != cudaSuccess) return MINW_ECUDA;
         if ((st = mark()) != MINW_OK) return st;
     }
