@@ -188,14 +188,10 @@ __device__ __forceinline__ uint32_t spread4(uint32_t m, int g) {
     return (((m >> (4 * g)) & 0xFu) * 0x00204081u) & 0x01010101u;
 }
 
-// Stores the planes (sign, then the non-zero mask for 2 bits or the magnitude
-// code |k - 3| for 3 bits; bits of channels >= nvalid cleared) and the E4M3
-// codes (ncodes = 16 or 32 bytes; the second 16 only when nvalid > 16) of
-// OUTB-bit levels given by their masks M[0 .. levels - 2].
+// Planes of OUTB-bit levels from their masks: sign, then the non-zero mask
+// (2 bits) or the magnitude code |k - 3| (3 bits), one bit per channel.
 template <int OUTB>
-__device__ __forceinline__ void store_level_masks(const uint32_t *M, int nvalid, int ncodes, uint32_t *planes, int NWo,
-                                                  uint8_t *codes) {
-    uint32_t P[3];
+__device__ __forceinline__ void level_planes(const uint32_t *M, uint32_t *P) {
     if constexpr (OUTB == 1) {
         P[0] = M[0];
     } else if constexpr (OUTB == 2) {
@@ -206,28 +202,42 @@ __device__ __forceinline__ void store_level_masks(const uint32_t *M, int nvalid,
         P[1] = M[0] | (M[2] & ~M[1]) | (M[4] & ~M[3]) | ~M[5];     // |k - 3| in {1, 3}
         P[2] = M[1] | ~M[4];                                        // |k - 3| in {2, 3}
     }
+}
+
+// E4M3 codes of channels 4g .. 4g + 3 (one byte each) from the planes.
+template <int OUTB>
+__device__ __forceinline__ uint32_t level_code_word(const uint32_t *P, int g) {
+    if constexpr (OUTB == 1) {
+        return (spread4(P[0], g) * 0x80u) | 0x38383838u;
+    } else if constexpr (OUTB == 2) {
+        return spread4(P[1], g) * 0x38u + spread4(P[0], g) * 0x80u;
+    } else {
+        const uint32_t c0 = P[1], c1 = P[2];
+        return spread4(c0, g) * 0x08u + spread4(c0 & ~c1, g) * 0x30u + spread4(c1, g) * 0x40u +
+               spread4(P[0] & (c0 | c1), g) * 0x80u;
+    }
+}
+
+// Stores the planes (bits of channels >= nvalid cleared) and the E4M3 codes
+// (ncodes = 16 or 32 bytes; the second 16 only when nvalid > 16) of OUTB-bit
+// levels given by their masks M[0 .. levels - 2].
+template <int OUTB>
+__device__ __forceinline__ void store_level_masks(const uint32_t *M, int nvalid, int ncodes, uint32_t *planes, int NWo,
+                                                  uint8_t *codes) {
+    uint32_t P[3];
+    level_planes<OUTB>(M, P);
     if (planes != nullptr) {
         const uint32_t vm = nvalid >= 32 ? 0xffffffffu : ((1u << nvalid) - 1u);
 #pragma unroll
         for (int u = 0; u < OUTB; ++u) planes[u * NWo] = P[u] & vm;
     }
     if (codes != nullptr) {
-        uint32_t cw[8];
-#pragma unroll
-        for (int g = 0; g < 8; ++g) {
-            if constexpr (OUTB == 1) {
-                cw[g] = (spread4(P[0], g) * 0x80u) | 0x38383838u;
-            } else if constexpr (OUTB == 2) {
-                cw[g] = spread4(P[1], g) * 0x38u + spread4(P[0], g) * 0x80u;
-            } else {
-                const uint32_t c0 = P[1], c1 = P[2];
-                cw[g] = spread4(c0, g) * 0x08u + spread4(c0 & ~c1, g) * 0x30u + spread4(c1, g) * 0x40u +
-                        spread4(P[0] & (c0 | c1), g) * 0x80u;
-            }
-        }
         uint4 *dst = reinterpret_cast<uint4 *>(codes);
-        dst[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
-        if (nvalid > 16 && ncodes > 16) dst[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
+        dst[0] = make_uint4(level_code_word<OUTB>(P, 0), level_code_word<OUTB>(P, 1), level_code_word<OUTB>(P, 2),
+                            level_code_word<OUTB>(P, 3));
+        if (nvalid > 16 && ncodes > 16)
+            dst[1] = make_uint4(level_code_word<OUTB>(P, 4), level_code_word<OUTB>(P, 5), level_code_word<OUTB>(P, 6),
+                                level_code_word<OUTB>(P, 7));
     }
 }
 

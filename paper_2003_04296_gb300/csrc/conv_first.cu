@@ -15,7 +15,7 @@ namespace minw {
 
 
 constexpr int FIRST_NT = 256;                   // 8 warps
-constexpr int FIRST_PX = 2;                     // output pixels per thread (32 apart)
+constexpr int FIRST_PX = 4;                     // output pixels per thread (16 apart)
 
 // Two fp32 lanes in one 64-bit register for the packed fma.rn.f32x2: each
 // lane is an IEEE fmaf of its own, so a chain of them is bit-identical to
@@ -80,10 +80,10 @@ __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_gr
 // rx at (rx % S) * Ws + rx / S, so that threads reading neighbouring output
 // pixels read neighbouring words for any stride): the next tile's patch
 // arrives by cp.async while the current one is computed.  Warp = 32 output
-// channels x 64 pixels; a thread holds two pixels (32 apart) x 32 channels as
-// 16 channel pairs and per tap does two patch loads, eight broadcast 128-bit
-// weight loads and 32 packed fma.rn.f32x2, one fmaf chain per output over
-// (c, ky, kx) in that order.  Zero padding: the accumulator starts at +0 and
+// channels x 64 pixels; a thread holds four pixels (16 apart) x 16 channels
+// as 8 channel pairs and per tap does four patch loads, four 128-bit weight
+// loads (one address per half warp) and 32 packed fma.rn.f32x2, one fmaf
+// chain per output over (c, ky, kx) in that order.  Zero padding: the accumulator starts at +0 and
 // a sum that rounds to zero is +0, so it is never -0 and fmaf(0, w, acc) ==
 // acc: the padded taps change nothing, exactly as skipping them.  The
 // epilogue turns each pixel's 32 channels into level masks (the sign bits of
@@ -167,11 +167,15 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
         }
     }
 
+    // warp = 32 channels x 64 pixels; lane = (channel half h, pixel l16):
+    // 4 pixels (16 apart) x 16 channels per thread
     const int g = warp % tl.groups, pb = warp / tl.groups;
+    const int h = lane >> 4, l16 = lane & 15;
     const int NWo = (a.O + 31) >> 5;
     const int gch = min(32, ochan - g * 32);                     // live channels of this warp (may be <= 0)
+    const int hch = gch - 16 * h;                                // live channels of this half (may be <= 0)
     const int ob = o0 + g * 32;
-    const float *wg = sW + g * 32;
+    const float *wg = sW + g * 32 + h * 16;
     constexpr int NL = OUTB == 0 ? 1 : (OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7));
     for (int buf = 0; t < total; t += gridDim.x, buf ^= 1) {
         const int tn = t + (int)gridDim.x;
@@ -192,19 +196,19 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
         bool live[FIRST_PX];
 #pragma unroll
         for (int i = 0; i < FIRST_PX; ++i) {
-            const int p = p0 + pb * 64 + lane + 32 * i;
+            const int p = p0 + pb * 64 + l16 + 16 * i;
             live[i] = p < pend;
             pix[i] = live[i] ? p : p0;
             const int yy = pix[i] / a.Wo, xx = pix[i] - yy * a.Wo;
             pofs[i] = (yy - y_first) * st * RP + xx;
         }
-        if (live[0] && gch > 0) {
+        if (p0 + pb * 64 < pend && gch > 0) {                   // warp-uniform: the epilogue shuffles
             // accumulators of channel pairs (2j, 2j + 1), packed for fma.rn.f32x2
-            unsigned long long acc[FIRST_PX][16];
+            unsigned long long acc[FIRST_PX][8];
 #pragma unroll
             for (int i = 0; i < FIRST_PX; ++i)
 #pragma unroll
-                for (int o = 0; o < 16; ++o) acc[i][o] = 0ull;
+                for (int o = 0; o < 8; ++o) acc[i][o] = 0ull;
             for (int c = 0; c < a.C; ++c) {
 #pragma unroll (KH ? KH : 1)
                 for (int ky = 0; ky < kh; ++ky) {
@@ -222,7 +226,7 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
                         for (int i = 0; i < FIRST_PX; ++i) xv[i] = dup2((ph == 0 ? xp[i] : xp[i] + ph * Ws)[xo]);
                         const ulonglong2 *w2 = reinterpret_cast<const ulonglong2 *>(wrow + kx * OCB);
 #pragma unroll
-                        for (int o4 = 0; o4 < 8; ++o4) {
+                        for (int o4 = 0; o4 < 4; ++o4) {
                             const ulonglong2 w = w2[o4];
 #pragma unroll
                             for (int i = 0; i < FIRST_PX; ++i) {
@@ -239,9 +243,9 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
                 for (int i = 0; i < FIRST_PX; ++i) {
                     if (!live[i]) continue;
 #pragma unroll
-                    for (int oc = 0; oc < 32; ++oc) {
-                        if (oc < gch) {
-                            const int o = ob + oc;
+                    for (int oc = 0; oc < 16; ++oc) {
+                        if (oc < hch) {
+                            const int o = ob + 16 * h + oc;
                             float y = fmaf(lane2(acc[i][oc >> 1], oc & 1), __ldg(a.scale + o), __ldg(a.shift + o));
                             if (OUTB > 0) y = fminf(fmaxf(y, -1.0f), 1.0f);
                             a.y_out[((long long)b * a.O + o) * npix + pix[i]] = y;
@@ -250,33 +254,49 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
                 }
             }
             if constexpr (OUTB > 0) {
-                // level masks: bit oc of M[i][u] = [sigma * acc < T_u], from the sign of
-                // fmaf(acc, sigma, -T_u); each channel's breakpoints serve both pixels
-                uint32_t M[FIRST_PX][NL - 1];
+                // level masks of this half's 16 channels: bit oc of M = [sigma * acc < T_u], from the
+                // sign of fmaf(acc, sigma, -T_u); then the two halves make the 32-channel word
+                const float *thb = sT + (g * 32 + 16 * h) * 8;
+                uint32_t MM[FIRST_PX][NL - 1];
 #pragma unroll
                 for (int i = 0; i < FIRST_PX; ++i)
 #pragma unroll
-                    for (int u = 0; u < NL - 1; ++u) M[i][u] = 0u;
+                    for (int u = 0; u < NL - 1; ++u) MM[i][u] = 0u;
 #pragma unroll
-                for (int oc = 31; oc >= 0; --oc) {
-                    const float *th = sT + (g * 32 + oc) * 8;
+                for (int oc = 15; oc >= 0; --oc) {
+                    const float *th = thb + oc * 8;
                     const float sg = th[NL - 1];
 #pragma unroll
                     for (int u = 0; u < NL - 1; ++u) {
                         const float nt = th[u];
 #pragma unroll
                         for (int i = 0; i < FIRST_PX; ++i)
-                            M[i][u] = __funnelshift_l(__float_as_uint(fmaf(lane2(acc[i][oc >> 1], oc & 1), sg, nt)),
-                                                      M[i][u], 1);
+                            MM[i][u] = __funnelshift_l(__float_as_uint(fmaf(lane2(acc[i][oc >> 1], oc & 1), sg, nt)),
+                                                       MM[i][u], 1);
                     }
                 }
 #pragma unroll
                 for (int i = 0; i < FIRST_PX; ++i) {
+                    uint32_t *M = MM[i];
+#pragma unroll
+                    for (int u = 0; u < NL - 1; ++u) {
+                        const uint32_t other = __shfl_xor_sync(0xffffffffu, M[u], 16);
+                        M[u] = h ? (other | (M[u] << 16)) : (M[u] | (other << 16));
+                    }
                     if (!live[i]) continue;
                     const long long m = (long long)b * npix + pix[i];
-                    store_level_masks<OUTB>(M[i], gch, 32,
-                                            a.planes_out ? a.planes_out + (m * OUTB) * NWo + (ob >> 5) : nullptr, NWo,
-                                            a.codes_out ? a.codes_out + m * a.O + ob : nullptr);
+                    uint32_t P[3];
+                    level_planes<OUTB>(M, P);
+                    if (a.planes_out != nullptr && h == 0) {
+                        const uint32_t vm = gch >= 32 ? 0xffffffffu : ((1u << gch) - 1u);
+                        uint32_t *dst = a.planes_out + (m * OUTB) * NWo + (ob >> 5);
+#pragma unroll
+                        for (int u = 0; u < OUTB; ++u) dst[u * NWo] = P[u] & vm;
+                    }
+                    if (a.codes_out != nullptr && hch > 0)
+                        *reinterpret_cast<uint4 *>(a.codes_out + m * a.O + ob + 16 * h) =
+                            make_uint4(level_code_word<OUTB>(P, 4 * h), level_code_word<OUTB>(P, 4 * h + 1),
+                                       level_code_word<OUTB>(P, 4 * h + 2), level_code_word<OUTB>(P, 4 * h + 3));
                 }
             }
         }
