@@ -54,7 +54,10 @@ struct Params {
     int B, C, H, W, O, kh, kw, pad, Ho, Wo;
     int stride;                // 1 or 2 (TMA element strides)
     int ck;                    // bytes (= channels) per K chunk: 128 (128-byte swizzle) or 64 (64-byte swizzle)
-    uint32_t a_bytes;          // activation box bytes per stage: 128 rows x ck
+    uint32_t a_bytes;          // activation box bytes of one K block: 128 rows x ck
+    uint32_t b_bytes;          // weight box bytes of one K block: BN rows x ck
+    int kps;                   // K blocks per pipeline stage (1 or 2): a stage holds kps activation
+                               // boxes, then kps weight boxes, and is released by one commit
     int bw, bh, bb, nbx, nby, nbb, ntn;
     int BN, nck, nk, S;
     uint32_t stage_bytes, idesc, tmem_cols;
@@ -476,7 +479,7 @@ __global__ void __launch_bounds__(NT, 1)
             const bool act = warp == 0;
             const CUtensorMap *map = act ? &tmA : &tmB;
             asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
-            const uint32_t bytes = act ? p.a_bytes : p.stage_bytes - p.a_bytes;   // weights: all cl slices
+            const uint32_t bytes = act ? p.a_bytes : p.b_bytes;   // per K block; weights: all cl slices
             const int bslice = p.BN / p.cl;        // weight rows this CTA loads (and multicasts)
             int g = 0, s = 0, lap = 0;             // stages issued, ring slot, ring lap
             bool alive = true;
@@ -491,23 +494,27 @@ __global__ void __launch_bounds__(NT, 1)
                 const int tap0 = kb / p.nck;
                 int c0 = (kb - tap0 * p.nck) * p.ck, ky = tap0 / p.kw, kx = tap0 - (tap0 / p.kw) * p.kw;
                 int kcol = kb * p.ck;
-                for (int ks = kb; ks < ke; ++ks, ++g) {
+                for (int ks = kb; ks < ke; ks += p.kps, ++g) {
                     // slot reuse: wait until the MMAs of the previous lap released it
                     if (lap > 0 && !mbar_wait(&empty[s], (lap - 1) & 1)) { alive = false; break; }
                     uint8_t *sa = smem + (size_t)s * p.stage_bytes;
-                    mbar_expect_tx(&full[s], bytes);
-                    if (act)
-                        tma_load_4d(sa, &tmA, &full[s], c0, x0 + kx, y0 + ky, b0);
-                    else if (p.cl == 1)
-                        tma_load_2d(sa + p.a_bytes, &tmB, &full[s], kcol, o0);
-                    else
-                        tma_load_2d_mc(sa + p.a_bytes + (size_t)crank * bslice * p.ck, &tmB, &full[s], kcol,
-                                       o0 + crank * bslice, cmask);
-                    kcol += p.ck;
-                    c0 += p.ck;
-                    if (c0 == p.C) {
-                        c0 = 0;
-                        if (++kx == p.kw) { kx = 0; ++ky; }
+                    const int n = min(p.kps, ke - ks);            // K blocks in this stage
+                    mbar_expect_tx(&full[s], (uint32_t)n * bytes);
+                    for (int j = 0; j < n; ++j) {
+                        if (act)
+                            tma_load_4d(sa + (size_t)j * p.a_bytes, &tmA, &full[s], c0, x0 + kx, y0 + ky, b0);
+                        else if (p.cl == 1)
+                            tma_load_2d(sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes, &tmB, &full[s], kcol, o0);
+                        else
+                            tma_load_2d_mc(sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes +
+                                               (size_t)crank * bslice * p.ck,
+                                           &tmB, &full[s], kcol, o0 + crank * bslice, cmask);
+                        kcol += p.ck;
+                        c0 += p.ck;
+                        if (c0 == p.C) {
+                            c0 = 0;
+                            if (++kx == p.kw) { kx = 0; ++ky; }
+                        }
                     }
                     if (++s == p.S) { s = 0; ++lap; }
                 }
@@ -532,8 +539,9 @@ __global__ void __launch_bounds__(NT, 1)
             // stage minimal (descriptors advance by a constant per ring slot,
             // the K = 32 steps are unrolled).
             const uint32_t sbase = smem_u32(smem);
-            const uint64_t adesc0 = sw_desc(sbase, p.ck), bdesc0 = sw_desc(sbase + p.a_bytes, p.ck);
+            const uint64_t adesc0 = sw_desc(sbase, p.ck), bdesc0 = sw_desc(sbase + p.kps * p.a_bytes, p.ck);
             const uint32_t dstep = p.stage_bytes >> 4;     // start-address step of one ring slot
+            const uint32_t astep = p.a_bytes >> 4, bstep = p.b_bytes >> 4;   // second K block of a stage
             const bool k128 = p.ck == 128;                 // four K = 32 steps per stage, else two
             const uint32_t idesc = p.idesc;
             for (int w = blockIdx.x; w < items && alive; w += gridDim.x, ++i) {
@@ -544,16 +552,26 @@ __global__ void __launch_bounds__(NT, 1)
                 fence_after();
                 const uint32_t tmem_d = tmem_base + (uint32_t)(ab * p.BN);
                 uint32_t acc = 0u;
-                for (int ks = kb; ks < ke; ++ks) {
+                for (int ks = kb; ks < ke; ks += p.kps) {
                     if (!mbar_wait(&full[s], fphase)) { alive = false; break; }
                     fence_after();
                     const uint64_t off = (uint64_t)((uint32_t)s * dstep);
-                    const uint64_t ad = adesc0 + off, bd = bdesc0 + off;
+                    uint64_t ad = adesc0 + off, bd = bdesc0 + off;
                     mma_f8(tmem_d, ad, bd, idesc, acc);
                     mma_f8(tmem_d, ad + 2, bd + 2, idesc, 1u);
                     if (k128) {
                         mma_f8(tmem_d, ad + 4, bd + 4, idesc, 1u);
                         mma_f8(tmem_d, ad + 6, bd + 6, idesc, 1u);
+                    }
+                    if (p.kps == 2 && ks + 1 < ke) {
+                        ad += astep;
+                        bd += bstep;
+                        mma_f8(tmem_d, ad, bd, idesc, 1u);
+                        mma_f8(tmem_d, ad + 2, bd + 2, idesc, 1u);
+                        if (k128) {
+                            mma_f8(tmem_d, ad + 4, bd + 4, idesc, 1u);
+                            mma_f8(tmem_d, ad + 6, bd + 6, idesc, 1u);
+                        }
                     }
                     acc = 1u;
                     if (p.cl == 1)
@@ -986,6 +1004,16 @@ static int cluster_pref() {
     return v;
 }
 
+// K blocks per stage the kernel may use (MINW_TC_KPS = 1 keeps one; 2 by default).
+static int kps_pref() {
+    static int v = -1;
+    if (v < 0) {
+        const char *e = getenv("MINW_TC_KPS");
+        v = (e && atoi(e) == 1) ? 1 : 2;
+    }
+    return v;
+}
+
 static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_pref()) {
     Params &p = pl.p;
     p = Params{};
@@ -1001,10 +1029,14 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     p.ntn = (a.O + p.BN - 1) / p.BN;
     p.nlev = a.quant_out ? num_levels(a.qo.bits) : 0;
     p.thr = a.thr;
-    p.stage_bytes = p.a_bytes + (uint32_t)(p.BN * p.ck);
+    p.b_bytes = (uint32_t)(p.BN * p.ck);
     const size_t o32 = ((size_t)a.O + 31) & ~(size_t)31;
     const size_t thr_bytes = a.quant_out ? (o32 * p.nlev + o32 / 32 + 10) * sizeof(float) : 0;
     const size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes;
+    // two K blocks per stage (one commit per 8 or 4 MMAs) when three such stages fit
+    const size_t blk = (size_t)p.a_bytes + p.b_bytes;
+    p.kps = (kps_pref() != 1 && p.nk >= 2 && budget / (2 * blk) >= 3) ? 2 : 1;
+    p.stage_bytes = (uint32_t)(p.kps * blk);
     int S = (int)(budget / p.stage_bytes);
     if (S > 8) S = 8;
     if (S < 2) return MINW_EUNSUPPORTED;
