@@ -293,7 +293,6 @@ def run_gpu(args, rank, world, local_rank):
     logits = torch.empty((BATCH, net.out_features), dtype=torch.float32, device=dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
-    net.enable_timing(True)
     macs, q_ops_idx = wl.op_macs()
     nl = net.launches
     assert len(macs) == nl, (len(macs), nl)
@@ -314,10 +313,19 @@ def run_gpu(args, rank, world, local_rank):
             ev0[k].record(stream)
             net.forward(x, logits)
             ev1[k].record(stream)
-            layer_ms += np.array(net.layer_times())   # waits for this step only
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
+    # per-kernel durations: the same K steps again with an event after every
+    # layer (events between kernels stop a kernel's set-up from overlapping the
+    # previous one's tail, so the timed steps above run without them)
+    net.enable_timing(True)
+    for k in range(args.steps):
+        flush.zero_()
+        net.forward(x, logits)
+        layer_ms += np.array(net.layer_times())
+    net.enable_timing(False)
+    torch.cuda.synchronize()
     for k in range(args.steps):
         step_ms.append(ev0[k].elapsed_time(ev1[k]))
     ms = sum(step_ms) / len(step_ms)
@@ -390,6 +398,8 @@ def run_gpu(args, rank, world, local_rank):
             "config": wl.config(world),
             "eff_tops": eff_tops,
             "layer_ms": [round(v, 5) for v in layer_ms.tolist()],
+            "layer_ms_note": "per-op CUDA-event durations from a second pass of the same steps with an event "
+                             "after every op; the timed steps run without them",
             "roofline": roofline, "cpu_baseline": cpu,
             "e2e": {"value": BATCH * world / e2e_sec, "unit": "images/s",
                     "h2d_bytes_per_step": int(x_host.numel() * 4),
@@ -402,7 +412,7 @@ def run_gpu(args, rank, world, local_rank):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["minw", "reference"], default="minw")
     ap.add_argument("--workload", choices=["cifar_convnet", "resnet18"], default="cifar_convnet")

@@ -4,6 +4,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "../../include/minw.h"
 
 #if defined(__CUDA_ARCH__) && (__CUDA_ARCH__ != 1030)
@@ -241,6 +243,15 @@ __device__ __forceinline__ void store_level_masks(const uint32_t *M, int nvalid,
     }
 }
 
+// Programmatic dependent launch: the kernels of a forward are launched so
+// that the next one may start (its set-up: barriers, TMEM, breakpoints,
+// weights) while the previous one finishes.  Each waits here before it reads
+// what an earlier kernel wrote or writes what an earlier kernel reads, and
+// lets its own dependents launch once its CTAs run.  Both are no-ops when
+// the launch did not ask for it.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
+
 // A breakpoint held for the mask test: -T, with -0 replaced by +0, so that
 // fmaf(acc, sigma, -T) is never -0 and its sign bit is exactly [sigma * acc < T].
 __host__ __device__ __forceinline__ float mask_breakpoint(float T) { return T == 0.0f ? 0.0f : -T; }
@@ -254,5 +265,24 @@ bool aligned16(const void *p);
 bool valid_quant(const minw_quant *q);
 int num_sms();
 minw_status launch_status();
+bool pdl_enabled();                 // MINW_PDL=0 turns programmatic dependent launch off
+
+// Kernel launch on stream s that may overlap the previous kernel in the
+// stream (programmatic stream serialization); the kernel calls pdl_wait()
+// before its dependent accesses.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl_enabled() ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
 
 }  // namespace minw_host

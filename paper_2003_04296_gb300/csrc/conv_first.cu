@@ -131,7 +131,6 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
     };
 
     int t = blockIdx.x;
-    if (t < total) load_patch(t, 0);
 
     // weights: prepared [K][O] levels (coalesced), else the latent [O][K] array
     const int osh = OCB == 64 ? 6 : 5;
@@ -169,6 +168,9 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
 
     // warp = 32 channels x 64 pixels; lane = (channel half h, pixel l16):
     // 4 pixels (16 apart) x 16 channels per thread
+    pdl_trigger();                                               // set-up done
+    pdl_wait();                                                  // the image and the output buffer are shared
+    if (t < total) load_patch(t, 0);
     const int g = warp % tl.groups, pb = warp / tl.groups;
     const int h = lane >> 4, l16 = lane & 15;
     const int NWo = (a.O + 31) >> 5;
@@ -363,8 +365,8 @@ static minw_status launch_first_shape(const FirstArgs &a, const FirstTile &tl, c
     int gx = (2 * sms + octiles - 1) / octiles;
     if (gx > total) gx = total;
     const dim3 grid((unsigned)gx, (unsigned)octiles);
-    kern<<<grid, FIRST_NT, tl.smem, s>>>(a, tl);
-    return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
+    if (minw_host::launch_pdl(kern, grid, dim3(FIRST_NT), tl.smem, s, a, tl) != cudaSuccess) return MINW_ECUDA;
+    return MINW_OK;
 }
 
 template <int OUTB>

@@ -472,11 +472,13 @@ __global__ void __launch_bounds__(NT, 1)
     if (p.cl > 1) cluster_sync_all();         // every barrier of the cluster is initialised
     fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    pdl_trigger();                            // set-up done: the next kernel may start its own
 
     if (warp == 0 || warp == B_WARP) {
         if (lane == 0) {
             // ---------------- TMA producers: warp 0 activations, warp 6 weights ----------------
             const bool act = warp == 0;
+            if (act) pdl_wait();                  // activations come from the previous kernel
             const CUtensorMap *map = act ? &tmA : &tmB;
             asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
             const uint32_t bytes = act ? p.a_bytes : p.b_bytes;   // per K block; weights: all cl slices
@@ -585,6 +587,7 @@ __global__ void __launch_bounds__(NT, 1)
         }
     } else if (warp < B_WARP) {
         // ---------------- epilogue: warps 2..9 ----------------
+        pdl_wait();                               // outputs, shortcuts and partial sums are shared with other kernels
         const int q = warp & 3;                   // TMEM lane quarter of this warp
         const int half_cols = (warp - 2) >> 2;    // which half of the accumulator columns
         const int r = q * 32 + lane;              // tile row = output pixel
@@ -825,6 +828,8 @@ __global__ void __launch_bounds__(NT, 1)
 // partial-sum loads coalesce and plane words assemble with shuffles.
 template <int OUTB>
 __global__ void __launch_bounds__(256) splitk_reduce_kernel(const Params p, const float *__restrict__ thr) {
+    pdl_wait();
+    pdl_trigger();
     constexpr int NL = OUTB == 0 ? 1 : (OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7));
     const int tiles_m = p.nbx * p.nby * p.nbb;
     const int tiles = tiles_m * p.ntn;
@@ -1222,24 +1227,27 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
         pm.y_out = nullptr;
     }
     if (pm.cl == 1) {
-        kern<<<pl.grid, tc::NT, pl.smem, s>>>(pl.tmA, pl.tmB, pm);
+        if (minw_host::launch_pdl(kern, pl.grid, dim3(tc::NT), pl.smem, s, pl.tmA, pl.tmB, pm) != cudaSuccess) return MINW_ECUDA;
     } else {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = pl.grid;
         cfg.blockDim = dim3(tc::NT);
         cfg.dynamicSmemBytes = pl.smem;
         cfg.stream = s;
-        cudaLaunchAttribute attr[1];
+        cudaLaunchAttribute attr[2];
         attr[0].id = cudaLaunchAttributeClusterDimension;
         attr[0].val.clusterDim.x = (unsigned)pm.cl;
         attr[0].val.clusterDim.y = 1;
         attr[0].val.clusterDim.z = 1;
+        attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[1].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
         // a persistent grid: no more clusters than can be resident at once
         const int maxc = tc::max_active_clusters(reinterpret_cast<const void *>(kern), pm.cl, pl.smem, cfg);
         if (maxc < 1) return MINW_EUNSUPPORTED;
         if ((int)cfg.gridDim.x > maxc * pm.cl) cfg.gridDim.x = (unsigned)(maxc * pm.cl);
+        cfg.numAttrs = minw_host::pdl_enabled() ? 2 : 1;
         if (cudaLaunchKernelEx(&cfg, kern, pl.tmA, pl.tmB, pm) != cudaSuccess) return MINW_ECUDA;
     }
     if (split) {
@@ -1247,10 +1255,10 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
         const long long threads = (long long)tiles_m * 128 * ((a.O + 31) / 32) * 8;
         const unsigned blocks = (unsigned)((threads + 255) / 256);
         switch (outb) {
-            case 1: tc::splitk_reduce_kernel<1><<<blocks, 256, 0, s>>>(pl.p, thr); break;
-            case 2: tc::splitk_reduce_kernel<2><<<blocks, 256, 0, s>>>(pl.p, thr); break;
-            case 3: tc::splitk_reduce_kernel<3><<<blocks, 256, 0, s>>>(pl.p, thr); break;
-            default: tc::splitk_reduce_kernel<0><<<blocks, 256, 0, s>>>(pl.p, thr); break;
+            case 1: minw_host::launch_pdl(tc::splitk_reduce_kernel<1>, dim3(blocks), dim3(256), 0, s, pl.p, thr); break;
+            case 2: minw_host::launch_pdl(tc::splitk_reduce_kernel<2>, dim3(blocks), dim3(256), 0, s, pl.p, thr); break;
+            case 3: minw_host::launch_pdl(tc::splitk_reduce_kernel<3>, dim3(blocks), dim3(256), 0, s, pl.p, thr); break;
+            default: minw_host::launch_pdl(tc::splitk_reduce_kernel<0>, dim3(blocks), dim3(256), 0, s, pl.p, thr); break;
         }
     }
     return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;

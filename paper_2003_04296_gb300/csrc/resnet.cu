@@ -55,6 +55,8 @@ __device__ __forceinline__ uint32_t ordered_to_codes(uint32_t o) {
 __global__ void __launch_bounds__(256) pool_levels_kernel(const uint8_t *__restrict__ in, int B, int H, int W, int C,
                                                           const float *__restrict__ scale, uint8_t *__restrict__ out,
                                                           int Ho, int Wo) {
+    pdl_wait();
+    pdl_trigger();
     const int groups = C >> 4;
     const long long total = (long long)B * Ho * Wo * groups;
     for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < total;
@@ -102,6 +104,8 @@ __global__ void __launch_bounds__(256) pool_levels_kernel(const uint8_t *__restr
 // then one division.
 __global__ void __launch_bounds__(256) avgpool_levels_kernel(const uint8_t *__restrict__ X, int B, int HW, int C,
                                                              float unit, float *__restrict__ pooled) {
+    pdl_wait();
+    pdl_trigger();
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= B * C) return;
     const int b = i / C, c = i - b * C;
@@ -122,6 +126,8 @@ __global__ void __launch_bounds__(HEAD_IMGS * HEAD_CLS) fc_head_kernel(const flo
                                                                        const float *__restrict__ shift,
                                                                        float *__restrict__ logits) {
     extern __shared__ float sp[];                    // [HEAD_IMGS][C]
+    pdl_wait();
+    pdl_trigger();
     const int b0 = blockIdx.y * HEAD_IMGS;
     const int nimg = min(HEAD_IMGS, B - b0);
     const int tid = threadIdx.y * HEAD_CLS + threadIdx.x;
@@ -416,7 +422,8 @@ minw_status resnet_forward(minw_net *net, const float *x, int B, float *logits, 
         const int sms = num_sms() > 0 ? num_sms() : 152;
         long long g = (items + 255) / 256;
         if (g > sms * 8LL) g = sms * 8LL;
-        pool_levels_kernel<<<(unsigned)g, 256, 0, s>>>(R->S, B, R->Hs, R->Hs, 64, R->stem_scale, R->X, R->Hp, R->Hp);
+        launch_pdl(pool_levels_kernel, dim3((unsigned)g), dim3(256), 0, s, (const uint8_t *)R->S, B, R->Hs, R->Hs, 64,
+                   (const float *)R->stem_scale, R->X, R->Hp, R->Hp);
         if (cudaGetLastError() != cudaSuccess) return MINW_ECUDA;
         if ((st = mark()) != MINW_OK) return st;
     }
@@ -434,11 +441,12 @@ minw_status resnet_forward(minw_net *net, const float *x, int B, float *logits, 
     {
         const ResConv &last = R->blocks[7].c2;
         const int HW = last.Ho * last.Wo;
-        avgpool_levels_kernel<<<(unsigned)((B * 512 + 255) / 256), 256, 0, s>>>(X, B, HW, 512, unit, R->pooled);
+        launch_pdl(avgpool_levels_kernel, dim3((unsigned)((B * 512 + 255) / 256)), dim3(256), 0, s, (const uint8_t *)X,
+                   B, HW, 512, unit, R->pooled);
         const size_t smem = sizeof(float) * HEAD_IMGS * 512;
         const dim3 grid((unsigned)((R->classes + HEAD_CLS - 1) / HEAD_CLS), (unsigned)((B + HEAD_IMGS - 1) / HEAD_IMGS));
-        fc_head_kernel<<<grid, dim3(HEAD_CLS, HEAD_IMGS), smem, s>>>(R->pooled, B, 512, R->fc_wt, R->classes,
-                                                                    R->fc_scale, R->fc_shift, logits);
+        launch_pdl(fc_head_kernel, grid, dim3(HEAD_CLS, HEAD_IMGS), smem, s, (const float *)R->pooled, B, 512,
+                   (const float *)R->fc_wt, R->classes, (const float *)R->fc_scale, (const float *)R->fc_shift, logits);
         if (cudaGetLastError() != cudaSuccess) return MINW_ECUDA;
         if ((st = mark()) != MINW_OK) return st;
     }
