@@ -412,7 +412,8 @@ def run_gpu(args, rank, world, local_rank):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed steps (default 1000 for the ConvNet, 100 for ResNet-18: about a second)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["minw", "reference"], default="minw")
     ap.add_argument("--workload", choices=["cifar_convnet", "resnet18"], default="cifar_convnet")
@@ -424,6 +425,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--skip-cpu", action="store_true")
     args = ap.parse_args()
+    if args.steps is None:
+        args.steps = 1000 if args.workload == "cifar_convnet" else 100
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
