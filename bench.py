@@ -237,9 +237,40 @@ def oracle_images_per_s(wl, x, max_seconds):
     return done / dt, done, dt
 
 
+def run_reference_sweep(args):
+    """The oracle on the sweep: one image per step through the fp64 level
+    convolution, cycling through the nine bit-width pairs."""
+    from oracle import oracle as Or
+    from paper_2003_04296_gb300.inputs import DEFAULT_THR
+    p = sweep_problem()
+    mac_img = 14 * 14 * 512 * 512 * 9
+    times = []
+    for k in range(args.warmup + args.steps):
+        ba, bw = SWEEP_PAIRS[k % len(SWEEP_PAIRS)]
+        a_lv = Or.quantize(p["x"][k % 256:k % 256 + 1], ba, DEFAULT_THR[ba])
+        w_lv = Or.quantize(p["w"], bw, DEFAULT_THR[bw], p["w_scale"])
+        t0 = time.perf_counter()
+        Or.conv2d_levels(a_lv, w_lv, 1, 1, ba, bw)
+        if k >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    sec = sum(times) / len(times)
+    tops = 2.0 * mac_img / sec / 1e12
+    sample = "one image per step (of 256) through the fp64 oracle convolution, the nine pairs in turn"
+    line = {"metric": METRIC, "value": tops, "unit": "effective TOPS (2 x MAC / s)", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
+            "impl": "reference", "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": sweep_config(args.gpus),
+            "cpu_baseline": {"value": tops, "unit": "effective TOPS", "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": tops, "unit": "effective TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_reference(args, rank):
     if rank != 0:
         return 0
+    if args.workload == "sweep":
+        return run_reference_sweep(args)
     wl = Workload(args.workload, args)
     x = wl.images(0)
     B = wl.batch
@@ -409,6 +440,166 @@ def run_gpu(args, rank, world, local_rank):
     return 0
 
 
+# ------------------------------------------------------------------ sweep --
+
+SWEEP_PAIRS = [(a, w) for a in (1, 2, 3) for w in (1, 2, 3)]
+
+
+def sweep_problem():
+    from paper_2003_04296_gb300.inputs import conv_problem
+    return conv_problem(5, 256, 512, 14, 14, 512, 3, 3, 1, 1, 1, 1, x_dist="normal", w_sigma=1.0)
+
+
+def sweep_config(n_gpus):
+    return {"workload": "conv3x3_bitwidth_sweep_256x512x14x14_to512", "batch_per_gpu": 256,
+            "global_batch": 256 * n_gpus, "input": "256x512x14x14 fp32 N(0,1), weights 512x512x3x3 N(0,1)",
+            "pairs": "(bits_a, bits_w) in {1,2,3}^2, each a 3x3/1/1 convolution to int32 accumulators",
+            "aqe": "AQE forward (alpha 0.75) and backward on the same 25.7M-element tensor",
+            "parallelism": f"replicas x{n_gpus} (batch-sharded, no collective)", "l2": L2_NOTE}
+
+
+def run_sweep(args, rank, world, local_rank):
+    """One step: quantize the input to level codes and convolve it with the
+    weight codes for each of the nine bit-width pairs (int32 accumulators),
+    then the AQE forward and backward on the same tensor."""
+    import torch
+    import torch.distributed as dist
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    import __graft_entry__ as g
+    if rank == 0:
+        g.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2003_04296_gb300 import minw
+    from paper_2003_04296_gb300.inputs import DEFAULT_THR, aqe_problem
+    p = sweep_problem()
+    B, C, H, W, O = 256, 512, 14, 14, 512
+    x = torch.from_numpy(p["x"]).to(dev)
+    w = torch.from_numpy(p["w"]).to(dev)
+    ws = torch.from_numpy(p["w_scale"]).to(dev)
+    g_np = aqe_problem(55, x.numel())["g"]
+    gy = torch.from_numpy(g_np).to(dev)
+    a8 = {b: torch.empty((B, H, W, C), dtype=torch.uint8, device=dev) for b in (1, 2, 3)}
+    w8 = {b: torch.empty((O, 3, 3, C), dtype=torch.uint8, device=dev) for b in (1, 2, 3)}
+    for b in (1, 2, 3):
+        minw.minw_pack_weight_codes(w, minw.quant(b, DEFAULT_THR[b]), w8[b], channel_scale=ws)
+    acc = torch.empty((B, O, H, W), dtype=torch.int32, device=dev)
+    y = torch.empty_like(x)
+    gx = torch.empty_like(x)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(ev=None):
+        for b in (1, 2, 3):
+            minw.aqe_quantize_codes(x, minw.quant(b, DEFAULT_THR[b]), a8[b])
+        for i, (ba, bw) in enumerate(SWEEP_PAIRS):
+            if ev is not None:
+                ev[i][0].record(stream)
+            minw.minw_conv2d_codes(a8[ba], B, C, H, W, ba, w8[bw], O, 3, 3, bw, 1, 1, acc_out=acc)
+            if ev is not None:
+                ev[i][1].record(stream)
+        if ev is not None:
+            ev[9][0].record(stream)
+        minw.aqe_forward(x, y, 0.75, minw.quant(2, DEFAULT_THR[2]))
+        if ev is not None:
+            ev[9][1].record(stream)
+        minw.aqe_backward(x, gy, gx, 0.75)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    e0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    e1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clk:
+        for k in range(args.steps):
+            flush.zero_()
+            e0[k].record(stream)
+            step()
+            e1[k].record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+    ms = sum(e0[k].elapsed_time(e1[k]) for k in range(args.steps)) / args.steps
+    t = torch.tensor([ms], device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_max = float(t.item())
+    # per-kernel durations: the same steps again with events around the convolutions and the AQE forward
+    conv_ms = np.zeros(len(SWEEP_PAIRS))
+    aqe_ms = 0.0
+    for k in range(args.steps):
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
+        flush.zero_()
+        step(ev)
+        torch.cuda.synchronize()
+        conv_ms += np.array([ev[i][0].elapsed_time(ev[i][1]) for i in range(9)])
+        aqe_ms += ev[9][0].elapsed_time(ev[9][1])
+    conv_ms /= args.steps
+    aqe_ms /= args.steps
+
+    # end to end: the fp32 input from pinned host memory, the step, the last accumulators back to the host
+    x_host = torch.from_numpy(p["x"]).pin_memory()
+    acc_host = torch.empty(acc.shape, dtype=torch.int32).pin_memory()
+    e2e_steps = min(args.steps, 20)
+    e2e_s = []
+    for k in range(e2e_steps + 1):
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        x.copy_(x_host, non_blocking=True)
+        step()
+        acc_host.copy_(acc, non_blocking=True)
+        torch.cuda.synchronize()
+        if k:
+            e2e_s.append(time.perf_counter() - t0)
+    e2e_sec = sum(e2e_s) / len(e2e_s)
+    if rank != 0:
+        return 0
+
+    mac = B * H * W * O * C * 9
+    value = 2.0 * mac * len(SWEEP_PAIRS) * world / (ms_max * 1e-3) / 1e12
+    achieved = 2.0 * mac * len(SWEEP_PAIRS) / (conv_ms.sum() * 1e-3) / 1e12
+    roofline = {"bound": "tensor", "kernel": "conv_tc_kernel (tcgen05 kind::f8f6f4, 9 bit-width pairs)",
+                "achieved": achieved, "peak": FP8_TFLOPS, "unit": "TFLOP/s", "frac": achieved / FP8_TFLOPS,
+                "traffic": None,
+                "peak_basis": f"measured dense bf16 {BF16_TFLOPS:.1f} TFLOP/s (burst) x 2 for FP8 "
+                              "(nominal fp8/bf16 ratio), of measured"}
+    aqe_bytes = 8.0 * x.numel()
+    aqe_roof = {"bound": "hbm", "kernel": "aqe_forward_kernel", "achieved": aqe_bytes / (aqe_ms * 1e-3) / 1e9,
+                "peak": HBM_GBS, "unit": "GB/s", "frac": aqe_bytes / (aqe_ms * 1e-3) / 1e9 / HBM_GBS,
+                "algorithmic_bytes": aqe_bytes, "peak_basis": "measured copy bandwidth, of measured"}
+    cpu = None
+    if world == 1 and not args.skip_cpu:
+        from oracle import oracle as Or
+        xs = p["x"][:1]
+        a_lv = Or.quantize(xs, 1, DEFAULT_THR[1])
+        w_lv = Or.quantize(p["w"], 1, DEFAULT_THR[1], p["w_scale"])
+        t0 = time.perf_counter()
+        n = 0
+        while True:
+            Or.conv2d_levels(a_lv, w_lv, 1, 1, 1, 1)
+            n += 1
+            if time.perf_counter() - t0 > args.cpu_seconds / 2:
+                break
+        dt = time.perf_counter() - t0
+        cpu = {"value": 2.0 * (mac / B) * n / dt / 1e12, "unit": "effective TOPS", "cores": 1, "kind": "oracle",
+               "sample": f"{n} single-image 1-bit x 1-bit convolutions (fp64 oracle, {dt:.1f} s)"}
+    line = {"metric": METRIC, "value": value, "unit": "effective TOPS (2 x MAC / s)", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "e4m3", "data": "synthetic", "config": sweep_config(world),
+            "conv_ms": [round(v, 5) for v in conv_ms.tolist()], "aqe_forward_ms": round(aqe_ms, 5),
+            "roofline": roofline, "aqe_roofline": aqe_roof, "cpu_baseline": cpu,
+            "e2e": {"value": 2.0 * mac * len(SWEEP_PAIRS) * world / e2e_sec / 1e12, "unit": "effective TOPS",
+                    "h2d_bytes_per_step": int(x_host.numel() * 4), "d2h_bytes_per_step": int(acc_host.numel() * 4)},
+            "gpu_launches": 14 * args.steps, "clocks": clk.summary()}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -416,7 +607,7 @@ def main():
                     help="timed steps (default 1000 for the ConvNet, 100 for ResNet-18: about a second)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["minw", "reference"], default="minw")
-    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18"], default="cifar_convnet")
+    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "sweep"], default="cifar_convnet")
     ap.add_argument("--bits-a", type=int, default=1, help="CIFAR ConvNet activation bits")
     ap.add_argument("--bits-w", type=int, default=1, help="CIFAR ConvNet weight bits")
     ap.add_argument("--bits-a-resnet", type=int, default=3)
@@ -426,7 +617,7 @@ def main():
     ap.add_argument("--skip-cpu", action="store_true")
     args = ap.parse_args()
     if args.steps is None:
-        args.steps = 1000 if args.workload == "cifar_convnet" else 100
+        args.steps = {"cifar_convnet": 1000, "resnet18": 100, "sweep": 20}[args.workload]
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -439,6 +630,8 @@ def main():
         torch.cuda.set_device(local_rank)
         dist.init_process_group("nccl")
     try:
+        if args.workload == "sweep":
+            return run_sweep(args, rank, world, local_rank)
         return run_gpu(args, rank, world, local_rank)
     finally:
         if world > 1:
