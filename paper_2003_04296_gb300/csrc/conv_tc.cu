@@ -56,6 +56,9 @@ struct Params {
     int ck;                    // bytes (= channels) per K chunk: 128 (128-byte swizzle) or 64 (64-byte swizzle)
     uint32_t a_bytes;          // activation box bytes of one K block: 128 rows x ck
     uint32_t b_bytes;          // weight box bytes of one K block: BN rows x ck
+    int trans;                 // 1: tile = 128 output channels (MMA M) x 256 pixels (MMA N)
+    int mrows;                 // output pixels per tile: 128, or 256 when trans
+    int acc_cols;              // TMEM columns of one accumulator: BN, or 256 when trans
     int kps;                   // K blocks per pipeline stage (1 or 2): a stage holds kps activation
                                // boxes, then kps weight boxes, and is released by one commit
     int bw, bh, bb, nbx, nby, nbb, ntn;
@@ -243,6 +246,20 @@ __device__ __forceinline__ uint32_t planes_k(int k) {
     if constexpr (OUTB == 1) return k ? 0u : 1u;
     else if constexpr (OUTB == 2) return (0x203u >> (4 * k)) & 0x3u;
     else return (uint32_t)((06420357ull >> (3 * k)) & 7ull);
+}
+
+// 32 x 32 bit transpose across a warp: lane l holds row l; on return lane j
+// holds column j (bit c of lane j's word = bit j of lane c's word).
+__device__ __forceinline__ uint32_t transpose32(uint32_t a, int lane) {
+    const uint32_t ms[5] = {0xFFFF0000u, 0xFF00FF00u, 0xF0F0F0F0u, 0xCCCCCCCCu, 0xAAAAAAAAu};
+#pragma unroll
+    for (int k = 0; k < 5; ++k) {
+        const int j = 16 >> k;
+        const uint32_t m = ms[k];
+        const uint32_t q = __shfl_xor_sync(0xffffffffu, a, j);
+        a = (lane & j) ? (((q >> j) & ~m) | (a & m)) : ((a & ~m) | ((q << j) & m));
+    }
+    return a;
 }
 
 // Epilogue of one 32-column chunk (16 when tail16 is false) of exact
@@ -552,13 +569,19 @@ __global__ void __launch_bounds__(NT, 1)
                 const int kb = (int)((long long)kp * p.nk / p.ksplit), ke = (int)((long long)(kp + 1) * p.nk / p.ksplit);
                 if (use > 0 && !mbar_wait(&tempty[ab], (use - 1) & 1)) break;
                 fence_after();
-                const uint32_t tmem_d = tmem_base + (uint32_t)(ab * p.BN);
+                const uint32_t tmem_d = tmem_base + (uint32_t)(ab * p.acc_cols);
                 uint32_t acc = 0u;
                 for (int ks = kb; ks < ke; ks += p.kps) {
                     if (!mbar_wait(&full[s], fphase)) { alive = false; break; }
                     fence_after();
                     const uint64_t off = (uint64_t)((uint32_t)s * dstep);
                     uint64_t ad = adesc0 + off, bd = bdesc0 + off;
+                    if (p.trans) {            // weights are the MMA's A operand (M = channels)
+                        const uint64_t t_ = ad;
+                        ad = bd;
+                        bd = t_;
+                    }
+                    const uint32_t as_ = p.trans ? bstep : astep, bs_ = p.trans ? astep : bstep;
                     mma_f8(tmem_d, ad, bd, idesc, acc);
                     mma_f8(tmem_d, ad + 2, bd + 2, idesc, 1u);
                     if (k128) {
@@ -566,8 +589,8 @@ __global__ void __launch_bounds__(NT, 1)
                         mma_f8(tmem_d, ad + 6, bd + 6, idesc, 1u);
                     }
                     if (p.kps == 2 && ks + 1 < ke) {
-                        ad += astep;
-                        bd += bstep;
+                        ad += as_;
+                        bd += bs_;
                         mma_f8(tmem_d, ad, bd, idesc, 1u);
                         mma_f8(tmem_d, ad + 2, bd + 2, idesc, 1u);
                         if (k128) {
@@ -610,7 +633,69 @@ __global__ void __launch_bounds__(NT, 1)
         const int cbeg = half_cols ? cmid : 0, cend = half_cols ? nch : cmid;
         int i = 0;
         bool dead = false;           // a bounded wait ran out: skip work, keep the barrier sequence
-        for (int w = blockIdx.x; w < items; w += gridDim.x, ++i) {
+        if constexpr (OUTB > 0) {
+            if (p.trans) {
+                // tile = 128 channels (TMEM lanes) x 256 pixels (columns): this warp holds
+                // channels 32 q + lane of pixel columns [128 half, 128 half + 128)
+                const int oq = 32 * q;
+                for (int w = blockIdx.x; w < items; w += gridDim.x, ++i) {
+                    const int ab = i & 1, use = i >> 1;
+                    const int tn = w / tiles_m, tm = w - tn * tiles_m;
+                    const int xb = tm % p.nbx, yb = (tm / p.nbx) % p.nby, bbk = tm / (p.nbx * p.nby);
+                    const int oc = tn * p.BN + oq + lane;          // this lane's channel
+                    float nt[NL - 1], sg;
+#pragma unroll
+                    for (int u = 0; u < NL - 1; ++u) nt[u] = sthr[oc * NL + u];
+                    sg = sthr[oc * NL + NL - 1];
+                    const uint32_t sig = ssig[(tn * p.BN + oq) >> 5];
+                    if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
+                    fence_after();
+                    for (int c = 4 * half_cols; c < 4 * half_cols + 4 && !dead; ++c) {
+                        __syncwarp();
+                        uint32_t v[32];
+                        tmem_ld32(tmem_base + ((uint32_t)oq << 16) + (uint32_t)(ab * p.acc_cols + c * 32), v);
+                        uint32_t M[NL - 1];
+#pragma unroll
+                        for (int u = 0; u < NL - 1; ++u) {
+                            uint32_t wd = 0u;          // bit j: [sigma * acc < T_u] at pixel column 32 c + j
+#pragma unroll
+                            for (int j = 31; j >= 0; --j)
+                                wd = __funnelshift_l(__float_as_uint(fmaf(__uint_as_float(v[j]), sg, nt[u])), wd, 1);
+                            M[u] = transpose32(wd, lane);     // lane j: bit k = channel oq + k at column 32 c + j
+                        }
+                        if (p.pool) {
+#pragma unroll
+                            for (int u = 0; u < NL - 1; ++u) {
+                                const uint32_t m = M[u];
+                                const uint32_t n1 = __shfl_xor_sync(0xffffffffu, m, 1);
+                                const uint32_t a1 = m & n1, o1 = m | n1;
+                                const uint32_t a2 = a1 & __shfl_xor_sync(0xffffffffu, a1, p.bw);
+                                const uint32_t o2 = o1 | __shfl_xor_sync(0xffffffffu, o1, p.bw);
+                                M[u] = (sig & a2) | (~sig & o2);
+                            }
+                        }
+                        const int r = c * 32 + lane;                    // tile row (pixel) of this lane
+                        const int b = bbk * p.bb + r / (p.bh * p.bw);
+                        const int y = yb * p.bh + (r / p.bw) % p.bh;
+                        const int x = xb * p.bw + r % p.bw;
+                        const bool valid = b < p.B && y < p.Ho && x < p.Wo;
+                        const bool writer = valid && (!p.pool || ((x & 1) == 0 && (y & 1) == 0));
+                        if (writer) {
+                            const int yp = p.pool ? y / 2 : y, xp = p.pool ? x / 2 : x;
+                            const long long opix = ((long long)b * Hp + yp) * Wp + xp;
+                            const int ob = tn * p.BN + oq;
+                            store_level_masks<OUTB>(M, 32, 32,
+                                                    p.planes_out ? p.planes_out + (opix * OUTB) * NWo + (ob >> 5) : nullptr,
+                                                    NWo, p.codes_out ? p.codes_out + opix * p.O + ob : nullptr);
+                        }
+                    }
+                    fence_before();
+                    __syncwarp();
+                    if (lane == 0 && !dead) mbar_arrive(&tempty[ab]);
+                }
+            }
+        }
+        for (int w = blockIdx.x; w < items && !p.trans; w += gridDim.x, ++i) {
             const int ab = i & 1, use = i >> 1;
             const int t = w / p.ksplit, kp = w - t * p.ksplit;
             const int tn = t / tiles_m, tm = t - tn * tiles_m;
@@ -966,14 +1051,15 @@ struct Plan {
     float *thr_ws;      // split-K: breakpoints computed into the workspace (nullable)
 };
 
-static bool plan_shape(const ConvArgs &a, Params &p) {
+static bool plan_shape(const ConvArgs &a, Params &p, int rows = 128) {
     if ((a.stride != 1 && a.stride != 2) || a.C % 64 != 0 || a.pad >= a.kh || a.pad >= a.kw) return false;
     int bw = pow2_ceil(a.Wo);
+    if (bw > rows) bw = rows;
     if (bw > 128) bw = 128;
     if (a.pool && bw > 16) bw = 16;
     int bh = pow2_ceil(a.Ho);
-    if (bh > 128 / bw) bh = 128 / bw;
-    const int bb = 128 / (bw * bh);
+    if (bh > rows / bw) bh = rows / bw;
+    const int bb = rows / (bw * bh);
     if (a.pool && (bw < 2 || bh < 2)) return false;
     p.bw = bw; p.bh = bh; p.bb = bb;
     p.nbx = (a.Wo + bw - 1) / bw;
@@ -1019,15 +1105,45 @@ static int kps_pref() {
     return v;
 }
 
+// Channel-major tiles (MINW_TC_TRANS=0 turns them off): a 128-channel layer
+// whose only output is the next layer's levels runs as 128 channels x 256
+// pixels, so each MMA has N = 256 (the tensor pipe's full rate).
+static int trans_pref() {
+    static int v = -1;
+    if (v < 0) {
+        const char *e = getenv("MINW_TC_TRANS");
+        v = (e && e[0] == '0') ? 0 : 1;
+    }
+    return v;
+}
+
+static bool trans_eligible(const ConvArgs &a) {
+    return trans_pref() && a.O == 128 && a.quant_out && (a.codes_out != nullptr || a.planes_out != nullptr) &&
+           a.acc_out == nullptr && a.y_out == nullptr && a.res_codes == nullptr && a.res_f32 == nullptr &&
+           a.y_nhwc == nullptr && a.ksplit <= 1;
+}
+
 static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_pref()) {
     Params &p = pl.p;
     p = Params{};
-    if (!plan_shape(a, p)) return MINW_EUNSUPPORTED;
+    p.trans = 0;
+    if (trans_eligible(a)) {
+        // only when the 256-pixel tiles cover the image without padding and leave
+        // at least four tiles per SM (else the 128-pixel tiles balance better)
+        Params q{};
+        const int sms_ = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
+        if (plan_shape(a, q, 256) && a.Wo % q.bw == 0 && a.Ho % q.bh == 0 &&
+            (long long)q.nbx * q.nby * ((a.B + q.bb - 1) / q.bb) >= 4LL * sms_)
+            p.trans = 1;
+    }
+    p.mrows = p.trans ? 256 : 128;
+    if (!plan_shape(a, p, p.mrows)) return MINW_EUNSUPPORTED;
+    if (p.trans) p.BN = 128;
     p.B = a.B; p.C = a.C; p.H = a.H; p.W = a.W; p.O = a.O; p.kh = a.kh; p.kw = a.kw; p.pad = a.pad;
     p.Ho = a.Ho; p.Wo = a.Wo;
     p.stride = a.stride;
     p.ck = (a.C % 128 == 0) ? 128 : 64;
-    p.a_bytes = (uint32_t)(128 * p.ck);
+    p.a_bytes = (uint32_t)(p.mrows * p.ck);
     p.nck = a.C / p.ck;
     p.nk = a.kh * a.kw * p.nck;
     p.nbb = (a.B + p.bb - 1) / p.bb;
@@ -1046,9 +1162,12 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     if (S > 8) S = 8;
     if (S < 2) return MINW_EUNSUPPORTED;
     p.S = S;
-    p.idesc = (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(p.BN >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+    // MMA N: the output channels, or the 256 pixels of a channel-major tile (M = 128 either way)
+    const int mma_n = p.trans ? 256 : p.BN;
+    p.acc_cols = mma_n;
+    p.idesc = (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(mma_n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
     uint32_t cols = 32;
-    while ((int)cols < 2 * p.BN) cols <<= 1;          // two accumulators
+    while ((int)cols < 2 * mma_n) cols <<= 1;         // two accumulators
     p.tmem_cols = cols;
     p.acc_out = a.acc_out; p.y_out = a.y_out; p.scale = a.scale; p.shift = a.shift;
     p.pool = a.pool; p.quant_out = a.quant_out; p.qo = a.qo;
@@ -1060,7 +1179,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
     p.ksplit = 1;
     pl.thr_ws = nullptr;
-    if (a.workspace != nullptr && !a.pool) {
+    if (a.workspace != nullptr && !a.pool && !p.trans) {
         // workspace: [breakpoints, when not given][ksplit partial-sum slices]
         const size_t tb = (a.quant_out && a.thr == nullptr) ? thr_ws_bytes(a.O, p.nlev) : 0;
         const size_t sb = slice_bytes(tiles, p.BN);
@@ -1084,7 +1203,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     // (padding the pixel tiles to a multiple of cl may add at most 1/8)
     const int tiles_m = p.nbx * p.nby * p.nbb;
     p.cl = 1;
-    if (p.ksplit == 1) {
+    if (p.ksplit == 1 && !p.trans) {
         int cl = cl_max;
         while (cl > 1 && (p.BN % (8 * cl) != 0 || ((tiles_m + cl - 1) / cl * cl - tiles_m) * 8 > tiles_m)) cl >>= 1;
         p.cl = cl;
