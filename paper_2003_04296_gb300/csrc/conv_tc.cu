@@ -643,14 +643,20 @@ __global__ void __launch_bounds__(NT, 1)
                     const int tn = w / tiles_m, tm = w - tn * tiles_m;
                     const int xb = tm % p.nbx, yb = (tm / p.nbx) % p.nby, bbk = tm / (p.nbx * p.nby);
                     const int oc = tn * p.BN + oq + lane;          // this lane's channel
-                    float nt[NL - 1], sg;
+                    const bool qlive = tn * p.BN + oq < p.O;       // 64-channel layers: half the lanes are padding
+                    float nt[NL - 1], sg = 1.0f;
+                    uint32_t sig = 0u;
 #pragma unroll
-                    for (int u = 0; u < NL - 1; ++u) nt[u] = sthr[oc * NL + u];
-                    sg = sthr[oc * NL + NL - 1];
-                    const uint32_t sig = ssig[(tn * p.BN + oq) >> 5];
+                    for (int u = 0; u < NL - 1; ++u) nt[u] = 0.0f;
+                    if (qlive) {
+#pragma unroll
+                        for (int u = 0; u < NL - 1; ++u) nt[u] = sthr[oc * NL + u];
+                        sg = sthr[oc * NL + NL - 1];
+                        sig = ssig[(tn * p.BN + oq) >> 5];
+                    }
                     if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
                     fence_after();
-                    for (int c = 4 * half_cols; c < 4 * half_cols + 4 && !dead; ++c) {
+                    for (int c = 4 * half_cols; c < 4 * half_cols + 4 && !dead && qlive; ++c) {
                         __syncwarp();
                         uint32_t v[32];
                         tmem_ld32(tmem_base + ((uint32_t)oq << 16) + (uint32_t)(ab * p.acc_cols + c * 32), v);
@@ -1117,8 +1123,26 @@ static int trans_pref() {
     return v;
 }
 
+// Tile of 256 pixels (bb images x bh rows x bw columns) that covers the output
+// image exactly, widest rows first; pooling keeps 2x2 windows inside a warp.
+static bool trans_shape(const ConvArgs &a, Params &p) {
+    if ((a.stride != 1 && a.stride != 2) || a.C % 64 != 0 || a.pad >= a.kh || a.pad >= a.kw) return false;
+    for (int bw = 128; bw >= 1; bw >>= 1) {
+        if (a.Wo % bw != 0 || (a.pool && (bw > 16 || bw < 2))) continue;
+        for (int bh = 256 / bw; bh >= 1; bh >>= 1) {
+            if (a.Ho % bh != 0 || (a.pool && bh < 2)) continue;
+            p.bw = bw; p.bh = bh; p.bb = 256 / (bw * bh);
+            p.nbx = a.Wo / bw;
+            p.nby = a.Ho / bh;
+            p.BN = 128;
+            return true;
+        }
+    }
+    return false;
+}
+
 static bool trans_eligible(const ConvArgs &a) {
-    return trans_pref() && a.O == 128 && a.quant_out && (a.codes_out != nullptr || a.planes_out != nullptr) &&
+    return trans_pref() && (a.O == 128 || a.O == 64) && a.quant_out && (a.codes_out != nullptr || a.planes_out != nullptr) &&
            a.acc_out == nullptr && a.y_out == nullptr && a.res_codes == nullptr && a.res_f32 == nullptr &&
            a.y_nhwc == nullptr && a.ksplit <= 1;
 }
@@ -1132,13 +1156,10 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
         // at least four tiles per SM (else the 128-pixel tiles balance better)
         Params q{};
         const int sms_ = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
-        if (plan_shape(a, q, 256) && a.Wo % q.bw == 0 && a.Ho % q.bh == 0 &&
-            (long long)q.nbx * q.nby * ((a.B + q.bb - 1) / q.bb) >= 4LL * sms_)
-            p.trans = 1;
+        if (trans_shape(a, q) && (long long)q.nbx * q.nby * ((a.B + q.bb - 1) / q.bb) >= 4LL * sms_) p.trans = 1;
     }
     p.mrows = p.trans ? 256 : 128;
-    if (!plan_shape(a, p, p.mrows)) return MINW_EUNSUPPORTED;
-    if (p.trans) p.BN = 128;
+    if (p.trans ? !trans_shape(a, p) : !plan_shape(a, p)) return MINW_EUNSUPPORTED;
     p.B = a.B; p.C = a.C; p.H = a.H; p.W = a.W; p.O = a.O; p.kh = a.kh; p.kw = a.kw; p.pad = a.pad;
     p.Ho = a.Ho; p.Wo = a.Wo;
     p.stride = a.stride;

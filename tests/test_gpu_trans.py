@@ -1,7 +1,8 @@
 """GPU parity of the channel-major tensor-core tiles (128 output channels x
-256 pixels, used for 128-channel layers whose only output is the next layer's
-levels): a 128 -> 128 convolution with and without the 2x2 pool, for each
-output bit width, against the oracle's levels, planes and codes."""
+256 pixels, used for 64- and 128-channel layers whose only output is the next
+layer's levels; a 64-channel layer pads the tile with zero weights): 128 -> 128
+and 64 -> 64 convolutions with and without the 2x2 pool, for each output bit
+width, against the oracle's levels, planes and codes."""
 import numpy as np
 import pytest
 
@@ -31,13 +32,15 @@ def M(dev):
     return minw
 
 
+@pytest.mark.parametrize("ch", [128, 64])
 @pytest.mark.parametrize("bits", [1, 2, 3])
 @pytest.mark.parametrize("pool", [0, 1])
-def test_channel_major_tiles(dev, M, bits, pool):
+def test_channel_major_tiles(dev, M, bits, pool, ch):
     # 160 images of 32x32: 640 pixel tiles of 256 (>= 4 per SM), blocks that tile the image exactly;
     # the images are independent, so the oracle checks three of them
-    B, C, H, W, O_ = 160, 128, 32, 32, 128
-    p = conv_problem(300 + bits + 10 * pool, B, C, H, W, O_, bits_a=bits, bits_w=bits, x_dist="normal", w_sigma=0.05)
+    B, C, H, W, O_ = 160, ch, 32, 32, ch
+    p = conv_problem(300 + bits + 10 * pool + ch, B, C, H, W, O_, bits_a=bits, bits_w=bits, x_dist="normal",
+                     w_sigma=0.05)
     a8 = torch.empty((B, H, W, C), dtype=torch.uint8, device=dev)
     w8 = torch.empty((O_, 3, 3, C), dtype=torch.uint8, device=dev)
     M.aqe_quantize_codes(dev_tensor(p["x"], dev), M.quant(bits, p["thr_a"]), a8)
