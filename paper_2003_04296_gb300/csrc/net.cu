@@ -11,6 +11,7 @@
 // (c, h, w) = OIHW weight order).
 #include <cuda_runtime.h>
 #include <stdint.h>
+#include <stdlib.h>
 
 #include <vector>
 
@@ -24,6 +25,8 @@ static void net_free(minw_net *n) {
     if (n->res) resnet_free(n);
     for (void *p : n->owned) cudaFree(p);
     for (cudaEvent_t e : n->events) cudaEventDestroy(e);
+    if (n->gexec) cudaGraphExecDestroy(n->gexec);
+    if (n->cap_stream) cudaStreamDestroy(n->cap_stream);
     delete n;
 }
 
@@ -193,12 +196,21 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
     return MINW_OK;
 }
 
-minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits, void *stream) {
-    if (!net || !x || !logits || B <= 0 || B > net->max_batch) return MINW_EINVAL;
-    if (net->kind == 1) return resnet_forward(net, x, B, logits, (cudaStream_t)stream);
+// MINW_GRAPH=0 enqueues every kernel on every call instead of replaying the
+// captured forward.
+static bool graphs_enabled() {
+    static int v = -1;
+    if (v < 0) {
+        const char *e = getenv("MINW_GRAPH");
+        v = (e && e[0] == '0') ? 0 : 1;
+    }
+    return v == 1;
+}
+
+static minw_status forward_enqueue(minw_net *net, const float *x, int32_t B, float *logits, cudaStream_t cs) {
+    if (net->kind == 1) return resnet_forward(net, x, B, logits, cs);
     const int nl = (int)net->L.size();
     int cur = 0;
-    cudaStream_t cs = (cudaStream_t)stream;
     if (net->timing && cudaEventRecord(net->events[0], cs) != cudaSuccess) return MINW_ECUDA;
     for (int l = 0; l < nl; ++l) {
         const LayerPlan &P = net->L[l];
@@ -253,6 +265,47 @@ minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits
         cur ^= 1;
     }
     return MINW_OK;
+}
+
+// The forward's kernels are captured once into a CUDA graph on a stream the
+// net owns and replayed on the caller's stream while the input and logits
+// pointers and the batch stay the same (any change re-captures); per-layer
+// timing enqueues the kernels directly, and so does a call made while the
+// caller's stream is itself being captured.
+minw_status minw_forward(minw_net *net, const float *x, int32_t B, float *logits, void *stream) {
+    if (!net || !x || !logits || B <= 0 || B > net->max_batch) return MINW_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (net->timing || !graphs_enabled() || cudaStreamIsCapturing(s, &cap) != cudaSuccess ||
+        cap != cudaStreamCaptureStatusNone)
+        return forward_enqueue(net, x, B, logits, s);
+    if (net->gexec == nullptr || net->gx != x || net->glogits != logits || net->gB != B) {
+        if (net->cap_stream == nullptr &&
+            cudaStreamCreateWithFlags(&net->cap_stream, cudaStreamNonBlocking) != cudaSuccess)
+            return MINW_ECUDA;
+        if (cudaStreamBeginCapture(net->cap_stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
+            return MINW_ECUDA;
+        const minw_status st = forward_enqueue(net, x, B, logits, net->cap_stream);
+        cudaGraph_t g = nullptr;
+        const cudaError_t ce = cudaStreamEndCapture(net->cap_stream, &g);
+        if (st != MINW_OK || ce != cudaSuccess || g == nullptr) {
+            if (g) cudaGraphDestroy(g);
+            cudaGetLastError();
+            return st != MINW_OK ? st : MINW_ECUDA;
+        }
+        if (net->gexec) cudaGraphExecDestroy(net->gexec);
+        net->gexec = nullptr;
+        const cudaError_t ie = cudaGraphInstantiate(&net->gexec, g, 0);
+        cudaGraphDestroy(g);
+        if (ie != cudaSuccess) {
+            net->gexec = nullptr;
+            return MINW_ECUDA;
+        }
+        net->gx = x;
+        net->glogits = logits;
+        net->gB = B;
+    }
+    return cudaGraphLaunch(net->gexec, s) == cudaSuccess ? MINW_OK : MINW_ECUDA;
 }
 
 minw_status minw_forward_host(minw_net *net, const float *x_host, int32_t B, float *logits_host,

@@ -44,6 +44,12 @@ struct minw_net {
     size_t ws_bytes = 0;
     std::vector<cudaEvent_t> events;  // [0] before the first layer, [l+1] after layer l
     bool timing = false;
+    // the forward captured once as a CUDA graph (per input, logits and batch) and replayed
+    cudaStream_t cap_stream = nullptr;
+    cudaGraphExec_t gexec = nullptr;
+    const float *gx = nullptr;
+    float *glogits = nullptr;
+    int gB = 0;
 };
 
 
