@@ -1111,9 +1111,10 @@ static int kps_pref() {
     return v;
 }
 
-// Channel-major tiles (MINW_TC_TRANS=0 turns them off): a 128-channel layer
-// whose only output is the next layer's levels runs as 128 channels x 256
-// pixels, so each MMA has N = 256 (the tensor pipe's full rate).
+// Channel-major tiles (MINW_TC_TRANS=0 turns them off): a 64- or 128-channel
+// layer whose only output is the next layer's levels runs as 128 channels (a
+// 64-channel layer pads with zero weights) x 256 pixels, so each MMA has
+// N = 256 (the tensor pipe's full rate).
 static int trans_pref() {
     static int v = -1;
     if (v < 0) {
@@ -1153,10 +1154,17 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     p.trans = 0;
     if (trans_eligible(a)) {
         // only when the 256-pixel tiles cover the image without padding and leave
-        // at least four tiles per SM (else the 128-pixel tiles balance better)
+        // at least two tiles per SM (MINW_TC_TRANS_MIN), else the 128-pixel tiles
+        // balance better
         Params q{};
         const int sms_ = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
-        if (trans_shape(a, q) && (long long)q.nbx * q.nby * ((a.B + q.bb - 1) / q.bb) >= 4LL * sms_) p.trans = 1;
+        static int min_tiles = -1;
+        if (min_tiles < 0) {
+            const char *e = getenv("MINW_TC_TRANS_MIN");
+            min_tiles = e ? atoi(e) : 2;
+        }
+        if (trans_shape(a, q) && (long long)q.nbx * q.nby * ((a.B + q.bb - 1) / q.bb) >= (long long)min_tiles * sms_)
+            p.trans = 1;
     }
     p.mrows = p.trans ? 256 : 128;
     if (p.trans ? !trans_shape(a, p) : !plan_shape(a, p)) return MINW_EUNSUPPORTED;
