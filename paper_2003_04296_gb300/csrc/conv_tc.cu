@@ -656,18 +656,59 @@ __global__ void __launch_bounds__(NT, 1)
                     }
                     if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
                     fence_after();
+                    const bool tres = p.res_codes != nullptr || p.res_f32 != nullptr;
+                    float sc = 0.0f, sh = 0.0f, ny[NL - 1];
+#pragma unroll
+                    for (int u = 0; u < NL - 1; ++u) ny[u] = syt[u];
+                    if (tres && qlive) {
+                        sc = __ldg(p.scale + oc);
+                        sh = __ldg(p.shift + oc);
+                    }
                     for (int c = 4 * half_cols; c < 4 * half_cols + 4 && !dead && qlive; ++c) {
                         __syncwarp();
                         uint32_t v[32];
                         tmem_ld32(tmem_base + ((uint32_t)oq << 16) + (uint32_t)(ab * p.acc_cols + c * 32), v);
+                        const int r = c * 32 + lane;                    // tile row (pixel) of this lane
+                        const int b = bbk * p.bb + r / (p.bh * p.bw);
+                        const int y = yb * p.bh + (r / p.bw) % p.bh;
+                        const int x = xb * p.bw + r % p.bw;
+                        const bool valid = b < p.B && y < p.Ho && x < p.Wo;
                         uint32_t M[NL - 1];
+                        if (tres) {
+                            // residual block: y = BN(acc) + shortcut at (pixel j, this lane's channel), then the
+                            // quantizer's breakpoints on y; pixel j's index comes from lane j
+                            // (all 32 loads issue before the first use; a pixel past the batch reads pixel 0)
+                            const long long pix = valid ? (((long long)b * p.Ho + y) * p.Wo + x) * p.O : 0;
+                            float yv[32];
+                            if (p.res_codes != nullptr) {
+                                uint32_t cb[32];
 #pragma unroll
-                        for (int u = 0; u < NL - 1; ++u) {
-                            uint32_t wd = 0u;          // bit j: [sigma * acc < T_u] at pixel column 32 c + j
+                                for (int j = 0; j < 32; ++j) cb[j] = __ldg(p.res_codes + oc + __shfl_sync(0xffffffffu, pix, j));
 #pragma unroll
-                            for (int j = 31; j >= 0; --j)
-                                wd = __funnelshift_l(__float_as_uint(fmaf(__uint_as_float(v[j]), sg, nt[u])), wd, 1);
-                            M[u] = transpose32(wd, lane);     // lane j: bit k = channel oq + k at column 32 c + j
+                                for (int j = 0; j < 32; ++j)
+                                    yv[j] = fmaf(__uint_as_float(v[j]), sc, sh) + code_units(cb[j]) * p.res_unit;
+                            } else {
+#pragma unroll
+                                for (int j = 0; j < 32; ++j) yv[j] = __ldg(p.res_f32 + oc + __shfl_sync(0xffffffffu, pix, j));
+#pragma unroll
+                                for (int j = 0; j < 32; ++j) yv[j] = fmaf(__uint_as_float(v[j]), sc, sh) + yv[j];
+                            }
+#pragma unroll
+                            for (int u = 0; u < NL - 1; ++u) {
+                                uint32_t wd = 0u;
+#pragma unroll
+                                for (int j = 31; j >= 0; --j) wd = __funnelshift_l(__float_as_uint(yv[j] + ny[u]), wd, 1);
+                                M[u] = transpose32(wd, lane);
+                            }
+                        } else {
+#pragma unroll
+                            for (int u = 0; u < NL - 1; ++u) {
+                                uint32_t wd = 0u;          // bit j: [sigma * acc < T_u] at pixel column 32 c + j
+#pragma unroll
+                                for (int j = 31; j >= 0; --j)
+                                    wd = __funnelshift_l(__float_as_uint(fmaf(__uint_as_float(v[j]), sg, nt[u])), wd, 1);
+                                M[u] = transpose32(wd, lane);     // lane j: bit k = channel oq + k at column 32 c + j
+                            }
                         }
                         if (p.pool) {
 #pragma unroll
@@ -680,11 +721,6 @@ __global__ void __launch_bounds__(NT, 1)
                                 M[u] = (sig & a2) | (~sig & o2);
                             }
                         }
-                        const int r = c * 32 + lane;                    // tile row (pixel) of this lane
-                        const int b = bbk * p.bb + r / (p.bh * p.bw);
-                        const int y = yb * p.bh + (r / p.bw) % p.bh;
-                        const int x = xb * p.bw + r % p.bw;
-                        const bool valid = b < p.B && y < p.Ho && x < p.Wo;
                         const bool writer = valid && (!p.pool || ((x & 1) == 0 && (y & 1) == 0));
                         if (writer) {
                             const int yp = p.pool ? y / 2 : y, xp = p.pool ? x / 2 : x;
@@ -1112,9 +1148,9 @@ static int kps_pref() {
 }
 
 // Channel-major tiles (MINW_TC_TRANS=0 turns them off): a 64- or 128-channel
-// layer whose only output is the next layer's levels runs as 128 channels (a
-// 64-channel layer pads with zero weights) x 256 pixels, so each MMA has
-// N = 256 (the tensor pipe's full rate).
+// layer whose only output is the next layer's levels (a residual block's too,
+// at 128 channels) runs as 128 channels (a 64-channel layer pads with zero
+// weights) x 256 pixels, so each MMA has N = 256 (the tensor pipe's full rate).
 static int trans_pref() {
     static int v = -1;
     if (v < 0) {
@@ -1144,8 +1180,9 @@ static bool trans_shape(const ConvArgs &a, Params &p) {
 
 static bool trans_eligible(const ConvArgs &a) {
     return trans_pref() && (a.O == 128 || a.O == 64) && a.quant_out && (a.codes_out != nullptr || a.planes_out != nullptr) &&
-           a.acc_out == nullptr && a.y_out == nullptr && a.res_codes == nullptr && a.res_f32 == nullptr &&
-           a.y_nhwc == nullptr && a.ksplit <= 1;
+           a.acc_out == nullptr && a.y_out == nullptr && a.y_nhwc == nullptr && a.ksplit <= 1 &&
+           (a.res_codes == nullptr && a.res_f32 == nullptr ||
+            (a.O == 128 && !a.pool));     // a 64-channel residual layer keeps pixel-major tiles (all 8 warps busy)
 }
 
 static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_pref()) {

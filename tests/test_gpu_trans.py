@@ -69,3 +69,51 @@ def test_channel_major_tiles(dev, M, bits, pool, ch):
     want_codes = np.vectorize(_CODE.get)(units.transpose(0, 2, 3, 1)).astype(np.uint8)
     assert np.array_equal(codes.cpu().numpy()[pick], want_codes)
     assert np.array_equal(planes_view(planes, B, Hp, Wp, bits, O_)[pick], O.pack(lv, bits))
+
+
+@pytest.mark.parametrize("ch", [128, 64])
+@pytest.mark.parametrize("bits", [1, 2, 3])
+@pytest.mark.parametrize("shortcut", ["codes", "f32"])
+def test_channel_major_residual(dev, M, bits, ch, shortcut):
+    """Residual block in channel-major tiles: y = fmaf(acc, scale, shift) +
+    shortcut, HardTanh, quantize; the shortcut is a level-code tensor (identity
+    path) or fp32 NHWC (downsample path).  Each lane holds one channel, so the
+    shortcut of pixel j comes through lane j's pixel index.  (A 64-channel
+    residual layer runs in pixel-major tiles: the same check covers it.)"""
+    B, C, H, W, O_ = 160, ch, 32, 32, ch
+    p = conv_problem(500 + bits + ch, B, C, H, W, O_, bits_a=bits, bits_w=bits, x_dist="normal", w_sigma=0.05)
+    a8 = torch.empty((B, H, W, C), dtype=torch.uint8, device=dev)
+    w8 = torch.empty((O_, 3, 3, C), dtype=torch.uint8, device=dev)
+    M.aqe_quantize_codes(dev_tensor(p["x"], dev), M.quant(bits, p["thr_a"]), a8)
+    M.minw_pack_weight_codes(dev_tensor(p["w"], dev), M.quant(bits, p["thr_w"]), w8,
+                             channel_scale=dev_tensor(p["w_scale"], dev))
+    qo = M.quant(bits, DEFAULT_THR[bits])
+    r = np.random.default_rng(600 + bits + ch)
+    if shortcut == "codes":
+        xs = (r.standard_normal((B, O_, H, W)) * 0.7).astype(np.float32)
+        res = O.quantize(xs, bits, DEFAULT_THR[bits]).astype(np.float32)
+        res_codes = torch.empty((B, H, W, O_), dtype=torch.uint8, device=dev)
+        M.aqe_quantize_codes(dev_tensor(xs, dev), qo, res_codes)
+        kw = dict(res_codes=res_codes, res_bits=bits)
+    else:
+        res = (r.standard_normal((B, O_, H, W)) * 0.5).astype(np.float32)
+        kw = dict(res_f32=dev_tensor(res.transpose(0, 2, 3, 1), dev))
+    codes = torch.empty((B, H, W, O_), dtype=torch.uint8, device=dev)
+    planes = torch.empty(M.packed_words(B, O_, H, W, bits), dtype=torch.int32, device=dev)
+    for out in ("codes", "planes"):
+        M.minw_conv_block_codes_ex(a8, B, C, H, W, bits, w8, O_, 3, 3, bits, 1, 1, 0, dev_tensor(p["scale"], dev),
+                                   dev_tensor(p["shift"], dev), q_out=qo,
+                                   codes_out=codes if out == "codes" else None,
+                                   planes_out=planes if out == "planes" else None, **kw)
+    torch.cuda.synchronize()
+    assert M.minw_get_last_device_error() == M.MINW_OK
+    pick = [0, 77, B - 1]
+    al = O.quantize(p["x"][pick], bits, p["thr_a"])
+    wl = O.quantize(p["w"], bits, p["thr_w"], p["w_scale"])
+    acc = O.conv2d_levels(al, wl, 1, 1, bits, bits)
+    y = O.hardtanh((O.affine(acc, p["scale"], p["shift"]) + res[pick]).astype(np.float32))
+    lv = O.quantize(y, bits, DEFAULT_THR[bits])
+    units = np.rint(lv * (4 if bits == 3 else 1)).astype(int)
+    want_codes = np.vectorize(_CODE.get)(units.transpose(0, 2, 3, 1)).astype(np.uint8)
+    assert np.array_equal(codes.cpu().numpy()[pick], want_codes)
+    assert np.array_equal(planes_view(planes, B, H, W, bits, O_)[pick], O.pack(lv, bits))
