@@ -43,6 +43,7 @@ struct FirstTile {
     int Ws;           // patch columns per stride phase
     int RP;           // patch row pitch (stride x Ws)
     int K;            // C x kh x kw
+    int nb;           // input patch buffers (2 or 3: the patch of tile t + (nb - 1) G is in flight)
     size_t smem;      // bytes of dynamic shared memory
 };
 
@@ -59,7 +60,11 @@ static FirstTile first_tile(const FirstArgs &a) {
     t.Ws = (Win + a.stride - 1) / a.stride;
     t.RP = t.Ws * a.stride;
     t.K = a.C * a.kh * a.kw;
-    t.smem = sizeof(float) * ((size_t)t.K * t.OCB + (size_t)t.OCB * 8 + 2 * (size_t)a.C * t.Rmax * t.RP);
+    // three patch buffers (two tiles of look-ahead) where two CTAs still fit on an SM
+    const size_t fixed = sizeof(float) * ((size_t)t.K * t.OCB + (size_t)t.OCB * 8);
+    const size_t pbytes = sizeof(float) * (size_t)a.C * t.Rmax * t.RP;
+    t.nb = fixed + 3 * pbytes <= 112 * 1024 ? 3 : 2;
+    t.smem = fixed + t.nb * pbytes;
     return t;
 }
 
@@ -79,7 +84,9 @@ __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_gr
 // patches [C][rows][columns] (zero padded; columns split by stride phase, column
 // rx at (rx % S) * Ws + rx / S, so that threads reading neighbouring output
 // pixels read neighbouring words for any stride): the next tile's patch
-// arrives by cp.async while the current one is computed.  Warp = 32 output
+// arrives by cp.async while the current one is computed (and, where shared
+// memory allows, the one after it: a small patch takes about as long to
+// arrive as a tile takes to compute).  Warp = 32 output
 // channels x 64 pixels; a thread holds four pixels (16 apart) x 16 channels
 // as 8 channel pairs and per tap does four patch loads, four 128-bit weight
 // loads (one address per half warp) and 32 packed fma.rn.f32x2, one fmaf
@@ -97,7 +104,7 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
     const size_t patch = (size_t)a.C * tl.Rmax * RP;
     float *sW = reinterpret_cast<float *>(smem4);                 // [K][OCB]
     float *sT = sW + (size_t)K * OCB;                             // [OCB][8] -breakpoints, sigma
-    float *sX0 = sT + OCB * 8;                                    // [2][C][Rmax][RP]
+    float *sX0 = sT + OCB * 8;                                    // [nb][C][Rmax][RP]
 
     const int o0 = blockIdx.y * OCB;
     const int ochan = min(OCB, a.O - o0);
@@ -170,7 +177,14 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
     // 4 pixels (16 apart) x 16 channels per thread
     pdl_trigger();                                               // set-up done
     pdl_wait();                                                  // the image and the output buffer are shared
-    if (t < total) load_patch(t, 0);
+    // one cp.async group per tile slot (empty past the end), so that the wait count is fixed
+    const int nb = tl.nb;
+    for (int j = 0; j < nb - 1; ++j) {
+        if (t + j * (int)gridDim.x < total)
+            load_patch(t + j * (int)gridDim.x, j);
+        else
+            cp_async_commit();
+    }
     const int g = warp % tl.groups, pb = warp / tl.groups;
     const int h = lane >> 4, l16 = lane & 15;
     const int NWo = (a.O + 31) >> 5;
@@ -179,14 +193,17 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
     const int ob = o0 + g * 32;
     const float *wg = sW + g * 32 + h * 16;
     constexpr int NL = OUTB == 0 ? 1 : (OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7));
-    for (int buf = 0; t < total; t += gridDim.x, buf ^= 1) {
-        const int tn = t + (int)gridDim.x;
-        if (tn < total) {
-            load_patch(tn, buf ^ 1);
+    for (int buf = 0; t < total; t += gridDim.x, buf = buf + 1 == nb ? 0 : buf + 1) {
+        const int tn = t + (nb - 1) * (int)gridDim.x;
+        const int bn = buf == 0 ? nb - 1 : buf - 1;              // the slot tile t - G used
+        if (tn < total)
+            load_patch(tn, bn);
+        else
+            cp_async_commit();
+        if (nb == 3)
+            cp_async_wait<2>();
+        else
             cp_async_wait<1>();
-        } else {
-            cp_async_wait<0>();
-        }
         __syncthreads();                                         // patch t (and the weights) visible
 
         const int b = t / tl.tiles;
@@ -302,7 +319,7 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
                 }
             }
         }
-        __syncthreads();                                         // buffer buf is free for tile t + 2 G
+        __syncthreads();                                         // buffer buf is free for tile t + nb G
     }
 }
 
