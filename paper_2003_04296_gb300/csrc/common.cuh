@@ -1,6 +1,7 @@
 // common.cuh -- shared device helpers of libminw.so (sm_103a only).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -266,6 +267,12 @@ bool valid_quant(const minw_quant *q);
 int num_sms();
 minw_status launch_status();
 bool pdl_enabled();                 // MINW_PDL=0 turns programmatic dependent launch off
+
+// cuTensorMapEncodeTiled from the driver (nullptr when it is unavailable).
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn tensor_map_encoder();
 
 // Kernel launch on stream s that may overlap the previous kernel in the
 // stream (programmatic stream serialization); the kernel calls pdl_wait()

@@ -8,6 +8,8 @@
 // See conv_first_kernel for the tiling.
 #include <cuda_runtime.h>
 #include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
 
 #include "kernels.cuh"
 
@@ -34,20 +36,84 @@ __device__ __forceinline__ float lane2(unsigned long long v, int hi) {
     return hi ? hi_ : lo_;
 }
 
+// Shared-memory loads by 32-bit shared address (the address arithmetic of
+// the tap loop stays in 32-bit registers with immediate offsets).
+__device__ __forceinline__ float lds_f32(uint32_t a) {
+    float v;
+    asm volatile("ld.shared.f32 %0, [%1];\n" : "=f"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ void lds_2x64(uint32_t a, unsigned long long &x, unsigned long long &y) {
+    asm volatile("ld.shared.v2.u64 {%0, %1}, [%2];\n" : "=l"(x), "=l"(y) : "r"(a));
+}
+
+// Error flag of this file's bounded waits (read with the tensor-core
+// kernels' flag by minw_get_last_device_error).
+__device__ int g_first_error = 0;
+
+constexpr long long FIRST_WAIT_CYCLES = 1ll << 31;
+
+__device__ __forceinline__ uint32_t saddr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void fbar_init(uint64_t *bar) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;\n" ::"r"(saddr(bar)));
+}
+
+__device__ __forceinline__ bool fbar_try_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, 100000;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(saddr(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait for a patch: false (and the error flag set) after about a second.
+__device__ __forceinline__ bool fbar_wait(uint64_t *bar, uint32_t parity) {
+    if (fbar_try_wait(bar, parity)) return true;
+    const long long t0 = clock64();
+    while (!fbar_try_wait(bar, parity)) {
+        if (clock64() - t0 > FIRST_WAIT_CYCLES) {
+            atomicExch(&g_first_error, 1);
+            return false;
+        }
+    }
+    return true;
+}
+
+// One box of the image [B][C][H][W] (x, y, c, b from the origin given) into
+// shared memory, completing its bytes on bar.  Zero outside the image.
+__device__ __forceinline__ void patch_tma(void *dst, const CUtensorMap *map, uint64_t *bar, uint32_t bytes, int x,
+                                          int y, int b) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(saddr(bar)), "r"(bytes)
+                 : "memory");
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6];\n" ::"r"(saddr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(0), "r"(b), "r"(saddr(bar))
+        : "memory");
+}
+
 struct FirstTile {
     int OCB;          // output channels per CTA (32 or 64)
     int groups;       // 32-channel groups per CTA
     int PB;           // output pixels per CTA (64 per pixel block, 8 / groups blocks)
     int tiles;        // CTAs along the pixels of one image
     int Rmax;         // input patch rows
-    int Ws;           // patch columns per stride phase
-    int RP;           // patch row pitch (stride x Ws)
+    int Ws;           // patch columns per stride phase (cp.async patches)
+    int RP;           // patch row pitch: stride x Ws, or the box width (TMA patches)
     int K;            // C x kh x kw
     int nb;           // input patch buffers (2 or 3: the patch of tile t + (nb - 1) G is in flight)
+    int tma;          // patches as one TMA box each (row-major columns from x0, zero padded)
+    int x0;           // TMA patches: first image column of the box (a multiple of 4, <= -pad)
+    int xsh;          // TMA patches: box column of image column -pad (-pad - x0)
+    int xoff;         // float offset of the first patch buffer (a multiple of 32: 128-byte aligned)
+    int pstride;      // floats per patch buffer (a multiple of 32)
     size_t smem;      // bytes of dynamic shared memory
 };
 
-static FirstTile first_tile(const FirstArgs &a) {
+static FirstTile first_tile(const FirstArgs &a, bool tma) {
     FirstTile t;
     t.OCB = a.O > 32 ? 64 : 32;
     t.groups = t.OCB / 32;
@@ -60,9 +126,16 @@ static FirstTile first_tile(const FirstArgs &a) {
     t.Ws = (Win + a.stride - 1) / a.stride;
     t.RP = t.Ws * a.stride;
     t.K = a.C * a.kh * a.kw;
+    // TMA box: image columns x0 .. x0 + RP - 1 with x0 rounded down to 16 bytes
+    t.x0 = -((a.pad + 3) / 4) * 4;
+    t.xsh = -a.pad - t.x0;
+    t.tma = tma && (Win + t.xsh + 3) / 4 * 4 <= 256 && t.Rmax <= 256 && a.C <= 256;
+    if (t.tma) t.RP = (Win + t.xsh + 3) / 4 * 4;
+    t.xoff = (t.K * t.OCB + t.OCB * 8 + 31) / 32 * 32;
+    t.pstride = (a.C * t.Rmax * t.RP + 31) / 32 * 32;
     // three patch buffers (two tiles of look-ahead) where two CTAs still fit on an SM
-    const size_t fixed = sizeof(float) * ((size_t)t.K * t.OCB + (size_t)t.OCB * 8);
-    const size_t pbytes = sizeof(float) * (size_t)a.C * t.Rmax * t.RP;
+    const size_t fixed = sizeof(float) * (size_t)t.xoff + 3 * sizeof(uint64_t);
+    const size_t pbytes = sizeof(float) * (size_t)t.pstride;
     t.nb = fixed + 3 * pbytes <= 112 * 1024 ? 3 : 2;
     t.smem = fixed + t.nb * pbytes;
     return t;
@@ -95,16 +168,21 @@ __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_gr
 // acc: the padded taps change nothing, exactly as skipping them.  The
 // epilogue turns each pixel's 32 channels into level masks (the sign bits of
 // fmaf(acc, sigma, -T)) and stores planes or codes from them.  KH, KW, S = 0:
-// runtime shape.
-template <int OUTB, int KH, int KW, int S>
-__global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs a, const FirstTile tl) {
+// runtime shape.  TM: each patch is one TMA box of the image (rows of RP
+// columns from x0, zero outside the image, completion on an mbarrier per
+// buffer), not per-word cp.async copies split by stride phase; a thread then
+// reads its pixels' words S apart (16 lanes on 16 distinct banks for S <= 2).
+template <int OUTB, int KH, int KW, int S, bool TM>
+__global__ void __launch_bounds__(FIRST_NT, 2)
+    conv_first_kernel(const FirstArgs a, const FirstTile tl, const __grid_constant__ CUtensorMap tmX) {
     extern __shared__ float4 smem4[];
     const int kh = KH ? KH : a.kh, kw = KW ? KW : a.kw, st = S ? S : a.stride;
     const int OCB = tl.OCB, K = tl.K, RP = tl.RP, Ws = tl.Ws;
-    const size_t patch = (size_t)a.C * tl.Rmax * RP;
+    const size_t patch = (size_t)tl.pstride;
     float *sW = reinterpret_cast<float *>(smem4);                 // [K][OCB]
     float *sT = sW + (size_t)K * OCB;                             // [OCB][8] -breakpoints, sigma
-    float *sX0 = sT + OCB * 8;                                    // [nb][C][Rmax][RP]
+    float *sX0 = sW + tl.xoff;                                    // [nb][C][Rmax][RP]
+    uint64_t *fullb = reinterpret_cast<uint64_t *>(sX0 + (size_t)tl.nb * patch);   // [nb] TMA patch arrivals
 
     const int o0 = blockIdx.y * OCB;
     const int ochan = min(OCB, a.O - o0);
@@ -117,6 +195,11 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
     auto load_patch = [&](int t, int buf) {
         const int b = t / tl.tiles;
         const int p0 = (t - b * tl.tiles) * tl.PB;
+        if constexpr (TM) {       // one thread: the whole patch as one box
+            patch_tma(sX0 + buf * patch, &tmX, &fullb[buf], (uint32_t)(sizeof(float) * a.C * tl.Rmax * RP), tl.x0,
+                      (p0 / a.Wo) * st - a.pad, b);
+            return;
+        }
         const int pend = min(p0 + tl.PB, npix);
         const int y_first = p0 / a.Wo, y_last = (pend - 1) / a.Wo;
         const int rows_in = (y_last - y_first) * st + kh;
@@ -173,18 +256,27 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
         }
     }
 
+    if (TM && threadIdx.x == 0) {
+        for (int j = 0; j < tl.nb; ++j) fbar_init(&fullb[j]);
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    __syncthreads();                                             // barriers initialised
+
     // warp = 32 channels x 64 pixels; lane = (channel half h, pixel l16):
     // 4 pixels (16 apart) x 16 channels per thread
     pdl_trigger();                                               // set-up done
     pdl_wait();                                                  // the image and the output buffer are shared
-    // one cp.async group per tile slot (empty past the end), so that the wait count is fixed
+    // TMA: thread 0 issues; cp.async: one group per tile slot (empty past the
+    // end), so that the wait count is fixed
     const int nb = tl.nb;
     for (int j = 0; j < nb - 1; ++j) {
-        if (t + j * (int)gridDim.x < total)
-            load_patch(t + j * (int)gridDim.x, j);
-        else
+        if (t + j * (int)gridDim.x < total) {
+            if (!TM || threadIdx.x == 0) load_patch(t + j * (int)gridDim.x, j);
+        } else if (!TM) {
             cp_async_commit();
+        }
     }
+    bool dead = false;                                           // a patch wait ran out: skip the work
     const int g = warp % tl.groups, pb = warp / tl.groups;
     const int h = lane >> 4, l16 = lane & 15;
     const int NWo = (a.O + 31) >> 5;
@@ -193,18 +285,23 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
     const int ob = o0 + g * 32;
     const float *wg = sW + g * 32 + h * 16;
     constexpr int NL = OUTB == 0 ? 1 : (OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7));
-    for (int buf = 0; t < total; t += gridDim.x, buf = buf + 1 == nb ? 0 : buf + 1) {
+    for (int buf = 0, it = 0; t < total; t += gridDim.x, buf = buf + 1 == nb ? 0 : buf + 1, ++it) {
         const int tn = t + (nb - 1) * (int)gridDim.x;
         const int bn = buf == 0 ? nb - 1 : buf - 1;              // the slot tile t - G used
-        if (tn < total)
-            load_patch(tn, bn);
-        else
-            cp_async_commit();
-        if (nb == 3)
-            cp_async_wait<2>();
-        else
-            cp_async_wait<1>();
-        __syncthreads();                                         // patch t (and the weights) visible
+        if constexpr (TM) {
+            if (tn < total && threadIdx.x == 0 && !dead) load_patch(tn, bn);
+            if (!dead && !fbar_wait(&fullb[buf], (uint32_t)(it / nb) & 1u)) dead = true;
+        } else {
+            if (tn < total)
+                load_patch(tn, bn);
+            else
+                cp_async_commit();
+            if (nb == 3)
+                cp_async_wait<2>();
+            else
+                cp_async_wait<1>();
+        }
+        dead = __syncthreads_or(dead);                           // patch t (and the weights) visible
 
         const int b = t / tl.tiles;
         const int p0 = (t - b * tl.tiles) * tl.PB;
@@ -219,38 +316,41 @@ __global__ void __launch_bounds__(FIRST_NT, 2) conv_first_kernel(const FirstArgs
             live[i] = p < pend;
             pix[i] = live[i] ? p : p0;
             const int yy = pix[i] / a.Wo, xx = pix[i] - yy * a.Wo;
-            pofs[i] = (yy - y_first) * st * RP + xx;
+            pofs[i] = (yy - y_first) * st * RP + (TM ? xx * st + tl.xsh : xx);
         }
-        if (p0 + pb * 64 < pend && gch > 0) {                   // warp-uniform: the epilogue shuffles
+        if (p0 + pb * 64 < pend && gch > 0 && !dead) {          // warp-uniform: the epilogue shuffles
             // accumulators of channel pairs (2j, 2j + 1), packed for fma.rn.f32x2
             unsigned long long acc[FIRST_PX][8];
 #pragma unroll
             for (int i = 0; i < FIRST_PX; ++i)
 #pragma unroll
                 for (int o = 0; o < 8; ++o) acc[i][o] = 0ull;
+            const uint32_t xs = (uint32_t)__cvta_generic_to_shared(sX);
+            const uint32_t ws = (uint32_t)__cvta_generic_to_shared(wg);
+            uint32_t xa[FIRST_PX];
+#pragma unroll
+            for (int i = 0; i < FIRST_PX; ++i) xa[i] = xs + 4u * (uint32_t)pofs[i];
             for (int c = 0; c < a.C; ++c) {
 #pragma unroll (KH ? KH : 1)
                 for (int ky = 0; ky < kh; ++ky) {
-                    const float *xrow = sX + ((size_t)c * tl.Rmax + ky) * RP;
-                    const float *wrow = wg + (size_t)((c * kh + ky) * kw) * OCB;
-                    const float *xp[FIRST_PX];
-#pragma unroll
-                    for (int i = 0; i < FIRST_PX; ++i) xp[i] = xrow + pofs[i];
+                    const uint32_t ro = 4u * (uint32_t)((c * tl.Rmax + ky) * RP);
+                    const uint32_t wr = ws + 4u * (uint32_t)((c * kh + ky) * kw * OCB);
 #pragma unroll (KW ? KW : 1)
                     for (int kx = 0; kx < kw; ++kx) {
                         // tap column kx: stride phase kx % S, offset kx / S within the phase
-                        const int ph = kx % st, xo = kx / st;
+                        const uint32_t xo = ro + 4u * (uint32_t)(TM ? kx : (kx % st) * Ws + kx / st);
                         unsigned long long xv[FIRST_PX];
 #pragma unroll
-                        for (int i = 0; i < FIRST_PX; ++i) xv[i] = dup2((ph == 0 ? xp[i] : xp[i] + ph * Ws)[xo]);
-                        const ulonglong2 *w2 = reinterpret_cast<const ulonglong2 *>(wrow + kx * OCB);
+                        for (int i = 0; i < FIRST_PX; ++i) xv[i] = dup2(lds_f32(xa[i] + xo));
+                        const uint32_t wk = wr + 4u * (uint32_t)(kx * OCB);
 #pragma unroll
                         for (int o4 = 0; o4 < 4; ++o4) {
-                            const ulonglong2 w = w2[o4];
+                            unsigned long long wx, wy;
+                            lds_2x64(wk + 16u * o4, wx, wy);
 #pragma unroll
                             for (int i = 0; i < FIRST_PX; ++i) {
-                                ffma2(acc[i][2 * o4], xv[i], w.x);
-                                ffma2(acc[i][2 * o4 + 1], xv[i], w.y);
+                                ffma2(acc[i][2 * o4], xv[i], wx);
+                                ffma2(acc[i][2 * o4 + 1], xv[i], wy);
                             }
                         }
                     }
@@ -366,10 +466,11 @@ minw_status launch_thresholds_f32(const float *scale, const float *shift, int O,
     return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
 }
 
-template <int OUTB, int KH, int KW, int S>
-static minw_status launch_first_shape(const FirstArgs &a, const FirstTile &tl, cudaStream_t s) {
+template <int OUTB, int KH, int KW, int S, bool TM>
+static minw_status launch_first_shape(const FirstArgs &a, const FirstTile &tl, const CUtensorMap &tm,
+                                      cudaStream_t s) {
     static size_t configured = 0;
-    void (*kern)(const FirstArgs, const FirstTile) = conv_first_kernel<OUTB, KH, KW, S>;
+    void (*kern)(const FirstArgs, const FirstTile, const CUtensorMap) = conv_first_kernel<OUTB, KH, KW, S, TM>;
     if (tl.smem > configured) {
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tl.smem) != cudaSuccess)
             return MINW_ECUDA;
@@ -382,27 +483,72 @@ static minw_status launch_first_shape(const FirstArgs &a, const FirstTile &tl, c
     int gx = (2 * sms + octiles - 1) / octiles;
     if (gx > total) gx = total;
     const dim3 grid((unsigned)gx, (unsigned)octiles);
-    if (minw_host::launch_pdl(kern, grid, dim3(FIRST_NT), tl.smem, s, a, tl) != cudaSuccess) return MINW_ECUDA;
+    if (minw_host::launch_pdl(kern, grid, dim3(FIRST_NT), tl.smem, s, a, tl, tm) != cudaSuccess) return MINW_ECUDA;
     return MINW_OK;
 }
 
+static bool tma_shape(const FirstArgs &a) {
+    return (a.kh == 3 && a.kw == 3 && a.stride == 1) || (a.kh == 7 && a.kw == 7 && a.stride == 2);
+}
+
 template <int OUTB>
-static minw_status launch_first_bits(const FirstArgs &a, const FirstTile &tl, cudaStream_t s) {
-    if (a.kh == 3 && a.kw == 3 && a.stride == 1) return launch_first_shape<OUTB, 3, 3, 1>(a, tl, s);
-    if (a.kh == 7 && a.kw == 7 && a.stride == 2) return launch_first_shape<OUTB, 7, 7, 2>(a, tl, s);
-    return launch_first_shape<OUTB, 0, 0, 0>(a, tl, s);
+static minw_status launch_first_bits(const FirstArgs &a, const FirstTile &tl, const CUtensorMap &tm, cudaStream_t s) {
+    if (a.kh == 3 && a.kw == 3 && a.stride == 1)
+        return tl.tma ? launch_first_shape<OUTB, 3, 3, 1, true>(a, tl, tm, s)
+                      : launch_first_shape<OUTB, 3, 3, 1, false>(a, tl, tm, s);
+    if (a.kh == 7 && a.kw == 7 && a.stride == 2)
+        return tl.tma ? launch_first_shape<OUTB, 7, 7, 2, true>(a, tl, tm, s)
+                      : launch_first_shape<OUTB, 7, 7, 2, false>(a, tl, tm, s);
+    return launch_first_shape<OUTB, 0, 0, 0, false>(a, tl, tm, s);
+}
+
+// Patches by TMA (MINW_FIRST_TMA=0: per-word cp.async) where the image rows
+// are 16-byte multiples at a 16-byte aligned base and the box fits the limits.
+static bool first_tma_pref() {
+    static int v = -1;
+    if (v < 0) {
+        const char *e = getenv("MINW_FIRST_TMA");
+        v = (e && e[0] == '0') ? 0 : 1;
+    }
+    return v != 0;
+}
+
+int take_first_error() {
+    int flag = 0;
+    if (cudaMemcpyFromSymbol(&flag, g_first_error, sizeof(int)) != cudaSuccess) return -1;
+    if (flag) {
+        const int zero = 0;
+        if (cudaMemcpyToSymbol(g_first_error, &zero, sizeof(int)) != cudaSuccess) return -1;
+    }
+    return flag;
 }
 
 minw_status launch_conv_first(const FirstArgs &a, cudaStream_t s) {
-    const FirstTile tl = first_tile(a);
+    const bool tma_ok = first_tma_pref() && tma_shape(a) && a.W % 4 == 0 && minw_host::aligned16(a.x) &&
+                        minw_host::tensor_map_encoder() != nullptr;
+    FirstTile tl = first_tile(a, tma_ok);
+    CUtensorMap tm;
+    memset(&tm, 0, sizeof(tm));
+    if (tl.tma) {
+        const cuuint64_t dims[4] = {(cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.C, (cuuint64_t)a.B};
+        const cuuint64_t strides[3] = {(cuuint64_t)a.W * 4, (cuuint64_t)a.H * a.W * 4,
+                                       (cuuint64_t)a.C * a.H * a.W * 4};
+        const cuuint32_t box[4] = {(cuuint32_t)tl.RP, (cuuint32_t)tl.Rmax, (cuuint32_t)a.C, 1u};
+        const cuuint32_t es[4] = {1u, 1u, 1u, 1u};
+        if (minw_host::tensor_map_encoder()(&tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float *>(a.x), dims,
+                                            strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                            CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            tl = first_tile(a, false);
+    }
     if (tl.smem > 200 * 1024) return MINW_EUNSUPPORTED;
     if (a.codes_out != nullptr && a.O % 16 != 0) return MINW_EUNSUPPORTED;
     const int outb = a.quant_out ? a.qo.bits : 0;
     switch (outb) {
-        case 1: return launch_first_bits<1>(a, tl, s);
-        case 2: return launch_first_bits<2>(a, tl, s);
-        case 3: return launch_first_bits<3>(a, tl, s);
-        default: return launch_first_bits<0>(a, tl, s);
+        case 1: return launch_first_bits<1>(a, tl, tm, s);
+        case 2: return launch_first_bits<2>(a, tl, tm, s);
+        case 3: return launch_first_bits<3>(a, tl, tm, s);
+        default: return launch_first_bits<0>(a, tl, tm, s);
     }
 }
 

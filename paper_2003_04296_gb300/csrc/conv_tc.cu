@@ -1062,23 +1062,6 @@ __global__ void thresholds_kernel(const float *__restrict__ scale, const float *
 // host side
 // ---------------------------------------------------------------------------
 
-typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
-                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-static EncodeTiledFn encode_fn() {
-    static EncodeTiledFn fn = nullptr;
-    if (fn == nullptr) {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    }
-    return fn;
-}
-
 static int pow2_ceil(int v) {
     int p = 1;
     while (p < v) p <<= 1;
@@ -1275,7 +1258,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
         p.cl = cl;
     }
     p.tiles_mp = (tiles_m + p.cl - 1) / p.cl * p.cl;
-    EncodeTiledFn enc = encode_fn();
+    minw_host::EncodeTiledFn enc = minw_host::tensor_map_encoder();
     if (enc == nullptr) return MINW_ECUDA;
     const CUtensorMapSwizzle swz = p.ck == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
     {
@@ -1458,7 +1441,21 @@ extern "C" minw_status minw_get_last_device_error(void *stream) {
     if (flag) {
         const int zero = 0;
         if (cudaMemcpyToSymbol(minw::g_device_error, &zero, sizeof(int)) != cudaSuccess) return MINW_ECUDA;
-        return MINW_ETIMEOUT;
     }
-    return MINW_OK;
+    const int first = minw::take_first_error();
+    if (first < 0) return MINW_ECUDA;
+    return (flag || first) ? MINW_ETIMEOUT : MINW_OK;
+}
+
+minw_host::EncodeTiledFn minw_host::tensor_map_encoder() {
+    static EncodeTiledFn fn = nullptr;
+    if (fn == nullptr) {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    }
+    return fn;
 }

@@ -59,6 +59,8 @@ struct FirstArgs {
 
 // Launchers (host).  Return MINW_OK or an error status.
 minw_status launch_conv_first(const FirstArgs &a, cudaStream_t s);
+// The first-layer kernels' timeout flag: 1 if set (and clears it), 0, or -1 on a CUDA error.
+int take_first_error();
 minw_status launch_ythresholds(const QParams &q, float *out, cudaStream_t s);
 minw_status launch_first_weights(const float *w, int O, int K, int quant_w, const QParams &qw, const float *cscale,
                                  float *wt, cudaStream_t s);
