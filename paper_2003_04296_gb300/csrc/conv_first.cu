@@ -30,6 +30,11 @@ __device__ __forceinline__ unsigned long long dup2(float x) {
 __device__ __forceinline__ void ffma2(unsigned long long &acc, unsigned long long a, unsigned long long b) {
     asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(acc) : "l"(a), "l"(b));
 }
+__device__ __forceinline__ unsigned long long fma2(unsigned long long a, unsigned long long b, unsigned long long c) {
+    unsigned long long d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
 __device__ __forceinline__ float lane2(unsigned long long v, int hi) {
     float lo_, hi_;
     asm("mov.b64 {%0, %1}, %2;" : "=f"(lo_), "=f"(hi_) : "l"(v));
@@ -41,6 +46,11 @@ __device__ __forceinline__ float lane2(unsigned long long v, int hi) {
 __device__ __forceinline__ float lds_f32(uint32_t a) {
     float v;
     asm volatile("ld.shared.f32 %0, [%1];\n" : "=f"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ unsigned long long lds_u64(uint32_t a) {
+    unsigned long long v;
+    asm volatile("ld.shared.u64 %0, [%1];\n" : "=l"(v) : "r"(a));
     return v;
 }
 __device__ __forceinline__ void lds_2x64(uint32_t a, unsigned long long &x, unsigned long long &y) {
@@ -180,7 +190,7 @@ __global__ void __launch_bounds__(FIRST_NT, 2)
     const int OCB = tl.OCB, K = tl.K, RP = tl.RP, Ws = tl.Ws;
     const size_t patch = (size_t)tl.pstride;
     float *sW = reinterpret_cast<float *>(smem4);                 // [K][OCB]
-    float *sT = sW + (size_t)K * OCB;                             // [OCB][8] -breakpoints, sigma
+    float *sT = sW + (size_t)K * OCB;                             // [8][OCB] -breakpoints, sigma (row 7)
     float *sX0 = sW + tl.xoff;                                    // [nb][C][Rmax][RP]
     uint64_t *fullb = reinterpret_cast<uint64_t *>(sX0 + (size_t)tl.nb * patch);   // [nb] TMA patch arrivals
 
@@ -240,7 +250,7 @@ __global__ void __launch_bounds__(FIRST_NT, 2)
     }
     // breakpoints held for the mask test: (-T_1 .. -T_{n-1}, sigma); padding channels never reached
     if (a.quant_out && threadIdx.x < OCB) {
-        float *th = sT + threadIdx.x * 8;
+        float th[8];
         const int o = o0 + threadIdx.x;
         const int nl = num_levels(a.qo.bits);
         if (threadIdx.x >= ochan) {
@@ -254,6 +264,9 @@ __global__ void __launch_bounds__(FIRST_NT, 2)
             }
             for (int u = 0; u < nl - 1; ++u) th[u] = mask_breakpoint(th[u]);
         }
+        // channel-fastest rows (a channel pair is one 64-bit word); sigma in row 7
+        for (int u = 0; u < nl - 1; ++u) sT[u * OCB + threadIdx.x] = th[u];
+        sT[7 * OCB + threadIdx.x] = th[nl - 1];
     }
 
     if (TM && threadIdx.x == 0) {
@@ -374,24 +387,26 @@ __global__ void __launch_bounds__(FIRST_NT, 2)
             }
             if constexpr (OUTB > 0) {
                 // level masks of this half's 16 channels: bit oc of M = [sigma * acc < T_u], from the
-                // sign of fmaf(acc, sigma, -T_u); then the two halves make the 32-channel word
-                const float *thb = sT + (g * 32 + 16 * h) * 8;
+                // sign of fmaf(acc, sigma, -T_u) (one packed fma.rn.f32x2 per channel pair); then the
+                // two halves make the 32-channel word
+                const uint32_t tb = (uint32_t)__cvta_generic_to_shared(sT + g * 32 + 16 * h);
                 uint32_t MM[FIRST_PX][NL - 1];
 #pragma unroll
                 for (int i = 0; i < FIRST_PX; ++i)
 #pragma unroll
                     for (int u = 0; u < NL - 1; ++u) MM[i][u] = 0u;
 #pragma unroll
-                for (int oc = 15; oc >= 0; --oc) {
-                    const float *th = thb + oc * 8;
-                    const float sg = th[NL - 1];
+                for (int j = 7; j >= 0; --j) {                   // channels 2j + 1, 2j (high bit first)
+                    const unsigned long long sg = lds_u64(tb + 4u * (uint32_t)(7 * OCB + 2 * j));
 #pragma unroll
                     for (int u = 0; u < NL - 1; ++u) {
-                        const float nt = th[u];
+                        const unsigned long long nt = lds_u64(tb + 4u * (uint32_t)(u * OCB + 2 * j));
 #pragma unroll
-                        for (int i = 0; i < FIRST_PX; ++i)
-                            MM[i][u] = __funnelshift_l(__float_as_uint(fmaf(lane2(acc[i][oc >> 1], oc & 1), sg, nt)),
-                                                       MM[i][u], 1);
+                        for (int i = 0; i < FIRST_PX; ++i) {
+                            const unsigned long long r = fma2(acc[i][j], sg, nt);
+                            MM[i][u] = __funnelshift_l(__float_as_uint(lane2(r, 1)), MM[i][u], 1);
+                            MM[i][u] = __funnelshift_l(__float_as_uint(lane2(r, 0)), MM[i][u], 1);
+                        }
                     }
                 }
 #pragma unroll
