@@ -68,6 +68,8 @@ struct Params {
     int nlev;                  // levels of the output quantizer
     int ksplit;                // K slices per output tile (1: no split)
     int cl;                    // CTAs per cluster sharing each weight box (1, 2 or 4; 1 when split)
+    int pair;                  // CTA pairs (cl = 2): one cta_group::2 MMA of M = 256 pixels per pair, each
+                               // CTA holding its 128 pixels and half of the weight rows
     int tiles_mp;              // pixel tiles per channel tile, padded to a multiple of cl
     int32_t *part;             // split-K: int32 partial sums [ksplit][tiles][128][BN]
     // residual blocks: y = BN(acc) + shortcut, then HardTanh + quantize
@@ -203,6 +205,76 @@ __device__ __forceinline__ void mma_commit_mc(uint64_t *bar, uint16_t mask) {
             smem_u32(bar)),
         "h"(mask)
         : "memory");
+}
+
+// CTA pairs (cta_group::2).  The even CTA of a cluster of two issues each MMA
+// for both: A = the pair's 256 pixel rows (128 in each CTA's shared memory),
+// B = the 256 weight rows (128 in each), D = 128 accumulator lanes in each
+// CTA's tensor memory.  Loads of both CTAs complete on the even CTA's barrier.
+__device__ __forceinline__ void mma_f8_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                            uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
+}
+
+// Arrive on the barrier at this offset in both CTAs of the pair once the
+// pair's MMAs issued so far have completed.
+__device__ __forceinline__ void mma_commit_pair(uint64_t *bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n" ::"r"(
+            smem_u32(bar)),
+        "h"((uint16_t)3)
+        : "memory");
+}
+
+// Shared::cluster address of the object at this offset in CTA 0 of the cluster.
+__device__ __forceinline__ uint32_t cta0_addr(const void *p) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, 0;\n" : "=r"(r) : "r"(smem_u32(p)));
+    return r;
+}
+
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];\n" ::"r"(cluster_addr) : "memory");
+}
+
+// Tile loads of a pair: into this CTA's shared memory, completing on the
+// barrier at a shared::cluster address (the even CTA's).
+__device__ __forceinline__ void tma_load_4d_pair(void *dst, const CUtensorMap *map, uint32_t bar, int c0, int c1,
+                                                 int c2, int c3) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6];\n" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void tma_load_2d_pair(void *dst, const CUtensorMap *map, uint32_t bar, int c0, int c1) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];\n" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
+        : "memory");
+}
+
+// Bounded wait with cluster-scope acquire (arrivals from the other CTA of a pair).
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity) {
+    const long long t0 = clock64();
+    while (true) {
+        uint32_t ok;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, 100000;\n"
+            " selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(ok)
+            : "r"(smem_u32(bar)), "r"(parity)
+            : "memory");
+        if (ok) return true;
+        if (clock64() - t0 > WAIT_CYCLES) {
+            atomicExch(&g_device_error, 1);
+            return false;
+        }
+    }
 }
 
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
@@ -393,7 +465,8 @@ __device__ __forceinline__ void resid_chunk(uint32_t taddr, bool full32, const P
 }
 
 // OUTB: bits of the quantized output (0 when the launch writes none).
-template <int OUTB>
+// PAIR: CTA pairs with cta_group::2 MMAs (a kernel uses one CTA group only).
+template <int OUTB, bool PAIR>
 __global__ void __launch_bounds__(NT, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const Params p) {
@@ -429,19 +502,27 @@ __global__ void __launch_bounds__(NT, 1)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < p.S; ++s) {
-            mbar_init(&full[s], 2);               // one arrival per TMA issuing warp
-            mbar_init(&empty[s], p.cl);           // one release per CTA reading the weight box
+            mbar_init(&full[s], 2);               // one arrival per TMA issuing warp (pairs: CTA 0's)
+            mbar_init(&empty[s], PAIR ? 1 : p.cl);   // one release per CTA reading the weight box
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
-            mbar_init(&tempty[i], EPI_WARPS);
+            mbar_init(&tempty[i], PAIR ? 2 * EPI_WARPS : EPI_WARPS);   // pairs: both CTAs' epilogues
         }
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(tmem_slot)),
-                     "r"(p.tmem_cols));
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n");
+        if constexpr (PAIR) {      // one warp of each CTA of the pair allocates the same columns in both
+            asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(
+                             smem_u32(tmem_slot)),
+                         "r"(p.tmem_cols));
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;\n");
+        } else {
+            asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(
+                             smem_u32(tmem_slot)),
+                         "r"(p.tmem_cols));
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n");
+        }
     }
     // output-quantizer breakpoints of every channel, in shared memory
     if constexpr (OUTB > 0) {
@@ -500,6 +581,9 @@ __global__ void __launch_bounds__(NT, 1)
             asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
             const uint32_t bytes = act ? p.a_bytes : p.b_bytes;   // per K block; weights: all cl slices
             const int bslice = p.BN / p.cl;        // weight rows this CTA loads (and multicasts)
+            // pairs: this operand's loads of both CTAs complete on CTA 0's barrier, whose
+            // producers alone arrive (expecting both CTAs' bytes)
+            const bool arrive = !PAIR || crank == 0;
             int g = 0, s = 0, lap = 0;             // stages issued, ring slot, ring lap
             bool alive = true;
             for (int w = blockIdx.x; w < items && alive; w += gridDim.x) {
@@ -518,9 +602,16 @@ __global__ void __launch_bounds__(NT, 1)
                     if (lap > 0 && !mbar_wait(&empty[s], (lap - 1) & 1)) { alive = false; break; }
                     uint8_t *sa = smem + (size_t)s * p.stage_bytes;
                     const int n = min(p.kps, ke - ks);            // K blocks in this stage
-                    mbar_expect_tx(&full[s], (uint32_t)n * bytes);
+                    if (arrive) mbar_expect_tx(&full[s], (uint32_t)n * bytes * (PAIR ? 2u : 1u));
+                    const uint32_t fb = PAIR ? cta0_addr(&full[s]) : 0u;
                     for (int j = 0; j < n; ++j) {
-                        if (act)
+                        if constexpr (PAIR) {
+                            if (act)
+                                tma_load_4d_pair(sa + (size_t)j * p.a_bytes, &tmA, fb, c0, x0 + kx, y0 + ky, b0);
+                            else
+                                tma_load_2d_pair(sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes, &tmB, fb,
+                                                 kcol, o0 + crank * bslice);
+                        } else if (act)
                             tma_load_4d(sa + (size_t)j * p.a_bytes, &tmA, &full[s], c0, x0 + kx, y0 + ky, b0);
                         else if (p.cl == 1)
                             tma_load_2d(sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes, &tmB, &full[s], kcol, o0);
@@ -538,18 +629,20 @@ __global__ void __launch_bounds__(NT, 1)
                     if (++s == p.S) { s = 0; ++lap; }
                 }
             }
-            // drain: every issued load has landed before the CTA can exit
+            // drain: every issued load has landed before the CTA can exit (pairs: the
+            // MMAs that read the last stages have completed)
             for (int j = g > p.S ? g - p.S : 0; j < g; ++j)
-                if (!mbar_wait(&full[j % p.S], (j / p.S) & 1)) break;
+                if (!(PAIR ? mbar_wait(&empty[j % p.S], (j / p.S) & 1) : mbar_wait(&full[j % p.S], (j / p.S) & 1)))
+                    break;
             // clusters: every CTA's release of every slot has arrived here too
             // (no remote arrival may reach this shared memory after exit)
-            if (p.cl > 1 && !act)
+            if (p.cl > 1 && !act && !PAIR)
                 for (int j = g > p.S ? g - p.S : 0; j < g; ++j)
                     if (!mbar_wait(&empty[j % p.S], (j / p.S) & 1)) break;
         }
     } else if (warp == 1) {
-        if (lane == 0) {
-            // ---------------- MMA issuer ----------------
+        if (lane == 0 && (!PAIR || crank == 0)) {
+            // ---------------- MMA issuer (pairs: CTA 0 issues for both) ----------------
             int s = 0, i = 0;
             uint32_t fphase = 0;
             bool alive = true;
@@ -567,10 +660,18 @@ __global__ void __launch_bounds__(NT, 1)
                 const int ab = i & 1, use = i >> 1;
                 const int t = w / p.ksplit, kp = w - t * p.ksplit;
                 const int kb = (int)((long long)kp * p.nk / p.ksplit), ke = (int)((long long)(kp + 1) * p.nk / p.ksplit);
-                if (use > 0 && !mbar_wait(&tempty[ab], (use - 1) & 1)) break;
+                if (use > 0 && !(PAIR ? mbar_wait_cluster(&tempty[ab], (use - 1) & 1)
+                                        : mbar_wait(&tempty[ab], (use - 1) & 1)))
+                    break;
                 fence_after();
                 const uint32_t tmem_d = tmem_base + (uint32_t)(ab * p.acc_cols);
                 uint32_t acc = 0u;
+                auto mma = [&](uint64_t ad_, uint64_t bd_, uint32_t a_) {
+                    if constexpr (PAIR)
+                        mma_f8_pair(tmem_d, ad_, bd_, idesc, a_);
+                    else
+                        mma_f8(tmem_d, ad_, bd_, idesc, a_);
+                };
                 for (int ks = kb; ks < ke; ks += p.kps) {
                     if (!mbar_wait(&full[s], fphase)) { alive = false; break; }
                     fence_after();
@@ -582,30 +683,35 @@ __global__ void __launch_bounds__(NT, 1)
                         bd = t_;
                     }
                     const uint32_t as_ = p.trans ? bstep : astep, bs_ = p.trans ? astep : bstep;
-                    mma_f8(tmem_d, ad, bd, idesc, acc);
-                    mma_f8(tmem_d, ad + 2, bd + 2, idesc, 1u);
+                    mma(ad, bd, acc);
+                    mma(ad + 2, bd + 2, 1u);
                     if (k128) {
-                        mma_f8(tmem_d, ad + 4, bd + 4, idesc, 1u);
-                        mma_f8(tmem_d, ad + 6, bd + 6, idesc, 1u);
+                        mma(ad + 4, bd + 4, 1u);
+                        mma(ad + 6, bd + 6, 1u);
                     }
                     if (p.kps == 2 && ks + 1 < ke) {
                         ad += as_;
                         bd += bs_;
-                        mma_f8(tmem_d, ad, bd, idesc, 1u);
-                        mma_f8(tmem_d, ad + 2, bd + 2, idesc, 1u);
+                        mma(ad, bd, 1u);
+                        mma(ad + 2, bd + 2, 1u);
                         if (k128) {
-                            mma_f8(tmem_d, ad + 4, bd + 4, idesc, 1u);
-                            mma_f8(tmem_d, ad + 6, bd + 6, idesc, 1u);
+                            mma(ad + 4, bd + 4, 1u);
+                            mma(ad + 6, bd + 6, 1u);
                         }
                     }
                     acc = 1u;
-                    if (p.cl == 1)
+                    if constexpr (PAIR)
+                        mma_commit_pair(&empty[s]);              // both CTAs' slots are free
+                    else if (p.cl == 1)
                         mma_commit(&empty[s]);
                     else
                         mma_commit_mc(&empty[s], cmask);     // the slot is free in every CTA's view
                     if (++s == p.S) { s = 0; fphase ^= 1; }
                 }
-                mma_commit(&tfull[ab]);
+                if constexpr (PAIR)
+                    mma_commit_pair(&tfull[ab]);
+                else
+                    mma_commit(&tfull[ab]);
             }
         }
     } else if (warp < B_WARP) {
@@ -625,6 +731,13 @@ __global__ void __launch_bounds__(NT, 1)
         // mask epilogue (a layer whose only output is the next layer's levels):
         // this warp's 32-column chunks
         const bool resid = p.res_codes != nullptr || p.res_f32 != nullptr || p.y_nhwc != nullptr;
+        // the accumulator is drained: CTA 1 of a pair tells CTA 0, which issues the MMAs
+        auto tempty_arrive = [&](uint64_t *bar) {
+            if (PAIR && crank == 1)
+                mbar_arrive_cluster(cta0_addr(bar));
+            else
+                mbar_arrive(bar);
+        };
         const bool masked = OUTB > 0 && p.ksplit == 1 && p.acc_out == nullptr && p.y_out == nullptr && !resid;
         // residual epilogue without per-element fp32 outputs: the same chunks
         const bool rmasked = p.ksplit == 1 && p.acc_out == nullptr && p.y_out == nullptr && !p.pool && resid &&
@@ -733,7 +846,7 @@ __global__ void __launch_bounds__(NT, 1)
                     }
                     fence_before();
                     __syncwarp();
-                    if (lane == 0 && !dead) mbar_arrive(&tempty[ab]);
+                    if (lane == 0 && !dead) tempty_arrive(&tempty[ab]);
                 }
             }
         }
@@ -768,7 +881,7 @@ __global__ void __launch_bounds__(NT, 1)
                     }
                     fence_before();
                     __syncwarp();
-                    if (lane == 0 && !dead) mbar_arrive(&tempty[ab]);
+                    if (lane == 0 && !dead) tempty_arrive(&tempty[ab]);
                     continue;
                 }
             }
@@ -784,7 +897,7 @@ __global__ void __launch_bounds__(NT, 1)
                 }
                 fence_before();
                 __syncwarp();
-                if (lane == 0 && !dead) mbar_arrive(&tempty[ab]);
+                if (lane == 0 && !dead) tempty_arrive(&tempty[ab]);
                 continue;
             }
 
@@ -938,15 +1051,24 @@ __global__ void __launch_bounds__(NT, 1)
             }
             fence_before();
             __syncwarp();
-            if (lane == 0 && !dead) mbar_arrive(&tempty[ab]);      // the accumulator can be reused
+            if (lane == 0 && !dead) tempty_arrive(&tempty[ab]);      // the accumulator can be reused
         }
     }
     __syncthreads();
-    if (warp == 1) {
-        fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(p.tmem_cols));
+    if constexpr (PAIR) {
+        // both CTAs are done with the pair's tensor memory and barriers; one warp of each frees it
+        cluster_sync_all();
+        if (warp == 1) {
+            fence_after();
+            asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(p.tmem_cols));
+        }
+    } else {
+        if (warp == 1) {
+            fence_after();
+            asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(p.tmem_cols));
+        }
+        if (p.cl > 1) cluster_sync_all();         // no CTA leaves while a peer may still address it
     }
-    if (p.cl > 1) cluster_sync_all();         // no CTA leaves while a peer may still address it
 }
 
 // Split-K second pass: sums the K slices of every accumulator and runs the
@@ -1120,6 +1242,19 @@ static int cluster_pref() {
     return v;
 }
 
+// CTA pairs with cta_group::2 MMAs for 256-channel layers with long K loops
+// (MINW_TC_PAIR = 0 turns them off).  Each CTA then loads half the weight
+// rows per K block, and one MMA instruction covers both SMs; short K loops
+// (< 18 K blocks) measured faster single.
+static int pair_pref() {
+    static int v = -1;
+    if (v < 0) {
+        const char *e = getenv("MINW_TC_PAIR");
+        v = (e && e[0] == '0') ? 0 : 1;
+    }
+    return v;
+}
+
 // K blocks per stage the kernel may use (MINW_TC_KPS = 1 keeps one; 2 by default).
 static int kps_pref() {
     static int v = -1;
@@ -1199,7 +1334,15 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     p.ntn = (a.O + p.BN - 1) / p.BN;
     p.nlev = a.quant_out ? num_levels(a.qo.bits) : 0;
     p.thr = a.thr;
-    p.b_bytes = (uint32_t)(p.BN * p.ck);
+    // CTA pairs (MINW_TC_PAIR): 256-channel tiles of a layer that is not split along K
+    {
+        const int sms_ = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
+        const int tiles_ = p.nbx * p.nby * p.nbb * p.ntn;
+        const int ks_ = (a.workspace != nullptr && !a.pool) ? (a.ksplit > 0 ? a.ksplit : auto_ksplit(tiles_, p.nk, sms_))
+                                                            : 1;
+        p.pair = (pair_pref() && !p.trans && p.BN == 256 && a.O % 256 == 0 && p.nk >= 18 && ks_ <= 1) ? 1 : 0;
+    }
+    p.b_bytes = (uint32_t)((p.pair ? p.BN / 2 : p.BN) * p.ck);   // pairs: each CTA holds half the weight rows
     const size_t o32 = ((size_t)a.O + 31) & ~(size_t)31;
     const size_t thr_bytes = a.quant_out ? (o32 * p.nlev + o32 / 32 + 10) * sizeof(float) : 0;
     const size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes;
@@ -1214,7 +1357,8 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     // MMA N: the output channels, or the 256 pixels of a channel-major tile (M = 128 either way)
     const int mma_n = p.trans ? 256 : p.BN;
     p.acc_cols = mma_n;
-    p.idesc = (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(mma_n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+    p.idesc = (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(mma_n >> 3) << 17) |
+              ((uint32_t)((p.pair ? 256 : 128) >> 4) << 24);
     uint32_t cols = 32;
     while ((int)cols < 2 * mma_n) cols <<= 1;         // two accumulators
     p.tmem_cols = cols;
@@ -1228,7 +1372,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
     p.ksplit = 1;
     pl.thr_ws = nullptr;
-    if (a.workspace != nullptr && !a.pool && !p.trans) {
+    if (a.workspace != nullptr && !a.pool && !p.trans && !p.pair) {
         // workspace: [breakpoints, when not given][ksplit partial-sum slices]
         const size_t tb = (a.quant_out && a.thr == nullptr) ? thr_ws_bytes(a.O, p.nlev) : 0;
         const size_t sb = slice_bytes(tiles, p.BN);
@@ -1251,8 +1395,8 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     // of one channel tile together; each loads BN / cl weight rows for all
     // (padding the pixel tiles to a multiple of cl may add at most 1/8)
     const int tiles_m = p.nbx * p.nby * p.nbb;
-    p.cl = 1;
-    if (p.ksplit == 1 && !p.trans) {
+    p.cl = p.pair ? 2 : 1;
+    if (p.ksplit == 1 && !p.trans && !p.pair) {
         int cl = cl_max;
         while (cl > 1 && (p.BN % (8 * cl) != 0 || ((tiles_m + cl - 1) / cl * cl - tiles_m) * 8 > tiles_m)) cl >>= 1;
         p.cl = cl;
@@ -1375,13 +1519,20 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
     const bool split = pl.p.ksplit > 1;
     const int kout = split ? 0 : outb;            // the split main pass writes only partial sums
     static size_t configured[4] = {0, 0, 0, 0};
-    void (*kern)(const CUtensorMap, const CUtensorMap, const tc::Params) =
-        kout == 1 ? tc::conv_tc_kernel<1> : kout == 2 ? tc::conv_tc_kernel<2> : kout == 3 ? tc::conv_tc_kernel<3>
-                                                                                         : tc::conv_tc_kernel<0>;
-    if (pl.smem > configured[kout]) {
+    typedef void (*TcKernel)(const CUtensorMap, const CUtensorMap, const tc::Params);
+    static const TcKernel kernels[2][4] = {
+        {tc::conv_tc_kernel<0, false>, tc::conv_tc_kernel<1, false>, tc::conv_tc_kernel<2, false>,
+         tc::conv_tc_kernel<3, false>},
+        {tc::conv_tc_kernel<0, true>, tc::conv_tc_kernel<1, true>, tc::conv_tc_kernel<2, true>,
+         tc::conv_tc_kernel<3, true>}};
+    static size_t configured_pair[4] = {0, 0, 0, 0};
+    const int kp = pl.p.pair ? 1 : 0;
+    TcKernel kern = kernels[kp][kout];
+    size_t &conf = kp ? configured_pair[kout] : configured[kout];
+    if (pl.smem > conf) {
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem) != cudaSuccess)
             return MINW_ECUDA;
-        configured[kout] = pl.smem;
+        conf = pl.smem;
     }
     const float *thr = a.thr;
     if (split && a.quant_out && thr == nullptr && !conv_tc_residual(a)) {

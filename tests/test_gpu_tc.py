@@ -291,7 +291,7 @@ def test_weight_multicast_clusters(dev, cl):
     (MINW_TC_CLUSTER, read once per process): the CIFAR-layer shapes still match
     the oracle bit for bit.  Batch 26 leaves 13 pixel tiles in the 8x8 layers,
     so one cluster also walks a padding tile.  Runs in a child process with the
-    variable set."""
+    variable set (and CTA pairs off, which would take the 256-channel layers)."""
     import subprocess
     import sys
     code = (
@@ -310,7 +310,7 @@ def test_weight_multicast_clusters(dev, cl):
         "assert np.array_equal(out.cpu().numpy(), N.convnet_forward(p, x))\n"
         "print('ok')\n")
     import os
-    env = dict(os.environ, MINW_TC_CLUSTER=str(cl))
+    env = dict(os.environ, MINW_TC_CLUSTER=str(cl), MINW_TC_PAIR="0")
     root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
     r = subprocess.run([sys.executable, "-c", code], cwd=root, env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stderr[-2000:]
