@@ -343,10 +343,11 @@ __device__ __forceinline__ uint32_t transpose32(uint32_t a, int lane) {
 // level index is k = #{u : bit clear}.  A 2x2 max pool of the accumulators
 // maps to the masks: for sigma = +1 the pooled level is the window's largest
 // (M pooled = AND over the window), for sigma = -1 its smallest (OR).  Bit
-// planes and E4M3 codes follow from the masks with bitwise logic.
+// planes and E4M3 codes follow from the masks with bitwise logic.  th: the
+// chunk's first channel in rows of tstride floats (-T_1 .. -T_{n-1}, sigma).
 template <int OUTB>
-__device__ __forceinline__ void mask_chunk(uint32_t taddr, bool full32, const float *th, uint32_t sig, int pool,
-                                           int bw, bool writer, int nvalid, uint32_t *planes, int NWo,
+__device__ __forceinline__ void mask_chunk(uint32_t taddr, bool full32, const float *th, int tstride, uint32_t sig,
+                                           int pool, int bw, bool writer, int nvalid, uint32_t *planes, int NWo,
                                            uint8_t *codes) {
     constexpr int NL = OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7);
     uint32_t v[32];
@@ -364,13 +365,23 @@ __device__ __forceinline__ void mask_chunk(uint32_t taddr, bool full32, const fl
     uint32_t M[NL - 1];
 #pragma unroll
     for (int u = 0; u < NL - 1; ++u) M[u] = 0u;
+    // breakpoints of four channels per 128-bit load (rows of tstride floats, channel fastest)
 #pragma unroll
-    for (int j = 31; j >= 0; --j) {
-        const float a = __uint_as_float(v[j]);
-        const float sg = th[j * NL + NL - 1];
+    for (int j4 = 7; j4 >= 0; --j4) {
+        const float4 sg4 = *reinterpret_cast<const float4 *>(th + (NL - 1) * tstride + 4 * j4);
+        float4 nt4[NL - 1];
 #pragma unroll
-        for (int u = 0; u < NL - 1; ++u)
-            M[u] = __funnelshift_l(__float_as_uint(fmaf(a, sg, th[j * NL + u])), M[u], 1);
+        for (int u = 0; u < NL - 1; ++u) nt4[u] = *reinterpret_cast<const float4 *>(th + u * tstride + 4 * j4);
+        const float sg[4] = {sg4.x, sg4.y, sg4.z, sg4.w};
+#pragma unroll
+        for (int jj = 3; jj >= 0; --jj) {
+            const float a = __uint_as_float(v[4 * j4 + jj]);
+#pragma unroll
+            for (int u = 0; u < NL - 1; ++u) {
+                const float nt = jj == 0 ? nt4[u].x : jj == 1 ? nt4[u].y : jj == 2 ? nt4[u].z : nt4[u].w;
+                M[u] = __funnelshift_l(__float_as_uint(fmaf(a, sg[jj], nt)), M[u], 1);
+            }
+        }
     }
     if (pool) {
 #pragma unroll
@@ -475,8 +486,8 @@ __global__ void __launch_bounds__(NT, 1)
     // pointer arithmetic on the shared array keeps the shared address space
     uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     constexpr int NL = OUTB == 0 ? 1 : (OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7));
-    // breakpoints [O32][NL] (channels padded to a multiple of 32), then the
-    // per-32-channel masks of channels with sigma = +1
+    // breakpoints [NL][O32] (channels padded to a multiple of 32, channel
+    // fastest), then the per-32-channel masks of channels with sigma = +1
     const int O32 = (p.O + 31) & ~31;
     float *sthr = reinterpret_cast<float *>(smem + (size_t)p.S * p.stage_bytes);
     const int thr_floats = OUTB ? O32 * NL : 0;
@@ -528,21 +539,25 @@ __global__ void __launch_bounds__(NT, 1)
     if constexpr (OUTB > 0) {
         // held as (-T_1 .. -T_{n-1}, sigma) with -0 stored as +0, so that
         // fmaf(acc, sigma, -T) is never -0 and its sign bit is [sigma * acc < T]
+        // rows u = 0 .. NL - 1 of O32 channels each (channel fastest: four channels per 128-bit load)
         if (p.thr != nullptr) {
             for (int i = threadIdx.x; i < p.O * NL; i += NT) {
                 const float x = __ldg(p.thr + i);
-                sthr[i] = (i % NL == NL - 1) ? x : mask_breakpoint(x);
+                const int o = i / NL, u = i - o * NL;
+                sthr[u * O32 + o] = (u == NL - 1) ? x : mask_breakpoint(x);
             }
         } else if (p.res_codes == nullptr && p.res_f32 == nullptr) {
             // (a residual block quantizes y + shortcut: no per-channel breakpoints on acc)
             for (int o = threadIdx.x; o < p.O; o += NT) {
-                float *t = sthr + o * NL;
+                float t[8];
                 channel_thresholds(__ldg(p.scale + o), __ldg(p.shift + o), p.qo, t);
-                for (int u = 0; u < NL - 1; ++u) t[u] = mask_breakpoint(t[u]);
+                for (int u = 0; u < NL; ++u) sthr[u * O32 + o] = (u == NL - 1) ? t[u] : mask_breakpoint(t[u]);
             }
         }
-        for (int i = p.O * NL + threadIdx.x; i < thr_floats; i += NT)        // padding channels
-            sthr[i] = ((i % NL) == NL - 1) ? 1.0f : 0.0f;
+        for (int i = p.O * NL + threadIdx.x; i < thr_floats; i += NT) {      // padding channels
+            const int k = i - p.O * NL, o = p.O + k / NL, u = k % NL;
+            sthr[u * O32 + o] = (u == NL - 1) ? 1.0f : 0.0f;
+        }
         if (p.res_codes != nullptr || p.res_f32 != nullptr) {       // level of y = #{u : y >= T_u}
             if (p.ythr != nullptr) {
                 if (threadIdx.x < NL - 1) syt[threadIdx.x] = mask_breakpoint(__ldg(p.ythr + threadIdx.x));
@@ -763,8 +778,8 @@ __global__ void __launch_bounds__(NT, 1)
                     for (int u = 0; u < NL - 1; ++u) nt[u] = 0.0f;
                     if (qlive) {
 #pragma unroll
-                        for (int u = 0; u < NL - 1; ++u) nt[u] = sthr[oc * NL + u];
-                        sg = sthr[oc * NL + NL - 1];
+                        for (int u = 0; u < NL - 1; ++u) nt[u] = sthr[u * O32 + oc];
+                        sg = sthr[(NL - 1) * O32 + oc];
                         sig = ssig[(tn * p.BN + oq) >> 5];
                     }
                     if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
@@ -874,7 +889,7 @@ __global__ void __launch_bounds__(NT, 1)
                         if (ob >= p.O) break;                      // no channel of this tile left
                         __syncwarp();
                         mask_chunk<OUTB>(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * p.BN + c * 32),
-                                         c * 32 + 32 <= p.BN, sthr + ob * NL, p.pool ? ssig[ob >> 5] : 0u, p.pool,
+                                         c * 32 + 32 <= p.BN, sthr + ob, O32, p.pool ? ssig[ob >> 5] : 0u, p.pool,
                                          p.bw, writer, p.O - ob,
                                          p.planes_out ? p.planes_out + (opix * OUTB) * NWo + (ob >> 5) : nullptr,
                                          NWo, p.codes_out ? p.codes_out + opix * p.O + ob : nullptr);
@@ -979,11 +994,10 @@ __global__ void __launch_bounds__(NT, 1)
 #pragma unroll
                         for (int j = 0; j < 16; ++j) {
                             const int o = min(ob + j, p.O - 1);
-                            const float *th = sthr + o * NL;
-                            const float vv = a[j] * th[NL - 1];
+                            const float vv = a[j] * sthr[(NL - 1) * O32 + o];
                             int k = 0;
 #pragma unroll
-                            for (int u = 0; u < NL - 1; ++u) k += (vv + th[u] >= 0.0f) ? 1 : 0;   // th = -T
+                            for (int u = 0; u < NL - 1; ++u) k += (vv + sthr[u * O32 + o] >= 0.0f) ? 1 : 0;   // -T
                             kq[j] = k;
                         }
                         if (p.codes_out != nullptr) {

@@ -51,38 +51,43 @@ __device__ __forceinline__ uint32_t ordered_to_codes(uint32_t o) {
 // 3x3 / stride 2 / pad 1 pooling of level codes [B][H][W][C] -> [B][Ho][Wo][C]:
 // per channel the max of the levels when the stem's BN scale is >= 0, the min
 // otherwise (padded taps skipped).  Thread = one output pixel x 16 channels;
-// the codes are compared as order-preserving bytes, four per word.
+// the codes are compared as order-preserving bytes, four per word.  Index
+// arithmetic in 32 bits (the host keeps B Ho Wo C / 16 below 2^31); the
+// max/min byte selectors of each channel group sit in shared memory.
 __global__ void __launch_bounds__(256) pool_levels_kernel(const uint8_t *__restrict__ in, int B, int H, int W, int C,
                                                           const float *__restrict__ scale, uint8_t *__restrict__ out,
                                                           int Ho, int Wo) {
+    __shared__ uint32_t sup[64];                     // C / 4 words: 0xFF bytes where the scale is >= 0
+    for (int i = threadIdx.x; i < (C >> 2); i += blockDim.x) {
+        uint32_t m = 0u;
+        for (int j = 0; j < 4; ++j) m |= (__ldg(scale + 4 * i + j) >= 0.0f ? 0xFFu : 0u) << (8 * j);
+        sup[i] = m;
+    }
+    __syncthreads();
     pdl_wait();
     pdl_trigger();
-    const int groups = C >> 4;
-    const long long total = (long long)B * Ho * Wo * groups;
-    for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-         t += (long long)gridDim.x * blockDim.x) {
-        const int g = (int)(t % groups);
-        const long long pix = t / groups;
-        const int xo = (int)(pix % Wo);
-        const int yo = (int)((pix / Wo) % Ho);
-        const int b = (int)(pix / ((long long)Wo * Ho));
-        uint32_t up[4], mx[4], mn[4];
+    const unsigned groups = (unsigned)C >> 4;
+    const unsigned total = (unsigned)B * (unsigned)Ho * (unsigned)Wo * groups;
+    for (unsigned t = blockIdx.x * blockDim.x + threadIdx.x; t < total; t += gridDim.x * blockDim.x) {
+        const unsigned g = t % groups, pix = t / groups;
+        const unsigned xo = pix % (unsigned)Wo, r = pix / (unsigned)Wo;
+        const unsigned yo = r % (unsigned)Ho, b = r / (unsigned)Ho;
+        uint32_t mx[4], mn[4];
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-            uint32_t m = 0u;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) m |= (__ldg(scale + g * 16 + 4 * q + j) >= 0.0f ? 0xFFu : 0u) << (8 * j);
-            up[q] = m;
             mx[q] = 0x00000000u;
             mn[q] = 0xFFFFFFFFu;
         }
+        const uint8_t *base = in + ((size_t)b * H * W) * C + g * 16;
+#pragma unroll
         for (int ky = 0; ky < 3; ++ky) {
-            const int yi = 2 * yo - 1 + ky;
+            const int yi = 2 * (int)yo - 1 + ky;
             if (yi < 0 || yi >= H) continue;
+#pragma unroll
             for (int kx = 0; kx < 3; ++kx) {
-                const int xi = 2 * xo - 1 + kx;
+                const int xi = 2 * (int)xo - 1 + kx;
                 if (xi < 0 || xi >= W) continue;
-                const uint4 v = __ldg(reinterpret_cast<const uint4 *>(in + (((long long)b * H + yi) * W + xi) * C + g * 16));
+                const uint4 v = __ldg(reinterpret_cast<const uint4 *>(base + ((size_t)yi * W + xi) * C));
                 const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
@@ -92,10 +97,13 @@ __global__ void __launch_bounds__(256) pool_levels_kernel(const uint8_t *__restr
                 }
             }
         }
-        uint32_t r[4];
+        uint32_t res[4];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) r[q] = ordered_to_codes((mx[q] & up[q]) | (mn[q] & ~up[q]));
-        *reinterpret_cast<uint4 *>(out + pix * C + g * 16) = make_uint4(r[0], r[1], r[2], r[3]);
+        for (int q = 0; q < 4; ++q) {
+            const uint32_t up = sup[4 * g + q];
+            res[q] = ordered_to_codes((mx[q] & up) | (mn[q] & ~up));
+        }
+        *reinterpret_cast<uint4 *>(out + (size_t)pix * C + g * 16) = make_uint4(res[0], res[1], res[2], res[3]);
     }
 }
 
@@ -419,6 +427,7 @@ minw_status resnet_forward(minw_net *net, const float *x, int B, float *logits, 
     // stem pool on levels -> X [B][Hp][Hp][64]
     {
         const long long items = (long long)B * R->Hp * R->Hp * 4;
+        if (items >= (1ll << 31)) return MINW_EUNSUPPORTED;
         const int sms = num_sms() > 0 ? num_sms() : 152;
         long long g = (items + 255) / 256;
         if (g > sms * 8LL) g = sms * 8LL;
