@@ -68,6 +68,8 @@ struct Params {
     int nlev;                  // levels of the output quantizer
     int ksplit;                // K slices per output tile (1: no split)
     int cl;                    // CTAs per cluster sharing each weight box (1, 2 or 4; 1 when split)
+    int dup;                   // channel-major 64-channel layer: the weight rows loaded twice (MMA rows
+                               // 64 .. 127 repeat 0 .. 63), so that all eight epilogue warps hold channels
     int pair;                  // CTA pairs (cl = 2): one cta_group::2 MMA of M = 256 pixels per pair, each
                                // CTA holding its 128 pixels and half of the weight rows
     int tiles_mp;              // pixel tiles per channel tile, padded to a multiple of cl
@@ -628,9 +630,11 @@ __global__ void __launch_bounds__(NT, 1)
                                                  kcol, o0 + crank * bslice);
                         } else if (act)
                             tma_load_4d(sa + (size_t)j * p.a_bytes, &tmA, &full[s], c0, x0 + kx, y0 + ky, b0);
-                        else if (p.cl == 1)
-                            tma_load_2d(sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes, &tmB, &full[s], kcol, o0);
-                        else
+                        else if (p.cl == 1) {
+                            uint8_t *sb = sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes;
+                            tma_load_2d(sb, &tmB, &full[s], kcol, o0);
+                            if (p.dup) tma_load_2d(sb + (size_t)64 * p.ck, &tmB, &full[s], kcol, o0);
+                        } else
                             tma_load_2d_mc(sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes +
                                                (size_t)crank * bslice * p.ck,
                                            &tmB, &full[s], kcol, o0 + crank * bslice, cmask);
@@ -764,8 +768,11 @@ __global__ void __launch_bounds__(NT, 1)
         if constexpr (OUTB > 0) {
             if (p.trans) {
                 // tile = 128 channels (TMEM lanes) x 256 pixels (columns): this warp holds
-                // channels 32 q + lane of pixel columns [128 half, 128 half + 128)
-                const int oq = 32 * q;
+                // channels 32 q + lane of pixel columns [128 half, 128 half + 128); with the
+                // weights loaded twice (64 channels), channels 32 (q & 1) + lane of the 64
+                // columns [64 (2 (q >> 1) + half), + 64)
+                const int oq = 32 * (p.dup ? (q & 1) : q);
+                const int cq = p.dup ? 2 : 4, cb = p.dup ? 2 * (2 * (q >> 1) + half_cols) : 4 * half_cols;
                 for (int w = blockIdx.x; w < items; w += gridDim.x, ++i) {
                     const int ab = i & 1, use = i >> 1;
                     const int tn = w / tiles_m, tm = w - tn * tiles_m;
@@ -792,7 +799,7 @@ __global__ void __launch_bounds__(NT, 1)
                         sc = __ldg(p.scale + oc);
                         sh = __ldg(p.shift + oc);
                     }
-                    for (int c = 4 * half_cols; c < 4 * half_cols + 4 && !dead && qlive; ++c) {
+                    for (int c = cb; c < cb + cq && !dead && qlive; ++c) {
                         __syncwarp();
                         uint32_t v[32];
                         tmem_ld32(tmem_base + ((uint32_t)oq << 16) + (uint32_t)(ab * p.acc_cols + c * 32), v);
@@ -1256,6 +1263,18 @@ static int cluster_pref() {
     return v;
 }
 
+// Channel-major 64-channel tiles with the weight rows loaded twice (MINW_TC_DUP
+// = 0 pads with zero rows instead): the epilogue of a tile then spreads over
+// all eight epilogue warps, two 32-pixel chunks each instead of four.
+static int dup_pref() {
+    static int v = -1;
+    if (v < 0) {
+        const char *e = getenv("MINW_TC_DUP");
+        v = (e && e[0] == '0') ? 0 : 1;
+    }
+    return v;
+}
+
 // CTA pairs with cta_group::2 MMAs for 256-channel layers with long K loops
 // (MINW_TC_PAIR = 0 turns them off).  Each CTA then loads half the weight
 // rows per K block, and one MMA instruction covers both SMs; short K loops
@@ -1280,9 +1299,10 @@ static int kps_pref() {
 }
 
 // Channel-major tiles (MINW_TC_TRANS=0 turns them off): a 64- or 128-channel
-// layer whose only output is the next layer's levels (a residual block's too,
-// at 128 channels) runs as 128 channels (a 64-channel layer pads with zero
-// weights) x 256 pixels, so each MMA has N = 256 (the tensor pipe's full rate).
+// layer whose only output is the next layer's levels (a residual block's too)
+// runs as 128 channels (a 64-channel layer repeats its weight rows, or pads
+// with zero rows) x 256 pixels, so each MMA has N = 256 (the tensor pipe's
+// full rate).
 static int trans_pref() {
     static int v = -1;
     if (v < 0) {
@@ -1314,7 +1334,7 @@ static bool trans_eligible(const ConvArgs &a) {
     return trans_pref() && (a.O == 128 || a.O == 64) && a.quant_out && (a.codes_out != nullptr || a.planes_out != nullptr) &&
            a.acc_out == nullptr && a.y_out == nullptr && a.y_nhwc == nullptr && a.ksplit <= 1 &&
            (a.res_codes == nullptr && a.res_f32 == nullptr ||
-            (a.O == 128 && !a.pool));     // a 64-channel residual layer keeps pixel-major tiles (all 8 warps busy)
+            ((a.O == 128 || (a.O == 64 && dup_pref())) && !a.pool));   // residual: all 8 warps hold channels
 }
 
 static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_pref()) {
@@ -1337,6 +1357,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     }
     p.mrows = p.trans ? 256 : 128;
     if (p.trans ? !trans_shape(a, p) : !plan_shape(a, p)) return MINW_EUNSUPPORTED;
+    p.dup = (p.trans && a.O == 64 && dup_pref()) ? 1 : 0;
     p.B = a.B; p.C = a.C; p.H = a.H; p.W = a.W; p.O = a.O; p.kh = a.kh; p.kw = a.kw; p.pad = a.pad;
     p.Ho = a.Ho; p.Wo = a.Wo;
     p.stride = a.stride;
@@ -1434,7 +1455,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
         const long long K = (long long)a.kh * a.kw * a.C;
         const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)a.O};
         const cuuint64_t strides[1] = {(cuuint64_t)K};
-        const cuuint32_t box[2] = {(cuuint32_t)p.ck, (cuuint32_t)(p.BN / p.cl)};
+        const cuuint32_t box[2] = {(cuuint32_t)p.ck, (cuuint32_t)(p.dup ? 64 : p.BN / p.cl)};
         const cuuint32_t es[2] = {1u, 1u};
         if (enc(&pl.tmB, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(a.wgt8), dims, strides, box, es,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,

@@ -1,8 +1,9 @@
 """GPU parity of the channel-major tensor-core tiles (128 output channels x
 256 pixels, used for 64- and 128-channel layers whose only output is the next
-layer's levels; a 64-channel layer pads the tile with zero weights): 128 -> 128
-and 64 -> 64 convolutions with and without the 2x2 pool, for each output bit
-width, against the oracle's levels, planes and codes."""
+layer's levels; a 64-channel layer loads its weight rows twice, or pads with
+zero rows when MINW_TC_DUP=0): 128 -> 128 and 64 -> 64 convolutions with and
+without the 2x2 pool, for each output bit width, residual blocks, against the
+oracle's levels, planes and codes."""
 import numpy as np
 import pytest
 
@@ -78,8 +79,9 @@ def test_channel_major_residual(dev, M, bits, ch, shortcut):
     """Residual block in channel-major tiles: y = fmaf(acc, scale, shift) +
     shortcut, HardTanh, quantize; the shortcut is a level-code tensor (identity
     path) or fp32 NHWC (downsample path).  Each lane holds one channel, so the
-    shortcut of pixel j comes through lane j's pixel index.  (A 64-channel
-    residual layer runs in pixel-major tiles: the same check covers it.)"""
+    shortcut of pixel j comes through lane j's pixel index.  A 64-channel layer
+    loads its weight rows twice, so that each epilogue warp takes 64 pixel
+    columns of 32 channels."""
     B, C, H, W, O_ = 160, ch, 32, 32, ch
     p = conv_problem(500 + bits + ch, B, C, H, W, O_, bits_a=bits, bits_w=bits, x_dist="normal", w_sigma=0.05)
     a8 = torch.empty((B, H, W, C), dtype=torch.uint8, device=dev)
@@ -117,3 +119,23 @@ def test_channel_major_residual(dev, M, bits, ch, shortcut):
     want_codes = np.vectorize(_CODE.get)(units.transpose(0, 2, 3, 1)).astype(np.uint8)
     assert np.array_equal(codes.cpu().numpy()[pick], want_codes)
     assert np.array_equal(planes_view(planes, B, H, W, bits, O_)[pick], O.pack(lv, bits))
+
+
+def test_channel_major_zero_rows():
+    """MINW_TC_DUP=0 (read once per process, so in a child): 64-channel tiles
+    padded with zero weight rows give the same levels."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    code = (
+        "import torch\n"
+        "from paper_2003_04296_gb300 import minw\n"
+        "import tests.test_gpu_trans as T\n"
+        "dev = torch.device('cuda:0')\n"
+        "for bits in (1, 3):\n"
+        "    T.test_channel_major_tiles(dev, minw, bits, 1, 64)\n"
+        "print('ok')\n")
+    env = dict(os.environ, MINW_TC_DUP="0")
+    r = subprocess.run([sys.executable, "-c", code], cwd=root, env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stderr[-2000:]
