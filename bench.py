@@ -454,7 +454,8 @@ def sweep_config(n_gpus):
     return {"workload": "conv3x3_bitwidth_sweep_256x512x14x14_to512", "batch_per_gpu": 256,
             "global_batch": 256 * n_gpus, "input": "256x512x14x14 fp32 N(0,1), weights 512x512x3x3 N(0,1)",
             "pairs": "(bits_a, bits_w) in {1,2,3}^2, each a 3x3/1/1 convolution to int32 accumulators",
-            "aqe": "AQE forward (alpha 0.75) and backward on the same 25.7M-element tensor",
+            "aqe": "AQE forward (alpha 0.75) and backward on the same 25.7M-element tensor (the stochastic forward, "
+                   "Eq. our, is timed beside the steps)",
             "parallelism": f"replicas x{n_gpus} (batch-sharded, no collective)", "l2": L2_NOTE}
 
 
@@ -505,6 +506,11 @@ def run_sweep(args, rank, world, local_rank):
         if ev is not None:
             ev[9][1].record(stream)
         minw.aqe_backward(x, gy, gx, 0.75)
+        if ev is not None:
+            # outside the timed steps: the stochastic forward (Eq. our, z from Philox4x64-10)
+            ev[10][0].record(stream)
+            minw.aqe_forward_stochastic(x, y, 0.75, 2026, 0)
+            ev[10][1].record(stream)
 
     for _ in range(max(args.warmup, 3)):
         step()
@@ -530,16 +536,18 @@ def run_sweep(args, rank, world, local_rank):
     ms_max = float(t.item())
     # per-kernel durations: the same steps again with events around the convolutions and the AQE forward
     conv_ms = np.zeros(len(SWEEP_PAIRS))
-    aqe_ms = 0.0
+    aqe_ms = sto_ms = 0.0
     for k in range(args.steps):
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(11)]
         flush.zero_()
         step(ev)
         torch.cuda.synchronize()
         conv_ms += np.array([ev[i][0].elapsed_time(ev[i][1]) for i in range(9)])
         aqe_ms += ev[9][0].elapsed_time(ev[9][1])
+        sto_ms += ev[10][0].elapsed_time(ev[10][1])
     conv_ms /= args.steps
     aqe_ms /= args.steps
+    sto_ms /= args.steps
 
     # end to end: the fp32 input from pinned host memory, the step, the last accumulators back to the host
     x_host = torch.from_numpy(p["x"]).pin_memory()
@@ -572,6 +580,10 @@ def run_sweep(args, rank, world, local_rank):
     aqe_roof = {"bound": "hbm", "kernel": "aqe_forward_kernel", "achieved": aqe_bytes / (aqe_ms * 1e-3) / 1e9,
                 "peak": HBM_GBS, "unit": "GB/s", "frac": aqe_bytes / (aqe_ms * 1e-3) / 1e9 / HBM_GBS,
                 "algorithmic_bytes": aqe_bytes, "peak_basis": "measured copy bandwidth, of measured"}
+    sto_roof = {"bound": "hbm", "kernel": "aqe_forward_stochastic_kernel (Eq. our, Philox4x64-10 noise)",
+                "achieved": aqe_bytes / (sto_ms * 1e-3) / 1e9, "peak": HBM_GBS, "unit": "GB/s",
+                "frac": aqe_bytes / (sto_ms * 1e-3) / 1e9 / HBM_GBS, "algorithmic_bytes": aqe_bytes,
+                "peak_basis": "measured copy bandwidth, of measured"}
     cpu = None
     if world == 1 and not args.skip_cpu:
         from oracle import oracle as Or
@@ -592,7 +604,8 @@ def run_sweep(args, rank, world, local_rank):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "e4m3", "data": "synthetic", "config": sweep_config(world),
             "conv_ms": [round(v, 5) for v in conv_ms.tolist()], "aqe_forward_ms": round(aqe_ms, 5),
-            "roofline": roofline, "aqe_roofline": aqe_roof, "cpu_baseline": cpu,
+            "aqe_stochastic_ms": round(sto_ms, 5),
+            "roofline": roofline, "aqe_roofline": aqe_roof, "aqe_stochastic_roofline": sto_roof, "cpu_baseline": cpu,
             "e2e": {"value": 2.0 * mac * len(SWEEP_PAIRS) * world / e2e_sec / 1e12, "unit": "effective TOPS",
                     "h2d_bytes_per_step": int(x_host.numel() * 4), "d2h_bytes_per_step": int(acc_host.numel() * 4)},
             "gpu_launches": 14 * args.steps, "clocks": clk.summary()}

@@ -92,6 +92,19 @@ MINW_API int32_t minw_version(void);
 MINW_API minw_status aqe_forward(const float *x, float *y, int64_t n, float alpha,
                         const minw_quant *q, void *stream);
 
+/* Stochastic AQE forward, Eq. our (Sec. III-A): y = alpha * sign(x - z) +
+ * (1 - alpha) * x with z ~ U[-1, 1) and sign(0) = -1, evaluated in fp32 as
+ * fmaf(alpha, x > z ? 1 : -1, (1 - alpha) * x).  The noise of element i is a
+ * pure function of (seed, offset, i): 32-bit word i mod 8 of
+ * Philox4x64-10(counter = (offset + i / 8, 0, 0, 0), key = (seed, 0))
+ * (Salmon et al., SC 2011; the low half of each 64-bit output first), mapped
+ * to z = (u >> 8) * 2^-23 - 1.  Successive calls advance offset by
+ * ceil(n / 8) for fresh noise.  x, y: n floats (may alias), 16-byte aligned.
+ * Errors: MINW_EINVAL for n < 0, null pointers, misalignment, alpha outside
+ * [0, 1].  The backward is aqe_backward (Eq. activation). */
+MINW_API minw_status aqe_forward_stochastic(const float *x, float *y, int64_t n, float alpha,
+                                            uint64_t seed, uint64_t offset, void *stream);
+
 /* AQE backward, Eq. activation / Eq. weight:
  * gx = (|x| <= 1) ? gy * (2 * alpha) : 0   (fp32, one rounding).
  * x, gy, gx: n floats (gx may alias gy). */

@@ -109,6 +109,62 @@ void orc_aqe_backward(const float *x, const float *g, int64_t n, double alpha,
 }
 
 /* ------------------------------------------------------------------------ */
+/* Stochastic AQE (Eq. our): h = alpha sign(a - z) + (1 - alpha) a, z ~ U[-1,1] */
+/* ------------------------------------------------------------------------ */
+
+/* Philox4x64-10 (Salmon, Moraes, Dror, Shaw, "Parallel random numbers: as
+ * easy as 1, 2, 3", SC 2011): ten rounds of two 64 x 64 -> 128-bit products
+ * on the counter, the key bumped by the Weyl constants between rounds. */
+void orc_philox4x64_10(const uint64_t ctr[4], const uint64_t key[2], uint64_t out[4])
+{
+    const uint64_t M0 = 0xD2E7470EE14C6C93ull, M1 = 0xCA5A826395121157ull;
+    const uint64_t W0 = 0x9E3779B97F4A7C15ull, W1 = 0xBB67AE8584CAA73Bull;
+    uint64_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3];
+    uint64_t k0 = key[0], k1 = key[1];
+    for (int r = 0; r < 10; ++r) {
+        const unsigned __int128 p0 = (unsigned __int128)M0 * c0;
+        const unsigned __int128 p1 = (unsigned __int128)M1 * c2;
+        const uint64_t hi0 = (uint64_t)(p0 >> 64), lo0 = (uint64_t)p0;
+        const uint64_t hi1 = (uint64_t)(p1 >> 64), lo1 = (uint64_t)p1;
+        c0 = hi1 ^ c1 ^ k0;
+        c1 = lo1;
+        c2 = hi0 ^ c3 ^ k1;
+        c3 = lo0;
+        k0 += W0;
+        k1 += W1;
+    }
+    out[0] = c0; out[1] = c1; out[2] = c2; out[3] = c3;
+}
+
+/* The noise of element i: 32-bit word (i mod 8) of philox4x64_10(counter =
+ * (offset + i / 8, 0, 0, 0), key = (seed, 0)) (words in order, low half of each
+ * 64-bit output first), u -> z = (u >> 8) 2^-23 - 1, a point of the 2^-23 grid
+ * on [-1, 1) (exact in fp32). */
+float orc_noise(uint64_t i, uint64_t seed, uint64_t offset)
+{
+    const uint64_t ctr[4] = {offset + (i >> 3), 0, 0, 0};
+    const uint64_t key[2] = {seed, 0};
+    uint64_t r[4];
+    orc_philox4x64_10(ctr, key, r);
+    const uint64_t w = r[(i & 7) >> 1];
+    const uint32_t u = (i & 1) ? (uint32_t)(w >> 32) : (uint32_t)w;
+    return (float)((double)(u >> 8) * (1.0 / 8388608.0) - 1.0);
+}
+
+/* Eq. our with the sign of Eq. sign (sign(0) = -1): y in fp64, the noise and
+ * the decision s = [a > z] exactly as drawn. */
+void orc_aqe_forward_stochastic(const float *x, int64_t n, double alpha, uint64_t seed, uint64_t offset,
+                                double *y, float *z)
+{
+    for (int64_t i = 0; i < n; ++i) {
+        const float zi = orc_noise((uint64_t)i, seed, offset);
+        const double s = ((double)x[i] - (double)zi > 0.0) ? 1.0 : -1.0;
+        y[i] = alpha * s + (1.0 - alpha) * (double)x[i];
+        if (z) z[i] = zi;
+    }
+}
+
+/* ------------------------------------------------------------------------ */
 /* Bit-plane packing of quantized levels                                     */
 /* ------------------------------------------------------------------------ */
 

@@ -36,6 +36,9 @@ def lib():
         L.orc_quantize.argtypes = [P, i64, i64, i32, P, P, P]
         L.orc_aqe_forward.argtypes = [P, i64, f64, i32, P, f32, P]
         L.orc_aqe_backward.argtypes = [P, P, i64, f64, P]
+        u64 = ctypes.c_uint64
+        L.orc_philox4x64_10.argtypes = [P, P, P]
+        L.orc_aqe_forward_stochastic.argtypes = [P, i64, f64, u64, u64, P, P]
         L.orc_pack.argtypes = [P, i32, i32, i32, i32, i32, P]
         L.orc_conv2d.restype = i32
         L.orc_conv2d.argtypes = [P, i32, i32, i32, i32, P, i32, i32, i32, i32, i32, i32, P]
@@ -117,6 +120,28 @@ def aqe_backward(x, g, alpha):
     gx = np.empty(x.shape, dtype=np.float64)
     lib().orc_aqe_backward(_p(x), _p(g), x.size, float(alpha), _p(gx))
     return gx
+
+
+def philox4x64_10(counter, key):
+    """Philox4x64-10 block (Salmon et al., SC 2011): 4 x uint64 counter,
+    2 x uint64 key -> 4 x uint64."""
+    c = np.ascontiguousarray(counter, dtype=np.uint64)
+    k = np.ascontiguousarray(key, dtype=np.uint64)
+    out = np.empty(4, dtype=np.uint64)
+    lib().orc_philox4x64_10(_p(c), _p(k), _p(out))
+    return out
+
+
+def aqe_forward_stochastic(x, alpha, seed, offset=0):
+    """Eq. our: alpha sign(a - z) + (1 - alpha) a in fp64, z ~ U[-1, 1) drawn
+    from Philox4x64-10 (element i: counter offset + i // 8, key (seed, 0),
+    32-bit word i mod 8).  Returns (y, z)."""
+    x = _f32(x)
+    y = np.empty(x.shape, dtype=np.float64)
+    z = np.empty(x.shape, dtype=np.float32)
+    lib().orc_aqe_forward_stochastic(_p(x), x.size, float(alpha), int(seed) & (2**64 - 1),
+                                     int(offset) & (2**64 - 1), _p(y), _p(z))
+    return y, z
 
 
 def pack(levels, bits):

@@ -39,6 +39,82 @@ __global__ void __launch_bounds__(256) aqe_forward_kernel(const float *__restric
         y[i] = aqe_fwd1(x[i], alpha, oma, q);
 }
 
+// ---------------------------------------------------------------------------
+// Stochastic AQE (Eq. our): alpha sign(a - z) + (1 - alpha) a with z ~ U[-1, 1)
+// from a counter-based generator, so that any element's noise is a pure
+// function of (seed, offset, index).
+// ---------------------------------------------------------------------------
+
+// Philox4x64-10 (Salmon, Moraes, Dror, Shaw, SC 2011): ten rounds of two
+// 64 x 64 -> 128-bit products on the counter, the key bumped by the Weyl
+// constants between rounds.
+__device__ __forceinline__ void philox4x64_10(uint64_t c[4], uint64_t k0, uint64_t k1) {
+    const uint64_t M0 = 0xD2E7470EE14C6C93ull, M1 = 0xCA5A826395121157ull;
+    const uint64_t W0 = 0x9E3779B97F4A7C15ull, W1 = 0xBB67AE8584CAA73Bull;
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        const uint64_t hi0 = __umul64hi(M0, c[0]), lo0 = M0 * c[0];
+        const uint64_t hi1 = __umul64hi(M1, c[2]), lo1 = M1 * c[2];
+        const uint64_t n0 = hi1 ^ c[1] ^ k0, n2 = hi0 ^ c[3] ^ k1;
+        c[0] = n0;
+        c[1] = lo1;
+        c[2] = n2;
+        c[3] = lo0;
+        k0 += W0;
+        k1 += W1;
+    }
+}
+
+// z = (u >> 8) 2^-23 - 1: a point of the 2^-23 grid on [-1, 1), exact in fp32.
+__device__ __forceinline__ float noise_of(uint32_t u) { return (float)(u >> 8) * 1.1920928955078125e-7f - 1.0f; }
+
+__device__ __forceinline__ float aqe_sto1(float x, float z, float alpha, float oma) {
+    return fmaf(alpha, x > z ? 1.0f : -1.0f, oma * x);      // sign(x - z), sign(0) = -1
+}
+
+// Thread = one block of eight elements: one Philox4x64-10 call (counter
+// offset + block, key (seed, 0)) gives the eight 32-bit noise words, low half
+// of each 64-bit output first; two 128-bit loads and stores.
+__global__ void __launch_bounds__(256) aqe_forward_stochastic_kernel(const float *__restrict__ x,
+                                                                     float *__restrict__ y, int64_t n,
+                                                                     float alpha, float oma, uint64_t seed,
+                                                                     uint64_t offset) {
+    const int64_t nb = (n + 7) >> 3;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nb; b += stride) {
+        const int64_t i0 = b << 3;
+        const bool whole = i0 + 8 <= n;
+        // the loads first, so that they are in flight during the generator's rounds
+        float v[8];
+        if (whole) {
+            const float4 *x4 = reinterpret_cast<const float4 *>(x + i0);
+            const float4 v0 = __ldcs(x4), v1 = __ldcs(x4 + 1);
+            v[0] = v0.x; v[1] = v0.y; v[2] = v0.z; v[3] = v0.w;
+            v[4] = v1.x; v[5] = v1.y; v[6] = v1.z; v[7] = v1.w;
+        } else {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) v[j] = i0 + j < n ? x[i0 + j] : 0.0f;
+        }
+        uint64_t c[4] = {offset + (uint64_t)b, 0ull, 0ull, 0ull};
+        philox4x64_10(c, seed, 0ull);
+        float r[8];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            r[2 * j] = aqe_sto1(v[2 * j], noise_of((uint32_t)c[j]), alpha, oma);
+            r[2 * j + 1] = aqe_sto1(v[2 * j + 1], noise_of((uint32_t)(c[j] >> 32)), alpha, oma);
+        }
+        if (whole) {
+            float4 *y4 = reinterpret_cast<float4 *>(y + i0);
+            __stcs(y4, make_float4(r[0], r[1], r[2], r[3]));
+            __stcs(y4 + 1, make_float4(r[4], r[5], r[6], r[7]));
+        } else {
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (i0 + j < n) y[i0 + j] = r[j];
+        }
+    }
+}
+
 __device__ __forceinline__ float aqe_bwd1(float x, float g, float two_alpha) {
     return (fabsf(x) <= 1.0f) ? g * two_alpha : 0.0f;
 }
@@ -384,6 +460,17 @@ minw_status aqe_forward(const float *x, float *y, int64_t n, float alpha, const 
     const QParams qp = to_qparams(q);
     const int64_t g = grid_for(n / 4 + 1, 256);
     aqe_forward_kernel<<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(x, y, n, alpha, 1.0f - alpha, qp);
+    return launch_status();
+}
+
+minw_status aqe_forward_stochastic(const float *x, float *y, int64_t n, float alpha, uint64_t seed,
+                                   uint64_t offset, void *stream) {
+    if (n < 0 || !(alpha >= 0.0f && alpha <= 1.0f)) return MINW_EINVAL;
+    if (n == 0) return MINW_OK;
+    if (!x || !y || !aligned16(x) || !aligned16(y)) return MINW_EINVAL;
+    const int64_t g = grid_for((n + 7) / 8, 256);
+    aqe_forward_stochastic_kernel<<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(x, y, n, alpha, 1.0f - alpha, seed,
+                                                                                offset);
     return launch_status();
 }
 

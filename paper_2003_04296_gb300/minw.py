@@ -64,6 +64,7 @@ SIGNATURES = {
     "minw_version": (_I32, []),
     "aqe_forward": (ctypes.c_int, [_P, _P, _I64, _F, _QP, _P]),
     "aqe_backward": (ctypes.c_int, [_P, _P, _P, _I64, _F, _P]),
+    "aqe_forward_stochastic": (ctypes.c_int, [_P, _P, _I64, _F, ctypes.c_uint64, ctypes.c_uint64, _P]),
     "aqe_quantize_pack": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _F, _P, _P, _P]),
     "aqe_backward_masked": (ctypes.c_int, [_P, _P, _P, _I64, _F, _P]),
     "minw_pack_weights": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
@@ -180,6 +181,14 @@ def packed_words(N, C, H, W, bits):
 def aqe_forward(x, y, alpha, q, stream=None):
     _check(lib().aqe_forward(_ptr(x), _ptr(y), x.numel(), float(alpha), ctypes.byref(q), _stream(stream)),
            "aqe_forward")
+
+
+def aqe_forward_stochastic(x, y, alpha, seed, offset=0, stream=None):
+    """Eq. our: alpha sign(x - z) + (1 - alpha) x, z ~ U[-1, 1) from
+    Philox4x64-10 keyed by seed; offset advances the counter (ceil(n / 8) per
+    call for fresh noise)."""
+    _check(lib().aqe_forward_stochastic(_ptr(x), _ptr(y), x.numel(), float(alpha), int(seed) & (2**64 - 1),
+                                        int(offset) & (2**64 - 1), _stream(stream)), "aqe_forward_stochastic")
 
 
 def aqe_backward(x, gy, gx, alpha, stream=None):

@@ -105,3 +105,79 @@ def test_weight_form_is_same_rule():
     g = np.ones_like(w)
     gx = O.aqe_backward(w, g, 0.75)
     assert np.array_equal(gx, np.where(np.abs(w) <= 1, 1.5, 0.0))
+
+
+# ---------------------------------------------------------------------------
+# Stochastic AQE (Eq. our) with the counter-based generator
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("key,counter", [
+    ((0x0123456789ABCDEF, 0xFEDCBA9876543210), (1, 0, 0, 0)),
+    ((0, 0), (7, 0, 0, 0)),
+    ((2**64 - 1, 2**64 - 1), (3, 2**64 - 1, 5, 2**63)),
+    ((12345, 0), (0, 1, 0, 0)),            # numpy's carry from counter word 0 into word 1
+])
+def test_philox_matches_numpy(key, counter):
+    """The oracle's Philox4x64-10 block equals numpy's Philox bit generator
+    (same published algorithm; numpy advances its 256-bit counter by one
+    before each block, so counter c comes from a generator started at c - 1)."""
+    c = [int(v) for v in counter]
+    prev = list(c)
+    for w in range(4):                     # c - 1 with borrow across the four words
+        if prev[w] > 0:
+            prev[w] -= 1
+            break
+        prev[w] = 2**64 - 1
+    bg = np.random.Philox(key=np.array(key, dtype=np.uint64), counter=np.array(prev, dtype=np.uint64))
+    want = bg.random_raw(4)
+    got = O.philox4x64_10(np.array(c, dtype=np.uint64), np.array(key, dtype=np.uint64))
+    assert np.array_equal(got, want)
+
+
+def test_noise_grid_and_uniformity():
+    """z lies on the 2^-23 grid of [-1, 1) and is uniform: mean, variance and
+    a 64-bin chi-square over 2^20 draws within their 5-sigma bounds."""
+    n = 1 << 20
+    _, z = O.aqe_forward_stochastic(np.zeros(n, dtype=np.float32), 0.5, seed=7, offset=0)
+    z = z.astype(np.float64)
+    assert z.min() >= -1.0 and z.max() < 1.0
+    k = (z + 1.0) * 2.0 ** 23
+    assert np.array_equal(k, np.rint(k))
+    assert abs(z.mean()) < 5 * np.sqrt(1 / 3 / n)
+    assert abs(z.var() - 1 / 3) < 5 * np.sqrt(4 / 45 / n)
+    counts = np.histogram(z, bins=64, range=(-1.0, 1.0))[0]
+    exp = n / 64
+    chi2 = np.sum((counts - exp) ** 2 / exp)
+    assert chi2 < 63 + 5 * np.sqrt(2 * 63)
+
+
+@pytest.mark.parametrize("alpha", [0.25, 0.75])
+def test_stochastic_theorem1_expectation(alpha):
+    """Theorem 1's premise on the oracle's own draws: (h^ - (1 - alpha) a) / alpha
+    = sign(a - z) averages to max(-1, min(1, a)) (Monte Carlo within 5 sigma),
+    and each draw is exactly +-1 around the identity term."""
+    m = 1 << 16
+    for j, a in enumerate([-1.4, -0.5, 0.0, 0.3, 0.95, 2.0]):
+        x = np.full(m, a, dtype=np.float32)
+        y, z = O.aqe_forward_stochastic(x, alpha, seed=100 + j, offset=3)
+        s = (y - (1.0 - alpha) * np.float64(np.float32(a))) / alpha
+        np.testing.assert_allclose(np.abs(s), 1.0, rtol=0, atol=1e-9)
+        assert np.array_equal(s > 0, x.astype(np.float64) > z)
+        exact = float(np.clip(np.float32(a), -1.0, 1.0))
+        sig = np.sqrt(max(1 - exact ** 2, 1e-12) / m)
+        assert abs(s.mean() - exact) <= 5 * sig + 2.0 ** -22
+
+
+def test_stochastic_limits_and_counter_layout():
+    """alpha = 1 gives sign(a - z) in {-1, 1}, alpha = 0 the identity; element
+    i at offset o draws the same noise as element i - 8k at offset o + k, and
+    another seed draws other noise."""
+    x = np.random.default_rng(3).standard_normal(1000).astype(np.float32)
+    y1, z1 = O.aqe_forward_stochastic(x, 1.0, seed=9, offset=5)
+    assert np.array_equal(np.abs(y1), np.ones_like(y1))
+    y0, _ = O.aqe_forward_stochastic(x, 0.0, seed=9, offset=5)
+    assert np.array_equal(y0, x.astype(np.float64))
+    _, z2 = O.aqe_forward_stochastic(x[:1000 - 24], 1.0, seed=9, offset=5 + 3)
+    assert np.array_equal(z2, z1[24:])
+    _, z3 = O.aqe_forward_stochastic(x, 1.0, seed=10, offset=5)
+    assert np.mean(z3 == z1) < 0.01
