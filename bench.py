@@ -145,6 +145,23 @@ class Workload:
                 "parallelism": par, "l2": L2_NOTE}
 
 
+def max_over_ranks(v, world, device):
+    """The largest v over the ranks (every rank gets it): the slowest replica
+    sets the job's time."""
+    import torch
+    t = torch.tensor([float(v)], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(units_per_rank, world, seconds):
+    """Whole-job throughput of independent replicas (weak scaling): every
+    rank processes units_per_rank in `seconds` (the max over ranks)."""
+    return units_per_rank * world / seconds
+
+
 def layer_macs(net_p, hw=32):
     """MACs per image of each layer, in network order."""
     out = []
@@ -359,11 +376,7 @@ def run_gpu(args, rank, world, local_rank):
     torch.cuda.synchronize()
     for k in range(args.steps):
         step_ms.append(ev0[k].elapsed_time(ev1[k]))
-    ms = sum(step_ms) / len(step_ms)
-    t = torch.tensor([ms], device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms_max = float(t.item())
+    ms_max = max_over_ranks(sum(step_ms) / len(step_ms), world, dev)
 
     # end to end through the public API: pinned host input -> logits on host
     x_host = torch.from_numpy(x_np).pin_memory()
@@ -380,10 +393,7 @@ def run_gpu(args, rank, world, local_rank):
         t0 = time.perf_counter()
         net.forward_host(x_host, out_host)
         e2e_s.append(time.perf_counter() - t0)
-    e2e = torch.tensor([sum(e2e_s) / len(e2e_s)], device=dev)
-    if world > 1:
-        dist.all_reduce(e2e, op=dist.ReduceOp.MAX)
-    e2e_sec = float(e2e.item())
+    e2e_sec = max_over_ranks(sum(e2e_s) / len(e2e_s), world, dev)
 
     if rank != 0:
         return 0
@@ -391,8 +401,8 @@ def run_gpu(args, rank, world, local_rank):
     clocks = clk.summary()
     layer_ms /= args.steps
     total_macs = sum(macs) * BATCH
-    value = BATCH * world / (ms_max * 1e-3)
-    eff_tops = 2.0 * total_macs * world / (ms_max * 1e-3) / 1e12
+    value = replica_throughput(BATCH, world, ms_max * 1e-3)
+    eff_tops = replica_throughput(2.0 * total_macs, world, ms_max * 1e-3) / 1e12
 
     # roofline of the dominant kernel: the quantized convolution (every op in q_ops_idx)
     variants = net.layer_variants()
@@ -432,7 +442,7 @@ def run_gpu(args, rank, world, local_rank):
             "layer_ms_note": "per-op CUDA-event durations from a second pass of the same steps with an event "
                              "after every op; the timed steps run without them",
             "roofline": roofline, "cpu_baseline": cpu,
-            "e2e": {"value": BATCH * world / e2e_sec, "unit": "images/s",
+            "e2e": {"value": replica_throughput(BATCH, world, e2e_sec), "unit": "images/s",
                     "h2d_bytes_per_step": int(x_host.numel() * 4),
                     "d2h_bytes_per_step": int(out_host.numel() * 4)},
             "gpu_launches": net.kernels * args.steps, "clocks": clocks}
@@ -530,10 +540,7 @@ def run_sweep(args, rank, world, local_rank):
         if world > 1:
             dist.barrier()
     ms = sum(e0[k].elapsed_time(e1[k]) for k in range(args.steps)) / args.steps
-    t = torch.tensor([ms], device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms_max = float(t.item())
+    ms_max = max_over_ranks(ms, world, dev)
     # per-kernel durations: the same steps again with events around the convolutions and the AQE forward
     conv_ms = np.zeros(len(SWEEP_PAIRS))
     aqe_ms = sto_ms = 0.0
@@ -564,12 +571,12 @@ def run_sweep(args, rank, world, local_rank):
         torch.cuda.synchronize()
         if k:
             e2e_s.append(time.perf_counter() - t0)
-    e2e_sec = sum(e2e_s) / len(e2e_s)
+    e2e_sec = max_over_ranks(sum(e2e_s) / len(e2e_s), world, dev)
     if rank != 0:
         return 0
 
     mac = B * H * W * O * C * 9
-    value = 2.0 * mac * len(SWEEP_PAIRS) * world / (ms_max * 1e-3) / 1e12
+    value = replica_throughput(2.0 * mac * len(SWEEP_PAIRS), world, ms_max * 1e-3) / 1e12
     achieved = 2.0 * mac * len(SWEEP_PAIRS) / (conv_ms.sum() * 1e-3) / 1e12
     roofline = {"bound": "tensor", "kernel": "conv_tc_kernel (tcgen05 kind::f8f6f4, 9 bit-width pairs)",
                 "achieved": achieved, "peak": FP8_TFLOPS, "unit": "TFLOP/s", "frac": achieved / FP8_TFLOPS,
