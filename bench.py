@@ -497,6 +497,13 @@ def run_sweep(args, rank, world, local_rank):
         minw.minw_pack_weight_codes(w, minw.quant(b, DEFAULT_THR[b]), w8[b], channel_scale=ws)
     acc = torch.empty((B, O, H, W), dtype=torch.int32, device=dev)
     y = torch.empty_like(x)
+    # weight-only layer at the same shape (bf16 activations x 1-bit weights), timed beside the steps
+    xb = torch.empty((B, H, W, C), dtype=torch.int16, device=dev)
+    wb = torch.empty((O, 3, 3, C), dtype=torch.int16, device=dev)
+    minw.minw_to_bf16_nhwc(x, xb)
+    minw.minw_pack_weight_bf16(w, minw.quant(1, DEFAULT_THR[1]), wb, channel_scale=ws)
+    yw = torch.empty((B, O, H, W), dtype=torch.float32, device=dev)
+    sc1, sh0 = torch.ones(O, device=dev), torch.zeros(O, device=dev)
     gx = torch.empty_like(x)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
@@ -521,6 +528,9 @@ def run_sweep(args, rank, world, local_rank):
             ev[10][0].record(stream)
             minw.aqe_forward_stochastic(x, y, 0.75, 2026, 0)
             ev[10][1].record(stream)
+            ev[11][0].record(stream)
+            minw.minw_conv2d_bf16(xb, B, C, H, W, wb, O, 3, 3, 1, 1, 1, 0, sc1, sh0, yw)
+            ev[11][1].record(stream)
 
     for _ in range(max(args.warmup, 3)):
         step()
@@ -543,18 +553,20 @@ def run_sweep(args, rank, world, local_rank):
     ms_max = max_over_ranks(ms, world, dev)
     # per-kernel durations: the same steps again with events around the convolutions and the AQE forward
     conv_ms = np.zeros(len(SWEEP_PAIRS))
-    aqe_ms = sto_ms = 0.0
+    aqe_ms = sto_ms = wo_ms = 0.0
     for k in range(args.steps):
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(11)]
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(12)]
         flush.zero_()
         step(ev)
         torch.cuda.synchronize()
         conv_ms += np.array([ev[i][0].elapsed_time(ev[i][1]) for i in range(9)])
         aqe_ms += ev[9][0].elapsed_time(ev[9][1])
         sto_ms += ev[10][0].elapsed_time(ev[10][1])
+        wo_ms += ev[11][0].elapsed_time(ev[11][1])
     conv_ms /= args.steps
     aqe_ms /= args.steps
     sto_ms /= args.steps
+    wo_ms /= args.steps
 
     # end to end: the fp32 input from pinned host memory, the step, the last accumulators back to the host
     x_host = torch.from_numpy(p["x"]).pin_memory()
@@ -591,6 +603,10 @@ def run_sweep(args, rank, world, local_rank):
                 "achieved": aqe_bytes / (sto_ms * 1e-3) / 1e9, "peak": HBM_GBS, "unit": "GB/s",
                 "frac": aqe_bytes / (sto_ms * 1e-3) / 1e9 / HBM_GBS, "algorithmic_bytes": aqe_bytes,
                 "peak_basis": "measured copy bandwidth, of measured"}
+    wo_tf = 2.0 * mac / (wo_ms * 1e-3) / 1e12
+    wonly = {"kernel": "conv_tc_kernel<0, false, true> (tcgen05 kind::f16: bf16 activations x 1-bit weights)",
+             "ms": round(wo_ms, 5), "achieved": wo_tf, "peak": BF16_TFLOPS, "unit": "TFLOP/s",
+             "frac": wo_tf / BF16_TFLOPS, "peak_basis": "measured dense bf16 TFLOP/s (burst), of measured"}
     cpu = None
     if world == 1 and not args.skip_cpu:
         from oracle import oracle as Or
@@ -612,7 +628,8 @@ def run_sweep(args, rank, world, local_rank):
             "scaling": "weak", "vs_baseline": None, "dtype": "e4m3", "data": "synthetic", "config": sweep_config(world),
             "conv_ms": [round(v, 5) for v in conv_ms.tolist()], "aqe_forward_ms": round(aqe_ms, 5),
             "aqe_stochastic_ms": round(sto_ms, 5),
-            "roofline": roofline, "aqe_roofline": aqe_roof, "aqe_stochastic_roofline": sto_roof, "cpu_baseline": cpu,
+            "roofline": roofline, "aqe_roofline": aqe_roof, "aqe_stochastic_roofline": sto_roof,
+            "weight_only_bf16": wonly, "cpu_baseline": cpu,
             "e2e": {"value": 2.0 * mac * len(SWEEP_PAIRS) * world / e2e_sec / 1e12, "unit": "effective TOPS",
                     "h2d_bytes_per_step": int(x_host.numel() * 4), "d2h_bytes_per_step": int(acc_host.numel() * 4)},
             "gpu_launches": 14 * args.steps, "clocks": clk.summary()}

@@ -229,6 +229,38 @@ MINW_API minw_status minw_conv_block_codes(const uint8_t *act, int32_t B, int32_
                                            uint8_t *codes_out, uint32_t *planes_out,
                                            float *y_out, void *stream);
 
+/* ---------------------------------------------------------------------- */
+/* Weight-only quantized convolution (Sec. IV, the XNOR / SHIFT ADDER       */
+/* layers of Tables II-IV: full-precision activations, 1-3-bit weights)    */
+/* ---------------------------------------------------------------------- */
+
+/* fp32 NCHW [B][C][H][W] -> bf16 NHWC [B][H][W][C], round to nearest even. */
+MINW_API minw_status minw_to_bf16_nhwc(const float *x, int32_t B, int32_t C, int32_t H, int32_t W,
+                                       uint16_t *out, void *stream);
+
+/* Quantize latent weights [O][C][kh][kw] (Eq. sign / tnn / qnn at x *
+ * channel_scale[o], or q->scale when channel_scale is null) into bf16 level
+ * values in integer units [O][kh][kw][C]: +-1 (1-bit), {-1, 0, 1} (2-bit),
+ * {0, +-1, +-2, +-4} (3-bit, quarters), all exact in bf16.  out 16-byte
+ * aligned, C % 8 == 0 (else MINW_EUNSUPPORTED). */
+MINW_API minw_status minw_pack_weight_bf16(const float *w, int32_t O, int32_t C, int32_t kh, int32_t kw,
+                                           const minw_quant *q, const float *channel_scale, uint16_t *out,
+                                           void *stream);
+
+/* Weight-only quantized convolution on the tcgen05 tensor cores (kind::f16,
+ * bf16 x bf16 -> fp32 in TMEM): acc[b][o][y][x] = sum over (ky, kx, c) of
+ * act * wgt with the accumulation order of the tensor core (not the oracle's),
+ * then [2x2 / 2 max pool] and y_out = fmaf(acc, scale[o], shift[o]) fp32 NCHW
+ * (no HardTanh, no quantizer: the next layer's activations stay full
+ * precision).  act: bf16 NHWC [B][H][W][C]; wgt: bf16 [O][kh][kw][C] from
+ * minw_pack_weight_bf16 (bits_w documents it).  Supported: stride 1 or 2,
+ * C % 64 == 0, pad < kh, kw, even output size when pooling.  Errors:
+ * MINW_EINVAL (arguments), MINW_EUNSUPPORTED (shape). */
+MINW_API minw_status minw_conv2d_bf16(const uint16_t *act, int32_t B, int32_t C, int32_t H, int32_t W,
+                                      const uint16_t *wgt, int32_t O, int32_t kh, int32_t kw, int32_t bits_w,
+                                      int32_t stride, int32_t pad, int32_t pool, const float *scale,
+                                      const float *shift, float *y_out, void *stream);
+
 /* Extra inputs and outputs of a residual block (ResNet-style MINW-Net,
  * where the paper leaves the block wiring open).  Host struct.
  * res_codes (nullable): shortcut as level codes [B][Hp][Wp][O] of bit width

@@ -241,6 +241,53 @@ int orc_conv2d(const double *a, int B, int C, int H, int W,
 }
 
 /* ------------------------------------------------------------------------ */
+/* Weight-only quantized layers (Sec. IV: full-precision activations times  */
+/* 1-3-bit weights, the XNOR / SHIFT ADDER rows of Tables II-IV)             */
+/* ------------------------------------------------------------------------ */
+
+/* bf16 of an fp32 value, round to nearest, ties to even (the 8 most
+ * significant bits of the significand are kept): the fp32 value of it.
+ * NaN stays NaN. */
+float orc_bf16_round(float x)
+{
+    uint32_t u;
+    memcpy(&u, &x, 4);
+    if ((u & 0x7F800000u) == 0x7F800000u && (u & 0x007FFFFFu)) return x;
+    const uint32_t lsb = (u >> 16) & 1u;
+    u = (u + 0x7FFFu + lsb) & 0xFFFF0000u;
+    float r;
+    memcpy(&r, &u, 4);
+    return r;
+}
+
+/* Direct convolution in fp64 of real activations a [B][C][H][W] with weights
+ * w [O][C][kh][kw], zero padding: the exact real-valued accumulator (every
+ * product of a bf16 value and a level is exact, and so is the fp64 sum at
+ * these sizes up to its own rounding). */
+void orc_conv2d_real(const double *a, int B, int C, int H, int W,
+                     const double *w, int O, int kh, int kw, int stride, int pad, double *out)
+{
+    int Ho = (H + 2 * pad - kh) / stride + 1;
+    int Wo = (W + 2 * pad - kw) / stride + 1;
+    for (int b = 0; b < B; ++b)
+        for (int o = 0; o < O; ++o)
+            for (int yo = 0; yo < Ho; ++yo)
+                for (int xo = 0; xo < Wo; ++xo) {
+                    double s = 0.0;
+                    for (int c = 0; c < C; ++c)
+                        for (int ky = 0; ky < kh; ++ky)
+                            for (int kx = 0; kx < kw; ++kx) {
+                                int yi = yo * stride - pad + ky;
+                                int xi = xo * stride - pad + kx;
+                                if (yi < 0 || yi >= H || xi < 0 || xi >= W) continue;
+                                s += a[(((size_t)b * C + c) * H + yi) * W + xi] *
+                                     w[(((size_t)o * C + c) * kh + ky) * kw + kx];
+                            }
+                    out[(((size_t)b * O + o) * Ho + yo) * Wo + xo] = s;
+                }
+}
+
+/* ------------------------------------------------------------------------ */
 /* Layer pieces around the convolution (Sec. III-E)                          */
 /* ------------------------------------------------------------------------ */
 

@@ -40,6 +40,9 @@ def lib():
         L.orc_philox4x64_10.argtypes = [P, P, P]
         L.orc_aqe_forward_stochastic.argtypes = [P, i64, f64, u64, u64, P, P]
         L.orc_pack.argtypes = [P, i32, i32, i32, i32, i32, P]
+        L.orc_bf16_round.restype = f32
+        L.orc_bf16_round.argtypes = [f32]
+        L.orc_conv2d_real.argtypes = [P, i32, i32, i32, i32, P, i32, i32, i32, i32, i32, P]
         L.orc_conv2d.restype = i32
         L.orc_conv2d.argtypes = [P, i32, i32, i32, i32, P, i32, i32, i32, i32, i32, i32, P]
         L.orc_maxpool_i32.argtypes = [P, i32, i32, i32, i32, i32, i32, P]
@@ -171,6 +174,39 @@ def conv2d_levels(a_lv, w_lv, stride, pad, bits_a, bits_w):
     if rc != 0:
         raise ArithmeticError("non-integral accumulator")
     return acc
+
+
+def bf16_round(x):
+    """fp32 -> bf16 (round to nearest, ties to even), returned as fp32 values."""
+    x = _f32(x)
+    f = lib().orc_bf16_round
+    return np.array([f(float(v)) for v in x.reshape(-1)], dtype=np.float32).reshape(x.shape)
+
+
+def conv2d_real(a, w, stride, pad):
+    """Zero-padded fp64 convolution of real activations a [B][C][H][W] with
+    weights w [O][C][kh][kw] (the weight-only layers' exact accumulator)."""
+    a = np.ascontiguousarray(a, dtype=np.float64)
+    w = np.ascontiguousarray(w, dtype=np.float64)
+    B, C, H, W = a.shape
+    O, Cw, kh, kw = w.shape
+    assert C == Cw
+    Ho = (H + 2 * pad - kh) // stride + 1
+    Wo = (W + 2 * pad - kw) // stride + 1
+    out = np.empty((B, O, Ho, Wo), dtype=np.float64)
+    lib().orc_conv2d_real(_p(a), B, C, H, W, _p(w), O, kh, kw, stride, pad, _p(out))
+    return out
+
+
+def maxpool_f64(x, k=2, s=2):
+    """k x k / s max pooling of fp64 [B][C][H][W] (no padding)."""
+    B, C, H, W = x.shape
+    Ho, Wo = (H - k) // s + 1, (W - k) // s + 1
+    out = np.full((B, C, Ho, Wo), -np.inf)
+    for dy in range(k):
+        for dx in range(k):
+            out = np.maximum(out, x[:, :, dy:dy + s * (Ho - 1) + 1:s, dx:dx + s * (Wo - 1) + 1:s])
+    return out
 
 
 def maxpool_i32(acc, k=2, s=2):

@@ -2,6 +2,7 @@
 // the fused quantize + bit-plane pack of activations (Eq. inference) and the
 // packing of latent weights.  All of them stream HBM: 128-bit loads where the
 // layout allows, grids sized from the SM count.
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 #include <stdlib.h>
@@ -379,6 +380,49 @@ __global__ void weight_codes_kernel(const float *__restrict__ w, int O, int C, i
     }
 }
 
+// Weights [O][C][kh][kw] -> bf16 level values in integer units [O][kh][kw][C]
+// (1, 2 or 4 for the 3-bit magnitudes, all exact in bf16): one thread per
+// 8 channels, one 128-bit store.
+__global__ void weight_bf16_kernel(const float *__restrict__ w, int O, int C, int kh, int kw, QParams q,
+                                   const float *__restrict__ cscale, uint16_t *__restrict__ out) {
+    const int G = C >> 3;
+    const int taps = kh * kw;
+    const int64_t total = (int64_t)O * taps * G;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        const int g = (int)(t % G);
+        const int tap = (int)((t / G) % taps);
+        const int o = (int)(t / ((int64_t)G * taps));
+        const float s = cscale ? cscale[o] : q.scale;
+        uint32_t wd[4];
+        for (int j = 0; j < 4; ++j) {
+            const int c = g * 8 + 2 * j;
+            const float lo = (float)level_units(w[((int64_t)o * C + c) * taps + tap] * s, q);
+            const float hi = (float)level_units(w[((int64_t)o * C + c + 1) * taps + tap] * s, q);
+            wd[j] = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(lo)) |
+                    ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(hi)) << 16);
+        }
+        *reinterpret_cast<uint4 *>(out + ((int64_t)o * taps + tap) * C + g * 8) = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+    }
+}
+
+// fp32 NCHW -> bf16 NHWC, round to nearest even: one thread per output element
+// of a 32 x 32 (channel, pixel) tile transposed through shared memory.
+__global__ void to_bf16_nhwc_kernel(const float *__restrict__ x, int C, int HW, uint16_t *__restrict__ out) {
+    __shared__ float tile[32][33];
+    const int b = blockIdx.z, c0 = blockIdx.y * 32, p0 = blockIdx.x * 32;
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int c = c0 + i, p = p0 + threadIdx.x;
+        tile[i][threadIdx.x] = (c < C && p < HW) ? x[((int64_t)b * C + c) * HW + p] : 0.0f;
+    }
+    __syncthreads();
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int p = p0 + i, c = c0 + threadIdx.x;
+        if (c < C && p < HW)
+            out[((int64_t)b * HW + p) * C + c] = __bfloat16_as_ushort(__float2bfloat16_rn(tile[threadIdx.x][i]));
+    }
+}
+
 }  // namespace minw
 
 // ===========================================================================
@@ -571,6 +615,27 @@ minw_status minw_pack_weight_codes(const float *w, int32_t O, int32_t C, int32_t
     const int64_t g = grid_for(items, 256);
     weight_codes_kernel<<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(w, O, C, kh, kw, to_qparams(q),
                                                                       channel_scale, codes);
+    return launch_status();
+}
+
+minw_status minw_pack_weight_bf16(const float *w, int32_t O, int32_t C, int32_t kh, int32_t kw,
+                                  const minw_quant *q, const float *channel_scale, uint16_t *out, void *stream) {
+    if (O <= 0 || C <= 0 || kh <= 0 || kw <= 0 || !valid_quant(q) || !w || !out) return MINW_EINVAL;
+    if (C % 8 != 0 || !aligned16(out)) return MINW_EUNSUPPORTED;
+    const int64_t items = (int64_t)O * kh * kw * (C / 8);
+    const int64_t g = grid_for(items, 256);
+    weight_bf16_kernel<<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(w, O, C, kh, kw, to_qparams(q),
+                                                                     channel_scale, out);
+    return launch_status();
+}
+
+minw_status minw_to_bf16_nhwc(const float *x, int32_t B, int32_t C, int32_t H, int32_t W, uint16_t *out,
+                              void *stream) {
+    if (B <= 0 || C <= 0 || H <= 0 || W <= 0 || !x || !out) return MINW_EINVAL;
+    const int64_t HW = (int64_t)H * W;
+    if (HW > (1ll << 30) || B > 65535 || (C + 31) / 32 > 65535) return MINW_EUNSUPPORTED;
+    const dim3 grid((unsigned)((HW + 31) / 32), (unsigned)((C + 31) / 32), (unsigned)B);
+    to_bf16_nhwc_kernel<<<grid, dim3(32, 8), 0, (cudaStream_t)stream>>>(x, C, (int)HW, out);
     return launch_status();
 }
 

@@ -133,6 +133,26 @@ minw_status minw_conv2d_codes(const uint8_t *act, int32_t B, int32_t C, int32_t 
     return launch_conv_tc(a, (cudaStream_t)stream);
 }
 
+minw_status minw_conv2d_bf16(const uint16_t *act, int32_t B, int32_t C, int32_t H, int32_t W, const uint16_t *wgt,
+                             int32_t O, int32_t kh, int32_t kw, int32_t bits_w, int32_t stride, int32_t pad,
+                             int32_t pool, const float *scale, const float *shift, float *y_out, void *stream) {
+    ConvArgs a;
+    minw_status st = make_codes_args(a, reinterpret_cast<const uint8_t *>(act), B, C, H, W, 1,
+                                     reinterpret_cast<const uint8_t *>(wgt), O, kh, kw, bits_w, stride, pad);
+    if (st != MINW_OK) return st;
+    if (!scale || !shift || !y_out) return MINW_EINVAL;
+    if (pool != 0 && pool != 1) return MINW_EINVAL;
+    if (pool && ((a.Ho & 1) || (a.Wo & 1))) return MINW_EUNSUPPORTED;
+    if ((long long)B * H * W * C >= (1ll << 39)) return MINW_EUNSUPPORTED;
+    a.bf16 = 1;
+    a.bits_a = 0;
+    a.scale = scale;
+    a.shift = shift;
+    a.pool = pool;
+    a.y_out = y_out;
+    return launch_conv_tc(a, (cudaStream_t)stream);
+}
+
 minw_status minw_conv_block_codes(const uint8_t *act, int32_t B, int32_t C, int32_t H, int32_t W,
                                   int32_t bits_a, const uint8_t *wgt, int32_t O, int32_t kh, int32_t kw,
                                   int32_t bits_w, int32_t stride, int32_t pad, int32_t pool, const float *scale,

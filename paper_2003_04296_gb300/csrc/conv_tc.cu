@@ -53,9 +53,12 @@ constexpr long long WAIT_CYCLES = 1ll << 31;
 struct Params {
     int B, C, H, W, O, kh, kw, pad, Ho, Wo;
     int stride;                // 1 or 2 (TMA element strides)
-    int ck;                    // bytes (= channels) per K chunk: 128 (128-byte swizzle) or 64 (64-byte swizzle)
-    uint32_t a_bytes;          // activation box bytes of one K block: 128 rows x ck
-    uint32_t b_bytes;          // weight box bytes of one K block: BN rows x ck
+    int ck;                    // channels per K chunk
+    int esize;                 // operand bytes: 1 (E4M3 level codes) or 2 (bf16)
+    int cb;                    // bytes of one row of a K chunk: 128 (128-byte swizzle) or 64 (64-byte swizzle);
+                               // = ck for E4M3 level codes, 2 ck for bf16 operands
+    uint32_t a_bytes;          // activation box bytes of one K block: 128 rows x cb
+    uint32_t b_bytes;          // weight box bytes of one K block: BN rows x cb
     int trans;                 // 1: tile = 128 output channels (MMA M) x 256 pixels (MMA N)
     int mrows;                 // output pixels per tile: 128, or 256 when trans
     int acc_cols;              // TMEM columns of one accumulator: BN, or 256 when trans
@@ -207,6 +210,16 @@ __device__ __forceinline__ void mma_commit_mc(uint64_t *bar, uint16_t mask) {
             smem_u32(bar)),
         "h"(mask)
         : "memory");
+}
+
+// bf16 x bf16 -> fp32 (weight-only quantized layers: full-precision bf16
+// activations, weights at their exact level values).
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
 }
 
 // CTA pairs (cta_group::2).  The even CTA of a cluster of two issues each MMA
@@ -479,7 +492,9 @@ __device__ __forceinline__ void resid_chunk(uint32_t taddr, bool full32, const P
 
 // OUTB: bits of the quantized output (0 when the launch writes none).
 // PAIR: CTA pairs with cta_group::2 MMAs (a kernel uses one CTA group only).
-template <int OUTB, bool PAIR>
+// BF16: bf16 operands (kind::f16), else E4M3 level codes (kind::f8f6f4); both
+// consume 32 bytes of K per MMA step.
+template <int OUTB, bool PAIR, bool BF16>
 __global__ void __launch_bounds__(NT, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const Params p) {
@@ -633,10 +648,10 @@ __global__ void __launch_bounds__(NT, 1)
                         else if (p.cl == 1) {
                             uint8_t *sb = sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes;
                             tma_load_2d(sb, &tmB, &full[s], kcol, o0);
-                            if (p.dup) tma_load_2d(sb + (size_t)64 * p.ck, &tmB, &full[s], kcol, o0);
+                            if (p.dup) tma_load_2d(sb + (size_t)64 * p.cb, &tmB, &full[s], kcol, o0);
                         } else
                             tma_load_2d_mc(sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes +
-                                               (size_t)crank * bslice * p.ck,
+                                               (size_t)crank * bslice * p.cb,
                                            &tmB, &full[s], kcol, o0 + crank * bslice, cmask);
                         kcol += p.ck;
                         c0 += p.ck;
@@ -670,10 +685,10 @@ __global__ void __launch_bounds__(NT, 1)
             // stage minimal (descriptors advance by a constant per ring slot,
             // the K = 32 steps are unrolled).
             const uint32_t sbase = smem_u32(smem);
-            const uint64_t adesc0 = sw_desc(sbase, p.ck), bdesc0 = sw_desc(sbase + p.kps * p.a_bytes, p.ck);
+            const uint64_t adesc0 = sw_desc(sbase, p.cb), bdesc0 = sw_desc(sbase + p.kps * p.a_bytes, p.cb);
             const uint32_t dstep = p.stage_bytes >> 4;     // start-address step of one ring slot
             const uint32_t astep = p.a_bytes >> 4, bstep = p.b_bytes >> 4;   // second K block of a stage
-            const bool k128 = p.ck == 128;                 // four K = 32 steps per stage, else two
+            const bool k128 = p.cb == 128;                 // four 32-byte K steps per K block, else two
             const uint32_t idesc = p.idesc;
             for (int w = blockIdx.x; w < items && alive; w += gridDim.x, ++i) {
                 const int ab = i & 1, use = i >> 1;
@@ -688,6 +703,8 @@ __global__ void __launch_bounds__(NT, 1)
                 auto mma = [&](uint64_t ad_, uint64_t bd_, uint32_t a_) {
                     if constexpr (PAIR)
                         mma_f8_pair(tmem_d, ad_, bd_, idesc, a_);
+                    else if constexpr (BF16)
+                        mma_bf16(tmem_d, ad_, bd_, idesc, a_);
                     else
                         mma_f8(tmem_d, ad_, bd_, idesc, a_);
                 };
@@ -1361,8 +1378,10 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     p.B = a.B; p.C = a.C; p.H = a.H; p.W = a.W; p.O = a.O; p.kh = a.kh; p.kw = a.kw; p.pad = a.pad;
     p.Ho = a.Ho; p.Wo = a.Wo;
     p.stride = a.stride;
-    p.ck = (a.C % 128 == 0) ? 128 : 64;
-    p.a_bytes = (uint32_t)(p.mrows * p.ck);
+    p.esize = a.bf16 ? 2 : 1;
+    p.cb = (a.C * p.esize % 128 == 0) ? 128 : 64;
+    p.ck = p.cb / p.esize;
+    p.a_bytes = (uint32_t)(p.mrows * p.cb);
     p.nck = a.C / p.ck;
     p.nk = a.kh * a.kw * p.nck;
     p.nbb = (a.B + p.bb - 1) / p.bb;
@@ -1375,9 +1394,10 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
         const int tiles_ = p.nbx * p.nby * p.nbb * p.ntn;
         const int ks_ = (a.workspace != nullptr && !a.pool) ? (a.ksplit > 0 ? a.ksplit : auto_ksplit(tiles_, p.nk, sms_))
                                                             : 1;
-        p.pair = (pair_pref() && !p.trans && p.BN == 256 && a.O % 256 == 0 && p.nk >= 18 && ks_ <= 1) ? 1 : 0;
+        p.pair = (pair_pref() && !a.bf16 && !p.trans && p.BN == 256 && a.O % 256 == 0 && p.nk >= 18 && ks_ <= 1)
+                     ? 1 : 0;
     }
-    p.b_bytes = (uint32_t)((p.pair ? p.BN / 2 : p.BN) * p.ck);   // pairs: each CTA holds half the weight rows
+    p.b_bytes = (uint32_t)((p.pair ? p.BN / 2 : p.BN) * p.cb);   // pairs: each CTA holds half the weight rows
     const size_t o32 = ((size_t)a.O + 31) & ~(size_t)31;
     const size_t thr_bytes = a.quant_out ? (o32 * p.nlev + o32 / 32 + 10) * sizeof(float) : 0;
     const size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes;
@@ -1392,7 +1412,9 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     // MMA N: the output channels, or the 256 pixels of a channel-major tile (M = 128 either way)
     const int mma_n = p.trans ? 256 : p.BN;
     p.acc_cols = mma_n;
-    p.idesc = (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(mma_n >> 3) << 17) |
+    // D fp32; A and B E4M3 (kind::f8f6f4) or bf16 (kind::f16)
+    const uint32_t fmt = a.bf16 ? 1u : 0u;
+    p.idesc = (1u << 4) | (fmt << 7) | (fmt << 10) | ((uint32_t)(mma_n >> 3) << 17) |
               ((uint32_t)((p.pair ? 256 : 128) >> 4) << 24);
     uint32_t cols = 32;
     while ((int)cols < 2 * mma_n) cols <<= 1;         // two accumulators
@@ -1407,7 +1429,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
     p.ksplit = 1;
     pl.thr_ws = nullptr;
-    if (a.workspace != nullptr && !a.pool && !p.trans && !p.pair) {
+    if (a.workspace != nullptr && !a.pool && !p.trans && !p.pair && !a.bf16) {
         // workspace: [breakpoints, when not given][ksplit partial-sum slices]
         const size_t tb = (a.quant_out && a.thr == nullptr) ? thr_ws_bytes(a.O, p.nlev) : 0;
         const size_t sb = slice_bytes(tiles, p.BN);
@@ -1439,14 +1461,17 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     p.tiles_mp = (tiles_m + p.cl - 1) / p.cl * p.cl;
     minw_host::EncodeTiledFn enc = minw_host::tensor_map_encoder();
     if (enc == nullptr) return MINW_ECUDA;
-    const CUtensorMapSwizzle swz = p.ck == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+    const CUtensorMapSwizzle swz = p.cb == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+    const CUtensorMapDataType dt = a.bf16 ? CU_TENSOR_MAP_DATA_TYPE_UINT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8;
+    const cuuint64_t es_ = (cuuint64_t)p.esize;
     {
         const cuuint64_t dims[4] = {(cuuint64_t)a.C, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.B};
-        const cuuint64_t strides[3] = {(cuuint64_t)a.C, (cuuint64_t)a.W * a.C, (cuuint64_t)a.H * a.W * a.C};
+        const cuuint64_t strides[3] = {(cuuint64_t)a.C * es_, (cuuint64_t)a.W * a.C * es_,
+                                       (cuuint64_t)a.H * a.W * a.C * es_};
         const cuuint32_t sd = (cuuint32_t)p.stride;
         const cuuint32_t box[4] = {(cuuint32_t)p.ck, (cuuint32_t)p.bw * sd, (cuuint32_t)p.bh * sd, (cuuint32_t)p.bb};
         const cuuint32_t es[4] = {1u, sd, sd, 1u};
-        if (enc(&pl.tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<uint8_t *>(a.act8), dims, strides, box, es,
+        if (enc(&pl.tmA, dt, 4, const_cast<uint8_t *>(a.act8), dims, strides, box, es,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return MINW_ECUDA;
@@ -1454,10 +1479,10 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     {
         const long long K = (long long)a.kh * a.kw * a.C;
         const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)a.O};
-        const cuuint64_t strides[1] = {(cuuint64_t)K};
+        const cuuint64_t strides[1] = {(cuuint64_t)K * es_};
         const cuuint32_t box[2] = {(cuuint32_t)p.ck, (cuuint32_t)(p.dup ? 64 : p.BN / p.cl)};
         const cuuint32_t es[2] = {1u, 1u};
-        if (enc(&pl.tmB, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(a.wgt8), dims, strides, box, es,
+        if (enc(&pl.tmB, dt, 2, const_cast<uint8_t *>(a.wgt8), dims, strides, box, es,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return MINW_ECUDA;
@@ -1517,18 +1542,21 @@ size_t conv_tc_min_split_bytes(const ConvArgs &a) {
     return tc::thr_ws_bytes(a.O, 7) + 2 * tc::slice_bytes(tiles, p.BN);
 }
 
+static bool conv_tc_residual(const ConvArgs &a) {
+    return a.res_codes != nullptr || a.res_f32 != nullptr || a.y_nhwc != nullptr;
+}
+
 bool conv_tc_supported(const ConvArgs &a) {
     tc::Params p{};
     if (!tc::plan_shape(a, p)) return false;
+    // bf16 operands: real-valued accumulators, so fp32 BN outputs only
+    if (a.bf16 && (a.quant_out || a.acc_out != nullptr || a.y_out == nullptr || conv_tc_residual(a))) return false;
     if (a.quant_out && (size_t)a.O * num_levels(a.qo.bits) * sizeof(float) > 64 * 1024) return false;
     if (a.quant_out && a.codes_out != nullptr && a.O % 16 != 0) return false;
     if (a.acc_out != nullptr && a.pool) return false;
     return true;
 }
 
-static bool conv_tc_residual(const ConvArgs &a) {
-    return a.res_codes != nullptr || a.res_f32 != nullptr || a.y_nhwc != nullptr;
-}
 
 int conv_tc_launches(const ConvArgs &a) {
     if (a.workspace == nullptr || a.pool) return 1;
@@ -1556,14 +1584,14 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
     static size_t configured[4] = {0, 0, 0, 0};
     typedef void (*TcKernel)(const CUtensorMap, const CUtensorMap, const tc::Params);
     static const TcKernel kernels[2][4] = {
-        {tc::conv_tc_kernel<0, false>, tc::conv_tc_kernel<1, false>, tc::conv_tc_kernel<2, false>,
-         tc::conv_tc_kernel<3, false>},
-        {tc::conv_tc_kernel<0, true>, tc::conv_tc_kernel<1, true>, tc::conv_tc_kernel<2, true>,
-         tc::conv_tc_kernel<3, true>}};
-    static size_t configured_pair[4] = {0, 0, 0, 0};
+        {tc::conv_tc_kernel<0, false, false>, tc::conv_tc_kernel<1, false, false>,
+         tc::conv_tc_kernel<2, false, false>, tc::conv_tc_kernel<3, false, false>},
+        {tc::conv_tc_kernel<0, true, false>, tc::conv_tc_kernel<1, true, false>, tc::conv_tc_kernel<2, true, false>,
+         tc::conv_tc_kernel<3, true, false>}};
+    static size_t configured_pair[4] = {0, 0, 0, 0}, configured_bf16 = 0;
     const int kp = pl.p.pair ? 1 : 0;
-    TcKernel kern = kernels[kp][kout];
-    size_t &conf = kp ? configured_pair[kout] : configured[kout];
+    TcKernel kern = a.bf16 ? tc::conv_tc_kernel<0, false, true> : kernels[kp][kout];
+    size_t &conf = a.bf16 ? configured_bf16 : kp ? configured_pair[kout] : configured[kout];
     if (pl.smem > conf) {
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem) != cudaSuccess)
             return MINW_ECUDA;

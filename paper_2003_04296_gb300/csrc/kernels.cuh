@@ -23,9 +23,10 @@ struct ConvArgs {
     QParams qo;            // quantizer of the output
     uint32_t *planes_out;  // [B][Hp][Wp][qo.bits][ceil(O/32)] (nullable)
     uint8_t *codes_out;    // [B][Hp][Wp][O] E4M3 level codes (nullable; O % 16 == 0)
-    // tensor-core operands: E4M3 level codes
+    // tensor-core operands: E4M3 level codes, or bf16 values when bf16 is set
     const uint8_t *act8;   // [B][H][W][C]
     const uint8_t *wgt8;   // [O][kh][kw][C]
+    int bf16;              // operands are bf16 (weight-only quantized layers): fp32 outputs only
     const float *thr;      // output-quantizer breakpoints [O][levels] (nullable: computed in-kernel)
     // residual blocks (tensor-core path): y = BN(acc) + shortcut before HardTanh + quantize
     const uint8_t *res_codes;  // shortcut as level codes [B][Hp][Wp][O] (nullable)

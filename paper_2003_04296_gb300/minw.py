@@ -65,6 +65,10 @@ SIGNATURES = {
     "aqe_forward": (ctypes.c_int, [_P, _P, _I64, _F, _QP, _P]),
     "aqe_backward": (ctypes.c_int, [_P, _P, _P, _I64, _F, _P]),
     "aqe_forward_stochastic": (ctypes.c_int, [_P, _P, _I64, _F, ctypes.c_uint64, ctypes.c_uint64, _P]),
+    "minw_to_bf16_nhwc": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _P]),
+    "minw_pack_weight_bf16": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
+    "minw_conv2d_bf16": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32, _I32, _I32,
+                                        _I32, _P, _P, _P, _P]),
     "aqe_quantize_pack": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _F, _P, _P, _P]),
     "aqe_backward_masked": (ctypes.c_int, [_P, _P, _P, _I64, _F, _P]),
     "minw_pack_weights": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
@@ -189,6 +193,24 @@ def aqe_forward_stochastic(x, y, alpha, seed, offset=0, stream=None):
     call for fresh noise)."""
     _check(lib().aqe_forward_stochastic(_ptr(x), _ptr(y), x.numel(), float(alpha), int(seed) & (2**64 - 1),
                                         int(offset) & (2**64 - 1), _stream(stream)), "aqe_forward_stochastic")
+
+
+def minw_to_bf16_nhwc(x, out, stream=None):
+    """fp32 NCHW -> bf16 NHWC (out: a uint16 or bfloat16 tensor [B][H][W][C])."""
+    B, C, H, W = x.shape
+    _check(lib().minw_to_bf16_nhwc(_ptr(x), B, C, H, W, _ptr(out), _stream(stream)), "minw_to_bf16_nhwc")
+
+
+def minw_pack_weight_bf16(w, q, out, channel_scale=None, stream=None):
+    """Latent weights [O][C][kh][kw] -> bf16 level values [O][kh][kw][C]."""
+    O, C, kh, kw = w.shape
+    _check(lib().minw_pack_weight_bf16(_ptr(w), O, C, kh, kw, ctypes.byref(q), _ptr(channel_scale), _ptr(out),
+                                       _stream(stream)), "minw_pack_weight_bf16")
+
+
+def minw_conv2d_bf16(act, B, C, H, W, wgt, O, kh, kw, bits_w, stride, pad, pool, scale, shift, y_out, stream=None):
+    _check(lib().minw_conv2d_bf16(_ptr(act), B, C, H, W, _ptr(wgt), O, kh, kw, bits_w, stride, pad, int(pool),
+                                  _ptr(scale), _ptr(shift), _ptr(y_out), _stream(stream)), "minw_conv2d_bf16")
 
 
 def aqe_backward(x, gy, gx, alpha, stream=None):

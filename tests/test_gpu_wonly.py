@@ -1,0 +1,140 @@
+"""GPU parity of the weight-only quantized convolution (full-precision bf16
+activations times 1-3-bit weights on the tcgen05 tensor cores, kind::f16)
+against the oracle, through the C ABI: the bf16 NHWC conversion and the bf16
+level weights bit for bit, and the convolution within the bound of fp32
+accumulation (the tensor core's summation order is its own):
+|y - y_ref| <= |scale| K 2^-23 A + 2^-23 |y_ref|, with A = sum |x w| of the
+output, which covers rounding or truncating additions; a wrong product, tap
+or channel breaks it by orders of magnitude."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from oracle import oracle as O  # noqa: E402
+from paper_2003_04296_gb300.inputs import DEFAULT_THR  # noqa: E402
+from tests._gpu import dev_tensor  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dev():
+    import __graft_entry__ as g
+    g.build()
+    assert torch.cuda.is_available()
+    return torch.device("cuda:0")
+
+
+@pytest.fixture(scope="module")
+def M(dev):
+    from paper_2003_04296_gb300 import minw
+    return minw
+
+
+def _operands(dev, M, x, w, bits, cs):
+    B, C, H, W = x.shape
+    O_, _, kh, kw = w.shape
+    xb = torch.empty((B, H, W, C), dtype=torch.int16, device=dev)
+    wb = torch.empty((O_, kh, kw, C), dtype=torch.int16, device=dev)
+    M.minw_to_bf16_nhwc(dev_tensor(x, dev), xb)
+    M.minw_pack_weight_bf16(dev_tensor(w, dev), M.quant(bits, DEFAULT_THR[bits]), wb,
+                            channel_scale=dev_tensor(cs, dev))
+    return xb, wb
+
+
+def _bf16_values(t):
+    """int16 bit patterns of bf16 -> fp32 values (upper half of the word)."""
+    u = t.cpu().numpy().view(np.uint16).astype(np.uint32) << 16
+    return u.view(np.float32)
+
+
+@pytest.mark.parametrize("shape", [(2, 64, 5, 7), (1, 128, 3, 9), (3, 96, 4, 4)])
+def test_to_bf16_nhwc(dev, M, shape):
+    x = (np.random.default_rng(sum(shape)).standard_normal(shape) * 3).astype(np.float32)
+    B, C, H, W = shape
+    out = torch.empty((B, H, W, C), dtype=torch.int16, device=dev)
+    M.minw_to_bf16_nhwc(dev_tensor(x, dev), out)
+    want = O.bf16_round(x).transpose(0, 2, 3, 1)
+    assert np.array_equal(_bf16_values(out).view(np.uint32), want.view(np.uint32))
+
+
+@pytest.mark.parametrize("bits", [1, 2, 3])
+def test_pack_weight_bf16(dev, M, bits):
+    w = np.random.default_rng(bits).normal(0, 0.05, (24, 64, 3, 3)).astype(np.float32)
+    cs = (1.0 / np.abs(w.reshape(24, -1)).max(1)).astype(np.float32)
+    out = torch.empty((24, 3, 3, 64), dtype=torch.int16, device=dev)
+    M.minw_pack_weight_bf16(dev_tensor(w, dev), M.quant(bits, DEFAULT_THR[bits]), out,
+                            channel_scale=dev_tensor(cs, dev))
+    units = O.quantize(w, bits, DEFAULT_THR[bits], cs) * 2.0 ** O.units_shift(bits)
+    assert np.array_equal(_bf16_values(out).astype(np.float64), units.transpose(0, 2, 3, 1))
+
+
+CASES = [(2, 64, 10, 12, 96, 1, 0), (3, 128, 9, 9, 128, 2, 0), (2, 256, 8, 8, 256, 1, 1), (1, 64, 7, 7, 320, 1, 0)]
+
+
+@pytest.mark.parametrize("case", CASES)
+@pytest.mark.parametrize("bits", [1, 2, 3])
+def test_conv2d_bf16(dev, M, case, bits):
+    B, C, H, W, O_, s, pool = case
+    r = np.random.default_rng(1000 * bits + sum(case))
+    x = r.standard_normal((B, C, H, W)).astype(np.float32)
+    w = r.normal(0, 0.05, (O_, C, 3, 3)).astype(np.float32)
+    cs = (1.0 / np.abs(w.reshape(O_, -1)).max(1)).astype(np.float32)
+    scale = r.normal(0.01, 0.005, O_).astype(np.float32)
+    shift = r.normal(0, 0.1, O_).astype(np.float32)
+    xb, wb = _operands(dev, M, x, w, bits, cs)
+    Ho, Wo = (H - 1) // s + 1, (W - 1) // s + 1
+    Hp, Wp = (Ho // 2, Wo // 2) if pool else (Ho, Wo)
+    y = torch.full((B, O_, Hp, Wp), np.nan, dtype=torch.float32, device=dev)
+    M.minw_conv2d_bf16(xb, B, C, H, W, wb, O_, 3, 3, bits, s, 1, pool, dev_tensor(scale, dev),
+                       dev_tensor(shift, dev), y)
+    torch.cuda.synchronize()
+    xr = O.bf16_round(x).astype(np.float64)
+    wu = O.quantize(w, bits, DEFAULT_THR[bits], cs) * 2.0 ** O.units_shift(bits)
+    acc = O.conv2d_real(xr, wu, s, 1)
+    A = O.conv2d_real(np.abs(xr), np.abs(wu), s, 1)
+    if pool:
+        acc, A = O.maxpool_f64(acc), O.maxpool_f64(A)
+    sc = scale.astype(np.float64)[None, :, None, None]
+    yref = acc * sc + shift.astype(np.float64)[None, :, None, None]
+    K = C * 9
+    bound = np.abs(sc) * K * 2.0 ** -23 * A + 2.0 ** -23 * np.abs(yref) + 1e-30
+    err = np.abs(y.cpu().numpy().astype(np.float64) - yref)
+    assert (err <= bound).all(), f"worst err/bound {np.max(err / bound)}"
+
+
+def test_conv2d_bf16_sweep_shape_sampled(dev, M):
+    """The bit-width sweep's shape, 256 x 512 x 14 x 14 -> 512 (3x3, K = 4608),
+    with 1-bit weights: images 0 and 255 against the oracle."""
+    B, C, H, W, O_ = 256, 512, 14, 14, 512
+    r = np.random.default_rng(77)
+    x = r.standard_normal((B, C, H, W)).astype(np.float32)
+    w = r.standard_normal((O_, C, 3, 3)).astype(np.float32)
+    cs = np.ones(O_, dtype=np.float32)
+    scale = np.full(O_, 1.0 / 64, dtype=np.float32)
+    shift = np.zeros(O_, dtype=np.float32)
+    xb, wb = _operands(dev, M, x, w, 1, cs)
+    y = torch.empty((B, O_, H, W), dtype=torch.float32, device=dev)
+    M.minw_conv2d_bf16(xb, B, C, H, W, wb, O_, 3, 3, 1, 1, 1, 0, dev_tensor(scale, dev), dev_tensor(shift, dev), y)
+    torch.cuda.synchronize()
+    pick = [0, B - 1]
+    xr = O.bf16_round(x[pick]).astype(np.float64)
+    wu = O.quantize(w, 1, DEFAULT_THR[1])
+    acc = O.conv2d_real(xr, wu, 1, 1)
+    A = O.conv2d_real(np.abs(xr), np.abs(wu), 1, 1)
+    yref = acc / 64.0
+    bound = (1.0 / 64) * C * 9 * 2.0 ** -23 * A + 2.0 ** -23 * np.abs(yref) + 1e-30
+    err = np.abs(y.cpu().numpy()[pick].astype(np.float64) - yref)
+    assert (err <= bound).all(), f"worst err/bound {np.max(err / bound)}"
+
+
+def test_conv2d_bf16_errors(dev, M):
+    xb = torch.zeros((1, 4, 4, 32), dtype=torch.int16, device=dev)
+    wb = torch.zeros((8, 3, 3, 32), dtype=torch.int16, device=dev)
+    sc = torch.ones(8, device=dev)
+    y = torch.empty((1, 8, 4, 4), device=dev)
+    with pytest.raises(M.MinwError):
+        M.minw_conv2d_bf16(xb, 1, 32, 4, 4, wb, 8, 3, 3, 1, 1, 1, 0, sc, sc, y)     # C % 64 != 0
+    with pytest.raises(M.MinwError):
+        M.minw_conv2d_bf16(xb, 1, 32, 4, 4, wb, 8, 3, 3, 1, 1, 1, 0, sc, sc, None)  # no output
