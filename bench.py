@@ -604,7 +604,7 @@ def run_sweep(args, rank, world, local_rank):
                 "frac": aqe_bytes / (sto_ms * 1e-3) / 1e9 / HBM_GBS, "algorithmic_bytes": aqe_bytes,
                 "peak_basis": "measured copy bandwidth, of measured"}
     wo_tf = 2.0 * mac / (wo_ms * 1e-3) / 1e12
-    wonly = {"kernel": "conv_tc_kernel<0, false, true> (tcgen05 kind::f16: bf16 activations x 1-bit weights)",
+    wonly = {"kernel": "conv_tc_kernel<0, true, true> (tcgen05 kind::f16, CTA pairs: bf16 activations x 1-bit weights)",
              "ms": round(wo_ms, 5), "achieved": wo_tf, "peak": BF16_TFLOPS, "unit": "TFLOP/s",
              "frac": wo_tf / BF16_TFLOPS, "peak_basis": "measured dense bf16 TFLOP/s (burst), of measured"}
     cpu = None

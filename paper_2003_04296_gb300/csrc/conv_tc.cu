@@ -234,6 +234,14 @@ __device__ __forceinline__ void mma_f8_pair(uint32_t tmem_d, uint64_t adesc, uin
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
 }
 
+__device__ __forceinline__ void mma_bf16_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                              uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
+}
+
 // Arrive on the barrier at this offset in both CTAs of the pair once the
 // pair's MMAs issued so far have completed.
 __device__ __forceinline__ void mma_commit_pair(uint64_t *bar) {
@@ -701,7 +709,9 @@ __global__ void __launch_bounds__(NT, 1)
                 const uint32_t tmem_d = tmem_base + (uint32_t)(ab * p.acc_cols);
                 uint32_t acc = 0u;
                 auto mma = [&](uint64_t ad_, uint64_t bd_, uint32_t a_) {
-                    if constexpr (PAIR)
+                    if constexpr (PAIR && BF16)
+                        mma_bf16_pair(tmem_d, ad_, bd_, idesc, a_);
+                    else if constexpr (PAIR)
                         mma_f8_pair(tmem_d, ad_, bd_, idesc, a_);
                     else if constexpr (BF16)
                         mma_bf16(tmem_d, ad_, bd_, idesc, a_);
@@ -1394,8 +1404,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
         const int tiles_ = p.nbx * p.nby * p.nbb * p.ntn;
         const int ks_ = (a.workspace != nullptr && !a.pool) ? (a.ksplit > 0 ? a.ksplit : auto_ksplit(tiles_, p.nk, sms_))
                                                             : 1;
-        p.pair = (pair_pref() && !a.bf16 && !p.trans && p.BN == 256 && a.O % 256 == 0 && p.nk >= 18 && ks_ <= 1)
-                     ? 1 : 0;
+        p.pair = (pair_pref() && !p.trans && p.BN == 256 && a.O % 256 == 0 && p.nk >= 18 && ks_ <= 1) ? 1 : 0;
     }
     p.b_bytes = (uint32_t)((p.pair ? p.BN / 2 : p.BN) * p.cb);   // pairs: each CTA holds half the weight rows
     const size_t o32 = ((size_t)a.O + 31) & ~(size_t)31;
@@ -1588,10 +1597,11 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
          tc::conv_tc_kernel<2, false, false>, tc::conv_tc_kernel<3, false, false>},
         {tc::conv_tc_kernel<0, true, false>, tc::conv_tc_kernel<1, true, false>, tc::conv_tc_kernel<2, true, false>,
          tc::conv_tc_kernel<3, true, false>}};
-    static size_t configured_pair[4] = {0, 0, 0, 0}, configured_bf16 = 0;
+    static size_t configured_pair[4] = {0, 0, 0, 0}, configured_bf16[2] = {0, 0};
     const int kp = pl.p.pair ? 1 : 0;
-    TcKernel kern = a.bf16 ? tc::conv_tc_kernel<0, false, true> : kernels[kp][kout];
-    size_t &conf = a.bf16 ? configured_bf16 : kp ? configured_pair[kout] : configured[kout];
+    TcKernel kern = a.bf16 ? (kp ? tc::conv_tc_kernel<0, true, true> : tc::conv_tc_kernel<0, false, true>)
+                           : kernels[kp][kout];
+    size_t &conf = a.bf16 ? configured_bf16[kp] : kp ? configured_pair[kout] : configured[kout];
     if (pl.smem > conf) {
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem) != cudaSuccess)
             return MINW_ECUDA;
