@@ -84,7 +84,9 @@ class Workload:
         self.name = name
         if name == "cifar_convnet":
             self.batch, self.seed = 256, 2
-            self.params = I.convnet_params(self.seed, bits_a=args.bits_a, bits_w=args.bits_w)
+            self.model = getattr(args, "model", "A")
+            self.params = I.convnet_params(self.seed, bits_a=args.bits_a, bits_w=args.bits_w,
+                                           **I.CIFAR_MODELS[self.model])
             self.bits = (args.bits_a, args.bits_w)
         else:
             self.batch, self.seed = 128, 4
@@ -133,9 +135,15 @@ class Workload:
         ba, bw = self.bits
         par = f"replicas x{n_gpus} (batch-sharded, no collective)"
         if self.name == "cifar_convnet":
-            return {"workload": f"cifar_convnet_fwd_a{ba}w{bw}", "batch_per_gpu": self.batch,
+            from paper_2003_04296_gb300.inputs import CIFAR_MODELS
+            m = CIFAR_MODELS[self.model]
+            w = m["widths"]
+            layers = (f"conv3x3 {w[0]},{w[1]},P,{w[2]},{w[3]},P,{w[4]},{w[5]},P; "
+                      f"fc {m['fcs'][0]},{m['fcs'][1]},10")
+            tag = "" if self.model == "A" else f"_model{self.model}"
+            return {"workload": f"cifar_convnet{tag}_fwd_a{ba}w{bw}", "batch_per_gpu": self.batch,
                     "global_batch": self.batch * n_gpus, "input": "3x32x32 fp32 U(-1,1)",
-                    "layers": "conv3x3 128,128,P,256,256,P,512,512,P; fc 1024,1024,10",
+                    "layers": layers,
                     "bits_a": ba, "bits_w": bw, "first_layer": "fp32 input, quantized weights",
                     "parallelism": par, "l2": L2_NOTE}
         return {"workload": f"resnet18_fwd_a{ba}w{bw}", "batch_per_gpu": self.batch,
@@ -647,6 +655,8 @@ def main():
     ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "sweep"], default="cifar_convnet")
     ap.add_argument("--bits-a", type=int, default=1, help="CIFAR ConvNet activation bits")
     ap.add_argument("--bits-w", type=int, default=1, help="CIFAR ConvNet weight bits")
+    ap.add_argument("--model", choices=["A", "B", "C", "D"], default="A",
+                    help="CIFAR ConvNet of Sec. IV-B (B-D: fewer channels)")
     ap.add_argument("--bits-a-resnet", type=int, default=3)
     ap.add_argument("--bits-w-resnet", type=int, default=3)
     ap.add_argument("--variant", type=int, default=0, help="0 auto, 1 popcount, 2 tensor cores")

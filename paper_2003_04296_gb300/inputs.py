@@ -119,6 +119,17 @@ def aqe_problem(seed, n, alpha=0.75):
     return dict(x=x, g=g, alpha=alpha)
 
 
+# The ConvNets of Sec. IV-B: Model A, then B with half the channels of every
+# convolution, C with B's convolutions and half the units of the hidden fully
+# connected layers, D with half of C's.
+CIFAR_MODELS = {
+    "A": dict(widths=(128, 128, 256, 256, 512, 512), fcs=(1024, 1024)),
+    "B": dict(widths=(64, 64, 128, 128, 256, 256), fcs=(1024, 1024)),
+    "C": dict(widths=(64, 64, 128, 128, 256, 256), fcs=(512, 512)),
+    "D": dict(widths=(64, 64, 128, 128, 256, 256), fcs=(256, 256)),
+}
+
+
 def convnet_params(seed, bits_a=1, bits_w=1, widths=(128, 128, 256, 256, 512, 512),
                    pools=(False, True, False, True, False, True), fcs=(1024, 1024),
                    classes=10, in_ch=3, hw=32, w_sigma=0.05):

@@ -60,6 +60,20 @@ def test_small_convnet_tensor_cores(dev, M, bits_a, bits_w):
     assert np.array_equal(got, ref)
 
 
+@pytest.mark.parametrize("model", ["B", "C", "D"])
+@pytest.mark.parametrize("bits_a,bits_w", [(1, 1), (2, 1)])
+def test_cifar_models_b_to_d(dev, M, model, bits_a, bits_w):
+    """Models B-D of Sec. IV-B (Model A with half the convolution channels,
+    then half the hidden FC units, twice) at 32 x 32, batch 20, against the
+    oracle's logits bit for bit."""
+    from paper_2003_04296_gb300.inputs import CIFAR_MODELS
+    net_p = convnet_params(60 + ord(model), bits_a=bits_a, bits_w=bits_w, **CIFAR_MODELS[model])
+    x = convnet_input(61 + ord(model), 20)
+    got = _run(dev, M, net_p, x, M.VARIANT_AUTO)
+    ref = N.convnet_forward(net_p, x)
+    assert np.array_equal(got, ref)
+
+
 def test_cifar_convnet_batch256_sampled(dev, M):
     """The full Model-A-shaped ConvNet (128-128-P-256-256-P-512-512-P,
     FC 1024-1024-10), 1-bit, batch 256; images 0 and 255 re-run by the oracle."""
