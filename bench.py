@@ -296,6 +296,9 @@ def run_reference(args, rank):
         return 0
     if args.workload == "sweep":
         return run_reference_sweep(args)
+    if args.workload == "fc_train":
+        print(json.dumps({"impl": "reference", "unavailable": "the CPU oracle arm covers the inference workloads only"}))
+        return 0
     wl = Workload(args.workload, args)
     x = wl.images(0)
     B = wl.batch
@@ -477,6 +480,92 @@ def sweep_config(n_gpus):
             "parallelism": f"replicas x{n_gpus} (batch-sharded, no collective)", "l2": L2_NOTE}
 
 
+def run_fc_train(args, rank, world, local_rank):
+    """Algorithm 1's training step of Model A's first fully connected layer
+    (8192 -> 1024, batch 256, 1-bit weights and activations, alpha 0.75): the
+    weight AQE, the forward product, the activation AQE and its backward mask,
+    the input and weight gradients, the mask of Eq. weight and the clipped
+    update, through minw_fc_train_step.  Its three tensor-core products hold
+    6 B K O flops; the roofline is the measured bf16 rate."""
+    import torch
+    import __graft_entry__ as g
+    if rank == 0:
+        g.build()
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    from paper_2003_04296_gb300 import minw
+    from paper_2003_04296_gb300.inputs import DEFAULT_THR
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    B, K, O = 256, 8192, 1024
+    r = np.random.default_rng(31 + 1000 * rank)
+    A = torch.from_numpy(np.clip(r.standard_normal((B, K)), -1.5, 1.5).astype(np.float32)).to(dev)
+    W = torch.from_numpy(r.uniform(-1, 1, (O, K)).astype(np.float32)).to(dev)
+    G = torch.from_numpy((r.standard_normal((B, O)) * 0.1).astype(np.float32)).to(dev)
+    a_out = torch.empty((B, O), device=dev)
+    g_in = torch.empty((B, K), device=dev)
+    ws = torch.empty(minw.minw_fc_train_workspace_bytes(B, K, O), dtype=torch.uint8, device=dev)
+    qw, qa = minw.quant(1, DEFAULT_THR[1]), minw.quant(1, DEFAULT_THR[1])
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        minw.minw_fc_train_step(A, W, G, 0.75, 1e-3, qw, qa, a_out, g_in, ws)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    e0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    e1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    with ClockSampler(local_rank) as clk:
+        for k in range(args.steps):
+            flush.zero_()
+            e0[k].record(stream)
+            step()
+            e1[k].record(stream)
+        torch.cuda.synchronize()
+    ms_max = max_over_ranks(sum(e0[k].elapsed_time(e1[k]) for k in range(args.steps)) / args.steps, world, dev)
+    # end to end: the batch and the upstream gradient from pinned host memory, the input gradient back
+    A_host = A.cpu().pin_memory()
+    G_host = G.cpu().pin_memory()
+    gin_host = torch.empty((B, K), dtype=torch.float32).pin_memory()
+    e2e_s = []
+    for k in range(min(args.steps, 20) + 1):
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        A.copy_(A_host, non_blocking=True)
+        G.copy_(G_host, non_blocking=True)
+        step()
+        gin_host.copy_(g_in, non_blocking=True)
+        torch.cuda.synchronize()
+        if k:
+            e2e_s.append(time.perf_counter() - t0)
+    e2e_sec = max_over_ranks(sum(e2e_s) / len(e2e_s), world, dev)
+    if rank != 0:
+        return 0
+    flops = 6.0 * B * K * O
+    achieved = flops / (ms_max * 1e-3) / 1e12
+    line = {"metric": "Algorithm 1 training step of a fully connected MINW layer: images/s",
+            "value": replica_throughput(B, world, ms_max * 1e-3), "unit": "images/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "fc_train_8192x1024_b256_a1w1", "batch_per_gpu": B, "global_batch": B * world,
+                       "layer": "FC 8192 -> 1024 (Model A's fc1), alpha 0.75, lr 1e-3, SGD + clip",
+                       "parallelism": f"replicas x{world} (no gradient all-reduce)", "l2": L2_NOTE},
+            "roofline": {"bound": "tensor", "kernel": "conv_tc_kernel<0, *, true> (three bf16 products)",
+                         "achieved": achieved, "peak": BF16_TFLOPS, "unit": "TFLOP/s",
+                         "frac": achieved / BF16_TFLOPS, "traffic": None,
+                         "peak_basis": "measured dense bf16 TFLOP/s (burst), of measured"},
+            "cpu_baseline": None,
+            "e2e": {"value": replica_throughput(B, world, e2e_sec), "unit": "images/s",
+                    "h2d_bytes_per_step": int(4 * (A.numel() + G.numel())), "d2h_bytes_per_step": int(4 * g_in.numel())},
+            "gpu_launches": 18 * args.steps, "clocks": clk.summary()}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_sweep(args, rank, world, local_rank):
     """One step: quantize the input to level codes and convolve it with the
     weight codes for each of the nine bit-width pairs (int32 accumulators),
@@ -652,7 +741,7 @@ def main():
                     help="timed steps (default 1000 for the ConvNet, 100 for ResNet-18: about a second)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["minw", "reference"], default="minw")
-    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "sweep"], default="cifar_convnet")
+    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "sweep", "fc_train"], default="cifar_convnet")
     ap.add_argument("--bits-a", type=int, default=1, help="CIFAR ConvNet activation bits")
     ap.add_argument("--bits-w", type=int, default=1, help="CIFAR ConvNet weight bits")
     ap.add_argument("--model", choices=["A", "B", "C", "D"], default="A",
@@ -664,7 +753,7 @@ def main():
     ap.add_argument("--skip-cpu", action="store_true")
     args = ap.parse_args()
     if args.steps is None:
-        args.steps = {"cifar_convnet": 1000, "resnet18": 100, "sweep": 20}[args.workload]
+        args.steps = {"cifar_convnet": 1000, "resnet18": 100, "sweep": 20, "fc_train": 200}[args.workload]
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -679,6 +768,8 @@ def main():
     try:
         if args.workload == "sweep":
             return run_sweep(args, rank, world, local_rank)
+        if args.workload == "fc_train":
+            return run_fc_train(args, rank, world, local_rank)
         return run_gpu(args, rank, world, local_rank)
     finally:
         if world > 1:

@@ -261,6 +261,41 @@ MINW_API minw_status minw_conv2d_bf16(const uint16_t *act, int32_t B, int32_t C,
                                       int32_t stride, int32_t pad, int32_t pool, const float *scale,
                                       const float *shift, float *y_out, void *stream);
 
+/* ---------------------------------------------------------------------- */
+/* Training step of a fully connected layer (Algorithm 1)                  */
+/* ---------------------------------------------------------------------- */
+
+/* out (bf16, round to nearest even, row-major (transpose ? cols : rows) x
+ * out_cols) = in (fp32 row-major rows x cols), transposed when transpose != 0,
+ * zero in the columns past the source's.  out_cols >= the source's columns. */
+MINW_API minw_status minw_bf16_matrix(const float *in, int32_t rows, int32_t cols, int32_t transpose,
+                                      int32_t out_cols, uint16_t *out, void *stream);
+
+/* The update of Algorithm 1 with a plain gradient step:
+ * w = min(1, max(-1, fmaf(-lr, g, w))), n floats in place. */
+MINW_API minw_status minw_sgd_clip(float *w, const float *g, int64_t n, float lr, void *stream);
+
+/* Bytes of device workspace minw_fc_train_step needs (0 for bad sizes). */
+MINW_API size_t minw_fc_train_workspace_bytes(int32_t B, int32_t K, int32_t O);
+
+/* One step of Algorithm 1 for a fully connected layer with input A [B][K]
+ * (fp32, the previous layer's AQE output or the network input), latent
+ * weights W [O][K] (fp32, updated in place) and the upstream gradient g_out
+ * [B][O] = dL/d(a_out):
+ *   W^ = fmaf(alpha, h_w(W), (1 - alpha) W)        (Eq. weight, q_w)
+ *   a~ = bf16(A) bf16(W^)^T                         (tensor cores, fp32 sums)
+ *   a_out = fmaf(alpha, h_a(a~), (1 - alpha) a~)    (Eq. activation, q_a; a_out = a~ when q_a is null: last layer)
+ *   g_a~ = 2 alpha g_out 1[|a~| <= 1]               (Eq. activation; g_out itself when q_a is null)
+ *   g_in = bf16(g_a~) bf16(W^)                      ([B][K], skipped when g_in is null)
+ *   g_W^ = bf16(g_a~)^T bf16(A)                     ([O][K])
+ *   W = min(1, max(-1, W - lr 2 alpha g_W^ 1[|W| <= 1]))   (Eq. weight, update and clip)
+ * Requirements: K % 64 == 0 and B % 64 == 0 (else MINW_EUNSUPPORTED), alpha in
+ * [0, 1], 16-byte aligned pointers, workspace of minw_fc_train_workspace_bytes. */
+MINW_API minw_status minw_fc_train_step(const float *A, float *W, const float *g_out, int32_t B, int32_t K,
+                                        int32_t O, float alpha, float lr, const minw_quant *q_w,
+                                        const minw_quant *q_a, float *a_out, float *g_in, void *workspace,
+                                        size_t workspace_bytes, void *stream);
+
 /* Extra inputs and outputs of a residual block (ResNet-style MINW-Net,
  * where the paper leaves the block wiring open).  Host struct.
  * res_codes (nullable): shortcut as level codes [B][Hp][Wp][O] of bit width

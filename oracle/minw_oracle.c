@@ -109,6 +109,37 @@ void orc_aqe_backward(const float *x, const float *g, int64_t n, double alpha,
 }
 
 /* ------------------------------------------------------------------------ */
+/* Training step pieces in the fp32 operations the step is defined with      */
+/* (Algorithm 1): each is one IEEE operation per element, written out        */
+/* ------------------------------------------------------------------------ */
+
+/* Eq. activation / Eq. weight forward in fp32: fmaf(alpha, h(x), (1 - alpha) x)
+ * with 1 - alpha and (1 - alpha) x each rounded to fp32. */
+void orc_aqe_forward_f32(const float *x, int64_t n, float alpha, int bits, const float *thr, float scale, float *y)
+{
+    const float oma = 1.0f - alpha;
+    for (int64_t i = 0; i < n; ++i) {
+        const float h = (float)orc_h(x[i], bits, thr, scale);
+        const float t = oma * x[i];
+        y[i] = fmaf(alpha, h, t);
+    }
+}
+
+/* Eq. activation / Eq. weight backward in fp32: (|x| <= 1) ? g (2 alpha) : 0. */
+void orc_aqe_backward_f32(const float *x, const float *g, int64_t n, float alpha, float *gx)
+{
+    const float two_alpha = 2.0f * alpha;
+    for (int64_t i = 0; i < n; ++i) gx[i] = (fabsf(x[i]) <= 1.0f) ? g[i] * two_alpha : 0.0f;
+}
+
+/* The update of Algorithm 1 with a plain gradient step and the clip:
+ * w = min(1, max(-1, fmaf(-lr, g, w))). */
+void orc_sgd_clip(float *w, const float *g, int64_t n, float lr)
+{
+    for (int64_t i = 0; i < n; ++i) w[i] = fminf(1.0f, fmaxf(-1.0f, fmaf(-lr, g[i], w[i])));
+}
+
+/* ------------------------------------------------------------------------ */
 /* Stochastic AQE (Eq. our): h = alpha sign(a - z) + (1 - alpha) a, z ~ U[-1,1] */
 /* ------------------------------------------------------------------------ */
 

@@ -36,6 +36,9 @@ def lib():
         L.orc_quantize.argtypes = [P, i64, i64, i32, P, P, P]
         L.orc_aqe_forward.argtypes = [P, i64, f64, i32, P, f32, P]
         L.orc_aqe_backward.argtypes = [P, P, i64, f64, P]
+        L.orc_aqe_forward_f32.argtypes = [P, i64, f32, i32, P, f32, P]
+        L.orc_aqe_backward_f32.argtypes = [P, P, i64, f32, P]
+        L.orc_sgd_clip.argtypes = [P, P, i64, f32]
         u64 = ctypes.c_uint64
         L.orc_philox4x64_10.argtypes = [P, P, P]
         L.orc_aqe_forward_stochastic.argtypes = [P, i64, f64, u64, u64, P, P]
@@ -123,6 +126,33 @@ def aqe_backward(x, g, alpha):
     gx = np.empty(x.shape, dtype=np.float64)
     lib().orc_aqe_backward(_p(x), _p(g), x.size, float(alpha), _p(gx))
     return gx
+
+
+def aqe_forward_f32(x, alpha, bits, thr=None, scale=1.0):
+    """Eq. activation / Eq. weight forward in the fp32 operations of a training
+    step: fmaf(alpha, h(x), (1 - alpha) x), each product rounded to fp32."""
+    x = _f32(x)
+    y = np.empty(x.shape, dtype=np.float32)
+    lib().orc_aqe_forward_f32(_p(x), x.size, float(np.float32(alpha)), bits, _p(_thr(thr)),
+                              float(np.float32(scale)), _p(y))
+    return y
+
+
+def aqe_backward_f32(x, g, alpha):
+    """Eq. activation / Eq. weight backward in fp32: (|x| <= 1) ? g (2 alpha) : 0."""
+    x, g = _f32(x), _f32(g)
+    gx = np.empty(x.shape, dtype=np.float32)
+    lib().orc_aqe_backward_f32(_p(x), _p(g), x.size, float(np.float32(alpha)), _p(gx))
+    return gx
+
+
+def sgd_clip(w, g, lr):
+    """Algorithm 1's update with a plain gradient step: min(1, max(-1, w - lr g))
+    (one fmaf), returned as a new fp32 array."""
+    w = _f32(w).copy()
+    g = _f32(g)
+    lib().orc_sgd_clip(_p(w), _p(g), w.size, float(np.float32(lr)))
+    return w
 
 
 def philox4x64_10(counter, key):

@@ -69,6 +69,11 @@ SIGNATURES = {
     "minw_pack_weight_bf16": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
     "minw_conv2d_bf16": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32, _I32, _I32,
                                         _I32, _P, _P, _P, _P]),
+    "minw_bf16_matrix": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _P]),
+    "minw_sgd_clip": (ctypes.c_int, [_P, _P, _I64, _F, _P]),
+    "minw_fc_train_workspace_bytes": (ctypes.c_size_t, [_I32, _I32, _I32]),
+    "minw_fc_train_step": (ctypes.c_int, [_P, _P, _P, _I32, _I32, _I32, _F, _F, _QP, _QP, _P, _P, _P,
+                                          ctypes.c_size_t, _P]),
     "aqe_quantize_pack": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _F, _P, _P, _P]),
     "aqe_backward_masked": (ctypes.c_int, [_P, _P, _P, _I64, _F, _P]),
     "minw_pack_weights": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
@@ -211,6 +216,33 @@ def minw_pack_weight_bf16(w, q, out, channel_scale=None, stream=None):
 def minw_conv2d_bf16(act, B, C, H, W, wgt, O, kh, kw, bits_w, stride, pad, pool, scale, shift, y_out, stream=None):
     _check(lib().minw_conv2d_bf16(_ptr(act), B, C, H, W, _ptr(wgt), O, kh, kw, bits_w, stride, pad, int(pool),
                                   _ptr(scale), _ptr(shift), _ptr(y_out), _stream(stream)), "minw_conv2d_bf16")
+
+
+def minw_bf16_matrix(x, out, transpose=False, stream=None):
+    """fp32 matrix [rows][cols] -> bf16 (int16 bit patterns), transposed when asked,
+    zero-padded to out's column count."""
+    rows, cols = x.shape
+    _check(lib().minw_bf16_matrix(_ptr(x), rows, cols, int(bool(transpose)), out.shape[1], _ptr(out),
+                                  _stream(stream)), "minw_bf16_matrix")
+
+
+def minw_sgd_clip(w, g, lr, stream=None):
+    _check(lib().minw_sgd_clip(_ptr(w), _ptr(g), w.numel(), float(lr), _stream(stream)), "minw_sgd_clip")
+
+
+def minw_fc_train_workspace_bytes(B, K, O):
+    return int(lib().minw_fc_train_workspace_bytes(B, K, O))
+
+
+def minw_fc_train_step(A, W, g_out, alpha, lr, q_w, q_a, a_out, g_in, workspace, stream=None):
+    """One Algorithm 1 step of a fully connected layer (W updated in place)."""
+    B, K = A.shape
+    O = W.shape[0]
+    nbytes = workspace.numel() * workspace.element_size()
+    _check(lib().minw_fc_train_step(_ptr(A), _ptr(W), _ptr(g_out), B, K, O, float(alpha), float(lr),
+                                    ctypes.byref(q_w), ctypes.byref(q_a) if q_a is not None else None,
+                                    _ptr(a_out), _ptr(g_in), _ptr(workspace), nbytes, _stream(stream)),
+           "minw_fc_train_step")
 
 
 def aqe_backward(x, gy, gx, alpha, stream=None):

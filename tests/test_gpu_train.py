@@ -1,0 +1,173 @@
+"""GPU parity of Algorithm 1's training step on a fully connected layer,
+through the C ABI.  Stage by stage, each GPU stage is checked against the
+oracle fed with the GPU's own inputs to that stage: the weight AQE forward
+and the activation AQE, the backward masks and the update bit for bit (one
+fp32 operation each), the bf16 operands bit for bit, and the three tensor-core
+products (forward, input gradient, weight gradient) within the bound of fp32
+accumulation, |err| <= K 2^-23 (|P| |Q|) for a product P Q with K terms.  Then
+minw_fc_train_step against the same stages run one by one, bit for bit."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from oracle import oracle as O  # noqa: E402
+from paper_2003_04296_gb300.inputs import DEFAULT_THR  # noqa: E402
+from tests._gpu import dev_tensor  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dev():
+    import __graft_entry__ as g
+    g.build()
+    assert torch.cuda.is_available()
+    return torch.device("cuda:0")
+
+
+@pytest.fixture(scope="module")
+def M(dev):
+    from paper_2003_04296_gb300 import minw
+    return minw
+
+
+def _bf16(t):
+    u = t.cpu().numpy().view(np.uint16).astype(np.uint32) << 16
+    return u.view(np.float32)
+
+
+def _check_product(got, P, Q):
+    """got ~ P @ Q (fp64 reference), within K 2^-23 (|P| @ |Q|)."""
+    ref = P.astype(np.float64) @ Q.astype(np.float64)
+    bound = P.shape[1] * 2.0 ** -23 * (np.abs(P).astype(np.float64) @ np.abs(Q).astype(np.float64)) + 1e-30
+    err = np.abs(got.astype(np.float64) - ref)
+    assert (err <= bound).all(), f"worst err/bound {np.max(err / bound)}"
+
+
+def _problem(seed, B, K, O_):
+    r = np.random.default_rng(seed)
+    A = np.clip(r.standard_normal((B, K)), -1.5, 1.5).astype(np.float32)
+    W = r.uniform(-1, 1, (O_, K)).astype(np.float32)
+    G = (r.standard_normal((B, O_)) * 0.1).astype(np.float32)
+    return A, W, G
+
+
+CASES = [(64, 128, 96, 0.75, 1, 1), (128, 256, 10, 0.3, 3, 2), (256, 1024, 512, 0.6, 2, 1)]
+
+
+@pytest.mark.parametrize("case", CASES)
+def test_train_stages(dev, M, case):
+    B, K, O_, alpha, bw, ba = case
+    A, W, G = _problem(sum(case[:3]), B, K, O_)
+    Op = (O_ + 63) // 64 * 64
+    qw, qa = M.quant(bw, DEFAULT_THR[bw]), M.quant(ba, DEFAULT_THR[ba])
+    At, Wt, Gt = dev_tensor(A, dev), dev_tensor(W, dev), dev_tensor(G, dev)
+    i16 = dict(dtype=torch.int16, device=dev)
+    # forward: W^ (Eq. weight), the bf16 operands, a~, a_out (Eq. activation)
+    what = torch.empty_like(Wt)
+    M.aqe_forward(Wt, what, alpha, qw)
+    what_np = what.cpu().numpy()
+    assert np.array_equal(what_np, O.aqe_forward_f32(W, alpha, bw, DEFAULT_THR[bw]))
+    wb, wtb = torch.empty((O_, K), **i16), torch.empty((K, Op), **i16)
+    ab, atb = torch.empty((B, K), **i16), torch.empty((K, B), **i16)
+    M.minw_bf16_matrix(what, wb)
+    M.minw_bf16_matrix(what, wtb, transpose=True)
+    M.minw_bf16_matrix(At, ab)
+    M.minw_bf16_matrix(At, atb, transpose=True)
+    Wq, Aq = O.bf16_round(what_np), O.bf16_round(A)
+    assert np.array_equal(_bf16(wb), Wq) and np.array_equal(_bf16(ab), Aq)
+    assert np.array_equal(_bf16(wtb)[:, :O_], Wq.T) and not _bf16(wtb)[:, O_:].any()
+    assert np.array_equal(_bf16(atb), Aq.T)
+    ones, zeros = torch.ones(max(K, O_), device=dev), torch.zeros(max(K, O_), device=dev)
+    at = torch.empty((B, O_), dtype=torch.float32, device=dev)
+    M.minw_conv2d_bf16(ab, B, K, 1, 1, wb, O_, 1, 1, bw, 1, 0, 0, ones, zeros, at)
+    at_np = at.cpu().numpy()
+    _check_product(at_np, Aq, Wq.T)
+    a_out = torch.empty_like(at)
+    M.aqe_forward(at, a_out, alpha, qa)
+    assert np.array_equal(a_out.cpu().numpy(), O.aqe_forward_f32(at_np, alpha, ba, DEFAULT_THR[ba]))
+    # backward: the mask of Eq. activation, g_in = g~ W^, g_W^ = g~^T A, Eq. weight's mask, the update
+    gat = torch.empty_like(at)
+    M.aqe_backward(at, Gt, gat, alpha)
+    gat_np = gat.cpu().numpy()
+    assert np.array_equal(gat_np, O.aqe_backward_f32(at_np, G, alpha))
+    gb, gtb = torch.empty((B, Op), **i16), torch.empty((O_, B), **i16)
+    M.minw_bf16_matrix(gat, gb)
+    M.minw_bf16_matrix(gat, gtb, transpose=True)
+    Gq = O.bf16_round(gat_np)
+    assert np.array_equal(_bf16(gb)[:, :O_], Gq) and np.array_equal(_bf16(gtb), Gq.T)
+    g_in = torch.empty((B, K), dtype=torch.float32, device=dev)
+    M.minw_conv2d_bf16(gb, B, Op, 1, 1, wtb, K, 1, 1, bw, 1, 0, 0, ones, zeros, g_in)
+    _check_product(g_in.cpu().numpy(), Gq, Wq)
+    gwhat = torch.empty((O_, K), dtype=torch.float32, device=dev)
+    M.minw_conv2d_bf16(gtb, O_, B, 1, 1, atb, K, 1, 1, bw, 1, 0, 0, ones, zeros, gwhat)
+    gwhat_np = gwhat.cpu().numpy()
+    _check_product(gwhat_np, Gq.T, Aq)
+    gw = torch.empty_like(Wt)
+    M.aqe_backward(Wt, gwhat, gw, alpha)
+    gw_np = gw.cpu().numpy()
+    assert np.array_equal(gw_np, O.aqe_backward_f32(W, gwhat_np, alpha))
+    Wn = Wt.clone()
+    M.minw_sgd_clip(Wn, gw, 0.05)
+    assert np.array_equal(Wn.cpu().numpy(), O.sgd_clip(W, gw_np, 0.05))
+
+
+@pytest.mark.parametrize("case", CASES)
+@pytest.mark.parametrize("last", [False, True])
+def test_train_step_matches_stages(dev, M, case, last):
+    """minw_fc_train_step runs the same kernels in the same order as the stages
+    above (the last layer: a_out = a~ and g~ = g_out): its a_out, g_in and
+    updated W equal theirs bit for bit."""
+    B, K, O_, alpha, bw, ba = case
+    A, W, G = _problem(7 + sum(case[:3]), B, K, O_)
+    qw, qa = M.quant(bw, DEFAULT_THR[bw]), (None if last else M.quant(ba, DEFAULT_THR[ba]))
+    At, Gt = dev_tensor(A, dev), dev_tensor(G, dev)
+    W1 = dev_tensor(W, dev)
+    a1 = torch.empty((B, O_), device=dev)
+    g1 = torch.empty((B, K), device=dev)
+    ws = torch.empty(M.minw_fc_train_workspace_bytes(B, K, O_), dtype=torch.uint8, device=dev)
+    M.minw_fc_train_step(At, W1, Gt, alpha, 0.05, qw, qa, a1, g1, ws)
+    # the same step by its stages
+    Op = (O_ + 63) // 64 * 64
+    i16 = dict(dtype=torch.int16, device=dev)
+    W2 = dev_tensor(W, dev)
+    what = torch.empty_like(W2)
+    M.aqe_forward(W2, what, alpha, qw)
+    wb, wtb = torch.empty((O_, K), **i16), torch.empty((K, Op), **i16)
+    ab, atb = torch.empty((B, K), **i16), torch.empty((K, B), **i16)
+    M.minw_bf16_matrix(what, wb)
+    M.minw_bf16_matrix(what, wtb, transpose=True)
+    M.minw_bf16_matrix(At, ab)
+    M.minw_bf16_matrix(At, atb, transpose=True)
+    ones, zeros = torch.ones(max(K, O_), device=dev), torch.zeros(max(K, O_), device=dev)
+    at = torch.empty((B, O_), device=dev)
+    M.minw_conv2d_bf16(ab, B, K, 1, 1, wb, O_, 1, 1, bw, 1, 0, 0, ones, zeros, at)
+    if last:
+        a2, gat = at, Gt
+    else:
+        a2, gat = torch.empty_like(at), torch.empty_like(at)
+        M.aqe_forward(at, a2, alpha, qa)
+        M.aqe_backward(at, Gt, gat, alpha)
+    gb, gtb = torch.empty((B, Op), **i16), torch.empty((O_, B), **i16)
+    M.minw_bf16_matrix(gat, gb)
+    M.minw_bf16_matrix(gat, gtb, transpose=True)
+    g2 = torch.empty((B, K), device=dev)
+    M.minw_conv2d_bf16(gb, B, Op, 1, 1, wtb, K, 1, 1, bw, 1, 0, 0, ones, zeros, g2)
+    gwhat = torch.empty((O_, K), device=dev)
+    M.minw_conv2d_bf16(gtb, O_, B, 1, 1, atb, K, 1, 1, bw, 1, 0, 0, ones, zeros, gwhat)
+    gw = torch.empty_like(W2)
+    M.aqe_backward(W2, gwhat, gw, alpha)
+    M.minw_sgd_clip(W2, gw, 0.05)
+    torch.cuda.synchronize()
+    assert torch.equal(a1, a2) and torch.equal(g1, g2) and torch.equal(W1, W2)
+    assert W1.abs().max().item() <= 1.0
+
+
+def test_train_step_errors(dev, M):
+    A = torch.zeros((64, 100), device=dev)
+    W = torch.zeros((8, 100), device=dev)
+    G = torch.zeros((64, 8), device=dev)
+    ws = torch.empty(1 << 20, dtype=torch.uint8, device=dev)
+    with pytest.raises(M.MinwError):       # K % 64 != 0
+        M.minw_fc_train_step(A, W, G, 0.5, 0.1, M.quant(1), None, torch.empty((64, 8), device=dev), None, ws)
