@@ -289,12 +289,17 @@ MINW_API size_t minw_fc_train_workspace_bytes(int32_t B, int32_t K, int32_t O);
  *   g_in = bf16(g_a~) bf16(W^)                      ([B][K], skipped when g_in is null)
  *   g_W^ = bf16(g_a~)^T bf16(A)                     ([O][K])
  *   W = min(1, max(-1, W - lr 2 alpha g_W^ 1[|W| <= 1]))   (Eq. weight, update and clip)
+ * a_pre (nullable, [B][O]) receives a~ when q_a is set (ignored without q_a,
+ * where a_out is a~ itself).
+ * A product with few output tiles and a long reduction adds its fp32 sums in K
+ * slices, slice by slice in a fixed order (deterministic, same bound).
  * Requirements: K % 64 == 0 and B % 64 == 0 (else MINW_EUNSUPPORTED), alpha in
- * [0, 1], 16-byte aligned pointers, workspace of minw_fc_train_workspace_bytes. */
+ * [0, 1], 16-byte aligned pointers, workspace of minw_fc_train_workspace_bytes
+ * (scratch: nothing in it survives the call). */
 MINW_API minw_status minw_fc_train_step(const float *A, float *W, const float *g_out, int32_t B, int32_t K,
                                         int32_t O, float alpha, float lr, const minw_quant *q_w,
-                                        const minw_quant *q_a, float *a_out, float *g_in, void *workspace,
-                                        size_t workspace_bytes, void *stream);
+                                        const minw_quant *q_a, float *a_out, float *g_in, float *a_pre,
+                                        void *workspace, size_t workspace_bytes, void *stream);
 
 /* Extra inputs and outputs of a residual block (ResNet-style MINW-Net,
  * where the paper leaves the block wiring open).  Host struct.

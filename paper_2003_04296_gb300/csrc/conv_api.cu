@@ -98,11 +98,12 @@ minw_status minw_conv_block(const uint32_t *act, int32_t B, int32_t C, int32_t H
 }
 
 static minw_status make_codes_args(ConvArgs &a, const uint8_t *act, int B, int C, int H, int W, int bits_a,
-                                   const uint8_t *wgt, int O, int kh, int kw, int bits_w, int stride, int pad) {
+                                   const uint8_t *wgt, int O, int kh, int kw, int bits_w, int stride, int pad,
+                                   bool check_ptrs = true) {
     if (B <= 0 || C <= 0 || H <= 0 || W <= 0 || O <= 0 || kh <= 0 || kw <= 0 || stride <= 0 || pad < 0)
         return MINW_EINVAL;
     if (bits_a < 1 || bits_a > 3 || bits_w < 1 || bits_w > 3) return MINW_EINVAL;
-    if (!act || !wgt || !aligned16(act) || !aligned16(wgt)) return MINW_EINVAL;
+    if (check_ptrs && (!act || !wgt || !aligned16(act) || !aligned16(wgt))) return MINW_EINVAL;
     if (C % 64 != 0 || (stride != 1 && stride != 2) || pad >= kh || pad >= kw) return MINW_EUNSUPPORTED;
     const int Ho = (H + 2 * pad - kh) / stride + 1;
     const int Wo = (W + 2 * pad - kw) / stride + 1;
@@ -116,6 +117,43 @@ static minw_status make_codes_args(ConvArgs &a, const uint8_t *act, int B, int C
     a.M = (long long)B * Ho * Wo;
     return MINW_OK;
 }
+
+}  // extern "C"
+
+namespace minw {
+
+minw_status conv2d_bf16(const uint16_t *act, int B, int C, int H, int W, const uint16_t *wgt, int O, int kh, int kw,
+                        int bits_w, int stride, int pad, int pool, const float *scale, const float *shift,
+                        float *y_out, void *workspace, size_t workspace_bytes, size_t *workspace_need,
+                        cudaStream_t s) {
+    ConvArgs a;
+    const bool query = workspace_need != nullptr;      // shape only: no pointer is used
+    minw_status st = make_codes_args(a, reinterpret_cast<const uint8_t *>(act), B, C, H, W, 1,
+                                     reinterpret_cast<const uint8_t *>(wgt), O, kh, kw, bits_w, stride, pad, !query);
+    if (st != MINW_OK) return st;
+    if (!query && (!scale || !shift || !y_out)) return MINW_EINVAL;
+    if (pool != 0 && pool != 1) return MINW_EINVAL;
+    if (pool && ((a.Ho & 1) || (a.Wo & 1))) return MINW_EUNSUPPORTED;
+    if ((long long)B * H * W * C >= (1ll << 39)) return MINW_EUNSUPPORTED;
+    a.bf16 = 1;
+    a.bits_a = 0;
+    a.scale = scale;
+    a.shift = shift;
+    a.pool = pool;
+    a.y_out = y_out;
+    if (query) {
+        *workspace_need = conv_tc_workspace_bytes(a);
+        return MINW_OK;
+    }
+    if (workspace != nullptr && !aligned16(workspace)) return MINW_EINVAL;
+    a.workspace = workspace;
+    a.workspace_bytes = workspace_bytes;
+    return launch_conv_tc(a, s);
+}
+
+}  // namespace minw
+
+extern "C" {
 
 minw_status minw_conv2d_codes(const uint8_t *act, int32_t B, int32_t C, int32_t H, int32_t W, int32_t bits_a,
                               const uint8_t *wgt, int32_t O, int32_t kh, int32_t kw, int32_t bits_w,
@@ -136,21 +174,8 @@ minw_status minw_conv2d_codes(const uint8_t *act, int32_t B, int32_t C, int32_t 
 minw_status minw_conv2d_bf16(const uint16_t *act, int32_t B, int32_t C, int32_t H, int32_t W, const uint16_t *wgt,
                              int32_t O, int32_t kh, int32_t kw, int32_t bits_w, int32_t stride, int32_t pad,
                              int32_t pool, const float *scale, const float *shift, float *y_out, void *stream) {
-    ConvArgs a;
-    minw_status st = make_codes_args(a, reinterpret_cast<const uint8_t *>(act), B, C, H, W, 1,
-                                     reinterpret_cast<const uint8_t *>(wgt), O, kh, kw, bits_w, stride, pad);
-    if (st != MINW_OK) return st;
-    if (!scale || !shift || !y_out) return MINW_EINVAL;
-    if (pool != 0 && pool != 1) return MINW_EINVAL;
-    if (pool && ((a.Ho & 1) || (a.Wo & 1))) return MINW_EUNSUPPORTED;
-    if ((long long)B * H * W * C >= (1ll << 39)) return MINW_EUNSUPPORTED;
-    a.bf16 = 1;
-    a.bits_a = 0;
-    a.scale = scale;
-    a.shift = shift;
-    a.pool = pool;
-    a.y_out = y_out;
-    return launch_conv_tc(a, (cudaStream_t)stream);
+    return minw::conv2d_bf16(act, B, C, H, W, wgt, O, kh, kw, bits_w, stride, pad, pool, scale, shift, y_out,
+                             nullptr, 0, nullptr, (cudaStream_t)stream);
 }
 
 minw_status minw_conv_block_codes(const uint8_t *act, int32_t B, int32_t C, int32_t H, int32_t W,

@@ -90,6 +90,9 @@ struct Params {
     QParams qo;
     uint32_t *planes_out;
     uint8_t *codes_out;
+    int rowst;                 // row-contiguous stores through a per-warp staging tile: the split-K
+                               // partial sums, and fp32 outputs of 1 x 1 images (fully connected)
+    int ystage;                // 32-bit words of the staging tiles (8 warps x 32 x 16, or 0)
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -502,6 +505,49 @@ __device__ __forceinline__ void resid_chunk(uint32_t taddr, bool full32, const P
 // PAIR: CTA pairs with cta_group::2 MMAs (a kernel uses one CTA group only).
 // BF16: bf16 operands (kind::f16), else E4M3 level codes (kind::f8f6f4); both
 // consume 32 bytes of K per MMA step.
+// Stores the 16 words u[] of each lane's tile row (row = lane) row-contiguously:
+// row rr goes to dst0 + rr * rstride + [0, 16), rows < nrows, columns < ncols.
+// The warp transposes through its 32 x 16-word shared tile in 16-byte chunks,
+// chunk m of row rr at rr * 4 + (m ^ ((rr >> 1) & 3)) (no bank conflict on the
+// writes nor on the reads), so that each 16-byte store instruction covers eight
+// 64-byte row segments.  With scale and shift, the words are fp32 accumulators
+// and column c stores fmaf(u, scale[c], shift[c]): after the transpose a lane
+// holds four fixed columns c = 4 (lane & 3) .. + 3, whose BN values the caller
+// passes in sc[] and sh[].
+__device__ __forceinline__ void rows_store16(uint32_t *sw, const uint32_t (&u)[16], int lane, uint32_t *dst0,
+                                             long long rstride, int nrows, int ncols,
+                                             const float *sc = nullptr, const float *sh = nullptr) {
+    uint4 *sw4 = reinterpret_cast<uint4 *>(sw);
+    __syncwarp();
+#pragma unroll
+    for (int m = 0; m < 4; ++m)
+        sw4[lane * 4 + (m ^ ((lane >> 1) & 3))] = make_uint4(u[4 * m], u[4 * m + 1], u[4 * m + 2], u[4 * m + 3]);
+    __syncwarp();
+    const int k = lane & 3, c = 4 * k;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int rr = 8 * i + (lane >> 2);
+        uint4 x = sw4[rr * 4 + (k ^ ((rr >> 1) & 3))];
+        if (sc != nullptr) {
+            x.x = __float_as_uint(fmaf(__uint_as_float(x.x), sc[0], sh[0]));
+            x.y = __float_as_uint(fmaf(__uint_as_float(x.y), sc[1], sh[1]));
+            x.z = __float_as_uint(fmaf(__uint_as_float(x.z), sc[2], sh[2]));
+            x.w = __float_as_uint(fmaf(__uint_as_float(x.w), sc[3], sh[3]));
+        }
+        if (rr < nrows) {
+            uint32_t *d = dst0 + (long long)rr * rstride + c;
+            if (c + 4 <= ncols && (reinterpret_cast<uintptr_t>(d) & 15) == 0) {
+                *reinterpret_cast<uint4 *>(d) = x;
+            } else {
+                if (c < ncols) d[0] = x.x;
+                if (c + 1 < ncols) d[1] = x.y;
+                if (c + 2 < ncols) d[2] = x.z;
+                if (c + 3 < ncols) d[3] = x.w;
+            }
+        }
+    }
+}
+
 template <int OUTB, bool PAIR, bool BF16>
 __global__ void __launch_bounds__(NT, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -520,7 +566,10 @@ __global__ void __launch_bounds__(NT, 1)
     const int sig_words = OUTB ? O32 / 32 : 0;
     // breakpoints of the output quantizer on y itself (residual blocks), held as -T
     float *syt = reinterpret_cast<float *>(ssig + ((sig_words + 1) & ~1));
-    uint64_t *full = reinterpret_cast<uint64_t *>(syt + (OUTB ? 8 : 0));
+    // staging tiles of the row-contiguous stores, one 32 x 16-word tile per epilogue warp
+    uint32_t *sy = reinterpret_cast<uint32_t *>(syt + (OUTB ? 8 : 0));
+    sy += (4u - ((smem_u32(sy) >> 2) & 3u)) & 3u;            // 16-byte aligned
+    uint64_t *full = reinterpret_cast<uint64_t *>(sy + p.ystage);
     uint64_t *empty = full + p.S;
     uint64_t *tfull = empty + p.S;            // [2] accumulator ready
     uint64_t *tempty = tfull + 2;             // [2] accumulator drained
@@ -1065,6 +1114,18 @@ __global__ void __launch_bounds__(NT, 1)
                 }
             };
 
+            // fully connected fp32 output: this warp's BN values, four columns a lane,
+            // loaded before the accumulator is ready (the loads overlap the MMAs)
+            float bsc[4] = {1.0f, 1.0f, 1.0f, 1.0f}, bsh[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            if (p.ksplit == 1 && p.rowst) {
+                const int oc = o0 + gbeg * 16 + 4 * lane;
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (4 * lane + e < (gend - gbeg) * 16 && oc + e < p.O) {
+                        bsc[e] = __ldg(p.scale + oc + e);
+                        bsh[e] = __ldg(p.shift + oc + e);
+                    }
+            }
             if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
             fence_after();
             int32_t *prow = p.part + (((size_t)kp * tiles + t) * 128 + r) * p.BN;
@@ -1086,15 +1147,46 @@ __global__ void __launch_bounds__(NT, 1)
                 float a[16];
 #pragma unroll
                 for (int j = 0; j < 16; ++j) a[j] = __uint_as_float(sub ? v32[16 + j] : v32[j]);
-                if (p.ksplit == 1) {
+                uint32_t *sw = sy + (warp - 2) * (32 * 16);
+                if (p.ksplit == 1 && p.rowst) {
+                    // fully connected output y[b][o]: rows b0 + rr of this warp, row-contiguous
+                    const int ob = o0 + ch * 16;
+                    uint32_t u[16];
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) u[j] = __float_as_uint(a[j]);
+                    // the BN values of columns 4 (lane & 3) .. + 3 of this group
+                    const int src = (ch - gbeg) * 4 + (lane & 3);
+                    float sc[4], sh[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        sc[e] = __shfl_sync(0xffffffffu, bsc[e], src);
+                        sh[e] = __shfl_sync(0xffffffffu, bsh[e], src);
+                    }
+                    const int b0 = b - lane;
+                    rows_store16(sw, u, lane, reinterpret_cast<uint32_t *>(p.y_out) + (long long)b0 * p.O + ob, p.O,
+                                 p.B - b0, p.O - ob, sc, sh);
+                } else if (p.ksplit == 1) {
                     finish(a, ch);
+                } else if (p.rowst) {
+                    // partial sums of this K slice (exact integers, or fp32 sums of bf16 products),
+                    // summed by splitk_reduce_kernel
+                    uint32_t u[16];
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) u[j] = BF16 ? __float_as_uint(a[j]) : (uint32_t)__float2int_rn(a[j]);
+                    rows_store16(sw, u, lane,
+                                 reinterpret_cast<uint32_t *>(p.part) + (((size_t)kp * tiles + t) * 128 + q * 32) * p.BN +
+                                     ch * 16,
+                                 p.BN, 32, 16);
                 } else {
-                    // exact integer partial sums of this K slice (summed by splitk_reduce_kernel)
                     int4 *dst = reinterpret_cast<int4 *>(prow + ch * 16);
 #pragma unroll
-                    for (int j = 0; j < 4; ++j)
-                        dst[j] = make_int4(__float2int_rn(a[4 * j]), __float2int_rn(a[4 * j + 1]),
-                                           __float2int_rn(a[4 * j + 2]), __float2int_rn(a[4 * j + 3]));
+                    for (int j = 0; j < 4; ++j) {
+                        int v[4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e)
+                            v[e] = BF16 ? __float_as_int(a[4 * j + e]) : __float2int_rn(a[4 * j + e]);
+                        dst[j] = make_int4(v[0], v[1], v[2], v[3]);
+                    }
                 }
             }
             fence_before();
@@ -1150,12 +1242,45 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const Params p, cons
     const bool inside = b < p.B && y < p.Ho && x < p.Wo;
     const bool valid = live && inside;
     int acc[4] = {0, 0, 0, 0};
+    float accf[4] = {0.0f, 0.0f, 0.0f, 0.0f};      // the accumulators as fp32
     if (valid) {
         const size_t slice4 = (size_t)tiles * 128 * p.BN / 4;
         const int4 *src = reinterpret_cast<const int4 *>(p.part + ((size_t)t * 128 + r) * p.BN + col);
-        for (int kp = 0; kp < p.ksplit; ++kp) {
-            const int4 v = __ldcs(src + kp * slice4);
-            acc[0] += v.x; acc[1] += v.y; acc[2] += v.z; acc[3] += v.w;
+        // four slices' loads in flight before their adds (the adds keep slice order)
+        if (p.esize == 2) {
+            // fp32 partial sums of bf16 products, added in slice order
+            const float4 *src4 = reinterpret_cast<const float4 *>(src);
+            int kp = 0;
+            for (; kp + 4 <= p.ksplit; kp += 4) {
+                float4 v[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) v[e] = __ldcs(src4 + (kp + e) * slice4);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    accf[0] += v[e].x; accf[1] += v[e].y; accf[2] += v[e].z; accf[3] += v[e].w;
+                }
+            }
+            for (; kp < p.ksplit; ++kp) {
+                const float4 v = __ldcs(src4 + kp * slice4);
+                accf[0] += v.x; accf[1] += v.y; accf[2] += v.z; accf[3] += v.w;
+            }
+        } else {
+            int kp = 0;
+            for (; kp + 4 <= p.ksplit; kp += 4) {
+                int4 v[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) v[e] = __ldcs(src + (kp + e) * slice4);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    acc[0] += v[e].x; acc[1] += v[e].y; acc[2] += v[e].z; acc[3] += v[e].w;
+                }
+            }
+            for (; kp < p.ksplit; ++kp) {
+                const int4 v = __ldcs(src + kp * slice4);
+                acc[0] += v.x; acc[1] += v.y; acc[2] += v.z; acc[3] += v.w;
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) accf[j] = (float)acc[j];
         }
     }
     const long long HoWo = (long long)p.Ho * p.Wo;
@@ -1170,19 +1295,27 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const Params p, cons
     if (valid && resid)
         for (int j = 0; j < 4; ++j)
             if (o + j < p.O) {
-                float yv = fmaf((float)acc[j], __ldg(p.scale + o + j), __ldg(p.shift + o + j));
+                float yv = fmaf(accf[j], __ldg(p.scale + o + j), __ldg(p.shift + o + j));
                 if (p.y_nhwc != nullptr) p.y_nhwc[pix * p.O + o + j] = yv;
                 if (p.res_codes != nullptr) yv += code_units(__ldg(p.res_codes + pix * p.O + o + j)) * p.res_unit;
                 else if (p.res_f32 != nullptr) yv += __ldg(p.res_f32 + pix * p.O + o + j);
                 yres[j] = yv;
             }
-    if (valid && p.y_out != nullptr)
-        for (int j = 0; j < 4; ++j)
-            if (o + j < p.O) {
-                float yv = resid ? yres[j] : fmaf((float)acc[j], __ldg(p.scale + o + j), __ldg(p.shift + o + j));
-                if (OUTB > 0) yv = fminf(fmaxf(yv, -1.0f), 1.0f);
-                p.y_out[((long long)b * p.O + o + j) * HoWo + (long long)y * p.Wo + x] = yv;
-            }
+    if (valid && p.y_out != nullptr) {
+        float yv4[4];
+        for (int j = 0; j < 4; ++j) {
+            const int oj = min(o + j, p.O - 1);
+            yv4[j] = resid ? yres[j] : fmaf(accf[j], __ldg(p.scale + oj), __ldg(p.shift + oj));
+            if (OUTB > 0) yv4[j] = fminf(fmaxf(yv4[j], -1.0f), 1.0f);
+        }
+        if (HoWo == 1 && o + 4 <= p.O && ((reinterpret_cast<uintptr_t>(p.y_out + (long long)b * p.O + o) & 15) == 0)) {
+            // fully connected output: four consecutive channels of one row
+            *reinterpret_cast<float4 *>(p.y_out + (long long)b * p.O + o) = make_float4(yv4[0], yv4[1], yv4[2], yv4[3]);
+        } else {
+            for (int j = 0; j < 4; ++j)
+                if (o + j < p.O) p.y_out[((long long)b * p.O + o + j) * HoWo + (long long)y * p.Wo + x] = yv4[j];
+        }
+    }
     if constexpr (OUTB > 0) {
         uint32_t code = 0u, bits[3] = {0u, 0u, 0u};
 #pragma unroll
@@ -1193,7 +1326,7 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const Params p, cons
                     k = level_index_of_y(yres[j], p.qo);
                 } else {
                     const float *th = thr + (o + j) * NL;
-                    const float v = (float)acc[j] * __ldg(th + NL - 1);
+                    const float v = accf[j] * __ldg(th + NL - 1);
 #pragma unroll
                     for (int u = 0; u < NL - 1; ++u) k += (v >= __ldg(th + u)) ? 1 : 0;
                 }
@@ -1274,6 +1407,9 @@ static int auto_ksplit(int tiles, int nk, int sms) {
     if (ks > nk / 4) ks = nk / 4;
     return ks < 2 ? 1 : ks;
 }
+// channels of one K chunk: 128-byte rows of E4M3 codes (64-byte rows when C is
+// not a multiple of 128), or 64 bf16 values
+static int chunk_channels(const ConvArgs &a) { return a.bf16 ? 64 : ((a.C % 128 == 0) ? 128 : 64); }
 static size_t slice_bytes(int tiles, int BN) { return (size_t)tiles * 128 * BN * sizeof(int32_t); }
 static size_t thr_ws_bytes(int O, int nlev) { return (((size_t)O * nlev * sizeof(float)) + 255) & ~(size_t)255; }
 
@@ -1409,7 +1545,14 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     p.b_bytes = (uint32_t)((p.pair ? p.BN / 2 : p.BN) * p.cb);   // pairs: each CTA holds half the weight rows
     const size_t o32 = ((size_t)a.O + 31) & ~(size_t)31;
     const size_t thr_bytes = a.quant_out ? (o32 * p.nlev + o32 / 32 + 10) * sizeof(float) : 0;
-    const size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes;
+    // staging tiles of the row-contiguous stores: a layer that may split along K,
+    // or whose fp32 output is a fully connected one (1 x 1 images)
+    const bool resid_ = a.res_codes != nullptr || a.res_f32 != nullptr || a.y_nhwc != nullptr;
+    const bool rowst_fc = !p.trans && a.y_out != nullptr && a.Ho == 1 && a.Wo == 1 && !a.pool && !a.quant_out &&
+                          a.acc_out == nullptr && !resid_;
+    const bool may_split = a.workspace != nullptr && !a.pool && !p.trans && !p.pair;
+    p.ystage = (rowst_fc || may_split) ? 8 * 32 * 16 : 0;
+    const size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes - (p.ystage ? (size_t)p.ystage * 4 + 16 : 0);
     // two K blocks per stage (one commit per 8 or 4 MMAs) when three such stages fit
     const size_t blk = (size_t)p.a_bytes + p.b_bytes;
     p.kps = (kps_pref() != 1 && p.nk >= 2 && budget / (2 * blk) >= 3) ? 2 : 1;
@@ -1438,7 +1581,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
     p.ksplit = 1;
     pl.thr_ws = nullptr;
-    if (a.workspace != nullptr && !a.pool && !p.trans && !p.pair && !a.bf16) {
+    if (a.workspace != nullptr && !a.pool && !p.trans && !p.pair) {
         // workspace: [breakpoints, when not given][ksplit partial-sum slices]
         const size_t tb = (a.quant_out && a.thr == nullptr) ? thr_ws_bytes(a.O, p.nlev) : 0;
         const size_t sb = slice_bytes(tiles, p.BN);
@@ -1460,6 +1603,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     // clusters sharing each weight box (multicast): cl CTAs walk pixel tiles
     // of one channel tile together; each loads BN / cl weight rows for all
     // (padding the pixel tiles to a multiple of cl may add at most 1/8)
+    p.rowst = (p.ystage > 0 && (p.ksplit > 1 || rowst_fc)) ? 1 : 0;
     const int tiles_m = p.nbx * p.nby * p.nbb;
     p.cl = p.pair ? 2 : 1;
     if (p.ksplit == 1 && !p.trans && !p.pair) {
@@ -1500,7 +1644,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     int grid = items < sms ? items : sms;
     grid -= grid % p.cl;
     pl.grid = dim3((unsigned)grid);
-    pl.smem = (size_t)p.S * p.stage_bytes + 1024 + 256 + thr_bytes;
+    pl.smem = (size_t)p.S * p.stage_bytes + 1024 + 256 + thr_bytes + (p.ystage ? (size_t)p.ystage * 4 + 16 : 0);
     // more than half of an SM's shared memory: exactly one CTA (and one TMEM
     // allocation) per SM
     if (pl.smem < 120 * 1024) pl.smem = 120 * 1024;
@@ -1533,7 +1677,7 @@ size_t conv_tc_workspace_bytes(const ConvArgs &a) {
     if (a.pool || !tc::plan_shape(a, p)) return 0;
     const int nbb = (a.B + p.bb - 1) / p.bb;
     const int tiles = p.nbx * p.nby * nbb * ((a.O + p.BN - 1) / p.BN);
-    const int nk = a.kh * a.kw * (a.C / ((a.C % 128 == 0) ? 128 : 64));
+    const int nk = a.kh * a.kw * (a.C / tc::chunk_channels(a));
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
     const int ks = tc::auto_ksplit(tiles, nk, sms);
     if (ks < 2) return 0;
@@ -1545,7 +1689,7 @@ size_t conv_tc_min_split_bytes(const ConvArgs &a) {
     if (a.pool || !tc::plan_shape(a, p)) return 0;
     const int nbb = (a.B + p.bb - 1) / p.bb;
     const int tiles = p.nbx * p.nby * nbb * ((a.O + p.BN - 1) / p.BN);
-    const int nk = a.kh * a.kw * (a.C / ((a.C % 128 == 0) ? 128 : 64));
+    const int nk = a.kh * a.kw * (a.C / tc::chunk_channels(a));
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
     if (tc::auto_ksplit(tiles, nk, sms) < 2) return 0;
     return tc::thr_ws_bytes(a.O, 7) + 2 * tc::slice_bytes(tiles, p.BN);

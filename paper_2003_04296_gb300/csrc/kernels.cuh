@@ -74,6 +74,12 @@ minw_status make_conv_args(ConvArgs &a, const uint32_t *act, int B, int C, int H
 int choose_variant(const ConvArgs &a, int requested);
 minw_status run_conv(const ConvArgs &a, int variant, cudaStream_t s);
 minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s);
+// bf16 convolution (minw_conv2d_bf16) with an optional split-K workspace;
+// with workspace_need set, only stores the workspace bytes the shape can use.
+minw_status conv2d_bf16(const uint16_t *act, int B, int C, int H, int W, const uint16_t *wgt, int O, int kh, int kw,
+                        int bits_w, int stride, int pad, int pool, const float *scale, const float *shift,
+                        float *y_out, void *workspace, size_t workspace_bytes, size_t *workspace_need,
+                        cudaStream_t s);
 bool conv_tc_supported(const ConvArgs &a);
 // Workspace the tensor-core path needs to split K for this shape (0: it does not split).
 size_t conv_tc_workspace_bytes(const ConvArgs &a);

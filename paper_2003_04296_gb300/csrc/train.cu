@@ -5,13 +5,14 @@
 // of Eq. activation, the input gradient g_a = g_a~ W^q, the weight gradient
 // g_W^q = g_a~^T a^q, the mask of Eq. weight, and the update with the clip to
 // [-1, 1].  The three products run on the tensor cores as 1 x 1 convolutions
-// of bf16 operands (conv_tc_kernel, kind::f16); the rest are elementwise
-// kernels here and in aqe.cu.
+// of bf16 operands (conv_tc_kernel, kind::f16); each operand is made in one
+// pass over its fp32 source (AQE, bf16 rounding, the transposed copy), and the
+// mask of Eq. weight is fused with the update.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include "common.cuh"
+#include "kernels.cuh"
 
 namespace minw {
 
@@ -47,11 +48,6 @@ __global__ void sgd_clip_kernel(float *__restrict__ w, const float *__restrict__
         w[i] = fminf(1.0f, fmaxf(-1.0f, fmaf(-lr, g[i], w[i])));
 }
 
-__global__ void fill_kernel(float *__restrict__ p, int64_t n, float v) {
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
-        p[i] = v;
-}
-
 static int64_t grid_of(int64_t n) {
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 152;
     int64_t g = (n + 255) / 256;
@@ -59,31 +55,182 @@ static int64_t grid_of(int64_t n) {
     return g < 1 ? 1 : g;
 }
 
-// Workspace of minw_fc_train_step: regions 256-byte aligned, in this order.
+__device__ __forceinline__ uint32_t bf16x2(float lo, float hi) {
+    return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(lo)) |
+           ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(hi)) << 16);
+}
+
+// The operand preparation of one product pair, in one pass over a row-major
+// fp32 matrix X [R][C]: v = f(X) as bf16 both row-major (vb [R][Cp], columns
+// C..Cp zero) and transposed (vtb [C][Rp], columns R..Rp zero), through a
+// 32 x 64 shared tile.
+//   MODE 0  weights: v = alpha h(W) + (1 - alpha) W (Eq. weight); also fills
+//           ones[0..M) = 1 and zeros[0..M) = 0 (the unit BN of the products)
+//   MODE 1  activations: v = a
+//   MODE 2  output gradients: with a_out, v = 2 alpha g 1[|a~| <= 1] (the
+//           backward of Eq. activation, X = a~, G = g) and a_out = alpha h(a~)
+//           + (1 - alpha) a~; without it (a layer without an activation
+//           quantizer), v = g
+// Every value takes the same fp32 operations as aqe_forward / aqe_backward.
+template <int MODE>
+__global__ void __launch_bounds__(256) prep_kernel(const float *__restrict__ X, const float *__restrict__ G, int R,
+                                                   int C, int Cp, int Rp, float alpha, QParams q,
+                                                   uint16_t *__restrict__ vb, uint16_t *__restrict__ vtb,
+                                                   float *__restrict__ a_out, float *__restrict__ ones,
+                                                   float *__restrict__ zeros, int M) {
+    __shared__ float tile[32][65];
+    const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 64;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;     // columns 4 tx .. 4 tx + 3 of rows ty, ty + 16
+    const float oma = 1.0f - alpha, two_alpha = 2.0f * alpha;
+    const int c = c0 + 4 * tx;
+    const bool vec = (C & 3) == 0 && c < C;                       // four columns inside, 16-byte aligned
+    // all loads first (two rows x four columns of X, and of G)
+    float x[2][4], g[2][4];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int r = r0 + ty + 16 * h;
+        const int64_t at = (int64_t)r * C + c;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) x[h][e] = g[h][e] = 0.0f;
+        if (r >= R) continue;
+        if (vec) {
+            const float4 x4 = *reinterpret_cast<const float4 *>(X + at);
+            x[h][0] = x4.x; x[h][1] = x4.y; x[h][2] = x4.z; x[h][3] = x4.w;
+            if (MODE == 2) {
+                const float4 g4 = *reinterpret_cast<const float4 *>(G + at);
+                g[h][0] = g4.x; g[h][1] = g4.y; g[h][2] = g4.z; g[h][3] = g4.w;
+            }
+        } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                if (c + e < C) {
+                    x[h][e] = X[at + e];
+                    if (MODE == 2) g[h][e] = G[at + e];
+                }
+        }
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int k = ty + 16 * h, r = r0 + k;
+        const int64_t at = (int64_t)r * C + c;
+        float v[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        if (r < R) {
+            float ao[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                if (c + e >= C) continue;
+                if (MODE == 0) {
+                    v[e] = fmaf(alpha, level_value(x[h][e] * q.scale, q), oma * x[h][e]);
+                } else if (MODE == 1) {
+                    v[e] = x[h][e];
+                } else if (a_out != nullptr) {
+                    ao[e] = fmaf(alpha, level_value(x[h][e] * q.scale, q), oma * x[h][e]);
+                    v[e] = (fabsf(x[h][e]) <= 1.0f) ? g[h][e] * two_alpha : 0.0f;
+                } else {
+                    v[e] = g[h][e];
+                }
+            }
+            if (MODE == 2 && a_out != nullptr) {
+                if (vec) {
+                    *reinterpret_cast<float4 *>(a_out + at) = make_float4(ao[0], ao[1], ao[2], ao[3]);
+                } else {
+                    for (int e = 0; e < 4; ++e)
+                        if (c + e < C) a_out[at + e] = ao[e];
+                }
+            }
+            uint16_t *dst = vb + (int64_t)r * Cp + c;
+            if (c + 3 < Cp && (Cp & 3) == 0)
+                *reinterpret_cast<uint2 *>(dst) = make_uint2(bf16x2(v[0], v[1]), bf16x2(v[2], v[3]));
+            else
+                for (int e = 0; e < 4; ++e)
+                    if (c + e < Cp) dst[e] = __bfloat16_as_ushort(__float2bfloat16_rn(v[e]));
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) tile[k][4 * tx + e] = v[e];
+    }
+    if (MODE == 0) {
+        const int64_t nthr = (int64_t)gridDim.x * gridDim.y * blockDim.x;
+        for (int64_t i = ((int64_t)blockIdx.y * gridDim.x + blockIdx.x) * blockDim.x + threadIdx.x; i < M; i += nthr) {
+            ones[i] = 1.0f;
+            zeros[i] = 0.0f;
+        }
+    }
+    __syncthreads();
+    // transposed: row c0 + cc of vtb, its 32 values r0 .. r0 + 31 as four 8-value runs
+    const int cc = threadIdx.x >> 2, part = threadIdx.x & 3;
+    const int ct = c0 + cc, rt = r0 + part * 8;
+    if (ct < C && rt < Rp) {
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) w[e] = bf16x2(tile[part * 8 + 2 * e][cc], tile[part * 8 + 2 * e + 1][cc]);
+        uint16_t *dst = vtb + (int64_t)ct * Rp + rt;
+        if (rt + 8 <= Rp && (Rp & 7) == 0) {
+            *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+        } else {
+            for (int e = 0; e < 8 && rt + e < Rp; ++e) dst[e] = (uint16_t)(w[e >> 1] >> (16 * (e & 1)));
+        }
+    }
+}
+
+// The mask of Eq. weight and the update, fused: w <- clip(w - lr 2 alpha g 1[|w| <= 1])
+// with the fp32 operations of aqe_backward followed by sgd_clip.
+__global__ void __launch_bounds__(256) update_kernel(float *__restrict__ w, const float *__restrict__ g, int64_t n,
+                                                     float two_alpha, float lr) {
+    const int64_t n4 = n >> 2, stride = (int64_t)gridDim.x * blockDim.x;
+    float4 *w4 = reinterpret_cast<float4 *>(w);
+    const float4 *g4 = reinterpret_cast<const float4 *>(g);
+    auto upd = [&](float x, float gx) {
+        const float gw = (fabsf(x) <= 1.0f) ? gx * two_alpha : 0.0f;
+        return fminf(1.0f, fmaxf(-1.0f, fmaf(-lr, gw, x)));
+    };
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
+        float4 x = w4[i];
+        const float4 gx = __ldcs(g4 + i);
+        x.x = upd(x.x, gx.x); x.y = upd(x.y, gx.y); x.z = upd(x.z, gx.z); x.w = upd(x.w, gx.w);
+        w4[i] = x;
+    }
+    for (int64_t i = (n4 << 2) + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride)
+        w[i] = upd(w[i], g[i]);
+}
+
+// Workspace of minw_fc_train_step: regions 256-byte aligned, in this order;
+// split holds the K-sliced partial sums of the products.
 struct TrainLayout {
-    size_t what, wb, wtb, ab, atb, at, gat, gb, gtb, gwhat, gw, ones, zeros, total;
+    size_t wb, wtb, ab, atb, at, gb, gtb, gwhat, ones, zeros, split, split_bytes, total;
 };
 
 static size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 static TrainLayout train_layout(int B, int K, int O) {
-    const size_t Op = (size_t)((O + 63) / 64 * 64), M = (size_t)(K > O ? K : O);
+    const int Op = (O + 63) / 64 * 64;
+    const size_t M = (size_t)(K > O ? K : O);
+    // split-K partial sums: the largest need of the three products
+    size_t need = 0;
+    auto want = [&](int nb, int c, int o) {
+        size_t w = 0;
+        if (conv2d_bf16(nullptr, nb, c, 1, 1, nullptr, o, 1, 1, 1, 1, 0, 0, nullptr, nullptr, nullptr, nullptr, 0, &w,
+                        nullptr) == MINW_OK &&
+            w > need)
+            need = w;
+    };
+    want(B, K, O);        // forward
+    want(B, Op, K);       // input gradient
+    want(O, B, K);        // weight gradient
     TrainLayout L;
     size_t off = 0;
     auto take = [&](size_t bytes) { const size_t r = off; off += al256(bytes); return r; };
-    L.what = take(4 * (size_t)O * K);
     L.wb = take(2 * (size_t)O * K);
     L.wtb = take(2 * (size_t)K * Op);
     L.ab = take(2 * (size_t)B * K);
     L.atb = take(2 * (size_t)K * B);
     L.at = take(4 * (size_t)B * O);
-    L.gat = take(4 * (size_t)B * O);
     L.gb = take(2 * (size_t)B * Op);
     L.gtb = take(2 * (size_t)O * B);
     L.gwhat = take(4 * (size_t)O * K);
-    L.gw = take(4 * (size_t)O * K);
     L.ones = take(4 * M);
     L.zeros = take(4 * M);
+    L.split_bytes = need;
+    L.split = take(need);
     L.total = off;
     return L;
 }
@@ -121,55 +268,55 @@ size_t minw_fc_train_workspace_bytes(int32_t B, int32_t K, int32_t O) {
 
 minw_status minw_fc_train_step(const float *A, float *W, const float *g_out, int32_t B, int32_t K, int32_t O,
                                float alpha, float lr, const minw_quant *q_w, const minw_quant *q_a, float *a_out,
-                               float *g_in, void *workspace, size_t workspace_bytes, void *stream) {
+                               float *g_in, float *a_pre, void *workspace, size_t workspace_bytes, void *stream) {
     if (B <= 0 || K <= 0 || O <= 0 || !A || !W || !g_out || !a_out || !q_w || !workspace) return MINW_EINVAL;
     if (!(alpha >= 0.0f && alpha <= 1.0f)) return MINW_EINVAL;
     if (!valid_quant(q_w) || (q_a && !valid_quant(q_a))) return MINW_EINVAL;
     if (K % 64 != 0 || B % 64 != 0) return MINW_EUNSUPPORTED;
     if (!aligned16(A) || !aligned16(W) || !aligned16(g_out) || !aligned16(a_out) || (g_in && !aligned16(g_in)) ||
+        (a_pre && !aligned16(a_pre)) ||
         !aligned16(workspace))
         return MINW_EINVAL;
     const TrainLayout L = train_layout(B, K, O);
     if (workspace_bytes < L.total) return MINW_EINVAL;
+    if ((int64_t)K * (O + 63) >= (1ll << 31) || (int64_t)B * K >= (1ll << 31)) return MINW_EUNSUPPORTED;
     cudaStream_t s = (cudaStream_t)stream;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
-    float *what = reinterpret_cast<float *>(ws + L.what), *at = reinterpret_cast<float *>(ws + L.at);
-    float *gat = reinterpret_cast<float *>(ws + L.gat), *gwhat = reinterpret_cast<float *>(ws + L.gwhat);
-    float *gw = reinterpret_cast<float *>(ws + L.gw);
+    float *at = a_pre ? a_pre : reinterpret_cast<float *>(ws + L.at), *gwhat = reinterpret_cast<float *>(ws + L.gwhat);
     float *ones = reinterpret_cast<float *>(ws + L.ones), *zeros = reinterpret_cast<float *>(ws + L.zeros);
     uint16_t *wb = reinterpret_cast<uint16_t *>(ws + L.wb), *wtb = reinterpret_cast<uint16_t *>(ws + L.wtb);
     uint16_t *ab = reinterpret_cast<uint16_t *>(ws + L.ab), *atb = reinterpret_cast<uint16_t *>(ws + L.atb);
     uint16_t *gb = reinterpret_cast<uint16_t *>(ws + L.gb), *gtb = reinterpret_cast<uint16_t *>(ws + L.gtb);
+    void *split = L.split_bytes ? ws + L.split : nullptr;
     const int Op = (O + 63) / 64 * 64, M = K > O ? K : O;
+    const QParams qw = to_qparams(q_w), qa = q_a ? to_qparams(q_a) : QParams{};
     minw_status st;
 #define TRY(x) do { if ((st = (x)) != MINW_OK) return st; } while (0)
-    fill_kernel<<<(unsigned)grid_of(M), 256, 0, s>>>(ones, M, 1.0f);
-    fill_kernel<<<(unsigned)grid_of(M), 256, 0, s>>>(zeros, M, 0.0f);
+    // 1.1 forward: W^ = alpha h(W) + (1 - alpha) W as bf16 [O][K] and [K][Op]; a as bf16 [B][K] and [K][B]
+    prep_kernel<0><<<dim3((unsigned)(K / 64), (unsigned)(Op / 32)), 256, 0, s>>>(
+        W, nullptr, O, K, K, Op, alpha, qw, wb, wtb, nullptr, ones, zeros, M);
+    prep_kernel<1><<<dim3((unsigned)(K / 64), (unsigned)(B / 32)), 256, 0, s>>>(
+        A, nullptr, B, K, K, B, 0.0f, qw, ab, atb, nullptr, nullptr, nullptr, 0);
     TRY(launch_status());
-    // 1.1 forward: W^ = alpha h(W) + (1 - alpha) W, a~ = a W^T, a_l = alpha h(a~) + (1 - alpha) a~
-    TRY(aqe_forward(W, what, (int64_t)O * K, alpha, q_w, stream));
-    TRY(minw_bf16_matrix(what, O, K, 0, K, wb, stream));
-    TRY(minw_bf16_matrix(what, O, K, 1, Op, wtb, stream));
-    TRY(minw_bf16_matrix(A, B, K, 0, K, ab, stream));
-    TRY(minw_bf16_matrix(A, B, K, 1, B, atb, stream));
-    float *fwd_out = q_a ? at : a_out;                 // the last layer emits a~ itself
-    TRY(minw_conv2d_bf16(ab, B, K, 1, 1, wb, O, 1, 1, q_w->bits, 1, 0, 0, ones, zeros, fwd_out, stream));
-    const float *g_at = g_out;
-    if (q_a) {
-        TRY(aqe_forward(at, a_out, (int64_t)B * O, alpha, q_a, stream));
-        // 1.2 backward through the activation AQE (Eq. activation): 2 alpha g 1[|a~| <= 1]
-        TRY(aqe_backward(at, g_out, gat, (int64_t)B * O, alpha, stream));
-        g_at = gat;
-    }
-    TRY(minw_bf16_matrix(g_at, B, O, 0, Op, gb, stream));
-    TRY(minw_bf16_matrix(g_at, B, O, 1, B, gtb, stream));
+    // a~ = a W^T  ([B][O], reduction over K); the last layer emits a~ itself
+    float *fwd_out = q_a ? at : a_out;
+    TRY(conv2d_bf16(ab, B, K, 1, 1, wb, O, 1, 1, q_w->bits, 1, 0, 0, ones, zeros, fwd_out, split, L.split_bytes,
+                    nullptr, s));
+    // 1.2 backward through the activation AQE (Eq. activation): g_a~ = 2 alpha g 1[|a~| <= 1], as bf16
+    // [B][Op] and [O][B]; a_l = alpha h(a~) + (1 - alpha) a~
+    prep_kernel<2><<<dim3((unsigned)(Op / 64), (unsigned)(B / 32)), 256, 0, s>>>(
+        q_a ? at : g_out, g_out, B, O, Op, B, alpha, qa, gb, gtb, q_a ? a_out : nullptr, nullptr, nullptr, 0);
+    TRY(launch_status());
     if (g_in)                                          // g_a = g_a~ W^  ([B][K], reduction over O)
-        TRY(minw_conv2d_bf16(gb, B, Op, 1, 1, wtb, K, 1, 1, q_w->bits, 1, 0, 0, ones, zeros, g_in, stream));
+        TRY(conv2d_bf16(gb, B, Op, 1, 1, wtb, K, 1, 1, q_w->bits, 1, 0, 0, ones, zeros, g_in, split, L.split_bytes,
+                        nullptr, s));
     // g_W^ = g_a~^T a  ([O][K], reduction over the batch)
-    TRY(minw_conv2d_bf16(gtb, O, B, 1, 1, atb, K, 1, 1, q_w->bits, 1, 0, 0, ones, zeros, gwhat, stream));
-    // 2. the mask of Eq. weight on the latent weights, then the update and the clip
-    TRY(aqe_backward(W, gwhat, gw, (int64_t)O * K, alpha, stream));
-    TRY(minw_sgd_clip(W, gw, (int64_t)O * K, lr, stream));
+    TRY(conv2d_bf16(gtb, O, B, 1, 1, atb, K, 1, 1, q_w->bits, 1, 0, 0, ones, zeros, gwhat, split, L.split_bytes,
+                    nullptr, s));
+    // 2. the mask of Eq. weight on the latent weights, the update and the clip
+    update_kernel<<<(unsigned)grid_of((int64_t)O * K / 4 + 1), 256, 0, s>>>(W, gwhat, (int64_t)O * K, 2.0f * alpha,
+                                                                            lr);
+    TRY(launch_status());
 #undef TRY
     return MINW_OK;
 }

@@ -72,7 +72,7 @@ SIGNATURES = {
     "minw_bf16_matrix": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _P]),
     "minw_sgd_clip": (ctypes.c_int, [_P, _P, _I64, _F, _P]),
     "minw_fc_train_workspace_bytes": (ctypes.c_size_t, [_I32, _I32, _I32]),
-    "minw_fc_train_step": (ctypes.c_int, [_P, _P, _P, _I32, _I32, _I32, _F, _F, _QP, _QP, _P, _P, _P,
+    "minw_fc_train_step": (ctypes.c_int, [_P, _P, _P, _I32, _I32, _I32, _F, _F, _QP, _QP, _P, _P, _P, _P,
                                           ctypes.c_size_t, _P]),
     "aqe_quantize_pack": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _F, _P, _P, _P]),
     "aqe_backward_masked": (ctypes.c_int, [_P, _P, _P, _I64, _F, _P]),
@@ -234,14 +234,16 @@ def minw_fc_train_workspace_bytes(B, K, O):
     return int(lib().minw_fc_train_workspace_bytes(B, K, O))
 
 
-def minw_fc_train_step(A, W, g_out, alpha, lr, q_w, q_a, a_out, g_in, workspace, stream=None):
-    """One Algorithm 1 step of a fully connected layer (W updated in place)."""
+def minw_fc_train_step(A, W, g_out, alpha, lr, q_w, q_a, a_out, g_in, workspace, a_pre=None, stream=None):
+    """One Algorithm 1 step of a fully connected layer (W updated in place;
+    a_pre, when given, receives the product before the activation AQE)."""
     B, K = A.shape
     O = W.shape[0]
     nbytes = workspace.numel() * workspace.element_size()
     _check(lib().minw_fc_train_step(_ptr(A), _ptr(W), _ptr(g_out), B, K, O, float(alpha), float(lr),
                                     ctypes.byref(q_w), ctypes.byref(q_a) if q_a is not None else None,
-                                    _ptr(a_out), _ptr(g_in), _ptr(workspace), nbytes, _stream(stream)),
+                                    _ptr(a_out), _ptr(g_in), _ptr(a_pre), _ptr(workspace), nbytes,
+                                    _stream(stream)),
            "minw_fc_train_step")
 
 
