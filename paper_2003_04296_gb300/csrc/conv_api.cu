@@ -125,7 +125,7 @@ namespace minw {
 minw_status conv2d_bf16(const uint16_t *act, int B, int C, int H, int W, const uint16_t *wgt, int O, int kh, int kw,
                         int bits_w, int stride, int pad, int pool, const float *scale, const float *shift,
                         float *y_out, void *workspace, size_t workspace_bytes, size_t *workspace_need,
-                        cudaStream_t s) {
+                        cudaStream_t s, int upd, float upd_lr, float upd_2a) {
     ConvArgs a;
     const bool query = workspace_need != nullptr;      // shape only: no pointer is used
     minw_status st = make_codes_args(a, reinterpret_cast<const uint8_t *>(act), B, C, H, W, 1,
@@ -148,6 +148,9 @@ minw_status conv2d_bf16(const uint16_t *act, int B, int C, int H, int W, const u
     if (workspace != nullptr && !aligned16(workspace)) return MINW_EINVAL;
     a.workspace = workspace;
     a.workspace_bytes = workspace_bytes;
+    a.upd = upd;
+    a.upd_lr = upd_lr;
+    a.upd_2a = upd_2a;
     return launch_conv_tc(a, s);
 }
 

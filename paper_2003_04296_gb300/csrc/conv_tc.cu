@@ -93,6 +93,8 @@ struct Params {
     int rowst;                 // row-contiguous stores through a per-warp staging tile: the split-K
                                // partial sums, and fp32 outputs of 1 x 1 images (fully connected)
     int ystage;                // 32-bit words of the staging tiles (8 warps x 32 x 16, or 0)
+    int upd;                   // fully connected output: y_out holds latent weights, updated in place
+    float upd_lr, upd_2a;      // (Algorithm 1: learning rate and 2 alpha of the mask of Eq. weight)
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -513,10 +515,17 @@ __device__ __forceinline__ void resid_chunk(uint32_t taddr, bool full32, const P
 // 64-byte row segments.  With scale and shift, the words are fp32 accumulators
 // and column c stores fmaf(u, scale[c], shift[c]): after the transpose a lane
 // holds four fixed columns c = 4 (lane & 3) .. + 3, whose BN values the caller
-// passes in sc[] and sh[].
+// passes in sc[] and sh[].  With upd, dst0 holds latent weights w and each
+// value g replaces its w by the clipped masked step of sgd_masked.
+__device__ __forceinline__ float sgd_masked(float w, float g, float lr, float two_alpha) {
+    const float gw = (fabsf(w) <= 1.0f) ? g * two_alpha : 0.0f;
+    return fminf(1.0f, fmaxf(-1.0f, fmaf(-lr, gw, w)));
+}
+
 __device__ __forceinline__ void rows_store16(uint32_t *sw, const uint32_t (&u)[16], int lane, uint32_t *dst0,
                                              long long rstride, int nrows, int ncols,
-                                             const float *sc = nullptr, const float *sh = nullptr) {
+                                             const float *sc = nullptr, const float *sh = nullptr,
+                                             bool upd = false, float lr = 0.0f, float two_alpha = 0.0f) {
     uint4 *sw4 = reinterpret_cast<uint4 *>(sw);
     __syncwarp();
 #pragma unroll
@@ -524,6 +533,26 @@ __device__ __forceinline__ void rows_store16(uint32_t *sw, const uint32_t (&u)[1
         sw4[lane * 4 + (m ^ ((lane >> 1) & 3))] = make_uint4(u[4 * m], u[4 * m + 1], u[4 * m + 2], u[4 * m + 3]);
     __syncwarp();
     const int k = lane & 3, c = 4 * k;
+    // the update's latent weights: all four loads in flight before any store
+    float4 wv[4];
+    if (upd) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int rr = 8 * i + (lane >> 2);
+            wv[i] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            if (rr < nrows) {
+                const float *wd = reinterpret_cast<const float *>(dst0 + (long long)rr * rstride + c);
+                if (c + 4 <= ncols && (reinterpret_cast<uintptr_t>(wd) & 15) == 0) {
+                    wv[i] = *reinterpret_cast<const float4 *>(wd);
+                } else {
+                    if (c < ncols) wv[i].x = wd[0];
+                    if (c + 1 < ncols) wv[i].y = wd[1];
+                    if (c + 2 < ncols) wv[i].z = wd[2];
+                    if (c + 3 < ncols) wv[i].w = wd[3];
+                }
+            }
+        }
+    }
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const int rr = 8 * i + (lane >> 2);
@@ -536,7 +565,23 @@ __device__ __forceinline__ void rows_store16(uint32_t *sw, const uint32_t (&u)[1
         }
         if (rr < nrows) {
             uint32_t *d = dst0 + (long long)rr * rstride + c;
-            if (c + 4 <= ncols && (reinterpret_cast<uintptr_t>(d) & 15) == 0) {
+            const bool v4 = c + 4 <= ncols && (reinterpret_cast<uintptr_t>(d) & 15) == 0;
+            if (upd) {
+                float *wd = reinterpret_cast<float *>(d);
+                float4 w = wv[i];
+                w.x = sgd_masked(w.x, __uint_as_float(x.x), lr, two_alpha);
+                w.y = sgd_masked(w.y, __uint_as_float(x.y), lr, two_alpha);
+                w.z = sgd_masked(w.z, __uint_as_float(x.z), lr, two_alpha);
+                w.w = sgd_masked(w.w, __uint_as_float(x.w), lr, two_alpha);
+                if (v4) {
+                    *reinterpret_cast<float4 *>(wd) = w;
+                } else {
+                    if (c < ncols) wd[0] = w.x;
+                    if (c + 1 < ncols) wd[1] = w.y;
+                    if (c + 2 < ncols) wd[2] = w.z;
+                    if (c + 3 < ncols) wd[3] = w.w;
+                }
+            } else if (v4) {
                 *reinterpret_cast<uint4 *>(d) = x;
             } else {
                 if (c < ncols) d[0] = x.x;
@@ -1125,6 +1170,14 @@ __global__ void __launch_bounds__(NT, 1)
                         bsc[e] = __ldg(p.scale + oc + e);
                         bsh[e] = __ldg(p.shift + oc + e);
                     }
+                if (p.upd && b < p.B) {
+                    // the latent weights of this lane's row into L2 while the MMAs run
+                    const int o1 = o0 + gbeg * 16;
+                    const int ncol = min((gend - gbeg) * 16, p.O - o1);
+                    const float *wrow = p.y_out + (long long)b * p.O + o1;
+                    for (int off = 0; off < ncol; off += 32)
+                        asm volatile("prefetch.global.L2 [%0];\n" ::"l"(wrow + off));
+                }
             }
             if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
             fence_after();
@@ -1164,7 +1217,7 @@ __global__ void __launch_bounds__(NT, 1)
                     }
                     const int b0 = b - lane;
                     rows_store16(sw, u, lane, reinterpret_cast<uint32_t *>(p.y_out) + (long long)b0 * p.O + ob, p.O,
-                                 p.B - b0, p.O - ob, sc, sh);
+                                 p.B - b0, p.O - ob, sc, sh, p.upd != 0, p.upd_lr, p.upd_2a);
                 } else if (p.ksplit == 1) {
                     finish(a, ch);
                 } else if (p.rowst) {
@@ -1223,13 +1276,14 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const Params p, cons
     const int tiles_m = p.nbx * p.nby * p.nbb;
     const int tiles = tiles_m * p.ntn;
     const int g32 = (p.O + 31) >> 5;                 // 32-channel groups
-    const long long total = (long long)tiles_m * 128 * g32 * 8;
-    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    // 32-bit index arithmetic: the host launches fewer than 2^31 threads
+    const uint32_t total = (uint32_t)tiles_m * 128u * (uint32_t)g32 * 8u;
+    const uint32_t idx = blockIdx.x * blockDim.x + threadIdx.x;
     const int lane8 = threadIdx.x & 7;
     if (idx - lane8 >= total) return;               // whole 8-lane groups leave together
-    const long long rowgrp = idx >> 3;
-    const int g = (int)(rowgrp % g32);
-    const long long rr = rowgrp / g32;
+    const uint32_t rowgrp = idx >> 3;
+    const int g = (int)(rowgrp % (uint32_t)g32);
+    const uint32_t rr = rowgrp / (uint32_t)g32;
     const int tm = (int)(rr >> 7), r = (int)(rr & 127);
     const int o = g * 32 + lane8 * 4;                // first of this thread's four channels
     const bool live = o < p.O;
@@ -1538,7 +1592,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     {
         const int sms_ = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
         const int tiles_ = p.nbx * p.nby * p.nbb * p.ntn;
-        const int ks_ = (a.workspace != nullptr && !a.pool) ? (a.ksplit > 0 ? a.ksplit : auto_ksplit(tiles_, p.nk, sms_))
+        const int ks_ = (a.workspace != nullptr && !a.pool && !a.upd) ? (a.ksplit > 0 ? a.ksplit : auto_ksplit(tiles_, p.nk, sms_))
                                                             : 1;
         p.pair = (pair_pref() && !p.trans && p.BN == 256 && a.O % 256 == 0 && p.nk >= 18 && ks_ <= 1) ? 1 : 0;
     }
@@ -1550,7 +1604,8 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     const bool resid_ = a.res_codes != nullptr || a.res_f32 != nullptr || a.y_nhwc != nullptr;
     const bool rowst_fc = !p.trans && a.y_out != nullptr && a.Ho == 1 && a.Wo == 1 && !a.pool && !a.quant_out &&
                           a.acc_out == nullptr && !resid_;
-    const bool may_split = a.workspace != nullptr && !a.pool && !p.trans && !p.pair;
+    const bool may_split = a.workspace != nullptr && !a.pool && !p.trans && !p.pair && !a.upd;
+    if (a.upd && !rowst_fc) return MINW_EUNSUPPORTED;     // the update runs in the row-contiguous epilogue
     p.ystage = (rowst_fc || may_split) ? 8 * 32 * 16 : 0;
     const size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes - (p.ystage ? (size_t)p.ystage * 4 + 16 : 0);
     // two K blocks per stage (one commit per 8 or 4 MMAs) when three such stages fit
@@ -1572,6 +1627,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     while ((int)cols < 2 * mma_n) cols <<= 1;         // two accumulators
     p.tmem_cols = cols;
     p.acc_out = a.acc_out; p.y_out = a.y_out; p.scale = a.scale; p.shift = a.shift;
+    p.upd = a.upd; p.upd_lr = a.upd_lr; p.upd_2a = a.upd_2a;
     p.pool = a.pool; p.quant_out = a.quant_out; p.qo = a.qo;
     p.planes_out = a.planes_out; p.codes_out = a.codes_out;
     p.res_codes = a.res_codes; p.res_unit = a.res_unit; p.res_f32 = a.res_f32; p.y_nhwc = a.y_nhwc;
@@ -1581,7 +1637,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
     p.ksplit = 1;
     pl.thr_ws = nullptr;
-    if (a.workspace != nullptr && !a.pool && !p.trans && !p.pair) {
+    if (a.workspace != nullptr && !a.pool && !p.trans && !p.pair && !a.upd) {
         // workspace: [breakpoints, when not given][ksplit partial-sum slices]
         const size_t tb = (a.quant_out && a.thr == nullptr) ? thr_ws_bytes(a.O, p.nlev) : 0;
         const size_t sb = slice_bytes(tiles, p.BN);
@@ -1593,6 +1649,8 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
             ks = 1;
         }
         if (ks > p.nk) ks = p.nk;
+        // the reduction's threads (one per four channels of a tile row) index in 32 bits
+        if ((long long)p.nbx * p.nby * p.nbb * 128 * ((a.O + 31) / 32) * 8 >= (1ll << 31)) ks = 1;
         if (ks > 1) {
             p.ksplit = ks;
             uint8_t *w = reinterpret_cast<uint8_t *>(a.workspace);
@@ -1789,6 +1847,7 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
     if (split) {
         const int tiles_m = pl.p.nbx * pl.p.nby * pl.p.nbb;
         const long long threads = (long long)tiles_m * 128 * ((a.O + 31) / 32) * 8;
+        if (threads >= (1ll << 31)) return MINW_EUNSUPPORTED;     // the reduction indexes in 32 bits
         const unsigned blocks = (unsigned)((threads + 255) / 256);
         switch (outb) {
             case 1: minw_host::launch_pdl(tc::splitk_reduce_kernel<1>, dim3(blocks), dim3(256), 0, s, pl.p, thr); break;

@@ -16,6 +16,11 @@ struct ConvArgs {
     // epilogue
     int32_t *acc_out;      // int32 NCHW, unpooled (nullable)
     float *y_out;          // fp32 NCHW after BN [+HardTanh] (nullable)
+    // weight update in place of the fp32 output (fully connected bf16 products):
+    // y_out holds latent weights w, and each BN output g replaces its w by
+    // min(1, max(-1, w - lr 2 alpha g 1[|w| <= 1]))
+    int upd;
+    float upd_lr, upd_2a;
     const float *scale;    // BN scale [O]
     const float *shift;    // BN shift [O]
     int pool;              // 2x2/2 max pool on the accumulator before BN
@@ -79,7 +84,7 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s);
 minw_status conv2d_bf16(const uint16_t *act, int B, int C, int H, int W, const uint16_t *wgt, int O, int kh, int kw,
                         int bits_w, int stride, int pad, int pool, const float *scale, const float *shift,
                         float *y_out, void *workspace, size_t workspace_bytes, size_t *workspace_need,
-                        cudaStream_t s);
+                        cudaStream_t s, int upd = 0, float upd_lr = 0.0f, float upd_2a = 0.0f);
 bool conv_tc_supported(const ConvArgs &a);
 // Workspace the tensor-core path needs to split K for this shape (0: it does not split).
 size_t conv_tc_workspace_bytes(const ConvArgs &a);

@@ -7,7 +7,8 @@
 // [-1, 1].  The three products run on the tensor cores as 1 x 1 convolutions
 // of bf16 operands (conv_tc_kernel, kind::f16); each operand is made in one
 // pass over its fp32 source (AQE, bf16 rounding, the transposed copy), and the
-// mask of Eq. weight is fused with the update.
+// weight-gradient product applies the mask of Eq. weight and the update in its
+// epilogue, so that the weight gradient never reaches memory.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -172,31 +173,10 @@ __global__ void __launch_bounds__(256) prep_kernel(const float *__restrict__ X, 
     }
 }
 
-// The mask of Eq. weight and the update, fused: w <- clip(w - lr 2 alpha g 1[|w| <= 1])
-// with the fp32 operations of aqe_backward followed by sgd_clip.
-__global__ void __launch_bounds__(256) update_kernel(float *__restrict__ w, const float *__restrict__ g, int64_t n,
-                                                     float two_alpha, float lr) {
-    const int64_t n4 = n >> 2, stride = (int64_t)gridDim.x * blockDim.x;
-    float4 *w4 = reinterpret_cast<float4 *>(w);
-    const float4 *g4 = reinterpret_cast<const float4 *>(g);
-    auto upd = [&](float x, float gx) {
-        const float gw = (fabsf(x) <= 1.0f) ? gx * two_alpha : 0.0f;
-        return fminf(1.0f, fmaxf(-1.0f, fmaf(-lr, gw, x)));
-    };
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
-        float4 x = w4[i];
-        const float4 gx = __ldcs(g4 + i);
-        x.x = upd(x.x, gx.x); x.y = upd(x.y, gx.y); x.z = upd(x.z, gx.z); x.w = upd(x.w, gx.w);
-        w4[i] = x;
-    }
-    for (int64_t i = (n4 << 2) + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride)
-        w[i] = upd(w[i], g[i]);
-}
-
 // Workspace of minw_fc_train_step: regions 256-byte aligned, in this order;
 // split holds the K-sliced partial sums of the products.
 struct TrainLayout {
-    size_t wb, wtb, ab, atb, at, gb, gtb, gwhat, ones, zeros, split, split_bytes, total;
+    size_t wb, wtb, ab, atb, at, gb, gtb, ones, zeros, split, split_bytes, total;
 };
 
 static size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -214,8 +194,7 @@ static TrainLayout train_layout(int B, int K, int O) {
             need = w;
     };
     want(B, K, O);        // forward
-    want(B, Op, K);       // input gradient
-    want(O, B, K);        // weight gradient
+    want(B, Op, K);       // input gradient (the weight gradient never splits: it updates W in its epilogue)
     TrainLayout L;
     size_t off = 0;
     auto take = [&](size_t bytes) { const size_t r = off; off += al256(bytes); return r; };
@@ -226,7 +205,6 @@ static TrainLayout train_layout(int B, int K, int O) {
     L.at = take(4 * (size_t)B * O);
     L.gb = take(2 * (size_t)B * Op);
     L.gtb = take(2 * (size_t)O * B);
-    L.gwhat = take(4 * (size_t)O * K);
     L.ones = take(4 * M);
     L.zeros = take(4 * M);
     L.split_bytes = need;
@@ -282,7 +260,7 @@ minw_status minw_fc_train_step(const float *A, float *W, const float *g_out, int
     if ((int64_t)K * (O + 63) >= (1ll << 31) || (int64_t)B * K >= (1ll << 31)) return MINW_EUNSUPPORTED;
     cudaStream_t s = (cudaStream_t)stream;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
-    float *at = a_pre ? a_pre : reinterpret_cast<float *>(ws + L.at), *gwhat = reinterpret_cast<float *>(ws + L.gwhat);
+    float *at = a_pre ? a_pre : reinterpret_cast<float *>(ws + L.at);
     float *ones = reinterpret_cast<float *>(ws + L.ones), *zeros = reinterpret_cast<float *>(ws + L.zeros);
     uint16_t *wb = reinterpret_cast<uint16_t *>(ws + L.wb), *wtb = reinterpret_cast<uint16_t *>(ws + L.wtb);
     uint16_t *ab = reinterpret_cast<uint16_t *>(ws + L.ab), *atb = reinterpret_cast<uint16_t *>(ws + L.atb);
@@ -310,13 +288,11 @@ minw_status minw_fc_train_step(const float *A, float *W, const float *g_out, int
     if (g_in)                                          // g_a = g_a~ W^  ([B][K], reduction over O)
         TRY(conv2d_bf16(gb, B, Op, 1, 1, wtb, K, 1, 1, q_w->bits, 1, 0, 0, ones, zeros, g_in, split, L.split_bytes,
                         nullptr, s));
-    // g_W^ = g_a~^T a  ([O][K], reduction over the batch)
-    TRY(conv2d_bf16(gtb, O, B, 1, 1, atb, K, 1, 1, q_w->bits, 1, 0, 0, ones, zeros, gwhat, split, L.split_bytes,
-                    nullptr, s));
-    // 2. the mask of Eq. weight on the latent weights, the update and the clip
-    update_kernel<<<(unsigned)grid_of((int64_t)O * K / 4 + 1), 256, 0, s>>>(W, gwhat, (int64_t)O * K, 2.0f * alpha,
-                                                                            lr);
-    TRY(launch_status());
+    // g_W^ = g_a~^T a  ([O][K], reduction over the batch), and in the same epilogue
+    // 2. the mask of Eq. weight on the latent weights, the update and the clip:
+    // W = min(1, max(-1, W - lr 2 alpha g_W^ 1[|W| <= 1])), element by element
+    TRY(conv2d_bf16(gtb, O, B, 1, 1, atb, K, 1, 1, q_w->bits, 1, 0, 0, ones, zeros, W, nullptr, 0, nullptr, s, 1, lr,
+                    2.0f * alpha));
 #undef TRY
     return MINW_OK;
 }
