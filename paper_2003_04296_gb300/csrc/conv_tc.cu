@@ -1452,14 +1452,16 @@ static bool plan_shape(const ConvArgs &a, Params &p, int rows = 128) {
     return true;
 }
 
-// Split-K: a shape with fewer output tiles than half the SMs and a long K
-// loop (>= 16 stages) splits it into slices of at least four stages, up to
-// one work item per SM.  Short K loops gain less than the second launch costs.
+// Split-K: a shape with fewer output tiles than a third of the SMs and a long
+// K loop (>= 16 stages) splits it into slices of at least four stages, up to
+// one work item per SM.  Short K loops gain less than the second launch costs,
+// and a split in two gains less than its second epilogue round (the partial
+// sums) and the reduction cost.
 static int auto_ksplit(int tiles, int nk, int sms) {
-    if (tiles * 2 > sms || nk < 16) return 1;
+    if (tiles * 3 > sms || nk < 16) return 1;
     int ks = sms / tiles;
     if (ks > nk / 4) ks = nk / 4;
-    return ks < 2 ? 1 : ks;
+    return ks < 3 ? 1 : ks;
 }
 // channels of one K chunk: 128-byte rows of E4M3 codes (64-byte rows when C is
 // not a multiple of 128), or 64 bf16 values
