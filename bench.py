@@ -297,8 +297,7 @@ def run_reference(args, rank):
     if args.workload == "sweep":
         return run_reference_sweep(args)
     if args.workload == "fc_train":
-        print(json.dumps({"impl": "reference", "unavailable": "the CPU oracle arm covers the inference workloads only"}))
-        return 0
+        return run_reference_fc_train(args)
     wl = Workload(args.workload, args)
     x = wl.images(0)
     B = wl.batch
@@ -494,6 +493,63 @@ def step_bytes(B, K, O):
                  + (2 * B * Op + 2 * K * Op + 4 * BK) + (2 * O * B + 2 * K * B + 8 * OK))
 
 
+FC_TRAIN_SHAPE = (256, 8192, 1024)       # batch, K, O: fc1 of the CIFAR model
+FC_TRAIN_ALPHA, FC_TRAIN_LR = 0.75, 1e-3
+
+
+def fc_train_problem(rank=0):
+    """Seeded input, latent weights and upstream gradient of the training
+    workload (fp32 numpy)."""
+    B, K, O = FC_TRAIN_SHAPE
+    r = np.random.default_rng(31 + 1000 * rank)
+    A = np.clip(r.standard_normal((B, K)), -1.5, 1.5).astype(np.float32)
+    W = r.uniform(-1, 1, (O, K)).astype(np.float32)
+    G = (r.standard_normal((B, O)) * 0.1).astype(np.float32)
+    return A, W, G
+
+
+def fc_train_oracle_rate(A, W, G, budget_s=10.0, warmup=1, max_steps=30):
+    """The oracle's training step (oracle.fc_train_step), timed on the host:
+    whole steps until budget_s seconds; returns (images/s, s per step, steps)."""
+    from oracle import oracle as Or
+    from paper_2003_04296_gb300.inputs import DEFAULT_THR
+    qw, qa = (1, DEFAULT_THR[1]), (1, DEFAULT_THR[1])
+    for _ in range(warmup):
+        Or.fc_train_step(A, W, G, FC_TRAIN_ALPHA, FC_TRAIN_LR, qw[0], qw[1], qa)
+    times = []
+    t_start = time.perf_counter()
+    while len(times) < max_steps and (not times or time.perf_counter() - t_start < budget_s):
+        t0 = time.perf_counter()
+        Or.fc_train_step(A, W, G, FC_TRAIN_ALPHA, FC_TRAIN_LR, qw[0], qw[1], qa)
+        times.append(time.perf_counter() - t0)
+    sec = sum(times) / len(times)
+    return A.shape[0] / sec, sec, len(times)
+
+
+def fc_train_config(world):
+    B, K, O = FC_TRAIN_SHAPE
+    return {"workload": "fc_train_8192x1024_b256_a1w1", "batch_per_gpu": B, "global_batch": B * world,
+            "layer": f"FC {K} -> {O} (Model A's fc1), alpha {FC_TRAIN_ALPHA}, lr {FC_TRAIN_LR}, SGD + clip",
+            "parallelism": f"replicas x{world} (no gradient all-reduce)", "l2": L2_NOTE}
+
+
+def run_reference_fc_train(args):
+    """The oracle's training step on the training workload, whole steps."""
+    A, W, G = fc_train_problem(0)
+    ips, sec, n = fc_train_oracle_rate(A, W, G, budget_s=1e9, warmup=args.warmup, max_steps=args.steps)
+    sample = (f"{n} full steps of the batch through oracle.fc_train_step (numpy's BLAS threads for the three fp64 "
+              "products, single-threaded C for the elementwise stages)")
+    line = {"metric": "Algorithm 1 training step of a fully connected MINW layer: images/s", "value": ips,
+            "unit": "images/s", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": sec * 1e3, "higher_is_better": True, "impl": "reference", "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": fc_train_config(args.gpus),
+            "cpu_baseline": {"value": ips, "unit": "images/s", "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": ips, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_fc_train(args, rank, world, local_rank):
     """Algorithm 1's training step of Model A's first fully connected layer
     (8192 -> 1024, batch 256, 1-bit weights and activations, alpha 0.75): the
@@ -514,11 +570,9 @@ def run_fc_train(args, rank, world, local_rank):
     from paper_2003_04296_gb300.inputs import DEFAULT_THR
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    B, K, O = 256, 8192, 1024
-    r = np.random.default_rng(31 + 1000 * rank)
-    A = torch.from_numpy(np.clip(r.standard_normal((B, K)), -1.5, 1.5).astype(np.float32)).to(dev)
-    W = torch.from_numpy(r.uniform(-1, 1, (O, K)).astype(np.float32)).to(dev)
-    G = torch.from_numpy((r.standard_normal((B, O)) * 0.1).astype(np.float32)).to(dev)
+    B, K, O = FC_TRAIN_SHAPE
+    A_np, W_np, G_np = fc_train_problem(rank)
+    A, W, G = (torch.from_numpy(x).to(dev) for x in (A_np, W_np, G_np))
     a_out = torch.empty((B, O), device=dev)
     g_in = torch.empty((B, K), device=dev)
     ws = torch.empty(minw.minw_fc_train_workspace_bytes(B, K, O), dtype=torch.uint8, device=dev)
@@ -527,7 +581,7 @@ def run_fc_train(args, rank, world, local_rank):
     stream = torch.cuda.current_stream()
 
     def step():
-        minw.minw_fc_train_step(A, W, G, 0.75, 1e-3, qw, qa, a_out, g_in, ws)
+        minw.minw_fc_train_step(A, W, G, FC_TRAIN_ALPHA, FC_TRAIN_LR, qw, qa, a_out, g_in, ws)
 
     for _ in range(max(args.warmup, 3)):
         step()
@@ -561,6 +615,13 @@ def run_fc_train(args, rank, world, local_rank):
     e2e_sec = max_over_ranks(sum(e2e_s) / len(e2e_s), world, dev)
     if rank != 0:
         return 0
+    cpu = None
+    if world == 1 and not args.skip_cpu:
+        ips, sec, n = fc_train_oracle_rate(A_np, W_np, G_np, budget_s=10.0)
+        cpu = {"value": ips, "unit": "images/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"{n} full steps of the same batch through oracle.fc_train_step ({sec * 1e3:.0f} ms "
+                         "each; numpy's BLAS threads for the three fp64 products, single-threaded C for the "
+                         "elementwise stages)"}
     flops = 6.0 * B * K * O
     nbytes = step_bytes(B, K, O)
     achieved = nbytes / (ms_max * 1e-3) / 1e9
@@ -568,9 +629,7 @@ def run_fc_train(args, rank, world, local_rank):
             "value": replica_throughput(B, world, ms_max * 1e-3), "unit": "images/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": "fc_train_8192x1024_b256_a1w1", "batch_per_gpu": B, "global_batch": B * world,
-                       "layer": "FC 8192 -> 1024 (Model A's fc1), alpha 0.75, lr 1e-3, SGD + clip",
-                       "parallelism": f"replicas x{world} (no gradient all-reduce)", "l2": L2_NOTE},
+            "config": fc_train_config(world),
             "roofline": {"bound": "hbm", "kernel": "the whole step (7 launches: 3 operand passes, 3 bf16 "
                                                    "tensor-core products, the forward's K-slice sum, the "
                                                    "update inside the weight-gradient epilogue)",
@@ -578,7 +637,7 @@ def run_fc_train(args, rank, world, local_rank):
                          "frac": achieved / HBM_GBS, "traffic": None, "bytes_per_step": nbytes,
                          "peak_basis": "measured HBM copy GB/s, of measured"},
             "tensor_tflops": flops / (ms_max * 1e-3) / 1e12,
-            "cpu_baseline": None,
+            "cpu_baseline": cpu,
             "e2e": {"value": replica_throughput(B, world, e2e_sec), "unit": "images/s",
                     "h2d_bytes_per_step": int(4 * (A.numel() + G.numel())), "d2h_bytes_per_step": int(4 * g_in.numel())},
             "gpu_launches": 7 * args.steps, "clocks": clk.summary()}

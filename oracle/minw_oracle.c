@@ -291,6 +291,12 @@ float orc_bf16_round(float x)
     return r;
 }
 
+/* orc_bf16_round over n values. */
+void orc_bf16_round_array(const float *x, int64_t n, float *out)
+{
+    for (int64_t i = 0; i < n; ++i) out[i] = orc_bf16_round(x[i]);
+}
+
 /* Direct convolution in fp64 of real activations a [B][C][H][W] with weights
  * w [O][C][kh][kw], zero padding: the exact real-valued accumulator (every
  * product of a bf16 value and a level is exact, and so is the fp64 sum at

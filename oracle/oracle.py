@@ -45,6 +45,7 @@ def lib():
         L.orc_pack.argtypes = [P, i32, i32, i32, i32, i32, P]
         L.orc_bf16_round.restype = f32
         L.orc_bf16_round.argtypes = [f32]
+        L.orc_bf16_round_array.argtypes = [P, i64, P]
         L.orc_conv2d_real.argtypes = [P, i32, i32, i32, i32, P, i32, i32, i32, i32, i32, P]
         L.orc_conv2d.restype = i32
         L.orc_conv2d.argtypes = [P, i32, i32, i32, i32, P, i32, i32, i32, i32, i32, i32, P]
@@ -209,8 +210,40 @@ def conv2d_levels(a_lv, w_lv, stride, pad, bits_a, bits_w):
 def bf16_round(x):
     """fp32 -> bf16 (round to nearest, ties to even), returned as fp32 values."""
     x = _f32(x)
-    f = lib().orc_bf16_round
-    return np.array([f(float(v)) for v in x.reshape(-1)], dtype=np.float32).reshape(x.shape)
+    out = np.empty(x.shape, dtype=np.float32)
+    lib().orc_bf16_round_array(_p(x), x.size, _p(out))
+    return out
+
+
+def bf16_round_scalar(v):
+    """bf16_round of one value, through the scalar C routine."""
+    return float(lib().orc_bf16_round(float(v)))
+
+
+def fc_train_step(A, W, G, alpha, lr, bits_w, thr_w, q_a=None):
+    """One step of Algorithm 1 on a fully connected layer with input A [B][K],
+    latent weights W [O][K] and upstream gradient G [B][O], in the order of
+    Algorithm 1: the weight AQE (Eq. weight, fp32), the forward product a~ of
+    the bf16 operands (fp64 sums, rounded to fp32), the activation AQE and its
+    backward mask (Eq. activation; skipped for the last layer, q_a None), the
+    input gradient g_in = bf16(g~) bf16(W^) and the weight gradient
+    g_W^ = bf16(g~)^T bf16(A) (fp64 sums, rounded to fp32), then the mask of
+    Eq. weight and the clipped update.  q_a = (bits, thr).  Returns
+    (a_out, g_in, W_new, a_pre) as fp32 arrays."""
+    A, W, G = _f32(A), _f32(W), _f32(G)
+    what = aqe_forward_f32(W, alpha, bits_w, thr_w)
+    Wq, Aq = bf16_round(what).astype(np.float64), bf16_round(A).astype(np.float64)
+    a_pre = (Aq @ Wq.T).astype(np.float32)
+    if q_a is None:
+        a_out, g_t = a_pre, G
+    else:
+        a_out = aqe_forward_f32(a_pre, alpha, q_a[0], q_a[1])
+        g_t = aqe_backward_f32(a_pre, G, alpha)
+    Gq = bf16_round(g_t).astype(np.float64)
+    g_in = (Gq @ Wq).astype(np.float32)
+    g_w = (Gq.T @ Aq).astype(np.float32)
+    W_new = sgd_clip(W, aqe_backward_f32(W, g_w, alpha), lr)
+    return a_out, g_in, W_new, a_pre
 
 
 def conv2d_real(a, w, stride, pad):

@@ -75,3 +75,76 @@ def test_backward_products_are_the_gradients():
     for (i, j) in [(0, 1), (4, 5), (2, 2)]:
         E = np.zeros_like(W); E[i, j] = h
         assert abs((f(A, W + E) - f(A, W - E)) / (2 * h) - gW[i, j]) < 1e-6
+
+
+def _bf16_torch(x):
+    """bf16 rounding by torch's conversion (independent of the oracle's)."""
+    torch = pytest.importorskip("torch")
+    return torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).to(torch.bfloat16).float().numpy()
+
+
+@pytest.mark.parametrize("last", [False, True])
+def test_fc_train_step_wiring(last):
+    """The composed step against properties it must have: a_pre is the fp32
+    rounding of the exact (rational) product of the bf16 operands; g_in and
+    the weight step are the gradients of sum(g~ * a~) with respect to the
+    bf16 input and weights (central differences in fp64), so a transposed or
+    swapped operand fails; the last layer passes g through unmasked."""
+    r = np.random.default_rng(11)
+    B, K, O_ = 3, 8, 4
+    A = np.clip(r.standard_normal((B, K)), -1.5, 1.5).astype(np.float32)
+    W = r.uniform(-1, 1, (O_, K)).astype(np.float32)
+    G = (r.standard_normal((B, O_)) * 0.5).astype(np.float32)
+    alpha, lr = 0.6, 0.125
+    q_a = None if last else (2, DEFAULT_THR[2])
+    a_out, g_in, W_new, a_pre = O.fc_train_step(A, W, G, alpha, lr, 1, DEFAULT_THR[1], q_a)
+    Wq = _bf16_torch(O.aqe_forward_f32(W, alpha, 1, DEFAULT_THR[1]))
+    Aq = _bf16_torch(A)
+    for i in range(B):
+        for o in range(O_):
+            exact = sum(Fraction(float(Aq[i, k])) * Fraction(float(Wq[o, k])) for k in range(K))
+            assert a_pre[i, o] == np.float32(float(exact))
+    if last:
+        assert np.array_equal(a_out, a_pre)
+        gt = G
+    else:
+        assert np.array_equal(a_out, O.aqe_forward_f32(a_pre, alpha, 2, DEFAULT_THR[2]))
+        gt = O.aqe_backward_f32(a_pre, G, alpha)
+    Gq = _bf16_torch(gt).astype(np.float64)
+    L = lambda A_, W_: np.sum(Gq * (A_ @ W_.T))
+    h = 1e-3
+    A64, W64 = Aq.astype(np.float64), Wq.astype(np.float64)
+    for i in range(B):
+        for k in range(K):
+            E = np.zeros_like(A64); E[i, k] = h
+            d = (L(A64 + E, W64) - L(A64 - E, W64)) / (2 * h)
+            assert abs(g_in[i, k] - d) <= 1e-6 * (1 + abs(d))
+    for o in range(O_):
+        for k in range(K):
+            E = np.zeros_like(W64); E[o, k] = h
+            d = (L(A64, W64 + E) - L(A64, W64 - E)) / (2 * h)
+            want = np.clip(W[o, k] - lr * 2 * alpha * d, -1.0, 1.0)     # |W| <= 1: the mask passes
+            assert abs(W_new[o, k] - want) <= 1e-6
+
+
+def test_fc_train_step_alpha_zero():
+    """alpha = 0: W^ = W, the masks' factor 2 alpha vanishes, so the weights
+    stay as they are and (hidden layer) the input gradient is zero."""
+    r = np.random.default_rng(12)
+    A = r.standard_normal((4, 16)).astype(np.float32)
+    W = r.uniform(-1, 1, (5, 16)).astype(np.float32)
+    G = r.standard_normal((4, 5)).astype(np.float32)
+    a_out, g_in, W_new, a_pre = O.fc_train_step(A, W, G, 0.0, 0.5, 2, DEFAULT_THR[2], (1, DEFAULT_THR[1]))
+    assert np.array_equal(W_new, W)
+    assert not g_in.any()
+    assert np.array_equal(a_out, a_pre)
+
+
+def test_bf16_round_array_matches_scalar():
+    """The array form of the oracle's bf16 rounding equals its scalar form,
+    ties and specials included."""
+    x = np.concatenate([_x(seed=21), np.array([1.00390625, 1.01171875, -2.0 ** -130, 3.0e38, np.inf, -np.inf],
+                                              dtype=np.float32)]).astype(np.float32)
+    got = O.bf16_round(x)
+    want = np.array([O.bf16_round_scalar(v) for v in x], dtype=np.float32)
+    assert np.array_equal(got, want)
