@@ -258,6 +258,7 @@ minw_status minw_fc_train_step(const float *A, float *W, const float *g_out, int
     const TrainLayout L = train_layout(B, K, O);
     if (workspace_bytes < L.total) return MINW_EINVAL;
     if ((int64_t)K * (O + 63) >= (1ll << 31) || (int64_t)B * K >= (1ll << 31)) return MINW_EUNSUPPORTED;
+    if ((O + 63) / 32 > 65535 || B / 32 > 65535) return MINW_EUNSUPPORTED;       // grid rows of the passes
     cudaStream_t s = (cudaStream_t)stream;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     float *at = a_pre ? a_pre : reinterpret_cast<float *>(ws + L.at);
