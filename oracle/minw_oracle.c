@@ -1,7 +1,8 @@
 /*
- * minw_oracle.c -- plain CPU oracle for the MINW-Net inference path and the
- * AQE quantizer (arXiv 2003.04296, "Propagating Asymptotic-Estimated Gradients
- * for Low Bitwidth Quantized Neural Networks").
+ * minw_oracle.c -- plain CPU oracle for the MINW-Net inference path, the
+ * AQE quantizer and the fp32 pieces of Algorithm 1's training step (arXiv
+ * 2003.04296, "Propagating Asymptotic-Estimated Gradients for Low Bitwidth
+ * Quantized Neural Networks").
  *
  * TEST INFRASTRUCTURE ONLY.  This file is the slow, obviously-correct
  * definition the CUDA path is checked against.  Only tests/, the smoke()
