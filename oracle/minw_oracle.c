@@ -325,6 +325,60 @@ void orc_conv2d_real(const double *a, int B, int C, int H, int W,
                 }
 }
 
+/* The two backward products of Algorithm 1 for a convolutional layer whose
+ * forward is orc_conv2d_real (a~ = a * W, zero padding), in fp64:
+ *   input gradient  g_a[b][c][y][x]   = sum over (o, yo, xo, ky, kx) with
+ *                   y = yo stride - pad + ky, x = xo stride - pad + kx of
+ *                   g[b][o][yo][xo] w[o][c][ky][kx]
+ *   weight gradient g_w[o][c][ky][kx] = sum over (b, yo, xo) of
+ *                   g[b][o][yo][xo] a[b][c][yo stride - pad + ky][xo stride - pad + kx]
+ *                   (taps outside the image contribute 0).
+ * Both walk the forward's index map directly: every (output, tap) pair of the
+ * forward adds its product to the input or weight it came from. */
+void orc_conv2d_input_grad(const double *g, int B, int O, int Ho, int Wo,
+                           const double *w, int C, int kh, int kw, int stride, int pad,
+                           int H, int W, double *ga)
+{
+    for (size_t i = 0; i < (size_t)B * C * H * W; ++i) ga[i] = 0.0;
+    for (int b = 0; b < B; ++b)
+        for (int o = 0; o < O; ++o)
+            for (int yo = 0; yo < Ho; ++yo)
+                for (int xo = 0; xo < Wo; ++xo) {
+                    const double gv = g[(((size_t)b * O + o) * Ho + yo) * Wo + xo];
+                    for (int c = 0; c < C; ++c)
+                        for (int ky = 0; ky < kh; ++ky)
+                            for (int kx = 0; kx < kw; ++kx) {
+                                int yi = yo * stride - pad + ky;
+                                int xi = xo * stride - pad + kx;
+                                if (yi < 0 || yi >= H || xi < 0 || xi >= W) continue;
+                                ga[(((size_t)b * C + c) * H + yi) * W + xi] +=
+                                    gv * w[(((size_t)o * C + c) * kh + ky) * kw + kx];
+                            }
+                }
+}
+
+void orc_conv2d_weight_grad(const double *g, int B, int O, int Ho, int Wo,
+                            const double *a, int C, int H, int W, int kh, int kw, int stride, int pad,
+                            double *gw)
+{
+    for (size_t i = 0; i < (size_t)O * C * kh * kw; ++i) gw[i] = 0.0;
+    for (int b = 0; b < B; ++b)
+        for (int o = 0; o < O; ++o)
+            for (int yo = 0; yo < Ho; ++yo)
+                for (int xo = 0; xo < Wo; ++xo) {
+                    const double gv = g[(((size_t)b * O + o) * Ho + yo) * Wo + xo];
+                    for (int c = 0; c < C; ++c)
+                        for (int ky = 0; ky < kh; ++ky)
+                            for (int kx = 0; kx < kw; ++kx) {
+                                int yi = yo * stride - pad + ky;
+                                int xi = xo * stride - pad + kx;
+                                if (yi < 0 || yi >= H || xi < 0 || xi >= W) continue;
+                                gw[(((size_t)o * C + c) * kh + ky) * kw + kx] +=
+                                    gv * a[(((size_t)b * C + c) * H + yi) * W + xi];
+                            }
+                }
+}
+
 /* ------------------------------------------------------------------------ */
 /* Layer pieces around the convolution (Sec. III-E)                          */
 /* ------------------------------------------------------------------------ */

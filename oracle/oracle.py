@@ -47,6 +47,8 @@ def lib():
         L.orc_bf16_round.argtypes = [f32]
         L.orc_bf16_round_array.argtypes = [P, i64, P]
         L.orc_conv2d_real.argtypes = [P, i32, i32, i32, i32, P, i32, i32, i32, i32, i32, P]
+        L.orc_conv2d_input_grad.argtypes = [P, i32, i32, i32, i32, P, i32, i32, i32, i32, i32, i32, i32, P]
+        L.orc_conv2d_weight_grad.argtypes = [P, i32, i32, i32, i32, P, i32, i32, i32, i32, i32, i32, i32, P]
         L.orc_conv2d.restype = i32
         L.orc_conv2d.argtypes = [P, i32, i32, i32, i32, P, i32, i32, i32, i32, i32, i32, P]
         L.orc_maxpool_i32.argtypes = [P, i32, i32, i32, i32, i32, i32, P]
@@ -259,6 +261,57 @@ def conv2d_real(a, w, stride, pad):
     out = np.empty((B, O, Ho, Wo), dtype=np.float64)
     lib().orc_conv2d_real(_p(a), B, C, H, W, _p(w), O, kh, kw, stride, pad, _p(out))
     return out
+
+
+def conv2d_input_grad(g, w, stride, pad, H, W):
+    """Algorithm 1's input gradient of a convolutional layer: the gradient of
+    sum(g * conv2d_real(a, w)) with respect to a [B][C][H][W] (fp64)."""
+    g = np.ascontiguousarray(g, dtype=np.float64)
+    w = np.ascontiguousarray(w, dtype=np.float64)
+    B, O, Ho, Wo = g.shape
+    O2, C, kh, kw = w.shape
+    assert O == O2
+    ga = np.empty((B, C, H, W), dtype=np.float64)
+    lib().orc_conv2d_input_grad(_p(g), B, O, Ho, Wo, _p(w), C, kh, kw, stride, pad, H, W, _p(ga))
+    return ga
+
+
+def conv2d_weight_grad(g, a, kh, kw, stride, pad):
+    """Algorithm 1's weight gradient of a convolutional layer: the gradient of
+    sum(g * conv2d_real(a, w)) with respect to w [O][C][kh][kw] (fp64)."""
+    g = np.ascontiguousarray(g, dtype=np.float64)
+    a = np.ascontiguousarray(a, dtype=np.float64)
+    B, O, Ho, Wo = g.shape
+    B2, C, H, W = a.shape
+    assert B == B2
+    gw = np.empty((O, C, kh, kw), dtype=np.float64)
+    lib().orc_conv2d_weight_grad(_p(g), B, O, Ho, Wo, _p(a), C, H, W, kh, kw, stride, pad, _p(gw))
+    return gw
+
+
+def conv_train_step(A, W, G, alpha, lr, bits_w, thr_w, stride, pad, q_a=None):
+    """Algorithm 1 on a convolutional layer, in the order of fc_train_step:
+    weight AQE (fp32), the forward convolution of the bf16 operands (fp64 sums
+    rounded to fp32), the activation AQE and its mask (q_a = (bits, thr); None
+    for a layer without an activation quantizer), the input and weight
+    gradients of the bf16 operands (fp64 sums rounded to fp32), then the mask
+    of Eq. weight and the clipped update.  A [B][C][H][W], W [O][C][kh][kw],
+    G [B][O][Ho][Wo].  Returns (a_out, g_in, W_new, a_pre)."""
+    A, W, G = _f32(A), _f32(W), _f32(G)
+    what = aqe_forward_f32(W, alpha, bits_w, thr_w)
+    Wq, Aq = bf16_round(what).astype(np.float64), bf16_round(A).astype(np.float64)
+    a_pre = conv2d_real(Aq, Wq, stride, pad).astype(np.float32)
+    if q_a is None:
+        a_out, g_t = a_pre, G
+    else:
+        a_out = aqe_forward_f32(a_pre, alpha, q_a[0], q_a[1])
+        g_t = aqe_backward_f32(a_pre, G, alpha)
+    Gq = bf16_round(g_t).astype(np.float64)
+    H, Wd = A.shape[2], A.shape[3]
+    g_in = conv2d_input_grad(Gq, Wq, stride, pad, H, Wd).astype(np.float32)
+    g_w = conv2d_weight_grad(Gq, Aq, W.shape[2], W.shape[3], stride, pad).astype(np.float32)
+    W_new = sgd_clip(W, aqe_backward_f32(W, g_w, alpha), lr)
+    return a_out, g_in, W_new, a_pre
 
 
 def maxpool_f64(x, k=2, s=2):

@@ -148,3 +148,65 @@ def test_bf16_round_array_matches_scalar():
     got = O.bf16_round(x)
     want = np.array([O.bf16_round_scalar(v) for v in x], dtype=np.float32)
     assert np.array_equal(got, want)
+
+
+@pytest.mark.parametrize("stride,pad,k", [(1, 1, 3), (2, 1, 3), (1, 0, 1), (2, 0, 2)])
+def test_conv_backward_products_match_autograd(stride, pad, k):
+    """The convolutional layer's input and weight gradients equal torch's
+    autograd of conv2d in float64 (an independent implementation), strided
+    and padded; a transposed or flipped kernel fails."""
+    torch = pytest.importorskip("torch")
+    r = np.random.default_rng(100 + stride * 10 + pad + k)
+    B, C, H, W, O_ = 2, 3, 7, 6, 4
+    a = r.standard_normal((B, C, H, W))
+    w = r.standard_normal((O_, C, k, k))
+    at = torch.tensor(a, requires_grad=True)
+    wt = torch.tensor(w, requires_grad=True)
+    y = torch.nn.functional.conv2d(at, wt, stride=stride, padding=pad)
+    g = r.standard_normal(tuple(y.shape))
+    (y * torch.tensor(g)).sum().backward()
+    assert np.allclose(O.conv2d_real(a, w, stride, pad), y.detach().numpy(), rtol=1e-12, atol=1e-12)
+    assert np.allclose(O.conv2d_input_grad(g, w, stride, pad, H, W), at.grad.numpy(), rtol=1e-12, atol=1e-12)
+    assert np.allclose(O.conv2d_weight_grad(g, a, k, k, stride, pad), wt.grad.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_conv_train_step_reduces_to_fc():
+    """A 1 x 1 convolution over 1 x 1 images is a fully connected layer: the
+    convolutional step equals fc_train_step bit for bit."""
+    r = np.random.default_rng(13)
+    B, K, O_ = 4, 16, 6
+    A = np.clip(r.standard_normal((B, K)), -1.5, 1.5).astype(np.float32)
+    W = r.uniform(-1, 1, (O_, K)).astype(np.float32)
+    G = (r.standard_normal((B, O_)) * 0.5).astype(np.float32)
+    for q_a in [None, (2, DEFAULT_THR[2])]:
+        fc = O.fc_train_step(A, W, G, 0.7, 0.25, 3, DEFAULT_THR[3], q_a)
+        cv = O.conv_train_step(A[:, :, None, None], W[:, :, None, None], G[:, :, None, None], 0.7, 0.25, 3,
+                               DEFAULT_THR[3], 1, 0, q_a)
+        for x, y in zip(fc, cv):
+            assert np.array_equal(x, y.reshape(x.shape))
+
+
+def test_conv_train_step_gradients():
+    """The convolutional step's input gradient and weight step are the
+    gradients of sum(g~ * a~) with respect to the bf16 operands (torch autograd
+    in float64 on torch-rounded bf16 operands), with the mask of Eq. weight
+    and the clip on the latent weights."""
+    torch = pytest.importorskip("torch")
+    r = np.random.default_rng(14)
+    A = np.clip(r.standard_normal((2, 4, 6, 6)), -1.5, 1.5).astype(np.float32)
+    W = r.uniform(-1.2, 1.2, (3, 4, 3, 3)).astype(np.float32)       # some |w| > 1: masked
+    G = (r.standard_normal((2, 3, 3, 3)) * 0.5).astype(np.float32)
+    alpha, lr = 0.5, 0.125
+    a_out, g_in, W_new, a_pre = O.conv_train_step(A, W, G, alpha, lr, 2, DEFAULT_THR[2], 2, 1, (1, DEFAULT_THR[1]))
+    Wq = torch.tensor(_bf16_torch(O.aqe_forward_f32(W, alpha, 2, DEFAULT_THR[2])).astype(np.float64),
+                      requires_grad=True)
+    Aq = torch.tensor(_bf16_torch(A).astype(np.float64), requires_grad=True)
+    y = torch.nn.functional.conv2d(Aq, Wq, stride=2, padding=1)
+    assert np.allclose(a_pre, y.detach().numpy(), rtol=2.0 ** -23, atol=1e-30)
+    gt = _bf16_torch(O.aqe_backward_f32(a_pre, G, alpha)).astype(np.float64)
+    (y * torch.tensor(gt)).sum().backward()
+    assert np.allclose(g_in, Aq.grad.numpy(), rtol=2.0 ** -23, atol=1e-30)
+    gw = Wq.grad.numpy()
+    want = np.clip(W - lr * np.where(np.abs(W) <= 1.0, 2 * alpha * gw, 0.0), -1.0, 1.0)
+    assert np.allclose(W_new, want, rtol=0, atol=1e-6)
+    assert np.array_equal(W_new[np.abs(W) > 1.0], np.clip(W[np.abs(W) > 1.0], -1, 1))
