@@ -265,14 +265,21 @@ MINW_API minw_status minw_conv2d_bf16(const uint16_t *act, int32_t B, int32_t C,
 /* Training step of a fully connected layer (Algorithm 1)                  */
 /* ---------------------------------------------------------------------- */
 
-/* out (bf16, round to nearest even, row-major (transpose ? cols : rows) x
- * out_cols) = in (fp32 row-major rows x cols), transposed when transpose != 0,
- * zero in the columns past the source's.  out_cols >= the source's columns. */
+/* The bf16 operands of Algorithm 1's training products (R21 reading: bf16
+ * operands, fp32 sums).  out (bf16, round to nearest even, row-major
+ * (transpose ? cols : rows) x out_cols) = in (fp32 row-major rows x cols),
+ * transposed when transpose != 0, zero in the columns past the source's.
+ * Caller-owned device buffers; asynchronous on stream.  MINW_EINVAL for null
+ * pointers, non-positive sizes or out_cols below the source's columns;
+ * MINW_EUNSUPPORTED past 65535 x 32 output rows. */
 MINW_API minw_status minw_bf16_matrix(const float *in, int32_t rows, int32_t cols, int32_t transpose,
                                       int32_t out_cols, uint16_t *out, void *stream);
 
-/* The update of Algorithm 1 with a plain gradient step:
- * w = min(1, max(-1, fmaf(-lr, g, w))), n floats in place. */
+/* The update of Algorithm 1 with a plain gradient step (update(W, g, eta)
+ * then the clip to [-1, 1]): w = min(1, max(-1, fmaf(-lr, g, w))), n fp32
+ * values of device memory in place (g is the already masked gradient).
+ * Asynchronous on stream; n == 0 does nothing; MINW_EINVAL for n < 0 or null
+ * pointers. */
 MINW_API minw_status minw_sgd_clip(float *w, const float *g, int64_t n, float lr, void *stream);
 
 /* Bytes of device workspace minw_fc_train_step needs (0 for bad sizes). */
@@ -295,7 +302,12 @@ MINW_API size_t minw_fc_train_workspace_bytes(int32_t B, int32_t K, int32_t O);
  * slices, slice by slice in a fixed order (deterministic, same bound).
  * Requirements: K % 64 == 0 and B % 64 == 0 (else MINW_EUNSUPPORTED), alpha in
  * [0, 1], 16-byte aligned pointers, workspace of minw_fc_train_workspace_bytes
- * (scratch: nothing in it survives the call). */
+ * (scratch: nothing in it survives the call).  All buffers are caller-owned
+ * device memory; the call is asynchronous on stream and launches 7-8 kernels.
+ * MINW_EINVAL: null A, W, g_out, a_out, q_w or workspace, an invalid quantizer,
+ * alpha outside [0, 1], a misaligned pointer or a short workspace;
+ * MINW_EUNSUPPORTED: the shapes above, or sizes past the kernels' 32-bit
+ * index and grid limits. */
 MINW_API minw_status minw_fc_train_step(const float *A, float *W, const float *g_out, int32_t B, int32_t K,
                                         int32_t O, float alpha, float lr, const minw_quant *q_w,
                                         const minw_quant *q_a, float *a_out, float *g_in, float *a_pre,
