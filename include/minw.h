@@ -303,7 +303,7 @@ MINW_API size_t minw_fc_train_workspace_bytes(int32_t B, int32_t K, int32_t O);
  * Requirements: K % 64 == 0 and B % 64 == 0 (else MINW_EUNSUPPORTED), alpha in
  * [0, 1], 16-byte aligned pointers, workspace of minw_fc_train_workspace_bytes
  * (scratch: nothing in it survives the call).  All buffers are caller-owned
- * device memory; the call is asynchronous on stream and launches 7-8 kernels.
+ * device memory; the call is asynchronous on stream and launches five to eight kernels.
  * MINW_EINVAL: null A, W, g_out, a_out, q_w or workspace, an invalid quantizer,
  * alpha outside [0, 1], a misaligned pointer or a short workspace;
  * MINW_EUNSUPPORTED: the shapes above, or sizes past the kernels' 32-bit
