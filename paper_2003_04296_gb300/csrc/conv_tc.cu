@@ -70,12 +70,12 @@ struct Params {
     const float *thr;          // precomputed breakpoints [O][nlev] (nullable)
     int nlev;                  // levels of the output quantizer
     int ksplit;                // K slices per output tile (1: no split)
-    int cl;                    // CTAs per cluster sharing each weight box (1, 2 or 4; 1 when split)
+    int cl;                    // CTAs per cluster: 2 for CTA pairs, else 1
     int dup;                   // channel-major 64-channel layer: the weight rows loaded twice (MMA rows
                                // 64 .. 127 repeat 0 .. 63), so that all eight epilogue warps hold channels
     int pair;                  // CTA pairs (cl = 2): one cta_group::2 MMA of M = 256 pixels per pair, each
                                // CTA holding its 128 pixels and half of the weight rows
-    int tiles_mp;              // pixel tiles per channel tile, padded to a multiple of cl
+    int tiles_mp;              // pixel tiles per channel tile, padded to a multiple of cl (even for pairs)
     int32_t *part;             // split-K: int32 partial sums [ksplit][tiles][128][BN]
     // residual blocks: y = BN(acc) + shortcut, then HardTanh + quantize
     const uint8_t *res_codes;  // shortcut as level codes [B][Hp][Wp][O] (nullable)
@@ -145,17 +145,6 @@ __device__ __forceinline__ void tma_load_4d(void *dst, const CUtensorMap *map, u
         : "memory");
 }
 
-// The same box delivered to every CTA of the cluster named in mask, at the
-// same shared-memory offset, completing bytes on each CTA's barrier there.
-__device__ __forceinline__ void tma_load_2d_mc(void *dst, const CUtensorMap *map, uint64_t *bar, int c0, int c1,
-                                               uint16_t mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
-        " [%0], [%1, {%2, %3}], [%4], %5;\n" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar)), "h"(mask)
-        : "memory");
-}
-
 __device__ __forceinline__ void cluster_sync_all() {
     asm volatile("barrier.cluster.arrive.release;\nbarrier.cluster.wait.acquire;\n" ::: "memory");
 }
@@ -193,38 +182,37 @@ __device__ __forceinline__ float code_units(uint32_t c) {
     return (c & 0x80u) ? -m : m;
 }
 
+// MMA issue.  The whole issuing warp executes these wrappers with warp-uniform
+// operands and one lane, chosen by elect.sync, issues the instruction: the
+// descriptors then stay in uniform registers.  Issued from a single divergent
+// thread instead, each tcgen05.mma costs that thread about 108 cycles (M = 128,
+// N <= 128) and a commit every four MMAs about 40 more; warp-uniform issue
+// runs at the tensor pipe's rate (64 cycles at N = 128, 128 at N = 256, with
+// the commit hidden).  The elected lane is the same for every call of a
+// converged warp, so its commits track the MMAs it issued.
+#define MINW_ELECT_PROLOGUE "{\n .reg .pred p, e;\n .reg .b32 r;\n setp.ne.b32 p, %4, 0;\n elect.sync r|e, 0xffffffff;\n"
+
 __device__ __forceinline__ void mma_f8(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                        uint32_t accumulate) {
-    asm volatile(
-        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
+    asm volatile(MINW_ELECT_PROLOGUE
+                 " @e tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+                 "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
 }
 
 __device__ __forceinline__ void mma_commit(uint64_t *bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(
+    asm volatile("{\n .reg .pred e;\n .reg .b32 r;\n elect.sync r|e, 0xffffffff;\n"
+                 " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}\n" ::"r"(
                      smem_u32(bar))
                  : "memory");
-}
-
-// Arrive on the barrier at this offset in every CTA of mask once the MMAs
-// issued so far have completed.
-__device__ __forceinline__ void mma_commit_mc(uint64_t *bar, uint16_t mask) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n" ::"r"(
-            smem_u32(bar)),
-        "h"(mask)
-        : "memory");
 }
 
 // bf16 x bf16 -> fp32 (weight-only quantized layers: full-precision bf16
 // activations, weights at their exact level values).
 __device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                          uint32_t accumulate) {
-    asm volatile(
-        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
+    asm volatile(MINW_ELECT_PROLOGUE
+                 " @e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+                 "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
 }
 
 // CTA pairs (cta_group::2).  The even CTA of a cluster of two issues each MMA
@@ -233,28 +221,25 @@ __device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64
 // CTA's tensor memory.  Loads of both CTAs complete on the even CTA's barrier.
 __device__ __forceinline__ void mma_f8_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                             uint32_t accumulate) {
-    asm volatile(
-        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
+    asm volatile(MINW_ELECT_PROLOGUE
+                 " @e tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+                 "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
 }
 
 __device__ __forceinline__ void mma_bf16_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                               uint32_t accumulate) {
-    asm volatile(
-        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
+    asm volatile(MINW_ELECT_PROLOGUE
+                 " @e tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+                 "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
 }
 
 // Arrive on the barrier at this offset in both CTAs of the pair once the
-// pair's MMAs issued so far have completed.
+// pair's MMAs issued so far have completed (an mbarrier signal to each CTA).
 __device__ __forceinline__ void mma_commit_pair(uint64_t *bar) {
-    asm volatile(
-        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n" ::"r"(
-            smem_u32(bar)),
-        "h"((uint16_t)3)
-        : "memory");
+    asm volatile("{\n .reg .pred e;\n .reg .b32 r;\n elect.sync r|e, 0xffffffff;\n"
+                 " @e tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n}\n"
+                 ::"r"(smem_u32(bar)), "h"((uint16_t)3)
+                 : "memory");
 }
 
 // Shared::cluster address of the object at this offset in CTA 0 of the cluster.
@@ -627,13 +612,12 @@ __global__ void __launch_bounds__(NT, 1)
     const int tiles_m = p.tiles_mp;
     const int tiles = tiles_m * p.ntn;
     const int items = tiles * p.ksplit;       // (output tile, K slice) work items
-    const uint16_t cmask = (uint16_t)((1u << p.cl) - 1u);
-    const int crank = p.cl > 1 ? (int)cluster_ctarank() : 0;
+    const int crank = PAIR ? (int)cluster_ctarank() : 0;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < p.S; ++s) {
             mbar_init(&full[s], 2);               // one arrival per TMA issuing warp (pairs: CTA 0's)
-            mbar_init(&empty[s], PAIR ? 1 : p.cl);   // one release per CTA reading the weight box
+            mbar_init(&empty[s], 1);              // one release per slot (pairs: CTA 0 commits to both CTAs)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
@@ -701,7 +685,7 @@ __global__ void __launch_bounds__(NT, 1)
     }
     fence_before();
     __syncthreads();
-    if (p.cl > 1) cluster_sync_all();         // every barrier of the cluster is initialised
+    if constexpr (PAIR) cluster_sync_all();   // every barrier of the pair is initialised
     fence_after();
     const uint32_t tmem_base = *tmem_slot;
     pdl_trigger();                            // set-up done: the next kernel may start its own
@@ -714,7 +698,7 @@ __global__ void __launch_bounds__(NT, 1)
             const CUtensorMap *map = act ? &tmA : &tmB;
             asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
             const uint32_t bytes = act ? p.a_bytes : p.b_bytes;   // per K block; weights: all cl slices
-            const int bslice = p.BN / p.cl;        // weight rows this CTA loads (and multicasts)
+            const int bslice = PAIR ? p.BN / 2 : p.BN;   // weight rows this CTA loads
             // pairs: this operand's loads of both CTAs complete on CTA 0's barrier, whose
             // producers alone arrive (expecting both CTAs' bytes)
             const bool arrive = !PAIR || crank == 0;
@@ -747,14 +731,11 @@ __global__ void __launch_bounds__(NT, 1)
                                                  kcol, o0 + crank * bslice);
                         } else if (act)
                             tma_load_4d(sa + (size_t)j * p.a_bytes, &tmA, &full[s], c0, x0 + kx, y0 + ky, b0);
-                        else if (p.cl == 1) {
+                        else {
                             uint8_t *sb = sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes;
                             tma_load_2d(sb, &tmB, &full[s], kcol, o0);
                             if (p.dup) tma_load_2d(sb + (size_t)64 * p.cb, &tmB, &full[s], kcol, o0);
-                        } else
-                            tma_load_2d_mc(sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes +
-                                               (size_t)crank * bslice * p.cb,
-                                           &tmB, &full[s], kcol, o0 + crank * bslice, cmask);
+                        }
                         kcol += p.ck;
                         c0 += p.ck;
                         if (c0 == p.C) {
@@ -770,22 +751,17 @@ __global__ void __launch_bounds__(NT, 1)
             for (int j = g > p.S ? g - p.S : 0; j < g; ++j)
                 if (!(PAIR ? mbar_wait(&empty[j % p.S], (j / p.S) & 1) : mbar_wait(&full[j % p.S], (j / p.S) & 1)))
                     break;
-            // clusters: every CTA's release of every slot has arrived here too
-            // (no remote arrival may reach this shared memory after exit)
-            if (p.cl > 1 && !act && !PAIR)
-                for (int j = g > p.S ? g - p.S : 0; j < g; ++j)
-                    if (!mbar_wait(&empty[j % p.S], (j / p.S) & 1)) break;
         }
     } else if (warp == 1) {
-        if (lane == 0 && (!PAIR || crank == 0)) {
+        if (!PAIR || crank == 0) {
             // ---------------- MMA issuer (pairs: CTA 0 issues for both) ----------------
+            // The whole warp runs this loop with warp-uniform values; one elected
+            // lane issues each MMA and commit (see mma_f8).  Every wait's outcome
+            // is made warp-uniform, so the warp stays converged.
             int s = 0, i = 0;
             uint32_t fphase = 0;
             bool alive = true;
-            // One thread issues every MMA, and each tcgen05.mma costs it on the
-            // order of a hundred cycles to issue: the loop keeps its own work per
-            // stage minimal (descriptors advance by a constant per ring slot,
-            // the K = 32 steps are unrolled).
+            // descriptors advance by a constant per ring slot, the K = 32 steps are unrolled
             const uint32_t sbase = smem_u32(smem);
             const uint64_t adesc0 = sw_desc(sbase, p.cb), bdesc0 = sw_desc(sbase + p.kps * p.a_bytes, p.cb);
             const uint32_t dstep = p.stage_bytes >> 4;     // start-address step of one ring slot
@@ -796,8 +772,8 @@ __global__ void __launch_bounds__(NT, 1)
                 const int ab = i & 1, use = i >> 1;
                 const int t = w / p.ksplit, kp = w - t * p.ksplit;
                 const int kb = (int)((long long)kp * p.nk / p.ksplit), ke = (int)((long long)(kp + 1) * p.nk / p.ksplit);
-                if (use > 0 && !(PAIR ? mbar_wait_cluster(&tempty[ab], (use - 1) & 1)
-                                        : mbar_wait(&tempty[ab], (use - 1) & 1)))
+                if (use > 0 && !__all_sync(0xffffffffu, PAIR ? mbar_wait_cluster(&tempty[ab], (use - 1) & 1)
+                                                             : mbar_wait(&tempty[ab], (use - 1) & 1)))
                     break;
                 fence_after();
                 const uint32_t tmem_d = tmem_base + (uint32_t)(ab * p.acc_cols);
@@ -813,7 +789,7 @@ __global__ void __launch_bounds__(NT, 1)
                         mma_f8(tmem_d, ad_, bd_, idesc, a_);
                 };
                 for (int ks = kb; ks < ke; ks += p.kps) {
-                    if (!mbar_wait(&full[s], fphase)) { alive = false; break; }
+                    if (!__all_sync(0xffffffffu, mbar_wait(&full[s], fphase))) { alive = false; break; }
                     fence_after();
                     const uint64_t off = (uint64_t)((uint32_t)s * dstep);
                     uint64_t ad = adesc0 + off, bd = bdesc0 + off;
@@ -842,10 +818,8 @@ __global__ void __launch_bounds__(NT, 1)
                     acc = 1u;
                     if constexpr (PAIR)
                         mma_commit_pair(&empty[s]);              // both CTAs' slots are free
-                    else if (p.cl == 1)
-                        mma_commit(&empty[s]);
                     else
-                        mma_commit_mc(&empty[s], cmask);     // the slot is free in every CTA's view
+                        mma_commit(&empty[s]);
                     if (++s == p.S) { s = 0; fphase ^= 1; }
                 }
                 if constexpr (PAIR)
@@ -1260,7 +1234,6 @@ __global__ void __launch_bounds__(NT, 1)
             fence_after();
             asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(p.tmem_cols));
         }
-        if (p.cl > 1) cluster_sync_all();         // no CTA leaves while a peer may still address it
     }
 }
 
@@ -1469,19 +1442,6 @@ static int chunk_channels(const ConvArgs &a) { return a.bf16 ? 64 : ((a.C % 128 
 static size_t slice_bytes(int tiles, int BN) { return (size_t)tiles * 128 * BN * sizeof(int32_t); }
 static size_t thr_ws_bytes(int O, int nlev) { return (((size_t)O * nlev * sizeof(float)) + 255) & ~(size_t)255; }
 
-// CTAs per cluster sharing each weight box (MINW_TC_CLUSTER = 1, 2 or 4;
-// 1 by default: the kernel is bound by MMA issue, not by the L2 -> shared
-// memory feed, and clusters of 2 or 4 measured 1-2 % slower on GB300).
-static int cluster_pref() {
-    static int v = -1;
-    if (v < 0) {
-        const char *e = getenv("MINW_TC_CLUSTER");
-        const int x = e ? atoi(e) : 1;
-        v = (x == 1 || x == 2 || x == 4) ? x : 1;
-    }
-    return v;
-}
-
 // Channel-major 64-channel tiles with the weight rows loaded twice (MINW_TC_DUP
 // = 0 pads with zero rows instead): the epilogue of a tile then spreads over
 // all eight epilogue warps, two 32-pixel chunks each instead of four.
@@ -1556,7 +1516,7 @@ static bool trans_eligible(const ConvArgs &a) {
             ((a.O == 128 || (a.O == 64 && dup_pref())) && !a.pool));   // residual: all 8 warps hold channels
 }
 
-static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_pref()) {
+static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     Params &p = pl.p;
     p = Params{};
     p.trans = 0;
@@ -1660,17 +1620,10 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, int cl_max = cluster_p
             p.part = reinterpret_cast<int32_t *>(w + tb);
         }
     }
-    // clusters sharing each weight box (multicast): cl CTAs walk pixel tiles
-    // of one channel tile together; each loads BN / cl weight rows for all
-    // (padding the pixel tiles to a multiple of cl may add at most 1/8)
     p.rowst = (p.ystage > 0 && (p.ksplit > 1 || rowst_fc)) ? 1 : 0;
     const int tiles_m = p.nbx * p.nby * p.nbb;
+    // CTA pairs walk pixel tiles two by two (an odd count gets one padded tile)
     p.cl = p.pair ? 2 : 1;
-    if (p.ksplit == 1 && !p.trans && !p.pair) {
-        int cl = cl_max;
-        while (cl > 1 && (p.BN % (8 * cl) != 0 || ((tiles_m + cl - 1) / cl * cl - tiles_m) * 8 > tiles_m)) cl >>= 1;
-        p.cl = cl;
-    }
     p.tiles_mp = (tiles_m + p.cl - 1) / p.cl * p.cl;
     minw_host::EncodeTiledFn enc = minw_host::tensor_map_encoder();
     if (enc == nullptr) return MINW_ECUDA;

@@ -283,34 +283,3 @@ def test_residual_block_epilogue(dev, M, shortcut, bits):
     assert np.array_equal(y.cpu().numpy(), yr)
     lv = O.quantize(yr, bits, DEFAULT_THR[bits])
     assert np.array_equal(decode_e4m3(codes.cpu().numpy()), (lv * 2.0 ** O.units_shift(bits)).transpose(0, 2, 3, 1))
-
-
-@pytest.mark.parametrize("cl", [2, 4])
-def test_weight_multicast_clusters(dev, cl):
-    """Clusters of 2 or 4 CTAs sharing each weight box by TMA multicast
-    (MINW_TC_CLUSTER, read once per process): the CIFAR-layer shapes still match
-    the oracle bit for bit.  Batch 26 leaves 13 pixel tiles in the 8x8 layers,
-    so one cluster also walks a padding tile.  Runs in a child process with the
-    variable set (and CTA pairs off, which would take the 256-channel layers)."""
-    import subprocess
-    import sys
-    code = (
-        "import numpy as np, torch\n"
-        "from oracle import network as N\n"
-        "from paper_2003_04296_gb300 import minw\n"
-        "from paper_2003_04296_gb300.inputs import convnet_input, convnet_params\n"
-        "dev = torch.device('cuda:0')\n"
-        "p = convnet_params(91, widths=(128, 128, 256, 256), pools=(False, True, False, True), fcs=(256,), hw=16)\n"
-        "x = convnet_input(92, 26, hw=16)\n"
-        "net = minw.Net(minw.layer_descs(p, dev), max_batch=26)\n"
-        "out = torch.empty((26, net.out_features), dtype=torch.float32, device=dev)\n"
-        "net.forward(torch.from_numpy(x).to(dev), out)\n"
-        "torch.cuda.synchronize()\n"
-        "assert minw.minw_get_last_device_error() == minw.MINW_OK\n"
-        "assert np.array_equal(out.cpu().numpy(), N.convnet_forward(p, x))\n"
-        "print('ok')\n")
-    import os
-    env = dict(os.environ, MINW_TC_CLUSTER=str(cl), MINW_TC_PAIR="0")
-    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-    r = subprocess.run([sys.executable, "-c", code], cwd=root, env=env, capture_output=True, text=True, timeout=600)
-    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stderr[-2000:]
