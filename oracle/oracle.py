@@ -222,28 +222,38 @@ def bf16_round_scalar(v):
     return float(lib().orc_bf16_round(float(v)))
 
 
-def fc_train_step(A, W, G, alpha, lr, bits_w, thr_w, q_a=None):
+def fc_train_step(A, W, G, alpha, lr, bits_w, thr_w, q_a=None, a_pre=None):
     """One step of Algorithm 1 on a fully connected layer with input A [B][K],
     latent weights W [O][K] and upstream gradient G [B][O], in the order of
-    Algorithm 1: the weight AQE (Eq. weight, fp32), the forward product a~ of
-    the bf16 operands (fp64 sums, rounded to fp32), the activation AQE and its
-    backward mask (Eq. activation; skipped for the last layer, q_a None), the
-    input gradient g_in = bf16(g~) bf16(W^) and the weight gradient
-    g_W^ = bf16(g~)^T bf16(A) (fp64 sums, rounded to fp32), then the mask of
-    Eq. weight and the clipped update.  q_a = (bits, thr).  Returns
-    (a_out, g_in, W_new, a_pre) as fp32 arrays."""
+    Algorithm 1 and at its precision (Sec. III-C: the weights and activations
+    entering the loss are full precision): the weight AQE W^ (Eq. weight,
+    fp32), the forward product a~ = A W^T (fp64 sums of the fp32 operands,
+    rounded to fp32), the activation AQE and its backward mask g~ (Eq.
+    activation; skipped for the last layer, q_a None), the input gradient
+    g_in = g~ W^ and the weight gradient g_W^ = g~^T A (fp64 sums of the fp32
+    operands, rounded to fp32), then the mask of Eq. weight and the clipped
+    update.  q_a = (bits, thr).
+
+    a_pre, when given, replaces the forward product a~ for the rest of the
+    step (a stage-wise check: the later stages of the oracle applied to the
+    forward product another implementation computed).
+
+    Returns (a_out, g_in, W_new, a_pre) as fp32 arrays."""
     A, W, G = _f32(A), _f32(W), _f32(G)
-    what = aqe_forward_f32(W, alpha, bits_w, thr_w)
-    Wq, Aq = bf16_round(what).astype(np.float64), bf16_round(A).astype(np.float64)
-    a_pre = (Aq @ Wq.T).astype(np.float32)
+    what = aqe_forward_f32(W, alpha, bits_w, thr_w).astype(np.float64)
+    A64 = A.astype(np.float64)
+    if a_pre is None:
+        a_pre = (A64 @ what.T).astype(np.float32)
+    else:
+        a_pre = _f32(a_pre)
     if q_a is None:
         a_out, g_t = a_pre, G
     else:
         a_out = aqe_forward_f32(a_pre, alpha, q_a[0], q_a[1])
         g_t = aqe_backward_f32(a_pre, G, alpha)
-    Gq = bf16_round(g_t).astype(np.float64)
-    g_in = (Gq @ Wq).astype(np.float32)
-    g_w = (Gq.T @ Aq).astype(np.float32)
+    g64 = g_t.astype(np.float64)
+    g_in = (g64 @ what).astype(np.float32)
+    g_w = (g64.T @ A64).astype(np.float32)
     W_new = sgd_clip(W, aqe_backward_f32(W, g_w, alpha), lr)
     return a_out, g_in, W_new, a_pre
 
@@ -289,27 +299,31 @@ def conv2d_weight_grad(g, a, kh, kw, stride, pad):
     return gw
 
 
-def conv_train_step(A, W, G, alpha, lr, bits_w, thr_w, stride, pad, q_a=None):
-    """Algorithm 1 on a convolutional layer, in the order of fc_train_step:
-    weight AQE (fp32), the forward convolution of the bf16 operands (fp64 sums
-    rounded to fp32), the activation AQE and its mask (q_a = (bits, thr); None
-    for a layer without an activation quantizer), the input and weight
-    gradients of the bf16 operands (fp64 sums rounded to fp32), then the mask
-    of Eq. weight and the clipped update.  A [B][C][H][W], W [O][C][kh][kw],
-    G [B][O][Ho][Wo].  Returns (a_out, g_in, W_new, a_pre)."""
+def conv_train_step(A, W, G, alpha, lr, bits_w, thr_w, stride, pad, q_a=None, a_pre=None):
+    """Algorithm 1 on a convolutional layer, in the order and at the precision
+    of fc_train_step: the weight AQE (fp32), the forward convolution of the
+    fp32 operands (fp64 sums rounded to fp32), the activation AQE and its mask
+    (q_a = (bits, thr); None for a layer without an activation quantizer), the
+    input and weight gradients of the fp32 operands (fp64 sums rounded to
+    fp32), then the mask of Eq. weight and the clipped update.  A [B][C][H][W],
+    W [O][C][kh][kw], G [B][O][Ho][Wo]; a_pre as in fc_train_step.  Returns
+    (a_out, g_in, W_new, a_pre)."""
     A, W, G = _f32(A), _f32(W), _f32(G)
-    what = aqe_forward_f32(W, alpha, bits_w, thr_w)
-    Wq, Aq = bf16_round(what).astype(np.float64), bf16_round(A).astype(np.float64)
-    a_pre = conv2d_real(Aq, Wq, stride, pad).astype(np.float32)
+    what = aqe_forward_f32(W, alpha, bits_w, thr_w).astype(np.float64)
+    A64 = A.astype(np.float64)
+    if a_pre is None:
+        a_pre = conv2d_real(A64, what, stride, pad).astype(np.float32)
+    else:
+        a_pre = _f32(a_pre)
     if q_a is None:
         a_out, g_t = a_pre, G
     else:
         a_out = aqe_forward_f32(a_pre, alpha, q_a[0], q_a[1])
         g_t = aqe_backward_f32(a_pre, G, alpha)
-    Gq = bf16_round(g_t).astype(np.float64)
+    g64 = g_t.astype(np.float64)
     H, Wd = A.shape[2], A.shape[3]
-    g_in = conv2d_input_grad(Gq, Wq, stride, pad, H, Wd).astype(np.float32)
-    g_w = conv2d_weight_grad(Gq, Aq, W.shape[2], W.shape[3], stride, pad).astype(np.float32)
+    g_in = conv2d_input_grad(g64, what, stride, pad, H, Wd).astype(np.float32)
+    g_w = conv2d_weight_grad(g64, A64, W.shape[2], W.shape[3], stride, pad).astype(np.float32)
     W_new = sgd_clip(W, aqe_backward_f32(W, g_w, alpha), lr)
     return a_out, g_in, W_new, a_pre
 

@@ -1,12 +1,25 @@
 """GPU parity of Algorithm 1's training step on a fully connected layer,
-through the C ABI.  Stage by stage, each GPU stage is checked against the
-oracle fed with the GPU's own inputs to that stage: the weight AQE forward
-and the activation AQE, the backward masks and the update bit for bit (one
-fp32 operation each), the bf16 operands bit for bit, and the three tensor-core
-products (forward, input gradient, weight gradient) within the bound of fp32
-accumulation, |err| <= K 2^-23 (|P| |Q|) for a product P Q with K terms.  Then
-minw_fc_train_step, whose fused passes and K-split products are checked
-against the oracle the same way."""
+through the C ABI.
+
+The building blocks are checked stage by stage against the oracle fed with
+the GPU's own inputs to each stage: the weight AQE forward and the activation
+AQE, the backward masks and the update bit for bit (one fp32 operation each),
+the bf16 conversions bit for bit, and the tensor-core products of given bf16
+operands within the bound of fp32 accumulation, K 2^-23 (|P| |Q|) for a
+product P Q with K terms.
+
+minw_fc_train_step is then checked against the oracle's step at the paper's
+precision (fp32 operands, fp64 sums).  The GPU forms its three products from
+bf16 roundings of the fp32 operands, so each product P Q differs from the
+exact one by at most
+
+    (2^-7 + 2^-16 + K 2^-23 (1 + 2^-8)^2) (|P| |Q|) + 2^-24 |P Q|
+
+(two operand roundings of relative size 2^-8 each, the fp32 accumulation, and
+the oracle's own rounding to fp32).  The stages after the forward product are
+compared with the oracle fed the GPU's forward product (its a_pre argument):
+a_out bit for bit, g_in within the bound, the updated weights within lr 2 alpha
+times the weight gradient's bound plus one fp32 ulp."""
 import numpy as np
 import pytest
 
@@ -114,23 +127,36 @@ def test_train_stages(dev, M, case):
     assert np.array_equal(Wn.cpu().numpy(), O.sgd_clip(W, gw_np, 0.05))
 
 
+def _step_bound(P, Q):
+    """Bound of a bf16-operand tensor-core product against the exact product
+    of the fp32 operands P [m][K] and Q [K][n] (the module docstring)."""
+    P64, Q64 = P.astype(np.float64), Q.astype(np.float64)
+    K = P.shape[1]
+    mag = np.abs(P64) @ np.abs(Q64)
+    return (2.0 ** -7 + 2.0 ** -16 + K * 2.0 ** -23 * (1 + 2.0 ** -8) ** 2) * mag + 2.0 ** -24 * np.abs(P64 @ Q64) + 1e-30
+
+
+def _within(got, ref, bound, what):
+    err = np.abs(got.astype(np.float64) - ref.astype(np.float64))
+    assert (err <= bound).all(), f"{what}: worst err/bound {np.max(err / bound)}"
+
+
 @pytest.mark.parametrize("case", CASES + [(256, 8192, 1024, 0.75, 1, 1)])
 @pytest.mark.parametrize("last", [False, True])
 def test_train_step(dev, M, case, last):
-    """minw_fc_train_step against the oracle.  Its operands are the bf16 of the
-    oracle's fp32 weight AQE and of the input; a~ (a_pre, or a_out for the last
-    layer) lies within the fp32 accumulation bound of Aq Wq^T; a_out and the
-    mask of Eq. activation equal the oracle's applied to that a~ bit for bit;
-    g_in lies within the bound of Gq Wq; the updated W within lr 2 alpha times
-    the weight gradient's bound (plus the half ulp of one fmaf) of the update
-    from the exact gradient.  (256, 8192, 1024) is fc1 of the CIFAR model at
-    the training bench's batch, whose forward product splits along K.  A second
-    step from the same inputs gives the same bits (the K slices add in a fixed
-    order)."""
+    """minw_fc_train_step against the oracle's Algorithm 1 step at the paper's
+    precision.  a~ (a_pre, or a_out for the last layer) lies within the
+    bf16-operand bound of the oracle's a~; with the GPU's a~ substituted, a_out
+    equals the oracle's bit for bit, g_in lies within the bound of g~ W^, and
+    the updated W within lr 2 alpha times the bound of g~^T A plus one fp32 ulp.
+    (256, 8192, 1024) is fc1 of the CIFAR model at the training bench's batch,
+    whose forward product splits along K.  A second step from the same inputs
+    gives the same bits (the K slices add in a fixed order)."""
     B, K, O_, alpha, bw, ba = case
     lr = 0.05
     A, W, G = _problem(7 + sum(case[:3]), B, K, O_)
     qw, qa = M.quant(bw, DEFAULT_THR[bw]), (None if last else M.quant(ba, DEFAULT_THR[ba]))
+    q_a = None if last else (ba, DEFAULT_THR[ba])
     At, Gt = dev_tensor(A, dev), dev_tensor(G, dev)
     ws = torch.empty(M.minw_fc_train_workspace_bytes(B, K, O_), dtype=torch.uint8, device=dev)
     outs = []
@@ -144,23 +170,20 @@ def test_train_step(dev, M, case, last):
     W1, a1, g1, pre = outs[0]
     for x, y in zip(outs[0], outs[1][:3]):
         assert np.array_equal(x, y)
-    Wq = O.bf16_round(O.aqe_forward_f32(W, alpha, bw, DEFAULT_THR[bw]))
-    Aq = O.bf16_round(A)
     at = a1 if last else pre
-    _check_product(at, Aq, Wq.T)
-    if last:
-        gat = G
-    else:
-        assert np.array_equal(a1, O.aqe_forward_f32(at, alpha, ba, DEFAULT_THR[ba]))
-        gat = O.aqe_backward_f32(at, G, alpha)
-    Gq = O.bf16_round(gat)
-    _check_product(g1, Gq, Wq)
-    gref = Gq.T.astype(np.float64) @ Aq.astype(np.float64)
-    gbound = B * 2.0 ** -23 * (np.abs(Gq.T).astype(np.float64) @ np.abs(Aq).astype(np.float64))
-    mask = np.abs(W) <= 1.0
-    Wref = np.clip(W.astype(np.float64) - lr * 2 * alpha * np.where(mask, gref, 0.0), -1.0, 1.0)
-    tol = lr * 2 * alpha * gbound + 2.0 ** -24
-    assert (np.abs(W1.astype(np.float64) - Wref) <= tol).all()
+    # the forward product against the paper-precision oracle's
+    what = O.aqe_forward_f32(W, alpha, bw, DEFAULT_THR[bw])
+    ref = O.fc_train_step(A, W, G, alpha, lr, bw, DEFAULT_THR[bw], q_a)
+    _within(at, ref[3], _step_bound(A, what.T), "a~")
+    # the later stages with the GPU's a~ substituted
+    a_ref, gin_ref, W_ref, _ = O.fc_train_step(A, W, G, alpha, lr, bw, DEFAULT_THR[bw], q_a, a_pre=at)
+    if not last:
+        assert np.array_equal(a1, a_ref)
+    gat = G if last else O.aqe_backward_f32(at, G, alpha)
+    _within(g1, gin_ref, _step_bound(gat, what), "g_in")
+    gb = _step_bound(gat.T, A)
+    gw_ref = gat.T.astype(np.float64) @ A.astype(np.float64)
+    _within(W1, W_ref, lr * 2 * alpha * (gb + 2.0 ** -24 * np.abs(gw_ref)) + 2.0 ** -23, "W")
     assert np.abs(W1).max() <= 1.0
 
 

@@ -85,11 +85,13 @@ def _bf16_torch(x):
 
 @pytest.mark.parametrize("last", [False, True])
 def test_fc_train_step_wiring(last):
-    """The composed step against properties it must have: a_pre is the fp32
-    rounding of the exact (rational) product of the bf16 operands; g_in and
-    the weight step are the gradients of sum(g~ * a~) with respect to the
-    bf16 input and weights (central differences in fp64), so a transposed or
-    swapped operand fails; the last layer passes g through unmasked."""
+    """The composed step against properties it must have, at the paper's
+    precision (fp32 operands): a_pre is the fp32 rounding of the exact
+    (rational) product of the fp32 input and the fp32 weight AQE; g_in and the
+    weight step are the gradients of sum(g~ * a~) with respect to the input
+    and the weights (central differences in fp64), so a transposed or swapped
+    operand fails; the last layer passes g through unmasked; a given a_pre
+    replaces the forward product for every later stage."""
     r = np.random.default_rng(11)
     B, K, O_ = 3, 8, 4
     A = np.clip(r.standard_normal((B, K)), -1.5, 1.5).astype(np.float32)
@@ -98,11 +100,10 @@ def test_fc_train_step_wiring(last):
     alpha, lr = 0.6, 0.125
     q_a = None if last else (2, DEFAULT_THR[2])
     a_out, g_in, W_new, a_pre = O.fc_train_step(A, W, G, alpha, lr, 1, DEFAULT_THR[1], q_a)
-    Wq = _bf16_torch(O.aqe_forward_f32(W, alpha, 1, DEFAULT_THR[1]))
-    Aq = _bf16_torch(A)
+    Wh = O.aqe_forward_f32(W, alpha, 1, DEFAULT_THR[1])
     for i in range(B):
         for o in range(O_):
-            exact = sum(Fraction(float(Aq[i, k])) * Fraction(float(Wq[o, k])) for k in range(K))
+            exact = sum(Fraction(float(A[i, k])) * Fraction(float(Wh[o, k])) for k in range(K))
             assert a_pre[i, o] == np.float32(float(exact))
     if last:
         assert np.array_equal(a_out, a_pre)
@@ -110,10 +111,10 @@ def test_fc_train_step_wiring(last):
     else:
         assert np.array_equal(a_out, O.aqe_forward_f32(a_pre, alpha, 2, DEFAULT_THR[2]))
         gt = O.aqe_backward_f32(a_pre, G, alpha)
-    Gq = _bf16_torch(gt).astype(np.float64)
-    L = lambda A_, W_: np.sum(Gq * (A_ @ W_.T))
+    g64 = gt.astype(np.float64)
+    L = lambda A_, W_: np.sum(g64 * (A_ @ W_.T))
     h = 1e-3
-    A64, W64 = Aq.astype(np.float64), Wq.astype(np.float64)
+    A64, W64 = A.astype(np.float64), Wh.astype(np.float64)
     for i in range(B):
         for k in range(K):
             E = np.zeros_like(A64); E[i, k] = h
@@ -125,6 +126,27 @@ def test_fc_train_step_wiring(last):
             d = (L(A64, W64 + E) - L(A64, W64 - E)) / (2 * h)
             want = np.clip(W[o, k] - lr * 2 * alpha * d, -1.0, 1.0)     # |W| <= 1: the mask passes
             assert abs(W_new[o, k] - want) <= 1e-6
+    # a substituted forward product drives the later stages
+    sub = (a_pre + np.float32(0.25)).astype(np.float32)
+    a2, g2, W2, p2 = O.fc_train_step(A, W, G, alpha, lr, 1, DEFAULT_THR[1], q_a, a_pre=sub)
+    assert np.array_equal(p2, sub)
+    if not last:
+        assert np.array_equal(a2, O.aqe_forward_f32(sub, alpha, 2, DEFAULT_THR[2]))
+        g2t = O.aqe_backward_f32(sub, G, alpha).astype(np.float64)
+        assert np.allclose(g2, g2t @ W64, rtol=2.0 ** -22, atol=1e-30)
+
+
+def test_fc_train_step_full_precision():
+    """The step keeps full precision: weights and inputs that bf16 cannot
+    represent (1 + 2^-12, 1 + 2^-20) give the fp32 rounding of the exact
+    product, not of a product of rounded operands."""
+    A = np.full((1, 64), 1.0 + 2.0 ** -12, dtype=np.float32)
+    W = np.full((2, 64), 0.5 + 2.0 ** -20, dtype=np.float32)
+    G = np.ones((1, 2), dtype=np.float32)
+    a_out, g_in, W_new, a_pre = O.fc_train_step(A, W, G, 0.0, 0.0, 1, DEFAULT_THR[1], None)
+    exact = 64 * Fraction(float(A[0, 0])) * Fraction(float(W[0, 0]))
+    assert a_pre[0, 0] == np.float32(float(exact)) and a_pre[0, 0] != np.float32(32.0)
+    assert g_in[0, 0] == np.float32(float(2 * Fraction(float(W[0, 0]))))
 
 
 def test_fc_train_step_alpha_zero():
@@ -187,10 +209,11 @@ def test_conv_train_step_reduces_to_fc():
 
 
 def test_conv_train_step_gradients():
-    """The convolutional step's input gradient and weight step are the
-    gradients of sum(g~ * a~) with respect to the bf16 operands (torch autograd
-    in float64 on torch-rounded bf16 operands), with the mask of Eq. weight
-    and the clip on the latent weights."""
+    """The convolutional step's forward product, input gradient and weight
+    step are those of the fp32 operands at full precision: torch autograd of
+    conv2d in float64 (an independent implementation) on the fp32 input and
+    weight AQE, with the mask of Eq. weight and the clip on the latent
+    weights."""
     torch = pytest.importorskip("torch")
     r = np.random.default_rng(14)
     A = np.clip(r.standard_normal((2, 4, 6, 6)), -1.5, 1.5).astype(np.float32)
@@ -198,12 +221,11 @@ def test_conv_train_step_gradients():
     G = (r.standard_normal((2, 3, 3, 3)) * 0.5).astype(np.float32)
     alpha, lr = 0.5, 0.125
     a_out, g_in, W_new, a_pre = O.conv_train_step(A, W, G, alpha, lr, 2, DEFAULT_THR[2], 2, 1, (1, DEFAULT_THR[1]))
-    Wq = torch.tensor(_bf16_torch(O.aqe_forward_f32(W, alpha, 2, DEFAULT_THR[2])).astype(np.float64),
-                      requires_grad=True)
-    Aq = torch.tensor(_bf16_torch(A).astype(np.float64), requires_grad=True)
+    Wq = torch.tensor(O.aqe_forward_f32(W, alpha, 2, DEFAULT_THR[2]).astype(np.float64), requires_grad=True)
+    Aq = torch.tensor(A.astype(np.float64), requires_grad=True)
     y = torch.nn.functional.conv2d(Aq, Wq, stride=2, padding=1)
     assert np.allclose(a_pre, y.detach().numpy(), rtol=2.0 ** -23, atol=1e-30)
-    gt = _bf16_torch(O.aqe_backward_f32(a_pre, G, alpha)).astype(np.float64)
+    gt = O.aqe_backward_f32(a_pre, G, alpha).astype(np.float64)
     (y * torch.tensor(gt)).sum().backward()
     assert np.allclose(g_in, Aq.grad.numpy(), rtol=2.0 ** -23, atol=1e-30)
     gw = Wq.grad.numpy()
