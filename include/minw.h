@@ -145,7 +145,10 @@ MINW_API minw_status minw_pack_weights(const float *w, int32_t O, int32_t C, int
 enum {
     MINW_VARIANT_AUTO = 0,    /* per-shape choice from measurements */
     MINW_VARIANT_POPC = 1,    /* bit-serial XNOR/AND + popcount on the integer pipe */
-    MINW_VARIANT_TC = 2       /* tcgen05 tensor cores on exact FP8 level values */
+    MINW_VARIANT_TC = 2,      /* tcgen05 tensor cores on exact level values: E2M1 operands where
+                                 the shape allows (C % 128 == 0), else E4M3 */
+    MINW_VARIANT_TC_E4M3 = 3, /* tensor cores on E4M3 operands only (a network request) */
+    MINW_VARIANT_TC_E2M1 = 4  /* reported for a network layer that runs on E2M1 operands */
 };
 
 /* Convolution of packed activations act [B][H][W][bits_a][C/32] with packed
@@ -207,6 +210,25 @@ MINW_API minw_status minw_pack_weight_codes(const float *w, int32_t O, int32_t C
                                             int32_t kw, const minw_quant *q,
                                             const float *channel_scale, uint8_t *codes,
                                             void *stream);
+
+/* "E2M1 codes" layout: the same levels as 4-bit FP4 E2M1 numbers, two
+ * channels per byte (channel 2j in the low nibble of byte j) -- 0 -> 0x0,
+ * +-1 -> 0x2/0xA, +-2 -> 0x4/0xC, +-4 -> 0x6/0xE.  Activations
+ * [N][H][W][C / 2] bytes, weights [O][kh][kw][C / 2].  The products are as
+ * exact as E4M3's; the tensor cores take them with unit block scales
+ * (tcgen05 kind::mxf4), at twice the K per instruction and half the bytes. */
+enum { MINW_CODES_E4M3 = 0, MINW_CODES_E2M1 = 1 };
+
+/* aqe_quantize_codes into E2M1 codes (C % 32 == 0). */
+MINW_API minw_status aqe_quantize_codes_e2m1(const float *x, int32_t B, int32_t C, int32_t H,
+                                             int32_t W, const minw_quant *q, uint8_t *codes,
+                                             void *stream);
+
+/* minw_pack_weight_codes into E2M1 codes [O][kh][kw][C / 2] (C % 16 == 0). */
+MINW_API minw_status minw_pack_weight_codes_e2m1(const float *w, int32_t O, int32_t C, int32_t kh,
+                                                 int32_t kw, const minw_quant *q,
+                                                 const float *channel_scale, uint8_t *codes,
+                                                 void *stream);
 
 /* minw_conv2d on codes operands, run on the tcgen05 tensor cores.
  * Supported: stride 1 or 2, C % 64 == 0, pad < kh, kw; otherwise
@@ -320,12 +342,22 @@ MINW_API minw_status minw_fc_train_step(const float *A, float *W, const float *g
  * res_f32 (nullable): shortcut as fp32 NHWC [B][Hp][Wp][O].
  * y_nhwc (nullable, output): the BN output before the shortcut, fp32 NHWC.
  * With a shortcut the block computes y = fmaf(acc, scale, shift) + shortcut
- * (one fp32 add), then HardTanh and the output quantizer. */
+ * (one fp32 add), then HardTanh and the output quantizer.
+ * in_format (MINW_CODES_E4M3 or MINW_CODES_E2M1): layout of act and wgt; E2M1
+ *   operands need C % 128 == 0 (else MINW_EUNSUPPORTED).
+ * out_format, res_format: layouts of codes_out and res_codes.
+ * acc_out (nullable, output): the exact int32 accumulators, NCHW, for a block
+ *   without pooling.
+ * A zero-initialised struct is the E4M3 block without extras. */
 typedef struct {
     const uint8_t *res_codes;
     int32_t res_bits;
     const float *res_f32;
     float *y_nhwc;
+    int32_t in_format;
+    int32_t out_format;
+    int32_t res_format;
+    int32_t *acc_out;
 } minw_block_extra;
 
 /* minw_conv_block_codes with the residual inputs / outputs of extra
@@ -456,7 +488,8 @@ MINW_API minw_status minw_net_enable_timing(minw_net *net, int32_t on);
 MINW_API minw_status minw_net_layer_times(minw_net *net, float *ms);
 
 /* Kernel chosen for each layer (host array of minw_net_launches() ints):
- * 0 for the fp32 first layer, else MINW_VARIANT_POPC or MINW_VARIANT_TC. */
+ * 0 for the fp32 first layer, else MINW_VARIANT_POPC, MINW_VARIANT_TC (E4M3
+ * operands) or MINW_VARIANT_TC_E2M1. */
 MINW_API minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants);
 
 /* ResNet-18-shaped MINW-Net (Table V's network).  The paper leaves the

@@ -327,9 +327,11 @@ __global__ void pack_weights_kernel(const float *__restrict__ w, int O, int C, i
 // Level codes: NCHW fp32 -> NHWC bytes (E4M3 levels), the tensor-core operand.
 // One warp owns 32 pixels x 32 channels of an image: lane l reads pixel p0+l of
 // each channel (coalesced along the row) and writes its 32 channel bytes with
-// two 16-byte stores.  C % 16 == 0.
+// two 16-byte stores.  C % 16 == 0.  With FP4 the codes are E2M1 nibbles, two
+// channels per byte (16 bytes per lane; C % 32 == 0).
 // ---------------------------------------------------------------------------
 
+template <bool FP4>
 __global__ void __launch_bounds__(256) quantize_codes_kernel(const float *__restrict__ x, int B, int C,
                                                              int HW, QParams q, uint8_t *__restrict__ codes) {
     const int groups = (C + 31) >> 5;
@@ -350,15 +352,29 @@ __global__ void __launch_bounds__(256) quantize_codes_kernel(const float *__rest
 #pragma unroll 8
         for (int c = 0; c < cmax; ++c) {
             const float v = __ldcs(x + ((int64_t)b * C + c0 + c) * HW + p);
-            w[c >> 2] |= (uint32_t)level_code_e4m3(level_units(v * q.scale, q)) << ((c & 3) * 8);
+            const int u = level_units(v * q.scale, q);
+            if (FP4)
+                w[c >> 3] |= level_code_e2m1(u) << ((c & 7) * 4);
+            else
+                w[c >> 2] |= (uint32_t)level_code_e4m3(u) << ((c & 3) * 8);
         }
-        uint4 *dst = reinterpret_cast<uint4 *>(codes + ((int64_t)b * HW + p) * C + c0);
-        dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
-        if (cmax > 16) dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+        if (FP4) {
+            uint8_t *dst = codes + ((((int64_t)b * HW + p) * C + c0) >> 1);
+            if (cmax > 16)
+                *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+            else
+                *reinterpret_cast<uint2 *>(dst) = make_uint2(w[0], w[1]);
+        } else {
+            uint4 *dst = reinterpret_cast<uint4 *>(codes + ((int64_t)b * HW + p) * C + c0);
+            dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+            if (cmax > 16) dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+        }
     }
 }
 
-// Weights [O][C][kh][kw] -> codes [O][kh][kw][C]: one thread per 16 channels.
+// Weights [O][C][kh][kw] -> codes [O][kh][kw][C]: one thread per 16 channels
+// (E4M3 bytes, or E2M1 nibbles with FP4).
+template <bool FP4>
 __global__ void weight_codes_kernel(const float *__restrict__ w, int O, int C, int kh, int kw, QParams q,
                                     const float *__restrict__ cscale, uint8_t *__restrict__ codes) {
     const int G = C >> 4;
@@ -373,10 +389,17 @@ __global__ void weight_codes_kernel(const float *__restrict__ w, int O, int C, i
         uint32_t wd[4] = {0u, 0u, 0u, 0u};
         for (int c = 0; c < 16; ++c) {
             const float v = w[((int64_t)o * C + g * 16 + c) * taps + tap];
-            wd[c >> 2] |= (uint32_t)level_code_e4m3(level_units(v * s, q)) << ((c & 3) * 8);
+            const int u = level_units(v * s, q);
+            if (FP4)
+                wd[c >> 3] |= level_code_e2m1(u) << ((c & 7) * 4);
+            else
+                wd[c >> 2] |= (uint32_t)level_code_e4m3(u) << ((c & 3) * 8);
         }
-        *reinterpret_cast<uint4 *>(codes + ((int64_t)o * taps + tap) * C + g * 16) =
-            make_uint4(wd[0], wd[1], wd[2], wd[3]);
+        if (FP4)
+            *reinterpret_cast<uint2 *>(codes + ((((int64_t)o * taps + tap) * C + g * 16) >> 1)) = make_uint2(wd[0], wd[1]);
+        else
+            *reinterpret_cast<uint4 *>(codes + ((int64_t)o * taps + tap) * C + g * 16) =
+                make_uint4(wd[0], wd[1], wd[2], wd[3]);
     }
 }
 
@@ -602,7 +625,19 @@ minw_status aqe_quantize_codes(const float *x, int32_t B, int32_t C, int32_t H, 
     if (HW > (1ll << 30)) return MINW_EUNSUPPORTED;
     const int64_t warps = (int64_t)B * ((C + 31) / 32) * ((HW + 31) / 32);
     const int64_t g = grid_for(warps * 32, 256);
-    quantize_codes_kernel<<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(x, B, C, (int)HW, to_qparams(q), codes);
+    quantize_codes_kernel<false><<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(x, B, C, (int)HW, to_qparams(q), codes);
+    return launch_status();
+}
+
+minw_status aqe_quantize_codes_e2m1(const float *x, int32_t B, int32_t C, int32_t H, int32_t W,
+                                    const minw_quant *q, uint8_t *codes, void *stream) {
+    if (B <= 0 || C <= 0 || H <= 0 || W <= 0 || !valid_quant(q) || !x || !codes) return MINW_EINVAL;
+    if (C % 32 != 0 || !aligned16(codes)) return MINW_EUNSUPPORTED;
+    const int64_t HW = (int64_t)H * W;
+    if (HW > (1ll << 30)) return MINW_EUNSUPPORTED;
+    const int64_t warps = (int64_t)B * ((C + 31) / 32) * ((HW + 31) / 32);
+    const int64_t g = grid_for(warps * 32, 256);
+    quantize_codes_kernel<true><<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(x, B, C, (int)HW, to_qparams(q), codes);
     return launch_status();
 }
 
@@ -613,8 +648,20 @@ minw_status minw_pack_weight_codes(const float *w, int32_t O, int32_t C, int32_t
     if (C % 16 != 0 || !aligned16(codes)) return MINW_EUNSUPPORTED;
     const int64_t items = (int64_t)O * kh * kw * (C / 16);
     const int64_t g = grid_for(items, 256);
-    weight_codes_kernel<<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(w, O, C, kh, kw, to_qparams(q),
-                                                                      channel_scale, codes);
+    weight_codes_kernel<false><<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(w, O, C, kh, kw, to_qparams(q),
+                                                                             channel_scale, codes);
+    return launch_status();
+}
+
+minw_status minw_pack_weight_codes_e2m1(const float *w, int32_t O, int32_t C, int32_t kh, int32_t kw,
+                                        const minw_quant *q, const float *channel_scale, uint8_t *codes,
+                                        void *stream) {
+    if (O <= 0 || C <= 0 || kh <= 0 || kw <= 0 || !valid_quant(q) || !w || !codes) return MINW_EINVAL;
+    if (C % 16 != 0 || !aligned16(codes)) return MINW_EUNSUPPORTED;
+    const int64_t items = (int64_t)O * kh * kw * (C / 16);
+    const int64_t g = grid_for(items, 256);
+    weight_codes_kernel<true><<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(w, O, C, kh, kw, to_qparams(q),
+                                                                            channel_scale, codes);
     return launch_status();
 }
 

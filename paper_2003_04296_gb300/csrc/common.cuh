@@ -73,6 +73,26 @@ __host__ __device__ __forceinline__ uint8_t level_code_e4m3(int v) {
     return (uint8_t)(((v < 0) ? 0x80u : 0u) | (e << 3));
 }
 
+// FP4 E2M1 encoding of a level in integer units (sign bit 3, exponent bits
+// 2-1 with bias 1, mantissa bit 0): 0 -> 0x0, +-1 -> 0x2/0xA, +-2 -> 0x4/0xC,
+// +-4 -> 0x6/0xE.  Every level is exact, so E2M1 products are exact too.  The
+// packed "E2M1 codes" layout holds two channels per byte, channel 2j in the
+// low nibble of byte j.
+__host__ __device__ __forceinline__ uint32_t level_code_e2m1(int v) {
+    if (v == 0) return 0u;
+    const int m = v < 0 ? -v : v;
+    const uint32_t c = (m == 4) ? 3u : (m == 2) ? 2u : 1u;
+    return ((v < 0) ? 8u : 0u) | (c << 1);
+}
+
+// Value in integer units of an E2M1 level code (low nibble of c).
+__host__ __device__ __forceinline__ float code_units_e2m1(uint32_t c) {
+    const uint32_t e = (c >> 1) & 3u;
+    if (e == 0u) return 0.0f;
+    const float m = (float)(1u << (e - 1u));
+    return (c & 8u) ? -m : m;
+}
+
 // ---------------------------------------------------------------------------
 // Output quantization as integer thresholds.
 //
@@ -221,12 +241,44 @@ __device__ __forceinline__ uint32_t level_code_word(const uint32_t *P, int g) {
     }
 }
 
+// Eight channels' bits (byte g of m) spread to the low bit of eight nibbles.
+__device__ __forceinline__ uint32_t spread8n(uint32_t m, int g) {
+    uint32_t x = (m >> (8 * g)) & 0xFFu;
+    x = (x | (x << 12)) & 0x000F000Fu;
+    x = (x | (x << 6)) & 0x03030303u;
+    x = (x | (x << 3)) & 0x11111111u;
+    return x;
+}
+
+// E2M1 codes of channels 8g .. 8g + 7 (one nibble each, channel 8g lowest)
+// from the planes: the nibble is sign * 8 + magnitude code * 2.
+template <int OUTB>
+__device__ __forceinline__ uint32_t level_code_word4(const uint32_t *P, int g) {
+    if constexpr (OUTB == 1) {
+        return (spread8n(P[0], g) * 8u) | 0x22222222u;
+    } else if constexpr (OUTB == 2) {
+        return spread8n(P[1], g) * 2u + spread8n(P[0], g) * 8u;
+    } else {
+        return spread8n(P[1], g) * 2u + spread8n(P[2], g) * 4u + spread8n(P[0] & (P[1] | P[2]), g) * 8u;
+    }
+}
+
+// E2M1 code of level index k of an OUTB-bit quantizer (packed nibble tables).
+template <int OUTB>
+__device__ __forceinline__ uint32_t code4_k(int k) {
+    if constexpr (OUTB == 1) return (0x2Au >> (4 * k)) & 0xFu;
+    else if constexpr (OUTB == 2) return (0x20Au >> (4 * k)) & 0xFu;
+    else return (0x6420ACEu >> (4 * k)) & 0xFu;
+}
+
 // Stores the planes (bits of channels >= nvalid cleared) and the E4M3 codes
 // (ncodes = 16 or 32 bytes; the second 16 only when nvalid > 16) of OUTB-bit
 // levels given by their masks M[0 .. levels - 2].
+// With codes4 the codes are E2M1 nibbles instead (codes then points at the
+// byte of the first channel: 16 bytes for 32 channels, 8 for 16).
 template <int OUTB>
 __device__ __forceinline__ void store_level_masks(const uint32_t *M, int nvalid, int ncodes, uint32_t *planes, int NWo,
-                                                  uint8_t *codes) {
+                                                  uint8_t *codes, bool codes4 = false) {
     uint32_t P[3];
     level_planes<OUTB>(M, P);
     if (planes != nullptr) {
@@ -234,7 +286,13 @@ __device__ __forceinline__ void store_level_masks(const uint32_t *M, int nvalid,
 #pragma unroll
         for (int u = 0; u < OUTB; ++u) planes[u * NWo] = P[u] & vm;
     }
-    if (codes != nullptr) {
+    if (codes != nullptr && codes4) {
+        if (nvalid > 16 && ncodes > 16)
+            *reinterpret_cast<uint4 *>(codes) = make_uint4(level_code_word4<OUTB>(P, 0), level_code_word4<OUTB>(P, 1),
+                                                           level_code_word4<OUTB>(P, 2), level_code_word4<OUTB>(P, 3));
+        else
+            *reinterpret_cast<uint2 *>(codes) = make_uint2(level_code_word4<OUTB>(P, 0), level_code_word4<OUTB>(P, 1));
+    } else if (codes != nullptr) {
         uint4 *dst = reinterpret_cast<uint4 *>(codes);
         dst[0] = make_uint4(level_code_word<OUTB>(P, 0), level_code_word<OUTB>(P, 1), level_code_word<OUTB>(P, 2),
                             level_code_word<OUTB>(P, 3));

@@ -215,15 +215,19 @@ minw_status minw_conv_block_codes_ex(const uint8_t *act, int32_t B, int32_t C, i
     ConvArgs a;
     minw_status st = make_codes_args(a, act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad);
     if (st != MINW_OK) return st;
-    if (!scale || !shift) return MINW_EINVAL;
     if (q_out && (!valid_quant(q_out) || (!planes_out && !codes_out))) return MINW_EINVAL;
     if (codes_out && (O % 16 != 0 || !aligned16(codes_out))) return MINW_EUNSUPPORTED;
     if (pool != 0 && pool != 1) return MINW_EINVAL;
     if (pool && ((a.Ho & 1) || (a.Wo & 1))) return MINW_EUNSUPPORTED;
     if (extra && extra->res_codes && extra->res_f32) return MINW_EINVAL;
     if (extra && extra->res_codes && (extra->res_bits < 1 || extra->res_bits > 3)) return MINW_EINVAL;
-    const bool any_out = q_out || y_out || (extra && extra->y_nhwc);
+    if (extra && ((unsigned)extra->in_format > 1u || (unsigned)extra->out_format > 1u ||
+                  (unsigned)extra->res_format > 1u))
+        return MINW_EINVAL;
+    if (extra && extra->acc_out && pool) return MINW_EUNSUPPORTED;
+    const bool any_out = q_out || y_out || (extra && (extra->y_nhwc || extra->acc_out));
     if (!any_out) return MINW_EINVAL;
+    if ((q_out || y_out || (extra && extra->y_nhwc)) && (!scale || !shift)) return MINW_EINVAL;
     a.scale = scale;
     a.shift = shift;
     a.pool = pool;
@@ -237,6 +241,10 @@ minw_status minw_conv_block_codes_ex(const uint8_t *act, int32_t B, int32_t C, i
         a.res_unit = extra->res_bits == 3 ? 0.25f : 1.0f;
         a.res_f32 = extra->res_f32;
         a.y_nhwc = extra->y_nhwc;
+        a.fp4 = extra->in_format == MINW_CODES_E2M1;
+        a.codes_out4 = extra->out_format == MINW_CODES_E2M1;
+        a.res_codes4 = extra->res_format == MINW_CODES_E2M1;
+        a.acc_out = extra->acc_out;
     }
     return launch_conv_tc(a, (cudaStream_t)stream);
 }

@@ -427,7 +427,10 @@ __global__ void __launch_bounds__(FIRST_NT, 2)
 #pragma unroll
                         for (int u = 0; u < OUTB; ++u) dst[u * NWo] = P[u] & vm;
                     }
-                    if (a.codes_out != nullptr && hch > 0)
+                    if (a.codes_out != nullptr && hch > 0 && a.codes4)
+                        *reinterpret_cast<uint2 *>(a.codes_out + ((m * a.O + ob + 16 * h) >> 1)) =
+                            make_uint2(level_code_word4<OUTB>(P, 2 * h), level_code_word4<OUTB>(P, 2 * h + 1));
+                    else if (a.codes_out != nullptr && hch > 0)
                         *reinterpret_cast<uint4 *>(a.codes_out + m * a.O + ob + 16 * h) =
                             make_uint4(level_code_word<OUTB>(P, 4 * h), level_code_word<OUTB>(P, 4 * h + 1),
                                        level_code_word<OUTB>(P, 4 * h + 2), level_code_word<OUTB>(P, 4 * h + 3));

@@ -95,6 +95,12 @@ struct Params {
     int ystage;                // 32-bit words of the staging tiles (8 warps x 32 x 16, or 0)
     int upd;                   // fully connected output: y_out holds latent weights, updated in place
     float upd_lr, upd_2a;      // (Algorithm 1: learning rate and 2 alpha of the mask of Eq. weight)
+    int fp4;                   // operands are E2M1 codes, two channels per byte (kind::mxf4, unit scales)
+    int out4;                  // codes_out receives E2M1 codes
+    int res4;                  // res_codes holds E2M1 codes
+    int nacc;                  // TMEM accumulators: 2 (the epilogue of one tile overlaps the MMAs of the
+                               // next) or 1 (E2M1 tiles of 256 columns: the scale factors take the rest)
+    uint32_t sf_col;           // E2M1 operands: TMEM column of A's unit scale factors (B's at + 32)
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -233,6 +239,25 @@ __device__ __forceinline__ void mma_bf16_pair(uint32_t tmem_d, uint64_t adesc, u
                  "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
 }
 
+// E2M1 x E2M1 -> fp32 with block scaling (kind::mxf4, 32 elements per
+// UE8M0 scale, K = 64 per instruction): every scale factor in tensor memory
+// is 2^0, so the products are the plain level products, exact like E4M3's.
+// The packed operands halve the bytes per K step, and the instruction covers
+// twice the K of an E4M3 one at the same issue cost.
+__device__ __forceinline__ void mma_f4(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                       uint32_t accumulate, uint32_t sfa, uint32_t sfb) {
+    asm volatile(MINW_ELECT_PROLOGUE
+                 " @e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%0], %1, %2, %3, [%5], [%6], p;\n}\n"
+                 ::"r"(tmem_d), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate), "r"(sfa), "r"(sfb));
+}
+
+__device__ __forceinline__ void mma_f4_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                            uint32_t accumulate, uint32_t sfa, uint32_t sfb) {
+    asm volatile(MINW_ELECT_PROLOGUE
+                 " @e tcgen05.mma.cta_group::2.kind::mxf4.block_scale.scale_vec::2X [%0], %1, %2, %3, [%5], [%6], p;\n}\n"
+                 ::"r"(tmem_d), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate), "r"(sfa), "r"(sfb));
+}
+
 // Arrive on the barrier at this offset in both CTAs of the pair once the
 // pair's MMAs issued so far have completed (an mbarrier signal to each CTA).
 __device__ __forceinline__ void mma_commit_pair(uint64_t *bar) {
@@ -361,7 +386,7 @@ __device__ __forceinline__ uint32_t transpose32(uint32_t a, int lane) {
 template <int OUTB>
 __device__ __forceinline__ void mask_chunk(uint32_t taddr, bool full32, const float *th, int tstride, uint32_t sig,
                                            int pool, int bw, bool writer, int nvalid, uint32_t *planes, int NWo,
-                                           uint8_t *codes) {
+                                           uint8_t *codes, bool codes4) {
     constexpr int NL = OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7);
     uint32_t v[32];
     if (full32) {
@@ -408,7 +433,7 @@ __device__ __forceinline__ void mask_chunk(uint32_t taddr, bool full32, const fl
         }
     }
     if (!writer) return;
-    store_level_masks<OUTB>(M, nvalid, full32 ? 32 : 16, planes, NWo, codes);
+    store_level_masks<OUTB>(M, nvalid, full32 ? 32 : 16, planes, NWo, codes, codes4);
 }
 
 // Epilogue of one 32-column chunk (16 when full32 is false) of a residual
@@ -449,7 +474,18 @@ __device__ __forceinline__ void resid_chunk(uint32_t taddr, bool full32, const P
             if (q4 * 4 < nvalid && q4 * 4 < ncol) dst[q4] = make_float4(y[4 * q4], y[4 * q4 + 1], y[4 * q4 + 2], y[4 * q4 + 3]);
     }
     if constexpr (OUTB > 0) {
-        if (p.res_codes != nullptr) {
+        if (p.res_codes != nullptr && p.res4) {
+            const uint2 *src = reinterpret_cast<const uint2 *>(p.res_codes + base / 2);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                if (h * 16 >= nvalid || h * 16 >= ncol) break;
+                const uint2 cv = __ldg(src + h);
+                const uint32_t cw[2] = {cv.x, cv.y};
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                    y[h * 16 + j] += code_units_e2m1(cw[j >> 3] >> (4 * (j & 7))) * p.res_unit;
+            }
+        } else if (p.res_codes != nullptr) {
             const uint4 *src = reinterpret_cast<const uint4 *>(p.res_codes + base);
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
@@ -484,14 +520,15 @@ __device__ __forceinline__ void resid_chunk(uint32_t taddr, bool full32, const P
 #pragma unroll
             for (int u = 0; u < NL - 1; ++u) M[u] = __funnelshift_l(__float_as_uint(y[j] + nt[u]), M[u], 1);
         store_level_masks<OUTB>(M, nvalid, ncol, p.planes_out ? p.planes_out + (opix * OUTB) * NWo + (ob >> 5) : nullptr,
-                                NWo, p.codes_out ? p.codes_out + base : nullptr);
+                                NWo, p.codes_out ? p.codes_out + (p.out4 ? base / 2 : base) : nullptr, p.out4 != 0);
     }
 }
 
 // OUTB: bits of the quantized output (0 when the launch writes none).
 // PAIR: CTA pairs with cta_group::2 MMAs (a kernel uses one CTA group only).
-// BF16: bf16 operands (kind::f16), else E4M3 level codes (kind::f8f6f4); both
-// consume 32 bytes of K per MMA step.
+// FMT: operand format -- 0 E4M3 level codes (kind::f8f6f4), 1 bf16 (kind::f16),
+// 2 E2M1 level codes (kind::mxf4); all three consume 32 bytes of K per MMA
+// step (32, 16 and 64 elements).
 // Stores the 16 words u[] of each lane's tile row (row = lane) row-contiguously:
 // row rr goes to dst0 + rr * rstride + [0, 16), rows < nrows, columns < ncols.
 // The warp transposes through its 32 x 16-word shared tile in 16-byte chunks,
@@ -578,7 +615,7 @@ __device__ __forceinline__ void rows_store16(uint32_t *sw, const uint32_t (&u)[1
     }
 }
 
-template <int OUTB, bool PAIR, bool BF16>
+template <int OUTB, bool PAIR, int FMT>
 __global__ void __launch_bounds__(NT, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const Params p) {
@@ -688,6 +725,23 @@ __global__ void __launch_bounds__(NT, 1)
     if constexpr (PAIR) cluster_sync_all();   // every barrier of the pair is initialised
     fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    if constexpr (FMT == 2) {
+        // unit scale factors (UE8M0 0x7F = 2^0) in 64 columns from sf_col, written
+        // by one warp per TMEM lane quarter (a pair: each CTA in its own tensor memory)
+        if (warp >= 2 && warp < 6) {
+            const uint32_t ta = tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + p.sf_col;
+#pragma unroll
+            for (int c = 0; c < 64; c += 8)
+                asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %1, %1, %1, %1, %1, %1, %1};\n" ::"r"(
+                                 ta + (uint32_t)c),
+                             "r"(0x7F7F7F7Fu));
+            asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory");
+        }
+        fence_before();
+        __syncthreads();
+        if constexpr (PAIR) cluster_sync_all();   // both CTAs' scale factors are in place
+        fence_after();
+    }
     pdl_trigger();                            // set-up done: the next kernel may start its own
 
     if (warp == 0 || warp == B_WARP) {
@@ -723,18 +777,20 @@ __global__ void __launch_bounds__(NT, 1)
                     if (arrive) mbar_expect_tx(&full[s], (uint32_t)n * bytes * (PAIR ? 2u : 1u));
                     const uint32_t fb = PAIR ? cta0_addr(&full[s]) : 0u;
                     for (int j = 0; j < n; ++j) {
+                        // tensor-map x coordinates: elements, or bytes for packed E2M1
+                        const int cx = FMT == 2 ? c0 >> 1 : c0, kx_ = FMT == 2 ? kcol >> 1 : kcol;
                         if constexpr (PAIR) {
                             if (act)
-                                tma_load_4d_pair(sa + (size_t)j * p.a_bytes, &tmA, fb, c0, x0 + kx, y0 + ky, b0);
+                                tma_load_4d_pair(sa + (size_t)j * p.a_bytes, &tmA, fb, cx, x0 + kx, y0 + ky, b0);
                             else
                                 tma_load_2d_pair(sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes, &tmB, fb,
-                                                 kcol, o0 + crank * bslice);
+                                                 kx_, o0 + crank * bslice);
                         } else if (act)
-                            tma_load_4d(sa + (size_t)j * p.a_bytes, &tmA, &full[s], c0, x0 + kx, y0 + ky, b0);
+                            tma_load_4d(sa + (size_t)j * p.a_bytes, &tmA, &full[s], cx, x0 + kx, y0 + ky, b0);
                         else {
                             uint8_t *sb = sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes;
-                            tma_load_2d(sb, &tmB, &full[s], kcol, o0);
-                            if (p.dup) tma_load_2d(sb + (size_t)64 * p.cb, &tmB, &full[s], kcol, o0);
+                            tma_load_2d(sb, &tmB, &full[s], kx_, o0);
+                            if (p.dup) tma_load_2d(sb + (size_t)64 * p.cb, &tmB, &full[s], kx_, o0);
                         }
                         kcol += p.ck;
                         c0 += p.ck;
@@ -768,8 +824,9 @@ __global__ void __launch_bounds__(NT, 1)
             const uint32_t astep = p.a_bytes >> 4, bstep = p.b_bytes >> 4;   // second K block of a stage
             const bool k128 = p.cb == 128;                 // four 32-byte K steps per K block, else two
             const uint32_t idesc = p.idesc;
+            const uint32_t sfa = tmem_base + p.sf_col, sfb = sfa + 32u;
             for (int w = blockIdx.x; w < items && alive; w += gridDim.x, ++i) {
-                const int ab = i & 1, use = i >> 1;
+                const int ab = p.nacc == 2 ? (i & 1) : 0, use = p.nacc == 2 ? (i >> 1) : i;
                 const int t = w / p.ksplit, kp = w - t * p.ksplit;
                 const int kb = (int)((long long)kp * p.nk / p.ksplit), ke = (int)((long long)(kp + 1) * p.nk / p.ksplit);
                 if (use > 0 && !__all_sync(0xffffffffu, PAIR ? mbar_wait_cluster(&tempty[ab], (use - 1) & 1)
@@ -779,12 +836,16 @@ __global__ void __launch_bounds__(NT, 1)
                 const uint32_t tmem_d = tmem_base + (uint32_t)(ab * p.acc_cols);
                 uint32_t acc = 0u;
                 auto mma = [&](uint64_t ad_, uint64_t bd_, uint32_t a_) {
-                    if constexpr (PAIR && BF16)
+                    if constexpr (PAIR && FMT == 1)
                         mma_bf16_pair(tmem_d, ad_, bd_, idesc, a_);
+                    else if constexpr (PAIR && FMT == 2)
+                        mma_f4_pair(tmem_d, ad_, bd_, idesc, a_, sfa, sfb);
                     else if constexpr (PAIR)
                         mma_f8_pair(tmem_d, ad_, bd_, idesc, a_);
-                    else if constexpr (BF16)
+                    else if constexpr (FMT == 1)
                         mma_bf16(tmem_d, ad_, bd_, idesc, a_);
+                    else if constexpr (FMT == 2)
+                        mma_f4(tmem_d, ad_, bd_, idesc, a_, sfa, sfb);
                     else
                         mma_f8(tmem_d, ad_, bd_, idesc, a_);
                 };
@@ -869,7 +930,7 @@ __global__ void __launch_bounds__(NT, 1)
                 const int oq = 32 * (p.dup ? (q & 1) : q);
                 const int cq = p.dup ? 2 : 4, cb = p.dup ? 2 * (2 * (q >> 1) + half_cols) : 4 * half_cols;
                 for (int w = blockIdx.x; w < items; w += gridDim.x, ++i) {
-                    const int ab = i & 1, use = i >> 1;
+                    const int ab = p.nacc == 2 ? (i & 1) : 0, use = p.nacc == 2 ? (i >> 1) : i;
                     const int tn = w / tiles_m, tm = w - tn * tiles_m;
                     const int xb = tm % p.nbx, yb = (tm / p.nbx) % p.nby, bbk = tm / (p.nbx * p.nby);
                     const int oc = tn * p.BN + oq + lane;          // this lane's channel
@@ -910,7 +971,16 @@ __global__ void __launch_bounds__(NT, 1)
                             // (all 32 loads issue before the first use; a pixel past the batch reads pixel 0)
                             const long long pix = valid ? (((long long)b * p.Ho + y) * p.Wo + x) * p.O : 0;
                             float yv[32];
-                            if (p.res_codes != nullptr) {
+                            if (p.res_codes != nullptr && p.res4) {
+                                uint32_t cb[32];
+#pragma unroll
+                                for (int j = 0; j < 32; ++j)
+                                    cb[j] = __ldg(p.res_codes + ((oc + __shfl_sync(0xffffffffu, pix, j)) >> 1));
+#pragma unroll
+                                for (int j = 0; j < 32; ++j)
+                                    yv[j] = fmaf(__uint_as_float(v[j]), sc, sh) +
+                                            code_units_e2m1(cb[j] >> (4 * (oc & 1))) * p.res_unit;
+                            } else if (p.res_codes != nullptr) {
                                 uint32_t cb[32];
 #pragma unroll
                                 for (int j = 0; j < 32; ++j) cb[j] = __ldg(p.res_codes + oc + __shfl_sync(0xffffffffu, pix, j));
@@ -958,7 +1028,8 @@ __global__ void __launch_bounds__(NT, 1)
                             const int ob = tn * p.BN + oq;
                             store_level_masks<OUTB>(M, 32, 32,
                                                     p.planes_out ? p.planes_out + (opix * OUTB) * NWo + (ob >> 5) : nullptr,
-                                                    NWo, p.codes_out ? p.codes_out + opix * p.O + ob : nullptr);
+                                                    NWo, p.codes_out ? p.codes_out + ((opix * p.O + ob) >> p.out4) : nullptr,
+                                                    p.out4 != 0);
                         }
                     }
                     fence_before();
@@ -968,7 +1039,7 @@ __global__ void __launch_bounds__(NT, 1)
             }
         }
         for (int w = blockIdx.x; w < items && !p.trans; w += gridDim.x, ++i) {
-            const int ab = i & 1, use = i >> 1;
+            const int ab = p.nacc == 2 ? (i & 1) : 0, use = p.nacc == 2 ? (i >> 1) : i;
             const int t = w / p.ksplit, kp = w - t * p.ksplit;
             const int tn = t / tiles_m, tm = t - tn * tiles_m;
             const int xb = tm % p.nbx, yb = (tm / p.nbx) % p.nby, bbk = tm / (p.nbx * p.nby);
@@ -994,7 +1065,8 @@ __global__ void __launch_bounds__(NT, 1)
                                          c * 32 + 32 <= p.BN, sthr + ob, O32, p.pool ? ssig[ob >> 5] : 0u, p.pool,
                                          p.bw, writer, p.O - ob,
                                          p.planes_out ? p.planes_out + (opix * OUTB) * NWo + (ob >> 5) : nullptr,
-                                         NWo, p.codes_out ? p.codes_out + opix * p.O + ob : nullptr);
+                                         NWo, p.codes_out ? p.codes_out + ((opix * p.O + ob) >> p.out4) : nullptr,
+                                         p.out4 != 0);
                     }
                     fence_before();
                     __syncwarp();
@@ -1050,7 +1122,7 @@ __global__ void __launch_bounds__(NT, 1)
                     // residual block: y = BN(acc) [+ shortcut], HardTanh, quantize,
                     // element by element in the fp32 order of the block
                     if (writer) {
-                        uint32_t cw[4] = {0u, 0u, 0u, 0u};
+                        uint32_t cw[4] = {0u, 0u, 0u, 0u}, cw4[2] = {0u, 0u};
                         uint32_t bits16[3] = {0u, 0u, 0u};
 #pragma unroll
                         for (int j = 0; j < 16; ++j) {
@@ -1058,7 +1130,11 @@ __global__ void __launch_bounds__(NT, 1)
                             if (o >= p.O) continue;
                             float yv = fmaf(a[j], __ldg(p.scale + o), __ldg(p.shift + o));
                             if (p.y_nhwc != nullptr) p.y_nhwc[opix * p.O + o] = yv;
-                            if (p.res_codes != nullptr) yv += code_units(__ldg(p.res_codes + opix * p.O + o)) * p.res_unit;
+                            if (p.res_codes != nullptr && p.res4)
+                                yv += code_units_e2m1(__ldg(p.res_codes + ((opix * p.O + o) >> 1)) >> (4 * (o & 1))) *
+                                      p.res_unit;
+                            else if (p.res_codes != nullptr)
+                                yv += code_units(__ldg(p.res_codes + opix * p.O + o)) * p.res_unit;
                             else if (p.res_f32 != nullptr) yv += __ldg(p.res_f32 + opix * p.O + o);
                             if (p.y_out != nullptr)
                                 p.y_out[(((long long)b * p.O + o) * Hp + yp) * Wp + xp] =
@@ -1066,13 +1142,16 @@ __global__ void __launch_bounds__(NT, 1)
                             if constexpr (OUTB > 0) {
                                 const int k = level_index_of_y(yv, p.qo);
                                 cw[j >> 2] |= code_k<OUTB>(k) << ((j & 3) * 8);
+                                cw4[j >> 3] |= code4_k<OUTB>(k) << ((j & 7) * 4);
                                 const uint32_t pb = planes_k<OUTB>(k);
 #pragma unroll
                                 for (int u = 0; u < OUTB; ++u) bits16[u] |= ((pb >> u) & 1u) << j;
                             }
                         }
                         if constexpr (OUTB > 0) {
-                            if (p.codes_out != nullptr)
+                            if (p.codes_out != nullptr && p.out4)
+                                *reinterpret_cast<uint2 *>(p.codes_out + ((opix * p.O + ob) >> 1)) = make_uint2(cw4[0], cw4[1]);
+                            else if (p.codes_out != nullptr)
                                 *reinterpret_cast<uint4 *>(p.codes_out + opix * p.O + ob) =
                                     make_uint4(cw[0], cw[1], cw[2], cw[3]);
                             if (p.planes_out != nullptr) {
@@ -1102,7 +1181,12 @@ __global__ void __launch_bounds__(NT, 1)
                             for (int u = 0; u < NL - 1; ++u) k += (vv + sthr[u * O32 + o] >= 0.0f) ? 1 : 0;   // -T
                             kq[j] = k;
                         }
-                        if (p.codes_out != nullptr) {
+                        if (p.codes_out != nullptr && p.out4) {
+                            uint32_t cw4[2] = {0u, 0u};
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) cw4[j >> 3] |= code4_k<OUTB>(kq[j]) << ((j & 7) * 4);
+                            *reinterpret_cast<uint2 *>(p.codes_out + ((opix * p.O + ob) >> 1)) = make_uint2(cw4[0], cw4[1]);
+                        } else if (p.codes_out != nullptr) {
                             uint32_t cw[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
                             for (int j = 0; j < 16; ++j) cw[j >> 2] |= code_k<OUTB>(kq[j]) << ((j & 3) * 8);
@@ -1199,7 +1283,7 @@ __global__ void __launch_bounds__(NT, 1)
                     // summed by splitk_reduce_kernel
                     uint32_t u[16];
 #pragma unroll
-                    for (int j = 0; j < 16; ++j) u[j] = BF16 ? __float_as_uint(a[j]) : (uint32_t)__float2int_rn(a[j]);
+                    for (int j = 0; j < 16; ++j) u[j] = FMT == 1 ? __float_as_uint(a[j]) : (uint32_t)__float2int_rn(a[j]);
                     rows_store16(sw, u, lane,
                                  reinterpret_cast<uint32_t *>(p.part) + (((size_t)kp * tiles + t) * 128 + q * 32) * p.BN +
                                      ch * 16,
@@ -1211,7 +1295,7 @@ __global__ void __launch_bounds__(NT, 1)
                         int v[4];
 #pragma unroll
                         for (int e = 0; e < 4; ++e)
-                            v[e] = BF16 ? __float_as_int(a[4 * j + e]) : __float2int_rn(a[4 * j + e]);
+                            v[e] = FMT == 1 ? __float_as_int(a[4 * j + e]) : __float2int_rn(a[4 * j + e]);
                         dst[j] = make_int4(v[0], v[1], v[2], v[3]);
                     }
                 }
@@ -1324,7 +1408,11 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const Params p, cons
             if (o + j < p.O) {
                 float yv = fmaf(accf[j], __ldg(p.scale + o + j), __ldg(p.shift + o + j));
                 if (p.y_nhwc != nullptr) p.y_nhwc[pix * p.O + o + j] = yv;
-                if (p.res_codes != nullptr) yv += code_units(__ldg(p.res_codes + pix * p.O + o + j)) * p.res_unit;
+                if (p.res_codes != nullptr && p.res4)
+                    yv += code_units_e2m1(__ldg(p.res_codes + ((pix * p.O + o + j) >> 1)) >> (4 * ((o + j) & 1))) *
+                          p.res_unit;
+                else if (p.res_codes != nullptr)
+                    yv += code_units(__ldg(p.res_codes + pix * p.O + o + j)) * p.res_unit;
                 else if (p.res_f32 != nullptr) yv += __ldg(p.res_f32 + pix * p.O + o + j);
                 yres[j] = yv;
             }
@@ -1344,7 +1432,7 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const Params p, cons
         }
     }
     if constexpr (OUTB > 0) {
-        uint32_t code = 0u, bits[3] = {0u, 0u, 0u};
+        uint32_t code = 0u, code4 = 0u, bits[3] = {0u, 0u, 0u};
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             if (valid && o + j < p.O) {
@@ -1358,12 +1446,18 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const Params p, cons
                     for (int u = 0; u < NL - 1; ++u) k += (v >= __ldg(th + u)) ? 1 : 0;
                 }
                 code |= code_k<OUTB>(k) << (8 * j);
+                code4 |= code4_k<OUTB>(k) << (4 * j);
                 const uint32_t pb = planes_k<OUTB>(k);
 #pragma unroll
                 for (int u = 0; u < OUTB; ++u) bits[u] |= ((pb >> u) & 1u) << (lane8 * 4 + j);
             }
         }
-        if (p.codes_out != nullptr && valid) *reinterpret_cast<uint32_t *>(p.codes_out + pix * p.O + o) = code;
+        if (p.codes_out != nullptr && valid) {
+            if (p.out4)
+                *reinterpret_cast<uint16_t *>(p.codes_out + ((pix * p.O + o) >> 1)) = (uint16_t)code4;
+            else
+                *reinterpret_cast<uint32_t *>(p.codes_out + pix * p.O + o) = code;
+        }
         if (p.planes_out != nullptr) {
 #pragma unroll
             for (int u = 0; u < OUTB; ++u) {
@@ -1438,7 +1532,10 @@ static int auto_ksplit(int tiles, int nk, int sms) {
 }
 // channels of one K chunk: 128-byte rows of E4M3 codes (64-byte rows when C is
 // not a multiple of 128), or 64 bf16 values
-static int chunk_channels(const ConvArgs &a) { return a.bf16 ? 64 : ((a.C % 128 == 0) ? 128 : 64); }
+static int chunk_channels(const ConvArgs &a) {
+    if (a.fp4) return (a.C % 256 == 0) ? 256 : 128;    // 128- or 64-byte rows of E2M1 pairs
+    return a.bf16 ? 64 : ((a.C % 128 == 0) ? 128 : 64);
+}
 static size_t slice_bytes(int tiles, int BN) { return (size_t)tiles * 128 * BN * sizeof(int32_t); }
 static size_t thr_ws_bytes(int O, int nlev) { return (((size_t)O * nlev * sizeof(float)) + 255) & ~(size_t)255; }
 
@@ -1541,8 +1638,13 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     p.Ho = a.Ho; p.Wo = a.Wo;
     p.stride = a.stride;
     p.esize = a.bf16 ? 2 : 1;
-    p.cb = (a.C * p.esize % 128 == 0) ? 128 : 64;
-    p.ck = p.cb / p.esize;
+    p.fp4 = a.fp4 ? 1 : 0;
+    p.out4 = a.codes_out4 ? 1 : 0;
+    p.res4 = a.res_codes4 ? 1 : 0;
+    // bytes of one pixel's channels: E2M1 packs two channels per byte
+    const int rowb = p.fp4 ? a.C / 2 : a.C * p.esize;
+    p.cb = (rowb % 128 == 0) ? 128 : 64;
+    p.ck = p.fp4 ? 2 * p.cb : p.cb / p.esize;
     p.a_bytes = (uint32_t)(p.mrows * p.cb);
     p.nck = a.C / p.ck;
     p.nk = a.kh * a.kw * p.nck;
@@ -1581,13 +1683,25 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     // MMA N: the output channels, or the 256 pixels of a channel-major tile (M = 128 either way)
     const int mma_n = p.trans ? 256 : p.BN;
     p.acc_cols = mma_n;
-    // D fp32; A and B E4M3 (kind::f8f6f4) or bf16 (kind::f16)
-    const uint32_t fmt = a.bf16 ? 1u : 0u;
-    p.idesc = (1u << 4) | (fmt << 7) | (fmt << 10) | ((uint32_t)(mma_n >> 3) << 17) |
-              ((uint32_t)((p.pair ? 256 : 128) >> 4) << 24);
-    uint32_t cols = 32;
-    while ((int)cols < 2 * mma_n) cols <<= 1;         // two accumulators
-    p.tmem_cols = cols;
+    // D fp32; A and B E4M3 (kind::f8f6f4), bf16 (kind::f16), or E2M1 with UE8M0
+    // block scales (kind::mxf4: formats E2M1 = 1, scale type bit 23)
+    const uint32_t mrows = (uint32_t)(p.pair ? 256 : 128);
+    if (p.fp4) {
+        p.idesc = (1u << 7) | (1u << 10) | ((uint32_t)(mma_n >> 3) << 17) | (1u << 23) | ((mrows >> 4) << 24);
+        // all 512 columns: the accumulators below column 448, the unit scale
+        // factors of A at 448 and of B at 480
+        p.tmem_cols = 512;
+        p.sf_col = 448;
+        p.nacc = 2 * mma_n <= 448 ? 2 : 1;
+    } else {
+        const uint32_t fmt = a.bf16 ? 1u : 0u;
+        p.idesc = (1u << 4) | (fmt << 7) | (fmt << 10) | ((uint32_t)(mma_n >> 3) << 17) | ((mrows >> 4) << 24);
+        uint32_t cols = 32;
+        while ((int)cols < 2 * mma_n) cols <<= 1;         // two accumulators
+        p.tmem_cols = cols;
+        p.sf_col = 0;
+        p.nacc = 2;
+    }
     p.acc_out = a.acc_out; p.y_out = a.y_out; p.scale = a.scale; p.shift = a.shift;
     p.upd = a.upd; p.upd_lr = a.upd_lr; p.upd_2a = a.upd_2a;
     p.pool = a.pool; p.quant_out = a.quant_out; p.qo = a.qo;
@@ -1630,12 +1744,14 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     const CUtensorMapSwizzle swz = p.cb == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
     const CUtensorMapDataType dt = a.bf16 ? CU_TENSOR_MAP_DATA_TYPE_UINT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8;
     const cuuint64_t es_ = (cuuint64_t)p.esize;
+    // tensor-map elements per pixel row and per K block: bytes for packed E2M1
+    const cuuint64_t cel = (cuuint64_t)(p.fp4 ? a.C / 2 : a.C);
+    const cuuint32_t kel = (cuuint32_t)(p.fp4 ? p.cb : p.ck);
     {
-        const cuuint64_t dims[4] = {(cuuint64_t)a.C, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.B};
-        const cuuint64_t strides[3] = {(cuuint64_t)a.C * es_, (cuuint64_t)a.W * a.C * es_,
-                                       (cuuint64_t)a.H * a.W * a.C * es_};
+        const cuuint64_t dims[4] = {cel, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.B};
+        const cuuint64_t strides[3] = {cel * es_, (cuuint64_t)a.W * cel * es_, (cuuint64_t)a.H * a.W * cel * es_};
         const cuuint32_t sd = (cuuint32_t)p.stride;
-        const cuuint32_t box[4] = {(cuuint32_t)p.ck, (cuuint32_t)p.bw * sd, (cuuint32_t)p.bh * sd, (cuuint32_t)p.bb};
+        const cuuint32_t box[4] = {kel, (cuuint32_t)p.bw * sd, (cuuint32_t)p.bh * sd, (cuuint32_t)p.bb};
         const cuuint32_t es[4] = {1u, sd, sd, 1u};
         if (enc(&pl.tmA, dt, 4, const_cast<uint8_t *>(a.act8), dims, strides, box, es,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -1643,10 +1759,10 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
             return MINW_ECUDA;
     }
     {
-        const long long K = (long long)a.kh * a.kw * a.C;
+        const long long K = (long long)a.kh * a.kw * cel;
         const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)a.O};
         const cuuint64_t strides[1] = {(cuuint64_t)K * es_};
-        const cuuint32_t box[2] = {(cuuint32_t)p.ck, (cuuint32_t)(p.dup ? 64 : p.BN / p.cl)};
+        const cuuint32_t box[2] = {kel, (cuuint32_t)(p.dup ? 64 : p.BN / p.cl)};
         const cuuint32_t es[2] = {1u, 1u};
         if (enc(&pl.tmB, dt, 2, const_cast<uint8_t *>(a.wgt8), dims, strides, box, es,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -1715,6 +1831,8 @@ static bool conv_tc_residual(const ConvArgs &a) {
 bool conv_tc_supported(const ConvArgs &a) {
     tc::Params p{};
     if (!tc::plan_shape(a, p)) return false;
+    // E2M1 operands: rows of 64 or 128 bytes (128 or 256 channels)
+    if (a.fp4 && (a.bf16 || a.C % 128 != 0)) return false;
     // bf16 operands: real-valued accumulators, so fp32 BN outputs only
     if (a.bf16 && (a.quant_out || a.acc_out != nullptr || a.y_out == nullptr || conv_tc_residual(a))) return false;
     if (a.quant_out && (size_t)a.O * num_levels(a.qo.bits) * sizeof(float) > 64 * 1024) return false;
@@ -1747,18 +1865,22 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
     const int outb = a.quant_out ? a.qo.bits : 0;
     const bool split = pl.p.ksplit > 1;
     const int kout = split ? 0 : outb;            // the split main pass writes only partial sums
-    static size_t configured[4] = {0, 0, 0, 0};
     typedef void (*TcKernel)(const CUtensorMap, const CUtensorMap, const tc::Params);
-    static const TcKernel kernels[2][4] = {
-        {tc::conv_tc_kernel<0, false, false>, tc::conv_tc_kernel<1, false, false>,
-         tc::conv_tc_kernel<2, false, false>, tc::conv_tc_kernel<3, false, false>},
-        {tc::conv_tc_kernel<0, true, false>, tc::conv_tc_kernel<1, true, false>, tc::conv_tc_kernel<2, true, false>,
-         tc::conv_tc_kernel<3, true, false>}};
-    static size_t configured_pair[4] = {0, 0, 0, 0}, configured_bf16[2] = {0, 0};
-    const int kp = pl.p.pair ? 1 : 0;
-    TcKernel kern = a.bf16 ? (kp ? tc::conv_tc_kernel<0, true, true> : tc::conv_tc_kernel<0, false, true>)
-                           : kernels[kp][kout];
-    size_t &conf = a.bf16 ? configured_bf16[kp] : kp ? configured_pair[kout] : configured[kout];
+    // [pair][E2M1][output bits]; bf16 operands have fp32 outputs only
+    static const TcKernel kernels[2][2][4] = {
+        {{tc::conv_tc_kernel<0, false, 0>, tc::conv_tc_kernel<1, false, 0>, tc::conv_tc_kernel<2, false, 0>,
+          tc::conv_tc_kernel<3, false, 0>},
+         {tc::conv_tc_kernel<0, false, 2>, tc::conv_tc_kernel<1, false, 2>, tc::conv_tc_kernel<2, false, 2>,
+          tc::conv_tc_kernel<3, false, 2>}},
+        {{tc::conv_tc_kernel<0, true, 0>, tc::conv_tc_kernel<1, true, 0>, tc::conv_tc_kernel<2, true, 0>,
+          tc::conv_tc_kernel<3, true, 0>},
+         {tc::conv_tc_kernel<0, true, 2>, tc::conv_tc_kernel<1, true, 2>, tc::conv_tc_kernel<2, true, 2>,
+          tc::conv_tc_kernel<3, true, 2>}}};
+    static size_t configured[2][2][4] = {}, configured_bf16[2] = {0, 0};
+    const int kp = pl.p.pair ? 1 : 0, kf = pl.p.fp4 ? 1 : 0;
+    TcKernel kern = a.bf16 ? (kp ? tc::conv_tc_kernel<0, true, 1> : tc::conv_tc_kernel<0, false, 1>)
+                           : kernels[kp][kf][kout];
+    size_t &conf = a.bf16 ? configured_bf16[kp] : configured[kp][kf][kout];
     if (pl.smem > conf) {
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem) != cudaSuccess)
             return MINW_ECUDA;

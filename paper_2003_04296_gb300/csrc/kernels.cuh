@@ -32,6 +32,9 @@ struct ConvArgs {
     const uint8_t *act8;   // [B][H][W][C]
     const uint8_t *wgt8;   // [O][kh][kw][C]
     int bf16;              // operands are bf16 (weight-only quantized layers): fp32 outputs only
+    int fp4;               // operands are E2M1 level codes, two channels per byte (C % 128 == 0)
+    int codes_out4;        // codes_out receives E2M1 codes [B][Hp][Wp][O / 2]
+    int res_codes4;        // res_codes holds E2M1 codes
     const float *thr;      // output-quantizer breakpoints [O][levels] (nullable: computed in-kernel)
     // residual blocks (tensor-core path): y = BN(acc) + shortcut before HardTanh + quantize
     const uint8_t *res_codes;  // shortcut as level codes [B][Hp][Wp][O] (nullable)
@@ -58,6 +61,7 @@ struct FirstArgs {
     QParams qo;
     uint32_t *planes_out;      // [B][Ho][Wo][qo.bits][ceil(O/32)] (nullable)
     uint8_t *codes_out;        // [B][Ho][Wo][O] E4M3 level codes (nullable)
+    int codes4;                // codes_out receives E2M1 codes [B][Ho][Wo][O / 2] instead
     float *y_out;              // [B][O][Ho][Wo] (nullable)
     const float *thr;          // fp32 breakpoints [O][8] (nullable: computed in-kernel)
     const float *wt;           // prepared weights [K][O] (levels when quantized; nullable: from w)

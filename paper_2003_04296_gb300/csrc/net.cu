@@ -44,7 +44,7 @@ extern "C" {
 minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int32_t max_batch,
                             int32_t variant, void *stream, minw_net **out) {
     if (!layers || n_layers < 2 || max_batch <= 0 || !out) return MINW_EINVAL;
-    if (variant < 0 || variant > 2) return MINW_EINVAL;
+    if (variant < 0 || variant > 3) return MINW_EINVAL;
     *out = nullptr;
     cudaStream_t s = (cudaStream_t)stream;
     minw_net *n = new minw_net();
@@ -130,8 +130,14 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
             a.pool = P.pool;
             a.quant_out = !last;
             if (!last) a.qo = to_qparams(&P.qo);
-            P.variant = choose_variant(a, variant);
+            P.variant = choose_variant(a, variant == MINW_VARIANT_TC_E4M3 ? MINW_VARIANT_TC : variant);
             if (P.variant == MINW_VARIANT_TC && !conv_tc_supported(a)) { net_free(n); return MINW_EUNSUPPORTED; }
+            if (P.variant == MINW_VARIANT_TC && variant != MINW_VARIANT_TC_E4M3) {
+                // E2M1 operands wherever the channels fill 64-byte rows
+                a.fp4 = 1;
+                P.in4 = conv_tc_supported(a) ? 1 : 0;
+                a.fp4 = P.in4;
+            }
             if (P.variant == MINW_VARIANT_TC) {
                 const size_t wb = conv_tc_workspace_bytes(a);
                 if (wb > n->ws_bytes) n->ws_bytes = wb;
@@ -151,7 +157,8 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
         if (P.in_codes) {
             const size_t bytes = (size_t)P.O * P.kh * P.kw * P.C;
             if ((st = net_alloc(n, &P.wcodes, bytes)) != MINW_OK) { net_free(n); return st; }
-            st = minw_pack_weight_codes(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, P.wcodes, stream);
+            st = P.in4 ? minw_pack_weight_codes_e2m1(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, P.wcodes, stream)
+                       : minw_pack_weight_codes(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, P.wcodes, stream);
             if (st == MINW_OK && l + 1 < n_layers) {
                 const QParams qo = to_qparams(&P.qo);
                 st = net_alloc(n, &P.thr, (size_t)P.O * num_levels(qo.bits));
@@ -167,7 +174,8 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
     for (int l = 0; l + 1 < n_layers; ++l) {
         const LayerPlan &P = n->L[l];
         const bool codes = n->L[l + 1].in_codes;
-        const size_t words = codes ? ((size_t)max_batch * P.Hp * P.Wp * P.O + 3) / 4
+        const size_t cbytes = (size_t)max_batch * P.Hp * P.Wp * P.O / (n->L[l + 1].in4 ? 2 : 1);
+        const size_t words = codes ? (cbytes + 3) / 4
                                    : (size_t)max_batch * P.Hp * P.Wp * P.d.bits_out * ((P.O + 31) / 32);
         if (words > max_words) max_words = words;
     }
@@ -230,6 +238,7 @@ static minw_status forward_enqueue(minw_net *net, const float *x, int32_t B, flo
             if (!last) a.qo = to_qparams(&P.qo);
             a.planes_out = out_codes ? nullptr : (uint32_t *)dst;
             a.codes_out = out_codes ? (uint8_t *)dst : nullptr;
+            a.codes4 = out_codes && net->L[l + 1].in4;
             a.y_out = last ? logits : nullptr;
             a.thr = P.thr;
             a.wt = P.wt;
@@ -246,7 +255,9 @@ static minw_status forward_enqueue(minw_net *net, const float *x, int32_t B, flo
             if (!last) a.qo = to_qparams(&P.qo);
             a.planes_out = (!last && !out_codes) ? (uint32_t *)dst : nullptr;
             a.codes_out = out_codes ? (uint8_t *)dst : nullptr;
+            a.codes_out4 = out_codes && net->L[l + 1].in4;
             a.y_out = last ? logits : nullptr;
+            a.fp4 = P.in4;
             if (P.in_codes) {
                 a.act8 = (const uint8_t *)src;
                 a.wgt8 = P.wcodes;
@@ -351,7 +362,8 @@ minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants) {
         for (int l = 0; l < n; ++l) variants[l] = (l >= 2 && l < n - 1) ? MINW_VARIANT_TC : 0;
         return MINW_OK;
     }
-    for (size_t l = 0; l < net->L.size(); ++l) variants[l] = l == 0 ? 0 : net->L[l].variant;
+    for (size_t l = 0; l < net->L.size(); ++l)
+        variants[l] = l == 0 ? 0 : net->L[l].in4 ? MINW_VARIANT_TC_E2M1 : net->L[l].variant;
     return MINW_OK;
 }
 
@@ -374,7 +386,7 @@ int32_t minw_net_kernels(const minw_net *net) {
         a.M = (long long)net->max_batch * P.Ho * P.Wo; a.pool = P.pool;
         a.quant_out = l + 1 < net->L.size();
         if (a.quant_out) a.qo = to_qparams(&P.qo);
-        a.act8 = P.wcodes; a.wgt8 = P.wcodes; a.thr = P.thr;
+        a.act8 = P.wcodes; a.wgt8 = P.wcodes; a.thr = P.thr; a.fp4 = P.in4;
         a.workspace = net->ws; a.workspace_bytes = net->ws_bytes;
         k += conv_tc_launches(a);
     }

@@ -18,6 +18,7 @@ struct LayerPlan {
     float *thr = nullptr;          // output-quantizer breakpoints (first layer: fp32 [O][8];
                                    // tensor-core layers: integer-valued [O][levels])
     int in_codes = 0;              // input arrives in the codes layout
+    int in4 = 0;                   // ... as E2M1 codes (two channels per byte; weights too)
     float *wlatent = nullptr;      // fp32 weights (first layer)
     float *wt = nullptr;           // first layer: weights prepared as [K][O] levels
     float *wscale = nullptr;       // per-channel weight prescale (first layer)

@@ -16,7 +16,8 @@ from . import build as _build
 _LIB = None
 
 MINW_OK, MINW_EINVAL, MINW_EUNSUPPORTED, MINW_ECUDA, MINW_ETIMEOUT, MINW_EDEVICE = range(6)
-VARIANT_AUTO, VARIANT_POPC, VARIANT_TC = 0, 1, 2
+VARIANT_AUTO, VARIANT_POPC, VARIANT_TC, VARIANT_TC_E4M3, VARIANT_TC_E2M1 = 0, 1, 2, 3, 4
+CODES_E4M3, CODES_E2M1 = 0, 1
 LAYER_CONV, LAYER_FC = 0, 1
 
 
@@ -32,7 +33,8 @@ class Quant(ctypes.Structure):
 
 class BlockExtra(ctypes.Structure):
     _fields_ = [("res_codes", ctypes.c_void_p), ("res_bits", ctypes.c_int32), ("res_f32", ctypes.c_void_p),
-                ("y_nhwc", ctypes.c_void_p)]
+                ("y_nhwc", ctypes.c_void_p), ("in_format", ctypes.c_int32), ("out_format", ctypes.c_int32),
+                ("res_format", ctypes.c_int32), ("acc_out", ctypes.c_void_p)]
 
 
 class LayerDesc(ctypes.Structure):
@@ -85,6 +87,8 @@ SIGNATURES = {
                                        _QP, _P, _I32, _P, _P, _QP, _P, _P, _P]),
     "aqe_quantize_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P]),
     "minw_pack_weight_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
+    "aqe_quantize_codes_e2m1": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P]),
+    "minw_pack_weight_codes_e2m1": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
     "minw_conv2d_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32,
                                          _I32, _I32, _P, _P, _P, _P, _P]),
     "minw_conv_block_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32,
@@ -308,6 +312,18 @@ def minw_pack_weight_codes(w, q, codes, channel_scale=None, stream=None):
                                         _ptr(codes), _stream(stream)), "minw_pack_weight_codes")
 
 
+def aqe_quantize_codes_e2m1(x, q, codes, stream=None):
+    B, C, H, W = x.shape
+    _check(lib().aqe_quantize_codes_e2m1(_ptr(x), B, C, H, W, ctypes.byref(q), _ptr(codes), _stream(stream)),
+           "aqe_quantize_codes_e2m1")
+
+
+def minw_pack_weight_codes_e2m1(w, q, codes, channel_scale=None, stream=None):
+    O, C, kh, kw = w.shape
+    _check(lib().minw_pack_weight_codes_e2m1(_ptr(w), O, C, kh, kw, ctypes.byref(q), _ptr(channel_scale),
+                                             _ptr(codes), _stream(stream)), "minw_pack_weight_codes_e2m1")
+
+
 def minw_conv2d_codes(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad, acc_out=None,
                       scale=None, shift=None, y_out=None, stream=None):
     _check(lib().minw_conv2d_codes(_ptr(act), B, C, H, W, bits_a, _ptr(wgt), O, kh, kw, bits_w, stride, pad,
@@ -326,12 +342,15 @@ def minw_conv_block_codes(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, strid
 
 def minw_conv_block_codes_ex(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad, pool, scale, shift,
                              q_out=None, codes_out=None, planes_out=None, y_out=None, res_codes=None, res_bits=0,
-                             res_f32=None, y_nhwc=None, stream=None):
+                             res_f32=None, y_nhwc=None, in_format=CODES_E4M3, out_format=CODES_E4M3,
+                             res_format=CODES_E4M3, acc_out=None, stream=None):
     ex = BlockExtra()
     ex.res_codes = res_codes.data_ptr() if res_codes is not None else None
     ex.res_bits = int(res_bits)
     ex.res_f32 = res_f32.data_ptr() if res_f32 is not None else None
     ex.y_nhwc = y_nhwc.data_ptr() if y_nhwc is not None else None
+    ex.in_format, ex.out_format, ex.res_format = int(in_format), int(out_format), int(res_format)
+    ex.acc_out = acc_out.data_ptr() if acc_out is not None else None
     _check(lib().minw_conv_block_codes_ex(_ptr(act), B, C, H, W, bits_a, _ptr(wgt), O, kh, kw, bits_w, stride, pad,
                                           int(pool), _ptr(scale), _ptr(shift),
                                           ctypes.byref(q_out) if q_out is not None else None, _ptr(codes_out),
@@ -456,7 +475,8 @@ class Net:
         return list(arr)
 
     def layer_variants(self):
-        """Kernel per layer: 0 fp32 first layer, VARIANT_POPC or VARIANT_TC."""
+        """Kernel per layer: 0 fp32 first layer, VARIANT_POPC, VARIANT_TC (E4M3
+        operands) or VARIANT_TC_E2M1."""
         n = self.launches
         arr = (ctypes.c_int32 * n)()
         _check(lib().minw_net_layer_variants(self._h, arr), "minw_net_layer_variants")
