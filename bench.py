@@ -68,7 +68,35 @@ def _captured_traffic(bound):
         return cap["dram_bytes_per_launch"]
     except (OSError, KeyError, ValueError):
         return None
-FP8_TFLOPS = 2.0 * BF16_TFLOPS
+FP8_TFLOPS = 2.0 * BF16_TFLOPS        # nominal dense FP8 / bf16 = 4.5 / 2.25
+FP4_TFLOPS = 6.0 * BF16_TFLOPS        # nominal dense FP4 / bf16 = 13.5 / 2.25
+# tcgen05 rates this repository's pipe probe measured on GB300 (one CTA per SM,
+# warp-uniform issue, M = 128, N = 256; bench.py --workload peaks re-measures them)
+PROBE_TFLOPS = {"e4m3": 4826.0, "e2m1": 9673.0, "bf16": 2418.0}
+
+
+def tensor_roofline(ops, kinds, ms):
+    """Roofline of quantized layers on the tensor cores, each at the peak of its
+    own operand kind ("e4m3" or "e2m1"): the time the layers would take at
+    those peaks over the time they took.  Returns the roofline dict."""
+    peak_of = {"e4m3": FP8_TFLOPS, "e2m1": FP4_TFLOPS}
+    t_ms = sum(ms)
+    t_roof = sum(o / (peak_of[k] * 1e12) for o, k in zip(ops, kinds)) * 1e3
+    t_probe = sum(o / (PROBE_TFLOPS[k] * 1e12) for o, k in zip(ops, kinds)) * 1e3
+    achieved = sum(ops) / (t_ms * 1e-3) / 1e12
+    names = sorted(set(kinds))
+    return {"bound": "tensor",
+            "kernel": "conv_tc_kernel (tcgen05 " + " + ".join(
+                {"e4m3": "kind::f8f6f4 E4M3", "e2m1": "kind::mxf4 E2M1"}[k] for k in names) + ")",
+            "achieved": achieved, "peak": sum(ops) / (t_roof * 1e-3) / 1e12, "unit": "TFLOP/s",
+            "frac": t_roof / t_ms, "traffic": None,
+            "peak_basis": f"per layer: measured dense bf16 {BF16_TFLOPS:.1f} TFLOP/s (burst) x 2 for E4M3 and x 6 for "
+                          "E2M1 layers (nominal FP8/FP4 to bf16 ratios), of measured",
+            "peak_probe": sum(ops) / (t_probe * 1e-3) / 1e12,
+            "frac_probe": t_probe / t_ms,
+            "probe_basis": "per layer: the tcgen05 rate of its kind measured by this repository's pipe probe "
+                           "(E4M3 4826, E2M1 9673 TFLOP/s at N = 256)",
+            "layer_kinds": kinds}
 
 
 L2_NOTE = "flushed between steps (256 MiB write outside the timed events)"
@@ -419,14 +447,12 @@ def run_gpu(args, rank, world, local_rank):
     q_ms = float(sum(layer_ms[i] for i in q_ops_idx))
     q_ops = 2.0 * sum(macs[i] for i in q_ops_idx) * BATCH
     achieved = q_ops / (q_ms * 1e-3) / 1e12
-    all_tc = all(variants[i] == minw.VARIANT_TC for i in q_ops_idx)
+    tc_kind = {minw.VARIANT_TC: "e4m3", minw.VARIANT_TC_E2M1: "e2m1"}
+    all_tc = all(variants[i] in tc_kind for i in q_ops_idx)
     if all_tc:
-        peak = FP8_TFLOPS
-        roofline = {"bound": "tensor", "kernel": "conv_tc_kernel (tcgen05 kind::f8f6f4, all quantized layers)",
-                    "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
-                    "traffic": None,
-                    "peak_basis": f"measured dense bf16 {BF16_TFLOPS:.1f} TFLOP/s (burst) x 2 for FP8 "
-                                  "(nominal fp8/bf16 ratio), of measured"}
+        roofline = tensor_roofline([2.0 * macs[i] * BATCH for i in q_ops_idx],
+                                   [tc_kind[variants[i]] for i in q_ops_idx],
+                                   [float(layer_ms[i]) for i in q_ops_idx])
     else:
         peak = POPC_PER_CLK_SM * 32 * 2 * SMS * SM_MAX_MHZ * 1e6 / 1e12
         roofline = {"bound": "alu", "kernel": "conv_popc_kernel (all quantized layers)",
@@ -444,7 +470,8 @@ def run_gpu(args, rank, world, local_rank):
 
     line = {"metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "e4m3" if all_tc else "b1",
+            "vs_baseline": None,
+            "dtype": ("+".join(sorted(set(roofline["layer_kinds"]))) if all_tc else "b1"),
             "data": "synthetic",
             "config": wl.config(world),
             "eff_tops": eff_tops,

@@ -385,6 +385,9 @@ MINW_API minw_status minw_conv_block_codes_ex(const uint8_t *act, int32_t B, int
  * concurrently.  With a split the call launches a second kernel that sums
  * the K slices and runs the epilogue. */
 MINW_API size_t minw_fc_workspace_bytes(int32_t B, int32_t K, int32_t O);
+/* K slices minw_fc_codes uses for this shape with a workspace of
+ * workspace_bytes (1: no split; 0: shape not supported).  Host-only query. */
+MINW_API int32_t minw_fc_ksplit(int32_t B, int32_t K, int32_t O, size_t workspace_bytes);
 MINW_API minw_status minw_fc_codes(const uint8_t *act, int32_t B, int32_t K, int32_t bits_a,
                                    const uint8_t *wgt, int32_t O, int32_t bits_w,
                                    const float *scale, const float *shift,
@@ -402,7 +405,10 @@ MINW_API minw_status minw_fc_codes(const uint8_t *act, int32_t B, int32_t K, int
  * allocates nothing (no cudaMalloc/cudaFree, no allocating library routine).
  * - The first call on each device looks up the array's device address
  *   (cudaGetSymbolAddress, with that device current); make that first call
- *   before any stream capture.
+ *   before any stream capture.  The address is kept for the life of the
+ *   process: after cudaDeviceReset (or anything else that ends the device's
+ *   primary context) it is stale, so a process that resets a device must not
+ *   call this entry point again on that device.
  * - Every call shares the one array.  Nothing in it needs to start at zero
  *   (each call overwrites what it reads) and it keeps the last call's
  *   contents; calls that overlap on the GPU (other streams, other threads)
@@ -540,6 +546,65 @@ MINW_API void minw_net_destroy(minw_net *net);
 /* Reads and clears the device error flag after synchronising `stream`:
  * MINW_OK, or MINW_ETIMEOUT when a bounded wait inside a kernel gave up. */
 MINW_API minw_status minw_get_last_device_error(void *stream);
+
+/* ---------------------------------------------------------------------- */
+/* Plan options (process-wide; no counterpart in the paper)                 */
+/* ---------------------------------------------------------------------- */
+
+/* Choices between kernel variants that compute the same results, and the
+ * limit of the kernels' bounded waits.  The defaults (1, 1, 2, 1, 2, 1, 1, 1,
+ * 1, 1, 2^31) are the measured fastest variants.  The options are read when a
+ * launch is planned: a change applies to standalone calls made after it and
+ * to networks created after it (a network keeps the plan it was created
+ * with, except pdl and graph, read at every forward).
+ * - cta_pairs: 256-channel layers with long K loops as CTA pairs (cta_group::2).
+ * - channel_major: 64- and 128-channel layers as 128-channel x 256-pixel tiles
+ *   when at least channel_major_min_tiles_per_sm such tiles per SM exist.
+ * - dup_weights: a 64-channel channel-major tile loads its weight rows twice
+ *   (else pads with zero rows).
+ * - kblocks_per_stage: K blocks per pipeline stage of the tensor-core kernel (1 or 2).
+ * - first_tma: first-layer input patches by TMA boxes (else per-word copies).
+ * - pdl: programmatic dependent launch between the kernels of a forward.
+ * - graph: minw_forward replays a captured CUDA graph.
+ * - tma_lanes: lanes of each TMA warp of the tensor-core kernel that issue
+ *   loads (1 to 8; each load keeps its issuing thread busy for about an L2
+ *   round trip, so more issuers keep more bytes in flight).
+ * - resident_weights: a tensor-core layer not split along K whose weights fit
+ *   in shared memory keeps them there for all of its tiles (each CTA then
+ *   works on one channel tile) instead of loading them per tile.
+ * - wait_cycles: SM clocks after which a bounded wait (TMA load, MMA, TMEM
+ *   hand-off) gives up; the kernel then finishes without its outputs and
+ *   minw_get_last_device_error reports MINW_ETIMEOUT. */
+typedef struct {
+    int32_t cta_pairs;
+    int32_t channel_major;
+    int32_t channel_major_min_tiles_per_sm;
+    int32_t dup_weights;
+    int32_t kblocks_per_stage;
+    int32_t first_tma;
+    int32_t pdl;
+    int32_t graph;
+    int32_t tma_lanes;
+    int32_t resident_weights;
+    int64_t wait_cycles;
+} minw_plan_options;
+
+/* Current options (host struct). */
+MINW_API minw_status minw_get_plan_options(minw_plan_options *out);
+/* Replace the options; NULL restores the defaults.  MINW_EINVAL on a
+ * kblocks_per_stage other than 1 or 2, tma_lanes outside 1..8 or a
+ * non-positive wait_cycles. */
+MINW_API minw_status minw_set_plan_options(const minw_plan_options *opt);
+
+/* Test hook of the timeout path (no counterpart in the paper): the next launch
+ * of the named kernel -- MINW_STALL_CONV_TC, the single-CTA tensor-core
+ * convolution, or MINW_STALL_CONV_FIRST, the first layer with TMA patches --
+ * first waits on a barrier that nothing completes.  That wait runs out after
+ * wait_cycles, the kernel skips its work, drains its own loads and frees its
+ * tensor memory, and minw_get_last_device_error reports MINW_ETIMEOUT once.
+ * One launch only; 0 cancels a pending request.  No GPU fault is involved. */
+enum { MINW_STALL_CONV_TC = 1, MINW_STALL_CONV_FIRST = 2 };
+MINW_API minw_status minw_test_stall_next_launch(int32_t kernel);
 
 #ifdef __cplusplus
 }

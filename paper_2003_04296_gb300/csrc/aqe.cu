@@ -476,15 +476,6 @@ int num_sms() {
     return sms;
 }
 
-bool pdl_enabled() {
-    static int v = -1;
-    if (v < 0) {
-        const char *e = getenv("MINW_PDL");
-        v = (e && e[0] == '0') ? 0 : 1;
-    }
-    return v == 1;
-}
-
 minw_status launch_status() {
     return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
 }

@@ -324,7 +324,9 @@ bool aligned16(const void *p);
 bool valid_quant(const minw_quant *q);
 int num_sms();
 minw_status launch_status();
-bool pdl_enabled();                 // MINW_PDL=0 turns programmatic dependent launch off
+bool pdl_enabled();                 // plan option pdl
+minw_plan_options plan_options();   // the process-wide plan options (runtime.cu)
+int take_stall(int which);          // 1 once after minw_test_stall_next_launch(which)
 
 // cuTensorMapEncodeTiled from the driver (nullptr when it is unavailable).
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,

@@ -257,6 +257,17 @@ size_t minw_fc_workspace_bytes(int32_t B, int32_t K, int32_t O) {
     return conv_tc_workspace_bytes(a);
 }
 
+int32_t minw_fc_ksplit(int32_t B, int32_t K, int32_t O, size_t workspace_bytes) {
+    if (B <= 0 || K <= 0 || O <= 0 || K % 128 != 0) return 0;
+    ConvArgs a{};
+    a.B = B; a.C = K; a.H = 1; a.W = 1; a.O = O; a.kh = 1; a.kw = 1; a.stride = 1; a.pad = 0;
+    a.Ho = 1; a.Wo = 1; a.NW = K / 32; a.M = B;
+    a.y_out = reinterpret_cast<float *>(256);           // shape planning only: never dereferenced
+    a.workspace = workspace_bytes ? reinterpret_cast<void *>(256) : nullptr;
+    a.workspace_bytes = workspace_bytes;
+    return conv_tc_ksplit(a);
+}
+
 minw_status minw_fc_codes(const uint8_t *act, int32_t B, int32_t K, int32_t bits_a, const uint8_t *wgt, int32_t O,
                           int32_t bits_w, const float *scale, const float *shift, const minw_quant *q_out,
                           uint8_t *codes_out, uint32_t *planes_out, float *y_out, int32_t *acc_out,

@@ -61,8 +61,6 @@ __device__ __forceinline__ void lds_2x64(uint32_t a, unsigned long long &x, unsi
 // kernels' flag by minw_get_last_device_error).
 __device__ int g_first_error = 0;
 
-constexpr long long FIRST_WAIT_CYCLES = 1ll << 31;
-
 __device__ __forceinline__ uint32_t saddr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
 __device__ __forceinline__ void fbar_init(uint64_t *bar) {
@@ -79,12 +77,13 @@ __device__ __forceinline__ bool fbar_try_wait(uint64_t *bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Bounded wait for a patch: false (and the error flag set) after about a second.
-__device__ __forceinline__ bool fbar_wait(uint64_t *bar, uint32_t parity) {
+// Bounded wait for a patch: false (and the error flag set) after limit SM
+// clocks (about a second by default).
+__device__ __forceinline__ bool fbar_wait(uint64_t *bar, uint32_t parity, long long limit) {
     if (fbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     while (!fbar_try_wait(bar, parity)) {
-        if (clock64() - t0 > FIRST_WAIT_CYCLES) {
+        if (clock64() - t0 > limit) {
             atomicExch(&g_first_error, 1);
             return false;
         }
@@ -144,7 +143,7 @@ static FirstTile first_tile(const FirstArgs &a, bool tma) {
     t.xoff = (t.K * t.OCB + t.OCB * 8 + 31) / 32 * 32;
     t.pstride = (a.C * t.Rmax * t.RP + 31) / 32 * 32;
     // three patch buffers (two tiles of look-ahead) where two CTAs still fit on an SM
-    const size_t fixed = sizeof(float) * (size_t)t.xoff + 3 * sizeof(uint64_t);
+    const size_t fixed = sizeof(float) * (size_t)t.xoff + 4 * sizeof(uint64_t);   // nb patch barriers + the stall test's
     const size_t pbytes = sizeof(float) * (size_t)t.pstride;
     t.nb = fixed + 3 * pbytes <= 112 * 1024 ? 3 : 2;
     t.smem = fixed + t.nb * pbytes;
@@ -192,7 +191,9 @@ __global__ void __launch_bounds__(FIRST_NT, 2)
     float *sW = reinterpret_cast<float *>(smem4);                 // [K][OCB]
     float *sT = sW + (size_t)K * OCB;                             // [8][OCB] -breakpoints, sigma (row 7)
     float *sX0 = sW + tl.xoff;                                    // [nb][C][Rmax][RP]
-    uint64_t *fullb = reinterpret_cast<uint64_t *>(sX0 + (size_t)tl.nb * patch);   // [nb] TMA patch arrivals
+    uint64_t *fullb = reinterpret_cast<uint64_t *>(sX0 + (size_t)tl.nb * patch);   // [nb] TMA patch arrivals, then
+                                                                                  // the timeout test's barrier
+    int issued[3] = {0, 0, 0}, landed[3] = {0, 0, 0};       // TMA patches per buffer (thread 0 issues them all)
 
     const int o0 = blockIdx.y * OCB;
     const int ochan = min(OCB, a.O - o0);
@@ -208,6 +209,7 @@ __global__ void __launch_bounds__(FIRST_NT, 2)
         if constexpr (TM) {       // one thread: the whole patch as one box
             patch_tma(sX0 + buf * patch, &tmX, &fullb[buf], (uint32_t)(sizeof(float) * a.C * tl.Rmax * RP), tl.x0,
                       (p0 / a.Wo) * st - a.pad, b);
+            ++issued[buf];
             return;
         }
         const int pend = min(p0 + tl.PB, npix);
@@ -270,7 +272,7 @@ __global__ void __launch_bounds__(FIRST_NT, 2)
     }
 
     if (TM && threadIdx.x == 0) {
-        for (int j = 0; j < tl.nb; ++j) fbar_init(&fullb[j]);
+        for (int j = 0; j <= tl.nb; ++j) fbar_init(&fullb[j]);
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     __syncthreads();                                             // barriers initialised
@@ -290,6 +292,8 @@ __global__ void __launch_bounds__(FIRST_NT, 2)
         }
     }
     bool dead = false;                                           // a patch wait ran out: skip the work
+    // timeout-path test: a wait on a barrier that nothing completes runs out
+    if (TM && a.stall && !fbar_wait(&fullb[tl.nb], 0u, a.wait_cycles)) dead = true;
     const int g = warp % tl.groups, pb = warp / tl.groups;
     const int h = lane >> 4, l16 = lane & 15;
     const int NWo = (a.O + 31) >> 5;
@@ -303,7 +307,12 @@ __global__ void __launch_bounds__(FIRST_NT, 2)
         const int bn = buf == 0 ? nb - 1 : buf - 1;              // the slot tile t - G used
         if constexpr (TM) {
             if (tn < total && threadIdx.x == 0 && !dead) load_patch(tn, bn);
-            if (!dead && !fbar_wait(&fullb[buf], (uint32_t)(it / nb) & 1u)) dead = true;
+            if (!dead) {
+                if (fbar_wait(&fullb[buf], (uint32_t)(it / nb) & 1u, a.wait_cycles))
+                    ++landed[buf];
+                else
+                    dead = true;
+            }
         } else {
             if (tn < total)
                 load_patch(tn, bn);
@@ -439,6 +448,13 @@ __global__ void __launch_bounds__(FIRST_NT, 2)
         }
         __syncthreads();                                         // buffer buf is free for tile t + nb G
     }
+    // a run that gave up leaves patches in flight: every one lands before the CTA exits
+    if (TM && threadIdx.x == 0)
+        for (int j = 0; j < tl.nb; ++j)
+            while (landed[j] < issued[j]) {
+                if (!fbar_wait(&fullb[j], (uint32_t)landed[j] & 1u, a.wait_cycles)) break;
+                ++landed[j];
+            }
 }
 
 // Weights of a first layer prepared once: [K][O] (output channel fastest),
@@ -501,7 +517,10 @@ static minw_status launch_first_shape(const FirstArgs &a, const FirstTile &tl, c
     int gx = (2 * sms + octiles - 1) / octiles;
     if (gx > total) gx = total;
     const dim3 grid((unsigned)gx, (unsigned)octiles);
-    if (minw_host::launch_pdl(kern, grid, dim3(FIRST_NT), tl.smem, s, a, tl, tm) != cudaSuccess) return MINW_ECUDA;
+    FirstArgs ar = a;
+    ar.wait_cycles = (long long)minw_host::plan_options().wait_cycles;
+    ar.stall = TM ? minw_host::take_stall(MINW_STALL_CONV_FIRST) : 0;
+    if (minw_host::launch_pdl(kern, grid, dim3(FIRST_NT), tl.smem, s, ar, tl, tm) != cudaSuccess) return MINW_ECUDA;
     return MINW_OK;
 }
 
@@ -520,16 +539,10 @@ static minw_status launch_first_bits(const FirstArgs &a, const FirstTile &tl, co
     return launch_first_shape<OUTB, 0, 0, 0, false>(a, tl, tm, s);
 }
 
-// Patches by TMA (MINW_FIRST_TMA=0: per-word cp.async) where the image rows
-// are 16-byte multiples at a 16-byte aligned base and the box fits the limits.
-static bool first_tma_pref() {
-    static int v = -1;
-    if (v < 0) {
-        const char *e = getenv("MINW_FIRST_TMA");
-        v = (e && e[0] == '0') ? 0 : 1;
-    }
-    return v != 0;
-}
+// Patches by TMA (plan option first_tma; else per-word cp.async) where the
+// image rows are 16-byte multiples at a 16-byte aligned base and the box fits
+// the limits.
+static bool first_tma_pref() { return minw_host::plan_options().first_tma != 0; }
 
 int take_first_error() {
     int flag = 0;

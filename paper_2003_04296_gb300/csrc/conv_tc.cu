@@ -48,7 +48,6 @@ constexpr int NT = 352;                 // 11 warps: TMA (A), MMA, 8 epilogue, T
 constexpr int EPI_WARPS = 8;            // two per TMEM lane quarter, each half of the columns
 constexpr int B_WARP = 2 + EPI_WARPS;   // the weight-box TMA warp
 
-constexpr long long WAIT_CYCLES = 1ll << 31;
 
 struct Params {
     int B, C, H, W, O, kh, kw, pad, Ho, Wo;
@@ -101,6 +100,13 @@ struct Params {
     int nacc;                  // TMEM accumulators: 2 (the epilogue of one tile overlaps the MMAs of the
                                // next) or 1 (E2M1 tiles of 256 columns: the scale factors take the rest)
     uint32_t sf_col;           // E2M1 operands: TMEM column of A's unit scale factors (B's at + 32)
+    long long wait_cycles;     // limit of every bounded wait (SM clocks)
+    int tlanes;                // lanes of each TMA warp that issue loads (stage g belongs to lane g % tlanes)
+    int wres;                  // resident weights: each CTA (pair) keeps one channel tile and holds all of its
+                               // weight K blocks in shared memory, loaded once; the ring carries activations
+                               // only, issued by both TMA warps in turn (no K split)
+    uint32_t wres_off;         // byte offset of the resident weights from the shared-memory base
+    int stall;                 // timeout-path test: the MMA issuer first waits on a barrier nothing completes
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -127,14 +133,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
 }
 
 // Bounded wait for the phase with the given parity; false (and the device
-// error flag set) when it does not complete within WAIT_CYCLES.  Each
+// error flag set) when it does not complete within limit SM clocks.  Each
 // try_wait may suspend the thread up to 100 us (the hint) until the phase
 // completes, so waiting warps do not take issue slots from the MMA thread.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, long long limit) {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     while (!mbar_try_wait(bar, parity)) {
-        if (clock64() - t0 > WAIT_CYCLES) {
+        if (clock64() - t0 > limit) {
             atomicExch(&g_device_error, 1);
             return false;
         }
@@ -297,7 +303,7 @@ __device__ __forceinline__ void tma_load_2d_pair(void *dst, const CUtensorMap *m
 }
 
 // Bounded wait with cluster-scope acquire (arrivals from the other CTA of a pair).
-__device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity, long long limit) {
     const long long t0 = clock64();
     while (true) {
         uint32_t ok;
@@ -308,7 +314,7 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity
             : "r"(smem_u32(bar)), "r"(parity)
             : "memory");
         if (ok) return true;
-        if (clock64() - t0 > WAIT_CYCLES) {
+        if (clock64() - t0 > limit) {
             atomicExch(&g_device_error, 1);
             return false;
         }
@@ -524,6 +530,21 @@ __device__ __forceinline__ void resid_chunk(uint32_t taddr, bool full32, const P
     }
 }
 
+// Work item n (0, 1, ...) of this CTA, or -1 past its last: an (output tile,
+// K slice) index w (tile t = w / ksplit, tile t = tn * tiles_m + tm).  By
+// default CTA b takes w = b, b + grid, ...; with resident weights, unit u
+// (a CTA, or a pair) keeps channel tile tn = u % ntn and walks its pixel
+// tiles (the pair's two CTAs on adjacent ones).
+__device__ __forceinline__ int cta_item(const Params &p, int n, int items, int tiles_m, int crank) {
+    if (!p.wres) {
+        const int w = (int)blockIdx.x + n * (int)gridDim.x;
+        return w < items ? w : -1;
+    }
+    const int units = (int)gridDim.x / p.cl, upt = units / p.ntn, u = (int)blockIdx.x / p.cl;
+    const int tm = (u / p.ntn + n * upt) * p.cl + crank;
+    return tm < tiles_m ? (u % p.ntn) * tiles_m + tm : -1;
+}
+
 // OUTB: bits of the quantized output (0 when the launch writes none).
 // PAIR: CTA pairs with cta_group::2 MMAs (a kernel uses one CTA group only).
 // FMT: operand format -- 0 E4M3 level codes (kind::f8f6f4), 1 bf16 (kind::f16),
@@ -627,7 +648,8 @@ __global__ void __launch_bounds__(NT, 1)
     // breakpoints [NL][O32] (channels padded to a multiple of 32, channel
     // fastest), then the per-32-channel masks of channels with sigma = +1
     const int O32 = (p.O + 31) & ~31;
-    float *sthr = reinterpret_cast<float *>(smem + (size_t)p.S * p.stage_bytes);
+    float *sthr = reinterpret_cast<float *>(smem + (size_t)p.S * p.stage_bytes +
+                                            (p.wres ? (size_t)p.nk * p.b_bytes : 0));   // after the resident weights
     const int thr_floats = OUTB ? O32 * NL : 0;
     uint32_t *ssig = reinterpret_cast<uint32_t *>(sthr + thr_floats);              // [O32 / 32]
     const int sig_words = OUTB ? O32 / 32 : 0;
@@ -640,7 +662,9 @@ __global__ void __launch_bounds__(NT, 1)
     uint64_t *empty = full + p.S;
     uint64_t *tfull = empty + p.S;            // [2] accumulator ready
     uint64_t *tempty = tfull + 2;             // [2] accumulator drained
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(tempty + 2);
+    uint64_t *tstall = tempty + 2;            // timeout-path test: a barrier nothing completes
+    uint64_t *wfull = tstall + 1;             // resident weights landed
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(wfull + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // pixel tiles padded to a multiple of the cluster size: the CTAs of a
@@ -653,13 +677,15 @@ __global__ void __launch_bounds__(NT, 1)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < p.S; ++s) {
-            mbar_init(&full[s], 2);               // one arrival per TMA issuing warp (pairs: CTA 0's)
+            mbar_init(&full[s], p.wres ? 1 : 2);  // one arrival per TMA warp loading the stage (pairs: CTA 0's)
             mbar_init(&empty[s], 1);              // one release per slot (pairs: CTA 0 commits to both CTAs)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
             mbar_init(&tempty[i], PAIR ? 2 * EPI_WARPS : EPI_WARPS);   // pairs: both CTAs' epilogues
         }
+        mbar_init(tstall, 1);
+        mbar_init(wfull, 1);
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     if (warp == 1) {
@@ -745,20 +771,45 @@ __global__ void __launch_bounds__(NT, 1)
     pdl_trigger();                            // set-up done: the next kernel may start its own
 
     if (warp == 0 || warp == B_WARP) {
-        if (lane == 0) {
-            // ---------------- TMA producers: warp 0 activations, warp 6 weights ----------------
-            const bool act = warp == 0;
-            if (act) pdl_wait();                  // activations come from the previous kernel
+        if (lane < p.tlanes) {
+            // ---------------- TMA producers: warp 0 activations, warp 10 weights ----------------
+            // Lane l of a warp owns the pipeline stages g with g % tlanes == l
+            // (own slot waits, own arrival on the stage's barrier).  With resident
+            // weights, warp 10 first loads every weight K block of its channel
+            // tile once, then both warps issue activation stages in turn.
+            const bool wwarp = warp == B_WARP;
+            const bool act = !wwarp || p.wres;     // this warp issues activation boxes
             const CUtensorMap *map = act ? &tmA : &tmB;
-            asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
-            const uint32_t bytes = act ? p.a_bytes : p.b_bytes;   // per K block; weights: all cl slices
+            if (lane == 0) asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+            const uint32_t bytes = act ? p.a_bytes : p.b_bytes;   // per K block
             const int bslice = PAIR ? p.BN / 2 : p.BN;   // weight rows this CTA loads
             // pairs: this operand's loads of both CTAs complete on CTA 0's barrier, whose
             // producers alone arrive (expecting both CTAs' bytes)
             const bool arrive = !PAIR || crank == 0;
-            int g = 0, s = 0, lap = 0;             // stages issued, ring slot, ring lap
+            const int nissue = p.wres ? 2 * p.tlanes : p.tlanes;          // issuers of this operand
+            const int myid = (p.wres && wwarp) ? p.tlanes + lane : lane;
+            if (p.wres && wwarp && lane == 0) {
+                // the channel tile's weights, all K blocks, once
+                const int o0 = (((int)blockIdx.x / p.cl) % p.ntn) * p.BN;
+                uint8_t *wres = smem + p.wres_off;
+                if (arrive) mbar_expect_tx(wfull, (uint32_t)p.nk * p.b_bytes * (PAIR ? 2u : 1u));
+                const uint32_t fb = PAIR ? cta0_addr(wfull) : 0u;
+                for (int kb = 0; kb < p.nk; ++kb) {
+                    const int kx_ = FMT == 2 ? (kb * p.ck) >> 1 : kb * p.ck;
+                    uint8_t *sb = wres + (size_t)kb * p.b_bytes;
+                    if constexpr (PAIR) {
+                        tma_load_2d_pair(sb, &tmB, fb, kx_, o0 + crank * bslice);
+                    } else {
+                        tma_load_2d(sb, &tmB, wfull, kx_, o0);
+                        if (p.dup) tma_load_2d(sb + (size_t)64 * p.cb, &tmB, wfull, kx_, o0);
+                    }
+                }
+            }
+            if (act) pdl_wait();                  // activations come from the previous kernel
+                                                  // (the weights above do not: they load before)
+            int g = 0, s = 0, lap = 0;             // stages walked, ring slot, ring lap
             bool alive = true;
-            for (int w = blockIdx.x; w < items && alive; w += gridDim.x) {
+            for (int n = 0, w; alive && (w = cta_item(p, n, items, tiles_m, crank)) >= 0; ++n) {
                 const int t = w / p.ksplit, kp = w - t * p.ksplit;
                 const int kb = (int)((long long)kp * p.nk / p.ksplit), ke = (int)((long long)(kp + 1) * p.nk / p.ksplit);
                 const int tn = t / tiles_m, tm = t - tn * tiles_m;
@@ -770,27 +821,30 @@ __global__ void __launch_bounds__(NT, 1)
                 int c0 = (kb - tap0 * p.nck) * p.ck, ky = tap0 / p.kw, kx = tap0 - (tap0 / p.kw) * p.kw;
                 int kcol = kb * p.ck;
                 for (int ks = kb; ks < ke; ks += p.kps, ++g) {
+                    const bool mine = g % nissue == myid;
                     // slot reuse: wait until the MMAs of the previous lap released it
-                    if (lap > 0 && !mbar_wait(&empty[s], (lap - 1) & 1)) { alive = false; break; }
+                    if (mine && lap > 0 && !mbar_wait(&empty[s], (lap - 1) & 1, p.wait_cycles)) { alive = false; break; }
                     uint8_t *sa = smem + (size_t)s * p.stage_bytes;
-                    const int n = min(p.kps, ke - ks);            // K blocks in this stage
-                    if (arrive) mbar_expect_tx(&full[s], (uint32_t)n * bytes * (PAIR ? 2u : 1u));
-                    const uint32_t fb = PAIR ? cta0_addr(&full[s]) : 0u;
-                    for (int j = 0; j < n; ++j) {
+                    const int nb = min(p.kps, ke - ks);           // K blocks in this stage
+                    if (mine && arrive) mbar_expect_tx(&full[s], (uint32_t)nb * bytes * (PAIR ? 2u : 1u));
+                    const uint32_t fb = (PAIR && mine) ? cta0_addr(&full[s]) : 0u;
+                    for (int j = 0; j < nb; ++j) {
                         // tensor-map x coordinates: elements, or bytes for packed E2M1
                         const int cx = FMT == 2 ? c0 >> 1 : c0, kx_ = FMT == 2 ? kcol >> 1 : kcol;
-                        if constexpr (PAIR) {
-                            if (act)
-                                tma_load_4d_pair(sa + (size_t)j * p.a_bytes, &tmA, fb, cx, x0 + kx, y0 + ky, b0);
-                            else
-                                tma_load_2d_pair(sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes, &tmB, fb,
-                                                 kx_, o0 + crank * bslice);
-                        } else if (act)
-                            tma_load_4d(sa + (size_t)j * p.a_bytes, &tmA, &full[s], cx, x0 + kx, y0 + ky, b0);
-                        else {
-                            uint8_t *sb = sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes;
-                            tma_load_2d(sb, &tmB, &full[s], kx_, o0);
-                            if (p.dup) tma_load_2d(sb + (size_t)64 * p.cb, &tmB, &full[s], kx_, o0);
+                        if (mine) {
+                            if constexpr (PAIR) {
+                                if (act)
+                                    tma_load_4d_pair(sa + (size_t)j * p.a_bytes, &tmA, fb, cx, x0 + kx, y0 + ky, b0);
+                                else
+                                    tma_load_2d_pair(sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes, &tmB, fb,
+                                                     kx_, o0 + crank * bslice);
+                            } else if (act)
+                                tma_load_4d(sa + (size_t)j * p.a_bytes, &tmA, &full[s], cx, x0 + kx, y0 + ky, b0);
+                            else {
+                                uint8_t *sb = sa + (size_t)p.kps * p.a_bytes + (size_t)j * p.b_bytes;
+                                tma_load_2d(sb, &tmB, &full[s], kx_, o0);
+                                if (p.dup) tma_load_2d(sb + (size_t)64 * p.cb, &tmB, &full[s], kx_, o0);
+                            }
                         }
                         kcol += p.ck;
                         c0 += p.ck;
@@ -802,11 +856,14 @@ __global__ void __launch_bounds__(NT, 1)
                     if (++s == p.S) { s = 0; ++lap; }
                 }
             }
-            // drain: every issued load has landed before the CTA can exit (pairs: the
-            // MMAs that read the last stages have completed)
+            // drain: every load this lane issued has landed before the CTA can exit
+            // (pairs: the MMAs that read the last stages have completed)
             for (int j = g > p.S ? g - p.S : 0; j < g; ++j)
-                if (!(PAIR ? mbar_wait(&empty[j % p.S], (j / p.S) & 1) : mbar_wait(&full[j % p.S], (j / p.S) & 1)))
+                if (j % nissue == myid &&
+                    !(PAIR ? mbar_wait(&empty[j % p.S], (j / p.S) & 1, p.wait_cycles)
+                           : mbar_wait(&full[j % p.S], (j / p.S) & 1, p.wait_cycles)))
                     break;
+            if (p.wres && wwarp && lane == 0 && (!PAIR || crank == 0)) mbar_wait(wfull, 0u, p.wait_cycles);
         }
     } else if (warp == 1) {
         if (!PAIR || crank == 0) {
@@ -820,17 +877,24 @@ __global__ void __launch_bounds__(NT, 1)
             // descriptors advance by a constant per ring slot, the K = 32 steps are unrolled
             const uint32_t sbase = smem_u32(smem);
             const uint64_t adesc0 = sw_desc(sbase, p.cb), bdesc0 = sw_desc(sbase + p.kps * p.a_bytes, p.cb);
+            const uint64_t wdesc0 = sw_desc(sbase + p.wres_off, p.cb);     // resident weights, K block 0
             const uint32_t dstep = p.stage_bytes >> 4;     // start-address step of one ring slot
             const uint32_t astep = p.a_bytes >> 4, bstep = p.b_bytes >> 4;   // second K block of a stage
             const bool k128 = p.cb == 128;                 // four 32-byte K steps per K block, else two
             const uint32_t idesc = p.idesc;
             const uint32_t sfa = tmem_base + p.sf_col, sfb = sfa + 32u;
-            for (int w = blockIdx.x; w < items && alive; w += gridDim.x, ++i) {
+            // timeout-path test (single CTAs): a wait that runs out; every other
+            // warp's next wait then runs out too, and the kernel winds down
+            if (!PAIR && p.stall && !__all_sync(0xffffffffu, mbar_wait(tstall, 0u, p.wait_cycles))) alive = false;
+            if (p.wres && alive && !__all_sync(0xffffffffu, PAIR ? mbar_wait_cluster(wfull, 0u, p.wait_cycles)
+                                                                 : mbar_wait(wfull, 0u, p.wait_cycles)))
+                alive = false;
+            for (int n = 0, w; alive && (w = cta_item(p, n, items, tiles_m, crank)) >= 0; ++n, ++i) {
                 const int ab = p.nacc == 2 ? (i & 1) : 0, use = p.nacc == 2 ? (i >> 1) : i;
                 const int t = w / p.ksplit, kp = w - t * p.ksplit;
                 const int kb = (int)((long long)kp * p.nk / p.ksplit), ke = (int)((long long)(kp + 1) * p.nk / p.ksplit);
-                if (use > 0 && !__all_sync(0xffffffffu, PAIR ? mbar_wait_cluster(&tempty[ab], (use - 1) & 1)
-                                                             : mbar_wait(&tempty[ab], (use - 1) & 1)))
+                if (use > 0 && !__all_sync(0xffffffffu, PAIR ? mbar_wait_cluster(&tempty[ab], (use - 1) & 1, p.wait_cycles)
+                                                             : mbar_wait(&tempty[ab], (use - 1) & 1, p.wait_cycles)))
                     break;
                 fence_after();
                 const uint32_t tmem_d = tmem_base + (uint32_t)(ab * p.acc_cols);
@@ -850,10 +914,11 @@ __global__ void __launch_bounds__(NT, 1)
                         mma_f8(tmem_d, ad_, bd_, idesc, a_);
                 };
                 for (int ks = kb; ks < ke; ks += p.kps) {
-                    if (!__all_sync(0xffffffffu, mbar_wait(&full[s], fphase))) { alive = false; break; }
+                    if (!__all_sync(0xffffffffu, mbar_wait(&full[s], fphase, p.wait_cycles))) { alive = false; break; }
                     fence_after();
                     const uint64_t off = (uint64_t)((uint32_t)s * dstep);
-                    uint64_t ad = adesc0 + off, bd = bdesc0 + off;
+                    uint64_t ad = adesc0 + off;
+                    uint64_t bd = p.wres ? wdesc0 + (uint64_t)((uint32_t)ks * bstep) : bdesc0 + off;
                     if (p.trans) {            // weights are the MMA's A operand (M = channels)
                         const uint64_t t_ = ad;
                         ad = bd;
@@ -929,7 +994,7 @@ __global__ void __launch_bounds__(NT, 1)
                 // columns [64 (2 (q >> 1) + half), + 64)
                 const int oq = 32 * (p.dup ? (q & 1) : q);
                 const int cq = p.dup ? 2 : 4, cb = p.dup ? 2 * (2 * (q >> 1) + half_cols) : 4 * half_cols;
-                for (int w = blockIdx.x; w < items; w += gridDim.x, ++i) {
+                for (int n = 0, w; (w = cta_item(p, n, items, tiles_m, crank)) >= 0; ++n, ++i) {
                     const int ab = p.nacc == 2 ? (i & 1) : 0, use = p.nacc == 2 ? (i >> 1) : i;
                     const int tn = w / tiles_m, tm = w - tn * tiles_m;
                     const int xb = tm % p.nbx, yb = (tm / p.nbx) % p.nby, bbk = tm / (p.nbx * p.nby);
@@ -945,7 +1010,7 @@ __global__ void __launch_bounds__(NT, 1)
                         sg = sthr[(NL - 1) * O32 + oc];
                         sig = ssig[(tn * p.BN + oq) >> 5];
                     }
-                    if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
+                    if (!dead && !mbar_wait(&tfull[ab], use & 1, p.wait_cycles)) dead = true;
                     fence_after();
                     const bool tres = p.res_codes != nullptr || p.res_f32 != nullptr;
                     float sc = 0.0f, sh = 0.0f, ny[NL - 1];
@@ -1038,7 +1103,7 @@ __global__ void __launch_bounds__(NT, 1)
                 }
             }
         }
-        for (int w = blockIdx.x; w < items && !p.trans; w += gridDim.x, ++i) {
+        for (int n = 0, w; !p.trans && (w = cta_item(p, n, items, tiles_m, crank)) >= 0; ++n, ++i) {
             const int ab = p.nacc == 2 ? (i & 1) : 0, use = p.nacc == 2 ? (i >> 1) : i;
             const int t = w / p.ksplit, kp = w - t * p.ksplit;
             const int tn = t / tiles_m, tm = t - tn * tiles_m;
@@ -1055,7 +1120,7 @@ __global__ void __launch_bounds__(NT, 1)
 
             if constexpr (OUTB > 0) {
                 if (masked) {
-                    if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
+                    if (!dead && !mbar_wait(&tfull[ab], use & 1, p.wait_cycles)) dead = true;
                     fence_after();
                     for (int c = cbeg; c < cend && !dead; ++c) {
                         const int ob = o0 + c * 32;
@@ -1075,7 +1140,7 @@ __global__ void __launch_bounds__(NT, 1)
                 }
             }
             if (rmasked) {
-                if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
+                if (!dead && !mbar_wait(&tfull[ab], use & 1, p.wait_cycles)) dead = true;
                 fence_after();
                 for (int c = cbeg; c < cend && !dead; ++c) {
                     const int ob = o0 + c * 32;
@@ -1237,7 +1302,7 @@ __global__ void __launch_bounds__(NT, 1)
                         asm volatile("prefetch.global.L2 [%0];\n" ::"l"(wrow + off));
                 }
             }
-            if (!dead && !mbar_wait(&tfull[ab], use & 1)) dead = true;
+            if (!dead && !mbar_wait(&tfull[ab], use & 1, p.wait_cycles)) dead = true;
             fence_after();
             int32_t *prow = p.part + (((size_t)kp * tiles + t) * 128 + r) * p.BN;
             uint32_t v32[32];
@@ -1539,54 +1604,14 @@ static int chunk_channels(const ConvArgs &a) {
 static size_t slice_bytes(int tiles, int BN) { return (size_t)tiles * 128 * BN * sizeof(int32_t); }
 static size_t thr_ws_bytes(int O, int nlev) { return (((size_t)O * nlev * sizeof(float)) + 255) & ~(size_t)255; }
 
-// Channel-major 64-channel tiles with the weight rows loaded twice (MINW_TC_DUP
-// = 0 pads with zero rows instead): the epilogue of a tile then spreads over
-// all eight epilogue warps, two 32-pixel chunks each instead of four.
-static int dup_pref() {
-    static int v = -1;
-    if (v < 0) {
-        const char *e = getenv("MINW_TC_DUP");
-        v = (e && e[0] == '0') ? 0 : 1;
-    }
-    return v;
-}
-
-// CTA pairs with cta_group::2 MMAs for 256-channel layers with long K loops
-// (MINW_TC_PAIR = 0 turns them off).  Each CTA then loads half the weight
-// rows per K block, and one MMA instruction covers both SMs; short K loops
-// (< 18 K blocks) measured faster single.
-static int pair_pref() {
-    static int v = -1;
-    if (v < 0) {
-        const char *e = getenv("MINW_TC_PAIR");
-        v = (e && e[0] == '0') ? 0 : 1;
-    }
-    return v;
-}
-
-// K blocks per stage the kernel may use (MINW_TC_KPS = 1 keeps one; 2 by default).
-static int kps_pref() {
-    static int v = -1;
-    if (v < 0) {
-        const char *e = getenv("MINW_TC_KPS");
-        v = (e && atoi(e) == 1) ? 1 : 2;
-    }
-    return v;
-}
-
-// Channel-major tiles (MINW_TC_TRANS=0 turns them off): a 64- or 128-channel
-// layer whose only output is the next layer's levels (a residual block's too)
-// runs as 128 channels (a 64-channel layer repeats its weight rows, or pads
-// with zero rows) x 256 pixels, so each MMA has N = 256 (the tensor pipe's
-// full rate).
-static int trans_pref() {
-    static int v = -1;
-    if (v < 0) {
-        const char *e = getenv("MINW_TC_TRANS");
-        v = (e && e[0] == '0') ? 0 : 1;
-    }
-    return v;
-}
+// Plan options (runtime.cu): channel-major 64-channel tiles with the weight
+// rows loaded twice (else zero rows), CTA pairs for 256-channel layers with
+// long K loops, K blocks per stage, channel-major tiles for 64- and
+// 128-channel layers.
+static int dup_pref() { return minw_host::plan_options().dup_weights != 0; }
+static int pair_pref() { return minw_host::plan_options().cta_pairs != 0; }
+static int kps_pref() { return minw_host::plan_options().kblocks_per_stage; }
+static int trans_pref() { return minw_host::plan_options().channel_major != 0; }
 
 // Tile of 256 pixels (bb images x bh rows x bw columns) that covers the output
 // image exactly, widest rows first; pooling keeps 2x2 windows inside a warp.
@@ -1613,21 +1638,18 @@ static bool trans_eligible(const ConvArgs &a) {
             ((a.O == 128 || (a.O == 64 && dup_pref())) && !a.pool));   // residual: all 8 warps hold channels
 }
 
-static minw_status make_plan(const ConvArgs &a, Plan &pl) {
+// encode = false plans the tiles and the split only (no tensor maps: no driver call).
+static minw_status make_plan(const ConvArgs &a, Plan &pl, bool encode = true) {
     Params &p = pl.p;
     p = Params{};
     p.trans = 0;
     if (trans_eligible(a)) {
         // only when the 256-pixel tiles cover the image without padding and leave
-        // at least two tiles per SM (MINW_TC_TRANS_MIN), else the 128-pixel tiles
+        // at least channel_major_min_tiles_per_sm tiles per SM, else the 128-pixel tiles
         // balance better
         Params q{};
         const int sms_ = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
-        static int min_tiles = -1;
-        if (min_tiles < 0) {
-            const char *e = getenv("MINW_TC_TRANS_MIN");
-            min_tiles = e ? atoi(e) : 2;
-        }
+        const int min_tiles = minw_host::plan_options().channel_major_min_tiles_per_sm;
         if (trans_shape(a, q) && (long long)q.nbx * q.nby * ((a.B + q.bb - 1) / q.bb) >= (long long)min_tiles * sms_)
             p.trans = 1;
     }
@@ -1671,15 +1693,41 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     const bool may_split = a.workspace != nullptr && !a.pool && !p.trans && !p.pair && !a.upd;
     if (a.upd && !rowst_fc) return MINW_EUNSUPPORTED;     // the update runs in the row-contiguous epilogue
     p.ystage = (rowst_fc || may_split) ? 8 * 32 * 16 : 0;
-    const size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes - (p.ystage ? (size_t)p.ystage * 4 + 16 : 0);
+    size_t budget = 224 * 1024 - 1024 - 256 - thr_bytes - (p.ystage ? (size_t)p.ystage * 4 + 16 : 0);
+    // resident weights (plan option resident_weights): a layer not split along K
+    // whose weights per CTA fit beside at least three activation stages, with
+    // at least as many CTA units as channel tiles and two or more pixel tiles
+    // per unit; it halves the loads per K block and frees the weight warp to
+    // issue activation stages
+    p.wres = 0;
+    p.wres_off = 0;
+    {
+        const int sms_ = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
+        const int tiles_ = p.nbx * p.nby * p.nbb * p.ntn;
+        const int ks_ = may_split ? (a.ksplit > 0 ? a.ksplit : auto_ksplit(tiles_, p.nk, sms_)) : 1;
+        const int cl_ = p.pair ? 2 : 1;
+        const int units = sms_ / cl_;
+        const int tiles_mp_ = (p.nbx * p.nby * p.nbb + cl_ - 1) / cl_ * cl_;
+        const size_t wbytes = (size_t)p.nk * p.b_bytes;
+        if (minw_host::plan_options().resident_weights && ks_ <= 1 && !rowst_fc && !a.upd && p.ntn <= units &&
+            tiles_mp_ / cl_ >= 2 * (units / p.ntn) && wbytes + 3 * (size_t)p.a_bytes <= budget) {
+            p.wres = 1;
+            budget -= wbytes;
+        }
+    }
     // two K blocks per stage (one commit per 8 or 4 MMAs) when three such stages fit
-    const size_t blk = (size_t)p.a_bytes + p.b_bytes;
+    const size_t blk = (size_t)p.a_bytes + (p.wres ? 0 : p.b_bytes);
     p.kps = (kps_pref() != 1 && p.nk >= 2 && budget / (2 * blk) >= 3) ? 2 : 1;
     p.stage_bytes = (uint32_t)(p.kps * blk);
     int S = (int)(budget / p.stage_bytes);
     if (S > 8) S = 8;
     if (S < 2) return MINW_EUNSUPPORTED;
     p.S = S;
+    if (p.wres) p.wres_off = (uint32_t)S * p.stage_bytes;
+    // lanes issuing TMA loads per producer warp (plan option tma_lanes), at most one per ring slot
+    p.tlanes = minw_host::plan_options().tma_lanes;
+    if (p.tlanes > p.S) p.tlanes = p.S;
+    if (p.tlanes < 1) p.tlanes = 1;
     // MMA N: the output channels, or the 256 pixels of a channel-major tile (M = 128 either way)
     const int mma_n = p.trans ? 256 : p.BN;
     p.acc_cols = mma_n;
@@ -1739,6 +1787,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     // CTA pairs walk pixel tiles two by two (an odd count gets one padded tile)
     p.cl = p.pair ? 2 : 1;
     p.tiles_mp = (tiles_m + p.cl - 1) / p.cl * p.cl;
+    if (!encode) return MINW_OK;
     minw_host::EncodeTiledFn enc = minw_host::tensor_map_encoder();
     if (enc == nullptr) return MINW_ECUDA;
     const CUtensorMapSwizzle swz = p.cb == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
@@ -1772,8 +1821,10 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl) {
     const int items = p.tiles_mp * p.ntn * p.ksplit;
     int grid = items < sms ? items : sms;
     grid -= grid % p.cl;
+    if (p.wres) grid = (sms / p.cl / p.ntn) * p.ntn * p.cl;     // whole units per channel tile
     pl.grid = dim3((unsigned)grid);
-    pl.smem = (size_t)p.S * p.stage_bytes + 1024 + 256 + thr_bytes + (p.ystage ? (size_t)p.ystage * 4 + 16 : 0);
+    pl.smem = (size_t)p.S * p.stage_bytes + (p.wres ? (size_t)p.nk * p.b_bytes : 0) + 1024 + 256 + thr_bytes +
+              (p.ystage ? (size_t)p.ystage * 4 + 16 : 0);
     // more than half of an SM's shared memory: exactly one CTA (and one TMEM
     // allocation) per SM
     if (pl.smem < 120 * 1024) pl.smem = 120 * 1024;
@@ -1842,6 +1893,12 @@ bool conv_tc_supported(const ConvArgs &a) {
 }
 
 
+int conv_tc_ksplit(const ConvArgs &a) {
+    if (!conv_tc_supported(a)) return 0;
+    tc::Plan pl;
+    return tc::make_plan(a, pl, false) == MINW_OK ? pl.p.ksplit : 0;
+}
+
 int conv_tc_launches(const ConvArgs &a) {
     if (a.workspace == nullptr || a.pool) return 1;
     tc::Plan pl;
@@ -1892,6 +1949,8 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
         thr = pl.thr_ws;
     }
     tc::Params pm = pl.p;
+    pm.wait_cycles = (long long)minw_host::plan_options().wait_cycles;
+    pm.stall = pl.p.pair ? 0 : minw_host::take_stall(MINW_STALL_CONV_TC);
     if (split) {
         pm.quant_out = 0;
         pm.acc_out = nullptr;

@@ -65,6 +65,8 @@ struct FirstArgs {
     float *y_out;              // [B][O][Ho][Wo] (nullable)
     const float *thr;          // fp32 breakpoints [O][8] (nullable: computed in-kernel)
     const float *wt;           // prepared weights [K][O] (levels when quantized; nullable: from w)
+    long long wait_cycles;     // limit of the bounded patch waits (set by the launcher)
+    int stall;                 // timeout-path test: first wait on a barrier nothing completes (set by the launcher)
 };
 
 // Launchers (host).  Return MINW_OK or an error status.
@@ -94,6 +96,8 @@ bool conv_tc_supported(const ConvArgs &a);
 size_t conv_tc_workspace_bytes(const ConvArgs &a);
 // Smallest workspace with which this shape still splits K (two slices); 0 when it does not split.
 size_t conv_tc_min_split_bytes(const ConvArgs &a);
+// K slices of the tensor-core plan for this shape and workspace (1: no split; 0: not supported).
+int conv_tc_ksplit(const ConvArgs &a);
 // Kernels one tensor-core launch issues for this shape and workspace (2 with a split).
 int conv_tc_launches(const ConvArgs &a);
 minw_status launch_thresholds(const float *scale, const float *shift, int O, const QParams &q, float *out,

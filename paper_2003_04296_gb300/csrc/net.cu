@@ -204,16 +204,9 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
     return MINW_OK;
 }
 
-// MINW_GRAPH=0 enqueues every kernel on every call instead of replaying the
-// captured forward.
-static bool graphs_enabled() {
-    static int v = -1;
-    if (v < 0) {
-        const char *e = getenv("MINW_GRAPH");
-        v = (e && e[0] == '0') ? 0 : 1;
-    }
-    return v == 1;
-}
+// Plan option graph = 0 enqueues every kernel on every call instead of
+// replaying the captured forward.
+static bool graphs_enabled() { return minw_host::plan_options().graph != 0; }
 
 static minw_status forward_enqueue(minw_net *net, const float *x, int32_t B, float *logits, cudaStream_t cs) {
     if (net->kind == 1) return resnet_forward(net, x, B, logits, cs);
@@ -357,9 +350,7 @@ minw_status minw_net_layer_times(minw_net *net, float *ms) {
 minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants) {
     if (!net || !variants) return MINW_EINVAL;
     if (net->kind == 1) {
-        // stem, pool, the block convolutions (tensor cores), head
-        const int n = minw_net_launches(net);
-        for (int l = 0; l < n; ++l) variants[l] = (l >= 2 && l < n - 1) ? MINW_VARIANT_TC : 0;
+        resnet_variants(net, variants);     // stem, pool, the block convolutions, head
         return MINW_OK;
     }
     for (size_t l = 0; l < net->L.size(); ++l)

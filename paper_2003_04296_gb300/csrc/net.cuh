@@ -57,5 +57,6 @@ struct minw_net {
 // Enqueue the residual network's forward (resnet.cu).
 minw_status resnet_forward(minw_net *net, const float *x, int B, float *logits, cudaStream_t s);
 int32_t resnet_ops(const minw_net *net);
+void resnet_variants(const minw_net *net, int32_t *variants);
 int32_t resnet_kernels(const minw_net *net);
 void resnet_free(minw_net *net);

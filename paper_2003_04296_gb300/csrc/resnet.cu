@@ -107,19 +107,25 @@ __global__ void __launch_bounds__(256) pool_levels_kernel(const uint8_t *__restr
     }
 }
 
-// Head, first part: global average pool of level codes [B][HW][C] -> fp32
-// [B][C]; thread = (image, channel), one fp32 sum over the pixels in order,
-// then one division.
+// Head, first part: global average pool of level codes [B][HW][C] (E4M3
+// bytes, or E2M1 nibbles with fp4) -> fp32 [B][C]; thread = (image, channel),
+// one fp32 sum over the pixels in order, then one division.
 __global__ void __launch_bounds__(256) avgpool_levels_kernel(const uint8_t *__restrict__ X, int B, int HW, int C,
-                                                             float unit, float *__restrict__ pooled) {
+                                                             float unit, int fp4, float *__restrict__ pooled) {
     pdl_wait();
     pdl_trigger();
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= B * C) return;
     const int b = i / C, c = i - b * C;
-    const uint8_t *src = X + (long long)b * HW * C + c;
     float s = 0.0f;
-    for (int p = 0; p < HW; ++p) s += (float)code_to_units(__ldg(src + (long long)p * C)) * unit;
+    if (fp4) {
+        const uint8_t *src = X + ((long long)b * HW * C + c) / 2;
+        const int sh = 4 * (c & 1);
+        for (int p = 0; p < HW; ++p) s += code_units_e2m1(__ldg(src + (long long)p * (C / 2)) >> sh) * unit;
+    } else {
+        const uint8_t *src = X + (long long)b * HW * C + c;
+        for (int p = 0; p < HW; ++p) s += (float)code_to_units(__ldg(src + (long long)p * C)) * unit;
+    }
     pooled[i] = s / (float)HW;
 }
 
@@ -160,6 +166,11 @@ __global__ void transpose_kernel(const float *__restrict__ in, int rows, int col
 }
 
 }  // namespace
+
+// Tensors of 128 channels or more are held as E2M1 codes (two channels per
+// byte), the 64-channel ones as E4M3 codes: a convolution's input and weights
+// follow its C, its quantized output (and a residual shortcut) its O.
+static int e2m1_channels(int c) { return c % 128 == 0 ? 1 : 0; }
 
 // One quantized convolution of a block.
 struct ResConv {
@@ -210,6 +221,7 @@ static ConvArgs conv_args(const ResConv &c, int B) {
     a.M = (long long)B * c.Ho * c.Wo;
     a.scale = c.scale; a.shift = c.shift;
     a.wgt8 = c.wcodes;
+    a.fp4 = e2m1_channels(c.C);
     return a;
 }
 
@@ -224,6 +236,20 @@ int32_t resnet_ops(const minw_net *net) {
     return ops;
 }
 
+// Variant of each op in forward order: 0 for the stem, its pool and the head,
+// MINW_VARIANT_TC or MINW_VARIANT_TC_E2M1 for the block convolutions.
+void resnet_variants(const minw_net *net, int32_t *variants) {
+    int k = 0;
+    variants[k++] = 0;
+    variants[k++] = 0;
+    for (const ResBlock &bk : net->res->blocks) {
+        variants[k++] = e2m1_channels(bk.c1.C) ? MINW_VARIANT_TC_E2M1 : MINW_VARIANT_TC;
+        if (bk.down) variants[k++] = e2m1_channels(bk.d.C) ? MINW_VARIANT_TC_E2M1 : MINW_VARIANT_TC;
+        variants[k++] = e2m1_channels(bk.c2.C) ? MINW_VARIANT_TC_E2M1 : MINW_VARIANT_TC;
+    }
+    variants[k++] = 0;
+}
+
 // Arguments of one block convolution: which = 0 conv1 (X -> V, quantized),
 // 1 the 1x1 / 2 shortcut (X -> D, fp32 BN output), 2 conv2 (V -> Y with the
 // shortcut added, quantized).
@@ -236,6 +262,7 @@ static ConvArgs block_conv(const minw_net *net, const ResBlock &bk, int which, i
         a.act8 = X;
         a.quant_out = 1; a.qo = to_qparams(&R->qa); a.thr = bk.c1.thr;
         a.codes_out = R->V;
+        a.codes_out4 = e2m1_channels(bk.c1.O);
     } else if (which == 1) {
         a.act8 = X;
         a.y_nhwc = R->D;
@@ -243,11 +270,13 @@ static ConvArgs block_conv(const minw_net *net, const ResBlock &bk, int which, i
         a.act8 = R->V;
         a.quant_out = 1; a.qo = to_qparams(&R->qa);
         a.codes_out = Y;
+        a.codes_out4 = e2m1_channels(bk.c2.O);
         a.ythr = R->ythr;
         if (bk.down) {
             a.res_f32 = R->D;
         } else {
             a.res_codes = X;
+            a.res_codes4 = e2m1_channels(bk.c2.O);
             a.res_unit = R->bits_a == 3 ? 0.25f : 1.0f;
         }
     }
@@ -341,8 +370,9 @@ extern "C" minw_status minw_resnet18_create(const minw_resnet18_desc *d, int32_t
             if (!x.c) continue;
             ResConv &c = *x.c;
             if ((st = alloc_owned(n, &c.wcodes, (size_t)c.O * c.k * c.k * c.C)) != MINW_OK) return fail(st);
-            if ((st = minw_pack_weight_codes(x.w, c.O, c.C, c.k, c.k, &qw, x.wsc, c.wcodes, stream)) != MINW_OK)
-                return fail(st);
+            st = e2m1_channels(c.C) ? minw_pack_weight_codes_e2m1(x.w, c.O, c.C, c.k, c.k, &qw, x.wsc, c.wcodes, stream)
+                                    : minw_pack_weight_codes(x.w, c.O, c.C, c.k, c.k, &qw, x.wsc, c.wcodes, stream);
+            if (st != MINW_OK) return fail(st);
             if ((st = copy_owned(n, &c.scale, x.sc, c.O, s)) != MINW_OK) return fail(st);
             if ((st = copy_owned(n, &c.shift, x.sh, c.O, s)) != MINW_OK) return fail(st);
             if (x.thr) {
@@ -451,7 +481,7 @@ minw_status resnet_forward(minw_net *net, const float *x, int B, float *logits, 
         const ResConv &last = R->blocks[7].c2;
         const int HW = last.Ho * last.Wo;
         launch_pdl(avgpool_levels_kernel, dim3((unsigned)((B * 512 + 255) / 256)), dim3(256), 0, s, (const uint8_t *)X,
-                   B, HW, 512, unit, R->pooled);
+                   B, HW, 512, unit, e2m1_channels(512), R->pooled);
         const size_t smem = sizeof(float) * HEAD_IMGS * 512;
         const dim3 grid((unsigned)((R->classes + HEAD_CLS - 1) / HEAD_CLS), (unsigned)((B + HEAD_IMGS - 1) / HEAD_IMGS));
         launch_pdl(fc_head_kernel, grid, dim3(HEAD_CLS, HEAD_IMGS), smem, s, (const float *)R->pooled, B, 512,

@@ -37,6 +37,17 @@ class BlockExtra(ctypes.Structure):
                 ("res_format", ctypes.c_int32), ("acc_out", ctypes.c_void_p)]
 
 
+class PlanOptions(ctypes.Structure):
+    _fields_ = [("cta_pairs", ctypes.c_int32), ("channel_major", ctypes.c_int32),
+                ("channel_major_min_tiles_per_sm", ctypes.c_int32), ("dup_weights", ctypes.c_int32),
+                ("kblocks_per_stage", ctypes.c_int32), ("first_tma", ctypes.c_int32), ("pdl", ctypes.c_int32),
+                ("graph", ctypes.c_int32), ("tma_lanes", ctypes.c_int32),
+                ("resident_weights", ctypes.c_int32), ("wait_cycles", ctypes.c_int64)]
+
+
+STALL_CONV_TC, STALL_CONV_FIRST = 1, 2
+
+
 class LayerDesc(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int32), ("C", ctypes.c_int32), ("H", ctypes.c_int32),
                 ("W", ctypes.c_int32), ("O", ctypes.c_int32), ("kh", ctypes.c_int32),
@@ -97,6 +108,10 @@ SIGNATURES = {
                                                 _I32, _I32, _I32, _P, _P, _QP, _P, _P, _P,
                                                 ctypes.POINTER(BlockExtra), _P]),
     "minw_fc_workspace_bytes": (ctypes.c_size_t, [_I32, _I32, _I32]),
+    "minw_fc_ksplit": (_I32, [_I32, _I32, _I32, ctypes.c_size_t]),
+    "minw_get_plan_options": (ctypes.c_int, [ctypes.POINTER(PlanOptions)]),
+    "minw_set_plan_options": (ctypes.c_int, [ctypes.POINTER(PlanOptions)]),
+    "minw_test_stall_next_launch": (ctypes.c_int, [_I32]),
     "minw_fc_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _P, _I32, _I32, _P, _P, _QP, _P, _P, _P, _P, _P,
                                      ctypes.c_size_t, _P]),
     "minw_fc_codes_noalloc": (ctypes.c_int, [_P, _I32, _I32, _I32, _P, _I32, _I32, _P, _P, _QP, _P, _P, _P, _P,
@@ -362,6 +377,11 @@ def minw_fc_workspace_bytes(B, K, O):
     return int(lib().minw_fc_workspace_bytes(B, K, O))
 
 
+def minw_fc_ksplit(B, K, O, workspace_bytes):
+    """K slices of minw_fc_codes for this shape and workspace size (host query)."""
+    return lib().minw_fc_ksplit(int(B), int(K), int(O), int(workspace_bytes))
+
+
 def minw_fc_codes(act, B, K, bits_a, wgt, O, bits_w, scale=None, shift=None, q_out=None, codes_out=None,
                   planes_out=None, y_out=None, acc_out=None, workspace=None, stream=None):
     nbytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
@@ -378,6 +398,28 @@ def minw_fc_codes_noalloc(act, B, K, bits_a, wgt, O, bits_w, scale=None, shift=N
                                        ctypes.byref(q_out) if q_out is not None else None, _ptr(codes_out),
                                        _ptr(planes_out), _ptr(y_out), _ptr(acc_out), _stream(stream)),
            "minw_fc_codes_noalloc")
+
+
+def get_plan_options():
+    o = PlanOptions()
+    _check(lib().minw_get_plan_options(ctypes.byref(o)), "minw_get_plan_options")
+    return {name: getattr(o, name) for name, _ in PlanOptions._fields_}
+
+
+def set_plan_options(opts=None, **changes):
+    """minw_set_plan_options: None and no changes restores the defaults;
+    otherwise the current options (or opts) updated with changes."""
+    if opts is None and not changes:
+        _check(lib().minw_set_plan_options(None), "minw_set_plan_options")
+        return
+    cur = dict(opts if opts is not None else get_plan_options())
+    cur.update(changes)
+    o = PlanOptions(**cur)
+    _check(lib().minw_set_plan_options(ctypes.byref(o)), "minw_set_plan_options")
+
+
+def minw_test_stall_next_launch(kernel):
+    _check(lib().minw_test_stall_next_launch(int(kernel)), "minw_test_stall_next_launch")
 
 
 def minw_get_last_device_error(stream=None):

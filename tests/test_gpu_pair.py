@@ -4,10 +4,6 @@ half of the weight rows), used for 256-channel layers with K loops of at
 least 18 K blocks: accumulators for several bit widths and strides with an
 odd number of pixel tiles (the pair's second tile is padding), the fused
 pooled block epilogue, and the same shapes with the pairs turned off."""
-import os
-import subprocess
-import sys
-
 import numpy as np
 import pytest
 
@@ -20,7 +16,6 @@ from tests._gpu import dev_tensor, planes_view  # noqa: E402
 pytestmark = pytest.mark.gpu
 
 _CODE = {0: 0x00, 1: 0x38, 2: 0x40, 4: 0x48, -1: 0xB8, -2: 0xC0, -4: 0xC8}
-ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 @pytest.fixture(scope="module")
@@ -98,24 +93,19 @@ def test_pair_pooled_block(dev, M, bits):
 
 
 def test_pairs_off(dev):
-    """MINW_TC_PAIR=0 (read once per process, so in a child): the same shapes on
-    single-CTA tiles give the same accumulators."""
-    code = (
-        "import numpy as np, torch\n"
-        "from paper_2003_04296_gb300 import minw\n"
-        "from tests.test_gpu_pair import CASES, _operands, _ref_acc\n"
-        "from paper_2003_04296_gb300.inputs import conv_problem\n"
-        "dev = torch.device('cuda:0')\n"
-        "for (B, C, H, W, O_, s) in CASES:\n"
-        "    p = conv_problem(900 + C // 64, B, C, H, W, O_, 3, 3, s, 1, 2, 2, w_sigma=0.5)\n"
-        "    act, wgt = _operands(dev, minw, p)\n"
-        "    Ho, Wo = (H - 1) // s + 1, (W - 1) // s + 1\n"
-        "    acc = torch.empty((B, O_, Ho, Wo), dtype=torch.int32, device=dev)\n"
-        "    minw.minw_conv2d_codes(act, B, C, H, W, 2, wgt, O_, 3, 3, 2, s, 1, acc_out=acc)\n"
-        "    torch.cuda.synchronize()\n"
-        "    assert minw.minw_get_last_device_error() == minw.MINW_OK\n"
-        "    assert np.array_equal(acc.cpu().numpy(), _ref_acc(p))\n"
-        "print('ok')\n")
-    env = dict(os.environ, MINW_TC_PAIR="0")
-    r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
-    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stderr[-2000:]
+    """Plan option cta_pairs = 0: the same shapes on single-CTA tiles give the
+    same accumulators."""
+    from paper_2003_04296_gb300 import minw
+    minw.set_plan_options(cta_pairs=0)
+    try:
+        for (B, C, H, W, O_, s) in CASES:
+            p = conv_problem(900 + C // 64, B, C, H, W, O_, 3, 3, s, 1, 2, 2, w_sigma=0.5)
+            act, wgt = _operands(dev, minw, p)
+            Ho, Wo = (H - 1) // s + 1, (W - 1) // s + 1
+            acc = torch.empty((B, O_, Ho, Wo), dtype=torch.int32, device=dev)
+            minw.minw_conv2d_codes(act, B, C, H, W, 2, wgt, O_, 3, 3, 2, s, 1, acc_out=acc)
+            torch.cuda.synchronize()
+            assert minw.minw_get_last_device_error() == minw.MINW_OK
+            assert np.array_equal(acc.cpu().numpy(), _ref_acc(p))
+    finally:
+        minw.set_plan_options()

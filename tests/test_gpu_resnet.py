@@ -71,7 +71,11 @@ def test_resnet_timing_and_variants(dev, M):
     var = net.layer_variants()
     net.close()
     assert len(ms) == len(var) == 22 and all(t >= 0.0 for t in ms)
-    assert var[0] == 0 and var[2:-1] == [M.VARIANT_TC] * 19
+    # block convolutions in forward order (conv1, [shortcut], conv2): inputs of
+    # 128 channels or more are E2M1 codes, the 64-channel ones E4M3
+    c_in = [64, 64, 64, 64, 64, 64, 128, 128, 128, 128, 128, 256, 256, 256, 256, 256, 512, 512, 512]
+    want = [M.VARIANT_TC_E2M1 if c % 128 == 0 else M.VARIANT_TC for c in c_in]
+    assert var[0] == 0 and var[1] == 0 and var[-1] == 0 and var[2:-1] == want
 
 
 def test_resnet_create_errors(dev, M):

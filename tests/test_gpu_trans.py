@@ -1,7 +1,7 @@
 """GPU parity of the channel-major tensor-core tiles (128 output channels x
 256 pixels, used for 64- and 128-channel layers whose only output is the next
 layer's levels; a 64-channel layer loads its weight rows twice, or pads with
-zero rows when MINW_TC_DUP=0): 128 -> 128 and 64 -> 64 convolutions with and
+zero rows with the plan option dup_weights = 0): 128 -> 128 and 64 -> 64 convolutions with and
 without the 2x2 pool, for each output bit width, residual blocks, against the
 oracle's levels, planes and codes."""
 import numpy as np
@@ -121,21 +121,12 @@ def test_channel_major_residual(dev, M, bits, ch, shortcut):
     assert np.array_equal(planes_view(planes, B, H, W, bits, O_)[pick], O.pack(lv, bits))
 
 
-def test_channel_major_zero_rows():
-    """MINW_TC_DUP=0 (read once per process, so in a child): 64-channel tiles
-    padded with zero weight rows give the same levels."""
-    import os
-    import subprocess
-    import sys
-    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-    code = (
-        "import torch\n"
-        "from paper_2003_04296_gb300 import minw\n"
-        "import tests.test_gpu_trans as T\n"
-        "dev = torch.device('cuda:0')\n"
-        "for bits in (1, 3):\n"
-        "    T.test_channel_major_tiles(dev, minw, bits, 1, 64)\n"
-        "print('ok')\n")
-    env = dict(os.environ, MINW_TC_DUP="0")
-    r = subprocess.run([sys.executable, "-c", code], cwd=root, env=env, capture_output=True, text=True, timeout=600)
-    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stderr[-2000:]
+def test_channel_major_zero_rows(dev, M):
+    """Plan option dup_weights = 0: 64-channel tiles padded with zero weight
+    rows give the same levels."""
+    M.set_plan_options(dup_weights=0)
+    try:
+        for bits in (1, 3):
+            test_channel_major_tiles(dev, M, bits, 1, 64)
+    finally:
+        M.set_plan_options()

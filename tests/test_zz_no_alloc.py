@@ -5,7 +5,9 @@ scratch is a fixed array inside the library.
 
 Checked through the C ABI against minw_fc_codes with a caller-allocated
 workspace, on two calls in a row, at the tolerance of the other GPU tests
-(exact integers and codes, fp32 within 1e-5 relative / 1e-6 absolute).
+(exact integers and codes, fp32 within 1e-5 relative / 1e-6 absolute), and
+against the oracle itself (exact accumulators, the BN output and the next
+layer's levels bit for bit).
 This file is collected last so that a run stopping at the first failure has
 already run every other test; it also passes on its own in a fresh process."""
 import numpy as np
@@ -13,6 +15,7 @@ import pytest
 
 torch = pytest.importorskip("torch")
 
+from oracle import oracle as O  # noqa: E402
 from paper_2003_04296_gb300.inputs import DEFAULT_THR, conv_problem  # noqa: E402
 from tests._gpu import assert_close, dev_tensor  # noqa: E402
 
@@ -50,9 +53,19 @@ def _outputs(dev, B, Oc, last):
     return acc, y, codes
 
 
+def _decode_e4m3(b):
+    """E4M3 bytes to values from the format's definition (normal numbers and 0)."""
+    b = b.astype(np.int64)
+    v = np.where(b & 0x80, -1.0, 1.0) * (1.0 + (b & 7) / 8.0) * np.power(2.0, ((b >> 3) & 0xF) - 7.0)
+    return np.where((b & 0x7F) == 0, 0.0, v)
+
+
 @pytest.mark.parametrize("B,K,Oc,ba,bw", [(256, 8192, 1024, 1, 1), (64, 4096, 512, 3, 3), (256, 2048, 10, 1, 1)])
 def test_noalloc_matches_workspace_entry_point(dev, M, B, K, Oc, ba, bw):
     p, act, wgt = _operands(dev, M, B, K, Oc, ba, bw, seed=B + K + Oc)
+    # the fixed array really carries a split of K for the shapes that split
+    if Oc >= 512:
+        assert M.minw_fc_ksplit(B, K, Oc, 8 << 20) > 1
     sc, sh = dev_tensor(p["scale"], dev), dev_tensor(p["shift"], dev)
     last = Oc % 16 != 0
     q = None if last else M.quant(ba, DEFAULT_THR[ba])
@@ -80,6 +93,18 @@ def test_noalloc_matches_workspace_entry_point(dev, M, B, K, Oc, ba, bw):
         if codes is not None:
             assert np.array_equal(codes.cpu().numpy(), codes_r.cpu().numpy())
     assert M.minw_get_last_device_error() == M.MINW_OK
+
+    # against the oracle: exact accumulators, BN (+ HardTanh), the next layer's levels
+    al = O.quantize(p["x"], ba, p["thr_a"])
+    wl = O.quantize(p["w"], bw, p["thr_w"], p["w_scale"])
+    ref = O.conv2d_levels(al, wl, 1, 0, ba, bw).reshape(B, Oc)
+    assert np.array_equal(acc.cpu().numpy(), ref)
+    yref = O.affine(ref, p["scale"], p["shift"])
+    if not last:
+        yref = O.hardtanh(yref)
+        lv = O.quantize(yref, ba, DEFAULT_THR[ba]) * 2.0 ** O.units_shift(ba)
+        assert np.array_equal(_decode_e4m3(codes.cpu().numpy()), lv)
+    assert np.array_equal(y.cpu().numpy(), yref)
 
 
 def test_noalloc_rejects_requests_beyond_the_fixed_scratch(dev, M):
