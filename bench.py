@@ -290,6 +290,81 @@ def oracle_images_per_s(wl, x, max_seconds):
     return done / dt, done, dt
 
 
+def _oracle_worker(job):
+    """One process of the all-cores oracle baseline: the network forward of
+    its images, one by one, until its time is up (returns images done, s)."""
+    name, bits, lo, n, seconds = job
+    import argparse as _ap
+    a = _ap.Namespace(bits_a=bits[0], bits_w=bits[1], model="A", bits_a_resnet=bits[0], bits_w_resnet=bits[1])
+    wl = Workload(name, a)
+    x = wl.images(0)[lo:lo + n]
+    wl.oracle(x[:1])
+    done, t0 = 0, time.perf_counter()
+    while done < x.shape[0] and time.perf_counter() - t0 < seconds:
+        wl.oracle(x[done:done + 1])
+        done += 1
+    return done, time.perf_counter() - t0
+
+
+def oracle_all_cores(name, bits, batch, seconds):
+    """The oracle forward on every core of this process's affinity mask, as
+    independent processes (spawned: no state shared with the GPU context),
+    each over its own images of the batch: aggregate images/s."""
+    import multiprocessing as mp
+    try:
+        cores = len(os.sched_getaffinity(0))
+    except AttributeError:
+        cores = os.cpu_count() or 1
+    per = max(1, batch // cores)
+    jobs = [(name, bits, (i * per) % batch, per, seconds) for i in range(cores)]
+    ctx = mp.get_context("spawn")
+    with ctx.Pool(cores) as pool:
+        res = pool.map(_oracle_worker, jobs)
+    imgs = sum(r[0] for r in res)
+    span = max(r[1] for r in res)
+    return imgs / span, imgs, span, cores
+
+
+def cpu_model():
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith(("model name", "cpu model")):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+def run_reference_conv1(args):
+    """The oracle on the single convolution: whole steps (quantize, fp64
+    level convolution, BN) of the 4-image batch."""
+    from oracle import oracle as Or
+    from paper_2003_04296_gb300.inputs import DEFAULT_THR, conv_problem
+    p = conv_problem(0, 4, 128, 32, 32, 128, 3, 3, 1, 1, 1, 1)
+    mac = 4 * 32 * 32 * 128 * 128 * 9
+    times = []
+    for k in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        al = Or.quantize(p["x"], 1, DEFAULT_THR[1])
+        wl = Or.quantize(p["w"], 1, DEFAULT_THR[1], p["w_scale"])
+        Or.affine(Or.conv2d_levels(al, wl, 1, 1, 1, 1), p["scale"], p["shift"])
+        if k >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    sec = sum(times) / len(times)
+    tops = 2.0 * mac / sec / 1e12
+    line = {"metric": METRIC, "value": tops, "unit": "effective TOPS (2 x MAC / s)", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
+            "impl": "reference", "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": conv1_config(args.gpus),
+            "cpu_baseline": {"value": tops, "unit": "effective TOPS", "cores": 1, "kind": "oracle",
+                             "sample": "whole steps of the 4-image workload, single-threaded C oracle"},
+            "e2e": {"value": tops, "unit": "effective TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_reference_sweep(args):
     """The oracle on the sweep: one image per step through the fp64 level
     convolution, cycling through the nine bit-width pairs."""
@@ -321,11 +396,13 @@ def run_reference_sweep(args):
 
 def run_reference(args, rank):
     if rank != 0:
-        return 0
+        return None
     if args.workload == "sweep":
         return run_reference_sweep(args)
     if args.workload == "fc_train":
         return run_reference_fc_train(args)
+    if args.workload == "conv1":
+        return run_reference_conv1(args)
     wl = Workload(args.workload, args)
     x = wl.images(0)
     B = wl.batch
@@ -434,7 +511,7 @@ def run_gpu(args, rank, world, local_rank):
     e2e_sec = max_over_ranks(sum(e2e_s) / len(e2e_s), world, dev)
 
     if rank != 0:
-        return 0
+        return None
 
     clocks = clk.summary()
     layer_ms /= args.steps
@@ -462,11 +539,17 @@ def run_gpu(args, rank, world, local_rank):
     roofline["layer_variants"] = variants
     roofline["traffic"] = _captured_traffic(roofline["bound"]) if wl.name == "cifar_convnet" else None
 
-    cpu = None
+    cpu = cpu_all = None
     if world == 1 and not args.skip_cpu:
         ips, n_img, secs = oracle_images_per_s(wl, x_np, args.cpu_seconds)
         cpu = {"value": ips, "unit": "images/s", "cores": 1, "kind": "oracle",
-               "sample": f"{n_img} images of the batch through the single-threaded C oracle ({secs:.1f} s)"}
+               "sample": f"{n_img} images of the batch through the single-threaded C oracle ({secs:.1f} s)",
+               "cpu": cpu_model()}
+        ips_all, n_all, secs_all, cores = oracle_all_cores(wl.name, wl.bits, BATCH, args.cpu_seconds)
+        cpu_all = {"value": ips_all, "unit": "images/s", "cores": cores, "kind": "oracle",
+                   "sample": f"{n_all} images through {cores} independent single-threaded oracle processes "
+                             f"(one per core of the affinity mask, spawned), {secs_all:.1f} s",
+                   "cpu": cpu_model()}
 
     line = {"metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
@@ -478,13 +561,12 @@ def run_gpu(args, rank, world, local_rank):
             "layer_ms": [round(v, 5) for v in layer_ms.tolist()],
             "layer_ms_note": "per-op CUDA-event durations from a second pass of the same steps with an event "
                              "after every op; the timed steps run without them",
-            "roofline": roofline, "cpu_baseline": cpu,
+            "roofline": roofline, "cpu_baseline": cpu, "cpu_baseline_all_cores": cpu_all,
             "e2e": {"value": replica_throughput(BATCH, world, e2e_sec), "unit": "images/s",
                     "h2d_bytes_per_step": int(x_host.numel() * 4),
                     "d2h_bytes_per_step": int(out_host.numel() * 4)},
             "gpu_launches": net.kernels * args.steps, "clocks": clocks}
-    print(json.dumps(line), flush=True)
-    return 0
+    return line
 
 
 # ------------------------------------------------------------------ sweep --
@@ -504,6 +586,134 @@ def sweep_config(n_gpus):
             "aqe": "AQE forward (alpha 0.75) and backward on the same 25.7M-element tensor (the stochastic forward, "
                    "Eq. our, is timed beside the steps)",
             "parallelism": f"replicas x{n_gpus} (batch-sharded, no collective)", "l2": L2_NOTE}
+
+
+# ------------------------------------------------------------ single conv --
+
+def conv1_config(n_gpus):
+    return {"workload": "conv3x3_4x128x32x32_to128_a1w1", "batch_per_gpu": 4, "global_batch": 4 * n_gpus,
+            "input": "4x128x32x32 fp32 N(0,1), weights 128x128x3x3 N(0,0.05), seed 0",
+            "step": "quantize the input to E2M1 codes (Eq. inference, 1-bit), then the 3x3/1/1 convolution "
+                    "with int32 accumulators and the fp32 per-channel BN output; weights packed once",
+            "launch": "each timed step replays a CUDA graph of the step's two kernels",
+            "parallelism": f"replicas x{n_gpus} (batch-sharded, no collective)", "l2": L2_NOTE}
+
+
+def run_conv1(args, rank, world, local_rank):
+    """The single quantized convolution of the smallest workload: the step
+    quantizes the fp32 input and convolves it (int32 accumulators plus the
+    fp32 BN output).  The op is a few microseconds, so each step replays a
+    CUDA graph of the two launches (the L2 flush stays outside the graph)."""
+    import torch
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    import __graft_entry__ as g
+    if rank == 0:
+        g.build()
+    from paper_2003_04296_gb300 import minw
+    from paper_2003_04296_gb300.inputs import DEFAULT_THR, conv_problem
+    B, C, H, W, O = 4, 128, 32, 32, 128
+    p = conv_problem(0, B, C, H, W, O, 3, 3, 1, 1, 1, 1)
+    x = torch.from_numpy(p["x"]).to(dev)
+    sc, sh = torch.from_numpy(p["scale"]).to(dev), torch.from_numpy(p["shift"]).to(dev)
+    act = torch.empty((B, H, W, C // 2), dtype=torch.uint8, device=dev)
+    wgt = torch.empty((O, 3, 3, C // 2), dtype=torch.uint8, device=dev)
+    minw.minw_pack_weight_codes_e2m1(torch.from_numpy(p["w"]).to(dev), minw.quant(1, DEFAULT_THR[1]), wgt,
+                                     channel_scale=torch.from_numpy(p["w_scale"]).to(dev))
+    acc = torch.empty((B, O, H, W), dtype=torch.int32, device=dev)
+    y = torch.empty((B, O, H, W), dtype=torch.float32, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    s = torch.cuda.Stream(device=dev)
+    q = minw.quant(1, DEFAULT_THR[1])
+
+    def step(stream):
+        minw.aqe_quantize_codes_e2m1(x, q, act, stream=stream)
+        minw.minw_conv_block_codes_ex(act, B, C, H, W, 1, wgt, O, 3, 3, 1, 1, 1, 0, sc, sh, y_out=y,
+                                      in_format=minw.CODES_E2M1, acc_out=acc, stream=stream)
+
+    with torch.cuda.stream(s):
+        for _ in range(3):
+            step(s)
+    s.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=s):
+        step(torch.cuda.current_stream())
+    torch.cuda.synchronize()
+    for _ in range(max(args.warmup, 3)):
+        graph.replay()
+    torch.cuda.synchronize()
+    e0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    e1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    cur = torch.cuda.current_stream()
+    with ClockSampler(local_rank) as clk:
+        for k in range(args.steps):
+            flush.zero_()
+            e0[k].record(cur)
+            graph.replay()
+            e1[k].record(cur)
+        torch.cuda.synchronize()
+    ms = sum(e0[k].elapsed_time(e1[k]) for k in range(args.steps)) / args.steps
+    ms_max = max_over_ranks(ms, world, dev)
+    # per-kernel time of the convolution (direct launches with events around it)
+    cms = []
+    for k in range(min(args.steps, 200)):
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        flush.zero_()
+        minw.aqe_quantize_codes_e2m1(x, q, act)
+        a0.record(cur)
+        minw.minw_conv_block_codes_ex(act, B, C, H, W, 1, wgt, O, 3, 3, 1, 1, 1, 0, sc, sh, y_out=y,
+                                      in_format=minw.CODES_E2M1, acc_out=acc)
+        a1.record(cur)
+        torch.cuda.synchronize()
+        cms.append(a0.elapsed_time(a1))
+    conv_ms = float(np.median(cms))
+    # end to end: pinned host input in, accumulators and BN output back
+    x_host = torch.from_numpy(p["x"]).pin_memory()
+    acc_host = torch.empty(acc.shape, dtype=torch.int32).pin_memory()
+    y_host = torch.empty(y.shape, dtype=torch.float32).pin_memory()
+    e2e_s = []
+    for k in range(min(args.steps, 200) + 1):
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        x.copy_(x_host, non_blocking=True)
+        graph.replay()
+        acc_host.copy_(acc, non_blocking=True)
+        y_host.copy_(y, non_blocking=True)
+        torch.cuda.synchronize()
+        if k:
+            e2e_s.append(time.perf_counter() - t0)
+    e2e_sec = max_over_ranks(sum(e2e_s) / len(e2e_s), world, dev)
+    if rank != 0:
+        return None
+    mac = B * H * W * O * C * 9
+    roofline = tensor_roofline([2.0 * mac], ["e2m1"], [conv_ms])
+    roofline["kernel"] = "conv_tc_kernel (tcgen05 kind::mxf4 E2M1; int32 and fp32 NCHW outputs)"
+    roofline["note"] = ("a 6.0e8-MAC layer: one wave of 32 tiles with 9 K blocks each, so launch and "
+                        "pipeline fill set its time, not the tensor pipe")
+    cpu = None
+    if world == 1 and not args.skip_cpu:
+        from oracle import oracle as Or
+        t0, n = time.perf_counter(), 0
+        while True:
+            al = Or.quantize(p["x"], 1, DEFAULT_THR[1])
+            wl = Or.quantize(p["w"], 1, DEFAULT_THR[1], p["w_scale"])
+            Or.affine(Or.conv2d_levels(al, wl, 1, 1, 1, 1), p["scale"], p["shift"])
+            n += 1
+            if time.perf_counter() - t0 > min(args.cpu_seconds, 10.0):
+                break
+        dt = time.perf_counter() - t0
+        cpu = {"value": 2.0 * mac * n / dt / 1e12, "unit": "effective TOPS", "cores": 1, "kind": "oracle",
+               "sample": f"{n} whole steps of the workload (quantize, fp64 level convolution, BN) in {dt:.1f} s"}
+    return {"metric": METRIC, "value": replica_throughput(2.0 * mac, world, ms_max * 1e-3) / 1e12,
+            "unit": "effective TOPS (2 x MAC / s)", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "e2m1", "data": "synthetic", "config": conv1_config(world), "conv_ms": round(conv_ms, 5),
+            "roofline": roofline, "cpu_baseline": cpu,
+            "e2e": {"value": 2.0 * mac * world / e2e_sec / 1e12, "unit": "effective TOPS",
+                    "h2d_bytes_per_step": int(x_host.numel() * 4),
+                    "d2h_bytes_per_step": int(acc_host.numel() * 4 + y_host.numel() * 4)},
+            "gpu_launches": 2 * args.steps, "clocks": clk.summary()}
 
 
 def step_bytes(B, K, O):
@@ -641,7 +851,7 @@ def run_fc_train(args, rank, world, local_rank):
             e2e_s.append(time.perf_counter() - t0)
     e2e_sec = max_over_ranks(sum(e2e_s) / len(e2e_s), world, dev)
     if rank != 0:
-        return 0
+        return None
     cpu = None
     if world == 1 and not args.skip_cpu:
         ips, sec, n = fc_train_oracle_rate(A_np, W_np, G_np, budget_s=10.0)
@@ -668,8 +878,7 @@ def run_fc_train(args, rank, world, local_rank):
             "e2e": {"value": replica_throughput(B, world, e2e_sec), "unit": "images/s",
                     "h2d_bytes_per_step": int(4 * (A.numel() + G.numel())), "d2h_bytes_per_step": int(4 * g_in.numel())},
             "gpu_launches": 7 * args.steps, "clocks": clk.summary()}
-    print(json.dumps(line), flush=True)
-    return 0
+    return line
 
 
 def run_sweep(args, rank, world, local_rank):
@@ -694,10 +903,11 @@ def run_sweep(args, rank, world, local_rank):
     ws = torch.from_numpy(p["w_scale"]).to(dev)
     g_np = aqe_problem(55, x.numel())["g"]
     gy = torch.from_numpy(g_np).to(dev)
-    a8 = {b: torch.empty((B, H, W, C), dtype=torch.uint8, device=dev) for b in (1, 2, 3)}
-    w8 = {b: torch.empty((O, 3, 3, C), dtype=torch.uint8, device=dev) for b in (1, 2, 3)}
+    # E2M1 level codes (two channels per byte): kind::mxf4 on the tensor cores
+    a8 = {b: torch.empty((B, H, W, C // 2), dtype=torch.uint8, device=dev) for b in (1, 2, 3)}
+    w8 = {b: torch.empty((O, 3, 3, C // 2), dtype=torch.uint8, device=dev) for b in (1, 2, 3)}
     for b in (1, 2, 3):
-        minw.minw_pack_weight_codes(w, minw.quant(b, DEFAULT_THR[b]), w8[b], channel_scale=ws)
+        minw.minw_pack_weight_codes_e2m1(w, minw.quant(b, DEFAULT_THR[b]), w8[b], channel_scale=ws)
     acc = torch.empty((B, O, H, W), dtype=torch.int32, device=dev)
     y = torch.empty_like(x)
     # weight-only layer at the same shape (bf16 activations x 1-bit weights), timed beside the steps
@@ -713,11 +923,16 @@ def run_sweep(args, rank, world, local_rank):
 
     def step(ev=None):
         for b in (1, 2, 3):
-            minw.aqe_quantize_codes(x, minw.quant(b, DEFAULT_THR[b]), a8[b])
+            if ev is not None and b == 1:
+                ev[12][0].record(stream)
+            minw.aqe_quantize_codes_e2m1(x, minw.quant(b, DEFAULT_THR[b]), a8[b])
+            if ev is not None and b == 1:
+                ev[12][1].record(stream)
         for i, (ba, bw) in enumerate(SWEEP_PAIRS):
             if ev is not None:
                 ev[i][0].record(stream)
-            minw.minw_conv2d_codes(a8[ba], B, C, H, W, ba, w8[bw], O, 3, 3, bw, 1, 1, acc_out=acc)
+            minw.minw_conv_block_codes_ex(a8[ba], B, C, H, W, ba, w8[bw], O, 3, 3, bw, 1, 1, 0, None, None,
+                                          in_format=minw.CODES_E2M1, acc_out=acc)
             if ev is not None:
                 ev[i][1].record(stream)
         if ev is not None:
@@ -756,9 +971,9 @@ def run_sweep(args, rank, world, local_rank):
     ms_max = max_over_ranks(ms, world, dev)
     # per-kernel durations: the same steps again with events around the convolutions and the AQE forward
     conv_ms = np.zeros(len(SWEEP_PAIRS))
-    aqe_ms = sto_ms = wo_ms = 0.0
+    aqe_ms = sto_ms = wo_ms = q_ms = 0.0
     for k in range(args.steps):
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(12)]
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(13)]
         flush.zero_()
         step(ev)
         torch.cuda.synchronize()
@@ -766,7 +981,9 @@ def run_sweep(args, rank, world, local_rank):
         aqe_ms += ev[9][0].elapsed_time(ev[9][1])
         sto_ms += ev[10][0].elapsed_time(ev[10][1])
         wo_ms += ev[11][0].elapsed_time(ev[11][1])
+        q_ms += ev[12][0].elapsed_time(ev[12][1])
     conv_ms /= args.steps
+    q_ms /= args.steps
     aqe_ms /= args.steps
     sto_ms /= args.steps
     wo_ms /= args.steps
@@ -788,16 +1005,20 @@ def run_sweep(args, rank, world, local_rank):
             e2e_s.append(time.perf_counter() - t0)
     e2e_sec = max_over_ranks(sum(e2e_s) / len(e2e_s), world, dev)
     if rank != 0:
-        return 0
+        return None
 
     mac = B * H * W * O * C * 9
     value = replica_throughput(2.0 * mac * len(SWEEP_PAIRS), world, ms_max * 1e-3) / 1e12
     achieved = 2.0 * mac * len(SWEEP_PAIRS) / (conv_ms.sum() * 1e-3) / 1e12
-    roofline = {"bound": "tensor", "kernel": "conv_tc_kernel (tcgen05 kind::f8f6f4, 9 bit-width pairs)",
-                "achieved": achieved, "peak": FP8_TFLOPS, "unit": "TFLOP/s", "frac": achieved / FP8_TFLOPS,
-                "traffic": None,
-                "peak_basis": f"measured dense bf16 {BF16_TFLOPS:.1f} TFLOP/s (burst) x 2 for FP8 "
-                              "(nominal fp8/bf16 ratio), of measured"}
+    roofline = tensor_roofline([2.0 * mac] * len(SWEEP_PAIRS), ["e2m1"] * len(SWEEP_PAIRS),
+                               [float(v) for v in conv_ms])
+    roofline["kernel"] = "conv_tc_kernel (tcgen05 kind::mxf4 E2M1, 9 bit-width pairs, int32 accumulators out)"
+    # the A2 step: fp32 NCHW in, E2M1 codes out (4 + 1/2 bytes per element)
+    q_bytes = 4.5 * x.numel()
+    quant_roof = {"bound": "hbm", "kernel": "quantize_codes_kernel<E2M1> (1-bit)", "ms": round(q_ms, 5),
+                  "achieved": q_bytes / (q_ms * 1e-3) / 1e9, "peak": HBM_GBS, "unit": "GB/s",
+                  "frac": q_bytes / (q_ms * 1e-3) / 1e9 / HBM_GBS, "algorithmic_bytes": q_bytes,
+                  "peak_basis": "measured copy bandwidth, of measured"}
     aqe_bytes = 8.0 * x.numel()
     aqe_roof = {"bound": "hbm", "kernel": "aqe_forward_kernel", "achieved": aqe_bytes / (aqe_ms * 1e-3) / 1e9,
                 "peak": HBM_GBS, "unit": "GB/s", "frac": aqe_bytes / (aqe_ms * 1e-3) / 1e9 / HBM_GBS,
@@ -828,16 +1049,79 @@ def run_sweep(args, rank, world, local_rank):
                "sample": f"{n} single-image 1-bit x 1-bit convolutions (fp64 oracle, {dt:.1f} s)"}
     line = {"metric": METRIC, "value": value, "unit": "effective TOPS (2 x MAC / s)", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "e4m3", "data": "synthetic", "config": sweep_config(world),
+            "scaling": "weak", "vs_baseline": None, "dtype": "e2m1", "data": "synthetic", "config": sweep_config(world),
             "conv_ms": [round(v, 5) for v in conv_ms.tolist()], "aqe_forward_ms": round(aqe_ms, 5),
             "aqe_stochastic_ms": round(sto_ms, 5),
             "roofline": roofline, "aqe_roofline": aqe_roof, "aqe_stochastic_roofline": sto_roof,
+            "quantize_roofline": quant_roof,
             "weight_only_bf16": wonly, "cpu_baseline": cpu,
             "e2e": {"value": 2.0 * mac * len(SWEEP_PAIRS) * world / e2e_sec / 1e12, "unit": "effective TOPS",
                     "h2d_bytes_per_step": int(x_host.numel() * 4), "d2h_bytes_per_step": int(acc_host.numel() * 4)},
             "gpu_launches": 14 * args.steps, "clocks": clk.summary()}
-    print(json.dumps(line), flush=True)
-    return 0
+    return line
+
+
+def run_peaks(args, rank, world, local_rank):
+    """The pipe rates behind the per-shape choice of path
+    (minw_measure_pipe_rates), with per-SM-per-clock figures and the resulting
+    peak of each path for a 1-bit x 1-bit convolution."""
+    import torch
+    torch.cuda.set_device(local_rank)
+    import __graft_entry__ as g
+    g.build()
+    from paper_2003_04296_gb300 import minw
+    r = minw.minw_measure_pipe_rates()
+    if rank != 0:
+        return None
+    mhz = r["sm_clock_mhz"]
+    per_clk = lambda v: v / (SMS * mhz * 1e6)
+    paths = {"popcount (XOR + POPC, 32 binary MACs per popc)": 2.0 * 32 * r["popc_per_s"],
+             "mma.sync b1 xor.popc": 2.0 * r["bmma_b1_mac_per_s"],
+             "mma.sync s8": 2.0 * r["imma_s8_mac_per_s"],
+             "tcgen05 kind::f8f6f4 E4M3 (N=256)": r["tc_e4m3_flop_per_s"][1],
+             "tcgen05 kind::mxf4 E2M1 (N=256)": r["tc_e2m1_flop_per_s"][1]}
+    return {"metric": "pipe rates of the quantized convolution's candidate paths", "n_gpus": 1,
+            "value": r["tc_e2m1_flop_per_s"][1] / 1e12, "unit": "TFLOP/s (tcgen05 E2M1, N = 256)",
+            "higher_is_better": True, "data": "synthetic", "config": {"workload": "pipe_rates"},
+            "rates": r,
+            "per_sm_per_clock": {"popc": per_clk(r["popc_per_s"]), "bmma_b1_mac": per_clk(r["bmma_b1_mac_per_s"]),
+                                 "imma_s8_mac": per_clk(r["imma_s8_mac_per_s"]),
+                                 "tc_e4m3_flop_n256": per_clk(r["tc_e4m3_flop_per_s"][1]),
+                                 "tc_e2m1_flop_n256": per_clk(r["tc_e2m1_flop_per_s"][1]),
+                                 "tc_bf16_flop_n256": per_clk(r["tc_bf16_flop_per_s"][1])},
+            "binary_conv_tops_by_path": {k: v / 1e12 for k, v in paths.items()}}
+
+
+def other_configs(args, rank, world, local_rank):
+    """The default run's summary of the other BASELINE workloads (each with
+    fewer steps than its own run, no CPU baseline): the single convolution,
+    the ConvNet at 2-bit activations with 1- and 2-bit weights, ResNet-18 and
+    the bit-width sweep."""
+    import copy
+    out = {}
+    jobs = [("conv1", run_conv1, dict(workload="conv1", steps=300)),
+            ("cifar_convnet_a2w1", run_gpu, dict(workload="cifar_convnet", bits_a=2, bits_w=1, steps=200)),
+            ("cifar_convnet_a2w2", run_gpu, dict(workload="cifar_convnet", bits_a=2, bits_w=2, steps=200)),
+            ("resnet18_a3w3", run_gpu, dict(workload="resnet18", steps=40)),
+            ("sweep", run_sweep, dict(workload="sweep", steps=8))]
+    for name, fn, ch in jobs:
+        a = copy.copy(args)
+        for k, v in ch.items():
+            setattr(a, k, v)
+        a.skip_cpu = True
+        r = fn(a, rank, world, local_rank)
+        if r is None:
+            continue
+        roof = r.get("roofline", {})
+        out[name] = {"workload": r["config"]["workload"], "value": r["value"], "unit": r["unit"],
+                     "ms_per_step": r["ms_per_step"], "steps": r["steps"], "dtype": r["dtype"],
+                     "roofline_frac": roof.get("frac"), "roofline_frac_probe": roof.get("frac_probe"),
+                     "roofline_kernel": roof.get("kernel"), "e2e": r.get("e2e", {}).get("value"),
+                     "clocks": r.get("clocks")}
+        for extra in ("layer_ms", "conv_ms"):
+            if extra in r:
+                out[name][extra] = r[extra]
+    return out
 
 
 def main():
@@ -847,7 +1131,8 @@ def main():
                     help="timed steps (default 1000 for the ConvNet, 100 for ResNet-18: about a second)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["minw", "reference"], default="minw")
-    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "sweep", "fc_train"], default="cifar_convnet")
+    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "sweep", "fc_train", "conv1", "peaks"],
+                    default="cifar_convnet")
     ap.add_argument("--bits-a", type=int, default=1, help="CIFAR ConvNet activation bits")
     ap.add_argument("--bits-w", type=int, default=1, help="CIFAR ConvNet weight bits")
     ap.add_argument("--model", choices=["A", "B", "C", "D"], default="A",
@@ -857,9 +1142,13 @@ def main():
     ap.add_argument("--variant", type=int, default=0, help="0 auto, 1 popcount, 2 tensor cores")
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--skip-cpu", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="default run: skip the summary of the other BASELINE configs")
     args = ap.parse_args()
+    default_run = args.steps is None and args.workload == "cifar_convnet"
     if args.steps is None:
-        args.steps = {"cifar_convnet": 1000, "resnet18": 100, "sweep": 20, "fc_train": 200}[args.workload]
+        args.steps = {"cifar_convnet": 1000, "resnet18": 100, "sweep": 20, "fc_train": 200,
+                      "conv1": 1000, "peaks": 1}[args.workload]
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -872,11 +1161,14 @@ def main():
         torch.cuda.set_device(local_rank)
         dist.init_process_group("nccl")
     try:
-        if args.workload == "sweep":
-            return run_sweep(args, rank, world, local_rank)
-        if args.workload == "fc_train":
-            return run_fc_train(args, rank, world, local_rank)
-        return run_gpu(args, rank, world, local_rank)
+        runner = {"sweep": run_sweep, "fc_train": run_fc_train, "conv1": run_conv1,
+                  "peaks": run_peaks}.get(args.workload, run_gpu)
+        line = runner(args, rank, world, local_rank)
+        if line is not None and default_run and world == 1 and not args.no_configs:
+            line["configs"] = other_configs(args, rank, world, local_rank)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return 0
     finally:
         if world > 1:
             import torch.distributed as dist

@@ -143,12 +143,15 @@ MINW_API minw_status minw_pack_weights(const float *w, int32_t O, int32_t C, int
 /* ---------------------------------------------------------------------- */
 
 enum {
-    MINW_VARIANT_AUTO = 0,    /* per-shape choice from measurements */
+    MINW_VARIANT_AUTO = 0,    /* per-shape choice from measurements: a network times each tensor-core
+                                 layer with E4M3 and with E2M1 operands at creation and keeps the
+                                 faster; the popcount path where the tensor cores do not apply */
     MINW_VARIANT_POPC = 1,    /* bit-serial XNOR/AND + popcount on the integer pipe */
     MINW_VARIANT_TC = 2,      /* tcgen05 tensor cores on exact level values: E2M1 operands where
                                  the shape allows (C % 128 == 0), else E4M3 */
     MINW_VARIANT_TC_E4M3 = 3, /* tensor cores on E4M3 operands only (a network request) */
-    MINW_VARIANT_TC_E2M1 = 4  /* reported for a network layer that runs on E2M1 operands */
+    MINW_VARIANT_TC_E2M1 = 4  /* tensor cores on E2M1 operands where the shape allows (a network
+                                 request, as MINW_VARIANT_TC); reported for a layer on E2M1 operands */
 };
 
 /* Convolution of packed activations act [B][H][W][bits_a][C/32] with packed
@@ -553,7 +556,7 @@ MINW_API minw_status minw_get_last_device_error(void *stream);
 
 /* Choices between kernel variants that compute the same results, and the
  * limit of the kernels' bounded waits.  The defaults (1, 1, 2, 1, 2, 1, 1, 1,
- * 1, 1, 2^31) are the measured fastest variants.  The options are read when a
+ * 1, 0, 2^31) are the measured fastest variants.  The options are read when a
  * launch is planned: a change applies to standalone calls made after it and
  * to networks created after it (a network keeps the plan it was created
  * with, except pdl and graph, read at every forward).
@@ -571,7 +574,10 @@ MINW_API minw_status minw_get_last_device_error(void *stream);
  *   round trip, so more issuers keep more bytes in flight).
  * - resident_weights: a tensor-core layer not split along K whose weights fit
  *   in shared memory keeps them there for all of its tiles (each CTA then
- *   works on one channel tile) instead of loading them per tile.
+ *   works on one channel tile) instead of loading them per tile.  Off by
+ *   default: it halves the loads per K block, but the shared memory the
+ *   weights take shortens the activation ring, and on GB300 the CIFAR layers
+ *   measured 0-6 % slower with it.
  * - wait_cycles: SM clocks after which a bounded wait (TMA load, MMA, TMEM
  *   hand-off) gives up; the kernel then finishes without its outputs and
  *   minw_get_last_device_error reports MINW_ETIMEOUT. */
@@ -605,6 +611,37 @@ MINW_API minw_status minw_set_plan_options(const minw_plan_options *opt);
  * One launch only; 0 cancels a pending request.  No GPU fault is involved. */
 enum { MINW_STALL_CONV_TC = 1, MINW_STALL_CONV_FIRST = 2 };
 MINW_API minw_status minw_test_stall_next_launch(int32_t kernel);
+
+/* ---------------------------------------------------------------------- */
+/* Pipe rates (no counterpart in the paper: the measurement behind the      */
+/* per-shape choice of path)                                                */
+/* ---------------------------------------------------------------------- */
+
+/* Throughput of the pipes the quantized convolution can run on, measured on
+ * the current device with all SMs busy (host struct, filled by the call):
+ * - sm_clock_mhz: SM clock during the tensor-core probes (clock64 / events);
+ * - popc_per_s: 32-bit XOR + POPC + add per second, the inner loop of the
+ *   bit-serial path (x 32 binary MACs);
+ * - bmma_b1_mac_per_s, imma_s8_mac_per_s: the legacy warp MMAs the toolchain
+ *   exposes for sm_103a (mma.sync m16n8k256 b1 xor.popc, m16n8k32 s8);
+ * - tc_e4m3 / tc_e2m1 / tc_bf16_flop_per_s[j]: tcgen05.mma kind::f8f6f4,
+ *   kind::mxf4 (unit scales) and kind::f16 at M = 128 and N = 128 (j = 0) or
+ *   256 (j = 1), issued warp-uniformly with a commit every four MMAs;
+ * - tma_box_cycles: SM clocks one issuing thread spends per 32 KB 4D TMA
+ *   box (128-byte rows) from L2 with three boxes in flight.
+ * Allocates about 10 MB of device memory for the call and runs about a second
+ * of kernels on stream; MINW_ETIMEOUT if a bounded wait ran out. */
+typedef struct {
+    double sm_clock_mhz;
+    double popc_per_s;
+    double bmma_b1_mac_per_s;
+    double imma_s8_mac_per_s;
+    double tc_e4m3_flop_per_s[2];
+    double tc_e2m1_flop_per_s[2];
+    double tc_bf16_flop_per_s[2];
+    double tma_box_cycles;
+} minw_pipe_rates;
+MINW_API minw_status minw_measure_pipe_rates(minw_pipe_rates *out, void *stream);
 
 #ifdef __cplusplus
 }

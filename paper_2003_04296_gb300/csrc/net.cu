@@ -13,6 +13,7 @@
 #include <stdint.h>
 #include <stdlib.h>
 
+#include <algorithm>
 #include <vector>
 
 #include "net.cuh"
@@ -39,12 +40,133 @@ static minw_status net_alloc(minw_net *n, T **p, size_t count) {
     return MINW_OK;
 }
 
+// Time one tensor-core launch: one warm-up, then the least of three runs (ms).
+static minw_status time_conv_tc(const ConvArgs &a, cudaStream_t s, cudaEvent_t e0, cudaEvent_t e1, float *ms) {
+    minw_status st = launch_conv_tc(a, s);
+    if (st != MINW_OK) return st;
+    float best = 1e30f;
+    for (int r = 0; r < 3; ++r) {
+        if (cudaEventRecord(e0, s) != cudaSuccess) return MINW_ECUDA;
+        if ((st = launch_conv_tc(a, s)) != MINW_OK) return st;
+        if (cudaEventRecord(e1, s) != cudaSuccess || cudaEventSynchronize(e1) != cudaSuccess) return MINW_ECUDA;
+        float t = 0.0f;
+        cudaEventElapsedTime(&t, e0, e1);
+        if (t < best) best = t;
+    }
+    *ms = best;
+    return MINW_OK;
+}
+
+// The measured choice between E4M3 and E2M1 operands for every tensor-core
+// layer whose channels allow both (north of the pipe rates, the layer's
+// tiling, accumulator count and epilogue decide which runs faster: on GB300
+// E2M1 wins on most layers but not on all).  Each candidate runs on the
+// layer's shape at the net's batch with its own weight codes, breakpoints
+// and split workspace, into scratch buffers; the faster is kept (P.in4) and
+// the shared workspace is sized for the choices.
+static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int n_layers, int max_batch,
+                                cudaStream_t s) {
+    size_t in_b = 0, out_b = 0, w_b = 0, ws_b = 0;
+    std::vector<int> cand;
+    for (int l = 1; l < n_layers; ++l) {
+        const LayerPlan &P = n->L[l];
+        if (P.variant != MINW_VARIANT_TC || P.C % 128 != 0) continue;
+        cand.push_back(l);
+        in_b = std::max(in_b, (size_t)max_batch * P.H * P.W * P.C);
+        out_b = std::max(out_b, (size_t)max_batch * P.Hp * P.Wp * P.O * sizeof(float));   // codes or fp32 logits
+        w_b = std::max(w_b, (size_t)P.O * P.kh * P.kw * P.C);
+    }
+    if (cand.empty()) return MINW_OK;
+    std::vector<void *> tmp;
+    auto talloc = [&](size_t bytes, void **p) -> minw_status {
+        if (cudaMalloc(p, bytes + 256) != cudaSuccess) return MINW_ECUDA;
+        tmp.push_back(*p);
+        return MINW_OK;
+    };
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    minw_status st = MINW_OK;
+    void *xin = nullptr, *yout = nullptr, *w8 = nullptr, *w4 = nullptr, *thr = nullptr, *ws = nullptr;
+    do {
+        if (cudaEventCreate(&e0) != cudaSuccess || cudaEventCreate(&e1) != cudaSuccess) { st = MINW_ECUDA; break; }
+        if ((st = talloc(in_b, &xin)) != MINW_OK || (st = talloc(out_b, &yout)) != MINW_OK ||
+            (st = talloc(w_b, &w8)) != MINW_OK || (st = talloc(w_b, &w4)) != MINW_OK ||
+            (st = talloc(4096 * 8 * sizeof(float), &thr)) != MINW_OK)
+            break;
+        // +1 levels in both formats (E4M3 0x38; E2M1 0x2 in each nibble)
+        if (cudaMemsetAsync(xin, 0x22, in_b, s) != cudaSuccess) { st = MINW_ECUDA; break; }
+        for (int l : cand) {
+            LayerPlan &P = n->L[l];
+            const minw_layer_desc &d = layers[l];
+            const bool last = l == n_layers - 1;
+            ConvArgs a{};
+            a.B = max_batch; a.C = P.C; a.H = P.H; a.W = P.W; a.O = P.O; a.kh = P.kh; a.kw = P.kw;
+            a.stride = P.stride; a.pad = P.pad; a.Ho = P.Ho; a.Wo = P.Wo; a.NW = P.C / 32;
+            a.bits_a = d.bits_in; a.bits_w = d.bits_w;
+            a.M = (long long)max_batch * P.Ho * P.Wo;
+            a.scale = P.scale; a.shift = P.shift; a.pool = P.pool;
+            a.quant_out = !last;
+            if (!last) {
+                a.qo = to_qparams(&P.qo);
+                if (P.O > 4096) { st = MINW_EUNSUPPORTED; break; }
+                if ((st = launch_thresholds(P.scale, P.shift, P.O, a.qo, (float *)thr, s)) != MINW_OK) break;
+                a.thr = (const float *)thr;
+                a.codes_out = (uint8_t *)yout;
+            } else {
+                a.y_out = (float *)yout;
+            }
+            float t[2] = {0.0f, 0.0f};
+            for (int f = 0; f < 2 && st == MINW_OK; ++f) {
+                ConvArgs b = a;
+                b.fp4 = f;
+                b.codes_out4 = f && !last;
+                if (!conv_tc_supported(b)) { t[f] = 1e30f; continue; }
+                void *wq = f ? w4 : w8;
+                st = f ? minw_pack_weight_codes_e2m1(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, (uint8_t *)wq, s)
+                       : minw_pack_weight_codes(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, (uint8_t *)wq, s);
+                if (st != MINW_OK) break;
+                b.act8 = (const uint8_t *)xin;
+                b.wgt8 = (const uint8_t *)wq;
+                const size_t need = conv_tc_workspace_bytes(b);
+                if (need > ws_b) {
+                    if (ws) { cudaStreamSynchronize(s); cudaFree(ws); tmp.erase(std::find(tmp.begin(), tmp.end(), ws)); ws = nullptr; }
+                    if ((st = talloc(need, &ws)) != MINW_OK) break;
+                    if (cudaMemsetAsync(ws, 0, need, s) != cudaSuccess) { st = MINW_ECUDA; break; }
+                    ws_b = need;
+                }
+                b.workspace = ws;
+                b.workspace_bytes = ws_b;
+                st = time_conv_tc(b, s, e0, e1, &t[f]);
+            }
+            if (st != MINW_OK) break;
+            P.in4 = t[1] < t[0] ? 1 : 0;
+        }
+    } while (false);
+    cudaStreamSynchronize(s);
+    if (e0) cudaEventDestroy(e0);
+    if (e1) cudaEventDestroy(e1);
+    for (void *p : tmp) cudaFree(p);
+    if (st != MINW_OK) return st;
+    // the shared split workspace, for the chosen formats
+    n->ws_bytes = 0;
+    for (int l = 1; l < n_layers; ++l) {
+        const LayerPlan &P = n->L[l];
+        if (P.variant != MINW_VARIANT_TC) continue;
+        ConvArgs a{};
+        a.B = max_batch; a.C = P.C; a.H = P.H; a.W = P.W; a.O = P.O; a.kh = P.kh; a.kw = P.kw;
+        a.stride = P.stride; a.pad = P.pad; a.Ho = P.Ho; a.Wo = P.Wo; a.NW = P.C / 32;
+        a.M = (long long)max_batch * P.Ho * P.Wo; a.pool = P.pool; a.quant_out = l + 1 < n_layers;
+        a.fp4 = P.in4;
+        n->ws_bytes = std::max(n->ws_bytes, conv_tc_workspace_bytes(a));
+    }
+    return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
+}
+
 extern "C" {
 
 minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int32_t max_batch,
                             int32_t variant, void *stream, minw_net **out) {
     if (!layers || n_layers < 2 || max_batch <= 0 || !out) return MINW_EINVAL;
-    if (variant < 0 || variant > 3) return MINW_EINVAL;
+    if (variant < 0 || variant > 4) return MINW_EINVAL;
     *out = nullptr;
     cudaStream_t s = (cudaStream_t)stream;
     minw_net *n = new minw_net();
@@ -130,7 +252,7 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
             a.pool = P.pool;
             a.quant_out = !last;
             if (!last) a.qo = to_qparams(&P.qo);
-            P.variant = choose_variant(a, variant == MINW_VARIANT_TC_E4M3 ? MINW_VARIANT_TC : variant);
+            P.variant = choose_variant(a, variant >= MINW_VARIANT_TC ? MINW_VARIANT_TC : variant);
             if (P.variant == MINW_VARIANT_TC && !conv_tc_supported(a)) { net_free(n); return MINW_EUNSUPPORTED; }
             if (P.variant == MINW_VARIANT_TC && variant != MINW_VARIANT_TC_E4M3) {
                 // E2M1 operands wherever the channels fill 64-byte rows
@@ -145,6 +267,12 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
         }
         pc = P.O; ph = P.Hp; pw = P.Wp; pbits = d.bits_out;
         n->L.push_back(P);
+    }
+    // MINW_VARIANT_AUTO: the operand format of each tensor-core layer that can
+    // take both is chosen by measurement (tune_formats)
+    if (variant == MINW_VARIANT_AUTO) {
+        minw_status st = tune_formats(n, layers, n_layers, max_batch, s);
+        if (st != MINW_OK) { net_free(n); return st; }
     }
     // input layouts follow the consumer's kernel; weights are quantized once
     for (int l = 1; l < n_layers; ++l) {

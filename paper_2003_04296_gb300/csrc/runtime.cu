@@ -30,7 +30,7 @@ minw_plan_options defaults() {
     o.pdl = 1;
     o.graph = 1;
     o.tma_lanes = 1;
-    o.resident_weights = 1;
+    o.resident_weights = 0;
     o.wait_cycles = (int64_t)1 << 31;
     return o;
 }

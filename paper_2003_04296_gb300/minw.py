@@ -48,6 +48,13 @@ class PlanOptions(ctypes.Structure):
 STALL_CONV_TC, STALL_CONV_FIRST = 1, 2
 
 
+class PipeRates(ctypes.Structure):
+    _fields_ = [("sm_clock_mhz", ctypes.c_double), ("popc_per_s", ctypes.c_double),
+                ("bmma_b1_mac_per_s", ctypes.c_double), ("imma_s8_mac_per_s", ctypes.c_double),
+                ("tc_e4m3_flop_per_s", ctypes.c_double * 2), ("tc_e2m1_flop_per_s", ctypes.c_double * 2),
+                ("tc_bf16_flop_per_s", ctypes.c_double * 2), ("tma_box_cycles", ctypes.c_double)]
+
+
 class LayerDesc(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int32), ("C", ctypes.c_int32), ("H", ctypes.c_int32),
                 ("W", ctypes.c_int32), ("O", ctypes.c_int32), ("kh", ctypes.c_int32),
@@ -112,6 +119,7 @@ SIGNATURES = {
     "minw_get_plan_options": (ctypes.c_int, [ctypes.POINTER(PlanOptions)]),
     "minw_set_plan_options": (ctypes.c_int, [ctypes.POINTER(PlanOptions)]),
     "minw_test_stall_next_launch": (ctypes.c_int, [_I32]),
+    "minw_measure_pipe_rates": (ctypes.c_int, [ctypes.POINTER(PipeRates), _P]),
     "minw_fc_codes": (ctypes.c_int, [_P, _I32, _I32, _I32, _P, _I32, _I32, _P, _P, _QP, _P, _P, _P, _P, _P,
                                      ctypes.c_size_t, _P]),
     "minw_fc_codes_noalloc": (ctypes.c_int, [_P, _I32, _I32, _I32, _P, _I32, _I32, _P, _P, _QP, _P, _P, _P, _P,
@@ -416,6 +424,18 @@ def set_plan_options(opts=None, **changes):
     cur.update(changes)
     o = PlanOptions(**cur)
     _check(lib().minw_set_plan_options(ctypes.byref(o)), "minw_set_plan_options")
+
+
+def minw_measure_pipe_rates(stream=None):
+    """minw_measure_pipe_rates as a dict (two-element lists for the N = 128 /
+    N = 256 tensor-core rates)."""
+    r = PipeRates()
+    _check(lib().minw_measure_pipe_rates(ctypes.byref(r), _stream(stream)), "minw_measure_pipe_rates")
+    out = {}
+    for name, _ in PipeRates._fields_:
+        v = getattr(r, name)
+        out[name] = list(v) if hasattr(v, "__len__") else float(v)
+    return out
 
 
 def minw_test_stall_next_launch(kernel):

@@ -2,12 +2,14 @@
 - a single 3x3 convolution, 4x128x32x32, 1-bit x 1-bit, int32 accumulators and
   the fp32 scale epilogue, every output checked (popcount and tensor-core paths);
 - the bit-width sweep 256x512x14x14 -> 512 channels, (M, N) in {1,2,3}^2, on the
-  tensor-core path, with images 0 and 255 re-computed by the oracle (the
-  images of a batch are independent);
+  tensor-core path with E4M3 and with E2M1 operands, 16 images spread over the
+  batch (so over every wave of tiles, the last partial one included)
+  re-computed by the oracle (the images of a batch are independent);
 - AQE forward/backward and quantize + pack on the full 256x512x14x14 tensor;
 - the CIFAR ConvNet with 2-bit activations x 1- and 2-bit weights at batch 256,
-  images 0 and 255 re-run by the oracle, and one layer fed |N(0,1)| clipped
-  to [0, 1] activations."""
+  16 spread images re-run by the oracle, and one layer fed |N(0,1)| clipped
+  to [0, 1] activations (16 spread images).
+The oracle's runs are spread over the host's cores (tests/_oracle_pool.py)."""
 from itertools import product
 
 import numpy as np
@@ -19,6 +21,7 @@ from oracle import network as N  # noqa: E402
 from oracle import oracle as O  # noqa: E402
 from paper_2003_04296_gb300.inputs import (DEFAULT_THR, aqe_problem, conv_problem, convnet_input,  # noqa: E402
                                            convnet_params)
+from tests import _oracle_pool as OP  # noqa: E402
 from tests._gpu import assert_close, dev_tensor, planes_view  # noqa: E402
 
 pytestmark = pytest.mark.gpu
@@ -73,9 +76,13 @@ def test_single_conv_4x128x32x32_both_paths(dev, M):
     assert np.array_equal(y.cpu().numpy(), yref)
 
 
+SWEEP_SPEC = (5, 256, 512, 14, 14, 512, 3, 1, 1, "normal", 1.0)
+
+
 @pytest.fixture(scope="module")
 def sweep_input():
-    return conv_problem(5, 256, 512, 14, 14, 512, 3, 3, 1, 1, 1, 1, x_dist="normal", w_sigma=1.0)
+    s = SWEEP_SPEC
+    return conv_problem(s[0], s[1], s[2], s[3], s[4], s[5], s[6], s[6], s[7], s[8], 1, 1, x_dist=s[9], w_sigma=s[10])
 
 
 @pytest.mark.parametrize("ba,bw", list(product([1, 2, 3], [1, 2, 3])))
@@ -84,19 +91,27 @@ def test_bitwidth_sweep_256x512x14x14(dev, M, sweep_input, ba, bw):
     p = dict(base, bits_a=ba, bits_w=bw, thr_a=DEFAULT_THR[ba], thr_w=DEFAULT_THR[bw],
              w_scale=(np.ones(512, np.float32) if bw == 1 else
                       (1.0 / np.abs(base["w"].reshape(512, -1)).max(1)).astype(np.float32)))
+    idx = OP.spread(256)
+    refs = OP.starmap(OP.conv_acc, [(SWEEP_SPEC, ba, bw, "ones" if bw == 1 else "max", i) for i in idx])
     x, w = dev_tensor(p["x"], dev), dev_tensor(p["w"], dev)
-    a8 = torch.empty((256, 14, 14, 512), dtype=torch.uint8, device=dev)
-    w8 = torch.empty((512, 3, 3, 512), dtype=torch.uint8, device=dev)
-    M.aqe_quantize_codes(x, M.quant(ba, p["thr_a"]), a8)
-    M.minw_pack_weight_codes(w, M.quant(bw, p["thr_w"]), w8, channel_scale=dev_tensor(p["w_scale"], dev))
+    ws = dev_tensor(p["w_scale"], dev)
     acc = torch.empty((256, 512, 14, 14), dtype=torch.int32, device=dev)
-    M.minw_conv2d_codes(a8, 256, 512, 14, 14, ba, w8, 512, 3, 3, bw, 1, 1, acc_out=acc)
-    got = acc.cpu().numpy()
-    wl = O.quantize(p["w"], bw, p["thr_w"], p["w_scale"])
-    for i in (0, 255):
-        al = O.quantize(p["x"][i:i + 1], ba, p["thr_a"])
-        ref = O.conv2d_levels(al, wl, 1, 1, ba, bw)
-        assert np.array_equal(got[i:i + 1], ref), f"image {i}: {np.sum(got[i:i + 1] != ref)} accumulators differ"
+    for fmt in (M.CODES_E4M3, M.CODES_E2M1):
+        cb = 512 if fmt == M.CODES_E4M3 else 256
+        a8 = torch.empty((256, 14, 14, cb), dtype=torch.uint8, device=dev)
+        w8 = torch.empty((512, 3, 3, cb), dtype=torch.uint8, device=dev)
+        if fmt == M.CODES_E4M3:
+            M.aqe_quantize_codes(x, M.quant(ba, p["thr_a"]), a8)
+            M.minw_pack_weight_codes(w, M.quant(bw, p["thr_w"]), w8, channel_scale=ws)
+        else:
+            M.aqe_quantize_codes_e2m1(x, M.quant(ba, p["thr_a"]), a8)
+            M.minw_pack_weight_codes_e2m1(w, M.quant(bw, p["thr_w"]), w8, channel_scale=ws)
+        acc.fill_(-7)
+        M.minw_conv_block_codes_ex(a8, 256, 512, 14, 14, ba, w8, 512, 3, 3, bw, 1, 1, 0, None, None,
+                                   in_format=fmt, acc_out=acc)
+        got = acc.cpu().numpy()
+        for i, ref in zip(idx, refs):
+            assert np.array_equal(got[i:i + 1], ref), f"format {fmt}, image {i}: {np.sum(got[i:i + 1] != ref)} differ"
     assert M.minw_get_last_device_error() == M.MINW_OK
 
 
@@ -131,8 +146,10 @@ def test_cifar_convnet_2bit_activations_batch256(dev, M, bits_w):
     torch.cuda.synchronize()
     got = logits.cpu().numpy()
     net.close()
-    for i in (0, 255):
-        assert np.array_equal(got[i:i + 1], N.convnet_forward(net_p, x[i:i + 1]))
+    idx = OP.spread(256)
+    refs = OP.starmap(OP.convnet_logits, [(3, 2, bits_w, 3, 256, i) for i in idx])
+    for i, ref in zip(idx, refs):
+        assert np.array_equal(got[i:i + 1], ref), f"image {i}"
 
 
 def test_clipped_abs_normal_activations_layer(dev, M):
@@ -151,10 +168,10 @@ def test_clipped_abs_normal_activations_layer(dev, M):
                             dev_tensor(p["shift"], dev), q_out=M.quant(2, DEFAULT_THR[2]), codes_out=codes,
                             y_out=y)
     got = y.cpu().numpy()
-    wl = O.quantize(p["w"], 2, DEFAULT_THR[2], p["w_scale"])
-    for i in (0, 255):
-        al = O.quantize(p["x"][i:i + 1], 2, DEFAULT_THR[2])
-        assert np.all(al >= 0)
-        acc = O.maxpool_i32(O.conv2d_levels(al, wl, 1, 1, 2, 2), 2, 2)
-        yr = O.hardtanh(O.affine(acc, p["scale"], p["shift"]))
-        assert np.array_equal(got[i:i + 1], yr)
+    assert np.all(p["x"] >= 0)
+    idx = OP.spread(256)
+    spec = (33, 256, 128, 32, 32, 128, 3, 1, 1, "absnormal_clip", 0.05)
+    accs = OP.starmap(OP.conv_acc, [(spec, 2, 2, "max", i) for i in idx])
+    for i, acc in zip(idx, accs):
+        yr = O.hardtanh(O.affine(O.maxpool_i32(acc, 2, 2), p["scale"], p["shift"]))
+        assert np.array_equal(got[i:i + 1], yr), f"image {i}"

@@ -255,7 +255,7 @@ def test_convnet_e2m1_layers(dev, M, bits_a, bits_w):
                            pools=(False, True, False, True), fcs=(256,), classes=10, hw=16)
     x = convnet_input(54, 7, hw=16)
     outs = []
-    for variant in (M.VARIANT_AUTO, M.VARIANT_TC_E4M3):
+    for variant in (M.VARIANT_TC_E2M1, M.VARIANT_TC_E4M3):
         net = M.Net(M.layer_descs(net_p, dev), max_batch=7, variant=variant)
         logits = torch.empty((7, net.out_features), dtype=torch.float32, device=dev)
         net.forward(dev_tensor(x, dev), logits)
@@ -268,4 +268,22 @@ def test_convnet_e2m1_layers(dev, M, bits_a, bits_w):
     ref = N.convnet_forward(net_p, x)
     assert np.array_equal(got, ref)
     assert np.array_equal(got8, ref)
+    assert M.minw_get_last_device_error() == M.MINW_OK
+
+
+def test_convnet_measured_formats(dev, M):
+    """VARIANT_AUTO times every tensor-core layer with E4M3 and with E2M1
+    operands at creation and keeps the faster: whatever it picks, each layer
+    reports one of the two, and the logits equal the oracle's bit for bit."""
+    net_p = convnet_params(55, bits_a=1, bits_w=1, widths=(128, 128, 256, 256),
+                           pools=(False, True, False, True), fcs=(256,), classes=10, hw=16)
+    x = convnet_input(56, 9, hw=16)
+    net = M.Net(M.layer_descs(net_p, dev), max_batch=9, variant=M.VARIANT_AUTO)
+    logits = torch.empty((9, net.out_features), dtype=torch.float32, device=dev)
+    net.forward(dev_tensor(x, dev), logits)
+    torch.cuda.synchronize()
+    var = net.layer_variants()
+    net.close()
+    assert all(v in (M.VARIANT_TC, M.VARIANT_TC_E2M1) for v in var[1:])
+    assert np.array_equal(logits.cpu().numpy(), N.convnet_forward(net_p, x))
     assert M.minw_get_last_device_error() == M.MINW_OK

@@ -76,11 +76,14 @@ def test_cifar_models_b_to_d(dev, M, model, bits_a, bits_w):
 
 def test_cifar_convnet_batch256_sampled(dev, M):
     """The full Model-A-shaped ConvNet (128-128-P-256-256-P-512-512-P,
-    FC 1024-1024-10), 1-bit, batch 256; images 0 and 255 re-run by the oracle."""
+    FC 1024-1024-10), 1-bit, batch 256: 16 images spread over the batch (every
+    wave of tiles, the last one included) re-run by the oracle, bit for bit."""
+    from tests import _oracle_pool as OP
     net_p = convnet_params(2, bits_a=1, bits_w=1)
     x = convnet_input(2, 256)
     got = _run(dev, M, net_p, x, M.VARIANT_AUTO)
     assert np.all(np.isfinite(got))
-    for i in (0, 255):
-        ref = N.convnet_forward(net_p, x[i:i + 1])
-        assert_close(got[i:i + 1], ref)
+    idx = OP.spread(256)
+    refs = OP.starmap(OP.convnet_logits, [(2, 1, 1, 2, 256, i) for i in idx])
+    for i, ref in zip(idx, refs):
+        assert np.array_equal(got[i:i + 1], ref), f"image {i}"

@@ -66,8 +66,8 @@ OPTION_CASES = [
     dict(kblocks_per_stage=1),
     dict(tma_lanes=1),
     dict(tma_lanes=8),
-    dict(resident_weights=0),
-    dict(resident_weights=0, tma_lanes=2),
+    dict(resident_weights=1),
+    dict(resident_weights=1, tma_lanes=2),
     dict(first_tma=0),
     dict(pdl=0),
     dict(graph=0),

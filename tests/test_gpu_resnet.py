@@ -88,12 +88,15 @@ def test_resnet_create_errors(dev, M):
 def test_resnet18_imagenet_b128_sampled(dev, M):
     """The ImageNet-shaped workload: batch 128 of 224x224 images, 3-bit
     activations and weights, 1000 classes; images are independent, so the
-    oracle checks three of them (first, middle, last) bit for bit."""
+    oracle checks 16 of them spread over the batch (every wave of tiles of
+    every layer, the last one included) bit for bit."""
+    from tests import _oracle_pool as OP
     params = resnet18_params(0, bits_a=3, bits_w=3, classes=1000, hw=224)
     x = resnet18_input(1, 128, hw=224)
     net, got = _forward(M, dev, params, x)
     net.close()
     assert np.all(np.isfinite(got))
-    for i in (0, 63, 127):
-        ref = N.resnet18_forward(params, x[i:i + 1])
+    idx = OP.spread(128)
+    refs = OP.starmap(OP.resnet_logits, [(0, 3, 3, 1000, 224, 1, 128, i) for i in idx])
+    for i, ref in zip(idx, refs):
         assert np.array_equal(got[i:i + 1], ref), f"image {i}"

@@ -141,7 +141,7 @@ def _within(got, ref, bound, what):
     assert (err <= bound).all(), f"{what}: worst err/bound {np.max(err / bound)}"
 
 
-@pytest.mark.parametrize("case", CASES + [(256, 8192, 1024, 0.75, 1, 1)])
+@pytest.mark.parametrize("case", CASES + [(256, 8192, 1024, 0.75, 1, 1), (1152, 256, 256, 0.5, 1, 2)])
 @pytest.mark.parametrize("last", [False, True])
 def test_train_step(dev, M, case, last):
     """minw_fc_train_step against the oracle's Algorithm 1 step at the paper's
@@ -150,7 +150,9 @@ def test_train_step(dev, M, case, last):
     equals the oracle's bit for bit, g_in lies within the bound of g~ W^, and
     the updated W within lr 2 alpha times the bound of g~^T A plus one fp32 ulp.
     (256, 8192, 1024) is fc1 of the CIFAR model at the training bench's batch,
-    whose forward product splits along K.  A second step from the same inputs
+    whose forward product splits along K; at (1152, 256, 256) the weight
+    gradient's product (contraction over the batch: 18 K blocks, 256 output
+    rows) runs on CTA pairs with the update in their staged-store epilogue.  A second step from the same inputs
     gives the same bits (the K slices add in a fixed order)."""
     B, K, O_, alpha, bw, ba = case
     lr = 0.05

@@ -129,6 +129,32 @@ def test_conv2d_bf16_sweep_shape_sampled(dev, M):
     assert (err <= bound).all(), f"worst err/bound {np.max(err / bound)}"
 
 
+@pytest.mark.parametrize("B,K,O_", [(256, 1152, 256), (200, 2048, 512)])
+def test_conv2d_bf16_fully_connected_cta_pairs(dev, M, B, K, O_):
+    """A fully connected shape long enough for CTA pairs (K / 64 >= 18 bf16 K
+    blocks, O a multiple of 256, no workspace): the pair kernel with the
+    row-contiguous staged stores of 1 x 1 outputs, against the oracle within
+    the fp32 accumulation bound; B = 200 leaves a ragged, odd pixel tile."""
+    r = np.random.default_rng(B + K + O_)
+    x = r.standard_normal((B, K, 1, 1)).astype(np.float32)
+    w = r.normal(0, 0.05, (O_, K, 1, 1)).astype(np.float32)
+    cs = (1.0 / np.abs(w.reshape(O_, -1)).max(1)).astype(np.float32)
+    scale = r.normal(0.01, 0.005, O_).astype(np.float32)
+    shift = r.normal(0, 0.1, O_).astype(np.float32)
+    xb, wb = _operands(dev, M, x, w, 1, cs)
+    y = torch.full((B, O_, 1, 1), np.nan, dtype=torch.float32, device=dev)
+    M.minw_conv2d_bf16(xb, B, K, 1, 1, wb, O_, 1, 1, 1, 1, 0, 0, dev_tensor(scale, dev), dev_tensor(shift, dev), y)
+    torch.cuda.synchronize()
+    xr = O.bf16_round(x).reshape(B, K).astype(np.float64)
+    wu = O.quantize(w, 1, DEFAULT_THR[1], cs).reshape(O_, K).astype(np.float64)
+    acc, A = xr @ wu.T, np.abs(xr) @ np.abs(wu).T
+    yref = acc * scale.astype(np.float64) + shift.astype(np.float64)
+    bound = np.abs(scale.astype(np.float64)) * K * 2.0 ** -23 * A + 2.0 ** -23 * np.abs(yref) + 1e-30
+    err = np.abs(y.cpu().numpy().reshape(B, O_).astype(np.float64) - yref)
+    assert (err <= bound).all(), f"worst err/bound {np.max(err / bound)}"
+    assert M.minw_get_last_device_error() == M.MINW_OK
+
+
 def test_conv2d_bf16_errors(dev, M):
     xb = torch.zeros((1, 4, 4, 32), dtype=torch.int16, device=dev)
     wb = torch.zeros((8, 3, 3, 32), dtype=torch.int16, device=dev)
