@@ -578,6 +578,11 @@ MINW_API minw_status minw_get_last_device_error(void *stream);
  *   default: it halves the loads per K block, but the shared memory the
  *   weights take shortens the activation ring, and on GB300 the CIFAR layers
  *   measured 0-6 % slower with it.
+ * - first_tensor_cores: a first layer whose output is the next layer's
+ *   levels (O a multiple of 64 up to 256) runs on the tensor cores with fp16
+ *   split operands and an error bound, recomputing exactly the outputs whose
+ *   level the bound leaves open (the levels are those of the fp32 chain
+ *   either way); else the fp32 chain runs on the CUDA cores for every output.
  * - wait_cycles: SM clocks after which a bounded wait (TMA load, MMA, TMEM
  *   hand-off) gives up; the kernel then finishes without its outputs and
  *   minw_get_last_device_error reports MINW_ETIMEOUT. */
@@ -592,6 +597,7 @@ typedef struct {
     int32_t graph;
     int32_t tma_lanes;
     int32_t resident_weights;
+    int32_t first_tensor_cores;
     int64_t wait_cycles;
 } minw_plan_options;
 

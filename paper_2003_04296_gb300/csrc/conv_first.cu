@@ -555,6 +555,7 @@ int take_first_error() {
 }
 
 minw_status launch_conv_first(const FirstArgs &a, cudaStream_t s) {
+    if (minw_host::plan_options().first_tensor_cores != 0 && first_tc_supported(a)) return launch_first_tc(a, s);
     const bool tma_ok = first_tma_pref() && tma_shape(a) && a.W % 4 == 0 && minw_host::aligned16(a.x) &&
                         minw_host::tensor_map_encoder() != nullptr;
     FirstTile tl = first_tile(a, tma_ok);

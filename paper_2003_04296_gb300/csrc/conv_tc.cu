@@ -2006,8 +2006,9 @@ extern "C" minw_status minw_get_last_device_error(void *stream) {
         if (cudaMemcpyToSymbol(minw::g_device_error, &zero, sizeof(int)) != cudaSuccess) return MINW_ECUDA;
     }
     const int first = minw::take_first_error();
-    if (first < 0) return MINW_ECUDA;
-    return (flag || first) ? MINW_ETIMEOUT : MINW_OK;
+    const int first_tc = minw::take_first_tc_error();
+    if (first < 0 || first_tc < 0) return MINW_ECUDA;
+    return (flag || first || first_tc) ? MINW_ETIMEOUT : MINW_OK;
 }
 
 minw_host::EncodeTiledFn minw_host::tensor_map_encoder() {

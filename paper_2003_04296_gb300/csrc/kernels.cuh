@@ -71,6 +71,11 @@ struct FirstArgs {
 
 // Launchers (host).  Return MINW_OK or an error status.
 minw_status launch_conv_first(const FirstArgs &a, cudaStream_t s);
+// The tensor-core first layer (conv_first_tc.cu): whether it applies, its
+// launch, and its timeout flag (as take_first_error).
+bool first_tc_supported(const FirstArgs &a);
+minw_status launch_first_tc(const FirstArgs &a, cudaStream_t s);
+int take_first_tc_error();
 // The first-layer kernels' timeout flag: 1 if set (and clears it), 0, or -1 on a CUDA error.
 int take_first_error();
 minw_status launch_ythresholds(const QParams &q, float *out, cudaStream_t s);

@@ -3,7 +3,8 @@
 //
 // The plan options pick between kernel variants that compute the same result
 // (CTA pairs, channel-major tiles, the 64-channel weight duplication, K blocks
-// per pipeline stage, TMA first-layer patches, programmatic dependent launch,
+// per pipeline stage, TMA first-layer patches, the tensor-core first layer,
+// programmatic dependent launch,
 // graph replay of a network forward) and set the limit of every bounded wait.
 // The defaults are the measured fastest choices; they are read when a launch
 // is planned, so a change applies to standalone calls made after it and to
@@ -31,6 +32,7 @@ minw_plan_options defaults() {
     o.graph = 1;
     o.tma_lanes = 1;
     o.resident_weights = 0;
+    o.first_tensor_cores = 1;
     o.wait_cycles = (int64_t)1 << 31;
     return o;
 }

@@ -42,7 +42,8 @@ class PlanOptions(ctypes.Structure):
                 ("channel_major_min_tiles_per_sm", ctypes.c_int32), ("dup_weights", ctypes.c_int32),
                 ("kblocks_per_stage", ctypes.c_int32), ("first_tma", ctypes.c_int32), ("pdl", ctypes.c_int32),
                 ("graph", ctypes.c_int32), ("tma_lanes", ctypes.c_int32),
-                ("resident_weights", ctypes.c_int32), ("wait_cycles", ctypes.c_int64)]
+                ("resident_weights", ctypes.c_int32), ("first_tensor_cores", ctypes.c_int32),
+                ("wait_cycles", ctypes.c_int64)]
 
 
 STALL_CONV_TC, STALL_CONV_FIRST = 1, 2

@@ -69,6 +69,8 @@ OPTION_CASES = [
     dict(resident_weights=1),
     dict(resident_weights=1, tma_lanes=2),
     dict(first_tma=0),
+    dict(first_tensor_cores=0),
+    dict(first_tensor_cores=0, first_tma=0),
     dict(pdl=0),
     dict(graph=0),
 ]
