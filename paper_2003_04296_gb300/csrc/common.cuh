@@ -327,6 +327,11 @@ minw_status launch_status();
 bool pdl_enabled();                 // plan option pdl
 minw_plan_options plan_options();   // the process-wide plan options (runtime.cu)
 int take_stall(int which);          // 1 once after minw_test_stall_next_launch(which)
+// Every kernel of the library asks for the largest shared-memory carve-out
+// of the SM (set once per kernel): consecutive kernels of a forward then need
+// no L1 / shared-memory reconfiguration of the SM between them, so the next
+// kernel's CTAs start as soon as an SM frees up.
+void max_shared_carveout(const void *kern);
 
 // cuTensorMapEncodeTiled from the driver (nullptr when it is unavailable).
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
@@ -349,6 +354,7 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = pdl_enabled() ? 1 : 0;
+    max_shared_carveout(reinterpret_cast<const void *>(kern));
     return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
 

@@ -664,7 +664,8 @@ __global__ void __launch_bounds__(NT, 1)
     uint64_t *tempty = tfull + 2;             // [2] accumulator drained
     uint64_t *tstall = tempty + 2;            // timeout-path test: a barrier nothing completes
     uint64_t *wfull = tstall + 1;             // resident weights landed
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(wfull + 1);
+    uint64_t *sfready = wfull + 1;            // E2M1: the unit scale factors are in tensor memory
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(sfready + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // pixel tiles padded to a multiple of the cluster size: the CTAs of a
@@ -686,6 +687,7 @@ __global__ void __launch_bounds__(NT, 1)
         }
         mbar_init(tstall, 1);
         mbar_init(wfull, 1);
+        mbar_init(sfready, PAIR ? 8 : 4);     // one arrival per filling warp (pairs: both CTAs' on CTA 0)
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     if (warp == 1) {
@@ -701,74 +703,15 @@ __global__ void __launch_bounds__(NT, 1)
             asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n");
         }
     }
-    // output-quantizer breakpoints of every channel, in shared memory
-    if constexpr (OUTB > 0) {
-        // held as (-T_1 .. -T_{n-1}, sigma) with -0 stored as +0, so that
-        // fmaf(acc, sigma, -T) is never -0 and its sign bit is [sigma * acc < T]
-        // rows u = 0 .. NL - 1 of O32 channels each (channel fastest: four channels per 128-bit load)
-        if (p.thr != nullptr) {
-            for (int i = threadIdx.x; i < p.O * NL; i += NT) {
-                const float x = __ldg(p.thr + i);
-                const int o = i / NL, u = i - o * NL;
-                sthr[u * O32 + o] = (u == NL - 1) ? x : mask_breakpoint(x);
-            }
-        } else if (p.res_codes == nullptr && p.res_f32 == nullptr) {
-            // (a residual block quantizes y + shortcut: no per-channel breakpoints on acc)
-            for (int o = threadIdx.x; o < p.O; o += NT) {
-                float t[8];
-                channel_thresholds(__ldg(p.scale + o), __ldg(p.shift + o), p.qo, t);
-                for (int u = 0; u < NL; ++u) sthr[u * O32 + o] = (u == NL - 1) ? t[u] : mask_breakpoint(t[u]);
-            }
-        }
-        for (int i = p.O * NL + threadIdx.x; i < thr_floats; i += NT) {      // padding channels
-            const int k = i - p.O * NL, o = p.O + k / NL, u = k % NL;
-            sthr[u * O32 + o] = (u == NL - 1) ? 1.0f : 0.0f;
-        }
-        if (p.res_codes != nullptr || p.res_f32 != nullptr) {       // level of y = #{u : y >= T_u}
-            if (p.ythr != nullptr) {
-                if (threadIdx.x < NL - 1) syt[threadIdx.x] = mask_breakpoint(__ldg(p.ythr + threadIdx.x));
-            } else if (threadIdx.x == 0) {
-                float t[8];
-                channel_thresholds_f32(1.0f, 0.0f, p.qo, t);         // a long serial search: callers cache it
-                for (int u = 0; u < NL - 1; ++u) syt[u] = mask_breakpoint(t[u]);
-            }
-        }
-        // sigma of a channel: the sign of its BN scale (+1 for 0)
-        for (int g = threadIdx.x; g < sig_words; g += NT) {
-            uint32_t m = 0u;
-            for (int j = 0; j < 32; ++j) {
-                const int o = g * 32 + j;
-                const float sg = o < p.O ? (p.thr != nullptr ? __ldg(p.thr + o * NL + NL - 1)
-                                                             : (__ldg(p.scale + o) < 0.0f ? -1.0f : 1.0f))
-                                         : 1.0f;
-                m |= (sg > 0.0f ? 1u : 0u) << j;
-            }
-            ssig[g] = m;
-        }
-    }
     fence_before();
     __syncthreads();
     if constexpr (PAIR) cluster_sync_all();   // every barrier of the pair is initialised
     fence_after();
     const uint32_t tmem_base = *tmem_slot;
-    if constexpr (FMT == 2) {
-        // unit scale factors (UE8M0 0x7F = 2^0) in 64 columns from sf_col, written
-        // by one warp per TMEM lane quarter (a pair: each CTA in its own tensor memory)
-        if (warp >= 2 && warp < 6) {
-            const uint32_t ta = tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + p.sf_col;
-#pragma unroll
-            for (int c = 0; c < 64; c += 8)
-                asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %1, %1, %1, %1, %1, %1, %1};\n" ::"r"(
-                                 ta + (uint32_t)c),
-                             "r"(0x7F7F7F7Fu));
-            asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory");
-        }
-        fence_before();
-        __syncthreads();
-        if constexpr (PAIR) cluster_sync_all();   // both CTAs' scale factors are in place
-        fence_after();
-    }
-    pdl_trigger();                            // set-up done: the next kernel may start its own
+    // set-up done: the next kernel may start its own.  The TMA producers start
+    // at once; the epilogue warps first write the E2M1 unit scale factors
+    // (the MMA issuer waits for them on sfready) and load the breakpoints.
+    pdl_trigger();
 
     if (warp == 0 || warp == B_WARP) {
         if (lane < p.tlanes) {
@@ -886,6 +829,11 @@ __global__ void __launch_bounds__(NT, 1)
             // timeout-path test (single CTAs): a wait that runs out; every other
             // warp's next wait then runs out too, and the kernel winds down
             if (!PAIR && p.stall && !__all_sync(0xffffffffu, mbar_wait(tstall, 0u, p.wait_cycles))) alive = false;
+            if (FMT == 2 && alive &&
+                !__all_sync(0xffffffffu, PAIR ? mbar_wait_cluster(sfready, 0u, p.wait_cycles)
+                                              : mbar_wait(sfready, 0u, p.wait_cycles)))
+                alive = false;
+            fence_after();
             if (p.wres && alive && !__all_sync(0xffffffffu, PAIR ? mbar_wait_cluster(wfull, 0u, p.wait_cycles)
                                                                  : mbar_wait(wfull, 0u, p.wait_cycles)))
                 alive = false;
@@ -956,6 +904,72 @@ __global__ void __launch_bounds__(NT, 1)
         }
     } else if (warp < B_WARP) {
         // ---------------- epilogue: warps 2..9 ----------------
+        const int et = threadIdx.x - 64;          // 0 .. 255
+        if constexpr (FMT == 2) {
+            // unit scale factors (UE8M0 0x7F = 2^0) in 64 columns from sf_col, written
+            // by one warp per TMEM lane quarter (a pair: each CTA in its own tensor memory)
+            if (warp < 6) {
+                const uint32_t ta = tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + p.sf_col;
+#pragma unroll
+                for (int c = 0; c < 64; c += 8)
+                    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %1, %1, %1, %1, %1, %1, %1};\n" ::"r"(
+                                     ta + (uint32_t)c),
+                                 "r"(0x7F7F7F7Fu));
+                asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory");
+                fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    if (PAIR && crank == 1)
+                        mbar_arrive_cluster(cta0_addr(sfready));
+                    else
+                        mbar_arrive(sfready);
+                }
+            }
+        }
+        // output-quantizer breakpoints of every channel, in shared memory
+        if constexpr (OUTB > 0) {
+            // held as (-T_1 .. -T_{n-1}, sigma) with -0 stored as +0, so that
+            // fmaf(acc, sigma, -T) is never -0 and its sign bit is [sigma * acc < T]
+            // rows u = 0 .. NL - 1 of O32 channels each (channel fastest: four channels per 128-bit load)
+            if (p.thr != nullptr) {
+                for (int i = et; i < p.O * NL; i += EPI_WARPS * 32) {
+                    const float x = __ldg(p.thr + i);
+                    const int o = i / NL, u = i - o * NL;
+                    sthr[u * O32 + o] = (u == NL - 1) ? x : mask_breakpoint(x);
+                }
+            } else if (p.res_codes == nullptr && p.res_f32 == nullptr) {
+                // (a residual block quantizes y + shortcut: no per-channel breakpoints on acc)
+                for (int o = et; o < p.O; o += EPI_WARPS * 32) {
+                    float t[8];
+                    channel_thresholds(__ldg(p.scale + o), __ldg(p.shift + o), p.qo, t);
+                    for (int u = 0; u < NL; ++u) sthr[u * O32 + o] = (u == NL - 1) ? t[u] : mask_breakpoint(t[u]);
+                }
+            }
+            for (int i = p.O * NL + et; i < thr_floats; i += EPI_WARPS * 32) {      // padding channels
+                const int k = i - p.O * NL, o = p.O + k / NL, u = k % NL;
+                sthr[u * O32 + o] = (u == NL - 1) ? 1.0f : 0.0f;
+            }
+            if (p.res_codes != nullptr || p.res_f32 != nullptr) {       // level of y = #{u : y >= T_u}
+                if (p.ythr != nullptr) {
+                    if (et < NL - 1) syt[et] = mask_breakpoint(__ldg(p.ythr + et));
+                } else if (et == 0) {
+                    float t[8];
+                    channel_thresholds_f32(1.0f, 0.0f, p.qo, t);         // a long serial search: callers cache it
+                    for (int u = 0; u < NL - 1; ++u) syt[u] = mask_breakpoint(t[u]);
+                }
+            }
+            // sigma of a channel: the sign of its BN scale (+1 for 0); one warp per
+            // 32-channel word, a lane per channel (one load latency for the word)
+            for (int g = warp - 2; g < sig_words; g += EPI_WARPS) {
+                const int o = g * 32 + lane;
+                const float sg = o < p.O ? (p.thr != nullptr ? __ldg(p.thr + o * NL + NL - 1)
+                                                             : (__ldg(p.scale + o) < 0.0f ? -1.0f : 1.0f))
+                                         : 1.0f;
+                const uint32_t m = __ballot_sync(0xffffffffu, sg > 0.0f);
+                if (lane == 0) ssig[g] = m;
+            }
+        }
+        asm volatile("bar.sync 1, %0;\n" ::"n"(EPI_WARPS * 32) : "memory");   // breakpoints in place
         pdl_wait();                               // outputs, shortcuts and partial sums are shared with other kernels
         const int q = warp & 3;                   // TMEM lane quarter of this warp
         const int half_cols = (warp - 2) >> 2;    // which half of the accumulator columns
@@ -1973,6 +1987,7 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s) {
         attr[1].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
+        minw_host::max_shared_carveout(reinterpret_cast<const void *>(kern));
         // a persistent grid: no more clusters than can be resident at once
         const int maxc = tc::max_active_clusters(reinterpret_cast<const void *>(kern), pm.cl, pl.smem, cfg);
         if (maxc < 1) return MINW_EUNSUPPORTED;

@@ -15,6 +15,7 @@
 
 #include <atomic>
 #include <mutex>
+#include <unordered_set>
 
 #include "kernels.cuh"
 
@@ -55,6 +56,14 @@ bool pdl_enabled() { return plan_options().pdl != 0; }
 int take_stall(int which) {
     int expected = which;
     return g_stall.compare_exchange_strong(expected, 0) ? 1 : 0;
+}
+
+void max_shared_carveout(const void *kern) {
+    static std::mutex mu;
+    static std::unordered_set<const void *> done;
+    std::lock_guard<std::mutex> lock(mu);
+    if (done.insert(kern).second)
+        cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
 }
 
 }  // namespace minw_host
