@@ -144,14 +144,19 @@ MINW_API minw_status minw_pack_weights(const float *w, int32_t O, int32_t C, int
 
 enum {
     MINW_VARIANT_AUTO = 0,    /* per-shape choice from measurements: a network times each tensor-core
-                                 layer with E4M3 and with E2M1 operands at creation and keeps the
-                                 faster; the popcount path where the tensor cores do not apply */
+                                 layer with E4M3 operands, with E2M1 operands and with E2M1 operands
+                                 as CTA pairs of 128-channel tiles at creation and keeps the fastest;
+                                 the popcount path where the tensor cores do not apply */
     MINW_VARIANT_POPC = 1,    /* bit-serial XNOR/AND + popcount on the integer pipe */
     MINW_VARIANT_TC = 2,      /* tcgen05 tensor cores on exact level values: E2M1 operands where
                                  the shape allows (C % 128 == 0), else E4M3 */
     MINW_VARIANT_TC_E4M3 = 3, /* tensor cores on E4M3 operands only (a network request) */
-    MINW_VARIANT_TC_E2M1 = 4  /* tensor cores on E2M1 operands where the shape allows (a network
+    MINW_VARIANT_TC_E2M1 = 4, /* tensor cores on E2M1 operands where the shape allows (a network
                                  request, as MINW_VARIANT_TC); reported for a layer on E2M1 operands */
+    MINW_VARIANT_TC_E2M1_PAIRS = 5  /* E2M1 operands as CTA pairs of 256 pixels x 128 channels where the
+                                 shape allows (output channels a multiple of 128, no K split): two
+                                 accumulators per CTA, so each tile's epilogue overlaps the next
+                                 tile's MMAs (a network request; reported for such a layer) */
 };
 
 /* Convolution of packed activations act [B][H][W][bits_a][C/32] with packed
@@ -498,7 +503,7 @@ MINW_API minw_status minw_net_layer_times(minw_net *net, float *ms);
 
 /* Kernel chosen for each layer (host array of minw_net_launches() ints):
  * 0 for the fp32 first layer, else MINW_VARIANT_POPC, MINW_VARIANT_TC (E4M3
- * operands) or MINW_VARIANT_TC_E2M1. */
+ * operands), MINW_VARIANT_TC_E2M1 or MINW_VARIANT_TC_E2M1_PAIRS. */
 MINW_API minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants);
 
 /* ResNet-18-shaped MINW-Net (Table V's network).  The paper leaves the

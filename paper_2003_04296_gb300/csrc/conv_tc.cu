@@ -331,6 +331,31 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
 }
 
+// 32 columns of this warp's 32 TMEM lanes, without waiting: tmem_wait_ld()
+// before the first use of v (it waits for every load this thread issued).
+__device__ __forceinline__ void tmem_ld32_nw(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
+        "%14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];\n"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
+          "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
+          "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
+
+// Sign bits of 32 values as one word (bit j = sign of x[j]), built as four
+// independent 8-bit chains so that the funnel shifts overlap.
+__device__ __forceinline__ uint32_t sign_word(const float (&x)[32]) {
+    uint32_t w[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int j = 7; j >= 0; --j)
+#pragma unroll
+        for (int k = 0; k < 4; ++k) w[k] = __funnelshift_l(__float_as_uint(x[8 * k + j]), w[k], 1);
+    return w[0] | (w[1] << 8) | (w[2] << 16) | (w[3] << 24);
+}
+
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
@@ -390,25 +415,27 @@ __device__ __forceinline__ uint32_t transpose32(uint32_t a, int lane) {
 // planes and E4M3 codes follow from the masks with bitwise logic.  th: the
 // chunk's first channel in rows of tstride floats (-T_1 .. -T_{n-1}, sigma).
 template <int OUTB>
-__device__ __forceinline__ void mask_chunk(uint32_t taddr, bool full32, const float *th, int tstride, uint32_t sig,
-                                           int pool, int bw, bool writer, int nvalid, uint32_t *planes, int NWo,
-                                           uint8_t *codes, bool codes4) {
+__device__ __forceinline__ void mask_chunk_regs(const uint32_t (&v)[32], bool full32, const float *th, int tstride,
+                                                uint32_t sig, int pool, int bw, bool writer, int nvalid,
+                                                uint32_t *planes, int NWo, uint8_t *codes, bool codes4) {
     constexpr int NL = OUTB == 1 ? 2 : (OUTB == 2 ? 3 : 7);
-    uint32_t v[32];
-    if (full32) {
-        tmem_ld32(taddr, v);
-    } else {
-        uint32_t v16[16];
-        tmem_ld16(taddr, v16);
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            v[j] = v16[j];
-            v[j + 16] = 0u;
-        }
-    }
     uint32_t M[NL - 1];
 #pragma unroll
     for (int u = 0; u < NL - 1; ++u) M[u] = 0u;
+    if constexpr (NL == 2) {
+        // one breakpoint: the 32 sign bits as four independent chains
+        float d[32];
+#pragma unroll
+        for (int j4 = 0; j4 < 8; ++j4) {
+            const float4 sg4 = *reinterpret_cast<const float4 *>(th + tstride + 4 * j4);
+            const float4 nt4 = *reinterpret_cast<const float4 *>(th + 4 * j4);
+            d[4 * j4] = fmaf(__uint_as_float(v[4 * j4]), sg4.x, nt4.x);
+            d[4 * j4 + 1] = fmaf(__uint_as_float(v[4 * j4 + 1]), sg4.y, nt4.y);
+            d[4 * j4 + 2] = fmaf(__uint_as_float(v[4 * j4 + 2]), sg4.z, nt4.z);
+            d[4 * j4 + 3] = fmaf(__uint_as_float(v[4 * j4 + 3]), sg4.w, nt4.w);
+        }
+        M[0] = sign_word(d);
+    } else
     // breakpoints of four channels per 128-bit load (rows of tstride floats, channel fastest)
 #pragma unroll
     for (int j4 = 7; j4 >= 0; --j4) {
@@ -440,6 +467,25 @@ __device__ __forceinline__ void mask_chunk(uint32_t taddr, bool full32, const fl
     }
     if (!writer) return;
     store_level_masks<OUTB>(M, nvalid, full32 ? 32 : 16, planes, NWo, codes, codes4);
+}
+
+template <int OUTB>
+__device__ __forceinline__ void mask_chunk(uint32_t taddr, bool full32, const float *th, int tstride, uint32_t sig,
+                                           int pool, int bw, bool writer, int nvalid, uint32_t *planes, int NWo,
+                                           uint8_t *codes, bool codes4) {
+    uint32_t v[32];
+    if (full32) {
+        tmem_ld32(taddr, v);
+    } else {
+        uint32_t v16[16];
+        tmem_ld16(taddr, v16);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            v[j] = v16[j];
+            v[j + 16] = 0u;
+        }
+    }
+    mask_chunk_regs<OUTB>(v, full32, th, tstride, sig, pool, bw, writer, nvalid, planes, NWo, codes, codes4);
 }
 
 // Epilogue of one 32-column chunk (16 when full32 is false) of a residual
@@ -1008,6 +1054,15 @@ __global__ void __launch_bounds__(NT, 1)
                 // columns [64 (2 (q >> 1) + half), + 64)
                 const int oq = 32 * (p.dup ? (q & 1) : q);
                 const int cq = p.dup ? 2 : 4, cb = p.dup ? 2 * (2 * (q >> 1) + half_cols) : 4 * half_cols;
+                // this lane's pixel of each of the warp's chunks, relative to the tile (tiles-invariant)
+                int crb[4], cry[4], crx[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int r = (cb + k) * 32 + lane;
+                    crb[k] = r / (p.bh * p.bw);
+                    cry[k] = (r / p.bw) % p.bh;
+                    crx[k] = r % p.bw;
+                }
                 for (int n = 0, w; (w = cta_item(p, n, items, tiles_m, crank)) >= 0; ++n, ++i) {
                     const int ab = p.nacc == 2 ? (i & 1) : 0, use = p.nacc == 2 ? (i >> 1) : i;
                     const int tn = w / tiles_m, tm = w - tn * tiles_m;
@@ -1034,7 +1089,62 @@ __global__ void __launch_bounds__(NT, 1)
                         sc = __ldg(p.scale + oc);
                         sh = __ldg(p.shift + oc);
                     }
-                    for (int c = cb; c < cb + cq && !dead && qlive; ++c) {
+                    // plain block epilogue of 1- and 2-bit outputs: two chunks at a time, their loads,
+                    // sign chains, transposes, pooling and stores interleaved (a 3-bit output's six
+                    // mask chains per chunk already overlap)
+#pragma unroll
+                    for (int k = 0; k < 4; k += 2) {
+                        if (NL > 3 || k >= cq || dead || !qlive || tres) break;
+                        __syncwarp();
+                        uint32_t v0[32], v1[32];
+                        const uint32_t ta = tmem_base + ((uint32_t)oq << 16) + (uint32_t)(ab * p.acc_cols + (cb + k) * 32);
+                        tmem_ld32_nw(ta, v0);
+                        tmem_ld32_nw(ta + 32u, v1);
+                        tmem_wait_ld();
+                        uint32_t M0[NL - 1], M1[NL - 1];
+#pragma unroll
+                        for (int u = 0; u < NL - 1; ++u) {
+                            float d0[32], d1[32];      // sigma * acc - T_u: sign bit j = [sigma * acc < T_u] at column j
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) {
+                                d0[j] = fmaf(__uint_as_float(v0[j]), sg, nt[u]);
+                                d1[j] = fmaf(__uint_as_float(v1[j]), sg, nt[u]);
+                            }
+                            M0[u] = transpose32(sign_word(d0), lane);   // lane j: bit k = channel oq + k at column j
+                            M1[u] = transpose32(sign_word(d1), lane);
+                        }
+                        if (p.pool) {
+#pragma unroll
+                            for (int u = 0; u < NL - 1; ++u) {
+                                const uint32_t m0 = M0[u], m1 = M1[u];
+                                const uint32_t n0 = __shfl_xor_sync(0xffffffffu, m0, 1), n1 = __shfl_xor_sync(0xffffffffu, m1, 1);
+                                const uint32_t a0 = m0 & n0, o0 = m0 | n0, a1 = m1 & n1, o1 = m1 | n1;
+                                const uint32_t a0b = a0 & __shfl_xor_sync(0xffffffffu, a0, p.bw);
+                                const uint32_t a1b = a1 & __shfl_xor_sync(0xffffffffu, a1, p.bw);
+                                const uint32_t o0b = o0 | __shfl_xor_sync(0xffffffffu, o0, p.bw);
+                                const uint32_t o1b = o1 | __shfl_xor_sync(0xffffffffu, o1, p.bw);
+                                M0[u] = (sig & a0b) | (~sig & o0b);
+                                M1[u] = (sig & a1b) | (~sig & o1b);
+                            }
+                        }
+#pragma unroll
+                        for (int h2 = 0; h2 < 2; ++h2) {
+                            const int b = bbk * p.bb + crb[k + h2];
+                            const int y = yb * p.bh + cry[k + h2];
+                            const int x = xb * p.bw + crx[k + h2];
+                            const bool valid = b < p.B && y < p.Ho && x < p.Wo;
+                            if (valid && (!p.pool || ((x & 1) == 0 && (y & 1) == 0))) {
+                                const int yp = p.pool ? y / 2 : y, xp = p.pool ? x / 2 : x;
+                                const long long opix = ((long long)b * Hp + yp) * Wp + xp;
+                                const int ob = tn * p.BN + oq;
+                                store_level_masks<OUTB>(h2 ? M1 : M0, 32, 32,
+                                                        p.planes_out ? p.planes_out + (opix * OUTB) * NWo + (ob >> 5) : nullptr,
+                                                        NWo, p.codes_out ? p.codes_out + ((opix * p.O + ob) >> p.out4) : nullptr,
+                                                        p.out4 != 0);
+                            }
+                        }
+                    }
+                    for (int c = cb; c < cb + cq && !dead && qlive && (tres || NL > 3); ++c) {
                         __syncwarp();
                         uint32_t v[32];
                         tmem_ld32(tmem_base + ((uint32_t)oq << 16) + (uint32_t)(ab * p.acc_cols + c * 32), v);
@@ -1695,6 +1805,13 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, bool encode = true) {
         const int ks_ = (a.workspace != nullptr && !a.pool && !a.upd) ? (a.ksplit > 0 ? a.ksplit : auto_ksplit(tiles_, p.nk, sms_))
                                                             : 1;
         p.pair = (pair_pref() && !p.trans && p.BN == 256 && a.O % 256 == 0 && p.nk >= 18 && ks_ <= 1) ? 1 : 0;
+        // E2M1 pairs of 128-channel tiles: each CTA accumulates 128 pixels x 128 channels, so two
+        // accumulators fit beside the scale factors (a 256-channel E2M1 tile has one)
+        if (a.pair_n128 && p.fp4 && !p.trans && a.O % 128 == 0 && ks_ <= 1 && !a.upd) {
+            p.BN = 128;
+            p.ntn = (a.O + 127) / 128;
+            p.pair = 1;
+        }
     }
     p.b_bytes = (uint32_t)((p.pair ? p.BN / 2 : p.BN) * p.cb);   // pairs: each CTA holds half the weight rows
     const size_t o32 = ((size_t)a.O + 31) & ~(size_t)31;
@@ -1911,6 +2028,12 @@ int conv_tc_ksplit(const ConvArgs &a) {
     if (!conv_tc_supported(a)) return 0;
     tc::Plan pl;
     return tc::make_plan(a, pl, false) == MINW_OK ? pl.p.ksplit : 0;
+}
+
+bool conv_tc_pairs128(const ConvArgs &a) {
+    if (!conv_tc_supported(a)) return false;
+    tc::Plan pl;
+    return tc::make_plan(a, pl, false) == MINW_OK && pl.p.pair && pl.p.BN == 128;
 }
 
 int conv_tc_launches(const ConvArgs &a) {

@@ -46,6 +46,8 @@ struct ConvArgs {
     void *workspace;       // nullable: no split
     size_t workspace_bytes;
     int ksplit;            // 0: chosen from the shape
+    int pair_n128;         // E2M1: CTA pairs of 256 pixels x 128 channels (two accumulators fit the tensor
+                           // memory beside the scale factors, so the epilogue overlaps the next MMAs)
 };
 
 // First-layer convolution on the fp32 image (see conv_first.cu).
@@ -103,6 +105,8 @@ size_t conv_tc_workspace_bytes(const ConvArgs &a);
 size_t conv_tc_min_split_bytes(const ConvArgs &a);
 // K slices of the tensor-core plan for this shape and workspace (1: no split; 0: not supported).
 int conv_tc_ksplit(const ConvArgs &a);
+// Whether the plan of this shape runs as CTA pairs of 128-channel E2M1 tiles (a.pair_n128 honoured).
+bool conv_tc_pairs128(const ConvArgs &a);
 // Kernels one tensor-core launch issues for this shape and workspace (2 with a split).
 int conv_tc_launches(const ConvArgs &a);
 minw_status launch_thresholds(const float *scale, const float *shift, int O, const QParams &q, float *out,

@@ -57,13 +57,14 @@ static minw_status time_conv_tc(const ConvArgs &a, cudaStream_t s, cudaEvent_t e
     return MINW_OK;
 }
 
-// The measured choice between E4M3 and E2M1 operands for every tensor-core
-// layer whose channels allow both (north of the pipe rates, the layer's
-// tiling, accumulator count and epilogue decide which runs faster: on GB300
-// E2M1 wins on most layers but not on all).  Each candidate runs on the
-// layer's shape at the net's batch with its own weight codes, breakpoints
-// and split workspace, into scratch buffers; the faster is kept (P.in4) and
-// the shared workspace is sized for the choices.
+// The measured choice of operands and tiling for every tensor-core layer whose
+// channels allow E2M1: E4M3 operands, E2M1 operands, or E2M1 as CTA pairs of
+// 128-channel tiles (pipe rates alone do not decide: the layer's tiling, its
+// accumulator count and its epilogue do; on GB300 E2M1 wins on most layers
+// but not on all).  Each candidate runs on the layer's shape at the net's
+// batch with its own weight codes, breakpoints and split workspace, into
+// scratch buffers; the fastest is kept (P.in4, P.pair128) and the shared
+// workspace is sized for the choices.
 static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int n_layers, int max_batch,
                                 cudaStream_t s) {
     size_t in_b = 0, out_b = 0, w_b = 0, ws_b = 0;
@@ -114,15 +115,18 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
             } else {
                 a.y_out = (float *)yout;
             }
-            float t[2] = {0.0f, 0.0f};
-            for (int f = 0; f < 2 && st == MINW_OK; ++f) {
+            // candidates: E4M3 operands, E2M1 operands, E2M1 as CTA pairs of 128-channel tiles
+            float t[3] = {0.0f, 0.0f, 0.0f};
+            for (int f = 0; f < 3 && st == MINW_OK; ++f) {
                 ConvArgs b = a;
-                b.fp4 = f;
+                b.fp4 = f ? 1 : 0;
+                b.pair_n128 = f == 2 ? 1 : 0;
                 b.codes_out4 = f && !last;
-                if (!conv_tc_supported(b)) { t[f] = 1e30f; continue; }
+                if (!conv_tc_supported(b) || (f == 2 && !conv_tc_pairs128(b))) { t[f] = 1e30f; continue; }
                 void *wq = f ? w4 : w8;
-                st = f ? minw_pack_weight_codes_e2m1(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, (uint8_t *)wq, s)
-                       : minw_pack_weight_codes(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, (uint8_t *)wq, s);
+                if (f < 2)
+                    st = f ? minw_pack_weight_codes_e2m1(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, (uint8_t *)wq, s)
+                           : minw_pack_weight_codes(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, (uint8_t *)wq, s);
                 if (st != MINW_OK) break;
                 b.act8 = (const uint8_t *)xin;
                 b.wgt8 = (const uint8_t *)wq;
@@ -138,7 +142,9 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
                 st = time_conv_tc(b, s, e0, e1, &t[f]);
             }
             if (st != MINW_OK) break;
-            P.in4 = t[1] < t[0] ? 1 : 0;
+            const int best = (t[1] < t[0]) ? (t[2] < t[1] ? 2 : 1) : (t[2] < t[0] ? 2 : 0);
+            P.in4 = best > 0 ? 1 : 0;
+            P.pair128 = best == 2 ? 1 : 0;
         }
     } while (false);
     cudaStreamSynchronize(s);
@@ -156,6 +162,7 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
         a.stride = P.stride; a.pad = P.pad; a.Ho = P.Ho; a.Wo = P.Wo; a.NW = P.C / 32;
         a.M = (long long)max_batch * P.Ho * P.Wo; a.pool = P.pool; a.quant_out = l + 1 < n_layers;
         a.fp4 = P.in4;
+        a.pair_n128 = P.pair128;
         n->ws_bytes = std::max(n->ws_bytes, conv_tc_workspace_bytes(a));
     }
     return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
@@ -166,7 +173,7 @@ extern "C" {
 minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int32_t max_batch,
                             int32_t variant, void *stream, minw_net **out) {
     if (!layers || n_layers < 2 || max_batch <= 0 || !out) return MINW_EINVAL;
-    if (variant < 0 || variant > 4) return MINW_EINVAL;
+    if (variant < 0 || variant > MINW_VARIANT_TC_E2M1_PAIRS) return MINW_EINVAL;
     *out = nullptr;
     cudaStream_t s = (cudaStream_t)stream;
     minw_net *n = new minw_net();
@@ -259,6 +266,11 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
                 a.fp4 = 1;
                 P.in4 = conv_tc_supported(a) ? 1 : 0;
                 a.fp4 = P.in4;
+                if (variant == MINW_VARIANT_TC_E2M1_PAIRS && P.in4) {
+                    a.pair_n128 = 1;
+                    P.pair128 = conv_tc_pairs128(a) ? 1 : 0;
+                    a.pair_n128 = P.pair128;
+                }
             }
             if (P.variant == MINW_VARIANT_TC) {
                 const size_t wb = conv_tc_workspace_bytes(a);
@@ -379,6 +391,7 @@ static minw_status forward_enqueue(minw_net *net, const float *x, int32_t B, flo
             a.codes_out4 = out_codes && net->L[l + 1].in4;
             a.y_out = last ? logits : nullptr;
             a.fp4 = P.in4;
+            a.pair_n128 = P.pair128;
             if (P.in_codes) {
                 a.act8 = (const uint8_t *)src;
                 a.wgt8 = P.wcodes;
@@ -482,7 +495,9 @@ minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants) {
         return MINW_OK;
     }
     for (size_t l = 0; l < net->L.size(); ++l)
-        variants[l] = l == 0 ? 0 : net->L[l].in4 ? MINW_VARIANT_TC_E2M1 : net->L[l].variant;
+        variants[l] = l == 0 ? 0
+                      : net->L[l].pair128 ? MINW_VARIANT_TC_E2M1_PAIRS
+                      : net->L[l].in4 ? MINW_VARIANT_TC_E2M1 : net->L[l].variant;
     return MINW_OK;
 }
 

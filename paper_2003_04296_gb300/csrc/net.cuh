@@ -19,6 +19,7 @@ struct LayerPlan {
                                    // tensor-core layers: integer-valued [O][levels])
     int in_codes = 0;              // input arrives in the codes layout
     int in4 = 0;                   // ... as E2M1 codes (two channels per byte; weights too)
+    int pair128 = 0;               // E2M1 tensor-core layer as CTA pairs of 128-channel tiles (measured choice)
     float *wlatent = nullptr;      // fp32 weights (first layer)
     float *wt = nullptr;           // first layer: weights prepared as [K][O] levels
     float *wscale = nullptr;       // per-channel weight prescale (first layer)

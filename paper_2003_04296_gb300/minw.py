@@ -16,7 +16,7 @@ from . import build as _build
 _LIB = None
 
 MINW_OK, MINW_EINVAL, MINW_EUNSUPPORTED, MINW_ECUDA, MINW_ETIMEOUT, MINW_EDEVICE = range(6)
-VARIANT_AUTO, VARIANT_POPC, VARIANT_TC, VARIANT_TC_E4M3, VARIANT_TC_E2M1 = 0, 1, 2, 3, 4
+VARIANT_AUTO, VARIANT_POPC, VARIANT_TC, VARIANT_TC_E4M3, VARIANT_TC_E2M1, VARIANT_TC_E2M1_PAIRS = 0, 1, 2, 3, 4, 5
 CODES_E4M3, CODES_E2M1 = 0, 1
 LAYER_CONV, LAYER_FC = 0, 1
 
