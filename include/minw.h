@@ -143,10 +143,12 @@ MINW_API minw_status minw_pack_weights(const float *w, int32_t O, int32_t C, int
 /* ---------------------------------------------------------------------- */
 
 enum {
-    MINW_VARIANT_AUTO = 0,    /* per-shape choice from measurements: a network times each tensor-core
-                                 layer with E4M3 operands, with E2M1 operands and with E2M1 operands
-                                 as CTA pairs of 128-channel tiles at creation and keeps the fastest;
-                                 the popcount path where the tensor cores do not apply */
+    MINW_VARIANT_AUTO = 0,    /* per-shape choice from measurements: at creation a network times each
+                                 layer the tensor cores cover with E4M3 operands, with E2M1 operands,
+                                 with E2M1 operands as CTA pairs of 128-channel tiles and on the
+                                 popcount path (bit-planes), and keeps the fastest (the times stay
+                                 readable through minw_net_layer_candidates); the popcount path
+                                 where the tensor cores do not apply */
     MINW_VARIANT_POPC = 1,    /* bit-serial XNOR/AND + popcount on the integer pipe */
     MINW_VARIANT_TC = 2,      /* tcgen05 tensor cores on exact level values: E2M1 operands where
                                  the shape allows (C % 128 == 0), else E4M3 */
@@ -343,6 +345,46 @@ MINW_API minw_status minw_fc_train_step(const float *A, float *W, const float *g
                                         const minw_quant *q_a, float *a_out, float *g_in, float *a_pre,
                                         void *workspace, size_t workspace_bytes, void *stream);
 
+/* Bytes of device workspace minw_conv_train_step needs for this shape (0
+ * for bad or unsupported sizes). */
+MINW_API size_t minw_conv_train_workspace_bytes(int32_t B, int32_t C, int32_t H, int32_t W, int32_t O, int32_t kh,
+                                                int32_t kw, int32_t stride, int32_t pad);
+
+/* One step of Algorithm 1 for a convolutional layer (the training branch
+ * treats convolutional and fully connected layers alike) with input A
+ * [B][C][H][W] (fp32 NCHW, the previous layer's AQE output or the network
+ * input), latent weights W [O][C][kh][kw] (fp32, updated in place) and the
+ * upstream gradient g_out [B][O][Ho][Wo] = dL/d(a_out), zero padding pad and
+ * stride stride:
+ *   W^ = fmaf(alpha, h_w(W), (1 - alpha) W)             (Eq. weight, q_w)
+ *   a~ = conv(bf16(A), bf16(W^))                         (tensor cores, fp32 sums)
+ *   a_out = fmaf(alpha, h_a(a~), (1 - alpha) a~)         (Eq. activation, q_a; a_out = a~ when q_a is null)
+ *   g_a~ = 2 alpha g_out 1[|a~| <= 1]                    (Eq. activation; g_out itself when q_a is null)
+ *   g_in = conv^T(bf16(g_a~), bf16(W^))                  ([B][C][H][W], skipped when g_in is null)
+ *   g_W^ = sum over b, y, x of bf16(g_a~) x bf16(A patch) ([O][C][kh][kw])
+ *   W = min(1, max(-1, W - lr 2 alpha g_W^ 1[|W| <= 1]))  (Eq. weight, update and clip)
+ * a_pre (nullable, [B][O][Ho][Wo]) receives a~ when q_a is set (ignored
+ * without q_a).  The three products take bf16 roundings of their fp32
+ * operands (the paper's operands are fp32: this is a precision departure
+ * with the per-product error bound of minw_fc_train_step), and the weight
+ * gradient's reduction over the pixels is split across the SMs and summed
+ * slice by slice in a fixed order (the same bits on every call).
+ * Requirements: C % 64 == 0, B Ho Wo % 64 == 0, stride 1 or 2, pad < kh and
+ * pad < kw (else MINW_EUNSUPPORTED); alpha in [0, 1]; 16-byte aligned
+ * pointers; workspace of minw_conv_train_workspace_bytes (scratch: nothing
+ * in it survives the call).  All buffers are caller-owned device memory; the
+ * call is asynchronous on stream and launches eight to eleven kernels (and a
+ * memset of the input gradient's spread image for stride 2 or O % 64 != 0).
+ * MINW_EINVAL: null A, W, g_out, a_out, q_w or workspace, an invalid
+ * quantizer, alpha outside [0, 1], a misaligned pointer or a short workspace;
+ * MINW_EUNSUPPORTED: the shapes above, or sizes past the kernels' index and
+ * grid limits. */
+MINW_API minw_status minw_conv_train_step(const float *A, float *W, const float *g_out, int32_t B, int32_t C,
+                                          int32_t H, int32_t Wd, int32_t O, int32_t kh, int32_t kw, int32_t stride,
+                                          int32_t pad, float alpha, float lr, const minw_quant *q_w,
+                                          const minw_quant *q_a, float *a_out, float *g_in, float *a_pre,
+                                          void *workspace, size_t workspace_bytes, void *stream);
+
 /* Extra inputs and outputs of a residual block (ResNet-style MINW-Net,
  * where the paper leaves the block wiring open).  Host struct.
  * res_codes (nullable): shortcut as level codes [B][Hp][Wp][O] of bit width
@@ -356,6 +398,11 @@ MINW_API minw_status minw_fc_train_step(const float *A, float *W, const float *g
  * out_format, res_format: layouts of codes_out and res_codes.
  * acc_out (nullable, output): the exact int32 accumulators, NCHW, for a block
  *   without pooling.
+ * e2m1_pairs: with E2M1 operands, run CTA pairs of 256 pixels x 128 channels
+ *   (two accumulators per CTA, so each tile's epilogue overlaps the next
+ *   tile's MMAs) where the shape allows it (O % 128 == 0); elsewhere, and for
+ *   E4M3 operands, the default tiling.  The results are the same integers
+ *   either way; only the speed differs, which is why callers measure both.
  * A zero-initialised struct is the E4M3 block without extras. */
 typedef struct {
     const uint8_t *res_codes;
@@ -366,6 +413,7 @@ typedef struct {
     int32_t out_format;
     int32_t res_format;
     int32_t *acc_out;
+    int32_t e2m1_pairs;
 } minw_block_extra;
 
 /* minw_conv_block_codes with the residual inputs / outputs of extra
@@ -505,6 +553,19 @@ MINW_API minw_status minw_net_layer_times(minw_net *net, float *ms);
  * 0 for the fp32 first layer, else MINW_VARIANT_POPC, MINW_VARIANT_TC (E4M3
  * operands), MINW_VARIANT_TC_E2M1 or MINW_VARIANT_TC_E2M1_PAIRS. */
 MINW_API minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants);
+
+/* The creation-time measurement behind layer `layer`'s kernel choice under
+ * MINW_VARIANT_AUTO (runtime introspection; the paper has no counterpart):
+ * ms (host array of 4 floats) receives the least of three timed launches of
+ * each candidate at the net's max_batch, in milliseconds, in the order E4M3
+ * operands, E2M1 operands, E2M1 CTA pairs of 128-channel tiles, popcount on
+ * bit-planes; -1 for a candidate the layer's shape does not allow, and -1 in
+ * every entry for the first layer and for nets not created with
+ * MINW_VARIANT_AUTO.  The kernel minw_net_layer_variants reports is the
+ * fastest entry.  MINW_EINVAL for a null argument or a layer out of range,
+ * MINW_EUNSUPPORTED for a residual network (its formats follow a fixed
+ * rule). */
+MINW_API minw_status minw_net_layer_candidates(const minw_net *net, int32_t layer, float *ms);
 
 /* ResNet-18-shaped MINW-Net (Table V's network).  The paper leaves the
  * residual wiring open; the reading implemented here:

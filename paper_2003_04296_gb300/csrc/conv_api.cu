@@ -245,6 +245,7 @@ minw_status minw_conv_block_codes_ex(const uint8_t *act, int32_t B, int32_t C, i
         a.codes_out4 = extra->out_format == MINW_CODES_E2M1;
         a.res_codes4 = extra->res_format == MINW_CODES_E2M1;
         a.acc_out = extra->acc_out;
+        a.pair_n128 = (extra->e2m1_pairs != 0 && a.fp4) ? 1 : 0;
     }
     return launch_conv_tc(a, (cudaStream_t)stream);
 }

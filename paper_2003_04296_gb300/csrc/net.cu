@@ -40,14 +40,16 @@ static minw_status net_alloc(minw_net *n, T **p, size_t count) {
     return MINW_OK;
 }
 
-// Time one tensor-core launch: one warm-up, then the least of three runs (ms).
-static minw_status time_conv_tc(const ConvArgs &a, cudaStream_t s, cudaEvent_t e0, cudaEvent_t e1, float *ms) {
-    minw_status st = launch_conv_tc(a, s);
+// Time one convolution launch on either path: one warm-up, then the least of
+// three runs (ms).
+static minw_status time_conv(const ConvArgs &a, bool popc, cudaStream_t s, cudaEvent_t e0, cudaEvent_t e1,
+                             float *ms) {
+    minw_status st = popc ? launch_conv_popc(a, s) : launch_conv_tc(a, s);
     if (st != MINW_OK) return st;
     float best = 1e30f;
     for (int r = 0; r < 3; ++r) {
         if (cudaEventRecord(e0, s) != cudaSuccess) return MINW_ECUDA;
-        if ((st = launch_conv_tc(a, s)) != MINW_OK) return st;
+        if ((st = popc ? launch_conv_popc(a, s) : launch_conv_tc(a, s)) != MINW_OK) return st;
         if (cudaEventRecord(e1, s) != cudaSuccess || cudaEventSynchronize(e1) != cudaSuccess) return MINW_ECUDA;
         float t = 0.0f;
         cudaEventElapsedTime(&t, e0, e1);
@@ -57,24 +59,27 @@ static minw_status time_conv_tc(const ConvArgs &a, cudaStream_t s, cudaEvent_t e
     return MINW_OK;
 }
 
-// The measured choice of operands and tiling for every tensor-core layer whose
-// channels allow E2M1: E4M3 operands, E2M1 operands, or E2M1 as CTA pairs of
-// 128-channel tiles (pipe rates alone do not decide: the layer's tiling, its
-// accumulator count and its epilogue do; on GB300 E2M1 wins on most layers
-// but not on all).  Each candidate runs on the layer's shape at the net's
-// batch with its own weight codes, breakpoints and split workspace, into
-// scratch buffers; the fastest is kept (P.in4, P.pair128) and the shared
-// workspace is sized for the choices.
+// The measured choice of kernel, operands and tiling for every layer the
+// tensor cores cover: E4M3 operands, E2M1 operands, E2M1 as CTA pairs of
+// 128-channel tiles, or bit-planes on the popcount path (pipe rates alone do
+// not decide: the layer's tiling, its accumulator count and its epilogue do;
+// on GB300 E2M1 wins on most layers but not on all).  Each candidate runs on
+// the layer's shape at the net's batch with its own weight codes or planes,
+// breakpoints and split workspace, into scratch buffers; the fastest is kept
+// (P.variant, P.in4, P.pair128), every candidate's time is kept in P.cand_ms,
+// and the shared workspace is sized for the choices.
 static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int n_layers, int max_batch,
                                 cudaStream_t s) {
     size_t in_b = 0, out_b = 0, w_b = 0, ws_b = 0;
     std::vector<int> cand;
     for (int l = 1; l < n_layers; ++l) {
         const LayerPlan &P = n->L[l];
-        if (P.variant != MINW_VARIANT_TC || P.C % 128 != 0) continue;
+        if (P.variant != MINW_VARIANT_TC) continue;
         cand.push_back(l);
+        // codes (one byte per channel at most) or bit-planes (3 bits per channel at most) in;
+        // codes, planes or fp32 logits out
         in_b = std::max(in_b, (size_t)max_batch * P.H * P.W * P.C);
-        out_b = std::max(out_b, (size_t)max_batch * P.Hp * P.Wp * P.O * sizeof(float));   // codes or fp32 logits
+        out_b = std::max(out_b, (size_t)max_batch * P.Hp * P.Wp * P.O * sizeof(float));
         w_b = std::max(w_b, (size_t)P.O * P.kh * P.kw * P.C);
     }
     if (cand.empty()) return MINW_OK;
@@ -87,11 +92,12 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
     cudaEvent_t e0 = nullptr, e1 = nullptr;
     minw_status st = MINW_OK;
     void *xin = nullptr, *yout = nullptr, *w8 = nullptr, *w4 = nullptr, *thr = nullptr, *ws = nullptr;
+    void *wpl = nullptr;
     do {
         if (cudaEventCreate(&e0) != cudaSuccess || cudaEventCreate(&e1) != cudaSuccess) { st = MINW_ECUDA; break; }
         if ((st = talloc(in_b, &xin)) != MINW_OK || (st = talloc(out_b, &yout)) != MINW_OK ||
             (st = talloc(w_b, &w8)) != MINW_OK || (st = talloc(w_b, &w4)) != MINW_OK ||
-            (st = talloc(4096 * 8 * sizeof(float), &thr)) != MINW_OK)
+            (st = talloc(w_b, &wpl)) != MINW_OK || (st = talloc(4096 * 8 * sizeof(float), &thr)) != MINW_OK)
             break;
         // +1 levels in both formats (E4M3 0x38; E2M1 0x2 in each nibble)
         if (cudaMemsetAsync(xin, 0x22, in_b, s) != cudaSuccess) { st = MINW_ECUDA; break; }
@@ -115,9 +121,24 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
             } else {
                 a.y_out = (float *)yout;
             }
-            // candidates: E4M3 operands, E2M1 operands, E2M1 as CTA pairs of 128-channel tiles
-            float t[3] = {0.0f, 0.0f, 0.0f};
-            for (int f = 0; f < 3 && st == MINW_OK; ++f) {
+            // candidates: E4M3 operands, E2M1 operands, E2M1 as CTA pairs of 128-channel tiles,
+            // bit-planes on the popcount path (its input: the same bytes read as planes; its
+            // output: planes, or the fp32 logits of the last layer)
+            float t[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            for (int f = 0; f < 4 && st == MINW_OK; ++f) {
+                if (f == 3) {
+                    ConvArgs b = a;
+                    b.thr = nullptr;
+                    b.codes_out = nullptr;
+                    if (!last) b.planes_out = (uint32_t *)yout;
+                    if ((st = minw_pack_weights(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, (uint32_t *)wpl, s)) !=
+                        MINW_OK)
+                        break;
+                    b.act = (const uint32_t *)xin;
+                    b.wgt = (const uint32_t *)wpl;
+                    st = time_conv(b, true, s, e0, e1, &t[f]);
+                    continue;
+                }
                 ConvArgs b = a;
                 b.fp4 = f ? 1 : 0;
                 b.pair_n128 = f == 2 ? 1 : 0;
@@ -139,11 +160,15 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
                 }
                 b.workspace = ws;
                 b.workspace_bytes = ws_b;
-                st = time_conv_tc(b, s, e0, e1, &t[f]);
+                st = time_conv(b, false, s, e0, e1, &t[f]);
             }
             if (st != MINW_OK) break;
-            const int best = (t[1] < t[0]) ? (t[2] < t[1] ? 2 : 1) : (t[2] < t[0] ? 2 : 0);
-            P.in4 = best > 0 ? 1 : 0;
+            int best = 0;
+            for (int f = 1; f < 4; ++f)
+                if (t[f] < t[best]) best = f;
+            for (int f = 0; f < 4; ++f) P.cand_ms[f] = t[f] < 1e29f ? t[f] : -1.0f;
+            P.variant = best == 3 ? MINW_VARIANT_POPC : MINW_VARIANT_TC;
+            P.in4 = (best == 1 || best == 2) ? 1 : 0;
             P.pair128 = best == 2 ? 1 : 0;
         }
     } while (false);
@@ -485,6 +510,14 @@ minw_status minw_net_layer_times(minw_net *net, float *ms) {
     if (cudaEventSynchronize(net->events.back()) != cudaSuccess) return MINW_ECUDA;
     for (size_t l = 0; l + 1 < net->events.size(); ++l)
         if (cudaEventElapsedTime(&ms[l], net->events[l], net->events[l + 1]) != cudaSuccess) return MINW_ECUDA;
+    return MINW_OK;
+}
+
+minw_status minw_net_layer_candidates(const minw_net *net, int32_t layer, float *ms) {
+    if (!net || !ms) return MINW_EINVAL;
+    if (net->kind == 1) return MINW_EUNSUPPORTED;
+    if (layer < 0 || layer >= (int32_t)net->L.size()) return MINW_EINVAL;
+    for (int f = 0; f < 4; ++f) ms[f] = net->L[layer].cand_ms[f];
     return MINW_OK;
 }
 

@@ -34,7 +34,7 @@ class Quant(ctypes.Structure):
 class BlockExtra(ctypes.Structure):
     _fields_ = [("res_codes", ctypes.c_void_p), ("res_bits", ctypes.c_int32), ("res_f32", ctypes.c_void_p),
                 ("y_nhwc", ctypes.c_void_p), ("in_format", ctypes.c_int32), ("out_format", ctypes.c_int32),
-                ("res_format", ctypes.c_int32), ("acc_out", ctypes.c_void_p)]
+                ("res_format", ctypes.c_int32), ("acc_out", ctypes.c_void_p), ("e2m1_pairs", ctypes.c_int32)]
 
 
 class PlanOptions(ctypes.Structure):
@@ -93,6 +93,9 @@ SIGNATURES = {
     "minw_bf16_matrix": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _P]),
     "minw_sgd_clip": (ctypes.c_int, [_P, _P, _I64, _F, _P]),
     "minw_fc_train_workspace_bytes": (ctypes.c_size_t, [_I32, _I32, _I32]),
+    "minw_conv_train_workspace_bytes": (ctypes.c_size_t, [_I32] * 9),
+    "minw_conv_train_step": (ctypes.c_int, [_P, _P, _P] + [_I32] * 9 + [_F, _F, _QP, _QP, _P, _P, _P, _P,
+                                            ctypes.c_size_t, _P]),
     "minw_fc_train_step": (ctypes.c_int, [_P, _P, _P, _I32, _I32, _I32, _F, _F, _QP, _QP, _P, _P, _P, _P,
                                           ctypes.c_size_t, _P]),
     "aqe_quantize_pack": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _F, _P, _P, _P]),
@@ -134,6 +137,7 @@ SIGNATURES = {
     "minw_net_enable_timing": (ctypes.c_int, [_P, _I32]),
     "minw_net_layer_times": (ctypes.c_int, [_P, _P]),
     "minw_net_layer_variants": (ctypes.c_int, [_P, _P]),
+    "minw_net_layer_candidates": (ctypes.c_int, [_P, ctypes.c_int32, _P]),
     "minw_net_launches": (_I32, [_P]),
     "minw_net_kernels": (_I32, [_P]),
     "minw_net_destroy": (None, [_P]),
@@ -275,6 +279,25 @@ def minw_fc_train_step(A, W, g_out, alpha, lr, q_w, q_a, a_out, g_in, workspace,
            "minw_fc_train_step")
 
 
+def minw_conv_train_workspace_bytes(B, C, H, W, O, kh, kw, stride, pad):
+    return int(lib().minw_conv_train_workspace_bytes(B, C, H, W, O, kh, kw, stride, pad))
+
+
+def minw_conv_train_step(A, W, g_out, stride, pad, alpha, lr, q_w, q_a, a_out, g_in, workspace, a_pre=None,
+                         stream=None):
+    """One Algorithm 1 step of a convolutional layer: A [B][C][H][W], W
+    [O][C][kh][kw] (updated in place), g_out [B][O][Ho][Wo]; a_pre, when
+    given, receives the convolution before the activation AQE."""
+    B, C, H, Wd = A.shape
+    O, _, kh, kw = W.shape
+    nbytes = workspace.numel() * workspace.element_size()
+    _check(lib().minw_conv_train_step(_ptr(A), _ptr(W), _ptr(g_out), B, C, H, Wd, O, kh, kw, int(stride), int(pad),
+                                      float(alpha), float(lr), ctypes.byref(q_w),
+                                      ctypes.byref(q_a) if q_a is not None else None, _ptr(a_out), _ptr(g_in),
+                                      _ptr(a_pre), _ptr(workspace), nbytes, _stream(stream)),
+           "minw_conv_train_step")
+
+
 def aqe_backward(x, gy, gx, alpha, stream=None):
     _check(lib().aqe_backward(_ptr(x), _ptr(gy), _ptr(gx), x.numel(), float(alpha), _stream(stream)),
            "aqe_backward")
@@ -367,8 +390,9 @@ def minw_conv_block_codes(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, strid
 def minw_conv_block_codes_ex(act, B, C, H, W, bits_a, wgt, O, kh, kw, bits_w, stride, pad, pool, scale, shift,
                              q_out=None, codes_out=None, planes_out=None, y_out=None, res_codes=None, res_bits=0,
                              res_f32=None, y_nhwc=None, in_format=CODES_E4M3, out_format=CODES_E4M3,
-                             res_format=CODES_E4M3, acc_out=None, stream=None):
+                             res_format=CODES_E4M3, acc_out=None, e2m1_pairs=False, stream=None):
     ex = BlockExtra()
+    ex.e2m1_pairs = int(bool(e2m1_pairs))
     ex.res_codes = res_codes.data_ptr() if res_codes is not None else None
     ex.res_bits = int(res_bits)
     ex.res_f32 = res_f32.data_ptr() if res_f32 is not None else None
@@ -539,10 +563,17 @@ class Net:
 
     def layer_variants(self):
         """Kernel per layer: 0 fp32 first layer, VARIANT_POPC, VARIANT_TC (E4M3
-        operands) or VARIANT_TC_E2M1."""
+        operands), VARIANT_TC_E2M1 or VARIANT_TC_E2M1_PAIRS."""
         n = self.launches
         arr = (ctypes.c_int32 * n)()
         _check(lib().minw_net_layer_variants(self._h, arr), "minw_net_layer_variants")
+        return list(arr)
+
+    def layer_candidates(self, layer):
+        """Creation-time milliseconds of layer `layer`'s candidates under
+        VARIANT_AUTO: [E4M3, E2M1, E2M1 pairs, popcount], -1 where not one."""
+        arr = (ctypes.c_float * 4)()
+        _check(lib().minw_net_layer_candidates(self._h, int(layer), arr), "minw_net_layer_candidates")
         return list(arr)
 
     @property

@@ -23,3 +23,10 @@ def assert_close(got, ref, rtol=1e-5, atol=1e-6):
     assert got.shape == ref.shape
     bad = np.abs(got - ref) > atol + rtol * np.abs(ref)
     assert not bad.any(), f"{bad.sum()} of {bad.size} outside tolerance; worst {np.max(np.abs(got - ref))}"
+
+
+def case_seed(*parts):
+    """A seed fixed by a test case's parameters (crc32 of their repr: unlike
+    hash(), the same in every process)."""
+    import zlib
+    return zlib.crc32(repr(parts).encode()) % 1000

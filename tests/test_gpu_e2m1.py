@@ -15,7 +15,7 @@ torch = pytest.importorskip("torch")
 from oracle import network as N  # noqa: E402
 from oracle import oracle as O  # noqa: E402
 from paper_2003_04296_gb300.inputs import DEFAULT_THR, conv_problem, convnet_input, convnet_params  # noqa: E402
-from tests._gpu import dev_tensor, planes_view  # noqa: E402
+from tests._gpu import case_seed, dev_tensor, planes_view  # noqa: E402
 
 pytestmark = pytest.mark.gpu
 
@@ -107,7 +107,7 @@ CASES = [
 @pytest.mark.parametrize("ba,bw", list(product([1, 2, 3], [1, 2, 3])))
 def test_conv_e2m1(dev, M, case, ba, bw):
     B, C, H, W, O_, k, stride, pad = case
-    p = conv_problem(hash((case, ba, bw, "e2m1")) % 1000, B, C, H, W, O_, k, k, stride, pad, ba, bw, w_sigma=0.5)
+    p = conv_problem(case_seed(case, ba, bw, "e2m1"), B, C, H, W, O_, k, k, stride, pad, ba, bw, w_sigma=0.5)
     act, wgt = _operands(dev, M, p)
     Ho, Wo = _out_hw(p)
     acc = torch.full((B, O_, Ho, Wo), -7, dtype=torch.int32, device=dev)
@@ -119,6 +119,35 @@ def test_conv_e2m1(dev, M, case, ba, bw):
     got = acc.cpu().numpy()
     assert np.array_equal(got, ref), f"{np.sum(got != ref)} of {ref.size} accumulators differ"
     assert np.array_equal(y.cpu().numpy(), O.affine(ref, p["scale"], p["shift"]))
+    assert M.minw_get_last_device_error() == M.MINW_OK
+
+
+PAIR_CASES = [
+    # B, C, H, W, O, k, stride, pad
+    (3, 512, 8, 8, 512, 3, 1, 1),     # odd pixel-tile count: the last pair holds one padded tile
+    (2, 256, 14, 14, 384, 3, 1, 1),   # 14x14 tiles overhang both edges, three 128-channel tiles
+    (4, 128, 16, 16, 128, 3, 2, 1),   # stride 2, one channel tile
+    (2, 128, 8, 8, 96, 3, 1, 1),      # O % 128 != 0: the request falls back to the default tiling
+]
+
+
+@pytest.mark.parametrize("case", PAIR_CASES)
+@pytest.mark.parametrize("ba,bw", [(1, 1), (2, 3), (3, 3)])
+def test_conv_e2m1_pairs_single_layer(dev, M, case, ba, bw):
+    """A single E2M1 convolution asked to run as CTA pairs of 256 pixels x
+    128 channels (minw_block_extra.e2m1_pairs): the same exact accumulators as
+    the oracle's, wherever the shape allows the pairs and where it does not."""
+    B, C, H, W, O_, k, stride, pad = case
+    seed = (7 * B + C + 3 * O_ + 5 * H + 11 * ba + 13 * bw) % 1000
+    p = conv_problem(seed, B, C, H, W, O_, k, k, stride, pad, ba, bw, w_sigma=0.5)
+    act, wgt = _operands(dev, M, p)
+    Ho, Wo = _out_hw(p)
+    acc = torch.full((B, O_, Ho, Wo), -7, dtype=torch.int32, device=dev)
+    M.minw_conv_block_codes_ex(act, B, C, H, W, ba, wgt, O_, k, k, bw, stride, pad, 0, None, None,
+                               in_format=M.CODES_E2M1, acc_out=acc, e2m1_pairs=True)
+    ref = _ref_acc(p)
+    got = acc.cpu().numpy()
+    assert np.array_equal(got, ref), f"{np.sum(got != ref)} of {ref.size} accumulators differ"
     assert M.minw_get_last_device_error() == M.MINW_OK
 
 

@@ -11,7 +11,7 @@ torch = pytest.importorskip("torch")
 
 from oracle import oracle as O  # noqa: E402
 from paper_2003_04296_gb300.inputs import DEFAULT_THR, aqe_problem, conv_problem  # noqa: E402
-from tests._gpu import assert_close, dev_tensor, planes_view, words  # noqa: E402
+from tests._gpu import case_seed, assert_close, dev_tensor, planes_view, words  # noqa: E402
 
 pytestmark = pytest.mark.gpu
 
@@ -144,7 +144,7 @@ def _conv_ref(p):
 @pytest.mark.parametrize("ba,bw", list(product([1, 2, 3], [1, 2, 3])))
 def test_conv2d_popc(dev, M, case, ba, bw):
     B, C, H, W, O_, k, s, pad = case
-    p = conv_problem(hash((case, ba, bw)) % 1000, B, C, H, W, O_, k, k, s, pad, ba, bw, w_sigma=0.5)
+    p = conv_problem(case_seed(case, ba, bw), B, C, H, W, O_, k, k, s, pad, ba, bw, w_sigma=0.5)
     _, _, acc, y = _conv_gpu(dev, M, p, M.VARIANT_POPC)
     ref = _conv_ref(p)
     assert np.array_equal(acc.cpu().numpy(), ref)

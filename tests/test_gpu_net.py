@@ -87,3 +87,32 @@ def test_cifar_convnet_batch256_sampled(dev, M):
     refs = OP.starmap(OP.convnet_logits, [(2, 1, 1, 2, 256, i) for i in idx])
     for i, ref in zip(idx, refs):
         assert np.array_equal(got[i:i + 1], ref), f"image {i}"
+
+
+@pytest.mark.parametrize("batch,bits", [(64, 1), (2, 2)])
+def test_auto_choice_is_the_measured_fastest(dev, M, batch, bits):
+    """MINW_VARIANT_AUTO times every layer the tensor cores cover on each
+    candidate (E4M3, E2M1, E2M1 CTA pairs, popcount on bit-planes) at creation
+    and keeps the fastest: the kernel each layer reports is the least of its
+    measured times, the popcount path was measured for every such layer, and
+    the net (whatever mix of layouts the measurement produced) still gives the
+    oracle's logits bit for bit.  Batch 2 makes the tensor-core tiles mostly
+    empty, where the popcount path can win."""
+    net_p = convnet_params(47, bits_a=bits, bits_w=bits, widths=(64, 128, 128, 256),
+                           pools=(False, True, False, True), fcs=(256,), classes=10, hw=16)
+    x = convnet_input(48, batch, hw=16)
+    net = M.Net(M.layer_descs(net_p, dev), max_batch=batch, variant=M.VARIANT_AUTO)
+    variants = net.layer_variants()
+    kind = {M.VARIANT_TC: 0, M.VARIANT_TC_E2M1: 1, M.VARIANT_TC_E2M1_PAIRS: 2, M.VARIANT_POPC: 3}
+    assert net.layer_candidates(0) == [-1.0] * 4
+    for layer in range(1, net.launches):
+        ms = net.layer_candidates(layer)
+        assert ms[0] > 0 and ms[3] > 0, (layer, ms)      # E4M3 and popcount cover every layer here
+        measured = [t if t >= 0 else np.inf for t in ms]
+        assert kind[variants[layer]] == int(np.argmin(measured)), (layer, variants[layer], ms)
+    logits = torch.empty((batch, net.out_features), dtype=torch.float32, device=dev)
+    net.forward(dev_tensor(x, dev), logits)
+    torch.cuda.synchronize()
+    got = logits.cpu().numpy()
+    net.close()
+    assert np.array_equal(got, N.convnet_forward(net_p, x))
