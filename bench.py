@@ -127,9 +127,15 @@ class Workload:
             return I.convnet_input(self.seed + 1000 * rank, self.batch)
         return I.resnet18_input(self.seed + 1000 * rank, self.batch)
 
-    def net(self, minw, dev, variant):
+    def net(self, minw, dev, variant, layer_variants=None):
         if self.name == "cifar_convnet":
-            return minw.Net(minw.layer_descs(self.params, dev), max_batch=self.batch, variant=variant)
+            descs = minw.layer_descs(self.params, dev)
+            if layer_variants:
+                # a plan measured by an earlier run, replayed (e.g. under a profiler, whose
+                # per-launch overhead would distort the creation-time measurement)
+                for d, v in zip(descs, layer_variants):
+                    d["variant"] = int(v)
+            return minw.Net(descs, max_batch=self.batch, variant=variant)
         return minw.Net.resnet18(self.params, self.batch, dev)
 
     def oracle(self, x):
@@ -401,6 +407,8 @@ def run_reference(args, rank):
         return run_reference_sweep(args)
     if args.workload == "fc_train":
         return run_reference_fc_train(args)
+    if args.workload == "conv_train":
+        return run_reference_conv_train(args)
     if args.workload == "conv1":
         return run_reference_conv1(args)
     wl = Workload(args.workload, args)
@@ -451,7 +459,8 @@ def run_gpu(args, rank, world, local_rank):
     wl = Workload(args.workload, args)
     BATCH = wl.batch
     x_np = wl.images(rank)
-    net = wl.net(minw, dev, args.variant)
+    lv = [int(v) for v in args.layer_variants.split(",")] if getattr(args, "layer_variants", None) else None
+    net = wl.net(minw, dev, args.variant, lv)
     x = torch.from_numpy(x_np).to(dev)
     logits = torch.empty((BATCH, net.out_features), dtype=torch.float32, device=dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
@@ -881,6 +890,196 @@ def run_fc_train(args, rank, world, local_rank):
     return line
 
 
+# --------------------------------------------------------- conv training --
+
+CONV_TRAIN_SHAPE = (256, 256, 16, 16, 256, 3, 1, 1)    # B, C, H, W, O, k, stride, pad: Model A's conv4
+CONV_TRAIN_ALPHA, CONV_TRAIN_LR = 0.75, 1e-3
+
+
+def conv_train_dims():
+    B, C, H, W, O, k, s, p = CONV_TRAIN_SHAPE
+    Ho, Wo = (H + 2 * p - k) // s + 1, (W + 2 * p - k) // s + 1
+    Hd, Wd = (Ho - 1) * s + 1 + (H + 2 * p - k) % s, (Wo - 1) * s + 1 + (W + 2 * p - k) % s
+    return B, C, H, W, O, k, s, p, Ho, Wo, Hd, Wd
+
+
+def conv_step_bytes():
+    """Bytes the convolutional training step's launches move at least, launch
+    by launch: the weight pass (W read; W^ written in the forward and the
+    flipped layouts), the input's bf16 NHWC copy and its transposed patches
+    (A read twice, both written), the forward product (bf16 input and W^
+    read, a~ written), the gradient pass (a~ and g read; a_out, g~ as rows
+    and as the spread NHWC image written), the input-gradient product (the
+    spread image and the flipped W^ read, g_in written), the weight-gradient
+    product (g~ rows and the patches read, the gradient written), and the
+    update (W and the gradient read, W written)."""
+    B, C, H, W, O, k, s, p, Ho, Wo, Hd, Wd = conv_train_dims()
+    Op = (O + 63) // 64 * 64
+    Kw, npix, x = C * k * k, B * Ho * Wo, B * C * H * W
+    return float((4 * O * Kw + 2 * O * Kw + 2 * Kw * Op)
+                 + (4 * x + 2 * x) + (4 * x + 2 * Kw * npix)
+                 + (2 * x + 2 * O * Kw + 4 * O * npix)
+                 + (8 * O * npix + 4 * O * npix + 2 * O * npix + 2 * B * Hd * Wd * Op)
+                 + (2 * B * Hd * Wd * Op + 2 * C * k * k * Op + 4 * x)
+                 + (2 * O * npix + 2 * Kw * npix + 4 * O * Kw)
+                 + 12 * O * Kw)
+
+
+def conv_min_bytes():
+    """The step's irreducible traffic: A, W and g read once, a~ (a_pre),
+    a_out, g_in and the updated W written once."""
+    B, C, H, W, O, k, s, p, Ho, Wo, Hd, Wd = conv_train_dims()
+    return float(4 * (B * C * H * W) * 2 + 4 * O * C * k * k * 2 + 4 * (B * O * Ho * Wo) * 3)
+
+
+def conv_train_problem(rank=0):
+    B, C, H, W, O, k, s, p, Ho, Wo, Hd, Wd = conv_train_dims()
+    r = np.random.default_rng(37 + 1000 * rank)
+    A = np.clip(r.standard_normal((B, C, H, W)), -1.5, 1.5).astype(np.float32)
+    Wl = r.uniform(-1, 1, (O, C, k, k)).astype(np.float32)
+    G = (r.standard_normal((B, O, Ho, Wo)) * 0.1).astype(np.float32)
+    return A, Wl, G
+
+
+def conv_train_config(world):
+    B, C, H, W, O, k, s, p, Ho, Wo, Hd, Wd = conv_train_dims()
+    return {"workload": f"conv_train_{C}to{O}_{H}x{W}_b{B}_a1w1", "batch_per_gpu": B, "global_batch": B * world,
+            "layer": f"conv {k}x{k}/{s}/{p} {C} -> {O} at {H}x{W} (Model A's conv4), alpha {CONV_TRAIN_ALPHA}, "
+                     f"lr {CONV_TRAIN_LR}, SGD + clip",
+            "parallelism": f"replicas x{world} (no gradient all-reduce)", "l2": L2_NOTE}
+
+
+def conv_train_oracle_rate(A, Wl, G, budget_s=10.0, images=2):
+    """The oracle's convolutional training step (oracle.conv_train_step) on
+    the first `images` images of the batch, repeated until budget_s seconds;
+    returns (images/s, seconds per sub-batch step, steps)."""
+    from oracle import oracle as Or
+    from paper_2003_04296_gb300.inputs import DEFAULT_THR
+    B, C, H, W, O, k, s, p, Ho, Wo, Hd, Wd = conv_train_dims()
+    a, g = A[:images], G[:images]
+    times = []
+    t_start = time.perf_counter()
+    while not times or time.perf_counter() - t_start < budget_s:
+        t0 = time.perf_counter()
+        Or.conv_train_step(a, Wl, g, CONV_TRAIN_ALPHA, CONV_TRAIN_LR, 1, DEFAULT_THR[1], s, p, (1, DEFAULT_THR[1]))
+        times.append(time.perf_counter() - t0)
+    sec = sum(times) / len(times)
+    return images / sec, sec, len(times)
+
+
+def run_reference_conv_train(args):
+    A, Wl, G = conv_train_problem(0)
+    steps = []
+    for _ in range(args.steps):
+        ips, sec, n = conv_train_oracle_rate(A, Wl, G, budget_s=0.0)
+        steps.append(sec)
+    sec = sum(steps) / len(steps)
+    ips = 2 / sec
+    line = {"metric": "Algorithm 1 training step of a convolutional MINW layer: images/s", "value": ips,
+            "unit": "images/s", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": sec * 1e3, "higher_is_better": True, "impl": "reference", "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": conv_train_config(args.gpus),
+            "cpu_baseline": {"value": ips, "unit": "images/s", "cores": 1, "kind": "oracle",
+                             "sample": "each step: oracle.conv_train_step on 2 images of the batch (single-threaded "
+                                       "C fp64 convolutions), scaled per image"},
+            "e2e": {"value": ips, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_conv_train(args, rank, world, local_rank):
+    """Algorithm 1's training step of Model A's conv4 (256 -> 256 channels,
+    16 x 16, 3 x 3, batch 256, 1-bit weights and activations, alpha 0.75)
+    through minw_conv_train_step: three bf16 tensor-core products (forward,
+    input gradient, weight gradient) and five operand and update passes.
+    Its roofline is HBM: the bytes its launches move at least
+    (conv_step_bytes), over the step's event time; the fraction of the
+    step's irreducible bytes (conv_min_bytes) is reported beside it."""
+    import torch
+    import __graft_entry__ as g
+    if rank == 0:
+        g.build()
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    from paper_2003_04296_gb300 import minw
+    from paper_2003_04296_gb300.inputs import DEFAULT_THR
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    B, C, H, W, O, k, s, p, Ho, Wo, Hd, Wd = conv_train_dims()
+    A_np, W_np, G_np = conv_train_problem(rank)
+    A, Wl, G = (torch.from_numpy(x).to(dev) for x in (A_np, W_np, G_np))
+    a_out = torch.empty((B, O, Ho, Wo), device=dev)
+    g_in = torch.empty((B, C, H, W), device=dev)
+    ws = torch.empty(minw.minw_conv_train_workspace_bytes(B, C, H, W, O, k, k, s, p), dtype=torch.uint8, device=dev)
+    qw, qa = minw.quant(1, DEFAULT_THR[1]), minw.quant(1, DEFAULT_THR[1])
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        minw.minw_conv_train_step(A, Wl, G, s, p, CONV_TRAIN_ALPHA, CONV_TRAIN_LR, qw, qa, a_out, g_in, ws)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    e0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    e1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    with ClockSampler(local_rank) as clk:
+        for kk in range(args.steps):
+            flush.zero_()
+            e0[kk].record(stream)
+            step()
+            e1[kk].record(stream)
+        torch.cuda.synchronize()
+    ms_max = max_over_ranks(sum(e0[kk].elapsed_time(e1[kk]) for kk in range(args.steps)) / args.steps, world, dev)
+    A_host = A.cpu().pin_memory()
+    G_host = G.cpu().pin_memory()
+    gin_host = torch.empty((B, C, H, W), dtype=torch.float32).pin_memory()
+    e2e_s = []
+    for kk in range(min(args.steps, 20) + 1):
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        A.copy_(A_host, non_blocking=True)
+        G.copy_(G_host, non_blocking=True)
+        step()
+        gin_host.copy_(g_in, non_blocking=True)
+        torch.cuda.synchronize()
+        if kk:
+            e2e_s.append(time.perf_counter() - t0)
+    e2e_sec = max_over_ranks(sum(e2e_s) / len(e2e_s), world, dev)
+    if rank != 0:
+        return None
+    cpu = None
+    if world == 1 and not args.skip_cpu:
+        ips, sec, n = conv_train_oracle_rate(A_np, W_np, G_np, budget_s=10.0)
+        cpu = {"value": ips, "unit": "images/s", "cores": 1, "kind": "oracle",
+               "sample": f"{n} steps of oracle.conv_train_step on 2 images of the batch ({sec:.2f} s each; "
+                         "single-threaded C fp64 convolutions), scaled per image"}
+    flops = 6.0 * B * Ho * Wo * O * C * k * k
+    nbytes = conv_step_bytes()
+    achieved = nbytes / (ms_max * 1e-3) / 1e9
+    line = {"metric": "Algorithm 1 training step of a convolutional MINW layer: images/s",
+            "value": replica_throughput(B, world, ms_max * 1e-3), "unit": "images/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": conv_train_config(world),
+            "roofline": {"bound": "hbm", "kernel": "the whole step (10 launches: weight, input and gradient "
+                                                   "passes, 3 bf16 tensor-core products, the weight gradient's "
+                                                   "slice sum, the update)",
+                         "achieved": achieved, "peak": HBM_GBS, "unit": "GB/s",
+                         "frac": achieved / HBM_GBS, "traffic": None, "bytes_per_step": nbytes,
+                         "frac_of_irreducible_bytes": conv_min_bytes() / (ms_max * 1e-3) / 1e9 / HBM_GBS,
+                         "irreducible_bytes": conv_min_bytes(),
+                         "peak_basis": "measured HBM copy GB/s, of measured"},
+            "tensor_tflops": flops / (ms_max * 1e-3) / 1e12,
+            "cpu_baseline": cpu,
+            "e2e": {"value": replica_throughput(B, world, e2e_sec), "unit": "images/s",
+                    "h2d_bytes_per_step": int(4 * (A.numel() + G.numel())), "d2h_bytes_per_step": int(4 * g_in.numel())},
+            "gpu_launches": 10 * args.steps, "clocks": clk.summary()}
+    return line
+
+
 def run_sweep(args, rank, world, local_rank):
     """One step: quantize the input to level codes and convolve it with the
     weight codes for each of the nine bit-width pairs (int32 accumulators),
@@ -1176,7 +1375,8 @@ def main():
                     help="timed steps (default 1000 for the ConvNet, 100 for ResNet-18: about a second)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["minw", "reference"], default="minw")
-    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "sweep", "fc_train", "conv1", "peaks"],
+    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "sweep", "fc_train", "conv_train", "conv1",
+                                           "peaks"],
                     default="cifar_convnet")
     ap.add_argument("--bits-a", type=int, default=1, help="CIFAR ConvNet activation bits")
     ap.add_argument("--bits-w", type=int, default=1, help="CIFAR ConvNet weight bits")
@@ -1185,6 +1385,9 @@ def main():
     ap.add_argument("--bits-a-resnet", type=int, default=3)
     ap.add_argument("--bits-w-resnet", type=int, default=3)
     ap.add_argument("--variant", type=int, default=0, help="0 auto, 1 popcount, 2 tensor cores")
+    ap.add_argument("--layer-variants", default=None,
+                    help="comma-separated kernel request per layer (the layer_variants of an earlier run): "
+                         "replays that measured plan instead of measuring at creation")
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--no-configs", action="store_true",
@@ -1192,7 +1395,7 @@ def main():
     args = ap.parse_args()
     default_run = args.steps is None and args.workload == "cifar_convnet"
     if args.steps is None:
-        args.steps = {"cifar_convnet": 1000, "resnet18": 100, "sweep": 20, "fc_train": 200,
+        args.steps = {"cifar_convnet": 1000, "resnet18": 100, "sweep": 20, "fc_train": 200, "conv_train": 50,
                       "conv1": 1000, "peaks": 1}[args.workload]
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -1206,7 +1409,7 @@ def main():
         torch.cuda.set_device(local_rank)
         dist.init_process_group("nccl")
     try:
-        runner = {"sweep": run_sweep, "fc_train": run_fc_train, "conv1": run_conv1,
+        runner = {"sweep": run_sweep, "fc_train": run_fc_train, "conv_train": run_conv_train, "conv1": run_conv1,
                   "peaks": run_peaks}.get(args.workload, run_gpu)
         line = runner(args, rank, world, local_rank)
         if line is not None and default_run and world == 1 and not args.no_configs:

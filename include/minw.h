@@ -297,9 +297,11 @@ MINW_API minw_status minw_conv2d_bf16(const uint16_t *act, int32_t B, int32_t C,
 /* Training step of a fully connected layer (Algorithm 1)                  */
 /* ---------------------------------------------------------------------- */
 
-/* The bf16 operands of Algorithm 1's training products (R21 reading: bf16
- * operands, fp32 sums).  out (bf16, round to nearest even, row-major
- * (transpose ? cols : rows) x out_cols) = in (fp32 row-major rows x cols),
+/* The bf16 operands of Algorithm 1's training products (bf16 roundings of
+ * the fp32 operands, fp32 sums: a precision departure from the paper's fp32
+ * training, with the error bound stated at minw_fc_train_step's products).
+ * out (bf16, round to nearest even, row-major (transpose ? cols : rows) x
+ * out_cols) = in (fp32 row-major rows x cols),
  * transposed when transpose != 0, zero in the columns past the source's.
  * Caller-owned device buffers; asynchronous on stream.  MINW_EINVAL for null
  * pointers, non-positive sizes or out_cols below the source's columns;
@@ -330,6 +332,11 @@ MINW_API size_t minw_fc_train_workspace_bytes(int32_t B, int32_t K, int32_t O);
  *   W = min(1, max(-1, W - lr 2 alpha g_W^ 1[|W| <= 1]))   (Eq. weight, update and clip)
  * a_pre (nullable, [B][O]) receives a~ when q_a is set (ignored without q_a,
  * where a_out is a~ itself).
+ * Each product P Q of K terms takes bf16 roundings of its fp32 operands (the
+ * paper trains on fp32 ones: a precision departure) and differs from the
+ * exact product of the fp32 operands by at most
+ * (2^-7 + 2^-16 + K 2^-23 (1 + 2^-8)^2) (|P| |Q|): the two operand roundings
+ * and the fp32 accumulation in any order.
  * A product with few output tiles and a long reduction adds its fp32 sums in K
  * slices, slice by slice in a fixed order (deterministic, same bound).
  * Requirements: K % 64 == 0 and B % 64 == 0 (else MINW_EUNSUPPORTED), alpha in
@@ -519,6 +526,14 @@ typedef struct {
     const float *w_scale;     /* per-output-channel prescale, nullable */
     const float *scale;       /* BN scale (length O) */
     const float *shift;       /* BN shift (length O) */
+    int32_t variant;          /* this layer's kernel request, in the values
+                                 minw_net_layer_variants reports; 0 follows the network's
+                                 request.  A non-zero request skips the layer's creation-time
+                                 measurement and runs: MINW_VARIANT_POPC the popcount path,
+                                 MINW_VARIANT_TC or _TC_E4M3 E4M3 operands, _TC_E2M1 E2M1
+                                 operands, _TC_E2M1_PAIRS E2M1 CTA pairs, each where the shape
+                                 allows it (a replay of a measured plan, e.g. under a profiler
+                                 whose overhead would distort the measurement) */
 } minw_layer_desc;
 
 typedef struct minw_net minw_net;

@@ -42,32 +42,31 @@ __global__ void __launch_bounds__(256) train_weights_kernel(const float *__restr
                                                             int Op, float alpha, QParams q, uint16_t *__restrict__ wf,
                                                             uint16_t *__restrict__ wd, float *__restrict__ ones,
                                                             float *__restrict__ zeros, int M) {
+    // element counts below 2^31 (checked by the host): 32-bit index arithmetic
     const float oma = 1.0f - alpha;
     const int khw = kh * kw;
-    const int64_t nf = (int64_t)O * khw * C, nd = (int64_t)C * khw * Op;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nf; i += stride) {
+    const int nf = O * khw * C, nd = C * khw * Op;
+    const int stride = gridDim.x * blockDim.x;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nf; i += stride) {
         // i = ((o kh + ky) kw + kx) C + c
-        const int c = (int)(i % C);
-        const int64_t r = i / C;
-        const int t = (int)(r % khw), o = (int)(r / khw);
-        const float x = W[((int64_t)o * C + c) * khw + t];
+        const int c = i % C, r = i / C;
+        const int t = r % khw, o = r / khw;
+        const float x = W[(o * C + c) * khw + t];
         wf[i] = bf16_bits(fmaf(alpha, level_value(x * q.scale, q), oma * x));
     }
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nd; i += stride) {
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nd; i += stride) {
         // i = ((c kh + ky) kw + kx) Op + o, source tap (kh - 1 - ky, kw - 1 - kx)
-        const int o = (int)(i % Op);
-        const int64_t r = i / Op;
-        const int t = (int)(r % khw), c = (int)(r / khw);
+        const int o = i % Op, r = i / Op;
+        const int t = r % khw, c = r / khw;
         float v = 0.0f;
         if (o < O) {
             const int ky = t / kw, kx = t - ky * kw;
-            const float x = W[((int64_t)o * C + c) * khw + (kh - 1 - ky) * kw + (kw - 1 - kx)];
+            const float x = W[(o * C + c) * khw + (kh - 1 - ky) * kw + (kw - 1 - kx)];
             v = fmaf(alpha, level_value(x * q.scale, q), oma * x);
         }
         wd[i] = bf16_bits(v);
     }
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < M; i += stride) {
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < M; i += stride) {
         ones[i] = 1.0f;
         zeros[i] = 0.0f;
     }
@@ -75,36 +74,58 @@ __global__ void __launch_bounds__(256) train_weights_kernel(const float *__restr
 
 // The input's patches, transposed: colT[(c kh + ky) kw + kx][n] =
 // bf16(A[b][c][y s - pad + ky][x s - pad + kx]) for output pixel n = (b Ho +
-// y) Wo + x, zero outside the image.  One thread writes eight consecutive
-// pixels of one row (a 16-byte store); for stride 1 the reads of a warp run
-// along an image row.
+// y) Wo + x, zero outside the image.  A thread takes eight consecutive pixels
+// n0 .. n0 + 7 of one channel c (blockIdx.y) and writes them for every tap:
+// kh kw 16-byte stores, each warp's store of a tap 512 contiguous bytes of
+// that tap's row.  The pixels' (b, y, x) come from one division and carries;
+// the taps' overlapping input reads hit L1, so each input value crosses from
+// L2 about once instead of once per tap.
 __global__ void __launch_bounds__(256) train_patches_kernel(const float *__restrict__ A, int B, int C, int H, int W,
                                                             int kh, int kw, int stride, int pad, int Ho, int Wo,
                                                             uint16_t *__restrict__ colT) {
-    const int64_t npix = (int64_t)B * Ho * Wo;
-    const int64_t groups = npix / 8;                      // npix % 8 == 0 (checked by the host)
-    const int64_t rows = (int64_t)C * kh * kw;
-    const int64_t total = rows * groups;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t row = i / groups;
-        const int64_t n0 = (i - row * groups) * 8;
-        const int kx = (int)(row % kw), ky = (int)((row / kw) % kh), c = (int)(row / ((int64_t)kh * kw));
-        uint32_t w[4];
+    const int HoWo = Ho * Wo;
+    const int npix = B * HoWo;                            // < 2^31 and a multiple of 8 (checked by the host)
+    const int c = blockIdx.y;
+    const int g = blockIdx.x * blockDim.x + threadIdx.x;
+    if (g >= npix / 8) return;
+    const int n0 = 8 * g;
+    // the eight pixels: image offset, first input row and column
+    int64_t base[8];
+    int iy0[8], ix0[8];
+    {
+        int b = n0 / HoWo;
+        const int r = n0 - b * HoWo;
+        int y = r / Wo, x = r - (r / Wo) * Wo;
 #pragma unroll
-        for (int e = 0; e < 8; e += 2) {
-            float v[2];
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int64_t n = n0 + e + h;
-                const int x = (int)(n % Wo);
-                const int64_t by = n / Wo;
-                const int y = (int)(by % Ho), b = (int)(by / Ho);
-                const int iy = y * stride - pad + ky, ix = x * stride - pad + kx;
-                v[h] = (iy >= 0 && iy < H && ix >= 0 && ix < W) ? A[(((int64_t)b * C + c) * H + iy) * W + ix] : 0.0f;
+        for (int e = 0; e < 8; ++e) {
+            base[e] = ((int64_t)b * C + c) * H * W;
+            iy0[e] = y * stride - pad;
+            ix0[e] = x * stride - pad;
+            if (++x == Wo) {
+                x = 0;
+                if (++y == Ho) {
+                    y = 0;
+                    ++b;
+                }
             }
-            w[e >> 1] = (uint32_t)bf16_bits(v[0]) | ((uint32_t)bf16_bits(v[1]) << 16);
         }
-        *reinterpret_cast<uint4 *>(colT + row * npix + n0) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+    for (int ky = 0; ky < kh; ++ky) {
+        for (int kx = 0; kx < kw; ++kx) {
+            uint32_t w[4];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const int iy = iy0[e] + ky, ix = ix0[e] + kx;
+                const float v = (iy >= 0 && iy < H && ix >= 0 && ix < W) ? __ldg(A + base[e] + (int64_t)iy * W + ix)
+                                                                          : 0.0f;
+                if (e & 1)
+                    w[e >> 1] |= (uint32_t)bf16_bits(v) << 16;
+                else
+                    w[e >> 1] = (uint32_t)bf16_bits(v);
+            }
+            const int64_t row = ((int64_t)c * kh + ky) * kw + kx;
+            *reinterpret_cast<uint4 *>(colT + row * npix + n0) = make_uint4(w[0], w[1], w[2], w[3]);
+        }
     }
 }
 
@@ -272,7 +293,9 @@ minw_status minw_conv_train_step(const float *A, float *Wt, const float *g_out, 
     if (!conv_train_shape(B, C, H, W, O, kh, kw, stride, pad, sh)) return MINW_EINVAL;
     if (sh.npix % 64 != 0 || sh.npix > INT32_MAX) return MINW_EUNSUPPORTED;
     // 32-bit grid limits of the gradient pass; 64-bit element indices everywhere else
-    if ((O + 31) / 32 > 65535 || B > 65535) return MINW_EUNSUPPORTED;
+    if ((O + 31) / 32 > 65535 || B > 65535 || C > 65535) return MINW_EUNSUPPORTED;
+
+    if ((int64_t)sh.Kw * (O > sh.Op ? O : sh.Op) >= (1ll << 31)) return MINW_EUNSUPPORTED;     // weight pass indices
     ConvTrainLayout L;
     minw_status st = conv_train_layout(B, C, H, W, O, kh, kw, stride, pad, L);
     if (st != MINW_OK) return st;
@@ -294,8 +317,10 @@ minw_status minw_conv_train_step(const float *A, float *Wt, const float *g_out, 
                                                                              wd, ones, zeros, M);
     TRY(launch_status());
     TRY(minw_to_bf16_nhwc(A, B, C, H, W, ab, stream));
-    train_patches_kernel<<<grid_for((int64_t)sh.Kw * (sh.npix / 8)), 256, 0, s>>>(A, B, C, H, W, kh, kw, stride, pad,
-                                                                                  sh.Ho, sh.Wo, colT);
+    {
+        const dim3 grid((unsigned)((sh.npix / 8 + 255) / 256), (unsigned)C);
+        train_patches_kernel<<<grid, 256, 0, s>>>(A, B, C, H, W, kh, kw, stride, pad, sh.Ho, sh.Wo, colT);
+    }
     TRY(launch_status());
     // a~ = a * W^ (fp32 NCHW [B][O][Ho][Wo]); the last layer emits a~ itself
     float *fwd_out = q_a ? at : a_out;

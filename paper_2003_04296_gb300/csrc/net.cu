@@ -74,7 +74,7 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
     std::vector<int> cand;
     for (int l = 1; l < n_layers; ++l) {
         const LayerPlan &P = n->L[l];
-        if (P.variant != MINW_VARIANT_TC) continue;
+        if (P.variant != MINW_VARIANT_TC || layers[l].variant != 0) continue;
         cand.push_back(l);
         // codes (one byte per channel at most) or bit-planes (3 bits per channel at most) in;
         // codes, planes or fp32 logits out
@@ -211,7 +211,11 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
         P.d = d;
         P.d.w = nullptr; P.d.w_scale = nullptr; P.d.scale = nullptr; P.d.shift = nullptr;
         const bool first = l == 0, last = l == n_layers - 1;
-        if (!d.w || !d.scale || !d.shift || d.O <= 0 || d.C <= 0 || d.H <= 0 || d.W <= 0) {
+        // this layer's request, in the values minw_net_layer_variants reports (there
+        // MINW_VARIANT_TC is a layer on E4M3 operands), else the network's
+        const int req = d.variant != 0 ? (d.variant == MINW_VARIANT_TC ? MINW_VARIANT_TC_E4M3 : d.variant) : variant;
+        if (!d.w || !d.scale || !d.shift || d.O <= 0 || d.C <= 0 || d.H <= 0 || d.W <= 0 || d.variant < 0 ||
+            d.variant > MINW_VARIANT_TC_E2M1_PAIRS) {
             net_free(n);
             return MINW_EINVAL;
         }
@@ -284,14 +288,14 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
             a.pool = P.pool;
             a.quant_out = !last;
             if (!last) a.qo = to_qparams(&P.qo);
-            P.variant = choose_variant(a, variant >= MINW_VARIANT_TC ? MINW_VARIANT_TC : variant);
+            P.variant = choose_variant(a, req >= MINW_VARIANT_TC ? MINW_VARIANT_TC : req);
             if (P.variant == MINW_VARIANT_TC && !conv_tc_supported(a)) { net_free(n); return MINW_EUNSUPPORTED; }
-            if (P.variant == MINW_VARIANT_TC && variant != MINW_VARIANT_TC_E4M3) {
+            if (P.variant == MINW_VARIANT_TC && req != MINW_VARIANT_TC_E4M3) {
                 // E2M1 operands wherever the channels fill 64-byte rows
                 a.fp4 = 1;
                 P.in4 = conv_tc_supported(a) ? 1 : 0;
                 a.fp4 = P.in4;
-                if (variant == MINW_VARIANT_TC_E2M1_PAIRS && P.in4) {
+                if (req == MINW_VARIANT_TC_E2M1_PAIRS && P.in4) {
                     a.pair_n128 = 1;
                     P.pair128 = conv_tc_pairs128(a) ? 1 : 0;
                     a.pair_n128 = P.pair128;

@@ -63,7 +63,7 @@ class LayerDesc(ctypes.Structure):
                 ("pool", ctypes.c_int32), ("bits_in", ctypes.c_int32), ("bits_w", ctypes.c_int32),
                 ("bits_out", ctypes.c_int32), ("thr_w", ctypes.c_float * 3),
                 ("thr_out", ctypes.c_float * 3), ("w", ctypes.c_void_p), ("w_scale", ctypes.c_void_p),
-                ("scale", ctypes.c_void_p), ("shift", ctypes.c_void_p)]
+                ("scale", ctypes.c_void_p), ("shift", ctypes.c_void_p), ("variant", ctypes.c_int32)]
 
 
 class ResNet18Desc(ctypes.Structure):
@@ -526,6 +526,7 @@ class Net:
             d.kh, d.kw, d.stride, d.pad, d.pool = L.get("kh", 1), L.get("kw", 1), L.get("stride", 1), \
                 L.get("pad", 0), int(L.get("pool", 0))
             d.bits_in, d.bits_w, d.bits_out = L["bits_in"], L["bits_w"], L["bits_out"]
+            d.variant = int(L.get("variant", 0))
             for i in range(3):
                 d.thr_w[i] = float(L["thr_w"][i])
                 d.thr_out[i] = float(L["thr_out"][i])

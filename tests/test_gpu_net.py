@@ -116,3 +116,30 @@ def test_auto_choice_is_the_measured_fastest(dev, M, batch, bits):
     got = logits.cpu().numpy()
     net.close()
     assert np.array_equal(got, N.convnet_forward(net_p, x))
+
+
+def test_per_layer_requests_replay_a_plan(dev, M):
+    """A per-layer kernel request (minw_layer_desc.variant) skips that layer's
+    measurement and runs the requested kernel: popcount, E4M3, E2M1 and E2M1
+    CTA pairs mixed in one net (each layer's input layout follows its
+    consumer), requested in the values minw_net_layer_variants reports
+    (VARIANT_TC: E4M3 operands) and reported back unchanged, with the oracle's
+    logits bit for bit."""
+    net_p = convnet_params(49, bits_a=2, bits_w=1, widths=(128, 128, 256, 256),
+                           pools=(False, True, False, True), fcs=(256,), classes=10, hw=16)
+    x = convnet_input(50, 24, hw=16)
+    req = [0, M.VARIANT_POPC, M.VARIANT_TC, M.VARIANT_TC_E2M1_PAIRS, M.VARIANT_TC_E2M1, M.VARIANT_POPC]
+    descs = M.layer_descs(net_p, dev)
+    assert len(descs) == len(req)
+    for d, v in zip(descs, req):
+        d["variant"] = v
+    net = M.Net(descs, max_batch=24, variant=M.VARIANT_AUTO)
+    assert net.layer_variants() == req
+    for layer in range(net.launches):
+        assert net.layer_candidates(layer) == [-1.0] * 4        # nothing measured
+    logits = torch.empty((24, net.out_features), dtype=torch.float32, device=dev)
+    net.forward(dev_tensor(x, dev), logits)
+    torch.cuda.synchronize()
+    got = logits.cpu().numpy()
+    net.close()
+    assert np.array_equal(got, N.convnet_forward(net_p, x))
