@@ -1343,11 +1343,11 @@ def other_configs(args, rank, world, local_rank):
     the bit-width sweep."""
     import copy
     out = {}
-    jobs = [("conv1", run_conv1, dict(workload="conv1", steps=300)),
-            ("cifar_convnet_a2w1", run_gpu, dict(workload="cifar_convnet", bits_a=2, bits_w=1, steps=200)),
-            ("cifar_convnet_a2w2", run_gpu, dict(workload="cifar_convnet", bits_a=2, bits_w=2, steps=200)),
-            ("resnet18_a3w3", run_gpu, dict(workload="resnet18", steps=40)),
-            ("sweep", run_sweep, dict(workload="sweep", steps=8))]
+    jobs = [("conv1", run_conv1, dict(workload="conv1", steps=3000)),
+            ("cifar_convnet_a2w1", run_gpu, dict(workload="cifar_convnet", bits_a=2, bits_w=1, steps=1500)),
+            ("cifar_convnet_a2w2", run_gpu, dict(workload="cifar_convnet", bits_a=2, bits_w=2, steps=1500)),
+            ("resnet18_a3w3", run_gpu, dict(workload="resnet18", steps=200)),
+            ("sweep", run_sweep, dict(workload="sweep", steps=40))]
     for name, fn, ch in jobs:
         a = copy.copy(args)
         for k, v in ch.items():
@@ -1372,7 +1372,8 @@ def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=None,
-                    help="timed steps (default 1000 for the ConvNet, 100 for ResNet-18: about a second)")
+                    help="timed steps (defaults give about half a second of timed work, so that the clock "
+                         "sampler sees several samples under load)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["minw", "reference"], default="minw")
     ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "sweep", "fc_train", "conv_train", "conv1",
@@ -1395,7 +1396,7 @@ def main():
     args = ap.parse_args()
     default_run = args.steps is None and args.workload == "cifar_convnet"
     if args.steps is None:
-        args.steps = {"cifar_convnet": 1000, "resnet18": 100, "sweep": 20, "fc_train": 200, "conv_train": 50,
+        args.steps = {"cifar_convnet": 4000, "resnet18": 400, "sweep": 100, "fc_train": 2000, "conv_train": 500,
                       "conv1": 1000, "peaks": 1}[args.workload]
 
     world = int(os.environ.get("WORLD_SIZE", "1"))

@@ -431,15 +431,25 @@ __global__ void weight_bf16_kernel(const float *__restrict__ w, int O, int C, in
 
 // fp32 NCHW -> bf16 NHWC, round to nearest even: one thread per output element
 // of a 32 x 32 (channel, pixel) tile transposed through shared memory.
-__global__ void to_bf16_nhwc_kernel(const float *__restrict__ x, int C, int HW, uint16_t *__restrict__ out) {
+// Block (32, 8): a 32-channel x 32-pixel tile of one image through shared
+// memory; each thread's four loads issue before its first shared-memory store.
+__global__ void __launch_bounds__(256) to_bf16_nhwc_kernel(const float *__restrict__ x, int C, int HW,
+                                                           uint16_t *__restrict__ out) {
     __shared__ float tile[32][33];
     const int b = blockIdx.z, c0 = blockIdx.y * 32, p0 = blockIdx.x * 32;
-    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+    float v[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int i = threadIdx.y + 8 * k;
         const int c = c0 + i, p = p0 + threadIdx.x;
-        tile[i][threadIdx.x] = (c < C && p < HW) ? x[((int64_t)b * C + c) * HW + p] : 0.0f;
+        v[k] = (c < C && p < HW) ? __ldg(x + ((int64_t)b * C + c) * HW + p) : 0.0f;
     }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) tile[threadIdx.y + 8 * k][threadIdx.x] = v[k];
     __syncthreads();
-    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int i = threadIdx.y + 8 * k;
         const int p = p0 + i, c = c0 + threadIdx.x;
         if (c < C && p < HW)
             out[((int64_t)b * HW + p) * C + c] = __bfloat16_as_ushort(__float2bfloat16_rn(tile[threadIdx.x][i]));

@@ -149,25 +149,40 @@ __global__ void __launch_bounds__(256) train_grad_kernel(const float *__restrict
     const int o0 = blockIdx.y * 32, p0 = blockIdx.x * 32;
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;      // 8 rows of 32
     const float oma = 1.0f - alpha, two_alpha = 2.0f * alpha;
-    for (int k = ty; k < 32; k += 8) {
+    // the four rows' loads first, then the arithmetic and the stores
+    float gl[4], xl[4];
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+        const int o = o0 + ty + 8 * kk, p = p0 + tx;
+        gl[kk] = xl[kk] = 0.0f;
+        if (o < O && p < HoWo) {
+            const int64_t idx = ((int64_t)b * O + o) * HoWo + p;
+            gl[kk] = __ldg(G + idx);
+            if (quant_a) xl[kk] = __ldg(at + idx);
+        }
+    }
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+        const int k = ty + 8 * kk;
         const int o = o0 + k, p = p0 + tx;
         float gv = 0.0f;
         if (o < O && p < HoWo) {
             const int64_t idx = ((int64_t)b * O + o) * HoWo + p;
-            const float g = G[idx];
             if (quant_a) {
-                const float x = at[idx];
+                const float x = xl[kk];
                 a_out[idx] = fmaf(alpha, level_value(x * qa.scale, qa), oma * x);
-                gv = (fabsf(x) <= 1.0f) ? g * two_alpha : 0.0f;
+                gv = (fabsf(x) <= 1.0f) ? gl[kk] * two_alpha : 0.0f;
             } else {
-                gv = g;
+                gv = gl[kk];
             }
             gT[(int64_t)o * npix + (int64_t)b * HoWo + p] = bf16_bits(gv);
         }
         tile[k][tx] = gv;
     }
     __syncthreads();
-    for (int k = ty; k < 32; k += 8) {
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+        const int k = ty + 8 * kk;
         const int p = p0 + k, o = o0 + tx;
         if (p < HoWo && o < O) {
             const int y = p / Wo, x = p - y * Wo;
