@@ -533,7 +533,8 @@ def run_gpu(args, rank, world, local_rank):
     q_ms = float(sum(layer_ms[i] for i in q_ops_idx))
     q_ops = 2.0 * sum(macs[i] for i in q_ops_idx) * BATCH
     achieved = q_ops / (q_ms * 1e-3) / 1e12
-    tc_kind = {minw.VARIANT_TC: "e4m3", minw.VARIANT_TC_E2M1: "e2m1", minw.VARIANT_TC_E2M1_PAIRS: "e2m1"}
+    tc_kind = {minw.VARIANT_TC: "e4m3", minw.VARIANT_TC_E2M1: "e2m1", minw.VARIANT_TC_E2M1_PAIRS: "e2m1",
+               minw.VARIANT_TC_E2M1_N128: "e2m1"}
     all_tc = all(variants[i] in tc_kind for i in q_ops_idx)
     if all_tc:
         roofline = tensor_roofline([2.0 * macs[i] * BATCH for i in q_ops_idx],

@@ -145,8 +145,9 @@ MINW_API minw_status minw_pack_weights(const float *w, int32_t O, int32_t C, int
 enum {
     MINW_VARIANT_AUTO = 0,    /* per-shape choice from measurements: at creation a network times each
                                  layer the tensor cores cover with E4M3 operands, with E2M1 operands,
-                                 with E2M1 operands as CTA pairs of 128-channel tiles and on the
-                                 popcount path (bit-planes), and keeps the fastest (the times stay
+                                 with E2M1 operands as CTA pairs of 128-channel tiles or as single-CTA
+                                 128-channel tiles, and on the popcount path (bit-planes), and keeps
+                                 the fastest (the times stay
                                  readable through minw_net_layer_candidates); the popcount path
                                  where the tensor cores do not apply */
     MINW_VARIANT_POPC = 1,    /* bit-serial XNOR/AND + popcount on the integer pipe */
@@ -155,10 +156,14 @@ enum {
     MINW_VARIANT_TC_E4M3 = 3, /* tensor cores on E4M3 operands only (a network request) */
     MINW_VARIANT_TC_E2M1 = 4, /* tensor cores on E2M1 operands where the shape allows (a network
                                  request, as MINW_VARIANT_TC); reported for a layer on E2M1 operands */
-    MINW_VARIANT_TC_E2M1_PAIRS = 5  /* E2M1 operands as CTA pairs of 256 pixels x 128 channels where the
+    MINW_VARIANT_TC_E2M1_PAIRS = 5, /* E2M1 operands as CTA pairs of 256 pixels x 128 channels where the
                                  shape allows (output channels a multiple of 128, no K split): two
                                  accumulators per CTA, so each tile's epilogue overlaps the next
                                  tile's MMAs (a network request; reported for such a layer) */
+    MINW_VARIANT_TC_E2M1_N128 = 6  /* E2M1 operands on single CTAs with 128-channel tiles (layers with
+                                 more than 128 output channels and pixel-major tiles): two accumulators
+                                 per CTA at half the MMA width (a network request; reported for such a
+                                 layer) */
 };
 
 /* Convolution of packed activations act [B][H][W][bits_a][C/32] with packed
@@ -566,7 +571,8 @@ MINW_API minw_status minw_net_layer_times(minw_net *net, float *ms);
 
 /* Kernel chosen for each layer (host array of minw_net_launches() ints):
  * 0 for the fp32 first layer, else MINW_VARIANT_POPC, MINW_VARIANT_TC (E4M3
- * operands), MINW_VARIANT_TC_E2M1 or MINW_VARIANT_TC_E2M1_PAIRS. */
+ * operands), MINW_VARIANT_TC_E2M1, MINW_VARIANT_TC_E2M1_PAIRS or
+ * MINW_VARIANT_TC_E2M1_N128. */
 MINW_API minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants);
 
 /* The creation-time measurement behind layer `layer`'s kernel choice under
@@ -574,7 +580,8 @@ MINW_API minw_status minw_net_layer_variants(const minw_net *net, int32_t *varia
  * ms (host array of 4 floats) receives the least of three timed launches of
  * each candidate at the net's max_batch, in milliseconds, in the order E4M3
  * operands, E2M1 operands, E2M1 CTA pairs of 128-channel tiles, popcount on
- * bit-planes; -1 for a candidate the layer's shape does not allow, and -1 in
+ * bit-planes, E2M1 single-CTA 128-channel tiles (ms: host array of 5
+ * floats); -1 for a candidate the layer's shape does not allow, and -1 in
  * every entry for the first layer and for nets not created with
  * MINW_VARIANT_AUTO.  The kernel minw_net_layer_variants reports is the
  * fastest entry.  MINW_EINVAL for a null argument or a layer out of range,

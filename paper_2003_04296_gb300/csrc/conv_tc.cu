@@ -1796,6 +1796,13 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, bool encode = true) {
     p.nk = a.kh * a.kw * p.nck;
     p.nbb = (a.B + p.bb - 1) / p.bb;
     p.ntn = (a.O + p.BN - 1) / p.BN;
+    // E2M1 tiles of 128 channels on single CTAs (request n128): a 256-channel E2M1 tile holds one
+    // accumulator beside the scale factors, a 128-channel one two, so that each tile's epilogue
+    // overlaps the next tile's MMAs (at half the MMA width)
+    if (a.n128 && a.fp4 && !p.trans && !a.pair_n128 && p.BN > 128) {
+        p.BN = 128;
+        p.ntn = (a.O + 127) / 128;
+    }
     p.nlev = a.quant_out ? num_levels(a.qo.bits) : 0;
     p.thr = a.thr;
     // CTA pairs (MINW_TC_PAIR): 256-channel tiles of a layer that is not split along K
@@ -2034,6 +2041,16 @@ bool conv_tc_pairs128(const ConvArgs &a) {
     if (!conv_tc_supported(a)) return false;
     tc::Plan pl;
     return tc::make_plan(a, pl, false) == MINW_OK && pl.p.pair && pl.p.BN == 128;
+}
+
+bool conv_tc_n128(const ConvArgs &a) {
+    if (!conv_tc_supported(a) || !a.n128 || !a.fp4) return false;
+    ConvArgs b = a;
+    b.n128 = 0;
+    tc::Plan pl, pl0;
+    // a change of tiling only: the default plan has wider single-CTA tiles
+    return tc::make_plan(a, pl, false) == MINW_OK && tc::make_plan(b, pl0, false) == MINW_OK && !pl.p.pair &&
+           !pl.p.trans && pl.p.BN == 128 && pl0.p.BN > 128;
 }
 
 int conv_tc_launches(const ConvArgs &a) {

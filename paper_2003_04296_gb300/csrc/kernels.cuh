@@ -46,6 +46,8 @@ struct ConvArgs {
     void *workspace;       // nullable: no split
     size_t workspace_bytes;
     int ksplit;            // 0: chosen from the shape
+    int n128;              // E2M1: single-CTA tiles of 128 pixels x 128 channels (two accumulators fit the
+                           // tensor memory beside the scale factors)
     int pair_n128;         // E2M1: CTA pairs of 256 pixels x 128 channels (two accumulators fit the tensor
                            // memory beside the scale factors, so the epilogue overlaps the next MMAs)
 };
@@ -107,6 +109,8 @@ size_t conv_tc_min_split_bytes(const ConvArgs &a);
 int conv_tc_ksplit(const ConvArgs &a);
 // Whether the plan of this shape runs as CTA pairs of 128-channel E2M1 tiles (a.pair_n128 honoured).
 bool conv_tc_pairs128(const ConvArgs &a);
+// Whether a.n128 changes this shape's plan to single-CTA 128-channel E2M1 tiles.
+bool conv_tc_n128(const ConvArgs &a);
 // Kernels one tensor-core launch issues for this shape and workspace (2 with a split).
 int conv_tc_launches(const ConvArgs &a);
 minw_status launch_thresholds(const float *scale, const float *shift, int O, const QParams &q, float *out,

@@ -124,8 +124,8 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
             // candidates: E4M3 operands, E2M1 operands, E2M1 as CTA pairs of 128-channel tiles,
             // bit-planes on the popcount path (its input: the same bytes read as planes; its
             // output: planes, or the fp32 logits of the last layer)
-            float t[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-            for (int f = 0; f < 4 && st == MINW_OK; ++f) {
+            float t[5] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+            for (int f = 0; f < 5 && st == MINW_OK; ++f) {
                 if (f == 3) {
                     ConvArgs b = a;
                     b.thr = nullptr;
@@ -142,8 +142,12 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
                 ConvArgs b = a;
                 b.fp4 = f ? 1 : 0;
                 b.pair_n128 = f == 2 ? 1 : 0;
+                b.n128 = f == 4 ? 1 : 0;
                 b.codes_out4 = f && !last;
-                if (!conv_tc_supported(b) || (f == 2 && !conv_tc_pairs128(b))) { t[f] = 1e30f; continue; }
+                if (!conv_tc_supported(b) || (f == 2 && !conv_tc_pairs128(b)) || (f == 4 && !conv_tc_n128(b))) {
+                    t[f] = 1e30f;
+                    continue;
+                }
                 void *wq = f ? w4 : w8;
                 if (f < 2)
                     st = f ? minw_pack_weight_codes_e2m1(d.w, P.O, P.C, P.kh, P.kw, &P.qw, d.w_scale, (uint8_t *)wq, s)
@@ -164,12 +168,13 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
             }
             if (st != MINW_OK) break;
             int best = 0;
-            for (int f = 1; f < 4; ++f)
+            for (int f = 1; f < 5; ++f)
                 if (t[f] < t[best]) best = f;
-            for (int f = 0; f < 4; ++f) P.cand_ms[f] = t[f] < 1e29f ? t[f] : -1.0f;
+            for (int f = 0; f < 5; ++f) P.cand_ms[f] = t[f] < 1e29f ? t[f] : -1.0f;
             P.variant = best == 3 ? MINW_VARIANT_POPC : MINW_VARIANT_TC;
-            P.in4 = (best == 1 || best == 2) ? 1 : 0;
+            P.in4 = (best == 1 || best == 2 || best == 4) ? 1 : 0;
             P.pair128 = best == 2 ? 1 : 0;
+            P.n128 = best == 4 ? 1 : 0;
         }
     } while (false);
     cudaStreamSynchronize(s);
@@ -188,6 +193,7 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
         a.M = (long long)max_batch * P.Ho * P.Wo; a.pool = P.pool; a.quant_out = l + 1 < n_layers;
         a.fp4 = P.in4;
         a.pair_n128 = P.pair128;
+        a.n128 = P.n128;
         n->ws_bytes = std::max(n->ws_bytes, conv_tc_workspace_bytes(a));
     }
     return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
@@ -198,7 +204,7 @@ extern "C" {
 minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int32_t max_batch,
                             int32_t variant, void *stream, minw_net **out) {
     if (!layers || n_layers < 2 || max_batch <= 0 || !out) return MINW_EINVAL;
-    if (variant < 0 || variant > MINW_VARIANT_TC_E2M1_PAIRS) return MINW_EINVAL;
+    if (variant < 0 || variant > MINW_VARIANT_TC_E2M1_N128) return MINW_EINVAL;
     *out = nullptr;
     cudaStream_t s = (cudaStream_t)stream;
     minw_net *n = new minw_net();
@@ -215,7 +221,7 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
         // MINW_VARIANT_TC is a layer on E4M3 operands), else the network's
         const int req = d.variant != 0 ? (d.variant == MINW_VARIANT_TC ? MINW_VARIANT_TC_E4M3 : d.variant) : variant;
         if (!d.w || !d.scale || !d.shift || d.O <= 0 || d.C <= 0 || d.H <= 0 || d.W <= 0 || d.variant < 0 ||
-            d.variant > MINW_VARIANT_TC_E2M1_PAIRS) {
+            d.variant > MINW_VARIANT_TC_E2M1_N128) {
             net_free(n);
             return MINW_EINVAL;
         }
@@ -299,6 +305,11 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
                     a.pair_n128 = 1;
                     P.pair128 = conv_tc_pairs128(a) ? 1 : 0;
                     a.pair_n128 = P.pair128;
+                }
+                if (req == MINW_VARIANT_TC_E2M1_N128 && P.in4) {
+                    a.n128 = 1;
+                    P.n128 = conv_tc_n128(a) ? 1 : 0;
+                    a.n128 = P.n128;
                 }
             }
             if (P.variant == MINW_VARIANT_TC) {
@@ -421,6 +432,7 @@ static minw_status forward_enqueue(minw_net *net, const float *x, int32_t B, flo
             a.y_out = last ? logits : nullptr;
             a.fp4 = P.in4;
             a.pair_n128 = P.pair128;
+            a.n128 = P.n128;
             if (P.in_codes) {
                 a.act8 = (const uint8_t *)src;
                 a.wgt8 = P.wcodes;
@@ -521,7 +533,7 @@ minw_status minw_net_layer_candidates(const minw_net *net, int32_t layer, float 
     if (!net || !ms) return MINW_EINVAL;
     if (net->kind == 1) return MINW_EUNSUPPORTED;
     if (layer < 0 || layer >= (int32_t)net->L.size()) return MINW_EINVAL;
-    for (int f = 0; f < 4; ++f) ms[f] = net->L[layer].cand_ms[f];
+    for (int f = 0; f < 5; ++f) ms[f] = net->L[layer].cand_ms[f];
     return MINW_OK;
 }
 
@@ -533,6 +545,7 @@ minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants) {
     }
     for (size_t l = 0; l < net->L.size(); ++l)
         variants[l] = l == 0 ? 0
+                      : net->L[l].n128 ? MINW_VARIANT_TC_E2M1_N128
                       : net->L[l].pair128 ? MINW_VARIANT_TC_E2M1_PAIRS
                       : net->L[l].in4 ? MINW_VARIANT_TC_E2M1 : net->L[l].variant;
     return MINW_OK;
@@ -558,6 +571,7 @@ int32_t minw_net_kernels(const minw_net *net) {
         a.quant_out = l + 1 < net->L.size();
         if (a.quant_out) a.qo = to_qparams(&P.qo);
         a.act8 = P.wcodes; a.wgt8 = P.wcodes; a.thr = P.thr; a.fp4 = P.in4;
+        a.pair_n128 = P.pair128; a.n128 = P.n128;
         a.workspace = net->ws; a.workspace_bytes = net->ws_bytes;
         k += conv_tc_launches(a);
     }

@@ -20,8 +20,10 @@ struct LayerPlan {
     int in_codes = 0;              // input arrives in the codes layout
     int in4 = 0;                   // ... as E2M1 codes (two channels per byte; weights too)
     int pair128 = 0;               // E2M1 tensor-core layer as CTA pairs of 128-channel tiles (measured choice)
-    float cand_ms[4] = {-1.0f, -1.0f, -1.0f, -1.0f};   // creation-time times of the candidates (MINW_VARIANT_AUTO):
-                                   // E4M3, E2M1, E2M1 pairs, popcount; -1 where not a candidate
+    int n128 = 0;                  // E2M1 tensor-core layer on single-CTA 128-channel tiles (measured choice)
+    float cand_ms[5] = {-1.0f, -1.0f, -1.0f, -1.0f, -1.0f};   // creation-time times of the candidates
+                                   // (MINW_VARIANT_AUTO): E4M3, E2M1, E2M1 pairs, popcount, E2M1 128-channel
+                                   // tiles; -1 where not a candidate
     float *wlatent = nullptr;      // fp32 weights (first layer)
     float *wt = nullptr;           // first layer: weights prepared as [K][O] levels
     float *wscale = nullptr;       // per-channel weight prescale (first layer)

@@ -17,6 +17,7 @@ _LIB = None
 
 MINW_OK, MINW_EINVAL, MINW_EUNSUPPORTED, MINW_ECUDA, MINW_ETIMEOUT, MINW_EDEVICE = range(6)
 VARIANT_AUTO, VARIANT_POPC, VARIANT_TC, VARIANT_TC_E4M3, VARIANT_TC_E2M1, VARIANT_TC_E2M1_PAIRS = 0, 1, 2, 3, 4, 5
+VARIANT_TC_E2M1_N128 = 6
 CODES_E4M3, CODES_E2M1 = 0, 1
 LAYER_CONV, LAYER_FC = 0, 1
 
@@ -564,7 +565,7 @@ class Net:
 
     def layer_variants(self):
         """Kernel per layer: 0 fp32 first layer, VARIANT_POPC, VARIANT_TC (E4M3
-        operands), VARIANT_TC_E2M1 or VARIANT_TC_E2M1_PAIRS."""
+        operands), VARIANT_TC_E2M1, VARIANT_TC_E2M1_PAIRS or VARIANT_TC_E2M1_N128."""
         n = self.launches
         arr = (ctypes.c_int32 * n)()
         _check(lib().minw_net_layer_variants(self._h, arr), "minw_net_layer_variants")
@@ -572,8 +573,9 @@ class Net:
 
     def layer_candidates(self, layer):
         """Creation-time milliseconds of layer `layer`'s candidates under
-        VARIANT_AUTO: [E4M3, E2M1, E2M1 pairs, popcount], -1 where not one."""
-        arr = (ctypes.c_float * 4)()
+        VARIANT_AUTO: [E4M3, E2M1, E2M1 pairs, popcount, E2M1 128-channel
+        tiles], -1 where not one."""
+        arr = (ctypes.c_float * 5)()
         _check(lib().minw_net_layer_candidates(self._h, int(layer), arr), "minw_net_layer_candidates")
         return list(arr)
 

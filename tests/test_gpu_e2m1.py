@@ -301,10 +301,10 @@ def test_convnet_e2m1_layers(dev, M, bits_a, bits_w):
 
 
 def test_convnet_measured_formats(dev, M):
-    """VARIANT_AUTO times every tensor-core layer with E4M3 operands, E2M1
-    operands and E2M1 CTA pairs at creation and keeps the fastest: whatever it
-    picks, each layer reports one of the three, and the logits equal the
-    oracle's bit for bit."""
+    """VARIANT_AUTO times every layer with E4M3 operands, E2M1 operands, E2M1
+    CTA pairs, E2M1 single-CTA 128-channel tiles and the popcount path at
+    creation and keeps the fastest: whatever it picks, each layer reports one
+    of them, and the logits equal the oracle's bit for bit."""
     net_p = convnet_params(55, bits_a=1, bits_w=1, widths=(128, 128, 256, 256),
                            pools=(False, True, False, True), fcs=(256,), classes=10, hw=16)
     x = convnet_input(56, 9, hw=16)
@@ -314,7 +314,8 @@ def test_convnet_measured_formats(dev, M):
     torch.cuda.synchronize()
     var = net.layer_variants()
     net.close()
-    assert all(v in (M.VARIANT_TC, M.VARIANT_TC_E2M1, M.VARIANT_TC_E2M1_PAIRS) for v in var[1:])
+    assert all(v in (M.VARIANT_TC, M.VARIANT_TC_E2M1, M.VARIANT_TC_E2M1_PAIRS, M.VARIANT_TC_E2M1_N128,
+                     M.VARIANT_POPC) for v in var[1:])
     assert np.array_equal(logits.cpu().numpy(), N.convnet_forward(net_p, x))
     assert M.minw_get_last_device_error() == M.MINW_OK
 
@@ -337,4 +338,25 @@ def test_convnet_e2m1_pairs(dev, M, bits_a, bits_w, batch):
     net.close()
     assert M.minw_get_last_device_error() == M.MINW_OK
     assert M.VARIANT_TC_E2M1_PAIRS in list(var[1:])
+    assert np.array_equal(logits.cpu().numpy(), N.convnet_forward(net_p, x))
+
+
+@pytest.mark.parametrize("bits_a,bits_w", [(1, 1), (2, 2), (3, 3)])
+@pytest.mark.parametrize("batch", [7, 32])
+def test_convnet_e2m1_n128(dev, M, bits_a, bits_w, batch):
+    """E2M1 layers on single CTAs with 128-channel tiles (two accumulators per
+    CTA at half the MMA width) for every layer with more than 128 output
+    channels, pooled and unpooled, the fully connected layer included: the
+    logits equal the oracle's bit for bit, and those layers report the plan."""
+    net_p = convnet_params(59, bits_a=bits_a, bits_w=bits_w, widths=(128, 256, 256, 384),
+                           pools=(False, True, False, True), fcs=(256,), classes=10, hw=16)
+    x = convnet_input(60, batch, hw=16)
+    net = M.Net(M.layer_descs(net_p, dev), max_batch=batch, variant=M.VARIANT_TC_E2M1_N128)
+    logits = torch.empty((batch, net.out_features), dtype=torch.float32, device=dev)
+    net.forward(dev_tensor(x, dev), logits)
+    torch.cuda.synchronize()
+    var = net.layer_variants()
+    net.close()
+    assert M.minw_get_last_device_error() == M.MINW_OK
+    assert var[1:].count(M.VARIANT_TC_E2M1_N128) >= 3, var
     assert np.array_equal(logits.cpu().numpy(), N.convnet_forward(net_p, x))

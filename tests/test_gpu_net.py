@@ -103,8 +103,9 @@ def test_auto_choice_is_the_measured_fastest(dev, M, batch, bits):
     x = convnet_input(48, batch, hw=16)
     net = M.Net(M.layer_descs(net_p, dev), max_batch=batch, variant=M.VARIANT_AUTO)
     variants = net.layer_variants()
-    kind = {M.VARIANT_TC: 0, M.VARIANT_TC_E2M1: 1, M.VARIANT_TC_E2M1_PAIRS: 2, M.VARIANT_POPC: 3}
-    assert net.layer_candidates(0) == [-1.0] * 4
+    kind = {M.VARIANT_TC: 0, M.VARIANT_TC_E2M1: 1, M.VARIANT_TC_E2M1_PAIRS: 2, M.VARIANT_POPC: 3,
+            M.VARIANT_TC_E2M1_N128: 4}
+    assert net.layer_candidates(0) == [-1.0] * 5
     for layer in range(1, net.launches):
         ms = net.layer_candidates(layer)
         assert ms[0] > 0 and ms[3] > 0, (layer, ms)      # E4M3 and popcount cover every layer here
@@ -120,15 +121,15 @@ def test_auto_choice_is_the_measured_fastest(dev, M, batch, bits):
 
 def test_per_layer_requests_replay_a_plan(dev, M):
     """A per-layer kernel request (minw_layer_desc.variant) skips that layer's
-    measurement and runs the requested kernel: popcount, E4M3, E2M1 and E2M1
-    CTA pairs mixed in one net (each layer's input layout follows its
+    measurement and runs the requested kernel: popcount, E4M3, E2M1 CTA pairs
+    and E2M1 single-CTA 128-channel tiles mixed in one net (each layer's input layout follows its
     consumer), requested in the values minw_net_layer_variants reports
     (VARIANT_TC: E4M3 operands) and reported back unchanged, with the oracle's
     logits bit for bit."""
     net_p = convnet_params(49, bits_a=2, bits_w=1, widths=(128, 128, 256, 256),
                            pools=(False, True, False, True), fcs=(256,), classes=10, hw=16)
     x = convnet_input(50, 24, hw=16)
-    req = [0, M.VARIANT_POPC, M.VARIANT_TC, M.VARIANT_TC_E2M1_PAIRS, M.VARIANT_TC_E2M1, M.VARIANT_POPC]
+    req = [0, M.VARIANT_POPC, M.VARIANT_TC, M.VARIANT_TC_E2M1_PAIRS, M.VARIANT_TC_E2M1_N128, M.VARIANT_POPC]
     descs = M.layer_descs(net_p, dev)
     assert len(descs) == len(req)
     for d, v in zip(descs, req):
@@ -136,7 +137,7 @@ def test_per_layer_requests_replay_a_plan(dev, M):
     net = M.Net(descs, max_batch=24, variant=M.VARIANT_AUTO)
     assert net.layer_variants() == req
     for layer in range(net.launches):
-        assert net.layer_candidates(layer) == [-1.0] * 4        # nothing measured
+        assert net.layer_candidates(layer) == [-1.0] * 5        # nothing measured
     logits = torch.empty((24, net.out_features), dtype=torch.float32, device=dev)
     net.forward(dev_tensor(x, dev), logits)
     torch.cuda.synchronize()
