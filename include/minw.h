@@ -284,6 +284,20 @@ MINW_API minw_status minw_pack_weight_bf16(const float *w, int32_t O, int32_t C,
                                            const minw_quant *q, const float *channel_scale, uint16_t *out,
                                            void *stream);
 
+/* Narrow layers (channel counts that are not a multiple of 64, as in the
+ * 16- and 32-channel stages of ResNet-110 or the 12-channel growth of
+ * DenseNet-100, Table III): the same conversions with the channels padded to
+ * Cp >= C (the row length of the output), channels C .. Cp written as 0.  A
+ * zero activation or weight adds exactly 0 to every product, so
+ * minw_conv2d_bf16 run with C = Cp (a multiple of 64) on both padded
+ * operands gives the product of the unpadded ones.  Cp % 8 == 0 for the
+ * weights (MINW_EUNSUPPORTED otherwise); MINW_EINVAL for Cp < C. */
+MINW_API minw_status minw_to_bf16_nhwc_pad(const float *x, int32_t B, int32_t C, int32_t H, int32_t W, int32_t Cp,
+                                           uint16_t *out, void *stream);
+MINW_API minw_status minw_pack_weight_bf16_pad(const float *w, int32_t O, int32_t C, int32_t kh, int32_t kw,
+                                               int32_t Cp, const minw_quant *q, const float *channel_scale,
+                                               uint16_t *out, void *stream);
+
 /* Weight-only quantized convolution on the tcgen05 tensor cores (kind::f16,
  * bf16 x bf16 -> fp32 in TMEM): acc[b][o][y][x] = sum over (ky, kx, c) of
  * act * wgt with the accumulation order of the tensor core (not the oracle's),

@@ -406,9 +406,10 @@ __global__ void weight_codes_kernel(const float *__restrict__ w, int O, int C, i
 // Weights [O][C][kh][kw] -> bf16 level values in integer units [O][kh][kw][C]
 // (1, 2 or 4 for the 3-bit magnitudes, all exact in bf16): one thread per
 // 8 channels, one 128-bit store.
-__global__ void weight_bf16_kernel(const float *__restrict__ w, int O, int C, int kh, int kw, QParams q,
+// out [O][kh][kw][Cp]: channels C .. Cp hold 0 (Cp >= C, a multiple of 8).
+__global__ void weight_bf16_kernel(const float *__restrict__ w, int O, int C, int Cp, int kh, int kw, QParams q,
                                    const float *__restrict__ cscale, uint16_t *__restrict__ out) {
-    const int G = C >> 3;
+    const int G = Cp >> 3;
     const int taps = kh * kw;
     const int64_t total = (int64_t)O * taps * G;
     for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
@@ -420,12 +421,12 @@ __global__ void weight_bf16_kernel(const float *__restrict__ w, int O, int C, in
         uint32_t wd[4];
         for (int j = 0; j < 4; ++j) {
             const int c = g * 8 + 2 * j;
-            const float lo = (float)level_units(w[((int64_t)o * C + c) * taps + tap] * s, q);
-            const float hi = (float)level_units(w[((int64_t)o * C + c + 1) * taps + tap] * s, q);
+            const float lo = c < C ? (float)level_units(w[((int64_t)o * C + c) * taps + tap] * s, q) : 0.0f;
+            const float hi = c + 1 < C ? (float)level_units(w[((int64_t)o * C + c + 1) * taps + tap] * s, q) : 0.0f;
             wd[j] = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(lo)) |
                     ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(hi)) << 16);
         }
-        *reinterpret_cast<uint4 *>(out + ((int64_t)o * taps + tap) * C + g * 8) = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+        *reinterpret_cast<uint4 *>(out + ((int64_t)o * taps + tap) * Cp + g * 8) = make_uint4(wd[0], wd[1], wd[2], wd[3]);
     }
 }
 
@@ -433,7 +434,8 @@ __global__ void weight_bf16_kernel(const float *__restrict__ w, int O, int C, in
 // of a 32 x 32 (channel, pixel) tile transposed through shared memory.
 // Block (32, 8): a 32-channel x 32-pixel tile of one image through shared
 // memory; each thread's four loads issue before its first shared-memory store.
-__global__ void __launch_bounds__(256) to_bf16_nhwc_kernel(const float *__restrict__ x, int C, int HW,
+// out [B][HW][Cp]: channels C .. Cp hold 0 (Cp >= C).
+__global__ void __launch_bounds__(256) to_bf16_nhwc_kernel(const float *__restrict__ x, int C, int Cp, int HW,
                                                            uint16_t *__restrict__ out) {
     __shared__ float tile[32][33];
     const int b = blockIdx.z, c0 = blockIdx.y * 32, p0 = blockIdx.x * 32;
@@ -451,8 +453,8 @@ __global__ void __launch_bounds__(256) to_bf16_nhwc_kernel(const float *__restri
     for (int k = 0; k < 4; ++k) {
         const int i = threadIdx.y + 8 * k;
         const int p = p0 + i, c = c0 + threadIdx.x;
-        if (c < C && p < HW)
-            out[((int64_t)b * HW + p) * C + c] = __bfloat16_as_ushort(__float2bfloat16_rn(tile[threadIdx.x][i]));
+        if (c < Cp && p < HW)
+            out[((int64_t)b * HW + p) * Cp + c] = __bfloat16_as_ushort(__float2bfloat16_rn(tile[threadIdx.x][i]));
     }
 }
 
@@ -666,25 +668,36 @@ minw_status minw_pack_weight_codes_e2m1(const float *w, int32_t O, int32_t C, in
     return launch_status();
 }
 
+minw_status minw_pack_weight_bf16_pad(const float *w, int32_t O, int32_t C, int32_t kh, int32_t kw, int32_t Cp,
+                                      const minw_quant *q, const float *channel_scale, uint16_t *out, void *stream) {
+    if (O <= 0 || C <= 0 || kh <= 0 || kw <= 0 || Cp < C || !valid_quant(q) || !w || !out) return MINW_EINVAL;
+    if (Cp % 8 != 0 || !aligned16(out)) return MINW_EUNSUPPORTED;
+    const int64_t items = (int64_t)O * kh * kw * (Cp / 8);
+    const int64_t g = grid_for(items, 256);
+    weight_bf16_kernel<<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(w, O, C, Cp, kh, kw, to_qparams(q),
+                                                                     channel_scale, out);
+    return launch_status();
+}
+
 minw_status minw_pack_weight_bf16(const float *w, int32_t O, int32_t C, int32_t kh, int32_t kw,
                                   const minw_quant *q, const float *channel_scale, uint16_t *out, void *stream) {
-    if (O <= 0 || C <= 0 || kh <= 0 || kw <= 0 || !valid_quant(q) || !w || !out) return MINW_EINVAL;
-    if (C % 8 != 0 || !aligned16(out)) return MINW_EUNSUPPORTED;
-    const int64_t items = (int64_t)O * kh * kw * (C / 8);
-    const int64_t g = grid_for(items, 256);
-    weight_bf16_kernel<<<(unsigned)g, 256, 0, (cudaStream_t)stream>>>(w, O, C, kh, kw, to_qparams(q),
-                                                                     channel_scale, out);
+    if (C > 0 && C % 8 != 0) return MINW_EUNSUPPORTED;
+    return minw_pack_weight_bf16_pad(w, O, C, kh, kw, C, q, channel_scale, out, stream);
+}
+
+minw_status minw_to_bf16_nhwc_pad(const float *x, int32_t B, int32_t C, int32_t H, int32_t W, int32_t Cp,
+                                  uint16_t *out, void *stream) {
+    if (B <= 0 || C <= 0 || H <= 0 || W <= 0 || Cp < C || !x || !out) return MINW_EINVAL;
+    const int64_t HW = (int64_t)H * W;
+    if (HW > (1ll << 30) || B > 65535 || (Cp + 31) / 32 > 65535) return MINW_EUNSUPPORTED;
+    const dim3 grid((unsigned)((HW + 31) / 32), (unsigned)((Cp + 31) / 32), (unsigned)B);
+    to_bf16_nhwc_kernel<<<grid, dim3(32, 8), 0, (cudaStream_t)stream>>>(x, C, Cp, (int)HW, out);
     return launch_status();
 }
 
 minw_status minw_to_bf16_nhwc(const float *x, int32_t B, int32_t C, int32_t H, int32_t W, uint16_t *out,
                               void *stream) {
-    if (B <= 0 || C <= 0 || H <= 0 || W <= 0 || !x || !out) return MINW_EINVAL;
-    const int64_t HW = (int64_t)H * W;
-    if (HW > (1ll << 30) || B > 65535 || (C + 31) / 32 > 65535) return MINW_EUNSUPPORTED;
-    const dim3 grid((unsigned)((HW + 31) / 32), (unsigned)((C + 31) / 32), (unsigned)B);
-    to_bf16_nhwc_kernel<<<grid, dim3(32, 8), 0, (cudaStream_t)stream>>>(x, C, (int)HW, out);
-    return launch_status();
+    return minw_to_bf16_nhwc_pad(x, B, C, H, W, C, out, stream);
 }
 
 }  // extern "C"

@@ -144,9 +144,15 @@ static minw_status tune_formats(minw_net *n, const minw_layer_desc *layers, int 
                 b.pair_n128 = f == 2 ? 1 : 0;
                 b.n128 = f == 4 ? 1 : 0;
                 b.codes_out4 = f && !last;
-                if (!conv_tc_supported(b) || (f == 2 && !conv_tc_pairs128(b)) || (f == 4 && !conv_tc_n128(b))) {
-                    t[f] = 1e30f;
-                    continue;
+                if (!conv_tc_supported(b)) { t[f] = 1e30f; continue; }
+                // the tiling the layer would run with: at run time it gets the net's split workspace
+                // (a layer that splits along K runs no CTA pairs); planning only reads the size
+                {
+                    ConvArgs c = b;
+                    const size_t wsn = conv_tc_workspace_bytes(c);
+                    c.workspace = wsn ? reinterpret_cast<void *>(256) : nullptr;
+                    c.workspace_bytes = wsn;
+                    if ((f == 2 && !conv_tc_pairs128(c)) || (f == 4 && !conv_tc_n128(c))) { t[f] = 1e30f; continue; }
                 }
                 void *wq = f ? w4 : w8;
                 if (f < 2)
@@ -301,14 +307,20 @@ minw_status minw_net_create(const minw_layer_desc *layers, int32_t n_layers, int
                 a.fp4 = 1;
                 P.in4 = conv_tc_supported(a) ? 1 : 0;
                 a.fp4 = P.in4;
+                // requested tilings, planned with the split workspace the layer gets at run time
+                // (a layer that splits along K runs no CTA pairs)
+                ConvArgs c = a;
+                const size_t wsn = conv_tc_workspace_bytes(c);
+                c.workspace = wsn ? reinterpret_cast<void *>(256) : nullptr;
+                c.workspace_bytes = wsn;
                 if (req == MINW_VARIANT_TC_E2M1_PAIRS && P.in4) {
-                    a.pair_n128 = 1;
-                    P.pair128 = conv_tc_pairs128(a) ? 1 : 0;
+                    c.pair_n128 = 1;
+                    P.pair128 = conv_tc_pairs128(c) ? 1 : 0;
                     a.pair_n128 = P.pair128;
                 }
                 if (req == MINW_VARIANT_TC_E2M1_N128 && P.in4) {
-                    a.n128 = 1;
-                    P.n128 = conv_tc_n128(a) ? 1 : 0;
+                    c.n128 = 1;
+                    P.n128 = conv_tc_n128(c) ? 1 : 0;
                     a.n128 = P.n128;
                 }
             }

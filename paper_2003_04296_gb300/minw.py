@@ -88,6 +88,8 @@ SIGNATURES = {
     "aqe_backward": (ctypes.c_int, [_P, _P, _P, _I64, _F, _P]),
     "aqe_forward_stochastic": (ctypes.c_int, [_P, _P, _I64, _F, ctypes.c_uint64, ctypes.c_uint64, _P]),
     "minw_to_bf16_nhwc": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _P]),
+    "minw_to_bf16_nhwc_pad": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _P]),
+    "minw_pack_weight_bf16_pad": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
     "minw_pack_weight_bf16": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
     "minw_conv2d_bf16": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32, _I32, _I32,
                                         _I32, _P, _P, _P, _P]),
@@ -244,6 +246,20 @@ def minw_pack_weight_bf16(w, q, out, channel_scale=None, stream=None):
     O, C, kh, kw = w.shape
     _check(lib().minw_pack_weight_bf16(_ptr(w), O, C, kh, kw, ctypes.byref(q), _ptr(channel_scale), _ptr(out),
                                        _stream(stream)), "minw_pack_weight_bf16")
+
+
+def minw_to_bf16_nhwc_pad(x, Cp, out, stream=None):
+    """fp32 NCHW -> bf16 NHWC with the channels padded to Cp (zeros) (out [B][H][W][Cp])."""
+    B, C, H, W = x.shape
+    _check(lib().minw_to_bf16_nhwc_pad(_ptr(x), B, C, H, W, int(Cp), _ptr(out), _stream(stream)),
+           "minw_to_bf16_nhwc_pad")
+
+
+def minw_pack_weight_bf16_pad(w, Cp, q, out, channel_scale=None, stream=None):
+    """Latent weights [O][C][kh][kw] -> bf16 level values [O][kh][kw][Cp], channels past C zero."""
+    O, C, kh, kw = w.shape
+    _check(lib().minw_pack_weight_bf16_pad(_ptr(w), O, C, kh, kw, int(Cp), ctypes.byref(q), _ptr(channel_scale),
+                                           _ptr(out), _stream(stream)), "minw_pack_weight_bf16_pad")
 
 
 def minw_conv2d_bf16(act, B, C, H, W, wgt, O, kh, kw, bits_w, stride, pad, pool, scale, shift, y_out, stream=None):

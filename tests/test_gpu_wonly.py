@@ -164,3 +164,60 @@ def test_conv2d_bf16_errors(dev, M):
         M.minw_conv2d_bf16(xb, 1, 32, 4, 4, wb, 8, 3, 3, 1, 1, 1, 0, sc, sc, y)     # C % 64 != 0
     with pytest.raises(M.MinwError):
         M.minw_conv2d_bf16(xb, 1, 32, 4, 4, wb, 8, 3, 3, 1, 1, 1, 0, sc, sc, None)  # no output
+
+
+# Narrow layers of the Table III networks (3-bit weights, full-precision activations):
+# B, C, H, W, O, k, stride, pad
+NARROW = [
+    (4, 16, 32, 32, 16, 3, 1, 1),     # ResNet-110 stage 1 (16 channels at 32 x 32)
+    (4, 16, 32, 32, 32, 3, 2, 1),     # ResNet-110 entering stage 2 (stride 2)
+    (4, 16, 32, 32, 32, 1, 2, 0),     # its 1 x 1 / 2 shortcut
+    (4, 32, 16, 16, 32, 3, 1, 1),     # ResNet-110 stage 2
+    (4, 48, 32, 32, 48, 1, 1, 0),     # DenseNet-BC-100 bottleneck (24 + 2 x 12 channels in, 4 x 12 out)
+    (4, 48, 32, 32, 12, 3, 1, 1),     # DenseNet-BC-100 3 x 3, growth 12
+    (4, 96, 16, 16, 48, 1, 1, 0),     # DenseNet-BC-100 transition (compression 1/2)
+]
+
+
+@pytest.mark.parametrize("case", NARROW)
+def test_conv2d_bf16_narrow_channels(dev, M, case):
+    """Channel counts that are not a multiple of 64 run on zero-padded
+    operands (minw_to_bf16_nhwc_pad, minw_pack_weight_bf16_pad; a zero adds
+    exactly 0 to every product): the padded conversions bit for bit, and the
+    convolution of the padded operands within the fp32-accumulation bound of
+    the oracle's product of the unpadded ones, 3-bit weights."""
+    B, C, H, W, O_, k, s, pad = case
+    bits = 3
+    Cp = (C + 63) // 64 * 64
+    r = np.random.default_rng(sum(case) * 7 + 3)
+    x = r.standard_normal((B, C, H, W)).astype(np.float32)
+    w = r.normal(0, 0.05, (O_, C, k, k)).astype(np.float32)
+    cs = (1.0 / np.abs(w.reshape(O_, -1)).max(1)).astype(np.float32)
+    scale = r.normal(0.01, 0.005, O_).astype(np.float32)
+    shift = r.normal(0, 0.1, O_).astype(np.float32)
+    xb = torch.full((B, H, W, Cp), 0x7FFF, dtype=torch.int16, device=dev)       # stale contents: overwritten
+    wb = torch.full((O_, k, k, Cp), 0x7FFF, dtype=torch.int16, device=dev)
+    M.minw_to_bf16_nhwc_pad(dev_tensor(x, dev), Cp, xb)
+    M.minw_pack_weight_bf16_pad(dev_tensor(w, dev), Cp, M.quant(bits, DEFAULT_THR[bits]), wb,
+                                channel_scale=dev_tensor(cs, dev))
+    xr = O.bf16_round(x)
+    wu = O.quantize(w, bits, DEFAULT_THR[bits], cs) * 2.0 ** O.units_shift(bits)
+    xv, wv = _bf16_values(xb), _bf16_values(wb)
+    assert np.array_equal(xv[..., :C].view(np.uint32), xr.transpose(0, 2, 3, 1).view(np.uint32))
+    assert not xv[..., C:].view(np.uint32).any()
+    assert np.array_equal(wv[..., :C].astype(np.float64), wu.transpose(0, 2, 3, 1))
+    assert not wv[..., C:].view(np.uint32).any()
+    Ho, Wo = (H + 2 * pad - k) // s + 1, (W + 2 * pad - k) // s + 1
+    y = torch.full((B, O_, Ho, Wo), np.nan, dtype=torch.float32, device=dev)
+    M.minw_conv2d_bf16(xb, B, Cp, H, W, wb, O_, k, k, bits, s, pad, 0, dev_tensor(scale, dev),
+                       dev_tensor(shift, dev), y)
+    torch.cuda.synchronize()
+    xr64 = xr.astype(np.float64)
+    acc = O.conv2d_real(xr64, wu, s, pad)
+    A = O.conv2d_real(np.abs(xr64), np.abs(wu), s, pad)
+    sc = scale.astype(np.float64)[None, :, None, None]
+    yref = acc * sc + shift.astype(np.float64)[None, :, None, None]
+    K = Cp * k * k
+    bound = np.abs(sc) * K * 2.0 ** -23 * A + 2.0 ** -23 * np.abs(yref) + 1e-30
+    err = np.abs(y.cpu().numpy().astype(np.float64) - yref)
+    assert (err <= bound).all(), f"worst err/bound {np.max(err / bound)}"
