@@ -116,6 +116,10 @@ class Workload:
             self.params = I.convnet_params(self.seed, bits_a=args.bits_a, bits_w=args.bits_w,
                                            **I.CIFAR_MODELS[self.model])
             self.bits = (args.bits_a, args.bits_w)
+        elif name == "wresnet110":
+            self.batch, self.seed = 128, 6
+            self.params = I.wresnet_params(self.seed, n=18, bits_w=3, classes=10, hw=32)
+            self.bits = (0, 3)
         else:
             self.batch, self.seed = 128, 4
             self.params = I.resnet18_params(self.seed, bits_a=args.bits_a_resnet, bits_w=args.bits_w_resnet)
@@ -125,6 +129,8 @@ class Workload:
         from paper_2003_04296_gb300 import inputs as I
         if self.name == "cifar_convnet":
             return I.convnet_input(self.seed + 1000 * rank, self.batch)
+        if self.name == "wresnet110":
+            return I.wresnet_input(self.seed + 1000 * rank, self.batch)
         return I.resnet18_input(self.seed + 1000 * rank, self.batch)
 
     def net(self, minw, dev, variant, layer_variants=None):
@@ -136,12 +142,16 @@ class Workload:
                 for d, v in zip(descs, layer_variants):
                     d["variant"] = int(v)
             return minw.Net(descs, max_batch=self.batch, variant=variant)
+        if self.name == "wresnet110":
+            return minw.Net.wresnet(self.params, self.batch, dev)
         return minw.Net.resnet18(self.params, self.batch, dev)
 
     def oracle(self, x):
         from oracle import network as N
         if self.name == "cifar_convnet":
             return N.convnet_forward(self.params, x)
+        if self.name == "wresnet110":
+            return N.wresnet_forward(self.params, x)
         return N.resnet18_forward(self.params, x)
 
     def op_macs(self):
@@ -150,6 +160,23 @@ class Workload:
         if self.name == "cifar_convnet":
             m = layer_macs(self.params)
             return m, list(range(1, len(m)))
+        if self.name == "wresnet110":
+            # ops: stem, its pass; per block conv1, pass, [shortcut], conv2, pass; head (unpadded MACs)
+            hw = self.params["hw"]
+            macs, q = [hw * hw * 16 * 27, 0], []
+            size, c_in = hw, 16
+            for blk in self.params["blocks"]:
+                o = blk["c1"]["w"].shape[0]
+                so = size // blk["stride"]
+                q.append(len(macs)); macs.append(so * so * o * c_in * 9)
+                macs.append(0)
+                if blk["down"] is not None:
+                    q.append(len(macs)); macs.append(so * so * o * c_in)
+                q.append(len(macs)); macs.append(so * so * o * o * 9)
+                macs.append(0)
+                size, c_in = so, o
+            macs.append(64 * self.params["classes"])
+            return macs, q
         hw = self.params["hw"]
         s = hw // 2
         macs = [s * s * 64 * 3 * 49, 0]
@@ -179,6 +206,13 @@ class Workload:
                     "global_batch": self.batch * n_gpus, "input": "3x32x32 fp32 U(-1,1)",
                     "layers": layers,
                     "bits_a": ba, "bits_w": bw, "first_layer": "fp32 input, quantized weights",
+                    "parallelism": par, "l2": L2_NOTE}
+        if self.name == "wresnet110":
+            return {"workload": "wresnet110_cifar_fwd_w3", "batch_per_gpu": self.batch,
+                    "global_batch": self.batch * n_gpus, "input": "3x32x32 fp32 U(-1,1)",
+                    "layers": "stem 3x3 16 (fp32 weights); 3 x 18 basic blocks 16-32-64 (3-bit weights, bf16 "
+                              "activations, 1x1/2 shortcuts entering stages 2-3); avgpool; fc 10 (fp32)",
+                    "bits_a": "full precision (bf16 into each convolution)", "bits_w": bw,
                     "parallelism": par, "l2": L2_NOTE}
         return {"workload": f"resnet18_fwd_a{ba}w{bw}", "batch_per_gpu": self.batch,
                 "global_batch": self.batch * n_gpus, "input": "3x224x224 fp32 N(0,1)",
@@ -535,8 +569,17 @@ def run_gpu(args, rank, world, local_rank):
     achieved = q_ops / (q_ms * 1e-3) / 1e12
     tc_kind = {minw.VARIANT_TC: "e4m3", minw.VARIANT_TC_E2M1: "e2m1", minw.VARIANT_TC_E2M1_PAIRS: "e2m1",
                minw.VARIANT_TC_E2M1_N128: "e2m1"}
+    if wl.name == "wresnet110":
+        tc_kind = {minw.VARIANT_TC: "bf16"}
     all_tc = all(variants[i] in tc_kind for i in q_ops_idx)
-    if all_tc:
+    if wl.name == "wresnet110":
+        roofline = {"bound": "tensor", "kernel": "conv_tc_kernel<0, *, bf16> (tcgen05 kind::f16, the 110 block "
+                                                 "and shortcut convolutions)",
+                    "achieved": achieved, "peak": BF16_TFLOPS, "unit": "TFLOP/s", "frac": achieved / BF16_TFLOPS,
+                    "traffic": None, "layer_kinds": ["bf16"] * len(q_ops_idx),
+                    "peak_basis": "measured dense bf16 TFLOP/s (burst), of measured; achieved counts the unpadded "
+                                  "MACs (16- and 32-channel layers run on operands padded to 64 channels)"}
+    elif all_tc:
         roofline = tensor_roofline([2.0 * macs[i] * BATCH for i in q_ops_idx],
                                    [tc_kind[variants[i]] for i in q_ops_idx],
                                    [float(layer_ms[i]) for i in q_ops_idx])
@@ -1377,8 +1420,8 @@ def main():
                          "sampler sees several samples under load)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["minw", "reference"], default="minw")
-    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "sweep", "fc_train", "conv_train", "conv1",
-                                           "peaks"],
+    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "wresnet110", "sweep", "fc_train",
+                                           "conv_train", "conv1", "peaks"],
                     default="cifar_convnet")
     ap.add_argument("--bits-a", type=int, default=1, help="CIFAR ConvNet activation bits")
     ap.add_argument("--bits-w", type=int, default=1, help="CIFAR ConvNet weight bits")
@@ -1397,7 +1440,8 @@ def main():
     args = ap.parse_args()
     default_run = args.steps is None and args.workload == "cifar_convnet"
     if args.steps is None:
-        args.steps = {"cifar_convnet": 4000, "resnet18": 400, "sweep": 100, "fc_train": 2000, "conv_train": 500,
+        args.steps = {"cifar_convnet": 4000, "resnet18": 400, "wresnet110": 500, "sweep": 100, "fc_train": 2000,
+                      "conv_train": 500,
                       "conv1": 1000, "peaks": 1}[args.workload]
 
     world = int(os.environ.get("WORLD_SIZE", "1"))

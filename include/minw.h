@@ -634,6 +634,59 @@ typedef struct {
 MINW_API minw_status minw_resnet18_create(const minw_resnet18_desc *desc, int32_t max_batch,
                                           void *stream, minw_net **out);
 
+/* The weight-only MINW-Net residual network of Table III (3-bit weights,
+ * full-precision activations; ResNet-110 for n = 18): a CIFAR ResNet-(6n+2)
+ * whose block convolutions multiply bf16 activations by N-bit weight levels
+ * on the tensor cores (the SHIFT ADDER layers of Sec. IV, as
+ * minw_conv2d_bf16), with fp32 first and last layers (Sec. III-E).  The
+ * paper leaves the block wiring open; the reading implemented here:
+ *   stem: fp32 3x3 conv 3 -> 16 (fp32 weights, pad 1; one fmaf chain per
+ *         output over (c, ky, kx)) -> BN -> HardTanh;
+ *   block (3 stages of n blocks, 16, 32 and 64 channels, stride 2 entering
+ *         stages 2 and 3): h = HardTanh(BN1(conv1(x))),
+ *         out = HardTanh(BN2(conv2(h)) + s) with s = x, or s = BN_d(conv_d(x))
+ *         for the 1x1 / 2 shortcut entering stages 2 and 3 (one fp32 add);
+ *         each convolution reads the bf16 rounding of its fp32 input;
+ *   head: global average pool (one fp32 sum in pixel order, one division) ->
+ *         fp32 fully connected layer [classes][64] -> BN -> fp32 logits.
+ * Block b (0 .. 3n - 1, stage b / n) has c1_*[b] [O][C][3][3] and
+ * c2_*[b] [O][O][3][3]; down_*[i] is the shortcut entering stage i + 2
+ * [O][C][1][1]; *_wscale: per-output-channel weight prescale (nullable);
+ * every block weight is quantized with (bits_w, thr_w) to levels in integer
+ * units.  The 16- and 32-channel layers run on operands padded to 64
+ * channels.  image_hw: a multiple of 4 (32 for CIFAR).  Device pointers, read
+ * during creation only.  minw_forward takes x [B][3][hw][hw] and writes
+ * logits [B][num_classes].  Errors: MINW_EINVAL (arguments, n outside
+ * 1 .. MINW_WRESNET_MAX_N), MINW_EUNSUPPORTED (sizes past the 32-bit index
+ * range), MINW_ECUDA. */
+#define MINW_WRESNET_MAX_N 18
+typedef struct {
+    int32_t n;
+    int32_t bits_w;
+    float thr_w[3];
+    int32_t image_hw, num_classes;
+    const float *stem_w, *stem_scale, *stem_shift;
+    const float *c1_w[3 * MINW_WRESNET_MAX_N], *c1_wscale[3 * MINW_WRESNET_MAX_N];
+    const float *c1_scale[3 * MINW_WRESNET_MAX_N], *c1_shift[3 * MINW_WRESNET_MAX_N];
+    const float *c2_w[3 * MINW_WRESNET_MAX_N], *c2_wscale[3 * MINW_WRESNET_MAX_N];
+    const float *c2_scale[3 * MINW_WRESNET_MAX_N], *c2_shift[3 * MINW_WRESNET_MAX_N];
+    const float *down_w[2], *down_wscale[2], *down_scale[2], *down_shift[2];
+    const float *fc_w, *fc_scale, *fc_shift;
+    int32_t keep_activations;   /* nonzero: keep every block's fp32 output for minw_wresnet_activation */
+} minw_wresnet_desc;
+
+MINW_API minw_status minw_wresnet_create(const minw_wresnet_desc *desc, int32_t max_batch, void *stream,
+                                         minw_net **out);
+
+/* Introspection of a net created with keep_activations (no counterpart in
+ * the paper): copies the fp32 NCHW output of stage-step `index` of the most
+ * recent forward -- 0 the stem's HardTanh output [B][16][hw][hw], b + 1 block
+ * b's output -- into dst (device memory of at least count floats), on stream.
+ * MINW_EINVAL for a net without kept activations, an index out of range or a
+ * short dst. */
+MINW_API minw_status minw_wresnet_activation(const minw_net *net, int32_t index, float *dst, size_t count,
+                                             void *stream);
+
 /* Number of layers (and of entries minw_net_layer_times fills). */
 MINW_API int32_t minw_net_launches(const minw_net *net);
 

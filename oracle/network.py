@@ -107,3 +107,58 @@ def resnet18_forward(net, x, keep=False):
     fc = net["fc"]
     logits = O.affine(O.linear_f32_seq(pooled, fc["w"]), fc["scale"], fc["shift"])
     return (logits, trace) if keep else logits
+
+
+def _wlevels(conv, bits_w, thr_w):
+    """A weight-only layer's weights: the levels of h in integer units
+    (quarters for 3-bit), exact in bf16."""
+    return O.quantize(conv["w"], bits_w, thr_w, conv["w_scale"]) * 2.0 ** O.units_shift(bits_w)
+
+
+def wconv(conv, a, stride, bits_w, thr_w):
+    """One weight-only convolution with its BN (the SHIFT ADDER layer of
+    Sec. IV): the fp32 activation rounded to bf16 (the layer's 16-bit input),
+    the product with the weight levels summed in fp64 and rounded to fp32,
+    then the BN map (fmaf).  Returns the fp32 BN output."""
+    k = conv["w"].shape[2]
+    ab = O.bf16_round(a).astype(np.float64)
+    acc = O.conv2d_real(ab, _wlevels(conv, bits_w, thr_w), stride, k // 2)
+    return O.affine(acc.astype(np.float32), conv["scale"], conv["shift"])
+
+
+def wresnet_block(blk, a, bits_w, thr_w):
+    """One block of the weight-only residual network: h = HardTanh(BN1(conv1(a))),
+    out = HardTanh(BN2(conv2(h)) + s), s = a or BN_d(conv_d(a)) (one fp32 add).
+    Returns (h, out)."""
+    h = O.hardtanh(wconv(blk["c1"], a, blk["stride"], bits_w, thr_w))
+    y2 = wconv(blk["c2"], h, 1, bits_w, thr_w)
+    s = a if blk["down"] is None else wconv(blk["down"], a, 2, bits_w, thr_w)
+    return h, O.hardtanh((y2 + s).astype(np.float32))
+
+
+def wresnet_head(net, a):
+    """Global average pool (one fp32 sum in pixel order, one division), the
+    fp32 fully connected layer (one fmaf chain) and its BN: the logits."""
+    fc = net["fc"]
+    return O.affine(O.linear_f32_seq(O.avgpool_f32(a), fc["w"]), fc["scale"], fc["shift"])
+
+
+def wresnet_forward(net, x, keep=False):
+    """Forward pass of the weight-only residual network of Table III built by
+    ``inputs.wresnet_params`` (a CIFAR ResNet-(6n+2), ResNet-110 for n = 18).
+    The paper leaves the wiring open; the reading followed:
+      stem : fp32 3x3 conv (fp32 weights, one fmaf chain per output) -> BN
+             -> HardTanh
+      block: wresnet_block; the stage entries (stride 2) take a 1x1 / 2
+             shortcut with quantized weights
+      head : wresnet_head.
+    With ``keep`` also returns every block's output (after the stem first)."""
+    bw, tw = net["bits_w"], net["thr_w"]
+    st = net["stem"]
+    a = O.hardtanh(O.affine(O.conv2d_f32_seq(x, st["w"], 1, 1), st["scale"], st["shift"]))
+    trace = [a]
+    for blk in net["blocks"]:
+        _, a = wresnet_block(blk, a, bw, tw)
+        trace.append(a)
+    logits = wresnet_head(net, a)
+    return (logits, trace) if keep else logits

@@ -24,6 +24,7 @@ using namespace minw_host;
 static void net_free(minw_net *n) {
     if (!n) return;
     if (n->res) resnet_free(n);
+    if (n->wres) wresnet_free(n);
     for (void *p : n->owned) cudaFree(p);
     for (cudaEvent_t e : n->events) cudaEventDestroy(e);
     if (n->gexec) cudaGraphExecDestroy(n->gexec);
@@ -402,6 +403,7 @@ static bool graphs_enabled() { return minw_host::plan_options().graph != 0; }
 
 static minw_status forward_enqueue(minw_net *net, const float *x, int32_t B, float *logits, cudaStream_t cs) {
     if (net->kind == 1) return resnet_forward(net, x, B, logits, cs);
+    if (net->kind == 2) return wresnet_forward(net, x, B, logits, cs);
     const int nl = (int)net->L.size();
     int cur = 0;
     if (net->timing && cudaEventRecord(net->events[0], cs) != cudaSuccess) return MINW_ECUDA;
@@ -543,7 +545,7 @@ minw_status minw_net_layer_times(minw_net *net, float *ms) {
 
 minw_status minw_net_layer_candidates(const minw_net *net, int32_t layer, float *ms) {
     if (!net || !ms) return MINW_EINVAL;
-    if (net->kind == 1) return MINW_EUNSUPPORTED;
+    if (net->kind != 0) return MINW_EUNSUPPORTED;
     if (layer < 0 || layer >= (int32_t)net->L.size()) return MINW_EINVAL;
     for (int f = 0; f < 5; ++f) ms[f] = net->L[layer].cand_ms[f];
     return MINW_OK;
@@ -553,6 +555,10 @@ minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants) {
     if (!net || !variants) return MINW_EINVAL;
     if (net->kind == 1) {
         resnet_variants(net, variants);     // stem, pool, the block convolutions, head
+        return MINW_OK;
+    }
+    if (net->kind == 2) {
+        wresnet_variants(net, variants);    // stem, its pass, per block conv1, pass, [shortcut], conv2, pass; head
         return MINW_OK;
     }
     for (size_t l = 0; l < net->L.size(); ++l)
@@ -565,13 +571,14 @@ minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants) {
 
 int32_t minw_net_launches(const minw_net *net) {
     if (!net) return 0;
-    return net->kind == 1 ? resnet_ops(net) : (int32_t)net->L.size();
+    return net->kind == 1 ? resnet_ops(net) : net->kind == 2 ? wresnet_ops(net) : (int32_t)net->L.size();
 }
 
 // Kernels one minw_forward issues (a split-K layer issues two).
 int32_t minw_net_kernels(const minw_net *net) {
     if (!net) return 0;
     if (net->kind == 1) return resnet_kernels(net);
+    if (net->kind == 2) return wresnet_kernels(net);
     int32_t k = 0;
     for (size_t l = 0; l < net->L.size(); ++l) {
         const LayerPlan &P = net->L[l];

@@ -34,10 +34,13 @@ struct LayerPlan {
 };
 
 struct ResNetPlan;   // resnet.cu
+struct WResPlan;     // wresnet.cu
 
 struct minw_net {
-    int kind = 0;                     // 0: sequential (minw_net_create), 1: residual (minw_resnet18_create)
+    int kind = 0;                     // 0: sequential (minw_net_create), 1: residual (minw_resnet18_create),
+                                      // 2: weight-only residual (minw_wresnet_create)
     ResNetPlan *res = nullptr;
+    WResPlan *wres = nullptr;
     std::vector<LayerPlan> L;
     int max_batch = 0;
     uint32_t *buf[2] = {nullptr, nullptr};
@@ -65,3 +68,10 @@ int32_t resnet_ops(const minw_net *net);
 void resnet_variants(const minw_net *net, int32_t *variants);
 int32_t resnet_kernels(const minw_net *net);
 void resnet_free(minw_net *net);
+
+// The weight-only residual network (wresnet.cu).
+minw_status wresnet_forward(minw_net *net, const float *x, int B, float *logits, cudaStream_t s);
+int32_t wresnet_ops(const minw_net *net);
+void wresnet_variants(const minw_net *net, int32_t *variants);
+int32_t wresnet_kernels(const minw_net *net);
+void wresnet_free(minw_net *net);

@@ -218,6 +218,56 @@ def resnet18_params(seed, bits_a=3, bits_w=3, classes=1000, hw=224, w_sigma=0.02
     return out
 
 
+# Second moment of a HardTanh output of a unit-variance input (the activations
+# the weight-only blocks consume); used only to size the synthetic BN maps.
+_HARDTANH_MS = 0.6
+
+
+def wresnet_params(seed, n=18, bits_w=3, classes=10, hw=32, w_sigma=0.05):
+    """Weight-only MINW-Net residual network of Table III (CIFAR ResNet-(6n+2),
+    ResNet-110 for n = 18): an fp32 3x3 stem 3 -> 16 (fp32 weights), three
+    stages of n basic blocks with 16, 32 and 64 channels (stride 2 and a 1x1
+    shortcut entering stages 2 and 3) whose weights are quantized to N-bit
+    levels while the activations stay full precision, and an fp32 classifier.
+    Latent weights ~ N(0, w_sigma); synthetic BN maps sized from the input and
+    level second moments (the block convolutions' outputs are in level
+    units)."""
+    r = rng(seed)
+    out = dict(n=n, bits_w=bits_w, thr_w=DEFAULT_THR[bits_w], classes=classes, hw=hw)
+    sw = f32(r.normal(0.0, w_sigma, (16, 3, 3, 3)))
+    g, b_ = r.normal(1.0, 0.1, 16), r.normal(0.0, 0.1, 16)
+    var = 27 * _LEVEL_MS[0] * w_sigma ** 2         # images U(-1, 1), fp32 weights
+    out["stem"] = dict(w=sw, scale=f32(g / np.sqrt(var + 1e-5)), shift=f32(b_))
+    unit2 = 4.0 ** _units(bits_w)
+
+    def wconv(o, c, k):
+        w = f32(r.normal(0.0, w_sigma, (o, c, k, k)))
+        ws = weight_prescale(w, bits_w)
+        gg, bb = r.normal(1.0, 0.1, o), r.normal(0.0, 0.1, o)
+        v = c * k * k * _HARDTANH_MS * weight_ms(w, ws, bits_w) * unit2
+        return dict(w=w, w_scale=ws, scale=f32(gg / np.sqrt(v + 1e-5)), shift=f32(bb), k=k)
+
+    blocks = []
+    c_in = 16
+    for stage, width in enumerate((16, 32, 64)):
+        for j in range(n):
+            stride = 2 if (stage > 0 and j == 0) else 1
+            blocks.append(dict(stride=stride, c1=wconv(width, c_in, 3), c2=wconv(width, width, 3),
+                               down=wconv(width, c_in, 1) if stride == 2 else None))
+            c_in = width
+    out["blocks"] = blocks
+    fw = f32(r.normal(0.0, w_sigma, (classes, 64)))
+    g, b_ = r.normal(1.0, 0.1, classes), r.normal(0.0, 0.1, classes)
+    var = 64 * _HARDTANH_MS * w_sigma ** 2
+    out["fc"] = dict(w=fw, scale=f32(g / np.sqrt(var + 1e-5)), shift=f32(b_))
+    return out
+
+
+def wresnet_input(seed, B, hw=32):
+    """CIFAR-shaped synthetic images, U(-1, 1)."""
+    return f32(rng(seed).uniform(-1.0, 1.0, (B, 3, hw, hw)))
+
+
 def resnet18_input(seed, B, hw=224):
     """ImageNet-shaped synthetic images, N(0, 1)."""
     return f32(rng(seed).standard_normal((B, 3, hw, hw)))

@@ -67,6 +67,24 @@ class LayerDesc(ctypes.Structure):
                 ("scale", ctypes.c_void_p), ("shift", ctypes.c_void_p), ("variant", ctypes.c_int32)]
 
 
+WRESNET_MAX_N = 18
+_NB = 3 * WRESNET_MAX_N
+
+
+class WResNetDesc(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int32), ("bits_w", ctypes.c_int32), ("thr_w", ctypes.c_float * 3),
+                ("image_hw", ctypes.c_int32), ("num_classes", ctypes.c_int32),
+                ("stem_w", ctypes.c_void_p), ("stem_scale", ctypes.c_void_p), ("stem_shift", ctypes.c_void_p),
+                ("c1_w", ctypes.c_void_p * _NB), ("c1_wscale", ctypes.c_void_p * _NB),
+                ("c1_scale", ctypes.c_void_p * _NB), ("c1_shift", ctypes.c_void_p * _NB),
+                ("c2_w", ctypes.c_void_p * _NB), ("c2_wscale", ctypes.c_void_p * _NB),
+                ("c2_scale", ctypes.c_void_p * _NB), ("c2_shift", ctypes.c_void_p * _NB),
+                ("down_w", ctypes.c_void_p * 2), ("down_wscale", ctypes.c_void_p * 2),
+                ("down_scale", ctypes.c_void_p * 2), ("down_shift", ctypes.c_void_p * 2),
+                ("fc_w", ctypes.c_void_p), ("fc_scale", ctypes.c_void_p), ("fc_shift", ctypes.c_void_p),
+                ("keep_activations", ctypes.c_int32)]
+
+
 class ResNet18Desc(ctypes.Structure):
     _fields_ = [("bits_a", ctypes.c_int32), ("bits_w", ctypes.c_int32), ("thr_a", ctypes.c_float * 3),
                 ("thr_w", ctypes.c_float * 3), ("image_hw", ctypes.c_int32), ("num_classes", ctypes.c_int32),
@@ -135,6 +153,9 @@ SIGNATURES = {
                                        ctypes.POINTER(ctypes.c_void_p)]),
     "minw_resnet18_create": (ctypes.c_int, [ctypes.POINTER(ResNet18Desc), _I32, _P,
                                             ctypes.POINTER(ctypes.c_void_p)]),
+    "minw_wresnet_create": (ctypes.c_int, [ctypes.POINTER(WResNetDesc), _I32, _P,
+                                           ctypes.POINTER(ctypes.c_void_p)]),
+    "minw_wresnet_activation": (ctypes.c_int, [_P, _I32, _P, ctypes.c_size_t, _P]),
     "minw_forward": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
     "minw_forward_host": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
     "minw_net_enable_timing": (ctypes.c_int, [_P, _I32]),
@@ -493,6 +514,54 @@ class Net:
 
     ``layers`` is a list of dicts with the minw_layer_desc fields; ``w``,
     ``w_scale``, ``scale`` and ``shift`` are device tensors."""
+
+    @classmethod
+    def wresnet(cls, params, max_batch, device, stream=None, keep_activations=False):
+        """minw_wresnet_create from a parameter dict shaped like
+        ``inputs.wresnet_params`` (latent fp32 weights, BN maps); the tensors
+        are copied to ``device`` for the call and released after it."""
+        d = WResNetDesc()
+        d.keep_activations = int(bool(keep_activations))
+        d.n, d.bits_w = params["n"], params["bits_w"]
+        for i in range(3):
+            d.thr_w[i] = float(params["thr_w"][i])
+        d.image_hw, d.num_classes = params["hw"], params["classes"]
+        keep = []
+
+        def dev(a):
+            t = torch.from_numpy(a).to(device).contiguous()
+            keep.append(t)
+            return t.data_ptr()
+        st = params["stem"]
+        d.stem_w, d.stem_scale, d.stem_shift = dev(st["w"]), dev(st["scale"]), dev(st["shift"])
+        nd = 0
+        for b, blk in enumerate(params["blocks"]):
+            c1, c2 = blk["c1"], blk["c2"]
+            d.c1_w[b], d.c1_wscale[b], d.c1_scale[b], d.c1_shift[b] = (dev(c1["w"]), dev(c1["w_scale"]),
+                                                                      dev(c1["scale"]), dev(c1["shift"]))
+            d.c2_w[b], d.c2_wscale[b], d.c2_scale[b], d.c2_shift[b] = (dev(c2["w"]), dev(c2["w_scale"]),
+                                                                      dev(c2["scale"]), dev(c2["shift"]))
+            if blk["down"] is not None:
+                c = blk["down"]
+                d.down_w[nd], d.down_wscale[nd] = dev(c["w"]), dev(c["w_scale"])
+                d.down_scale[nd], d.down_shift[nd] = dev(c["scale"]), dev(c["shift"])
+                nd += 1
+        fc = params["fc"]
+        d.fc_w, d.fc_scale, d.fc_shift = dev(fc["w"]), dev(fc["scale"]), dev(fc["shift"])
+        h = ctypes.c_void_p()
+        _check(lib().minw_wresnet_create(ctypes.byref(d), int(max_batch), _stream(stream), ctypes.byref(h)),
+               "minw_wresnet_create")
+        net = cls.__new__(cls)
+        net._h = h
+        net.max_batch = max_batch
+        net.out_features = params["classes"]
+        return net
+
+    def wresnet_activation(self, index, out, stream=None):
+        """minw_wresnet_activation: the fp32 output of stage-step `index` of
+        the most recent forward (0 the stem, b + 1 block b) into `out`."""
+        _check(lib().minw_wresnet_activation(self._h, int(index), _ptr(out), out.numel(), _stream(stream)),
+               "minw_wresnet_activation")
 
     @classmethod
     def resnet18(cls, params, max_batch, device, stream=None):
