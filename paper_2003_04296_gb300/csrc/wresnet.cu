@@ -34,9 +34,10 @@ namespace {
 
 // v = HardTanh(y + s) (s nullable: v = HardTanh(y)) over NCHW fp32 [B][C][HW]
 // (the fp32 operations of the oracle: one add, then the two clamps), written
-// as fp32 NCHW to z (nullable) and as bf16 NHWC [B][HW][Cp] to zb, channels
-// C .. Cp zero.  Block (32, 8): 32 channels x 32 pixels of one image through
-// shared memory; each thread's loads issue before its first store.
+// as fp32 NCHW to z (nullable) and as bf16 NHWC [B][HW][Cp] to zb (channels
+// C .. Cp are not written: the buffers hold zeros there from creation on).
+// Block (32, 8): 32 channels x 32 pixels of one image through shared memory;
+// each thread's loads issue before its first store.
 __global__ void __launch_bounds__(256) wres_post_kernel(const float *__restrict__ y, const float *__restrict__ s,
                                                         int C, int Cp, int HW, float *__restrict__ z,
                                                         uint16_t *__restrict__ zb) {
@@ -69,7 +70,7 @@ __global__ void __launch_bounds__(256) wres_post_kernel(const float *__restrict_
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
         const int p = p0 + threadIdx.y + 8 * k, c = c0 + threadIdx.x;
-        if (c < Cp && p < HW)
+        if (c < C && p < HW)
             zb[((int64_t)b * HW + p) * Cp + c] =
                 __bfloat16_as_ushort(__float2bfloat16_rn(tile[threadIdx.x][threadIdx.y + 8 * k]));
     }
@@ -140,8 +141,10 @@ struct WResPlan {
     std::vector<WBlock> blocks;
     float *fc_wt = nullptr, *fc_scale = nullptr, *fc_shift = nullptr;
     float *A[2] = {nullptr, nullptr};      // fp32 NCHW block activations (ping-pong)
-    uint16_t *AB[2] = {nullptr, nullptr};  // the same as padded bf16 NHWC
-    uint16_t *HB = nullptr;                // HardTanh(BN1(conv1)) as padded bf16 NHWC
+    // padded bf16 NHWC inputs of the convolutions, per stage (the channels past a stage's
+    // count stay zero from creation on): block outputs (ping-pong) and HardTanh(BN1(conv1))
+    uint16_t *AB[3][2] = {{nullptr, nullptr}, {nullptr, nullptr}, {nullptr, nullptr}};
+    uint16_t *HB[3] = {nullptr, nullptr, nullptr};
     float *Y1 = nullptr, *Y2 = nullptr, *S = nullptr;   // fp32 NCHW convolution outputs
     float *pooled = nullptr;
     std::vector<float *> keep;             // with keep_activations: the stem's and every block's fp32 output
@@ -167,7 +170,7 @@ static minw_status wcopy(minw_net *n, float **dst, const float *src, size_t coun
 
 static minw_status post(const float *y, const float *s, int B, int C, int HW, float *z, uint16_t *zb, cudaStream_t st) {
     const int Cp = pad64(C);
-    const dim3 grid((unsigned)((HW + 31) / 32), (unsigned)((Cp + 31) / 32), (unsigned)B);
+    const dim3 grid((unsigned)((HW + 31) / 32), (unsigned)((C + 31) / 32), (unsigned)B);
     wres_post_kernel<<<grid, dim3(32, 8), 0, st>>>(y, s, C, Cp, HW, z, zb);
     return cudaGetLastError() == cudaSuccess ? MINW_OK : MINW_ECUDA;
 }
@@ -232,31 +235,35 @@ minw_status wresnet_forward(minw_net *net, const float *x, int B, float *logits,
         if ((st = launch_conv_first(a, s)) != MINW_OK) return st;
         if ((st = mark()) != MINW_OK) return st;
         float *a0 = R->keep.empty() ? R->A[0] : R->keep[0];
-        if ((st = post(R->Y1, nullptr, B, 16, hw * hw, a0, R->AB[0], s)) != MINW_OK) return st;
+        if ((st = post(R->Y1, nullptr, B, 16, hw * hw, a0, R->AB[0][1], s)) != MINW_OK) return st;
         if ((st = mark()) != MINW_OK) return st;
     }
     int cur = 0, bi = 0;
     const float *acur = R->keep.empty() ? R->A[0] : R->keep[0];    // this block's fp32 input (its identity shortcut)
+    const uint16_t *xin = R->AB[0][1];                               // ... and its bf16 input
     for (const WBlock &bk : R->blocks) {
         float *anext = R->keep.empty() ? R->A[cur ^ 1] : R->keep[bi + 1];
+        const int stg = bi / R->n, j = bi - stg * R->n;
+        uint16_t *xout = R->AB[stg][j & 1];
         const int HWo = bk.c1.Ho * bk.c1.Wo;
-        if ((st = wconv(bk.c1, R->AB[cur], B, R->Y1, s, R->bits_w)) != MINW_OK) return st;
+        if ((st = wconv(bk.c1, xin, B, R->Y1, s, R->bits_w)) != MINW_OK) return st;
         if ((st = mark()) != MINW_OK) return st;
-        if ((st = post(R->Y1, nullptr, B, bk.c1.O, HWo, nullptr, R->HB, s)) != MINW_OK) return st;
+        if ((st = post(R->Y1, nullptr, B, bk.c1.O, HWo, nullptr, R->HB[stg], s)) != MINW_OK) return st;
         if ((st = mark()) != MINW_OK) return st;
         const float *sc = acur;
         if (bk.down) {
-            if ((st = wconv(bk.d, R->AB[cur], B, R->S, s, R->bits_w)) != MINW_OK) return st;
+            if ((st = wconv(bk.d, xin, B, R->S, s, R->bits_w)) != MINW_OK) return st;
             if ((st = mark()) != MINW_OK) return st;
             sc = R->S;
         }
-        if ((st = wconv(bk.c2, R->HB, B, R->Y2, s, R->bits_w)) != MINW_OK) return st;
+        if ((st = wconv(bk.c2, R->HB[stg], B, R->Y2, s, R->bits_w)) != MINW_OK) return st;
         if ((st = mark()) != MINW_OK) return st;
-        if ((st = post(R->Y2, sc, B, bk.c2.O, HWo, anext, R->AB[cur ^ 1], s)) != MINW_OK) return st;
+        if ((st = post(R->Y2, sc, B, bk.c2.O, HWo, anext, xout, s)) != MINW_OK) return st;
         if ((st = mark()) != MINW_OK) return st;
         cur ^= 1;
         ++bi;
         acur = anext;
+        xin = xout;
     }
     R->keep_B = B;
     {
@@ -363,11 +370,18 @@ extern "C" minw_status minw_wresnet_create(const minw_wresnet_desc *d, int32_t m
     }
     // activations: the stage-1 sizes are the largest (16 channels, 64 padded, at hw x hw)
     const size_t px = (size_t)max_batch * d->image_hw * d->image_hw;
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < 2; ++i)
         if ((st = walloc(n, &R->A[i], px * 16)) != MINW_OK) return fail(st);
-        if ((st = walloc(n, &R->AB[i], px * 64)) != MINW_OK) return fail(st);
+    for (int stg = 0; stg < 3; ++stg) {
+        const size_t e = px / ((size_t)1 << (2 * stg)) * 64;      // the stage's pixels x 64 padded channels
+        for (int i = 0; i < 3; ++i) {
+            uint16_t *b = nullptr;
+            if ((st = walloc(n, &b, e)) != MINW_OK) return fail(st);
+            if (cudaMemsetAsync(b, 0, e * sizeof(uint16_t), s) != cudaSuccess) return fail(MINW_ECUDA);
+            if (i < 2) R->AB[stg][i] = b; else R->HB[stg] = b;
+        }
     }
-    if ((st = walloc(n, &R->HB, px * 64)) != MINW_OK || (st = walloc(n, &R->Y1, px * 16)) != MINW_OK ||
+    if ((st = walloc(n, &R->Y1, px * 16)) != MINW_OK ||
         (st = walloc(n, &R->Y2, px * 16)) != MINW_OK || (st = walloc(n, &R->S, px * 16)) != MINW_OK)
         return fail(st);
     if (d->keep_activations) {
