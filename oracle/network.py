@@ -162,3 +162,57 @@ def wresnet_forward(net, x, keep=False):
         trace.append(a)
     logits = wresnet_head(net, a)
     return (logits, trace) if keep else logits
+
+
+def avgpool2_f32(t):
+    """2x2 / 2 average pool of fp32 [B][C][H][W]: ((t00 + t01) + t10) + t11 in
+    fp32, then times 1/4 (exact)."""
+    t = np.asarray(t, dtype=np.float32)
+    s = (t[:, :, 0::2, 0::2] + t[:, :, 0::2, 1::2]).astype(np.float32)
+    s = (s + t[:, :, 1::2, 0::2]).astype(np.float32)
+    s = (s + t[:, :, 1::2, 1::2]).astype(np.float32)
+    return (s * np.float32(0.25)).astype(np.float32)
+
+
+def wdense_layer(lay, F, bits_w, thr_w):
+    """One bottleneck layer of the weight-only DenseNet: h = HardTanh(BN(conv
+    1x1(F))), n = HardTanh(BN(conv 3x3(h))); returns (h, bf16(n)), the new
+    features in the 16-bit form the block holds them in."""
+    h = O.hardtanh(wconv(lay["b"], F, 1, bits_w, thr_w))
+    n = O.hardtanh(wconv(lay["c"], h, 1, bits_w, thr_w))
+    return h, O.bf16_round(n)
+
+
+def wdense_transition(conv, F, bits_w, thr_w):
+    """Transition: bf16(avgpool 2x2(HardTanh(BN(conv 1x1(F)))))."""
+    t = O.hardtanh(wconv(conv, F, 1, bits_w, thr_w))
+    return O.bf16_round(avgpool2_f32(t))
+
+
+def wdense_forward(net, x, keep=False):
+    """Forward pass of the weight-only DenseNet-BC of Table III built by
+    ``inputs.wdense_params`` (DenseNet-100 for 16 layers per block, growth
+    12).  The paper gives no wiring beyond DenseNet's; the reading followed
+    (the block order of Sec. III-E, conv -> BN -> HardTanh, in place of
+    DenseNet's pre-activation):
+      stem : fp32 3x3 conv (fp32 weights) -> BN -> HardTanh
+      block: features F, held as bf16 (the form every convolution reads); each
+             layer appends wdense_layer's growth channels
+      trans: wdense_transition (channels halved, 2x2 average pool)
+      head : global average pool of the last F (one fp32 sum in pixel order,
+             one division) -> fp32 FC -> BN.
+    With ``keep`` also returns each block's final features (bf16 values)."""
+    bw, tw = net["bits_w"], net["thr_w"]
+    st = net["stem"]
+    F = O.bf16_round(O.hardtanh(O.affine(O.conv2d_f32_seq(x, st["w"], 1, 1), st["scale"], st["shift"])))
+    finals = []
+    for bi, lay_list in enumerate(net["blocks"]):
+        for lay in lay_list:
+            _, nb = wdense_layer(lay, F, bw, tw)
+            F = np.concatenate([F, nb], axis=1)
+        finals.append(F)
+        if bi < len(net["trans"]):
+            F = wdense_transition(net["trans"][bi], F, bw, tw)
+    fc = net["fc"]
+    logits = O.affine(O.linear_f32_seq(O.avgpool_f32(F), fc["w"]), fc["scale"], fc["shift"])
+    return (logits, finals) if keep else logits

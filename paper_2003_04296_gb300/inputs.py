@@ -268,6 +268,51 @@ def wresnet_input(seed, B, hw=32):
     return f32(rng(seed).uniform(-1.0, 1.0, (B, 3, hw, hw)))
 
 
+def wdense_params(seed, layers=16, growth=12, bits_w=3, classes=10, hw=32, w_sigma=0.05):
+    """Weight-only MINW-Net DenseNet-BC of Table III (DenseNet-100 for
+    layers = 16, growth 12): an fp32 3x3 stem 3 -> 2 growth (fp32 weights),
+    three dense blocks of ``layers`` bottleneck layers (1x1 conv to 4 growth
+    channels, then 3x3 conv to growth channels, each with its BN and
+    HardTanh, concatenated onto the block's features), transitions with
+    compression 1/2 (1x1 conv, BN, HardTanh, 2x2 average pool), and an fp32
+    classifier.  Latent weights ~ N(0, w_sigma); BN maps as wresnet_params."""
+    r = rng(seed)
+    k = growth
+    out = dict(layers=layers, growth=k, bits_w=bits_w, thr_w=DEFAULT_THR[bits_w], classes=classes, hw=hw)
+    c0 = 2 * k
+    sw = f32(r.normal(0.0, w_sigma, (c0, 3, 3, 3)))
+    g, b_ = r.normal(1.0, 0.1, c0), r.normal(0.0, 0.1, c0)
+    var = 27 * _LEVEL_MS[0] * w_sigma ** 2
+    out["stem"] = dict(w=sw, scale=f32(g / np.sqrt(var + 1e-5)), shift=f32(b_))
+    unit2 = 4.0 ** _units(bits_w)
+
+    def wconv(o, c, kk):
+        w = f32(r.normal(0.0, w_sigma, (o, c, kk, kk)))
+        ws = weight_prescale(w, bits_w)
+        gg, bb = r.normal(1.0, 0.1, o), r.normal(0.0, 0.1, o)
+        v = c * kk * kk * _HARDTANH_MS * weight_ms(w, ws, bits_w) * unit2
+        return dict(w=w, w_scale=ws, scale=f32(gg / np.sqrt(v + 1e-5)), shift=f32(bb), k=kk)
+
+    blocks, trans = [], []
+    c = c0
+    for blk in range(3):
+        lay = []
+        for _ in range(layers):
+            lay.append(dict(b=wconv(4 * k, c, 1), c=wconv(k, 4 * k, 3)))
+            c += k
+        blocks.append(lay)
+        if blk < 2:
+            trans.append(wconv(c // 2, c, 1))
+            c //= 2
+    out["blocks"], out["trans"] = blocks, trans
+    fw = f32(r.normal(0.0, w_sigma, (classes, c)))
+    g, b_ = r.normal(1.0, 0.1, classes), r.normal(0.0, 0.1, classes)
+    var = c * _HARDTANH_MS * w_sigma ** 2
+    out["fc"] = dict(w=fw, scale=f32(g / np.sqrt(var + 1e-5)), shift=f32(b_))
+    out["features"] = c
+    return out
+
+
 def resnet18_input(seed, B, hw=224):
     """ImageNet-shaped synthetic images, N(0, 1)."""
     return f32(rng(seed).standard_normal((B, 3, hw, hw)))
