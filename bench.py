@@ -120,6 +120,10 @@ class Workload:
             self.batch, self.seed = 128, 6
             self.params = I.wresnet_params(self.seed, n=18, bits_w=3, classes=10, hw=32)
             self.bits = (0, 3)
+        elif name == "wdense100":
+            self.batch, self.seed = 128, 7
+            self.params = I.wdense_params(self.seed, layers=16, growth=12, bits_w=3, classes=10, hw=32)
+            self.bits = (0, 3)
         else:
             self.batch, self.seed = 128, 4
             self.params = I.resnet18_params(self.seed, bits_a=args.bits_a_resnet, bits_w=args.bits_w_resnet)
@@ -129,7 +133,7 @@ class Workload:
         from paper_2003_04296_gb300 import inputs as I
         if self.name == "cifar_convnet":
             return I.convnet_input(self.seed + 1000 * rank, self.batch)
-        if self.name == "wresnet110":
+        if self.name in ("wresnet110", "wdense100"):
             return I.wresnet_input(self.seed + 1000 * rank, self.batch)
         return I.resnet18_input(self.seed + 1000 * rank, self.batch)
 
@@ -144,6 +148,8 @@ class Workload:
             return minw.Net(descs, max_batch=self.batch, variant=variant)
         if self.name == "wresnet110":
             return minw.Net.wresnet(self.params, self.batch, dev)
+        if self.name == "wdense100":
+            return minw.Net.wdense(self.params, self.batch, dev)
         return minw.Net.resnet18(self.params, self.batch, dev)
 
     def oracle(self, x):
@@ -152,6 +158,8 @@ class Workload:
             return N.convnet_forward(self.params, x)
         if self.name == "wresnet110":
             return N.wresnet_forward(self.params, x)
+        if self.name == "wdense100":
+            return N.wdense_forward(self.params, x)
         return N.resnet18_forward(self.params, x)
 
     def op_macs(self):
@@ -161,7 +169,7 @@ class Workload:
             m = layer_macs(self.params)
             return m, list(range(1, len(m)))
         if self.name == "wresnet110":
-            # ops: stem, its pass; per block conv1, pass, [shortcut], conv2, pass; head (unpadded MACs)
+            # ops: stem, its pass; per block conv1 (HardTanh fused), [shortcut], conv2, pass; head (unpadded MACs)
             hw = self.params["hw"]
             macs, q = [hw * hw * 16 * 27, 0], []
             size, c_in = hw, 16
@@ -169,13 +177,28 @@ class Workload:
                 o = blk["c1"]["w"].shape[0]
                 so = size // blk["stride"]
                 q.append(len(macs)); macs.append(so * so * o * c_in * 9)
-                macs.append(0)
                 if blk["down"] is not None:
                     q.append(len(macs)); macs.append(so * so * o * c_in)
                 q.append(len(macs)); macs.append(so * so * o * o * 9)
                 macs.append(0)
                 size, c_in = so, o
             macs.append(64 * self.params["classes"])
+            return macs, q
+        if self.name == "wdense100":
+            # ops: stem, its pass; per layer 1x1, 3x3 (HardTanh fused in both); per transition conv, pool; head
+            P = self.params
+            hw, k = P["hw"], P["growth"]
+            macs, q = [hw * hw * 2 * k * 27, 0], []
+            for b, lay_list in enumerate(P["blocks"]):
+                px = (hw >> b) ** 2
+                for lay in lay_list:
+                    c = lay["b"]["w"].shape[1]
+                    q.append(len(macs)); macs.append(px * 4 * k * c)
+                    q.append(len(macs)); macs.append(px * k * 4 * k * 9)
+                if b < 2:
+                    t = P["trans"][b]["w"]
+                    q.append(len(macs)); macs += [px * t.shape[0] * t.shape[1], 0]
+            macs.append(P["features"] * P["classes"])
             return macs, q
         hw = self.params["hw"]
         s = hw // 2
@@ -212,6 +235,14 @@ class Workload:
                     "global_batch": self.batch * n_gpus, "input": "3x32x32 fp32 U(-1,1)",
                     "layers": "stem 3x3 16 (fp32 weights); 3 x 18 basic blocks 16-32-64 (3-bit weights, bf16 "
                               "activations, 1x1/2 shortcuts entering stages 2-3); avgpool; fc 10 (fp32)",
+                    "bits_a": "full precision (bf16 into each convolution)", "bits_w": bw,
+                    "parallelism": par, "l2": L2_NOTE}
+        if self.name == "wdense100":
+            return {"workload": "densenet100_bc_k12_cifar_fwd_w3", "batch_per_gpu": self.batch,
+                    "global_batch": self.batch * n_gpus, "input": "3x32x32 fp32 U(-1,1)",
+                    "layers": "stem 3x3 24 (fp32 weights); 3 dense blocks x 16 bottleneck layers (1x1 to 48, 3x3 "
+                              "to 12; 3-bit weights, bf16 activations) 24-216 / 108-300 / 150-342 channels; "
+                              "transitions 1x1 + 2x2 avgpool (compression 1/2); avgpool; fc 10 (fp32)",
                     "bits_a": "full precision (bf16 into each convolution)", "bits_w": bw,
                     "parallelism": par, "l2": L2_NOTE}
         return {"workload": f"resnet18_fwd_a{ba}w{bw}", "batch_per_gpu": self.batch,
@@ -569,7 +600,7 @@ def run_gpu(args, rank, world, local_rank):
     achieved = q_ops / (q_ms * 1e-3) / 1e12
     tc_kind = {minw.VARIANT_TC: "e4m3", minw.VARIANT_TC_E2M1: "e2m1", minw.VARIANT_TC_E2M1_PAIRS: "e2m1",
                minw.VARIANT_TC_E2M1_N128: "e2m1"}
-    if wl.name == "wresnet110":
+    if wl.name in ("wresnet110", "wdense100"):
         tc_kind = {minw.VARIANT_TC: "bf16"}
     all_tc = all(variants[i] in tc_kind for i in q_ops_idx)
     if wl.name == "wresnet110":
@@ -579,6 +610,14 @@ def run_gpu(args, rank, world, local_rank):
                     "traffic": None, "layer_kinds": ["bf16"] * len(q_ops_idx),
                     "peak_basis": "measured dense bf16 TFLOP/s (burst), of measured; achieved counts the unpadded "
                                   "MACs (16- and 32-channel layers run on operands padded to 64 channels)"}
+    elif wl.name == "wdense100":
+        roofline = {"bound": "tensor", "kernel": "conv_tc_kernel<0, *, bf16> (tcgen05 kind::f16, the 96 "
+                                                 "bottleneck-layer and 2 transition convolutions)",
+                    "achieved": achieved, "peak": BF16_TFLOPS, "unit": "TFLOP/s", "frac": achieved / BF16_TFLOPS,
+                    "traffic": None, "layer_kinds": ["bf16"] * len(q_ops_idx),
+                    "peak_basis": "measured dense bf16 TFLOP/s (burst), of measured; achieved counts the unpadded "
+                                  "MACs (each 1x1 reads its channels padded to a multiple of 64, the 3x3 its 48 "
+                                  "padded to 64, and the 3x3 computes 12 output channels of a 16-wide MMA)"}
     elif all_tc:
         roofline = tensor_roofline([2.0 * macs[i] * BATCH for i in q_ops_idx],
                                    [tc_kind[variants[i]] for i in q_ops_idx],
@@ -1381,16 +1420,19 @@ def run_peaks(args, rank, world, local_rank):
 
 
 def other_configs(args, rank, world, local_rank):
-    """The default run's summary of the other BASELINE workloads (each with
+    """The default run's summary of the other benchmark workloads (each with
     fewer steps than its own run, no CPU baseline): the single convolution,
-    the ConvNet at 2-bit activations with 1- and 2-bit weights, ResNet-18 and
-    the bit-width sweep."""
+    the ConvNet at 2-bit activations with 1- and 2-bit weights, ResNet-18, the
+    weight-only ResNet-110 and DenseNet-100 of Table III, and the bit-width
+    sweep."""
     import copy
     out = {}
     jobs = [("conv1", run_conv1, dict(workload="conv1", steps=3000)),
             ("cifar_convnet_a2w1", run_gpu, dict(workload="cifar_convnet", bits_a=2, bits_w=1, steps=1500)),
             ("cifar_convnet_a2w2", run_gpu, dict(workload="cifar_convnet", bits_a=2, bits_w=2, steps=1500)),
             ("resnet18_a3w3", run_gpu, dict(workload="resnet18", steps=200)),
+            ("wresnet110_w3", run_gpu, dict(workload="wresnet110", steps=200)),
+            ("densenet100_w3", run_gpu, dict(workload="wdense100", steps=100)),
             ("sweep", run_sweep, dict(workload="sweep", steps=40))]
     for name, fn, ch in jobs:
         a = copy.copy(args)
@@ -1420,8 +1462,8 @@ def main():
                          "sampler sees several samples under load)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["minw", "reference"], default="minw")
-    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "wresnet110", "sweep", "fc_train",
-                                           "conv_train", "conv1", "peaks"],
+    ap.add_argument("--workload", choices=["cifar_convnet", "resnet18", "wresnet110", "wdense100", "sweep",
+                                           "fc_train", "conv_train", "conv1", "peaks"],
                     default="cifar_convnet")
     ap.add_argument("--bits-a", type=int, default=1, help="CIFAR ConvNet activation bits")
     ap.add_argument("--bits-w", type=int, default=1, help="CIFAR ConvNet weight bits")
@@ -1436,11 +1478,12 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--no-configs", action="store_true",
-                    help="default run: skip the summary of the other BASELINE configs")
+                    help="default run: skip the summary of the other benchmark workloads")
     args = ap.parse_args()
     default_run = args.steps is None and args.workload == "cifar_convnet"
     if args.steps is None:
-        args.steps = {"cifar_convnet": 4000, "resnet18": 400, "wresnet110": 500, "sweep": 100, "fc_train": 2000,
+        args.steps = {"cifar_convnet": 4000, "resnet18": 400, "wresnet110": 500, "wdense100": 300, "sweep": 100,
+                      "fc_train": 2000,
                       "conv_train": 500,
                       "conv1": 1000, "peaks": 1}[args.workload]
 

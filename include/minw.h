@@ -312,6 +312,22 @@ MINW_API minw_status minw_conv2d_bf16(const uint16_t *act, int32_t B, int32_t C,
                                       int32_t stride, int32_t pad, int32_t pool, const float *scale,
                                       const float *shift, float *y_out, void *stream);
 
+/* The same convolution (no pool) with the next layer's input as its output:
+ * out[pixel][out_off + o] = bf16(HardTanh(fmaf(acc, scale[o], shift[o])))
+ * (the fp32 clamps to [-1, 1], one round-to-nearest-even), bf16 NHWC rows of
+ * out_ld elements per output pixel; the other elements of each row are not
+ * written (a DenseNet block appends its new channels to its feature buffer
+ * this way).  act: bf16 NHWC rows of ldc elements per pixel (0: C), of which
+ * the first C are read (ldc a multiple of 64, at least C).  The accumulators
+ * are those minw_conv2d_bf16 forms for the same operands, so out equals the
+ * bf16 rounding of HardTanh of its y_out.  Errors: MINW_EINVAL (arguments,
+ * out_ld < out_off + O), MINW_EUNSUPPORTED (shape, as minw_conv2d_bf16). */
+MINW_API minw_status minw_conv2d_bf16_hardtanh(const uint16_t *act, int32_t B, int32_t C, int32_t H, int32_t W,
+                                               int32_t ldc, const uint16_t *wgt, int32_t O, int32_t kh, int32_t kw,
+                                               int32_t bits_w, int32_t stride, int32_t pad, const float *scale,
+                                               const float *shift, uint16_t *out, int32_t out_ld, int32_t out_off,
+                                               void *stream);
+
 /* ---------------------------------------------------------------------- */
 /* Training step of a fully connected layer (Algorithm 1)                  */
 /* ---------------------------------------------------------------------- */
@@ -686,6 +702,69 @@ MINW_API minw_status minw_wresnet_create(const minw_wresnet_desc *desc, int32_t 
  * short dst. */
 MINW_API minw_status minw_wresnet_activation(const minw_net *net, int32_t index, float *dst, size_t count,
                                              void *stream);
+
+/* The weight-only MINW-Net DenseNet-BC of Table III (DenseNet-100 for
+ * layers = 16, growth k = 12, 3-bit weights): N-bit weights times
+ * full-precision (bf16) activations on the tensor cores for every layer
+ * inside the network, fp32 first and last layers (Sec. III-E).  The paper
+ * gives no wiring beyond DenseNet's; the reading implemented here keeps the
+ * block order conv -> BN -> HardTanh of Sec. III-E:
+ *   stem : fp32 3x3 conv 3 -> 2k (fp32 weights, pad 1, one fmaf chain per
+ *          output over (c, ky, kx)) -> BN -> HardTanh; the block's features
+ *          F start as its bf16 rounding;
+ *   layer: h = HardTanh(BN(conv 1x1 (F) to 4k channels)),
+ *          n = HardTanh(BN(conv 3x3 pad 1 (bf16(h)) to k channels)),
+ *          F <- concat(F, bf16(n)) along channels;
+ *   trans: between blocks, F <- bf16(avgpool 2x2(HardTanh(BN(conv 1x1 (F)
+ *          to floor(c / 2) channels)))), the pool ((v00 + v01) + v10) + v11
+ *          in fp32, times 1/4;
+ *   head : global average pool of the last F (one fp32 sum in pixel order,
+ *          one division) -> fp32 fully connected layer -> BN -> logits.
+ * Three blocks of `layers` layers; block b starts with c_b channels (c_0 =
+ * 2k) and its layer i reads c_b + i k.  Layer j = b * layers + i has b_*[j]
+ * [4k][c_b + i k][1][1] and c_*[j] [k][4k][3][3]; t_*[b] [c / 2][c][1][1] is
+ * the transition after block b (c its final channels); fc_w [classes][c]
+ * for the last block's c.  *_wscale: per-output-channel weight prescale
+ * (nullable); every convolution after the stem is quantized with (bits_w,
+ * thr_w) to levels in integer units.  Each block's features live in one bf16
+ * NHWC buffer of pad64(final c) channels per pixel that the layers append
+ * to in place (no concatenation copies); each 1x1 convolution reads the
+ * first pad64(c) channels of its rows (zero weights past c).  image_hw: a
+ * multiple of 4, at least 8.  Device pointers, read during creation only.
+ * minw_forward takes x [B][3][hw][hw] and writes logits [B][num_classes].
+ * Errors: MINW_EINVAL (arguments; layers outside 1 .. MINW_WDENSE_MAX_LAYERS,
+ * growth outside 1 .. 64), MINW_EUNSUPPORTED (sizes past the 32-bit index
+ * range, more than 1536 final channels), MINW_ECUDA. */
+#define MINW_WDENSE_MAX_LAYERS 32
+typedef struct {
+    int32_t layers, growth;
+    int32_t bits_w;
+    float thr_w[3];
+    int32_t image_hw, num_classes;
+    const float *stem_w, *stem_scale, *stem_shift;
+    const float *b_w[3 * MINW_WDENSE_MAX_LAYERS], *b_wscale[3 * MINW_WDENSE_MAX_LAYERS];
+    const float *b_scale[3 * MINW_WDENSE_MAX_LAYERS], *b_shift[3 * MINW_WDENSE_MAX_LAYERS];
+    const float *c_w[3 * MINW_WDENSE_MAX_LAYERS], *c_wscale[3 * MINW_WDENSE_MAX_LAYERS];
+    const float *c_scale[3 * MINW_WDENSE_MAX_LAYERS], *c_shift[3 * MINW_WDENSE_MAX_LAYERS];
+    const float *t_w[2], *t_wscale[2], *t_scale[2], *t_shift[2];
+    const float *fc_w, *fc_scale, *fc_shift;
+} minw_wdense_desc;
+
+MINW_API minw_status minw_wdense_create(const minw_wdense_desc *desc, int32_t max_batch, void *stream,
+                                        minw_net **out);
+
+/* Introspection (no counterpart in the paper): copies block `block`'s
+ * features after the most recent forward -- bf16 bit patterns, NHWC
+ * [B][h][h][*row] with *row = pad64(the block's final channels) elements per
+ * pixel, channels past the final count unspecified; h = image_hw >> block --
+ * into dst (device memory of at least count uint16), on stream, and stores
+ * the block's final channel count in *channels and the row length in *row
+ * (host pointers, nullable).  Block b's first c_b channels are the stem's
+ * or the previous transition's output, and channels c_b + i k .. + k the
+ * output of its layer i.  MINW_EINVAL for a net of another kind, a block
+ * outside 0 .. 2, no forward yet, or a short dst. */
+MINW_API minw_status minw_wdense_features(const minw_net *net, int32_t block, uint16_t *dst, size_t count,
+                                          int32_t *channels, int32_t *row, void *stream);
 
 /* Number of layers (and of entries minw_net_layer_times fills). */
 MINW_API int32_t minw_net_launches(const minw_net *net);

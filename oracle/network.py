@@ -213,6 +213,5 @@ def wdense_forward(net, x, keep=False):
         finals.append(F)
         if bi < len(net["trans"]):
             F = wdense_transition(net["trans"][bi], F, bw, tw)
-    fc = net["fc"]
-    logits = O.affine(O.linear_f32_seq(O.avgpool_f32(F), fc["w"]), fc["scale"], fc["shift"])
+    logits = wresnet_head(net, F)
     return (logits, finals) if keep else logits

@@ -125,8 +125,9 @@ namespace minw {
 minw_status conv2d_bf16(const uint16_t *act, int B, int C, int H, int W, const uint16_t *wgt, int O, int kh, int kw,
                         int bits_w, int stride, int pad, int pool, const float *scale, const float *shift,
                         float *y_out, void *workspace, size_t workspace_bytes, size_t *workspace_need,
-                        cudaStream_t s, int upd, float upd_lr, float upd_2a) {
+                        cudaStream_t s, int upd, float upd_lr, float upd_2a, int ldc) {
     ConvArgs a;
+    if (ldc != 0 && (ldc < C || ldc % 64 != 0)) return MINW_EINVAL;
     const bool query = workspace_need != nullptr;      // shape only: no pointer is used
     minw_status st = make_codes_args(a, reinterpret_cast<const uint8_t *>(act), B, C, H, W, 1,
                                      reinterpret_cast<const uint8_t *>(wgt), O, kh, kw, bits_w, stride, pad, !query);
@@ -134,8 +135,9 @@ minw_status conv2d_bf16(const uint16_t *act, int B, int C, int H, int W, const u
     if (!query && (!scale || !shift || !y_out)) return MINW_EINVAL;
     if (pool != 0 && pool != 1) return MINW_EINVAL;
     if (pool && ((a.Ho & 1) || (a.Wo & 1))) return MINW_EUNSUPPORTED;
-    if ((long long)B * H * W * C >= (1ll << 39)) return MINW_EUNSUPPORTED;
+    if ((long long)B * H * W * (ldc ? ldc : C) >= (1ll << 39)) return MINW_EUNSUPPORTED;
     a.bf16 = 1;
+    a.ldc = ldc;
     a.bits_a = 0;
     a.scale = scale;
     a.shift = shift;
@@ -151,6 +153,27 @@ minw_status conv2d_bf16(const uint16_t *act, int B, int C, int H, int W, const u
     a.upd = upd;
     a.upd_lr = upd_lr;
     a.upd_2a = upd_2a;
+    return launch_conv_tc(a, s);
+}
+
+minw_status conv2d_bf16_hardtanh(const uint16_t *act, int B, int C, int H, int W, int ldc, const uint16_t *wgt,
+                                 int O, int kh, int kw, int bits_w, int stride, int pad, const float *scale,
+                                 const float *shift, uint16_t *hb_out, int hb_ld, int hb_off, cudaStream_t s) {
+    ConvArgs a;
+    if (ldc != 0 && (ldc < C || ldc % 64 != 0)) return MINW_EINVAL;
+    if (!scale || !shift || !hb_out || hb_off < 0 || hb_ld < hb_off + O) return MINW_EINVAL;
+    minw_status st = make_codes_args(a, reinterpret_cast<const uint8_t *>(act), B, C, H, W, 1,
+                                     reinterpret_cast<const uint8_t *>(wgt), O, kh, kw, bits_w, stride, pad);
+    if (st != MINW_OK) return st;
+    if ((long long)B * H * W * (ldc ? ldc : C) >= (1ll << 39) || a.M * hb_ld >= (1ll << 39)) return MINW_EUNSUPPORTED;
+    a.bf16 = 1;
+    a.bits_a = 0;
+    a.ldc = ldc;
+    a.scale = scale;
+    a.shift = shift;
+    a.hb_out = hb_out;
+    a.hb_ld = hb_ld;
+    a.hb_off = hb_off;
     return launch_conv_tc(a, s);
 }
 
@@ -172,6 +195,14 @@ minw_status minw_conv2d_codes(const uint8_t *act, int32_t B, int32_t C, int32_t 
     a.scale = scale;
     a.shift = shift;
     return launch_conv_tc(a, (cudaStream_t)stream);
+}
+
+minw_status minw_conv2d_bf16_hardtanh(const uint16_t *act, int32_t B, int32_t C, int32_t H, int32_t W, int32_t ldc,
+                                      const uint16_t *wgt, int32_t O, int32_t kh, int32_t kw, int32_t bits_w,
+                                      int32_t stride, int32_t pad, const float *scale, const float *shift,
+                                      uint16_t *out, int32_t out_ld, int32_t out_off, void *stream) {
+    return minw::conv2d_bf16_hardtanh(act, B, C, H, W, ldc, wgt, O, kh, kw, bits_w, stride, pad, scale, shift, out,
+                                      out_ld, out_off, (cudaStream_t)stream);
 }
 
 minw_status minw_conv2d_bf16(const uint16_t *act, int32_t B, int32_t C, int32_t H, int32_t W, const uint16_t *wgt,

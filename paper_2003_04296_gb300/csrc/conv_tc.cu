@@ -30,6 +30,7 @@
 // runs out sets the device error flag read by minw_get_last_device_error, the
 // CTA stops issuing work, drains its own TMA loads and frees its TMEM.
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 #include <stdlib.h>
@@ -82,6 +83,8 @@ struct Params {
     const float *res_f32;      // shortcut as fp32 NHWC [B][Hp][Wp][O] (nullable)
     float *y_nhwc;             // BN output (before the shortcut) as fp32 NHWC (nullable)
     const float *ythr;         // breakpoints of the output quantizer on y (nullable: computed here)
+    uint16_t *hb_out;          // bf16 operands: HardTanh(BN(acc)) as bf16 NHWC rows of hb_ld, at hb_off
+    int hb_ld, hb_off;
     int32_t *acc_out;
     float *y_out;
     const float *scale, *shift;
@@ -1307,6 +1310,39 @@ __global__ void __launch_bounds__(NT, 1)
                         }
                     }
                 }
+                if (p.hb_out != nullptr && writer) {
+                    // weight-only networks: HardTanh(BN(acc)) (the fp32 fmaf, the two clamps, one
+                    // rounding to bf16) into this pixel's NHWC row, 16 channels of it
+                    uint32_t pk[8];
+#pragma unroll
+                    for (int j = 0; j < 16; j += 2) {
+                        uint32_t h2[2];
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) {
+                            const int o = min(ob + j + e, p.O - 1);
+                            const float yv = fmaf(a[j + e], __ldg(p.scale + o), __ldg(p.shift + o));
+                            h2[e] = __bfloat16_as_ushort(__float2bfloat16_rn(fminf(fmaxf(yv, -1.0f), 1.0f)));
+                        }
+                        pk[j >> 1] = h2[0] | (h2[1] << 16);
+                    }
+                    uint16_t *dst = p.hb_out + opix * p.hb_ld + p.hb_off + ob;
+                    const uintptr_t al = reinterpret_cast<uintptr_t>(dst);
+                    if (ob + 16 <= p.O && (al & 15) == 0) {
+                        reinterpret_cast<uint4 *>(dst)[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                        reinterpret_cast<uint4 *>(dst)[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+                    } else if ((al & 7) == 0) {
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) {
+                            if (ob + 4 * g + 4 <= p.O)
+                                reinterpret_cast<uint2 *>(dst)[g] = make_uint2(pk[2 * g], pk[2 * g + 1]);
+                            else
+                                for (int j = 4 * g; j < 4 * g + 4 && ob + j < p.O; ++j)
+                                    dst[j] = (uint16_t)(pk[j >> 1] >> (16 * (j & 1)));
+                        }
+                    } else {
+                        for (int j = 0; j < 16 && ob + j < p.O; ++j) dst[j] = (uint16_t)(pk[j >> 1] >> (16 * (j & 1)));
+                    }
+                }
                 if (resid) {
                     // residual block: y = BN(acc) [+ shortcut], HardTanh, quantize,
                     // element by element in the fp32 order of the block
@@ -1894,6 +1930,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, bool encode = true) {
     p.planes_out = a.planes_out; p.codes_out = a.codes_out;
     p.res_codes = a.res_codes; p.res_unit = a.res_unit; p.res_f32 = a.res_f32; p.y_nhwc = a.y_nhwc;
     p.ythr = a.ythr;
+    p.hb_out = a.hb_out; p.hb_ld = a.hb_ld; p.hb_off = a.hb_off;
 
     const int tiles = p.nbx * p.nby * p.nbb * p.ntn;
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;
@@ -1935,8 +1972,9 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, bool encode = true) {
     const cuuint64_t cel = (cuuint64_t)(p.fp4 ? a.C / 2 : a.C);
     const cuuint32_t kel = (cuuint32_t)(p.fp4 ? p.cb : p.ck);
     {
+        const cuuint64_t rel = (a.bf16 && a.ldc) ? (cuuint64_t)a.ldc : cel;     // elements per pixel row
         const cuuint64_t dims[4] = {cel, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.B};
-        const cuuint64_t strides[3] = {cel * es_, (cuuint64_t)a.W * cel * es_, (cuuint64_t)a.H * a.W * cel * es_};
+        const cuuint64_t strides[3] = {rel * es_, (cuuint64_t)a.W * rel * es_, (cuuint64_t)a.H * a.W * rel * es_};
         const cuuint32_t sd = (cuuint32_t)p.stride;
         const cuuint32_t box[4] = {kel, (cuuint32_t)p.bw * sd, (cuuint32_t)p.bh * sd, (cuuint32_t)p.bb};
         const cuuint32_t es[4] = {1u, sd, sd, 1u};
@@ -2023,7 +2061,10 @@ bool conv_tc_supported(const ConvArgs &a) {
     // E2M1 operands: rows of 64 or 128 bytes (128 or 256 channels)
     if (a.fp4 && (a.bf16 || a.C % 128 != 0)) return false;
     // bf16 operands: real-valued accumulators, so fp32 BN outputs only
-    if (a.bf16 && (a.quant_out || a.acc_out != nullptr || a.y_out == nullptr || conv_tc_residual(a))) return false;
+    if (a.bf16 && (a.quant_out || a.acc_out != nullptr || (a.y_out == nullptr) == (a.hb_out == nullptr) ||
+                   conv_tc_residual(a)))
+        return false;
+    if (a.hb_out != nullptr && (!a.bf16 || a.pool || a.workspace != nullptr || a.upd)) return false;
     if (a.quant_out && (size_t)a.O * num_levels(a.qo.bits) * sizeof(float) > 64 * 1024) return false;
     if (a.quant_out && a.codes_out != nullptr && a.O % 16 != 0) return false;
     if (a.acc_out != nullptr && a.pool) return false;

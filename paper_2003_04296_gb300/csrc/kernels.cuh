@@ -50,6 +50,12 @@ struct ConvArgs {
                            // tensor memory beside the scale factors)
     int pair_n128;         // E2M1: CTA pairs of 256 pixels x 128 channels (two accumulators fit the tensor
                            // memory beside the scale factors, so the epilogue overlaps the next MMAs)
+    int ldc;               // bf16 operands: elements between pixel rows of act8 (0: C); the product reads
+                           // channels 0 .. C of each row (the first C of a wider feature buffer)
+    // bf16 operands, in place of y_out: HardTanh(BN(acc)) rounded to bf16 into NHWC rows of hb_ld
+    // elements, channels hb_off .. hb_off + O of each (the next weight-only layer's input)
+    uint16_t *hb_out;
+    int hb_ld, hb_off;
 };
 
 // First-layer convolution on the fp32 image (see conv_first.cu).
@@ -99,7 +105,12 @@ minw_status launch_conv_tc(const ConvArgs &a, cudaStream_t s);
 minw_status conv2d_bf16(const uint16_t *act, int B, int C, int H, int W, const uint16_t *wgt, int O, int kh, int kw,
                         int bits_w, int stride, int pad, int pool, const float *scale, const float *shift,
                         float *y_out, void *workspace, size_t workspace_bytes, size_t *workspace_need,
-                        cudaStream_t s, int upd = 0, float upd_lr = 0.0f, float upd_2a = 0.0f);
+                        cudaStream_t s, int upd = 0, float upd_lr = 0.0f, float upd_2a = 0.0f, int ldc = 0);
+// The same convolution with the HardTanh + bf16 NHWC epilogue (ConvArgs::hb_out): input rows of
+// ldc elements (0: C), output rows of hb_ld elements at channel offset hb_off.
+minw_status conv2d_bf16_hardtanh(const uint16_t *act, int B, int C, int H, int W, int ldc, const uint16_t *wgt,
+                                 int O, int kh, int kw, int bits_w, int stride, int pad, const float *scale,
+                                 const float *shift, uint16_t *hb_out, int hb_ld, int hb_off, cudaStream_t s);
 bool conv_tc_supported(const ConvArgs &a);
 // Workspace the tensor-core path needs to split K for this shape (0: it does not split).
 size_t conv_tc_workspace_bytes(const ConvArgs &a);

@@ -25,6 +25,7 @@ static void net_free(minw_net *n) {
     if (!n) return;
     if (n->res) resnet_free(n);
     if (n->wres) wresnet_free(n);
+    if (n->wdense) wdense_free(n);
     for (void *p : n->owned) cudaFree(p);
     for (cudaEvent_t e : n->events) cudaEventDestroy(e);
     if (n->gexec) cudaGraphExecDestroy(n->gexec);
@@ -404,6 +405,7 @@ static bool graphs_enabled() { return minw_host::plan_options().graph != 0; }
 static minw_status forward_enqueue(minw_net *net, const float *x, int32_t B, float *logits, cudaStream_t cs) {
     if (net->kind == 1) return resnet_forward(net, x, B, logits, cs);
     if (net->kind == 2) return wresnet_forward(net, x, B, logits, cs);
+    if (net->kind == 3) return wdense_forward(net, x, B, logits, cs);
     const int nl = (int)net->L.size();
     int cur = 0;
     if (net->timing && cudaEventRecord(net->events[0], cs) != cudaSuccess) return MINW_ECUDA;
@@ -561,6 +563,10 @@ minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants) {
         wresnet_variants(net, variants);    // stem, its pass, per block conv1, pass, [shortcut], conv2, pass; head
         return MINW_OK;
     }
+    if (net->kind == 3) {
+        wdense_variants(net, variants);     // stem, its pass, per layer 1x1, pass, 3x3, pass; transitions; head
+        return MINW_OK;
+    }
     for (size_t l = 0; l < net->L.size(); ++l)
         variants[l] = l == 0 ? 0
                       : net->L[l].n128 ? MINW_VARIANT_TC_E2M1_N128
@@ -571,7 +577,10 @@ minw_status minw_net_layer_variants(const minw_net *net, int32_t *variants) {
 
 int32_t minw_net_launches(const minw_net *net) {
     if (!net) return 0;
-    return net->kind == 1 ? resnet_ops(net) : net->kind == 2 ? wresnet_ops(net) : (int32_t)net->L.size();
+    return net->kind == 1   ? resnet_ops(net)
+           : net->kind == 2 ? wresnet_ops(net)
+           : net->kind == 3 ? wdense_ops(net)
+                            : (int32_t)net->L.size();
 }
 
 // Kernels one minw_forward issues (a split-K layer issues two).
@@ -579,6 +588,7 @@ int32_t minw_net_kernels(const minw_net *net) {
     if (!net) return 0;
     if (net->kind == 1) return resnet_kernels(net);
     if (net->kind == 2) return wresnet_kernels(net);
+    if (net->kind == 3) return wdense_kernels(net);
     int32_t k = 0;
     for (size_t l = 0; l < net->L.size(); ++l) {
         const LayerPlan &P = net->L[l];

@@ -35,12 +35,15 @@ struct LayerPlan {
 
 struct ResNetPlan;   // resnet.cu
 struct WResPlan;     // wresnet.cu
+struct WDensePlan;   // wresnet.cu
 
 struct minw_net {
     int kind = 0;                     // 0: sequential (minw_net_create), 1: residual (minw_resnet18_create),
-                                      // 2: weight-only residual (minw_wresnet_create)
+                                      // 2: weight-only residual (minw_wresnet_create),
+                                      // 3: weight-only DenseNet-BC (minw_wdense_create)
     ResNetPlan *res = nullptr;
     WResPlan *wres = nullptr;
+    WDensePlan *wdense = nullptr;
     std::vector<LayerPlan> L;
     int max_batch = 0;
     uint32_t *buf[2] = {nullptr, nullptr};
@@ -75,3 +78,10 @@ int32_t wresnet_ops(const minw_net *net);
 void wresnet_variants(const minw_net *net, int32_t *variants);
 int32_t wresnet_kernels(const minw_net *net);
 void wresnet_free(minw_net *net);
+
+// The weight-only DenseNet-BC (wresnet.cu).
+minw_status wdense_forward(minw_net *net, const float *x, int B, float *logits, cudaStream_t s);
+int32_t wdense_ops(const minw_net *net);
+void wdense_variants(const minw_net *net, int32_t *variants);
+int32_t wdense_kernels(const minw_net *net);
+void wdense_free(minw_net *net);

@@ -85,6 +85,23 @@ class WResNetDesc(ctypes.Structure):
                 ("keep_activations", ctypes.c_int32)]
 
 
+WDENSE_MAX_LAYERS = 32
+_NL = 3 * WDENSE_MAX_LAYERS
+
+
+class WDenseDesc(ctypes.Structure):
+    _fields_ = [("layers", ctypes.c_int32), ("growth", ctypes.c_int32), ("bits_w", ctypes.c_int32),
+                ("thr_w", ctypes.c_float * 3), ("image_hw", ctypes.c_int32), ("num_classes", ctypes.c_int32),
+                ("stem_w", ctypes.c_void_p), ("stem_scale", ctypes.c_void_p), ("stem_shift", ctypes.c_void_p),
+                ("b_w", ctypes.c_void_p * _NL), ("b_wscale", ctypes.c_void_p * _NL),
+                ("b_scale", ctypes.c_void_p * _NL), ("b_shift", ctypes.c_void_p * _NL),
+                ("c_w", ctypes.c_void_p * _NL), ("c_wscale", ctypes.c_void_p * _NL),
+                ("c_scale", ctypes.c_void_p * _NL), ("c_shift", ctypes.c_void_p * _NL),
+                ("t_w", ctypes.c_void_p * 2), ("t_wscale", ctypes.c_void_p * 2),
+                ("t_scale", ctypes.c_void_p * 2), ("t_shift", ctypes.c_void_p * 2),
+                ("fc_w", ctypes.c_void_p), ("fc_scale", ctypes.c_void_p), ("fc_shift", ctypes.c_void_p)]
+
+
 class ResNet18Desc(ctypes.Structure):
     _fields_ = [("bits_a", ctypes.c_int32), ("bits_w", ctypes.c_int32), ("thr_a", ctypes.c_float * 3),
                 ("thr_w", ctypes.c_float * 3), ("image_hw", ctypes.c_int32), ("num_classes", ctypes.c_int32),
@@ -111,6 +128,8 @@ SIGNATURES = {
     "minw_pack_weight_bf16": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _QP, _P, _P, _P]),
     "minw_conv2d_bf16": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32, _I32, _I32,
                                         _I32, _P, _P, _P, _P]),
+    "minw_conv2d_bf16_hardtanh": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32, _I32,
+                                                 _I32, _P, _P, _P, _I32, _I32, _P]),
     "minw_bf16_matrix": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _P]),
     "minw_sgd_clip": (ctypes.c_int, [_P, _P, _I64, _F, _P]),
     "minw_fc_train_workspace_bytes": (ctypes.c_size_t, [_I32, _I32, _I32]),
@@ -156,6 +175,9 @@ SIGNATURES = {
     "minw_wresnet_create": (ctypes.c_int, [ctypes.POINTER(WResNetDesc), _I32, _P,
                                            ctypes.POINTER(ctypes.c_void_p)]),
     "minw_wresnet_activation": (ctypes.c_int, [_P, _I32, _P, ctypes.c_size_t, _P]),
+    "minw_wdense_create": (ctypes.c_int, [ctypes.POINTER(WDenseDesc), _I32, _P, ctypes.POINTER(ctypes.c_void_p)]),
+    "minw_wdense_features": (ctypes.c_int, [_P, _I32, _P, ctypes.c_size_t, ctypes.POINTER(ctypes.c_int32),
+                                            ctypes.POINTER(ctypes.c_int32), _P]),
     "minw_forward": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
     "minw_forward_host": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
     "minw_net_enable_timing": (ctypes.c_int, [_P, _I32]),
@@ -286,6 +308,13 @@ def minw_pack_weight_bf16_pad(w, Cp, q, out, channel_scale=None, stream=None):
 def minw_conv2d_bf16(act, B, C, H, W, wgt, O, kh, kw, bits_w, stride, pad, pool, scale, shift, y_out, stream=None):
     _check(lib().minw_conv2d_bf16(_ptr(act), B, C, H, W, _ptr(wgt), O, kh, kw, bits_w, stride, pad, int(pool),
                                   _ptr(scale), _ptr(shift), _ptr(y_out), _stream(stream)), "minw_conv2d_bf16")
+
+
+def minw_conv2d_bf16_hardtanh(act, B, C, H, W, ldc, wgt, O, kh, kw, bits_w, stride, pad, scale, shift, out,
+                              out_ld, out_off, stream=None):
+    _check(lib().minw_conv2d_bf16_hardtanh(_ptr(act), B, C, H, W, int(ldc), _ptr(wgt), O, kh, kw, bits_w, stride,
+                                           pad, _ptr(scale), _ptr(shift), _ptr(out), int(out_ld), int(out_off),
+                                           _stream(stream)), "minw_conv2d_bf16_hardtanh")
 
 
 def minw_bf16_matrix(x, out, transpose=False, stream=None):
@@ -562,6 +591,56 @@ class Net:
         the most recent forward (0 the stem, b + 1 block b) into `out`."""
         _check(lib().minw_wresnet_activation(self._h, int(index), _ptr(out), out.numel(), _stream(stream)),
                "minw_wresnet_activation")
+
+    @classmethod
+    def wdense(cls, params, max_batch, device, stream=None):
+        """minw_wdense_create from a parameter dict shaped like
+        ``inputs.wdense_params`` (latent fp32 weights, BN maps); the tensors
+        are copied to ``device`` for the call and released after it."""
+        d = WDenseDesc()
+        d.layers, d.growth, d.bits_w = params["layers"], params["growth"], params["bits_w"]
+        for i in range(3):
+            d.thr_w[i] = float(params["thr_w"][i])
+        d.image_hw, d.num_classes = params["hw"], params["classes"]
+        keep = []
+
+        def dev(a):
+            t = torch.from_numpy(a).to(device).contiguous()
+            keep.append(t)
+            return t.data_ptr()
+        st = params["stem"]
+        d.stem_w, d.stem_scale, d.stem_shift = dev(st["w"]), dev(st["scale"]), dev(st["shift"])
+        j = 0
+        for lay_list in params["blocks"]:
+            for lay in lay_list:
+                b, c = lay["b"], lay["c"]
+                d.b_w[j], d.b_wscale[j], d.b_scale[j], d.b_shift[j] = (dev(b["w"]), dev(b["w_scale"]),
+                                                                       dev(b["scale"]), dev(b["shift"]))
+                d.c_w[j], d.c_wscale[j], d.c_scale[j], d.c_shift[j] = (dev(c["w"]), dev(c["w_scale"]),
+                                                                       dev(c["scale"]), dev(c["shift"]))
+                j += 1
+        for i, t in enumerate(params["trans"]):
+            d.t_w[i], d.t_wscale[i], d.t_scale[i], d.t_shift[i] = (dev(t["w"]), dev(t["w_scale"]),
+                                                                   dev(t["scale"]), dev(t["shift"]))
+        fc = params["fc"]
+        d.fc_w, d.fc_scale, d.fc_shift = dev(fc["w"]), dev(fc["scale"]), dev(fc["shift"])
+        h = ctypes.c_void_p()
+        _check(lib().minw_wdense_create(ctypes.byref(d), int(max_batch), _stream(stream), ctypes.byref(h)),
+               "minw_wdense_create")
+        net = cls.__new__(cls)
+        net._h = h
+        net.max_batch = max_batch
+        net.out_features = params["classes"]
+        return net
+
+    def wdense_features(self, block, out, stream=None):
+        """minw_wdense_features: block `block`'s bf16 NHWC features after
+        the most recent forward into the int16 device tensor `out`; returns
+        (final channels, elements per pixel row)."""
+        c, r = ctypes.c_int32(), ctypes.c_int32()
+        _check(lib().minw_wdense_features(self._h, int(block), _ptr(out), out.numel(), ctypes.byref(c),
+                                          ctypes.byref(r), _stream(stream)), "minw_wdense_features")
+        return c.value, r.value
 
     @classmethod
     def resnet18(cls, params, max_batch, device, stream=None):

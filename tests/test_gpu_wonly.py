@@ -221,3 +221,63 @@ def test_conv2d_bf16_narrow_channels(dev, M, case):
     bound = np.abs(sc) * K * 2.0 ** -23 * A + 2.0 ** -23 * np.abs(yref) + 1e-30
     err = np.abs(y.cpu().numpy().astype(np.float64) - yref)
     assert (err <= bound).all(), f"worst err/bound {np.max(err / bound)}"
+
+
+# B, C, ldc, H, W, O, k, stride, out_ld, out_off
+HT_CASES = [
+    (4, 64, 256, 32, 32, 48, 1, 1, 64, 0),      # DenseNet-100 bottleneck: the first 64 of 256-element rows
+    (4, 64, 0, 32, 32, 12, 3, 1, 256, 36),      # DenseNet-100 3x3 appending 12 channels at 36 (8-byte aligned)
+    (3, 64, 0, 16, 16, 12, 3, 1, 320, 110),     # ... at 110 (4-byte aligned)
+    (2, 128, 0, 8, 8, 32, 3, 2, 64, 0),         # stride 2, 16-byte aligned rows
+    (2, 64, 128, 9, 7, 40, 3, 1, 48, 5),        # ragged tiles, odd offset
+]
+
+
+@pytest.mark.parametrize("case", HT_CASES)
+def test_conv2d_bf16_hardtanh(dev, M, case):
+    """The fused HardTanh + bf16 NHWC epilogue equals the bf16 rounding of
+    HardTanh of minw_conv2d_bf16's output on the same operands bit for bit
+    (the same accumulators), lands in channels out_off .. out_off + O of each
+    out_ld-element row and writes nothing else; inputs read from the first C
+    elements of ldc-element rows whose other elements hold values far out of
+    range (a read of them would show)."""
+    B, C, ldc, H, W, O_, k, s, ld, off = case
+    pad = k // 2
+    r = np.random.default_rng(sum(case) * 5 + 1)
+    Cf = ldc or C
+    x = r.standard_normal((B, Cf, H, W)).astype(np.float32)
+    x[:, C:] = 1e30
+    w = r.normal(0, 0.05, (O_, C, k, k)).astype(np.float32)
+    cs = (1.0 / np.abs(w.reshape(O_, -1)).max(1)).astype(np.float32)
+    scale = r.normal(0.02, 0.01, O_).astype(np.float32)
+    shift = r.normal(0, 0.3, O_).astype(np.float32)
+    bits = 3
+    xw = torch.empty((B, H, W, Cf), dtype=torch.int16, device=dev)
+    M.minw_to_bf16_nhwc(dev_tensor(x, dev), xw)
+    xc, wb = _operands(dev, M, np.ascontiguousarray(x[:, :C]), w, bits, cs)
+    Ho, Wo = (H + 2 * pad - k) // s + 1, (W + 2 * pad - k) // s + 1
+    sc, sh = dev_tensor(scale, dev), dev_tensor(shift, dev)
+    y = torch.empty((B, O_, Ho, Wo), dtype=torch.float32, device=dev)
+    M.minw_conv2d_bf16(xc, B, C, H, W, wb, O_, k, k, bits, s, pad, 0, sc, sh, y)
+    sentinel = 0x7F7F
+    out = torch.full((B, Ho, Wo, ld), sentinel, dtype=torch.int16, device=dev)
+    M.minw_conv2d_bf16_hardtanh(xw, B, C, H, W, ldc, wb, O_, k, k, bits, s, pad, sc, sh, out, ld, off)
+    torch.cuda.synchronize()
+    got = out.cpu().numpy().view(np.uint16)
+    want = O.bf16_round(np.clip(y.cpu().numpy(), -1.0, 1.0)).transpose(0, 2, 3, 1)
+    want_bits = (want.view(np.uint32) >> 16).astype(np.uint16)
+    assert np.array_equal(got[..., off:off + O_], want_bits)
+    rest = np.concatenate([got[..., :off].ravel(), got[..., off + O_:].ravel()])
+    assert (rest == sentinel).all()
+    assert M.minw_get_last_device_error() == M.MINW_OK
+
+
+def test_conv2d_bf16_hardtanh_errors(dev, M):
+    xb = torch.zeros((1, 4, 4, 64), dtype=torch.int16, device=dev)
+    wb = torch.zeros((8, 1, 1, 64), dtype=torch.int16, device=dev)
+    sc = torch.ones(8, device=dev)
+    out = torch.zeros((1, 4, 4, 16), dtype=torch.int16, device=dev)
+    with pytest.raises(M.MinwError):       # the row cannot hold channels 10 .. 18
+        M.minw_conv2d_bf16_hardtanh(xb, 1, 64, 4, 4, 0, wb, 8, 1, 1, 1, 1, 0, sc, sc, out, 16, 10)
+    with pytest.raises(M.MinwError):       # input rows shorter than C
+        M.minw_conv2d_bf16_hardtanh(xb, 1, 64, 4, 4, 32, wb, 8, 1, 1, 1, 1, 0, sc, sc, out, 16, 0)

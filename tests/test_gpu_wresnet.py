@@ -24,6 +24,7 @@ torch = pytest.importorskip("torch")
 from oracle import network as N  # noqa: E402
 from oracle import oracle as O  # noqa: E402
 from paper_2003_04296_gb300.inputs import wresnet_input, wresnet_params  # noqa: E402
+from tests._bounds import conv_bound as _conv_bound  # noqa: E402
 from tests._gpu import dev_tensor  # noqa: E402
 
 pytestmark = pytest.mark.gpu
@@ -41,25 +42,6 @@ def dev():
 def M(dev):
     from paper_2003_04296_gb300 import minw
     return minw
-
-
-def _levels(conv, bits, thr):
-    return O.quantize(conv["w"], bits, thr, conv["w_scale"]) * 2.0 ** O.units_shift(bits)
-
-
-def _conv_bound(conv, xb, y_ref, stride, bits, thr, dx=None):
-    """Bound on |y_gpu - y_ref| of one weight-only convolution + BN whose
-    bf16 input xb (fp64) is exact, or off by at most dx elementwise."""
-    k = conv["w"].shape[2]
-    wl = np.abs(_levels(conv, bits, thr))
-    sc = np.abs(conv["scale"].astype(np.float64))[None, :, None, None]
-    K = xb.shape[1] * k * k
-    mag = np.abs(xb) if dx is None else np.abs(xb) + dx
-    A = O.conv2d_real(mag, wl, stride, k // 2)
-    b = sc * K * 2.0 ** -23 * A + 2.0 ** -23 * np.abs(y_ref)
-    if dx is not None:
-        b = b + sc * O.conv2d_real(dx, wl, stride, k // 2)
-    return b
 
 
 def _check_block(blk, a, out_gpu, bits, thr):
