@@ -169,7 +169,8 @@ class Workload:
             m = layer_macs(self.params)
             return m, list(range(1, len(m)))
         if self.name == "wresnet110":
-            # ops: stem, its pass; per block conv1 (HardTanh fused), [shortcut], conv2, pass; head (unpadded MACs)
+            # ops: stem, its pass; per block conv1, [shortcut], conv2 (HardTanh and the shortcut add fused); head
+            # (unpadded MACs)
             hw = self.params["hw"]
             macs, q = [hw * hw * 16 * 27, 0], []
             size, c_in = hw, 16
@@ -180,7 +181,6 @@ class Workload:
                 if blk["down"] is not None:
                     q.append(len(macs)); macs.append(so * so * o * c_in)
                 q.append(len(macs)); macs.append(so * so * o * o * 9)
-                macs.append(0)
                 size, c_in = so, o
             macs.append(64 * self.params["classes"])
             return macs, q

@@ -313,9 +313,11 @@ MINW_API minw_status minw_conv2d_bf16(const uint16_t *act, int32_t B, int32_t C,
                                       const float *shift, float *y_out, void *stream);
 
 /* The same convolution (no pool) with the next layer's input as its output:
- * out[pixel][out_off + o] = bf16(HardTanh(fmaf(acc, scale[o], shift[o])))
- * (the fp32 clamps to [-1, 1], one round-to-nearest-even), bf16 NHWC rows of
- * out_ld elements per output pixel; the other elements of each row are not
+ * v = fmaf(acc, scale[o], shift[o]) [+ residual[b][o][y][x], one fp32 add:
+ * a residual block's shortcut, fp32 NCHW, nullable], clamped to [-1, 1]
+ * (HardTanh); out[pixel][out_off + o] = bf16(v) (round to nearest even),
+ * bf16 NHWC rows of out_ld elements per output pixel, and y_out (nullable)
+ * v as fp32 NCHW [B][O][Ho][Wo]; the other elements of each out row are not
  * written (a DenseNet block appends its new channels to its feature buffer
  * this way).  act: bf16 NHWC rows of ldc elements per pixel (0: C), of which
  * the first C are read (ldc a multiple of 64, at least C).  The accumulators
@@ -326,7 +328,7 @@ MINW_API minw_status minw_conv2d_bf16_hardtanh(const uint16_t *act, int32_t B, i
                                                int32_t ldc, const uint16_t *wgt, int32_t O, int32_t kh, int32_t kw,
                                                int32_t bits_w, int32_t stride, int32_t pad, const float *scale,
                                                const float *shift, uint16_t *out, int32_t out_ld, int32_t out_off,
-                                               void *stream);
+                                               const float *residual, float *y_out, void *stream);
 
 /* ---------------------------------------------------------------------- */
 /* Training step of a fully connected layer (Algorithm 1)                  */

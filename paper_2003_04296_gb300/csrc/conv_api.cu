@@ -158,7 +158,8 @@ minw_status conv2d_bf16(const uint16_t *act, int B, int C, int H, int W, const u
 
 minw_status conv2d_bf16_hardtanh(const uint16_t *act, int B, int C, int H, int W, int ldc, const uint16_t *wgt,
                                  int O, int kh, int kw, int bits_w, int stride, int pad, const float *scale,
-                                 const float *shift, uint16_t *hb_out, int hb_ld, int hb_off, cudaStream_t s) {
+                                 const float *shift, uint16_t *hb_out, int hb_ld, int hb_off, cudaStream_t s,
+                                 const float *res, float *z) {
     ConvArgs a;
     if (ldc != 0 && (ldc < C || ldc % 64 != 0)) return MINW_EINVAL;
     if (!scale || !shift || !hb_out || hb_off < 0 || hb_ld < hb_off + O) return MINW_EINVAL;
@@ -174,6 +175,8 @@ minw_status conv2d_bf16_hardtanh(const uint16_t *act, int B, int C, int H, int W
     a.hb_out = hb_out;
     a.hb_ld = hb_ld;
     a.hb_off = hb_off;
+    a.hb_res = res;
+    a.hb_z = z;
     return launch_conv_tc(a, s);
 }
 
@@ -200,9 +203,10 @@ minw_status minw_conv2d_codes(const uint8_t *act, int32_t B, int32_t C, int32_t 
 minw_status minw_conv2d_bf16_hardtanh(const uint16_t *act, int32_t B, int32_t C, int32_t H, int32_t W, int32_t ldc,
                                       const uint16_t *wgt, int32_t O, int32_t kh, int32_t kw, int32_t bits_w,
                                       int32_t stride, int32_t pad, const float *scale, const float *shift,
-                                      uint16_t *out, int32_t out_ld, int32_t out_off, void *stream) {
+                                      uint16_t *out, int32_t out_ld, int32_t out_off, const float *residual,
+                                      float *y_out, void *stream) {
     return minw::conv2d_bf16_hardtanh(act, B, C, H, W, ldc, wgt, O, kh, kw, bits_w, stride, pad, scale, shift, out,
-                                      out_ld, out_off, (cudaStream_t)stream);
+                                      out_ld, out_off, (cudaStream_t)stream, residual, y_out);
 }
 
 minw_status minw_conv2d_bf16(const uint16_t *act, int32_t B, int32_t C, int32_t H, int32_t W, const uint16_t *wgt,

@@ -83,8 +83,10 @@ struct Params {
     const float *res_f32;      // shortcut as fp32 NHWC [B][Hp][Wp][O] (nullable)
     float *y_nhwc;             // BN output (before the shortcut) as fp32 NHWC (nullable)
     const float *ythr;         // breakpoints of the output quantizer on y (nullable: computed here)
-    uint16_t *hb_out;          // bf16 operands: HardTanh(BN(acc)) as bf16 NHWC rows of hb_ld, at hb_off
+    uint16_t *hb_out;          // bf16 operands: HardTanh(BN(acc) [+ hb_res]) as bf16 NHWC rows of hb_ld, at hb_off
     int hb_ld, hb_off;
+    const float *hb_res;       // fp32 NCHW shortcut (nullable)
+    float *hb_z;               // fp32 NCHW copy of the HardTanh output (nullable)
     int32_t *acc_out;
     float *y_out;
     const float *scale, *shift;
@@ -1311,19 +1313,43 @@ __global__ void __launch_bounds__(NT, 1)
                     }
                 }
                 if (p.hb_out != nullptr && writer) {
-                    // weight-only networks: HardTanh(BN(acc)) (the fp32 fmaf, the two clamps, one
-                    // rounding to bf16) into this pixel's NHWC row, 16 channels of it
+                    // weight-only networks: HardTanh(BN(acc) [+ shortcut]) (the fp32 fmaf, one fp32
+                    // add, the two clamps, one rounding to bf16) into this pixel's NHWC row, 16
+                    // channels of it [and the fp32 value into NCHW]
                     uint32_t pk[8];
+                    if (p.hb_res == nullptr && p.hb_z == nullptr) {
 #pragma unroll
-                    for (int j = 0; j < 16; j += 2) {
-                        uint32_t h2[2];
+                        for (int j = 0; j < 16; j += 2) {
+                            uint32_t h2[2];
 #pragma unroll
-                        for (int e = 0; e < 2; ++e) {
-                            const int o = min(ob + j + e, p.O - 1);
-                            const float yv = fmaf(a[j + e], __ldg(p.scale + o), __ldg(p.shift + o));
-                            h2[e] = __bfloat16_as_ushort(__float2bfloat16_rn(fminf(fmaxf(yv, -1.0f), 1.0f)));
+                            for (int e = 0; e < 2; ++e) {
+                                const int o = min(ob + j + e, p.O - 1);
+                                const float yv = fmaf(a[j + e], __ldg(p.scale + o), __ldg(p.shift + o));
+                                h2[e] = __bfloat16_as_ushort(__float2bfloat16_rn(fminf(fmaxf(yv, -1.0f), 1.0f)));
+                            }
+                            pk[j >> 1] = h2[0] | (h2[1] << 16);
                         }
-                        pk[j >> 1] = h2[0] | (h2[1] << 16);
+                    } else {
+                        const long long nchw = ((long long)b * p.O * p.Ho + y) * p.Wo + x;     // channel 0
+                        const long long cst = (long long)p.Ho * p.Wo;
+                        float rv[16];
+#pragma unroll
+                        for (int j = 0; j < 16; ++j)
+                            rv[j] = p.hb_res != nullptr ? __ldg(p.hb_res + nchw + min(ob + j, p.O - 1) * cst) : 0.0f;
+#pragma unroll
+                        for (int j = 0; j < 16; j += 2) {
+                            uint32_t h2[2];
+#pragma unroll
+                            for (int e = 0; e < 2; ++e) {
+                                const int o = min(ob + j + e, p.O - 1);
+                                float yv = fmaf(a[j + e], __ldg(p.scale + o), __ldg(p.shift + o));
+                                if (p.hb_res != nullptr) yv = yv + rv[j + e];
+                                yv = fminf(fmaxf(yv, -1.0f), 1.0f);
+                                if (p.hb_z != nullptr && ob + j + e < p.O) p.hb_z[nchw + o * cst] = yv;
+                                h2[e] = __bfloat16_as_ushort(__float2bfloat16_rn(yv));
+                            }
+                            pk[j >> 1] = h2[0] | (h2[1] << 16);
+                        }
                     }
                     uint16_t *dst = p.hb_out + opix * p.hb_ld + p.hb_off + ob;
                     const uintptr_t al = reinterpret_cast<uintptr_t>(dst);
@@ -1930,7 +1956,7 @@ static minw_status make_plan(const ConvArgs &a, Plan &pl, bool encode = true) {
     p.planes_out = a.planes_out; p.codes_out = a.codes_out;
     p.res_codes = a.res_codes; p.res_unit = a.res_unit; p.res_f32 = a.res_f32; p.y_nhwc = a.y_nhwc;
     p.ythr = a.ythr;
-    p.hb_out = a.hb_out; p.hb_ld = a.hb_ld; p.hb_off = a.hb_off;
+    p.hb_out = a.hb_out; p.hb_ld = a.hb_ld; p.hb_off = a.hb_off; p.hb_res = a.hb_res; p.hb_z = a.hb_z;
 
     const int tiles = p.nbx * p.nby * p.nbb * p.ntn;
     const int sms = minw_host::num_sms() > 0 ? minw_host::num_sms() : 148;

@@ -56,6 +56,8 @@ struct ConvArgs {
     // elements, channels hb_off .. hb_off + O of each (the next weight-only layer's input)
     uint16_t *hb_out;
     int hb_ld, hb_off;
+    const float *hb_res;   // ... with a shortcut added before the HardTanh: fp32 NCHW [B][O][Ho][Wo] (nullable)
+    float *hb_z;           // ... and the HardTanh output also as fp32 NCHW (nullable)
 };
 
 // First-layer convolution on the fp32 image (see conv_first.cu).
@@ -110,7 +112,8 @@ minw_status conv2d_bf16(const uint16_t *act, int B, int C, int H, int W, const u
 // ldc elements (0: C), output rows of hb_ld elements at channel offset hb_off.
 minw_status conv2d_bf16_hardtanh(const uint16_t *act, int B, int C, int H, int W, int ldc, const uint16_t *wgt,
                                  int O, int kh, int kw, int bits_w, int stride, int pad, const float *scale,
-                                 const float *shift, uint16_t *hb_out, int hb_ld, int hb_off, cudaStream_t s);
+                                 const float *shift, uint16_t *hb_out, int hb_ld, int hb_off, cudaStream_t s,
+                                 const float *res = nullptr, float *z = nullptr);
 bool conv_tc_supported(const ConvArgs &a);
 // Workspace the tensor-core path needs to split K for this shape (0: it does not split).
 size_t conv_tc_workspace_bytes(const ConvArgs &a);

@@ -15,10 +15,12 @@
 // (conv2d_bf16): its input is the bf16 rounding of the fp32 activation, its
 // weights the exact levels as bf16, both held with their channels padded to
 // a multiple of 64 (zeros add nothing to a product), and its output the fp32
-// BN map in NCHW, or, for conv1, HardTanh of it rounded to bf16 straight into
-// conv2's padded NHWC input (the epilogue of conv2d_bf16_hardtanh).  A fused
-// pass after conv2 adds the shortcut, applies HardTanh and writes the next
-// input as padded bf16 NHWC, plus the fp32 NCHW copy a later shortcut reads.
+// BN map goes through the epilogue of conv2d_bf16_hardtanh: for conv1,
+// HardTanh of it rounded to bf16 straight into conv2's padded NHWC input; for
+// conv2, the shortcut added (one fp32 add), HardTanh, and the result written
+// both as the next block's padded bf16 NHWC input and as the fp32 NCHW copy a
+// later shortcut reads.  The 1x1 / 2 shortcut convolution writes its fp32
+// BN map (NCHW).
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -197,7 +199,7 @@ struct WResPlan {
     // count stay zero from creation on): block outputs (ping-pong) and HardTanh(BN1(conv1))
     uint16_t *AB[3][2] = {{nullptr, nullptr}, {nullptr, nullptr}, {nullptr, nullptr}};
     uint16_t *HB[3] = {nullptr, nullptr, nullptr};
-    float *Y1 = nullptr, *Y2 = nullptr, *S = nullptr;   // fp32 NCHW convolution outputs
+    float *Y1 = nullptr, *S = nullptr;     // fp32 NCHW outputs of the stem and of the shortcut convolutions
     float *pooled = nullptr;
     std::vector<float *> keep;             // with keep_activations: the stem's and every block's fp32 output
     std::vector<size_t> keep_elems;        // ... their sizes at max_batch
@@ -264,11 +266,11 @@ void wresnet_free(minw_net *net) {
 }
 
 // Ops timed by minw_net_layer_times, in forward order: the stem, its HardTanh
-// pass, per block conv1 (its HardTanh fused), [the shortcut], conv2, its pass,
-// the head.
+// pass, per block conv1 (its HardTanh fused), [the shortcut], conv2 (the
+// shortcut add and HardTanh fused), the head.
 int32_t wresnet_ops(const minw_net *net) {
     int ops = 3;
-    for (const WBlock &bk : net->wres->blocks) ops += bk.down ? 4 : 3;
+    for (const WBlock &bk : net->wres->blocks) ops += bk.down ? 3 : 2;
     return ops;
 }
 
@@ -281,7 +283,6 @@ void wresnet_variants(const minw_net *net, int32_t *v) {
         v[k++] = MINW_VARIANT_TC;
         if (bk.down) v[k++] = MINW_VARIANT_TC;
         v[k++] = MINW_VARIANT_TC;
-        v[k++] = 0;
     }
     while (k < n) v[k++] = 0;
 }
@@ -323,7 +324,6 @@ minw_status wresnet_forward(minw_net *net, const float *x, int B, float *logits,
         float *anext = R->keep.empty() ? R->A[cur ^ 1] : R->keep[bi + 1];
         const int stg = bi / R->n, j = bi - stg * R->n;
         uint16_t *xout = R->AB[stg][j & 1];
-        const int HWo = bk.c1.Ho * bk.c1.Wo;
         if ((st = wconv_ht(bk.c1, xin, 0, B, R->HB[stg], pad64(bk.c1.O), 0, s, R->bits_w)) != MINW_OK) return st;
         if ((st = mark()) != MINW_OK) return st;
         const float *sc = acur;
@@ -332,9 +332,10 @@ minw_status wresnet_forward(minw_net *net, const float *x, int B, float *logits,
             if ((st = mark()) != MINW_OK) return st;
             sc = R->S;
         }
-        if ((st = wconv(bk.c2, R->HB[stg], B, R->Y2, s, R->bits_w)) != MINW_OK) return st;
-        if ((st = mark()) != MINW_OK) return st;
-        if ((st = post(R->Y2, sc, B, bk.c2.O, HWo, anext, xout, s)) != MINW_OK) return st;
+        if ((st = conv2d_bf16_hardtanh(R->HB[stg], B, bk.c2.Cp, bk.c2.H, bk.c2.W, 0, bk.c2.wb, bk.c2.O, 3, 3,
+                                       R->bits_w, 1, 1, bk.c2.scale, bk.c2.shift, xout, pad64(bk.c2.O), 0, s, sc,
+                                       anext)) != MINW_OK)
+            return st;
         if ((st = mark()) != MINW_OK) return st;
         cur ^= 1;
         ++bi;
@@ -451,7 +452,7 @@ extern "C" minw_status minw_wresnet_create(const minw_wresnet_desc *d, int32_t m
         }
     }
     if ((st = walloc(n, &R->Y1, px * 16)) != MINW_OK ||
-        (st = walloc(n, &R->Y2, px * 16)) != MINW_OK || (st = walloc(n, &R->S, px * 16)) != MINW_OK)
+        (st = walloc(n, &R->S, px * 16)) != MINW_OK)
         return fail(st);
     if (d->keep_activations) {
         size_t e = px * 16;                               // the stem's output

@@ -129,7 +129,7 @@ SIGNATURES = {
     "minw_conv2d_bf16": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32, _I32, _I32,
                                         _I32, _P, _P, _P, _P]),
     "minw_conv2d_bf16_hardtanh": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _I32, _I32, _I32,
-                                                 _I32, _P, _P, _P, _I32, _I32, _P]),
+                                                 _I32, _P, _P, _P, _I32, _I32, _P, _P, _P]),
     "minw_bf16_matrix": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _P]),
     "minw_sgd_clip": (ctypes.c_int, [_P, _P, _I64, _F, _P]),
     "minw_fc_train_workspace_bytes": (ctypes.c_size_t, [_I32, _I32, _I32]),
@@ -311,10 +311,11 @@ def minw_conv2d_bf16(act, B, C, H, W, wgt, O, kh, kw, bits_w, stride, pad, pool,
 
 
 def minw_conv2d_bf16_hardtanh(act, B, C, H, W, ldc, wgt, O, kh, kw, bits_w, stride, pad, scale, shift, out,
-                              out_ld, out_off, stream=None):
+                              out_ld, out_off, residual=None, y_out=None, stream=None):
     _check(lib().minw_conv2d_bf16_hardtanh(_ptr(act), B, C, H, W, int(ldc), _ptr(wgt), O, kh, kw, bits_w, stride,
                                            pad, _ptr(scale), _ptr(shift), _ptr(out), int(out_ld), int(out_off),
-                                           _stream(stream)), "minw_conv2d_bf16_hardtanh")
+                                           _ptr(residual), _ptr(y_out), _stream(stream)),
+           "minw_conv2d_bf16_hardtanh")
 
 
 def minw_bf16_matrix(x, out, transpose=False, stream=None):

@@ -233,14 +233,15 @@ HT_CASES = [
 ]
 
 
-@pytest.mark.parametrize("case", HT_CASES)
-def test_conv2d_bf16_hardtanh(dev, M, case):
+@pytest.mark.parametrize("case,residual", [(c, False) for c in HT_CASES] + [(HT_CASES[3], True), (HT_CASES[4], True)])
+def test_conv2d_bf16_hardtanh(dev, M, case, residual):
     """The fused HardTanh + bf16 NHWC epilogue equals the bf16 rounding of
-    HardTanh of minw_conv2d_bf16's output on the same operands bit for bit
-    (the same accumulators), lands in channels out_off .. out_off + O of each
-    out_ld-element row and writes nothing else; inputs read from the first C
-    elements of ldc-element rows whose other elements hold values far out of
-    range (a read of them would show)."""
+    HardTanh of minw_conv2d_bf16's output [plus a shortcut, one fp32 add] on
+    the same operands bit for bit (the same accumulators), lands in channels
+    out_off .. out_off + O of each out_ld-element row and writes nothing
+    else, and its fp32 NCHW copy equals the clamped value; inputs read from
+    the first C elements of ldc-element rows whose other elements hold values
+    far out of range (a read of them would show)."""
     B, C, ldc, H, W, O_, k, s, ld, off = case
     pad = k // 2
     r = np.random.default_rng(sum(case) * 5 + 1)
@@ -261,10 +262,19 @@ def test_conv2d_bf16_hardtanh(dev, M, case):
     M.minw_conv2d_bf16(xc, B, C, H, W, wb, O_, k, k, bits, s, pad, 0, sc, sh, y)
     sentinel = 0x7F7F
     out = torch.full((B, Ho, Wo, ld), sentinel, dtype=torch.int16, device=dev)
-    M.minw_conv2d_bf16_hardtanh(xw, B, C, H, W, ldc, wb, O_, k, k, bits, s, pad, sc, sh, out, ld, off)
+    res = r.uniform(-1, 1, (B, O_, Ho, Wo)).astype(np.float32) if residual else None
+    z = torch.full((B, O_, Ho, Wo), np.nan, dtype=torch.float32, device=dev) if residual else None
+    M.minw_conv2d_bf16_hardtanh(xw, B, C, H, W, ldc, wb, O_, k, k, bits, s, pad, sc, sh, out, ld, off,
+                                residual=dev_tensor(res, dev) if residual else None, y_out=z)
     torch.cuda.synchronize()
     got = out.cpu().numpy().view(np.uint16)
-    want = O.bf16_round(np.clip(y.cpu().numpy(), -1.0, 1.0)).transpose(0, 2, 3, 1)
+    v = y.cpu().numpy()
+    if residual:
+        v = (v + res).astype(np.float32)
+    v = np.clip(v, -1.0, 1.0)
+    if residual:
+        assert np.array_equal(z.cpu().numpy(), v)
+    want = O.bf16_round(v).transpose(0, 2, 3, 1)
     want_bits = (want.view(np.uint32) >> 16).astype(np.uint16)
     assert np.array_equal(got[..., off:off + O_], want_bits)
     rest = np.concatenate([got[..., :off].ravel(), got[..., off + O_:].ravel()])
