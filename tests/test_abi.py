@@ -123,3 +123,54 @@ def test_train_workspace_layout(lib):
                                   None, fake, 1 << 30, None) == minw.MINW_EINVAL   # misaligned A
     assert lib.minw_fc_train_step(fake, fake, fake, 64, 128, 8, 0.5, 0.1, ctypes.byref(q), None, fake, None,
                                   None, fake, 16, None) == minw.MINW_EINVAL        # workspace too small
+
+
+def test_weight_only_nets_host_validation(lib):
+    """minw_wdense_create, minw_wresnet_create, minw_wdense_features and
+    minw_conv2d_bf16_hardtanh reject bad arguments before any device call."""
+    from paper_2003_04296_gb300 import minw
+    P = ctypes.c_void_p
+    fake = 4096                        # never dereferenced: validation fails first
+    out = P()
+
+    def dense(**kw):
+        d = minw.WDenseDesc()
+        d.layers, d.growth, d.bits_w, d.image_hw, d.num_classes = 16, 12, 3, 32, 10
+        for i, t in enumerate((0.75, 0.375, 0.125)):
+            d.thr_w[i] = t
+        d.stem_w = d.stem_scale = d.stem_shift = d.fc_w = d.fc_scale = d.fc_shift = fake
+        for j in range(3 * minw.WDENSE_MAX_LAYERS):
+            d.b_w[j] = d.b_scale[j] = d.b_shift[j] = d.c_w[j] = d.c_scale[j] = d.c_shift[j] = fake
+        for i in range(2):
+            d.t_w[i] = d.t_scale[i] = d.t_shift[i] = fake
+        for k, v in kw.items():
+            setattr(d, k, v)
+        return d
+
+    create = lambda d, mb=8: lib.minw_wdense_create(ctypes.byref(d), mb, None, ctypes.byref(out))
+    assert create(dense(), 0) == minw.MINW_EINVAL                       # batch
+    for bad in (dict(layers=0), dict(layers=minw.WDENSE_MAX_LAYERS + 1), dict(growth=0), dict(growth=65),
+                dict(bits_w=4), dict(image_hw=30), dict(image_hw=4), dict(num_classes=0), dict(stem_w=None)):
+        assert create(dense(**bad)) == minw.MINW_EINVAL, bad
+    d = dense()
+    d.c_shift[3 * 16 - 1] = None                                        # last layer's BN shift missing
+    assert create(d) == minw.MINW_EINVAL
+    d = dense()
+    d.thr_w[0], d.thr_w[2] = 0.1, 0.5                                   # thresholds not descending
+    assert create(d) == minw.MINW_EINVAL
+    # 32 layers of growth 64 end on 3616 channels: more than the head stages
+    assert create(dense(layers=32, growth=64)) == minw.MINW_EUNSUPPORTED
+    assert lib.minw_wdense_create(None, 8, None, ctypes.byref(out)) == minw.MINW_EINVAL
+    r = minw.WResNetDesc()
+    r.n, r.bits_w, r.image_hw, r.num_classes = 0, 3, 32, 10
+    assert lib.minw_wresnet_create(ctypes.byref(r), 8, None, ctypes.byref(out)) == minw.MINW_EINVAL
+    c, row = ctypes.c_int32(), ctypes.c_int32()
+    assert lib.minw_wdense_features(None, 0, P(fake), 1, ctypes.byref(c), ctypes.byref(row),
+                                    None) == minw.MINW_EINVAL
+    # the fused epilogue: a row too short for its channels, input rows shorter than C
+    assert lib.minw_conv2d_bf16_hardtanh(P(fake), 1, 64, 4, 4, 0, P(fake), 8, 1, 1, 1, 1, 0, P(fake), P(fake),
+                                         P(fake), 16, 10, None, None, None) == minw.MINW_EINVAL
+    assert lib.minw_conv2d_bf16_hardtanh(P(fake), 1, 64, 4, 4, 32, P(fake), 8, 1, 1, 1, 1, 0, P(fake), P(fake),
+                                         P(fake), 16, 0, None, None, None) == minw.MINW_EINVAL
+    assert lib.minw_conv2d_bf16_hardtanh(P(fake), 1, 64, 4, 4, 0, P(fake), 8, 1, 1, 1, 1, 0, None, P(fake),
+                                         P(fake), 16, 0, None, None, None) == minw.MINW_EINVAL
