@@ -1,4 +1,7 @@
-// wresnet.cu -- the weight-only MINW-Net residual network of Table III: a CIFAR
+// wresnet.cu -- the weight-only MINW-Net networks of Table III: the residual
+// network below, and the DenseNet-BC (DenseNet-100) after it.
+//
+// The residual network is a CIFAR
 // ResNet-(6n+2) (ResNet-110 for n = 18) whose block convolutions use N-bit
 // weights (the SHIFT ADDER rows: full-precision activations times level
 // weights, Sec. IV) and whose first and last layers keep fp32 weights
@@ -14,8 +17,8 @@
 // and 3.  Every block convolution runs on the bf16 tensor cores
 // (conv2d_bf16): its input is the bf16 rounding of the fp32 activation, its
 // weights the exact levels as bf16, both held with their channels padded to
-// a multiple of 64 (zeros add nothing to a product), and its output the fp32
-// BN map goes through the epilogue of conv2d_bf16_hardtanh: for conv1,
+// a multiple of 64 (zeros add nothing to a product), and its output, the fp32
+// BN map, goes through the epilogue of conv2d_bf16_hardtanh: for conv1,
 // HardTanh of it rounded to bf16 straight into conv2's padded NHWC input; for
 // conv2, the shortcut added (one fp32 add), HardTanh, and the result written
 // both as the next block's padded bf16 NHWC input and as the fp32 NCHW copy a
