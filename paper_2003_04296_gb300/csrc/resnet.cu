@@ -4,7 +4,7 @@
 // The paper fixes the layer block (QuantizedConv - [pool] - BN - HardTanh,
 // Sec. III-E), that the input of the first convolution stays fp32, and (for
 // ResNet-18, Table V's first footnote) that the first layer is not quantized.
-// It leaves the residual wiring open; this build reads it as
+// It leaves the residual wiring open; the reading implemented here:
 //   u = h(x)                       (block input, quantized levels)
 //   v = h(HardTanh(BN1(conv1(u))))
 //   y = BN2(conv2(v)) + s,  s = u (identity) or BN_d(conv_d(u)) (1x1 / 2)
