@@ -648,8 +648,8 @@ extern "C" minw_status minw_wdense_create(const minw_wdense_desc *d, int32_t max
     // the widest fp32 output (the stem's 2k channels, or a transition's) and bf16 buffer, at max_batch
     size_t y_px = (size_t)2 * k * hw * hw;
     for (int b = 0; b < 2; ++b) y_px = std::max(y_px, (size_t)(cfin[b] / 2) * (hw >> b) * (hw >> b));
-    if ((long long)max_batch * (long long)std::max((size_t)pad64(cfin[0]) * hw * hw, y_px) >= (1ll << 31))
-        return MINW_EUNSUPPORTED;
+    const size_t row_px = (size_t)std::max(pad64(cfin[0]), pad64(4 * k)) * hw * hw;   // block 1's buffer, HB
+    if ((long long)max_batch * (long long)std::max(row_px, y_px) >= (1ll << 31)) return MINW_EUNSUPPORTED;
     if (sizeof(float) * WHEAD_IMGS * cfin[2] > 48 * 1024) return MINW_EUNSUPPORTED;   // the head's staged features
     cudaStream_t s = (cudaStream_t)stream;
     minw_net *n = new minw_net();
