@@ -93,3 +93,31 @@ def test_avgpool_and_linear_bounds():
     ref = xf.astype(np.float64) @ wf.astype(np.float64).T + bf
     bound = 42 * 2.0 ** -24 * (np.abs(xf).astype(np.float64) @ np.abs(wf).astype(np.float64).T + np.abs(bf))
     assert np.all(np.abs(y - ref) <= bound)
+
+
+def test_linear_and_avgpool_order():
+    """The head's fixed operation order, which the GPU head reproduces bit for
+    bit: the fully connected layer is one fmaf chain over the features in
+    order (each step the exact x w + s rounded once) with the bias added last
+    (one rounding); the global average pool is one fp32 sum in pixel order
+    (each add rounded) and one division rounded once.  Exact rational
+    emulation of both."""
+    r = np.random.default_rng(6)
+    x = r.standard_normal((2, 9)).astype(np.float32)
+    w = r.standard_normal((3, 9)).astype(np.float32)
+    b = (r.standard_normal(3) * 4).astype(np.float32)
+    y = O.linear_f32_seq(x, w, b)
+    for i in range(2):
+        for o in range(3):
+            s = np.float32(0.0)
+            for k in range(9):
+                s = round_f32(Fraction(float(x[i, k])) * Fraction(float(w[o, k])) + Fraction(float(s)))
+            assert y[i, o] == round_f32(Fraction(float(s)) + Fraction(float(b[o])))
+    t = r.standard_normal((2, 3, 5, 3)).astype(np.float32)
+    avg = O.avgpool_f32(t)
+    for i in range(2):
+        for c in range(3):
+            s = np.float32(0.0)
+            for v in t[i, c].ravel():
+                s = round_f32(Fraction(float(s)) + Fraction(float(v)))
+            assert avg[i, c] == round_f32(Fraction(float(s)) / 15)

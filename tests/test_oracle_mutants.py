@@ -23,6 +23,7 @@ import tests.test_oracle_wresnet as TR
 _h, _quantize, _aqe_f, _aqe_b = O.h, O.quantize, O.aqe_forward, O.aqe_backward
 _pack, _conv, _conv_real = O.pack, O.conv2d_levels, O.conv2d_real
 _avg, _avg2, _fc_step = O.avgpool_f32, N.avgpool2_f32, O.fc_train_step
+_linear, _maxpool, _igrad, _wgrad = O.linear_f32_seq, O.maxpool_f32, O.conv2d_input_grad, O.conv2d_weight_grad
 
 
 def _pins_of(mod, name, params):
@@ -167,6 +168,42 @@ def avgpool2_shifted(t):
     return _avg2(np.roll(np.asarray(t, dtype=np.float32), -1, axis=3))
 
 
+def linear_bias_first(x, w, bias=None):
+    """The fully connected layer's chain started from the bias instead of
+    adding it last (each step x w + s in fp64, rounded to fp32)."""
+    x, w = np.asarray(x, dtype=np.float32), np.asarray(w, dtype=np.float32)
+    y = np.empty((x.shape[0], w.shape[0]), dtype=np.float32)
+    for i in range(x.shape[0]):
+        for o in range(w.shape[0]):
+            acc = np.float32(0.0 if bias is None else bias[o])
+            for k in range(x.shape[1]):
+                acc = np.float32(float(x[i, k]) * float(w[o, k]) + float(acc))
+            y[i, o] = acc
+    return y
+
+
+def maxpool_shifted(x, k, s, p):
+    """The pooling windows one column off."""
+    return _maxpool(np.roll(np.asarray(x, dtype=np.float32), 1, axis=3), k, s, p)
+
+
+def input_grad_flipped(g, w, stride, pad, H, W):
+    """The input gradient with unflipped taps (a correlation with W in place of its transpose)."""
+    return _igrad(g, np.ascontiguousarray(np.asarray(w)[:, :, ::-1, ::-1]), stride, pad, H, W)
+
+
+def weight_grad_flipped(g, a, kh, kw, stride, pad):
+    """The weight gradient with its taps reversed."""
+    return np.ascontiguousarray(_wgrad(g, a, kh, kw, stride, pad)[:, :, ::-1, ::-1])
+
+
+def wconv_no_bf16(conv, a, stride, bits_w, thr_w):
+    """A weight-only convolution that reads its fp32 input without the bf16 rounding (R19)."""
+    k = conv["w"].shape[2]
+    acc = O.conv2d_real(np.asarray(a, dtype=np.float64), N._wlevels(conv, bits_w, thr_w), stride, k // 2)
+    return O.affine(acc.astype(np.float32), conv["scale"], conv["shift"])
+
+
 def wdense_layer_no_hardtanh(lay, F, bits_w, thr_w):
     """The 3x3's HardTanh dropped."""
     h = O.hardtanh(N.wconv(lay["b"], F, 1, bits_w, thr_w))
@@ -229,6 +266,14 @@ MUTANTS = [
      _pins_of(TR, "test_small_wresnet_blocks", [(3,)])),
     ("training step: weight mask dropped", O, "fc_train_step", fc_step_unmasked_weights,
      _pins_of(TT, "test_fc_train_step_wiring", [(False,), (True,)])),
+    ("fully connected: bias first", O, "linear_f32_seq", linear_bias_first, [TE.test_linear_and_avgpool_order]),
+    ("max pool: shifted windows", O, "maxpool_f32", maxpool_shifted, [TE.test_maxpool_f32_vs_torch]),
+    ("input gradient: unflipped taps", O, "conv2d_input_grad", input_grad_flipped,
+     _pins_of(TT, "test_conv_backward_products_match_autograd", [(1, 1, 3)]) + [TT.test_conv_train_step_gradients]),
+    ("weight gradient: reversed taps", O, "conv2d_weight_grad", weight_grad_flipped,
+     _pins_of(TT, "test_conv_backward_products_match_autograd", [(1, 1, 3)]) + [TT.test_conv_train_step_gradients]),
+    ("weight-only conv: no bf16 input rounding", N, "wconv", wconv_no_bf16,
+     _pins_of(TR, "test_small_wresnet_blocks", [(3,)]) + _pins_of(TD, "test_small_wdense", [(3,)])),
 ]
 
 
