@@ -181,3 +181,20 @@ def test_stochastic_limits_and_counter_layout():
     assert np.array_equal(z2, z1[24:])
     _, z3 = O.aqe_forward_stochastic(x, 1.0, seed=10, offset=5)
     assert np.mean(z3 == z1) < 0.01
+
+
+def test_stochastic_noise_words_follow_r18():
+    """The noise of elements 8 c .. 8 c + 7 at offset o is the Philox4x64-10
+    block at counter (o + c, 0, 0, 0), key (seed, 0) (the block pinned to
+    numpy's generator above), split into its eight 32-bit words low half
+    first, each mapped to (u >> 8) 2^-23 - 1: a swapped half, word or
+    counter shows here though the noise statistics would not change."""
+    seed, offset = 0x9E3779B97F4A7C15, 11
+    _, z = O.aqe_forward_stochastic(np.zeros(24, dtype=np.float32), 0.5, seed=seed, offset=offset)
+    for c in range(3):
+        blk = O.philox4x64_10(np.array([offset + c, 0, 0, 0], dtype=np.uint64), np.array([seed, 0], dtype=np.uint64))
+        words = []
+        for w in blk:
+            words += [int(w) & 0xFFFFFFFF, int(w) >> 32]
+        want = np.array([(u >> 8) * 2.0 ** -23 - 1.0 for u in words], dtype=np.float32)
+        assert np.array_equal(z[8 * c:8 * c + 8], want)

@@ -24,6 +24,7 @@ _h, _quantize, _aqe_f, _aqe_b = O.h, O.quantize, O.aqe_forward, O.aqe_backward
 _pack, _conv, _conv_real = O.pack, O.conv2d_levels, O.conv2d_real
 _avg, _avg2, _fc_step = O.avgpool_f32, N.avgpool2_f32, O.fc_train_step
 _linear, _maxpool, _igrad, _wgrad = O.linear_f32_seq, O.maxpool_f32, O.conv2d_input_grad, O.conv2d_weight_grad
+_stoch = O.aqe_forward_stochastic
 
 
 def _pins_of(mod, name, params):
@@ -197,6 +198,17 @@ def weight_grad_flipped(g, a, kh, kw, stride, pad):
     return np.ascontiguousarray(_wgrad(g, a, kh, kw, stride, pad)[:, :, ::-1, ::-1])
 
 
+def stochastic_halves_swapped(x, alpha, seed, offset=0):
+    """The stochastic AQE drawing each 64-bit word's high half first."""
+    _, z = _stoch(x, alpha, seed, offset)
+    z = np.asarray(z).copy()
+    n2 = z.size // 2 * 2
+    z[:n2] = z[:n2].reshape(-1, 2)[:, ::-1].ravel()
+    xd = np.asarray(x, dtype=np.float32).astype(np.float64)
+    s = np.where(xd - z.astype(np.float64) > 0, 1.0, -1.0)
+    return alpha * s + (1.0 - alpha) * xd, z
+
+
 def wconv_no_bf16(conv, a, stride, bits_w, thr_w):
     """A weight-only convolution that reads its fp32 input without the bf16 rounding (R19)."""
     k = conv["w"].shape[2]
@@ -272,6 +284,9 @@ MUTANTS = [
      _pins_of(TT, "test_conv_backward_products_match_autograd", [(1, 1, 3)]) + [TT.test_conv_train_step_gradients]),
     ("weight gradient: reversed taps", O, "conv2d_weight_grad", weight_grad_flipped,
      _pins_of(TT, "test_conv_backward_products_match_autograd", [(1, 1, 3)]) + [TT.test_conv_train_step_gradients]),
+    ("stochastic AQE: high half first", O, "aqe_forward_stochastic", stochastic_halves_swapped,
+     [TA.test_stochastic_noise_words_follow_r18, TA.test_noise_grid_and_uniformity,
+      TA.test_stochastic_limits_and_counter_layout]),
     ("weight-only conv: no bf16 input rounding", N, "wconv", wconv_no_bf16,
      _pins_of(TR, "test_small_wresnet_blocks", [(3,)]) + _pins_of(TD, "test_small_wdense", [(3,)])),
 ]
