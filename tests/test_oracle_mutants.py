@@ -13,6 +13,7 @@ from paper_2003_04296_gb300.inputs import DEFAULT_THR
 import tests.test_oracle_aqe as TA
 import tests.test_oracle_epilogue as TE
 import tests.test_oracle_levels as TL
+import tests.test_oracle_network as TN
 import tests.test_oracle_pack_conv as TP
 import tests.test_oracle_train as TT
 import tests.test_oracle_wdense as TD
@@ -25,6 +26,7 @@ _pack, _conv, _conv_real = O.pack, O.conv2d_levels, O.conv2d_real
 _avg, _avg2, _fc_step = O.avgpool_f32, N.avgpool2_f32, O.fc_train_step
 _linear, _maxpool, _igrad, _wgrad = O.linear_f32_seq, O.maxpool_f32, O.conv2d_input_grad, O.conv2d_weight_grad
 _stoch = O.aqe_forward_stochastic
+_convnet_layer = N.convnet_layer
 
 
 def _pins_of(mod, name, params):
@@ -209,6 +211,14 @@ def stochastic_halves_swapped(x, alpha, seed, offset=0):
     return alpha * s + (1.0 - alpha) * xd, z
 
 
+def convnet_layer_hwc_flatten(layer, a, thr_a, thr_w):
+    """The first fully connected layer flattening its input in (h, w, c)
+    order instead of R14's (c, h, w)."""
+    if layer["kind"] != "conv" and layer["bits_in"] != 0 and np.ndim(a) == 4:
+        a = np.ascontiguousarray(np.asarray(a).transpose(0, 2, 3, 1)).reshape(np.shape(a))
+    return _convnet_layer(layer, a, thr_a, thr_w)
+
+
 def wconv_no_bf16(conv, a, stride, bits_w, thr_w):
     """A weight-only convolution that reads its fp32 input without the bf16 rounding (R19)."""
     k = conv["w"].shape[2]
@@ -287,6 +297,8 @@ MUTANTS = [
     ("stochastic AQE: high half first", O, "aqe_forward_stochastic", stochastic_halves_swapped,
      [TA.test_stochastic_noise_words_follow_r18, TA.test_noise_grid_and_uniformity,
       TA.test_stochastic_limits_and_counter_layout]),
+    ("ConvNet: flatten in (h, w, c) order", N, "convnet_layer", convnet_layer_hwc_flatten,
+     _pins_of(TN, "test_small_convnet_layerwise", [(1, 1), (2, 2)])),
     ("weight-only conv: no bf16 input rounding", N, "wconv", wconv_no_bf16,
      _pins_of(TR, "test_small_wresnet_blocks", [(3,)]) + _pins_of(TD, "test_small_wdense", [(3,)])),
 ]
