@@ -34,8 +34,8 @@ struct LayerPlan {
 };
 
 struct ResNetPlan;   // resnet.cu
-struct WResPlan;     // wresnet.cu
-struct WDensePlan;   // wresnet.cu
+struct WResPlan;     // wonly_nets.cu
+struct WDensePlan;   // wonly_nets.cu
 
 struct minw_net {
     int kind = 0;                     // 0: sequential (minw_net_create), 1: residual (minw_resnet18_create),
@@ -72,14 +72,14 @@ void resnet_variants(const minw_net *net, int32_t *variants);
 int32_t resnet_kernels(const minw_net *net);
 void resnet_free(minw_net *net);
 
-// The weight-only residual network (wresnet.cu).
+// The weight-only residual network (wonly_nets.cu).
 minw_status wresnet_forward(minw_net *net, const float *x, int B, float *logits, cudaStream_t s);
 int32_t wresnet_ops(const minw_net *net);
 void wresnet_variants(const minw_net *net, int32_t *variants);
 int32_t wresnet_kernels(const minw_net *net);
 void wresnet_free(minw_net *net);
 
-// The weight-only DenseNet-BC (wresnet.cu).
+// The weight-only DenseNet-BC (wonly_nets.cu).
 minw_status wdense_forward(minw_net *net, const float *x, int B, float *logits, cudaStream_t s);
 int32_t wdense_ops(const minw_net *net);
 void wdense_variants(const minw_net *net, int32_t *variants);

@@ -1,4 +1,4 @@
-// wresnet.cu -- the weight-only MINW-Net networks of Table III: the residual
+// wonly_nets.cu -- the weight-only MINW-Net networks of Table III: the residual
 // network below, and the DenseNet-BC (DenseNet-100) after it.
 //
 // The residual network is a CIFAR
