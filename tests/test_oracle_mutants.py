@@ -27,6 +27,7 @@ _avg, _avg2, _fc_step = O.avgpool_f32, N.avgpool2_f32, O.fc_train_step
 _linear, _maxpool, _igrad, _wgrad = O.linear_f32_seq, O.maxpool_f32, O.conv2d_input_grad, O.conv2d_weight_grad
 _stoch = O.aqe_forward_stochastic
 _convnet_layer = N.convnet_layer
+_maxpool_i32 = O.maxpool_i32
 
 
 def _pins_of(mod, name, params):
@@ -211,6 +212,24 @@ def stochastic_halves_swapped(x, alpha, seed, offset=0):
     return alpha * s + (1.0 - alpha) * xd, z
 
 
+def quantize_divided_scale(x, bits, thr=None, scale=None):
+    """The per-channel prescale (R7) applied as a division."""
+    if scale is None:
+        return _quantize(x, bits, thr, None)
+    return _quantize(x, bits, thr, (1.0 / np.asarray(scale, dtype=np.float64)).astype(np.float32))
+
+
+def maxpool_i32_shifted(acc, k=2, s=2):
+    """The integer pooling windows one row down (wrapping)."""
+    return _maxpool_i32(np.roll(np.asarray(acc), -1, axis=2), k, s)
+
+
+def conv_units_doubled(a_lv, w_lv, stride, pad, bits_a, bits_w):
+    """3-bit levels counted in units of 1/2 instead of 1/4 (a wrong integer scale)."""
+    acc = _conv(a_lv, w_lv, stride, pad, bits_a, bits_w)
+    return acc // 2 if 3 in (bits_a, bits_w) else acc
+
+
 def convnet_layer_hwc_flatten(layer, a, thr_a, thr_w):
     """The first fully connected layer flattening its input in (h, w, c)
     order instead of R14's (c, h, w)."""
@@ -297,6 +316,10 @@ MUTANTS = [
     ("stochastic AQE: high half first", O, "aqe_forward_stochastic", stochastic_halves_swapped,
      [TA.test_stochastic_noise_words_follow_r18, TA.test_noise_grid_and_uniformity,
       TA.test_stochastic_limits_and_counter_layout]),
+    ("quantize: prescale divided", O, "quantize", quantize_divided_scale, [TL.test_per_channel_scale_quantize]),
+    ("integer max pool: shifted windows", O, "maxpool_i32", maxpool_i32_shifted, [TE.test_maxpool_i32_vs_reshape]),
+    ("conv: 3-bit units of 1/2", O, "conv2d_levels", conv_units_doubled,
+     _pins_of(TP, "test_conv_matches_torch_float64", [(3, 1, 1, 1, 3), (1, 3, 1, 1, 3)])),
     ("ConvNet: flatten in (h, w, c) order", N, "convnet_layer", convnet_layer_hwc_flatten,
      _pins_of(TN, "test_small_convnet_layerwise", [(1, 1), (2, 2)])),
     ("weight-only conv: no bf16 input rounding", N, "wconv", wconv_no_bf16,
